@@ -1,0 +1,292 @@
+"""Plain fp64 CPU oracle for EG-MLA decode (test infrastructure only).
+
+This module is the parity reference for the CUDA path.  Only ``tests/``,
+``__graft_entry__.smoke()`` and the CPU-baseline leg of ``bench.py`` may import
+it; the library itself never does.  It shares no code with the CUDA path: the
+only common module is the seeded input generator, which holds none of the
+method's arithmetic.
+
+Everything is computed in float64 from the stored input bits (bf16 widened
+exactly), with no blocking, splitting, fusion or absorption beyond what each
+function's docstring states.  Citations are to the EG-MLA paper (arXiv
+2509.16686): section 3 ("Embedding Gated MLA", Eqs. 1-5), Appendix C (full
+formulas, Eqs. 1-14), Appendix E (the PyTorch listing), Table 5 and the Appendix
+F cache table.
+
+Reading of the gate placement (the paper is not self-consistent, see the
+repository design notes): the hot path gates the compressed latent,
+``c~ = LN_{d_c}(c (*) g)``, with ``g = G[id]`` the precomputed gate row of the
+inference variant EG-MLA-A (Section 5.2).  The paper-literal form that gates the
+up-projected keys/values (Eq. 5 applied after Eq. 2, as in the listing) is kept
+as ``decode_r0`` for documentation.
+
+Parity status: every function here is pinned by the tests in
+``tests/test_oracle_pins.py`` (library routines, closed forms, invariants, the
+paper's printed cache sizes).  ``decode_r0`` is pinned only against a PyTorch
+re-expression of the paper's listing on tiny inputs (parity unpinned beyond
+that: the paper prints no numeric example).
+"""
+from __future__ import annotations
+
+import math
+from typing import Iterable, Optional
+
+import numpy as np
+
+
+# --------------------------------------------------------------------------
+# storage
+# --------------------------------------------------------------------------
+def widen(x: np.ndarray, dtype: str) -> np.ndarray:
+    """Stored values -> float64.  bf16 arrives as uint16 bit patterns."""
+    if dtype == "bf16":
+        b = np.ascontiguousarray(x, dtype=np.uint16)
+        return (b.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    return np.asarray(x, dtype=np.float64)
+
+
+# --------------------------------------------------------------------------
+# paged latent cache (Table 5: the cache holds d_c + d_h^R values per token)
+# --------------------------------------------------------------------------
+def paged_position(block_table: np.ndarray, b: int, j: int, page_size: int):
+    """Logical position j of sequence b -> (physical page, slot in page)."""
+    return int(block_table[b, j // page_size]), j % page_size
+
+
+def gather_sequence(pool: np.ndarray, block_table: np.ndarray, b: int, length: int,
+                    page_size: int) -> np.ndarray:
+    """Rows 0..length-1 of sequence b, read through the block table one by one."""
+    rows = []
+    for j in range(length):
+        page, slot = paged_position(block_table, b, j, page_size)
+        rows.append(pool[page, slot])
+    if not rows:
+        return pool[:0, 0]
+    return np.stack(rows, axis=0)
+
+
+def append_latent(c_pool, kr_pool, id_pool, c_new, kr_new, ids_new, block_table, positions,
+                  page_size: int):
+    """Host scatter of each sequence's new token into its cache slot (Appendix C Eq. 1
+    and Eq. 10 produce c^KV and the rotated k^R; those two, plus the token id, are
+    what the cache keeps).  Returns new arrays; inputs are not modified.
+    A negative position means "nothing to append" for that sequence."""
+    c_pool, kr_pool = c_pool.copy(), kr_pool.copy()
+    id_pool = None if id_pool is None else id_pool.copy()
+    for b in range(positions.shape[0]):
+        pos = int(positions[b])
+        if pos < 0:
+            continue
+        page, slot = paged_position(block_table, b, pos, page_size)
+        c_pool[page, slot] = c_new[b]
+        kr_pool[page, slot] = kr_new[b]
+        if id_pool is not None and ids_new is not None:
+            id_pool[page, slot] = ids_new[b]
+    return c_pool, kr_pool, id_pool
+
+
+# --------------------------------------------------------------------------
+# gate (Section 3 Eqs. 3-5; inference variant EG-MLA-A in Section 5.2)
+# --------------------------------------------------------------------------
+def gate_table_from_embedding(emb: np.ndarray, w_ue: np.ndarray) -> np.ndarray:
+    """G[i] = W^UE Emb(i) for every vocabulary entry (Eqs. 3-4), precomputed once
+    as EG-MLA-A does at model-load time.  emb [V, d_e], w_ue [d_gate, d_e]."""
+    return np.asarray(emb, np.float64) @ np.asarray(w_ue, np.float64).T
+
+
+def layer_norm(x: np.ndarray, gamma: np.ndarray, beta: np.ndarray, eps: float) -> np.ndarray:
+    """LN over the last axis with biased variance and affine gamma/beta (the listing's
+    nn.LayerNorm with its default eps=1e-5)."""
+    mean = x.mean(axis=-1, keepdims=True)
+    var = ((x - mean) ** 2).mean(axis=-1, keepdims=True)
+    return (x - mean) / np.sqrt(var + eps) * gamma + beta
+
+
+def gated_latent(c: np.ndarray, g: np.ndarray, gamma, beta, eps: float) -> np.ndarray:
+    """Eq. 5 in latent space: c~ = LN(c (*) g); the Hadamard product comes first."""
+    return layer_norm(c * g, gamma, beta, eps)
+
+
+# --------------------------------------------------------------------------
+# attention for one decode query (Appendix C Eqs. 11-13)
+# --------------------------------------------------------------------------
+def softmax(s: np.ndarray) -> np.ndarray:
+    """Max-subtracted softmax over the last axis.  An empty axis gives an empty result."""
+    if s.shape[-1] == 0:
+        return s.copy()
+    m = s.max(axis=-1, keepdims=True)
+    e = np.exp(s - m)
+    return e / e.sum(axis=-1, keepdims=True)
+
+
+def _sequence_latents(case, b: int, gate: bool):
+    """(c~ [L, d_c], k^R [L, d_r]) of sequence b after the new token is appended."""
+    d = case.dims
+    L = int(case.seq_lens[b])
+    c_pool, kr_pool, id_pool = appended_pools(case)
+    c = widen(gather_sequence(c_pool, case.block_table, b, L, d.page_size), d.dtype)
+    kr = widen(gather_sequence(kr_pool, case.block_table, b, L, d.page_size), d.dtype)
+    if gate:
+        ids = gather_sequence(id_pool, case.block_table, b, L, d.page_size).astype(np.int64)
+        g = widen(case.gate_table, d.dtype)[ids] if L > 0 else np.zeros((0, d.d_c))
+        c_t = gated_latent(c, g, np.asarray(case.ln_gamma, np.float64),
+                           np.asarray(case.ln_beta, np.float64), d.ln_eps)
+    else:
+        c_t = c
+    return c_t, kr
+
+
+def appended_pools(case):
+    """The cache after this step's append (computed once per case and kept on it)."""
+    got = getattr(case, "_oracle_appended", None)
+    if got is None:
+        d = case.dims
+        got = append_latent(case.c_pool, case.kr_pool, case.id_pool, case.c_new, case.kr_new,
+                            case.ids_new, case.block_table, case.positions(), d.page_size)
+        case._oracle_appended = got
+    return got
+
+
+def head_probs_unabsorbed(case, b: int, h: int, gate: Optional[bool] = None):
+    """Softmax weights p_j of head h of sequence b over its L_b cached positions.
+
+    Keys are k_j = [W_UK,h c~_j ; k^R_j] (Eqs. 6 and 12, the RoPE key shared by all
+    heads and not gated), the query is q = [q^C ; q^R] (Eq. 11) and the scale is
+    1/sqrt(d_h + d_h^R) (Eq. 13)."""
+    d = case.dims
+    gate = d.gate if gate is None else gate
+    c_t, kr = _sequence_latents(case, b, gate)
+    qv = widen(case.q[b, h], d.dtype)
+    w_uk = widen(case.w_uk[h], d.dtype)               # [d_n, d_c]
+    k_c = c_t @ w_uk.T                                 # [L, d_n]   (Eq. 2 + split, Eq. 6)
+    k = np.concatenate([k_c, kr], axis=1)              # [L, d_n + d_r] (Eq. 12)
+    s = (k @ qv) * d.scale()                           # (Eq. 13)
+    return softmax(s), c_t
+
+
+def decode_unabsorbed(case, batches: Optional[Iterable[int]] = None,
+                      heads: Optional[Iterable[int]] = None, gate: Optional[bool] = None) -> np.ndarray:
+    """u_{t,i} = sum_j softmax_j(q_i . k_{j,i} / sqrt(d_h + d_h^R)) v_{j,i}   (Eq. 13)
+
+    with v_{j,i} = W_UV,i c~_j (Eq. 2 + split, Eq. 6): naive per-head MLA that
+    up-projects every cached latent.  Returns [B, H, d_v] float64 (rows of
+    unselected batches/heads are NaN).  A sequence of length 0 gives zeros."""
+    d = case.dims
+    gate = d.gate if gate is None else gate
+    B, H = case.batch, d.num_heads
+    out = np.full((B, H, d.d_v), np.nan)
+    bs = range(B) if batches is None else list(batches)
+    hs = range(H) if heads is None else list(heads)
+    for b in bs:
+        L = int(case.seq_lens[b])
+        if L == 0:
+            out[b, list(hs)] = 0.0
+            continue
+        c_t, kr = _sequence_latents(case, b, gate)
+        for h in hs:
+            qv = widen(case.q[b, h], d.dtype)
+            w_uk = widen(case.w_uk[h], d.dtype)
+            w_uv = widen(case.w_uv[h], d.dtype)
+            k = np.concatenate([c_t @ w_uk.T, kr], axis=1)
+            v = c_t @ w_uv.T                             # [L, d_v]
+            p = softmax((k @ qv) * d.scale())
+            out[b, h] = p @ v
+    return out
+
+
+def decode_absorbed(case, batches=None, heads=None, gate: Optional[bool] = None) -> np.ndarray:
+    """The same output computed in weight-absorbed form: q^ = W_UK,h^T q^C scores the
+    shared latent directly (q.(W c~) = (W^T q).c~), the latent-space output
+    o = sum_j p_j c~_j is formed first and W_UV,h is applied once at the end."""
+    d = case.dims
+    gate = d.gate if gate is None else gate
+    B, H = case.batch, d.num_heads
+    out = np.full((B, H, d.d_v), np.nan)
+    bs = range(B) if batches is None else list(batches)
+    hs = range(H) if heads is None else list(heads)
+    for b in bs:
+        L = int(case.seq_lens[b])
+        if L == 0:
+            out[b, list(hs)] = 0.0
+            continue
+        c_t, kr = _sequence_latents(case, b, gate)
+        for h in hs:
+            qv = widen(case.q[b, h], d.dtype)
+            q_nope, q_rope = qv[:d.d_nope], qv[d.d_nope:]
+            q_hat = widen(case.w_uk[h], d.dtype).T @ q_nope          # [d_c]
+            s = (c_t @ q_hat + kr @ q_rope) * d.scale()
+            o_lat = softmax(s) @ c_t                                 # [d_c]
+            out[b, h] = widen(case.w_uv[h], d.dtype) @ o_lat
+    return out
+
+
+def decode_r0(case, w_ukv_full: Optional[np.ndarray] = None, gate_r0: Optional[np.ndarray] = None,
+              ln_gamma_r0=None, ln_beta_r0=None, batches=None) -> np.ndarray:
+    """Paper-literal gating (Eq. 5 after Eq. 2, as the Appendix E listing does):
+    kv~ = LN_{H(d_n+d_v)}((W^UKV c) (*) g) over all heads at once, split per head
+    into k^C, v^C (Eq. 6), then Eqs. 11-13.  ``gate_r0`` [V, H(d_n+d_v)] is the
+    precomputed gate in that space and must be given.  W^UKV defaults to stacking
+    W_UK,h and W_UV,h per head, the row order of the listing's wkv_b.
+    Returns [B, H, d_v]."""
+    d = case.dims
+    B, H, dn, dv = case.batch, d.num_heads, d.d_nope, d.d_v
+    if w_ukv_full is None:
+        w_ukv_full = np.concatenate([widen(case.w_uk, d.dtype), widen(case.w_uv, d.dtype)], axis=1)
+        w_ukv_full = w_ukv_full.reshape(H * (dn + dv), d.d_c)
+    width = H * (dn + dv)
+    gamma = np.ones(width) if ln_gamma_r0 is None else np.asarray(ln_gamma_r0, np.float64)
+    beta = np.zeros(width) if ln_beta_r0 is None else np.asarray(ln_beta_r0, np.float64)
+    out = np.full((B, H, dv), np.nan)
+    bs = range(B) if batches is None else list(batches)
+    for b in bs:
+        L = int(case.seq_lens[b])
+        if L == 0:
+            out[b] = 0.0
+            continue
+        c_raw, kr = _sequence_latents(case, b, gate=False)
+        ids = gather_sequence(appended_pools(case)[2], case.block_table, b, L, d.page_size)
+        kv = c_raw @ w_ukv_full.T                                   # [L, H(dn+dv)]  Eq. 2
+        kv = layer_norm(kv * np.asarray(gate_r0, np.float64)[ids], gamma, beta, d.ln_eps)  # Eq. 5
+        kv = kv.reshape(L, H, dn + dv)
+        for h in range(H):
+            k = np.concatenate([kv[:, h, :dn], kr], axis=1)
+            v = kv[:, h, dn:]
+            p = softmax((k @ widen(case.q[b, h], d.dtype)) * d.scale())
+            out[b, h] = p @ v
+    return out
+
+
+# --------------------------------------------------------------------------
+# cache size (Table 5 and the Appendix F table)
+# --------------------------------------------------------------------------
+def kv_elements_per_token(kind: str, n_layers: int, *, n_heads: int = 0, d_head: int = 0,
+                          n_groups: int = 0, d_c: int = 0, d_rope: int = 0, r: int = 1) -> int:
+    """KV-cache elements stored per token over all layers (Table 5).
+
+    mha: 2 n_h d_h l;  gqa: 2 n_g d_h l;  mqa: 2 d_h l;  mla: (d_c + d_h^R) l;
+    egmla: (d_c / r + d_h^R) l  (d_c / r is the latent width the cache actually keeps)."""
+    if kind == "mha":
+        return 2 * n_heads * d_head * n_layers
+    if kind == "gqa":
+        return 2 * n_groups * d_head * n_layers
+    if kind == "mqa":
+        return 2 * d_head * n_layers
+    if kind == "mla":
+        return (d_c + d_rope) * n_layers
+    if kind == "egmla":
+        if d_c % r:
+            raise ValueError("d_c must be divisible by r")
+        return (d_c // r + d_rope) * n_layers
+    raise ValueError(kind)
+
+
+def kv_bytes_per_token(d_c: int, d_rope: int, n_layers: int, elem_bytes: int,
+                       with_token_id: bool) -> int:
+    """Bytes the paged cache keeps per token: (d_c + d_r) values per layer, plus the
+    4-byte token id per layer that read-time gating needs to find g = G[id]."""
+    return n_layers * ((d_c + d_rope) * elem_bytes + (4 if with_token_id else 0))
+
+
+def embedding_params(n_layers: int, vocab: int, d_e: int) -> int:
+    """Per-layer gate embedding tables: l * V * d_e parameters (Appendix A 'Embed Size')."""
+    return n_layers * vocab * d_e
