@@ -1,0 +1,391 @@
+"""Decode-step benchmark of libegmla on synthetic EG-MLA workloads.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c32k] [--impl reference]
+
+A step is one pass of the whole decode hot path for one batch: append of each
+sequence's new token to the paged latent cache, query absorption, the split-KV
+gated latent attention and the split merge with the W_UV up-projection.  The
+default workload is the 32K-context one (batch 8, 16 heads, d_c 256, RoPE 64,
+64-token pages permuted over a shared pool, vocabulary 32000), on which the
+roofline target of the hot path is stated.
+
+value: decode tokens/s (new tokens produced per second, all GPUs) with every
+input resident in HBM; the step is replayed from a CUDA graph over three
+rotating cache replicas (3 x 168 MB > L2), so the latent stream comes from HBM.
+e2e: the same metric through the C ABI from pinned HOST buffers, the per-step
+inputs copied in and the output copied back inside the timed region.
+roofline: the decode kernel's latent-cache bytes per launch divided by its own
+CUDA-event duration (a second pass of the same steps with per-launch events on
+the launching stream), against the measured HBM copy bandwidth.
+cpu_baseline / --impl reference: the fp64 oracle on the host cores on a bounded
+sample of the same workload, scaled to decode tokens/s.
+
+Multi-GPU (torchrun): every rank runs its own replica of the workload (the
+sequences are independent; no data-path collective); the slowest rank's time
+sets the aggregate.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "decode tokens/sec and latent-cache HBM GB/s (fraction of ~8 TB/s) vs ctx len"
+UNIT = "tokens/s"
+REPLICAS = 3
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--warmup", type=int, default=30)
+    ap.add_argument("--workload", default="c32k", choices=["c32k", "c4k", "ragged", "ragged_mla"])
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--splits", type=int, default=0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=0)
+    return ap.parse_args()
+
+
+def make_workload(name):
+    from paper_2509_16686_gb300 import synth
+    if name == "c32k":
+        case = synth.case_c32k(keep_logical=False)
+        desc = "c32k: batch 8 x context 32768, 16 heads, d_nope 128, d_rope 64, d_c 256, vocab 32000, " \
+               "64-token pages permuted over one pool, uniform ids"
+    elif name == "c4k":
+        case = synth.case_c4k(keep_logical=False)
+        desc = "c4k: batch 32 x context 4096, 16 heads, d_c 256, d_rope 64, vocab 32000, contiguous pages"
+    elif name == "ragged":
+        case = synth.case_ragged(keep_logical=False)
+        desc = "ragged: batch 128, contexts log-uniform [128, 16384], 16 heads, d_c 192, vocab 50000, Zipf(1.1) ids"
+    else:
+        case = synth.case_ragged(gate=False, keep_logical=False)
+        desc = "ragged_mla: plain-MLA baseline (gate off) at d_c 512 on the ragged lengths"
+    return case, desc
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+# ----------------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id):
+        self.gpu_id = gpu_id
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-lms", "100", "-i", str(self.gpu_id)], stdout=subprocess.PIPE,
+                                         stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.25)
+        return self
+
+    def __exit__(self, *a):
+        self.lines = []
+        if self.proc is not None:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for l in self.lines:
+            f = [x.strip() for x in l.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def nvsmi_id(torch, dev):
+    try:
+        u = str(torch.cuda.get_device_properties(dev).uuid)
+        return u if u.startswith("GPU-") else "GPU-" + u
+    except Exception:
+        return dev
+
+
+# ----------------------------------------------------------------------------- CPU oracle timing
+def oracle_sample_rate(case, budget_s):
+    """Decode tokens/s of the fp64 oracle on host cores, from a bounded sample:
+    whole heads of whole sequences while the budget lasts (at least one head)."""
+    from oracle import egmla_oracle as orc
+    B, H = case.batch, case.dims.num_heads
+    t0 = time.perf_counter()
+    heads_done = 0
+    b = 0
+    while True:
+        for h in range(H):
+            orc.decode_unabsorbed(case, batches=[b], heads=[h])
+            heads_done += 1
+            if time.perf_counter() - t0 > budget_s:
+                break
+        if time.perf_counter() - t0 > budget_s or b + 1 >= B:
+            break
+        b += 1
+    dt = time.perf_counter() - t0
+    # one decode token = all heads of one sequence
+    rate = (heads_done / H) / dt
+    sample = f"{heads_done} head(s) of {b + 1} sequence(s) at full context, {dt:.1f} s"
+    return rate, sample, dt
+
+
+def host_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def run_reference(args):
+    """The reference arm: the fp64 oracle on the host cores.  Each step computes one
+    head of sequence 0 over its first S cached tokens, S chosen so that the whole
+    run fits in about two minutes; the oracle's cost is linear in the context, so
+    the step time is scaled by (L / S) x heads to one decode token."""
+    import dataclasses
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    case, desc = make_workload(args.workload)
+    from oracle import egmla_oracle as orc
+    H = case.dims.num_heads
+    L = int(case.seq_lens[0])
+    n_steps = max(1, args.steps) + max(0, args.warmup)
+    probe = dataclasses.replace(case, seq_lens=case.seq_lens[:1].copy(), block_table=case.block_table[:1],
+                                q=case.q[:1], c_new=case.c_new[:1], kr_new=case.kr_new[:1],
+                                ids_new=case.ids_new[:1])
+    t0 = time.perf_counter()
+    orc.decode_unabsorbed(probe, batches=[0], heads=[0])
+    t_full = time.perf_counter() - t0           # includes the one-time append copy
+    t0 = time.perf_counter()
+    orc.decode_unabsorbed(probe, batches=[0], heads=[0])
+    t_full = min(t_full, time.perf_counter() - t0)
+    S = int(min(L, max(64, L * (110.0 / n_steps) / max(t_full, 1e-6))))
+    sub = dataclasses.replace(probe, seq_lens=np.array([S], dtype=np.int32))
+    orc.appended_pools(sub)
+    times = []
+    t_start = time.perf_counter()
+    for i in range(n_steps):
+        t1 = time.perf_counter()
+        orc.decode_unabsorbed(sub, batches=[0], heads=[i % H])
+        dt = time.perf_counter() - t1
+        if i >= args.warmup:
+            times.append(dt)
+        if time.perf_counter() - t_start > 170:
+            break
+    t_token = statistics.mean(times) * H * (L / S)
+    rate = 1.0 / t_token
+    line = {
+        "impl": "reference", "metric": METRIC, "value": rate, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": len(times), "warmup": args.warmup, "ms_per_step": t_token * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": desc, "batch": case.batch, "ctx": L},
+        "cpu_baseline": {"value": rate, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
+                         "sample": f"per step one head of one sequence over its first {S} of {L} cached "
+                                   f"tokens, scaled x{H} heads x{L / S:.1f} context"},
+        "e2e": {"value": rate, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ----------------------------------------------------------------------------- GPU arm
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    import torch
+    ws, rank, local = dist_env()
+    dist = None
+    if ws > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.cuda.current_device()
+
+    from paper_2509_16686_gb300 import _lib, device, synth  # noqa: F401
+    from oracle import egmla_oracle as orc  # CPU-baseline leg only
+
+    case, desc = make_workload(args.workload)
+    B = case.batch
+    d = case.dims
+    dcs = [device.upload(case, num_splits=args.splits)]
+    for _ in range(REPLICAS - 1):
+        r = device.upload(case, num_splits=args.splits)
+        dcs.append(r)
+    # all replicas share the weights, queries and outputs of the first
+    for r in dcs[1:]:
+        for name in ("q", "gate_table", "ln_gamma", "ln_beta", "w_uk", "w_uv", "out", "workspace", "status",
+                     "block_table", "seq_lens", "positions", "c_new", "kr_new", "ids_new"):
+            setattr(r, name, getattr(dcs[0], name))
+    stream = torch.cuda.Stream()
+    tokens_cached = int(case.seq_lens.astype(np.int64).sum())
+    elem = 2 if d.dtype == "bf16" else 4
+    id_bytes = 4 if d.gate else 0
+    cache_bytes = tokens_cached * ((d.d_c + d.d_rope) * elem + id_bytes)
+    splits = dcs[0].num_splits or _lib.eg_mla_default_num_splits()
+    launches_per_step = 4 if d.dtype == "bf16" else 3
+
+    # ---- warm-up, then capture one graph of REPLICAS steps (one per cache replica)
+    with torch.cuda.stream(stream):
+        for i in range(max(3, args.warmup)):
+            dcs[i % REPLICAS].step(stream)
+    stream.synchronize()
+    assert dcs[0].read_status() == 0, "device status after warm-up"
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        for r in dcs:
+            r.step(stream)
+    torch.cuda.synchronize()
+    reps = max(1, math.ceil(args.steps / REPLICAS))
+    steps = reps * REPLICAS
+    with torch.cuda.stream(stream):
+        for _ in range(2):
+            graph.replay()
+    torch.cuda.synchronize()
+
+    # ---- timed region: `steps` steps, barrier + sync on both sides
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(nvsmi_id(torch, dev)) as clk:
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize()
+        with torch.cuda.stream(stream):
+            ev0.record(stream)
+            for _ in range(reps):
+                graph.replay()
+            ev1.record(stream)
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+    elapsed_ms = ev0.elapsed_time(ev1)
+    if dist:
+        t = torch.tensor([elapsed_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+    assert dcs[0].read_status() == 0, "device status after timed region"
+    ms_per_step = elapsed_ms / steps
+    value = ws * B * steps / (elapsed_ms / 1e3)
+
+    # ---- the decode kernel alone: per-launch events on the launching stream
+    prof_steps = min(steps, 300)
+    _lib.eg_mla_profile_begin(prof_steps)
+    with torch.cuda.stream(stream):
+        for i in range(prof_steps):
+            dcs[i % REPLICAS].step(stream)
+    stream.synchronize()
+    ms_sum, n_l = _lib.eg_mla_profile_end()
+    k_ms = ms_sum / max(1, n_l)
+    achieved = cache_bytes / (k_ms * 1e-3) / 1e9
+    peaks_path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(peaks_path):
+        peak = float(json.load(open(peaks_path))["hbm_gbs"])
+        peak_src = "measured"
+    else:
+        peak, peak_src = 6800.0, "fallback"
+    traffic = None
+    tpath = os.path.join(ROOT, "profiles", "traffic.json")
+    if os.path.exists(tpath):
+        tj = json.load(open(tpath)).get(args.workload)
+        if tj:
+            traffic = tj.get("dram_bytes_per_launch")
+
+    # ---- end to end through the C ABI with host buffers
+    e2e_steps = args.e2e_steps or min(steps, 2000)
+    h_in = {k: getattr(dcs[0], k).cpu().pin_memory() for k in ("q", "c_new", "kr_new", "ids_new", "positions",
+                                                             "seq_lens")}
+    h_out = torch.empty(dcs[0].out.shape, dtype=dcs[0].out.dtype).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for t in h_in.values())
+    d2h = h_out.numel() * h_out.element_size()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for i in range(e2e_steps):
+            r = dcs[i % REPLICAS]
+            for k, t in h_in.items():
+                getattr(r, k).copy_(t, non_blocking=True)
+            r.step(stream)
+            h_out.copy_(r.out, non_blocking=True)
+        e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    if dist:
+        t = torch.tensor([e2e_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    e2e_value = ws * B * e2e_steps / (e2e_ms / 1e3)
+
+    # ---- CPU baseline (rank 0, N = 1 only)
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        rate, sample, _ = oracle_sample_rate(case, budget_s=12.0)
+        cpu = {"value": rate, "unit": UNIT, "cores": host_cores(), "kind": "oracle", "sample": sample}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": steps, "warmup": args.warmup,
+            "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": d.dtype, "data": "synthetic",
+            "config": {"workload": desc, "batch": B, "ctx_tokens_cached": tokens_cached, "splits": splits,
+                       "page_size": d.page_size, "l2": f"inputs larger than L2: {REPLICAS} rotating cache "
+                       f"replicas of {cache_bytes / 1e6:.0f} MB", "graph": "step replayed from a CUDA graph"},
+            "kv_cache_gbs": cache_bytes * steps / (elapsed_ms / 1e3) / 1e9 * 1.0,
+            "kv_bytes_per_token": (d.d_c + d.d_rope) * elem + id_bytes,
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": traffic, "kernel": "decode_tc_kernel",
+                         "kernel_ms": k_ms, "bytes_per_launch": cache_bytes, "peak_source": peak_src},
+            "cpu_baseline": cpu,
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "gpu_launches": steps * launches_per_step,
+            "clocks": clk.summary(),
+        }
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,223 @@
+/*
+ * egmla.h - C ABI of libegmla, the GB300 (sm_103a) decode hot path of EG-MLA
+ * (Embedding-Gated Multi-head Latent Attention, arXiv 2509.16686).
+ *
+ * The library implements one decode step of an EG-MLA attention layer over a
+ * paged latent KV cache:
+ *   - eg_mla_append_latent writes each sequence's new compressed latent c^KV
+ *     (Appendix C Eq. 1) and its rotated RoPE key k^R (Eq. 10), plus the token
+ *     id, into the cache.  The cache keeps (d_c + d_h^R) values per token per
+ *     layer (Table 5).
+ *   - eg_mla_decode reads the cache, gathers each cached token's gate row
+ *     g = G[id] (Section 3 Eqs. 3-4 in the table form of EG-MLA-A, Section 5.2),
+ *     applies the gate and LayerNorm to the latent as it is read,
+ *     c~ = LN(c (*) g) (Eq. 5 in latent space), and runs weight-absorbed MLA
+ *     (Eqs. 11-13): q^ = W_UK,h^T q^C scores the shared latent plus the shared
+ *     RoPE key with scale 1/sqrt(d_h + d_h^R), an online softmax with split-KV
+ *     partials is merged by log-sum-exp, and the latent-space output is
+ *     up-projected through W_UV,h.  It returns the per-head outputs u_{t,i}.
+ *
+ * Conventions shared by every call:
+ *   - Every pointer argument except `dims`, `bytes_out` and `out_splits` is a
+ *     DEVICE pointer to caller-owned memory.  The library never allocates,
+ *     frees or keeps device memory between calls.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Calls are asynchronous on that stream and never synchronise
+ *     the host.
+ *   - Host-side argument errors return a negative eg_mla_status and launch
+ *     nothing.  Errors found on the device (out-of-range page id or token id,
+ *     a pipeline wait that timed out) are written to *dev_status (a device
+ *     int32 that the caller zeroes; the first error wins); the host reads it
+ *     after synchronising.  dev_status may be NULL, in which case device
+ *     errors are not reported.
+ *   - Layouts are row-major and densely packed unless stated.  Model-dtype
+ *     tensors hold bf16 (EG_MLA_BF16) or fp32 (EG_MLA_FP32) elements;
+ *     ln_gamma/ln_beta are always fp32.
+ */
+#ifndef EGMLA_H
+#define EGMLA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  EG_MLA_OK = 0,
+  EG_MLA_ERR_INVALID_ARG = -1,   /* null pointer, bad size, misaligned buffer */
+  EG_MLA_ERR_UNSUPPORTED = -2,   /* dims outside the compiled kernel shapes */
+  EG_MLA_ERR_CUDA = -3,          /* a CUDA runtime call failed (launch, attribute) */
+  EG_MLA_ERR_OUT_OF_RANGE = -4,  /* device: page id >= num_pages or token id >= vocab */
+  EG_MLA_ERR_TIMEOUT = -5,       /* device: a pipeline wait exceeded its limit */
+  EG_MLA_ERR_WORKSPACE = -6      /* workspace too small or misaligned */
+} eg_mla_status;
+
+typedef enum { EG_MLA_BF16 = 0, EG_MLA_FP32 = 1 } eg_mla_dtype;
+
+typedef enum {
+  EG_MLA_GATE_NONE = 0,    /* plain MLA: the latent is used as cached (baseline) */
+  EG_MLA_GATE_MUL_LN = 1   /* EG-MLA: c~ = LN(c (*) G[id]) with affine gamma/beta */
+} eg_mla_gate_mode;
+
+/* Shapes of one attention layer.  d_v = value head dim (= d_nope in the paper's
+ * models, Appendix A).  softmax_scale <= 0 selects 1/sqrt(d_nope + d_rope)
+ * (Eq. 13); ln_eps <= 0 selects 1e-5 (nn.LayerNorm's default, listing of
+ * Appendix E). */
+typedef struct {
+  int32_t num_heads;
+  int32_t d_nope;
+  int32_t d_rope;
+  int32_t d_v;
+  int32_t d_c;
+  int32_t page_size;
+  int32_t vocab;
+  int32_t dtype;      /* eg_mla_dtype */
+  int32_t gate_mode;  /* eg_mla_gate_mode */
+  float softmax_scale;
+  float ln_eps;
+} eg_mla_dims;
+
+/* Supported shapes.
+ *   bf16 (tensor-core path): num_heads 16, d_rope 64, page_size 64,
+ *        d_c in {192, 256} with either gate mode, d_c 512 with EG_MLA_GATE_NONE;
+ *        d_nope, d_v multiples of 8 up to 256.
+ *   fp32: num_heads <= 16, d_c <= 512 and a multiple of 4, d_rope <= 64,
+ *        d_nope, d_v <= 256, page_size 64.
+ * Other shapes return EG_MLA_ERR_UNSUPPORTED. */
+
+/*
+ * eg_mla_append_latent - write one new token per sequence into the paged cache.
+ *
+ * Cache content per token is the compressed latent c^KV [d_c] (Appendix C
+ * Eq. 1), the rotated shared RoPE key k^R [d_rope] (Eq. 10; the listing of
+ * Appendix E rotates k_pe before it is used), and the token id i_t that the
+ * gate needs at read time (Section 3, Eq. 3).  Nothing is gated here: with
+ * latent-space gating the gate is applied when the latent is read.
+ *
+ *   c_pool       [num_pages, page_size, d_c]   model dtype, written
+ *   krope_pool   [num_pages, page_size, d_rope] model dtype, written
+ *   id_pool      [num_pages, page_size] int32, written; may be NULL (then
+ *                ids_new is ignored)
+ *   c_new        [batch, d_c], krope_new [batch, d_rope], ids_new [batch]
+ *   block_table  [batch, max_pages_per_seq] int32: logical page -> physical page
+ *   positions    [batch] int32: logical slot of the new token (= seq_len-1);
+ *                a negative position skips that sequence
+ * Device errors: a position whose page index is >= max_pages_per_seq or whose
+ * physical page is outside [0, num_pages) is skipped and reported as
+ * EG_MLA_ERR_OUT_OF_RANGE.  The copy is bit-exact.
+ */
+int eg_mla_append_latent(const eg_mla_dims* dims, void* c_pool, void* krope_pool,
+                         int32_t* id_pool, const void* c_new, const void* krope_new,
+                         const int32_t* ids_new, const int32_t* block_table,
+                         int32_t max_pages_per_seq, const int32_t* positions,
+                         int32_t batch, int32_t num_pages, int32_t* dev_status,
+                         void* stream);
+
+/*
+ * eg_mla_default_num_splits - the split count eg_mla_decode uses for
+ * num_splits = 0: one split-KV work unit per SM of the current device.
+ */
+int eg_mla_default_num_splits(int32_t* out_splits);
+
+/*
+ * eg_mla_decode_workspace_size - bytes of device workspace eg_mla_decode needs
+ * for this batch and split count (0 = default).  The workspace holds the page
+ * prefix sums, the absorbed queries q^ = W_UK,h^T q^C and the split-KV partial
+ * results (running max, denominator and un-normalised latent output per
+ * split, sequence and head).  Returns 0 for unsupported dims.
+ */
+size_t eg_mla_decode_workspace_size(const eg_mla_dims* dims, int32_t batch, int32_t num_splits);
+
+/*
+ * eg_mla_decode - one decode step of EG-MLA attention for `batch` sequences.
+ *
+ * For each sequence b and head h, with L_b = seq_lens[b] cached tokens
+ * (including the one just appended) and c~_j = LN(c_j (*) G[id_j]) over d_c
+ * (EG_MLA_GATE_MUL_LN) or c~_j = c_j (EG_MLA_GATE_NONE):
+ *   s_j   = scale * (q^_h . c~_j + q^R_h . k^R_j),  q^_h = W_UK,h^T q^C_h   (Eqs. 11-13)
+ *   u_b,h = W_UV,h sum_j softmax(s)_j c~_j                                    (Eq. 13, Eq. 6)
+ * which equals the paper's per-head attention with k^C = W_UK c~ and
+ * v^C = W_UV c~ (weight absorption).  A sequence with L_b = 0 gets u = 0.
+ *
+ *   q            [batch, num_heads, d_nope + d_rope] model dtype; RoPE already
+ *                applied to the last d_rope entries
+ *   c_pool, krope_pool, id_pool: the paged cache (see eg_mla_append_latent);
+ *                id_pool may be NULL for EG_MLA_GATE_NONE.  c_pool and
+ *                krope_pool must be 16-byte aligned.
+ *   block_table  [batch, max_pages_per_seq] int32
+ *   seq_lens     [batch] int32 (device), each <= max_seq_len
+ *   max_seq_len  host-side upper bound of seq_lens (<= max_pages_per_seq*page_size)
+ *   gate_table   [vocab, d_c] model dtype: G[i] = W^UE Emb(i) precomputed per
+ *                vocabulary entry (EG-MLA-A); ignored for EG_MLA_GATE_NONE
+ *   ln_gamma, ln_beta  [d_c] fp32, may be NULL (gamma = 1, beta = 0)
+ *   w_uk         [num_heads, d_nope, d_c] model dtype (the k_nope rows of the
+ *                listing's wkv_b weight viewed per head)
+ *   w_uv         [num_heads, d_v, d_c] model dtype (the v rows of wkv_b)
+ *   out          [batch, num_heads, d_v] model dtype, written
+ *   num_splits   number of split-KV work units (0 = eg_mla_default_num_splits);
+ *                the cache pages of all sequences are divided into this many
+ *                equal contiguous ranges
+ *   workspace    device buffer of at least eg_mla_decode_workspace_size()
+ *                bytes, 256-byte aligned; its content is scratch
+ * Returns EG_MLA_OK once the kernels are queued.  Device errors go to
+ * *dev_status; the content of `out` is then unspecified.
+ */
+int eg_mla_decode(const eg_mla_dims* dims, const void* q, const void* c_pool,
+                  const void* krope_pool, const int32_t* id_pool,
+                  const int32_t* block_table, int32_t max_pages_per_seq,
+                  const int32_t* seq_lens, int32_t max_seq_len, int32_t batch,
+                  int32_t num_pages, const void* gate_table, const float* ln_gamma,
+                  const float* ln_beta, const void* w_uk, const void* w_uv, void* out,
+                  int32_t num_splits, void* workspace, size_t workspace_bytes,
+                  int32_t* dev_status, void* stream);
+
+/*
+ * eg_mla_kv_bytes_per_token - bytes the paged cache keeps per token over
+ * n_layers layers: (d_c + d_rope) elements of the model dtype per layer
+ * (Table 5 with d_c the cached latent width), plus a 4-byte token id per
+ * layer when gating is on (read-time gating needs the id).  Host only.
+ */
+int eg_mla_kv_bytes_per_token(const eg_mla_dims* dims, int32_t n_layers, int64_t* bytes_out);
+
+/* eg_mla_status_string - static text for a status code. */
+const char* eg_mla_status_string(int status);
+
+/*
+ * eg_mla_debug_gather - test entry: runs the decode kernel's cache-read stage
+ * (TMA page loads through the block table and the token-id gate-row gather)
+ * and writes what it read for every cached position instead of attending.
+ * bf16 path only.  Outputs are dense per (sequence, logical position):
+ *   c_out [batch, max_seq_len, d_c], kr_out [batch, max_seq_len, d_rope],
+ *   ids_out [batch, max_seq_len] int32, g_out [batch, max_seq_len, d_c]
+ * Positions >= seq_lens[b] are left untouched.  Same argument rules and
+ * workspace as eg_mla_decode.
+ */
+int eg_mla_debug_gather(const eg_mla_dims* dims, const void* c_pool, const void* krope_pool,
+                        const int32_t* id_pool, const int32_t* block_table,
+                        int32_t max_pages_per_seq, const int32_t* seq_lens,
+                        int32_t max_seq_len, int32_t batch, int32_t num_pages,
+                        const void* gate_table, void* c_out, void* kr_out, int32_t* ids_out,
+                        void* g_out, int32_t num_splits, void* workspace,
+                        size_t workspace_bytes, int32_t* dev_status, void* stream);
+
+/*
+ * eg_mla_profile_begin / eg_mla_profile_end - per-launch timing of the split-KV
+ * decode kernel (the one that streams the latent cache).  After begin, every
+ * eg_mla_decode call records a CUDA event pair around that kernel's launch on
+ * its stream, for at most max_launches launches.  end synchronises on the
+ * events, returns the summed kernel time in milliseconds and the number of
+ * launches timed, releases the events and stops recording.  Host-side event
+ * objects only; not for use while a stream is being captured into a graph.
+ * Returns EG_MLA_ERR_CUDA if event creation fails, EG_MLA_ERR_INVALID_ARG for
+ * max_launches <= 0 or null outputs.
+ */
+int eg_mla_profile_begin(int32_t max_launches);
+int eg_mla_profile_end(double* ms_sum, int32_t* launches);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* EGMLA_H */

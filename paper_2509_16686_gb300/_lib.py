@@ -1,0 +1,211 @@
+"""ctypes binding of libegmla (include/egmla.h).
+
+Argument marshalling only: torch tensors are passed as raw device pointers and
+the current torch CUDA stream as the stream handle; every step of the decode
+path runs in the library's kernels.  There is no fallback: if the library
+cannot be built or loaded, ``load()`` raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+import threading
+from typing import Optional
+
+import torch
+
+from . import build as _build
+
+EG_MLA_OK = 0
+EG_MLA_ERR_INVALID_ARG = -1
+EG_MLA_ERR_UNSUPPORTED = -2
+EG_MLA_ERR_CUDA = -3
+EG_MLA_ERR_OUT_OF_RANGE = -4
+EG_MLA_ERR_TIMEOUT = -5
+EG_MLA_ERR_WORKSPACE = -6
+
+EG_MLA_BF16 = 0
+EG_MLA_FP32 = 1
+EG_MLA_GATE_NONE = 0
+EG_MLA_GATE_MUL_LN = 1
+
+EXPORTED = [
+    "eg_mla_append_latent",
+    "eg_mla_default_num_splits",
+    "eg_mla_decode_workspace_size",
+    "eg_mla_decode",
+    "eg_mla_kv_bytes_per_token",
+    "eg_mla_status_string",
+    "eg_mla_debug_gather",
+    "eg_mla_profile_begin",
+    "eg_mla_profile_end",
+]
+
+
+class EgMlaDims(ctypes.Structure):
+    _fields_ = [
+        ("num_heads", ctypes.c_int32),
+        ("d_nope", ctypes.c_int32),
+        ("d_rope", ctypes.c_int32),
+        ("d_v", ctypes.c_int32),
+        ("d_c", ctypes.c_int32),
+        ("page_size", ctypes.c_int32),
+        ("vocab", ctypes.c_int32),
+        ("dtype", ctypes.c_int32),
+        ("gate_mode", ctypes.c_int32),
+        ("softmax_scale", ctypes.c_float),
+        ("ln_eps", ctypes.c_float),
+    ]
+
+
+class EgMlaError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        super().__init__(f"{where}: {status_string(code)} ({code})")
+
+
+_lock = threading.Lock()
+_handle: Optional[ctypes.CDLL] = None
+
+
+def _declare(lib: ctypes.CDLL) -> None:
+    P, I32, SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_size_t
+    D = ctypes.POINTER(EgMlaDims)
+    lib.eg_mla_append_latent.argtypes = [D, P, P, P, P, P, P, P, I32, P, I32, I32, P, P]
+    lib.eg_mla_append_latent.restype = ctypes.c_int
+    lib.eg_mla_default_num_splits.argtypes = [ctypes.POINTER(I32)]
+    lib.eg_mla_default_num_splits.restype = ctypes.c_int
+    lib.eg_mla_decode_workspace_size.argtypes = [D, I32, I32]
+    lib.eg_mla_decode_workspace_size.restype = SZ
+    lib.eg_mla_decode.argtypes = [D, P, P, P, P, P, I32, P, I32, I32, I32, P, P, P, P, P, P, I32, P, SZ, P, P]
+    lib.eg_mla_decode.restype = ctypes.c_int
+    lib.eg_mla_kv_bytes_per_token.argtypes = [D, I32, ctypes.POINTER(ctypes.c_int64)]
+    lib.eg_mla_kv_bytes_per_token.restype = ctypes.c_int
+    lib.eg_mla_status_string.argtypes = [ctypes.c_int]
+    lib.eg_mla_status_string.restype = ctypes.c_char_p
+    lib.eg_mla_debug_gather.argtypes = [D, P, P, P, P, I32, P, I32, I32, I32, P, P, P, P, P, I32, P, SZ, P, P]
+    lib.eg_mla_debug_gather.restype = ctypes.c_int
+    lib.eg_mla_profile_begin.argtypes = [I32]
+    lib.eg_mla_profile_begin.restype = ctypes.c_int
+    lib.eg_mla_profile_end.argtypes = [ctypes.POINTER(ctypes.c_double), ctypes.POINTER(I32)]
+    lib.eg_mla_profile_end.restype = ctypes.c_int
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load(build_if_needed: bool = True) -> ctypes.CDLL:
+    """Load (building first if needed) the in-tree libegmla.so."""
+    global _handle
+    with _lock:
+        if _handle is None:
+            path = _build.build() if build_if_needed else _build.LIB
+            if not os.path.exists(path):
+                raise RuntimeError(f"libegmla not built: {path}")
+            lib = ctypes.CDLL(path)
+            _declare(lib)
+            _handle = lib
+    return _handle
+
+
+def status_string(code: int) -> str:
+    if _handle is None:
+        return f"status {code}"
+    return _handle.eg_mla_status_string(code).decode()
+
+
+def _check(code: int, where: str) -> None:
+    if code != EG_MLA_OK:
+        raise EgMlaError(code, where)
+
+
+def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("device tensor expected")
+    if not t.is_contiguous():
+        raise ValueError("contiguous tensor expected")
+    return t.data_ptr()
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream
+
+
+def make_dims(num_heads, d_nope, d_rope, d_v, d_c, vocab, dtype="bf16", gate=True, page_size=64,
+              softmax_scale=0.0, ln_eps=1e-5) -> EgMlaDims:
+    return EgMlaDims(num_heads, d_nope, d_rope, d_v, d_c, page_size, vocab,
+                     EG_MLA_BF16 if dtype == "bf16" else EG_MLA_FP32,
+                     EG_MLA_GATE_MUL_LN if gate else EG_MLA_GATE_NONE, softmax_scale, ln_eps)
+
+
+def eg_mla_default_num_splits() -> int:
+    out = ctypes.c_int32(0)
+    _check(load().eg_mla_default_num_splits(ctypes.byref(out)), "eg_mla_default_num_splits")
+    return int(out.value)
+
+
+def eg_mla_decode_workspace_size(dims: EgMlaDims, batch: int, num_splits: int = 0) -> int:
+    n = load().eg_mla_decode_workspace_size(ctypes.byref(dims), batch, num_splits)
+    if n == 0:
+        raise EgMlaError(EG_MLA_ERR_UNSUPPORTED, "eg_mla_decode_workspace_size")
+    return int(n)
+
+
+def eg_mla_kv_bytes_per_token(dims: EgMlaDims, n_layers: int) -> int:
+    out = ctypes.c_int64(0)
+    _check(load().eg_mla_kv_bytes_per_token(ctypes.byref(dims), n_layers, ctypes.byref(out)),
+           "eg_mla_kv_bytes_per_token")
+    return int(out.value)
+
+
+def eg_mla_append_latent(dims: EgMlaDims, c_pool, krope_pool, id_pool, c_new, krope_new, ids_new,
+                         block_table, positions, dev_status=None, stream=None) -> None:
+    code = load().eg_mla_append_latent(
+        ctypes.byref(dims), _ptr(c_pool), _ptr(krope_pool), _ptr(id_pool), _ptr(c_new), _ptr(krope_new),
+        _ptr(ids_new), _ptr(block_table), block_table.shape[1], _ptr(positions), positions.shape[0],
+        c_pool.shape[0], _ptr(dev_status), _stream(stream))
+    _check(code, "eg_mla_append_latent")
+
+
+def eg_mla_decode(dims: EgMlaDims, q, c_pool, krope_pool, id_pool, block_table, seq_lens, max_seq_len,
+                  gate_table, ln_gamma, ln_beta, w_uk, w_uv, out, workspace, num_splits=0,
+                  dev_status=None, stream=None) -> None:
+    code = load().eg_mla_decode(
+        ctypes.byref(dims), _ptr(q), _ptr(c_pool), _ptr(krope_pool), _ptr(id_pool), _ptr(block_table),
+        block_table.shape[1], _ptr(seq_lens), int(max_seq_len), seq_lens.shape[0], c_pool.shape[0],
+        _ptr(gate_table), _ptr(ln_gamma), _ptr(ln_beta), _ptr(w_uk), _ptr(w_uv), _ptr(out), num_splits,
+        _ptr(workspace), workspace.numel() * workspace.element_size(), _ptr(dev_status), _stream(stream))
+    _check(code, "eg_mla_decode")
+
+
+def eg_mla_debug_gather(dims: EgMlaDims, c_pool, krope_pool, id_pool, block_table, seq_lens, max_seq_len,
+                        gate_table, c_out, kr_out, ids_out, g_out, workspace, num_splits=0,
+                        dev_status=None, stream=None) -> None:
+    code = load().eg_mla_debug_gather(
+        ctypes.byref(dims), _ptr(c_pool), _ptr(krope_pool), _ptr(id_pool), _ptr(block_table),
+        block_table.shape[1], _ptr(seq_lens), int(max_seq_len), seq_lens.shape[0], c_pool.shape[0],
+        _ptr(gate_table), _ptr(c_out), _ptr(kr_out), _ptr(ids_out), _ptr(g_out), num_splits,
+        _ptr(workspace), workspace.numel() * workspace.element_size(), _ptr(dev_status), _stream(stream))
+    _check(code, "eg_mla_debug_gather")
+
+
+def eg_mla_profile_begin(max_launches: int) -> None:
+    _check(load().eg_mla_profile_begin(max_launches), "eg_mla_profile_begin")
+
+
+def eg_mla_profile_end():
+    """(summed decode-kernel milliseconds, launches timed)."""
+    ms = ctypes.c_double(0)
+    n = ctypes.c_int32(0)
+    _check(load().eg_mla_profile_end(ctypes.byref(ms), ctypes.byref(n)), "eg_mla_profile_end")
+    return float(ms.value), int(n.value)
+
+
+def default_scale(d_nope: int, d_rope: int) -> float:
+    return 1.0 / math.sqrt(d_nope + d_rope)

@@ -1,0 +1,355 @@
+// egmla_api.cu - the C ABI of libegmla: argument validation, workspace
+// carving, TMA descriptor encoding and kernel launches.  See include/egmla.h
+// for the contract of every entry point.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "../../include/egmla.h"
+#include "egmla_common.cuh"
+#include "egmla_kernels.h"
+
+namespace {
+
+using egmla::DecodeArgs;
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+int elem_bytes(const eg_mla_dims* d) { return d->dtype == EG_MLA_BF16 ? 2 : 4; }
+
+bool is_tc_path(const eg_mla_dims* d) { return d->dtype == EG_MLA_BF16; }
+
+// shape support; returns EG_MLA_OK or the error code
+int check_dims(const eg_mla_dims* d) {
+  if (d == nullptr) return EG_MLA_ERR_INVALID_ARG;
+  if (d->num_heads <= 0 || d->d_nope <= 0 || d->d_rope <= 0 || d->d_v <= 0 || d->d_c <= 0 ||
+      d->page_size <= 0 || d->vocab <= 0)
+    return EG_MLA_ERR_INVALID_ARG;
+  if (d->gate_mode != EG_MLA_GATE_NONE && d->gate_mode != EG_MLA_GATE_MUL_LN) return EG_MLA_ERR_INVALID_ARG;
+  if (d->page_size != egmla::kPage) return EG_MLA_ERR_UNSUPPORTED;
+  if (d->dtype == EG_MLA_BF16) {
+    if (d->num_heads != 16 || d->d_rope != 64) return EG_MLA_ERR_UNSUPPORTED;
+    if (!egmla::tc_supported(d->d_c, d->gate_mode)) return EG_MLA_ERR_UNSUPPORTED;
+    if (d->d_nope % 8 || d->d_nope > 256 || d->d_v % 8 || d->d_v > 256) return EG_MLA_ERR_UNSUPPORTED;
+    return EG_MLA_OK;
+  }
+  if (d->dtype == EG_MLA_FP32) {
+    if (d->num_heads > 16 || d->d_c > 512 || d->d_c % 4 || d->d_rope > 64 || d->d_rope % 4 ||
+        d->d_nope > 256 || d->d_v > 256)
+      return EG_MLA_ERR_UNSUPPORTED;
+    return EG_MLA_OK;
+  }
+  return EG_MLA_ERR_INVALID_ARG;
+}
+
+int resolve_splits(int32_t num_splits, int32_t* out) {
+  if (num_splits < 0) return EG_MLA_ERR_INVALID_ARG;
+  if (num_splits > 0) {
+    *out = num_splits;
+    return EG_MLA_OK;
+  }
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return EG_MLA_ERR_CUDA;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return EG_MLA_ERR_CUDA;
+  *out = sms > 0 ? sms : 1;
+  return EG_MLA_OK;
+}
+
+// cuTensorMapEncodeTiled through the runtime's driver entry point (no libcuda link)
+using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                              const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                              CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeFn get_encode() {
+  static EncodeFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeFn>(p);
+  });
+  return fn;
+}
+
+// 2D view [rows, cols] of a bf16 pool, boxes of 64 columns (128 bytes) x 64 rows,
+// 128-byte swizzle (the layout the MMA descriptors of the decode kernel expect)
+bool encode_pool_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols) {
+  EncodeFn enc = get_encode();
+  if (enc == nullptr) return false;
+  const cuuint64_t dims[2] = {cols, rows};
+  const cuuint64_t strides[1] = {cols * 2};
+  const cuuint32_t box[2] = {64, 64};
+  const cuuint32_t estr[2] = {1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+float resolve_scale(const eg_mla_dims* d) {
+  return d->softmax_scale > 0.f ? d->softmax_scale : 1.0f / std::sqrt(static_cast<float>(d->d_nope + d->d_rope));
+}
+
+int fill_decode_args(DecodeArgs& a, const eg_mla_dims* d, const void* c_pool, const void* krope_pool,
+                     const int32_t* id_pool, const int32_t* block_table, int32_t max_pages,
+                     const int32_t* seq_lens, int32_t max_seq_len, int32_t batch, int32_t num_pages,
+                     const void* gate_table, int32_t num_splits, void* workspace, size_t workspace_bytes,
+                     int32_t* dev_status) {
+  int rc = check_dims(d);
+  if (rc != EG_MLA_OK) return rc;
+  if (batch < 0 || num_pages <= 0 || max_pages <= 0 || max_seq_len < 0) return EG_MLA_ERR_INVALID_ARG;
+  if (static_cast<int64_t>(max_seq_len) > static_cast<int64_t>(max_pages) * d->page_size)
+    return EG_MLA_ERR_INVALID_ARG;
+  if (static_cast<int64_t>(num_pages) * d->page_size > INT32_MAX) return EG_MLA_ERR_UNSUPPORTED;
+  if (c_pool == nullptr || krope_pool == nullptr || block_table == nullptr || seq_lens == nullptr)
+    return EG_MLA_ERR_INVALID_ARG;
+  if (d->gate_mode == EG_MLA_GATE_MUL_LN && (id_pool == nullptr || gate_table == nullptr))
+    return EG_MLA_ERR_INVALID_ARG;
+  if (!aligned(c_pool, 16) || !aligned(krope_pool, 16) || (id_pool && !aligned(id_pool, 16)) ||
+      (gate_table && !aligned(gate_table, 16)))
+    return EG_MLA_ERR_INVALID_ARG;
+  int32_t splits = 0;
+  rc = resolve_splits(num_splits, &splits);
+  if (rc != EG_MLA_OK) return rc;
+  const egmla::WorkspaceLayout wl =
+      egmla::workspace_layout(batch, splits, d->num_heads, d->d_c, d->d_rope, is_tc_path(d));
+  if (workspace == nullptr || workspace_bytes < wl.total || !aligned(workspace, 256)) return EG_MLA_ERR_WORKSPACE;
+  std::memset(&a, 0, sizeof(a));
+  a.H = d->num_heads;
+  a.d_nope = d->d_nope;
+  a.d_rope = d->d_rope;
+  a.d_v = d->d_v;
+  a.d_c = d->d_c;
+  a.page_size = d->page_size;
+  a.vocab = d->vocab;
+  a.dtype = d->dtype;
+  a.gate = d->gate_mode == EG_MLA_GATE_MUL_LN ? 1 : 0;
+  a.scale_log2 = resolve_scale(d) * 1.4426950408889634f;
+  a.eps = d->ln_eps > 0.f ? d->ln_eps : 1e-5f;
+  a.c_pool = c_pool;
+  a.kr_pool = krope_pool;
+  a.id_pool = id_pool;
+  a.block_table = block_table;
+  a.max_pages = max_pages;
+  a.seq_lens = seq_lens;
+  a.max_seq_len = max_seq_len;
+  a.batch = batch;
+  a.num_pages = num_pages;
+  a.gate_table = gate_table;
+  a.num_splits = splits;
+  a.workspace = workspace;
+  a.status = dev_status;
+  return EG_MLA_OK;
+}
+
+int to_status(cudaError_t e) { return e == cudaSuccess ? EG_MLA_OK : EG_MLA_ERR_CUDA; }
+
+// per-launch event pairs around the split-KV kernel (eg_mla_profile_begin/end)
+struct Profiler {
+  std::mutex mu;
+  bool active = false;
+  std::vector<cudaEvent_t> ev;  // 2 per launch
+  int used = 0;
+} g_prof;
+
+void prof_mark(cudaStream_t st, bool before) {
+  std::lock_guard<std::mutex> lk(g_prof.mu);
+  if (!g_prof.active) return;
+  const int pairs = static_cast<int>(g_prof.ev.size() / 2);
+  if (before) {
+    if (g_prof.used < pairs) cudaEventRecord(g_prof.ev[2 * g_prof.used], st);
+  } else if (g_prof.used < pairs) {
+    cudaEventRecord(g_prof.ev[2 * g_prof.used + 1], st);
+    ++g_prof.used;
+  }
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* eg_mla_status_string(int status) {
+  switch (status) {
+    case EG_MLA_OK: return "ok";
+    case EG_MLA_ERR_INVALID_ARG: return "invalid argument";
+    case EG_MLA_ERR_UNSUPPORTED: return "unsupported shape";
+    case EG_MLA_ERR_CUDA: return "CUDA runtime error";
+    case EG_MLA_ERR_OUT_OF_RANGE: return "page id or token id out of range";
+    case EG_MLA_ERR_TIMEOUT: return "device pipeline wait timed out";
+    case EG_MLA_ERR_WORKSPACE: return "workspace too small or misaligned";
+    default: return "unknown status";
+  }
+}
+
+int eg_mla_kv_bytes_per_token(const eg_mla_dims* dims, int32_t n_layers, int64_t* bytes_out) {
+  if (dims == nullptr || bytes_out == nullptr || n_layers < 0) return EG_MLA_ERR_INVALID_ARG;
+  if (dims->d_c <= 0 || dims->d_rope < 0) return EG_MLA_ERR_INVALID_ARG;
+  const int64_t per_layer = static_cast<int64_t>(dims->d_c + dims->d_rope) * elem_bytes(dims) +
+                            (dims->gate_mode == EG_MLA_GATE_MUL_LN ? 4 : 0);
+  *bytes_out = per_layer * n_layers;
+  return EG_MLA_OK;
+}
+
+int eg_mla_default_num_splits(int32_t* out_splits) {
+  if (out_splits == nullptr) return EG_MLA_ERR_INVALID_ARG;
+  return resolve_splits(0, out_splits);
+}
+
+size_t eg_mla_decode_workspace_size(const eg_mla_dims* dims, int32_t batch, int32_t num_splits) {
+  if (check_dims(dims) != EG_MLA_OK || batch < 0) return 0;
+  int32_t splits = 0;
+  if (resolve_splits(num_splits, &splits) != EG_MLA_OK) return 0;
+  return egmla::workspace_layout(batch, splits, dims->num_heads, dims->d_c, dims->d_rope, is_tc_path(dims)).total;
+}
+
+int eg_mla_append_latent(const eg_mla_dims* dims, void* c_pool, void* krope_pool, int32_t* id_pool,
+                         const void* c_new, const void* krope_new, const int32_t* ids_new,
+                         const int32_t* block_table, int32_t max_pages_per_seq, const int32_t* positions,
+                         int32_t batch, int32_t num_pages, int32_t* dev_status, void* stream) {
+  int rc = check_dims(dims);
+  if (rc != EG_MLA_OK) return rc;
+  if (batch < 0 || num_pages <= 0 || max_pages_per_seq <= 0) return EG_MLA_ERR_INVALID_ARG;
+  if (batch == 0) return EG_MLA_OK;
+  if (!c_pool || !krope_pool || !c_new || !krope_new || !block_table || !positions) return EG_MLA_ERR_INVALID_ARG;
+  const int eb = elem_bytes(dims);
+  const int crb = dims->d_c * eb, krb = dims->d_rope * eb;
+  if (crb % 16 || krb % 16) return EG_MLA_ERR_UNSUPPORTED;
+  if (!aligned(c_pool, 16) || !aligned(krope_pool, 16) || !aligned(c_new, 16) || !aligned(krope_new, 16))
+    return EG_MLA_ERR_INVALID_ARG;
+  egmla::AppendArgs a;
+  a.c_pool = c_pool;
+  a.kr_pool = krope_pool;
+  a.id_pool = id_pool;
+  a.c_new = c_new;
+  a.kr_new = krope_new;
+  a.ids_new = ids_new;
+  a.block_table = block_table;
+  a.max_pages = max_pages_per_seq;
+  a.positions = positions;
+  a.batch = batch;
+  a.num_pages = num_pages;
+  a.page_size = dims->page_size;
+  a.c_row_bytes = crb;
+  a.kr_row_bytes = krb;
+  a.status = dev_status;
+  return to_status(egmla::launch_append(a, static_cast<cudaStream_t>(stream)));
+}
+
+int eg_mla_decode(const eg_mla_dims* dims, const void* q, const void* c_pool, const void* krope_pool,
+                  const int32_t* id_pool, const int32_t* block_table, int32_t max_pages_per_seq,
+                  const int32_t* seq_lens, int32_t max_seq_len, int32_t batch, int32_t num_pages,
+                  const void* gate_table, const float* ln_gamma, const float* ln_beta, const void* w_uk,
+                  const void* w_uv, void* out, int32_t num_splits, void* workspace, size_t workspace_bytes,
+                  int32_t* dev_status, void* stream) {
+  DecodeArgs a;
+  int rc = fill_decode_args(a, dims, c_pool, krope_pool, id_pool, block_table, max_pages_per_seq, seq_lens,
+                            max_seq_len, batch, num_pages, gate_table, num_splits, workspace, workspace_bytes,
+                            dev_status);
+  if (rc != EG_MLA_OK) return rc;
+  if (batch == 0) return EG_MLA_OK;
+  if (q == nullptr || w_uk == nullptr || w_uv == nullptr || out == nullptr) return EG_MLA_ERR_INVALID_ARG;
+  a.q = q;
+  a.ln_gamma = ln_gamma;
+  a.ln_beta = ln_beta;
+  a.w_uk = w_uk;
+  a.w_uv = w_uv;
+  a.out = out;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (is_tc_path(dims)) {
+    CUtensorMap maps[2];
+    const uint64_t rows = static_cast<uint64_t>(num_pages) * dims->page_size;
+    if (!encode_pool_map(&maps[0], c_pool, rows, dims->d_c) ||
+        !encode_pool_map(&maps[1], krope_pool, rows, dims->d_rope))
+      return EG_MLA_ERR_CUDA;
+    cudaError_t e = egmla::launch_prologue_tc(a, st);
+    if (e == cudaSuccess) {
+      prof_mark(st, true);
+      e = egmla::launch_decode_tc(a, maps, false, st);
+      prof_mark(st, false);
+    }
+    if (e == cudaSuccess) e = egmla::launch_combine(a, true, st);
+    return to_status(e);
+  }
+  cudaError_t e = egmla::launch_decode_f32(a, st);
+  if (e == cudaSuccess) e = egmla::launch_combine(a, false, st);
+  return to_status(e);
+}
+
+int eg_mla_profile_begin(int32_t max_launches) {
+  if (max_launches <= 0) return EG_MLA_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> lk(g_prof.mu);
+  for (cudaEvent_t e : g_prof.ev) cudaEventDestroy(e);
+  g_prof.ev.assign(2 * static_cast<size_t>(max_launches), nullptr);
+  for (auto& e : g_prof.ev)
+    if (cudaEventCreate(&e) != cudaSuccess) {
+      g_prof.ev.clear();
+      g_prof.active = false;
+      return EG_MLA_ERR_CUDA;
+    }
+  g_prof.used = 0;
+  g_prof.active = true;
+  return EG_MLA_OK;
+}
+
+int eg_mla_profile_end(double* ms_sum, int32_t* launches) {
+  if (ms_sum == nullptr || launches == nullptr) return EG_MLA_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> lk(g_prof.mu);
+  double total = 0.0;
+  int rc = EG_MLA_OK;
+  for (int i = 0; i < g_prof.used; ++i) {
+    float ms = 0.f;
+    if (cudaEventSynchronize(g_prof.ev[2 * i + 1]) != cudaSuccess ||
+        cudaEventElapsedTime(&ms, g_prof.ev[2 * i], g_prof.ev[2 * i + 1]) != cudaSuccess) {
+      rc = EG_MLA_ERR_CUDA;
+      break;
+    }
+    total += ms;
+  }
+  *ms_sum = total;
+  *launches = g_prof.used;
+  for (cudaEvent_t e : g_prof.ev) cudaEventDestroy(e);
+  g_prof.ev.clear();
+  g_prof.used = 0;
+  g_prof.active = false;
+  return rc;
+}
+
+int eg_mla_debug_gather(const eg_mla_dims* dims, const void* c_pool, const void* krope_pool,
+                        const int32_t* id_pool, const int32_t* block_table, int32_t max_pages_per_seq,
+                        const int32_t* seq_lens, int32_t max_seq_len, int32_t batch, int32_t num_pages,
+                        const void* gate_table, void* c_out, void* kr_out, int32_t* ids_out, void* g_out,
+                        int32_t num_splits, void* workspace, size_t workspace_bytes, int32_t* dev_status,
+                        void* stream) {
+  if (dims == nullptr || dims->dtype != EG_MLA_BF16 || dims->gate_mode != EG_MLA_GATE_MUL_LN ||
+      (dims->d_c != 192 && dims->d_c != 256))
+    return EG_MLA_ERR_UNSUPPORTED;
+  DecodeArgs a;
+  int rc = fill_decode_args(a, dims, c_pool, krope_pool, id_pool, block_table, max_pages_per_seq, seq_lens,
+                            max_seq_len, batch, num_pages, gate_table, num_splits, workspace, workspace_bytes,
+                            dev_status);
+  if (rc != EG_MLA_OK) return rc;
+  if (batch == 0) return EG_MLA_OK;
+  if (!c_out || !kr_out || !ids_out || !g_out) return EG_MLA_ERR_INVALID_ARG;
+  a.dump_c = c_out;
+  a.dump_kr = kr_out;
+  a.dump_ids = ids_out;
+  a.dump_g = g_out;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  CUtensorMap maps[2];
+  const uint64_t rows = static_cast<uint64_t>(num_pages) * dims->page_size;
+  if (!encode_pool_map(&maps[0], c_pool, rows, dims->d_c) || !encode_pool_map(&maps[1], krope_pool, rows, dims->d_rope))
+    return EG_MLA_ERR_CUDA;
+  a.q = nullptr;  // prologue computes the page prefix sums only
+  cudaError_t e = egmla::launch_prologue_tc(a, st);
+  if (e == cudaSuccess) e = egmla::launch_decode_tc(a, maps, true, st);
+  return to_status(e);
+}
+
+}  // extern "C"

@@ -1,0 +1,78 @@
+// egmla_common.cuh - launch-independent pieces shared by the decode kernels:
+// the workspace layout and the split-KV work schedule.
+//
+// Split-KV schedule.  The cache pages of all sequences are numbered globally in
+// sequence order (prefix sums cu_pages[b] = sum_{b'<b} ceil(L_b'/P)) and cut
+// into `num_splits` equal contiguous ranges of `chunk` pages, one per CTA.  A
+// CTA may therefore cover the tail of one sequence and the head of the next;
+// it emits one partial result (running max m, denominator l, un-normalised
+// latent output) per sequence it touches.  Partial slot of (CTA c, sequence b)
+// is c + b: the CTA ranges of consecutive sequences overlap in at most one CTA,
+// so these slots never collide and there are at most num_splits + batch of them.
+#pragma once
+#include <cstddef>
+#include <cstdint>
+
+namespace egmla {
+
+constexpr int kPage = 64;
+
+__host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Bytes of the per-sequence prepared query block of the tensor-core path:
+// q^ (*) gamma as a bf16 MMA operand [16 heads x d_c], q^R as a bf16 operand
+// [16 x d_rope], then per-head fp32 sums w_h = sum_f (q^ gamma)_hf and
+// b_h = q^_h . beta, padded to 16-byte multiples.
+__host__ __device__ inline size_t qprep_bytes_tc(int d_c, int d_rope) {
+  return static_cast<size_t>(16) * d_c * 2 + static_cast<size_t>(16) * d_rope * 2 + 128;
+}
+
+// fp32 path: q^ [H, d_c] and q^R [H, d_rope] in fp32.
+__host__ __device__ inline size_t qprep_bytes_f32(int H, int d_c, int d_rope) {
+  return align_up(static_cast<size_t>(H) * (d_c + d_rope) * 4, 16);
+}
+
+struct WorkspaceLayout {
+  size_t off_cu, off_qprep, off_ml, off_o, total;
+  size_t qprep_stride;
+  int num_slots;
+};
+
+__host__ __device__ inline WorkspaceLayout workspace_layout(int batch, int num_splits, int H, int d_c,
+                                                            int d_rope, bool tc_path) {
+  WorkspaceLayout w;
+  w.num_slots = num_splits + batch;
+  w.qprep_stride = tc_path ? qprep_bytes_tc(d_c, d_rope) : qprep_bytes_f32(H, d_c, d_rope);
+  size_t off = 0;
+  w.off_cu = off;
+  off = align_up(off + static_cast<size_t>(batch + 1) * 4, 256);
+  w.off_qprep = off;
+  off = align_up(off + static_cast<size_t>(batch) * w.qprep_stride, 256);
+  w.off_ml = off;
+  off = align_up(off + static_cast<size_t>(w.num_slots) * H * 2 * 4, 256);
+  w.off_o = off;
+  off = align_up(off + static_cast<size_t>(w.num_slots) * H * d_c * 4, 256);
+  w.total = off;
+  return w;
+}
+
+// pages per split for the total page count
+__host__ __device__ inline int split_chunk(int total_pages, int num_splits) {
+  int c = (total_pages + num_splits - 1) / num_splits;
+  return c < 1 ? 1 : c;
+}
+
+// first sequence whose page range contains global page g (cu has batch+1 entries,
+// non-decreasing, cu[0] = 0, g < cu[batch])
+__device__ inline int find_sequence(const int32_t* cu, int batch, int g) {
+  int lo = 0, hi = batch - 1;
+  while (lo < hi) {
+    int mid = (lo + hi + 1) >> 1;
+    if (__ldg(cu + mid) <= g) lo = mid; else hi = mid - 1;
+  }
+  // skip empty sequences that share the same start
+  while (lo < batch - 1 && __ldg(cu + lo + 1) <= g) ++lo;
+  return lo;
+}
+
+}  // namespace egmla

@@ -1,0 +1,69 @@
+// egmla_kernels.h - internal launch interface between the C-ABI layer
+// (egmla_api.cu) and the kernels.  Not part of the public ABI.
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+namespace egmla {
+
+struct AppendArgs {
+  void* c_pool;
+  void* kr_pool;
+  int32_t* id_pool;
+  const void* c_new;
+  const void* kr_new;
+  const int32_t* ids_new;
+  const int32_t* block_table;
+  int max_pages;
+  const int32_t* positions;
+  int batch, num_pages, page_size;
+  int c_row_bytes, kr_row_bytes;
+  int32_t* status;
+};
+
+struct DecodeArgs {
+  // shapes
+  int H, d_nope, d_rope, d_v, d_c, page_size, vocab;
+  int dtype;  // 0 bf16, 1 fp32
+  int gate;   // 0 none, 1 mul+LN
+  float scale_log2;  // softmax scale * log2(e)
+  float eps;
+  // tensors
+  const void* q;
+  const void* c_pool;
+  const void* kr_pool;
+  const int32_t* id_pool;
+  const int32_t* block_table;
+  int max_pages;
+  const int32_t* seq_lens;
+  int max_seq_len;
+  int batch, num_pages;
+  const void* gate_table;
+  const float* ln_gamma;
+  const float* ln_beta;
+  const void* w_uk;
+  const void* w_uv;
+  void* out;
+  int num_splits;
+  void* workspace;
+  int32_t* status;
+  // cache-read test entry outputs (eg_mla_debug_gather)
+  void* dump_c;
+  void* dump_kr;
+  int32_t* dump_ids;
+  void* dump_g;
+};
+
+cudaError_t launch_append(const AppendArgs& a, cudaStream_t st);
+cudaError_t launch_prologue_tc(const DecodeArgs& a, cudaStream_t st);
+cudaError_t launch_decode_f32(const DecodeArgs& a, cudaStream_t st);
+cudaError_t launch_combine(const DecodeArgs& a, bool tc_path, cudaStream_t st);
+// tensor-core split-KV kernel; `maps` = {c_pool map, kr_pool map}
+cudaError_t launch_decode_tc(const DecodeArgs& a, const CUtensorMap* maps, bool dump, cudaStream_t st);
+// true if the bf16 tensor-core path has a kernel for these shapes
+bool tc_supported(int d_c, int gate);
+
+}  // namespace egmla

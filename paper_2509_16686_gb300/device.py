@@ -1,0 +1,120 @@
+"""Device-side plumbing: upload a synthetic decode step to HBM and run it
+through the C ABI (append of the new token, then decode).
+
+PyTorch only allocates device memory and provides the stream here; the work
+itself is done by libegmla's kernels.
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import Optional
+
+import numpy as np
+import torch
+
+from . import _lib
+from .synth import Case
+
+
+def to_device_array(a: np.ndarray, dtype: str, device) -> torch.Tensor:
+    """Stored bits -> device tensor of the model dtype (bf16 from uint16 bits)."""
+    if dtype == "bf16" and a.dtype == np.uint16:
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(device)
+    if a.dtype == np.int32:
+        return torch.from_numpy(np.ascontiguousarray(a)).to(device)
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(device)
+
+
+def bf16_tensor_to_bits(t: torch.Tensor) -> np.ndarray:
+    return t.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
+
+
+@dataclasses.dataclass
+class DeviceCase:
+    dims: _lib.EgMlaDims
+    dtype: str
+    c_pool: torch.Tensor
+    kr_pool: torch.Tensor
+    id_pool: torch.Tensor
+    block_table: torch.Tensor
+    seq_lens: torch.Tensor
+    positions: torch.Tensor
+    c_new: torch.Tensor
+    kr_new: torch.Tensor
+    ids_new: torch.Tensor
+    q: torch.Tensor
+    gate_table: torch.Tensor
+    ln_gamma: torch.Tensor
+    ln_beta: torch.Tensor
+    w_uk: torch.Tensor
+    w_uv: torch.Tensor
+    out: torch.Tensor
+    workspace: torch.Tensor
+    status: torch.Tensor
+    max_seq_len: int
+    num_splits: int
+
+    @property
+    def batch(self) -> int:
+        return int(self.seq_lens.shape[0])
+
+    def append(self, stream=None) -> None:
+        _lib.eg_mla_append_latent(self.dims, self.c_pool, self.kr_pool, self.id_pool, self.c_new, self.kr_new,
+                                  self.ids_new, self.block_table, self.positions, self.status, stream)
+
+    def decode(self, stream=None, out: Optional[torch.Tensor] = None) -> torch.Tensor:
+        o = self.out if out is None else out
+        _lib.eg_mla_decode(self.dims, self.q, self.c_pool, self.kr_pool, self.id_pool, self.block_table,
+                           self.seq_lens, self.max_seq_len, self.gate_table, self.ln_gamma, self.ln_beta,
+                           self.w_uk, self.w_uv, o, self.workspace, self.num_splits, self.status, stream)
+        return o
+
+    def step(self, stream=None) -> torch.Tensor:
+        """One decode step: append the new token, then attend over the cache."""
+        self.append(stream)
+        return self.decode(stream)
+
+    def read_status(self) -> int:
+        return int(self.status.item())
+
+
+def dims_of(case: Case) -> _lib.EgMlaDims:
+    d = case.dims
+    return _lib.make_dims(d.num_heads, d.d_nope, d.d_rope, d.d_v, d.d_c, d.vocab, dtype=d.dtype, gate=d.gate,
+                          page_size=d.page_size, softmax_scale=d.softmax_scale, ln_eps=d.ln_eps)
+
+
+def upload(case: Case, device="cuda", num_splits: int = 0) -> DeviceCase:
+    d = case.dims
+    dt = d.dtype
+    dims = dims_of(case)
+    B = case.batch
+    ws_bytes = _lib.eg_mla_decode_workspace_size(dims, B, num_splits)
+    out_dtype = torch.bfloat16 if dt == "bf16" else torch.float32
+    return DeviceCase(
+        dims=dims, dtype=dt,
+        c_pool=to_device_array(case.c_pool, dt, device),
+        kr_pool=to_device_array(case.kr_pool, dt, device),
+        id_pool=to_device_array(case.id_pool, dt, device),
+        block_table=to_device_array(case.block_table, dt, device),
+        seq_lens=to_device_array(case.seq_lens, dt, device),
+        positions=to_device_array(case.positions(), dt, device),
+        c_new=to_device_array(case.c_new, dt, device),
+        kr_new=to_device_array(case.kr_new, dt, device),
+        ids_new=to_device_array(case.ids_new, dt, device),
+        q=to_device_array(case.q, dt, device),
+        gate_table=to_device_array(case.gate_table, dt, device),
+        ln_gamma=torch.from_numpy(case.ln_gamma.astype(np.float32)).to(device),
+        ln_beta=torch.from_numpy(case.ln_beta.astype(np.float32)).to(device),
+        w_uk=to_device_array(case.w_uk, dt, device),
+        w_uv=to_device_array(case.w_uv, dt, device),
+        out=torch.empty((B, d.num_heads, d.d_v), dtype=out_dtype, device=device),
+        workspace=torch.empty(ws_bytes, dtype=torch.uint8, device=device),
+        status=torch.zeros(1, dtype=torch.int32, device=device),
+        max_seq_len=int(case.seq_lens.max()) if B else 0,
+        num_splits=num_splits,
+    )
+
+
+def output_f64(t: torch.Tensor) -> np.ndarray:
+    return t.detach().float().cpu().numpy().astype(np.float64)

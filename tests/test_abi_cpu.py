@@ -1,0 +1,112 @@
+"""Host-side checks of the C ABI that need no GPU: the library builds and loads,
+exports every symbol include/egmla.h declares, and its host-only calls and
+argument validation behave as documented."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2509_16686_gb300 import _lib
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "egmla.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(eg_mla_[a-z_0-9]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    return _lib.load()
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert len(names) >= 7
+    for n in names:
+        assert hasattr(lib, n), n
+    assert sorted(_lib.EXPORTED) == names
+
+
+def test_dims_struct_matches_header():
+    src = open(os.path.join(ROOT, "include", "egmla.h")).read()
+    body = re.search(r"typedef struct \{(.*?)\} eg_mla_dims;", src, flags=re.S).group(1)
+    fields = re.findall(r"(int32_t|float)\s+([a-z_0-9, ]+);", body)
+    flat = []
+    for ty, names in fields:
+        for n in names.split(","):
+            flat.append((ty, n.strip()))
+    assert [n for _, n in flat] == [n for n, _ in _lib.EgMlaDims._fields_]
+    assert ctypes.sizeof(_lib.EgMlaDims) == 4 * len(flat)
+
+
+def test_status_strings(lib):
+    for code in range(0, -7, -1):
+        assert lib.eg_mla_status_string(code)
+    assert b"unknown" in lib.eg_mla_status_string(42)
+
+
+def test_kv_bytes_per_token():
+    d = _lib.make_dims(16, 128, 64, 128, 256, 32000)
+    assert _lib.eg_mla_kv_bytes_per_token(d, 1) == 644
+    assert _lib.eg_mla_kv_bytes_per_token(d, 24) == 24 * 644
+    d = _lib.make_dims(16, 128, 64, 128, 512, 50000, gate=False)
+    assert _lib.eg_mla_kv_bytes_per_token(d, 1) == 1152
+    d = _lib.make_dims(4, 32, 16, 32, 64, 1000, dtype="fp32")
+    assert _lib.eg_mla_kv_bytes_per_token(d, 1) == (64 + 16) * 4 + 4
+
+
+def test_workspace_size_and_shape_support():
+    d = _lib.make_dims(16, 128, 64, 128, 256, 32000)
+    n1 = _lib.eg_mla_decode_workspace_size(d, 8, 152)
+    n2 = _lib.eg_mla_decode_workspace_size(d, 8, 304)
+    assert n2 > n1 > 0 and n1 % 256 == 0
+    # partials: (splits + batch) x heads x (d_c + 2) floats dominate
+    assert n1 >= (152 + 8) * 16 * (256 + 2) * 4
+    bad = _lib.make_dims(8, 128, 64, 128, 256, 32000)          # bf16 path is built for 16 heads
+    assert _lib.load().eg_mla_decode_workspace_size(ctypes.byref(bad), 8, 152) == 0
+    bad = _lib.make_dims(16, 128, 64, 128, 512, 32000, gate=True)  # gated d_c 512 not built
+    assert _lib.load().eg_mla_decode_workspace_size(ctypes.byref(bad), 8, 152) == 0
+
+
+def test_invalid_arguments_are_rejected_before_launch(lib):
+    d = _lib.make_dims(16, 128, 64, 128, 256, 32000)
+    P = ctypes.c_void_p
+    fake = P(0x10000)  # never dereferenced: validation fails first
+    rc = lib.eg_mla_decode(ctypes.byref(d), fake, None, fake, fake, fake, 4, fake, 256, 2, 8, fake, None, None,
+                           fake, fake, fake, 152, fake, 1 << 20, None, None)
+    assert rc == _lib.EG_MLA_ERR_INVALID_ARG
+    # max_seq_len beyond the block table's reach
+    rc = lib.eg_mla_decode(ctypes.byref(d), fake, fake, fake, fake, fake, 4, fake, 257, 2, 8, fake, None, None,
+                           fake, fake, fake, 152, fake, 1 << 20, None, None)
+    assert rc == _lib.EG_MLA_ERR_INVALID_ARG
+    # workspace too small
+    rc = lib.eg_mla_decode(ctypes.byref(d), fake, fake, fake, fake, fake, 4, fake, 256, 2, 8, fake, None, None,
+                           fake, fake, fake, 152, fake, 16, None, None)
+    assert rc == _lib.EG_MLA_ERR_WORKSPACE
+    # misaligned cache pool
+    rc = lib.eg_mla_decode(ctypes.byref(d), fake, P(0x10008), fake, fake, fake, 4, fake, 256, 2, 8, fake, None,
+                           None, fake, fake, fake, 152, fake, 1 << 20, None, None)
+    assert rc == _lib.EG_MLA_ERR_INVALID_ARG
+    # unsupported shape
+    d2 = _lib.make_dims(16, 128, 32, 128, 256, 32000)
+    rc = lib.eg_mla_decode(ctypes.byref(d2), fake, fake, fake, fake, fake, 4, fake, 256, 2, 8, fake, None, None,
+                           fake, fake, fake, 152, fake, 1 << 20, None, None)
+    assert rc == _lib.EG_MLA_ERR_UNSUPPORTED
+    # append: null pool
+    rc = lib.eg_mla_append_latent(ctypes.byref(d), None, fake, fake, fake, fake, fake, fake, 4, fake, 2, 8, None,
+                                  None)
+    assert rc == _lib.EG_MLA_ERR_INVALID_ARG
+
+
+def test_library_has_no_oracle_dependency():
+    # the product path must not reach the test oracle
+    pkg = os.path.join(ROOT, "paper_2509_16686_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h")):
+                text = open(os.path.join(dirpath, f)).read()
+                assert "import oracle" not in text and "from oracle" not in text, f
