@@ -308,9 +308,13 @@ def main():
     value = ws * B * steps / (elapsed_ms / 1e3)
 
     # ---- the decode kernel alone: per-launch events on the launching stream
-    prof_steps = min(steps, 300)
+    prof_steps = min(steps, 200)
     _lib.eg_mla_profile_begin(prof_steps)
+    torch.cuda.synchronize()
     with torch.cuda.stream(stream):
+        # a spin kernel keeps the GPU busy while the host queues the steps, so the
+        # events bracket kernel execution rather than host launch gaps
+        torch.cuda._sleep(int(150e6))
         for i in range(prof_steps):
             dcs[i % REPLICAS].step(stream)
     stream.synchronize()

@@ -40,6 +40,7 @@ EXPORTED = [
     "eg_mla_debug_gather",
     "eg_mla_profile_begin",
     "eg_mla_profile_end",
+    "eg_mla_debug_set_trace",
 ]
 
 
@@ -90,6 +91,8 @@ def _declare(lib: ctypes.CDLL) -> None:
     lib.eg_mla_profile_begin.restype = ctypes.c_int
     lib.eg_mla_profile_end.argtypes = [ctypes.POINTER(ctypes.c_double), ctypes.POINTER(I32)]
     lib.eg_mla_profile_end.restype = ctypes.c_int
+    lib.eg_mla_debug_set_trace.argtypes = [P, ctypes.c_int64, I32]
+    lib.eg_mla_debug_set_trace.restype = ctypes.c_int
 
 
 def library_path() -> str:
@@ -205,6 +208,15 @@ def eg_mla_profile_end():
     n = ctypes.c_int32(0)
     _check(load().eg_mla_profile_end(ctypes.byref(ms), ctypes.byref(n)), "eg_mla_profile_end")
     return float(ms.value), int(n.value)
+
+
+def eg_mla_debug_set_trace(buf: Optional[torch.Tensor], ctas: int = 0) -> None:
+    """Set (or clear, with None) the decode kernel's pipeline trace buffer."""
+    if buf is None:
+        _check(load().eg_mla_debug_set_trace(None, 0, 0), "eg_mla_debug_set_trace")
+        return
+    _check(load().eg_mla_debug_set_trace(_ptr(buf), buf.numel() * buf.element_size(), ctas),
+           "eg_mla_debug_set_trace")
 
 
 def default_scale(d_nope: int, d_rope: int) -> float:

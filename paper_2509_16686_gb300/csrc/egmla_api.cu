@@ -159,6 +159,20 @@ struct Profiler {
   int used = 0;
 } g_prof;
 
+// optional pipeline trace buffer for the decode kernel (eg_mla_debug_set_trace)
+struct TraceCfg {
+  std::mutex mu;
+  void* buf = nullptr;
+  int ctas = 0, cap = 0;
+} g_trace;
+
+void apply_trace(DecodeArgs& a) {
+  std::lock_guard<std::mutex> lk(g_trace.mu);
+  a.trace = g_trace.buf;
+  a.trace_ctas = g_trace.ctas;
+  a.trace_cap = g_trace.cap;
+}
+
 void prof_mark(cudaStream_t st, bool before) {
   std::lock_guard<std::mutex> lk(g_prof.mu);
   if (!g_prof.active) return;
@@ -268,6 +282,7 @@ int eg_mla_decode(const eg_mla_dims* dims, const void* q, const void* c_pool, co
     if (!encode_pool_map(&maps[0], c_pool, rows, dims->d_c) ||
         !encode_pool_map(&maps[1], krope_pool, rows, dims->d_rope))
       return EG_MLA_ERR_CUDA;
+    apply_trace(a);
     cudaError_t e = egmla::launch_prologue_tc(a, st);
     if (e == cudaSuccess) {
       prof_mark(st, true);
@@ -280,6 +295,21 @@ int eg_mla_decode(const eg_mla_dims* dims, const void* q, const void* c_pool, co
   cudaError_t e = egmla::launch_decode_f32(a, st);
   if (e == cudaSuccess) e = egmla::launch_combine(a, false, st);
   return to_status(e);
+}
+
+int eg_mla_debug_set_trace(void* dev_buf, int64_t bytes, int32_t ctas) {
+  std::lock_guard<std::mutex> lk(g_trace.mu);
+  if (dev_buf == nullptr || bytes <= 0 || ctas <= 0) {
+    g_trace.buf = nullptr;
+    g_trace.ctas = g_trace.cap = 0;
+    return EG_MLA_OK;
+  }
+  const int64_t cap = bytes / (static_cast<int64_t>(ctas) * 4 * 16);
+  if (cap < 1 || !aligned(dev_buf, 16)) return EG_MLA_ERR_INVALID_ARG;
+  g_trace.buf = dev_buf;
+  g_trace.ctas = ctas;
+  g_trace.cap = static_cast<int>(cap > (1 << 20) ? (1 << 20) : cap);
+  return EG_MLA_OK;
 }
 
 int eg_mla_profile_begin(int32_t max_launches) {

@@ -79,55 +79,94 @@ __device__ __forceinline__ float block_sum_256(float v, float* red) {
   return s;
 }
 
-// Tensor-core path: block (b, h) computes q^_h = W_UK,h^T q^C_h in fp32 and stores
-// (q^ (*) gamma) as the bf16 B operand of the score MMA, laid out in 8x8 core
-// matrices (no swizzle, K-major): element (head n, feature k) at byte
-// (k/8)*256 + (n/8)*128 + (n%8)*16 + (k%8)*2.  q^R goes to the same layout.
-// The per-head sums w_h = sum_f bf16(q^ gamma)_f and b_h = q^_h . beta are the
-// terms the LayerNorm contributes after the MMA (see the decode kernel).
-__global__ void prologue_tc_kernel(const __nv_bfloat16* __restrict__ q,
-                                   const __nv_bfloat16* __restrict__ w_uk,
-                                   const float* __restrict__ gamma, const float* __restrict__ beta,
-                                   const int32_t* __restrict__ seq_lens, int batch, int d_nope,
-                                   int d_rope, int d_c, int page_size, uint8_t* __restrict__ qprep,
-                                   size_t qstride, int32_t* __restrict__ cu) {
-  __shared__ float qn[256];
-  __shared__ float red[8];
+// Tensor-core path: block (h, group of up to kQGroup sequences) computes
+// q^_{b,h} = W_UK,h^T q^C_{b,h} in fp32 (one latent feature per thread, W_UK,h
+// read once per group) and stores (q^ (*) gamma) as the bf16 B operand of the
+// score MMA, laid out in 8x8 core matrices (no swizzle, K-major): element
+// (head n, feature k) at byte (k/8)*256 + (n/8)*128 + (n%8)*16 + (k%8)*2.  q^R
+// goes to the same layout.  The per-head sums w_h = sum_f bf16(q^ gamma)_f and
+// b_h = q^_h . beta are the terms the LayerNorm contributes after the MMA.
+constexpr int kQGroup = 8;
+
+__global__ void __launch_bounds__(256)
+prologue_tc_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ w_uk,
+                   const float* __restrict__ gamma, const float* __restrict__ beta,
+                   const int32_t* __restrict__ seq_lens, int batch, int d_nope, int d_rope, int d_c,
+                   int page_size, uint8_t* __restrict__ qprep, size_t qstride, int32_t* __restrict__ cu) {
+  __shared__ float qn[kQGroup][256];
+  __shared__ float red[2][kQGroup][8];
   const int H = 16;
-  if (blockIdx.x == static_cast<unsigned>(batch * H)) {
+  const int ngroups = (batch + kQGroup - 1) / kQGroup;
+  if (blockIdx.x == static_cast<unsigned>(ngroups * H)) {
     page_prefix_sums(seq_lens, batch, page_size, cu);
     return;
   }
   if (q == nullptr) return;  // cache-read test entry: prefix sums only
-  const int b = blockIdx.x / H, h = blockIdx.x % H;
-  const __nv_bfloat16* qv = q + (static_cast<size_t>(b) * H + h) * (d_nope + d_rope);
-  for (int n = threadIdx.x; n < d_nope; n += blockDim.x) qn[n] = __bfloat162float(qv[n]);
+  const int h = blockIdx.x % H, b0 = (blockIdx.x / H) * kQGroup;
+  const int nb = min(kQGroup, batch - b0);
+  for (int i = threadIdx.x; i < kQGroup * d_nope; i += blockDim.x) {
+    const int j = i / d_nope, n = i % d_nope;
+    qn[j][n] = j < nb ? __bfloat162float(q[(static_cast<size_t>(b0 + j) * H + h) * (d_nope + d_rope) + n]) : 0.f;
+  }
   __syncthreads();
-  uint8_t* blk = qprep + static_cast<size_t>(b) * qstride;
   const __nv_bfloat16* w = w_uk + static_cast<size_t>(h) * d_nope * d_c;
-  float wpart = 0.f, bpart = 0.f;
+  float wpart[kQGroup], bpart[kQGroup];
+#pragma unroll
+  for (int j = 0; j < kQGroup; ++j) wpart[j] = bpart[j] = 0.f;
   for (int f = threadIdx.x; f < d_c; f += blockDim.x) {
-    float acc = 0.f;
-    for (int n = 0; n < d_nope; ++n) acc = fmaf(__bfloat162float(w[static_cast<size_t>(n) * d_c + f]), qn[n], acc);
+    float acc[kQGroup];
+#pragma unroll
+    for (int j = 0; j < kQGroup; ++j) acc[j] = 0.f;
+#pragma unroll 8
+    for (int n = 0; n < d_nope; ++n) {
+      const float wv = __bfloat162float(w[static_cast<size_t>(n) * d_c + f]);
+#pragma unroll
+      for (int j = 0; j < kQGroup; ++j) acc[j] = fmaf(wv, qn[j][n], acc[j]);
+    }
     const float gm = gamma ? gamma[f] : 1.f;
     const float bt = beta ? beta[f] : 0.f;
-    const __nv_bfloat16 bq = __float2bfloat16_rn(acc * gm);
     const size_t off = static_cast<size_t>(f / 8) * 256 + (h / 8) * 128 + (h % 8) * 16 + (f % 8) * 2;
-    *reinterpret_cast<__nv_bfloat16*>(blk + off) = bq;
-    wpart += __bfloat162float(bq);
-    bpart = fmaf(acc, bt, bpart);
+#pragma unroll
+    for (int j = 0; j < kQGroup; ++j) {
+      if (j >= nb) break;
+      const __nv_bfloat16 bq = __float2bfloat16_rn(acc[j] * gm);
+      *reinterpret_cast<__nv_bfloat16*>(qprep + static_cast<size_t>(b0 + j) * qstride + off) = bq;
+      wpart[j] += __bfloat162float(bq);
+      bpart[j] = fmaf(acc[j], bt, bpart[j]);
+    }
   }
-  uint8_t* rope = blk + static_cast<size_t>(H) * d_c * 2;
-  for (int r = threadIdx.x; r < d_rope; r += blockDim.x) {
+  for (int i = threadIdx.x; i < nb * d_rope; i += blockDim.x) {
+    const int j = i / d_rope, r = i % d_rope;
     const size_t off = static_cast<size_t>(r / 8) * 256 + (h / 8) * 128 + (h % 8) * 16 + (r % 8) * 2;
-    *reinterpret_cast<__nv_bfloat16*>(rope + off) = qv[d_nope + r];
+    *reinterpret_cast<__nv_bfloat16*>(qprep + static_cast<size_t>(b0 + j) * qstride + static_cast<size_t>(H) * d_c * 2 +
+                                      off) = q[(static_cast<size_t>(b0 + j) * H + h) * (d_nope + d_rope) + d_nope + r];
   }
-  const float wsum = block_sum_256(wpart, red);
-  const float bsum = block_sum_256(bpart, red);
-  if (threadIdx.x == 0) {
-    float* sums = reinterpret_cast<float*>(rope + static_cast<size_t>(H) * d_rope * 2);
-    sums[h] = wsum;
-    sums[16 + h] = bsum;
+  // per-sequence block sums of w and b
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int j = 0; j < kQGroup; ++j) {
+    float a = wpart[j], c = bpart[j];
+    for (int o = 16; o > 0; o >>= 1) {
+      a += __shfl_xor_sync(0xffffffffu, a, o);
+      c += __shfl_xor_sync(0xffffffffu, c, o);
+    }
+    if (lane == 0) {
+      red[0][j][warp] = a;
+      red[1][j][warp] = c;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x < nb) {
+    const int j = threadIdx.x;
+    float a = 0.f, c = 0.f;
+    for (int k = 0; k < (int)(blockDim.x >> 5); ++k) {
+      a += red[0][j][k];
+      c += red[1][j][k];
+    }
+    float* sums = reinterpret_cast<float*>(qprep + static_cast<size_t>(b0 + j) * qstride +
+                                           static_cast<size_t>(H) * (d_c + d_rope) * 2);
+    sums[h] = a;
+    sums[16 + h] = c;
   }
 }
 
@@ -173,65 +212,79 @@ __device__ __forceinline__ float from_f<float>(float v) { return v; }
 template <>
 __device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
 
-constexpr int kCombineRows = 8;
+// Block per (sequence b, head h), 256 threads.  The splits that covered b are
+// the CTAs c0..c1 of the page schedule; their partials sit in slots c + b.
+// M = max_s m_s; o = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s (m in log2
+// units); then u = W_UV,h o with two threads per output row.  A sequence of
+// length 0 gets u = 0.
+constexpr int kCombineThreads = 256;
+constexpr int kMaxSlotsSmem = 512;
 
 template <typename T>
-__global__ void combine_kernel(const int32_t* __restrict__ cu, const int32_t* __restrict__ seq_lens,
-                               const float* __restrict__ part_ml, const float* __restrict__ part_o,
-                               const T* __restrict__ w_uv, T* __restrict__ out, int batch, int H, int d_c,
-                               int d_v, int num_splits) {
-  extern __shared__ float olat[];  // [kCombineRows][d_c]
-  const int h = blockIdx.x;
-  const int b0 = blockIdx.y * kCombineRows;
-  const int rows = min(kCombineRows, batch - b0);
+__global__ void __launch_bounds__(kCombineThreads)
+combine_kernel(const int32_t* __restrict__ cu, const float* __restrict__ part_ml, const float* __restrict__ part_o,
+               const T* __restrict__ w_uv, T* __restrict__ out, int batch, int H, int d_c, int d_v,
+               int num_splits) {
+  extern __shared__ float olat[];  // [d_c]
+  __shared__ float wts[kMaxSlotsSmem];
+  __shared__ float red[32];
+  const int b = blockIdx.x / H, h = blockIdx.x % H;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int total = cu[batch];
   const int chunk = split_chunk(total, num_splits);
-  for (int i = 0; i < rows; ++i) {
-    const int b = b0 + i;
-    const int p0 = cu[b], p1 = cu[b + 1];
-    if (p1 <= p0) {
-      for (int f = threadIdx.x; f < d_c; f += blockDim.x) olat[i * d_c + f] = 0.f;
-      continue;
+  const int p0 = cu[b], p1 = cu[b + 1];
+  const int c0 = p0 / chunk;
+  const int n = p1 > p0 ? (p1 - 1) / chunk - c0 + 1 : 0;
+  if (n == 0) {
+    for (int f = tid; f < d_c; f += blockDim.x) olat[f] = 0.f;
+  } else {
+    // running max and denominator over the slots (n <= num_splits)
+    float mloc = -INFINITY;
+    for (int k = tid; k < n; k += blockDim.x) mloc = fmaxf(mloc, part_ml[(static_cast<size_t>(c0 + k + b) * H + h) * 2]);
+    for (int o = 16; o > 0; o >>= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, o));
+    if (lane == 0) red[warp] = mloc;
+    __syncthreads();
+    float M = red[0];
+    for (int k = 1; k < (int)(blockDim.x >> 5); ++k) M = fmaxf(M, red[k]);
+    __syncthreads();
+    float lloc = 0.f;
+    for (int k = tid; k < n; k += blockDim.x) {
+      const float* ml = part_ml + (static_cast<size_t>(c0 + k + b) * H + h) * 2;
+      const float wk = exp2f(ml[0] - M);
+      if (k < kMaxSlotsSmem) wts[k] = wk;
+      lloc = fmaf(wk, ml[1], lloc);
     }
-    // CTAs c0..c1 covered this sequence; its partials sit in slots c + b
-    const int c0 = p0 / chunk, c1 = (p1 - 1) / chunk;
-    float M = -INFINITY;
-    for (int c = c0; c <= c1; ++c) M = fmaxf(M, part_ml[(static_cast<size_t>(c + b) * H + h) * 2]);
+    for (int o = 16; o > 0; o >>= 1) lloc += __shfl_xor_sync(0xffffffffu, lloc, o);
+    if (lane == 0) red[warp] = lloc;
+    __syncthreads();
     float L = 0.f;
-    for (int c = c0; c <= c1; ++c) {
-      const float* ml = part_ml + (static_cast<size_t>(c + b) * H + h) * 2;
-      L = fmaf(exp2f(ml[0] - M), ml[1], L);
-    }
+    for (int k = 0; k < (int)(blockDim.x >> 5); ++k) L += red[k];
     const float invL = 1.f / L;
-    for (int f = threadIdx.x; f < d_c; f += blockDim.x) {
+    for (int f = tid; f < d_c; f += blockDim.x) {
       float acc = 0.f;
-      for (int c = c0; c <= c1; ++c) {
-        const size_t s = static_cast<size_t>(c + b) * H + h;
-        acc = fmaf(exp2f(part_ml[s * 2] - M), part_o[s * d_c + f], acc);
+#pragma unroll 8
+      for (int k = 0; k < n; ++k) {
+        const size_t s = static_cast<size_t>(c0 + k + b) * H + h;
+        const float wk = k < kMaxSlotsSmem ? wts[k] : exp2f(part_ml[s * 2] - M);
+        acc = fmaf(wk, part_o[s * d_c + f], acc);
       }
-      olat[i * d_c + f] = acc * invL;
+      olat[f] = acc * invL;
     }
   }
   __syncthreads();
-  // u[b][h][v] = sum_f W_UV[h][v][f] * olat[b][f]; warp per output row v, lanes over f
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  // u[v] = sum_f W_UV[h][v][f] olat[f]: a thread pair per row v, halves of f
   const T* wh = w_uv + static_cast<size_t>(h) * d_v * d_c;
-  for (int v = warp; v < d_v; v += nwarps) {
-    float acc[kCombineRows];
-#pragma unroll
-    for (int i = 0; i < kCombineRows; ++i) acc[i] = 0.f;
-    for (int f = lane; f < d_c; f += 32) {
-      const float wv = to_f<T>(wh[static_cast<size_t>(v) * d_c + f]);
-#pragma unroll
-      for (int i = 0; i < kCombineRows; ++i)
-        if (i < rows) acc[i] = fmaf(wv, olat[i * d_c + f], acc[i]);
+  const int half = tid & 1;
+  for (int base = 0; base < d_v; base += blockDim.x >> 1) {
+    const int v = base + (tid >> 1);
+    float acc = 0.f;
+    if (v < d_v) {
+      const T* row = wh + static_cast<size_t>(v) * d_c;
+#pragma unroll 8
+      for (int f = half; f < d_c; f += 2) acc = fmaf(to_f<T>(row[f]), olat[f], acc);
     }
-#pragma unroll
-    for (int i = 0; i < kCombineRows; ++i) {
-      float s = acc[i];
-      for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-      if (lane == 0 && i < rows) out[(static_cast<size_t>(b0 + i) * H + h) * d_v + v] = from_f<T>(s);
-    }
+    acc += __shfl_xor_sync(0xffffffffu, acc, 1);
+    if (half == 0 && v < d_v) out[(static_cast<size_t>(b) * H + h) * d_v + v] = from_f<T>(acc);
   }
 }
 
@@ -374,7 +427,8 @@ cudaError_t launch_prologue_tc(const DecodeArgs& a, cudaStream_t st) {
   // with the gate off the latent is used as cached: no LayerNorm affine to fold into q^
   const float* gamma = a.gate ? a.ln_gamma : nullptr;
   const float* beta = a.gate ? a.ln_beta : nullptr;
-  prologue_tc_kernel<<<a.batch * 16 + 1, 256, 0, st>>>(
+  const int ngroups = (a.batch + kQGroup - 1) / kQGroup;
+  prologue_tc_kernel<<<ngroups * 16 + 1, 256, 0, st>>>(
       static_cast<const __nv_bfloat16*>(a.q), static_cast<const __nv_bfloat16*>(a.w_uk), gamma, beta,
       a.seq_lens, a.batch, a.d_nope, a.d_rope, a.d_c, a.page_size, ws + wl.off_qprep, wl.qprep_stride,
       reinterpret_cast<int32_t*>(ws + wl.off_cu));
@@ -407,20 +461,19 @@ cudaError_t launch_decode_f32(const DecodeArgs& a, cudaStream_t st) {
 cudaError_t launch_combine(const DecodeArgs& a, bool tc_path, cudaStream_t st) {
   const WorkspaceLayout wl = workspace_layout(a.batch, a.num_splits, a.H, a.d_c, a.d_rope, tc_path);
   uint8_t* ws = static_cast<uint8_t*>(a.workspace);
-  dim3 grid(a.H, (a.batch + kCombineRows - 1) / kCombineRows);
-  const size_t smem = static_cast<size_t>(kCombineRows) * a.d_c * sizeof(float);
+  const size_t smem = static_cast<size_t>(a.d_c) * sizeof(float);
   const int32_t* cu = reinterpret_cast<const int32_t*>(ws + wl.off_cu);
   const float* ml = reinterpret_cast<const float*>(ws + wl.off_ml);
   const float* po = reinterpret_cast<const float*>(ws + wl.off_o);
+  const int grid = a.batch * a.H;
   if (a.dtype == 0) {
-    combine_kernel<__nv_bfloat16><<<grid, 256, smem, st>>>(cu, a.seq_lens, ml, po,
-                                                           static_cast<const __nv_bfloat16*>(a.w_uv),
-                                                           static_cast<__nv_bfloat16*>(a.out), a.batch, a.H,
-                                                           a.d_c, a.d_v, a.num_splits);
+    combine_kernel<__nv_bfloat16><<<grid, kCombineThreads, smem, st>>>(
+        cu, ml, po, static_cast<const __nv_bfloat16*>(a.w_uv), static_cast<__nv_bfloat16*>(a.out), a.batch, a.H,
+        a.d_c, a.d_v, a.num_splits);
   } else {
-    combine_kernel<float><<<grid, 256, smem, st>>>(cu, a.seq_lens, ml, po, static_cast<const float*>(a.w_uv),
-                                                   static_cast<float*>(a.out), a.batch, a.H, a.d_c, a.d_v,
-                                                   a.num_splits);
+    combine_kernel<float><<<grid, kCombineThreads, smem, st>>>(cu, ml, po, static_cast<const float*>(a.w_uv),
+                                                                static_cast<float*>(a.out), a.batch, a.H, a.d_c,
+                                                                a.d_v, a.num_splits);
   }
   return cudaGetLastError();
 }

@@ -55,6 +55,9 @@ struct DecodeArgs {
   void* dump_kr;
   int32_t* dump_ids;
   void* dump_g;
+  // pipeline event trace of the decode kernel (eg_mla_debug_set_trace)
+  void* trace;
+  int trace_ctas, trace_cap;
 };
 
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t st);
