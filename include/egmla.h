@@ -20,7 +20,9 @@
  * Conventions shared by every call:
  *   - Every pointer argument except `dims`, `bytes_out` and `out_splits` is a
  *     DEVICE pointer to caller-owned memory.  The library never allocates,
- *     frees or keeps device memory between calls.
+ *     frees or keeps device memory between calls; the one device buffer it
+ *     owns is the fixed static scratch array of eg_mla_decode_static, which
+ *     is part of the loaded module.
  *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
  *     stream).  Calls are asynchronous on that stream and never synchronise
  *     the host.
@@ -51,7 +53,8 @@ typedef enum {
   EG_MLA_ERR_CUDA = -3,          /* a CUDA runtime call failed (launch, attribute) */
   EG_MLA_ERR_OUT_OF_RANGE = -4,  /* device: page id >= num_pages or token id >= vocab */
   EG_MLA_ERR_TIMEOUT = -5,       /* device: a pipeline wait exceeded its limit */
-  EG_MLA_ERR_WORKSPACE = -6      /* workspace too small or misaligned */
+  EG_MLA_ERR_WORKSPACE = -6,     /* workspace too small or misaligned */
+  EG_MLA_ERR_SCRATCH_LIMIT = -7  /* needs more than EG_MLA_STATIC_SCRATCH_BYTES of static scratch */
 } eg_mla_status;
 
 typedef enum { EG_MLA_BF16 = 0, EG_MLA_FP32 = 1 } eg_mla_dtype;
@@ -172,6 +175,49 @@ int eg_mla_decode(const eg_mla_dims* dims, const void* q, const void* c_pool,
                   const float* ln_beta, const void* w_uk, const void* w_uv, void* out,
                   int32_t num_splits, void* workspace, size_t workspace_bytes,
                   int32_t* dev_status, void* stream);
+
+/* Size of the static device scratch array behind eg_mla_decode_static. */
+#define EG_MLA_STATIC_SCRATCH_BYTES ((size_t)16 << 20)
+
+/*
+ * eg_mla_decode_static - eg_mla_decode without a caller workspace.  The paper
+ * has no counterpart to this call: it is an interface choice of this library.
+ *
+ * Same arguments, results, validation and device-error reporting as
+ * eg_mla_decode, minus `workspace` and `workspace_bytes`: the scratch is a
+ * file-scope static device array of EG_MLA_STATIC_SCRATCH_BYTES (16 MiB),
+ * 256-byte aligned, compiled into the library.  The call allocates no device
+ * or pinned memory: no cudaMalloc/cudaFree and no allocating library routine.
+ * It serves callers that have no device memory to hand out per step, such as
+ * an engine that reserved all free HBM for the paged latent cache at start-up,
+ * or a C caller without a caching allocator that would otherwise pay a
+ * device-synchronising cudaFree inside the token loop.
+ *
+ *   - Size limit: if eg_mla_decode_workspace_size(dims, batch, num_splits)
+ *     exceeds EG_MLA_STATIC_SCRATCH_BYTES the call returns
+ *     EG_MLA_ERR_SCRATCH_LIMIT and launches nothing; use eg_mla_decode with a
+ *     workspace, or fewer splits, instead.  The limit covers, for example,
+ *     batch 128 at d_c = 512 with 152 splits (about 12 MB).
+ *   - Start-up: the first call on each device, with that device current,
+ *     looks up the array's device address (cudaGetSymbolAddress) and caches
+ *     it; make that first call before any stream capture begins.  A failed
+ *     lookup returns EG_MLA_ERR_CUDA.
+ *   - Zeroing: no part of the scratch needs to start at zero (every word the
+ *     kernels read from it is written earlier in the same call), so the call
+ *     runs no clearing pass.  *dev_status is the caller's, zeroed by the
+ *     caller, as for eg_mla_decode.
+ *   - Concurrency: there is one scratch array per device.  Calls on the same
+ *     device whose kernels may overlap (different streams without ordering,
+ *     or different host threads) race on it and corrupt each other's
+ *     results; serialise them, e.g. on one stream.
+ */
+int eg_mla_decode_static(const eg_mla_dims* dims, const void* q, const void* c_pool,
+                         const void* krope_pool, const int32_t* id_pool,
+                         const int32_t* block_table, int32_t max_pages_per_seq,
+                         const int32_t* seq_lens, int32_t max_seq_len, int32_t batch,
+                         int32_t num_pages, const void* gate_table, const float* ln_gamma,
+                         const float* ln_beta, const void* w_uk, const void* w_uv, void* out,
+                         int32_t num_splits, int32_t* dev_status, void* stream);
 
 /*
  * eg_mla_kv_bytes_per_token - bytes the paged cache keeps per token over

@@ -24,6 +24,10 @@ EG_MLA_ERR_CUDA = -3
 EG_MLA_ERR_OUT_OF_RANGE = -4
 EG_MLA_ERR_TIMEOUT = -5
 EG_MLA_ERR_WORKSPACE = -6
+EG_MLA_ERR_SCRATCH_LIMIT = -7
+
+# size of the library's static scratch array (EG_MLA_STATIC_SCRATCH_BYTES)
+STATIC_SCRATCH_BYTES = 16 << 20
 
 EG_MLA_BF16 = 0
 EG_MLA_FP32 = 1
@@ -35,6 +39,7 @@ EXPORTED = [
     "eg_mla_default_num_splits",
     "eg_mla_decode_workspace_size",
     "eg_mla_decode",
+    "eg_mla_decode_static",
     "eg_mla_kv_bytes_per_token",
     "eg_mla_status_string",
     "eg_mla_debug_gather",
@@ -81,6 +86,8 @@ def _declare(lib: ctypes.CDLL) -> None:
     lib.eg_mla_decode_workspace_size.restype = SZ
     lib.eg_mla_decode.argtypes = [D, P, P, P, P, P, I32, P, I32, I32, I32, P, P, P, P, P, P, I32, P, SZ, P, P]
     lib.eg_mla_decode.restype = ctypes.c_int
+    lib.eg_mla_decode_static.argtypes = [D, P, P, P, P, P, I32, P, I32, I32, I32, P, P, P, P, P, P, I32, P, P]
+    lib.eg_mla_decode_static.restype = ctypes.c_int
     lib.eg_mla_kv_bytes_per_token.argtypes = [D, I32, ctypes.POINTER(ctypes.c_int64)]
     lib.eg_mla_kv_bytes_per_token.restype = ctypes.c_int
     lib.eg_mla_status_string.argtypes = [ctypes.c_int]
@@ -185,6 +192,18 @@ def eg_mla_decode(dims: EgMlaDims, q, c_pool, krope_pool, id_pool, block_table, 
         _ptr(gate_table), _ptr(ln_gamma), _ptr(ln_beta), _ptr(w_uk), _ptr(w_uv), _ptr(out), num_splits,
         _ptr(workspace), workspace.numel() * workspace.element_size(), _ptr(dev_status), _stream(stream))
     _check(code, "eg_mla_decode")
+
+
+def eg_mla_decode_static(dims: EgMlaDims, q, c_pool, krope_pool, id_pool, block_table, seq_lens, max_seq_len,
+                         gate_table, ln_gamma, ln_beta, w_uk, w_uv, out, num_splits=0,
+                         dev_status=None, stream=None) -> None:
+    """eg_mla_decode on the library's static scratch array (no workspace argument)."""
+    code = load().eg_mla_decode_static(
+        ctypes.byref(dims), _ptr(q), _ptr(c_pool), _ptr(krope_pool), _ptr(id_pool), _ptr(block_table),
+        block_table.shape[1], _ptr(seq_lens), int(max_seq_len), seq_lens.shape[0], c_pool.shape[0],
+        _ptr(gate_table), _ptr(ln_gamma), _ptr(ln_beta), _ptr(w_uk), _ptr(w_uv), _ptr(out), num_splits,
+        _ptr(dev_status), _stream(stream))
+    _check(code, "eg_mla_decode_static")
 
 
 def eg_mla_debug_gather(dims: EgMlaDims, c_pool, krope_pool, id_pool, block_table, seq_lens, max_seq_len,

@@ -185,6 +185,41 @@ void prof_mark(cudaStream_t st, bool before) {
   }
 }
 
+// Static scratch of eg_mla_decode_static.  Callers that cannot hand the
+// decode a workspace (an engine that reserved all free HBM for the paged
+// latent cache at start-up, or a C caller without a caching allocator, whose
+// per-step cudaFree would synchronise the device inside the token loop) get
+// this module-owned array instead; no call allocates or frees device memory.
+// Nothing in it needs to start at zero: the prologue writes the page prefix
+// sums and prepared queries, the split-KV kernel writes every partial slot the
+// combine reads, all within the same call.  One array per device, so calls
+// whose kernels overlap on one device race on it.
+static __device__ __align__(256) unsigned char g_static_scratch[EG_MLA_STATIC_SCRATCH_BYTES];
+
+constexpr int kMaxDevices = 64;
+
+// device address of g_static_scratch, looked up once per device with that
+// device current (the lookup may load the module, so the first call belongs
+// before any stream capture)
+struct StaticScratch {
+  std::mutex mu;
+  void* ptr[kMaxDevices] = {};
+} g_static;
+
+int static_scratch(void** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return EG_MLA_ERR_CUDA;
+  if (dev < 0 || dev >= kMaxDevices) return EG_MLA_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lk(g_static.mu);
+  if (g_static.ptr[dev] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || p == nullptr) return EG_MLA_ERR_CUDA;
+    g_static.ptr[dev] = p;
+  }
+  *out = g_static.ptr[dev];
+  return EG_MLA_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -198,6 +233,8 @@ const char* eg_mla_status_string(int status) {
     case EG_MLA_ERR_OUT_OF_RANGE: return "page id or token id out of range";
     case EG_MLA_ERR_TIMEOUT: return "device pipeline wait timed out";
     case EG_MLA_ERR_WORKSPACE: return "workspace too small or misaligned";
+    case EG_MLA_ERR_SCRATCH_LIMIT:
+      return "problem needs more scratch than the static scratch array (EG_MLA_STATIC_SCRATCH_BYTES) holds";
     default: return "unknown status";
   }
 }
@@ -295,6 +332,25 @@ int eg_mla_decode(const eg_mla_dims* dims, const void* q, const void* c_pool, co
   cudaError_t e = egmla::launch_decode_f32(a, st);
   if (e == cudaSuccess) e = egmla::launch_combine(a, false, st);
   return to_status(e);
+}
+
+int eg_mla_decode_static(const eg_mla_dims* dims, const void* q, const void* c_pool, const void* krope_pool,
+                         const int32_t* id_pool, const int32_t* block_table, int32_t max_pages_per_seq,
+                         const int32_t* seq_lens, int32_t max_seq_len, int32_t batch, int32_t num_pages,
+                         const void* gate_table, const float* ln_gamma, const float* ln_beta, const void* w_uk,
+                         const void* w_uv, void* out, int32_t num_splits, int32_t* dev_status, void* stream) {
+  int rc = check_dims(dims);
+  if (rc != EG_MLA_OK) return rc;
+  if (batch < 0 || num_splits < 0) return EG_MLA_ERR_INVALID_ARG;
+  const size_t need = eg_mla_decode_workspace_size(dims, batch, num_splits);
+  if (need == 0) return EG_MLA_ERR_CUDA;  // dims were checked: only the SM-count query can fail
+  if (need > EG_MLA_STATIC_SCRATCH_BYTES) return EG_MLA_ERR_SCRATCH_LIMIT;
+  void* scratch = nullptr;
+  rc = static_scratch(&scratch);
+  if (rc != EG_MLA_OK) return rc;
+  return eg_mla_decode(dims, q, c_pool, krope_pool, id_pool, block_table, max_pages_per_seq, seq_lens, max_seq_len,
+                       batch, num_pages, gate_table, ln_gamma, ln_beta, w_uk, w_uv, out, num_splits, scratch,
+                       EG_MLA_STATIC_SCRATCH_BYTES, dev_status, stream);
 }
 
 int eg_mla_debug_set_trace(void* dev_buf, int64_t bytes, int32_t ctas) {
