@@ -19,7 +19,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libegmla.so")
 
-SOURCES = ["egmla_api.cu", "egmla_aux.cu", "egmla_decode_tc.cu"]
+SOURCES = ["egmla_api.cu", "egmla_aux.cu", "egmla_decode_tc.cu", "egmla_decode_wide.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

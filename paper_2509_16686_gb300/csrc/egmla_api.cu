@@ -93,6 +93,32 @@ bool encode_pool_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Latent pool as one 3-D box per page for the d_c <= 256 kernel: dims
+// {64 features, rows, d_c / 64 feature columns}, so that one copy writes the
+// page as its 128-byte-swizzled 64-feature columns one after another.
+bool encode_page_map_3d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols) {
+  EncodeFn enc = get_encode();
+  if (enc == nullptr) return false;
+  const cuuint64_t dims[3] = {64, rows, cols / 64};
+  const cuuint64_t strides[2] = {cols * 2, 128};
+  const cuuint32_t box[3] = {64, 64, static_cast<cuuint32_t>(cols / 64)};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// maps = {latent pool (3-D page box for d_c <= 256, 64x64 boxes otherwise), RoPE-key pool}
+bool encode_decode_maps(CUtensorMap (&maps)[2], const eg_mla_dims* d, const void* c_pool, const void* krope_pool,
+                        int32_t num_pages) {
+  std::memset(maps, 0, sizeof(maps));
+  const uint64_t rows = static_cast<uint64_t>(num_pages) * d->page_size;
+  const bool paged3d = d->d_c <= 256;
+  if (!(paged3d ? encode_page_map_3d(&maps[0], c_pool, rows, d->d_c) : encode_pool_map(&maps[0], c_pool, rows, d->d_c)))
+    return false;
+  return encode_pool_map(&maps[1], krope_pool, rows, d->d_rope);
+}
+
 float resolve_scale(const eg_mla_dims* d) {
   return d->softmax_scale > 0.f ? d->softmax_scale : 1.0f / std::sqrt(static_cast<float>(d->d_nope + d->d_rope));
 }
@@ -315,10 +341,7 @@ int eg_mla_decode(const eg_mla_dims* dims, const void* q, const void* c_pool, co
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   if (is_tc_path(dims)) {
     CUtensorMap maps[2];
-    const uint64_t rows = static_cast<uint64_t>(num_pages) * dims->page_size;
-    if (!encode_pool_map(&maps[0], c_pool, rows, dims->d_c) ||
-        !encode_pool_map(&maps[1], krope_pool, rows, dims->d_rope))
-      return EG_MLA_ERR_CUDA;
+    if (!encode_decode_maps(maps, dims, c_pool, krope_pool, num_pages)) return EG_MLA_ERR_CUDA;
     apply_trace(a);
     cudaError_t e = egmla::launch_prologue_tc(a, st);
     if (e == cudaSuccess) {
@@ -360,7 +383,7 @@ int eg_mla_debug_set_trace(void* dev_buf, int64_t bytes, int32_t ctas) {
     g_trace.ctas = g_trace.cap = 0;
     return EG_MLA_OK;
   }
-  const int64_t cap = bytes / (static_cast<int64_t>(ctas) * 4 * 16);
+  const int64_t cap = bytes / (static_cast<int64_t>(ctas) * egmla::kTraceRoles * 16);
   if (cap < 1 || !aligned(dev_buf, 16)) return EG_MLA_ERR_INVALID_ARG;
   g_trace.buf = dev_buf;
   g_trace.ctas = ctas;
@@ -429,9 +452,7 @@ int eg_mla_debug_gather(const eg_mla_dims* dims, const void* c_pool, const void*
   a.dump_g = g_out;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   CUtensorMap maps[2];
-  const uint64_t rows = static_cast<uint64_t>(num_pages) * dims->page_size;
-  if (!encode_pool_map(&maps[0], c_pool, rows, dims->d_c) || !encode_pool_map(&maps[1], krope_pool, rows, dims->d_rope))
-    return EG_MLA_ERR_CUDA;
+  if (!encode_decode_maps(maps, dims, c_pool, krope_pool, num_pages)) return EG_MLA_ERR_CUDA;
   a.q = nullptr;  // prologue computes the page prefix sums only
   cudaError_t e = egmla::launch_prologue_tc(a, st);
   if (e == cudaSuccess) e = egmla::launch_decode_tc(a, maps, true, st);

@@ -125,7 +125,7 @@ prologue_tc_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __r
     }
     const float gm = gamma ? gamma[f] : 1.f;
     const float bt = beta ? beta[f] : 0.f;
-    const size_t off = static_cast<size_t>(f / 8) * 256 + (h / 8) * 128 + (h % 8) * 16 + (f % 8) * 2;
+    const size_t off = qop_offset(h, f);
 #pragma unroll
     for (int j = 0; j < kQGroup; ++j) {
       if (j >= nb) break;
@@ -137,9 +137,8 @@ prologue_tc_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __r
   }
   for (int i = threadIdx.x; i < nb * d_rope; i += blockDim.x) {
     const int j = i / d_rope, r = i % d_rope;
-    const size_t off = static_cast<size_t>(r / 8) * 256 + (h / 8) * 128 + (h % 8) * 16 + (r % 8) * 2;
-    *reinterpret_cast<__nv_bfloat16*>(qprep + static_cast<size_t>(b0 + j) * qstride + static_cast<size_t>(H) * d_c * 2 +
-                                      off) = q[(static_cast<size_t>(b0 + j) * H + h) * (d_nope + d_rope) + d_nope + r];
+    const size_t off = qprep_lat_bytes(d_c) + qop_offset(h, r);
+    *reinterpret_cast<__nv_bfloat16*>(qprep + static_cast<size_t>(b0 + j) * qstride + off) = q[(static_cast<size_t>(b0 + j) * H + h) * (d_nope + d_rope) + d_nope + r];
   }
   // per-sequence block sums of w and b
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -163,8 +162,8 @@ prologue_tc_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __r
       a += red[0][j][k];
       c += red[1][j][k];
     }
-    float* sums = reinterpret_cast<float*>(qprep + static_cast<size_t>(b0 + j) * qstride +
-                                           static_cast<size_t>(H) * (d_c + d_rope) * 2);
+    float* sums = reinterpret_cast<float*>(qprep + static_cast<size_t>(b0 + j) * qstride + qprep_lat_bytes(d_c) +
+                                           qprep_rope_bytes(d_rope));
     sums[h] = a;
     sums[16 + h] = c;
   }

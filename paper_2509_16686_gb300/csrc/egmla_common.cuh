@@ -19,12 +19,25 @@ constexpr int kPage = 64;
 
 __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-// Bytes of the per-sequence prepared query block of the tensor-core path:
-// q^ (*) gamma as a bf16 MMA operand [16 heads x d_c], q^R as a bf16 operand
-// [16 x d_rope], then per-head fp32 sums w_h = sum_f (q^ gamma)_hf and
-// b_h = q^_h . beta, padded to 16-byte multiples.
-__host__ __device__ inline size_t qprep_bytes_tc(int d_c, int d_rope) {
-  return static_cast<size_t>(16) * d_c * 2 + static_cast<size_t>(16) * d_rope * 2 + 128;
+// Per-sequence prepared query block of the tensor-core path: q^ (*) gamma
+// [16 heads x d_c] and q^R [16 x d_rope] as bf16 MMA operands in 8x8 core
+// matrices, then per-head fp32 sums w_h = sum_f (q^ gamma)_hf and
+// b_h = q^_h . beta (16 + 16 floats, 128 bytes).  In every group of 8 columns
+// (512 bytes) heads 0-7 fill core-matrix row group 0 and heads 8-15 row group
+// 2.  Read as the A operand of an M = 64 MMA (row-group stride 128 B) the two
+// head halves land in TMEM lane quadrants 0 and 1; read as an N = 16 B operand
+// (row-group stride 256 B) they are its 16 rows.  The unused row groups are
+// never written.
+constexpr int kQGroupBytes = 512;
+__host__ __device__ constexpr size_t qop_offset(int h, int k) {
+  return static_cast<size_t>(k / 8) * kQGroupBytes + (h / 8) * 256 + (h % 8) * 16 + (k % 8) * 2;
+}
+__host__ __device__ constexpr size_t qprep_lat_bytes(int d_c) { return static_cast<size_t>(d_c / 8) * kQGroupBytes; }
+__host__ __device__ constexpr size_t qprep_rope_bytes(int d_rope) {
+  return static_cast<size_t>(d_rope / 8) * kQGroupBytes;
+}
+__host__ __device__ constexpr size_t qprep_bytes_tc(int d_c, int d_rope) {
+  return qprep_lat_bytes(d_c) + qprep_rope_bytes(d_rope) + 128;
 }
 
 // fp32 path: q^ [H, d_c] and q^R [H, d_rope] in fp32.

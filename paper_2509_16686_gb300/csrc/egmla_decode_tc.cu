@@ -1,31 +1,42 @@
-// egmla_decode_tc.cu - split-KV EG-MLA decode on sm_103a tensor cores.
+// egmla_decode_tc.cu - split-KV EG-MLA decode on sm_103a tensor cores for the
+// latent widths 192 and 256 (gated or plain).
 //
 // One CTA per split-KV work unit (see egmla_common.cuh for the schedule).  The
 // CTA streams its cache pages, one 64-token page per tile, through a ring of
 // shared-memory slots.  Four roles run concurrently on different tiles:
 //
-//   TMA (warp 0)      latent page [64 tok x d_c] and RoPE-key page [64 x 64] as
-//                     128-byte-swizzled boxes, plus the page's token ids.
-//   gate (warps 4-7, two threads per token, each half of the features)
-//                     g = G[id] gathered from global memory, z = c (*) g rounded
-//                     to bf16 and written back in place, and the LayerNorm
-//                     statistics mu, r = 1/sqrt(var + eps) of z (Eq. 5 over d_c).
-//   MMA (warp 1)      S_lat = Z Bq^T and S_rope = K^R Q^R^T on tcgen05 with fp32
-//                     accumulators in TMEM (M = 64 tokens, N = 16 heads, S
-//                     double-buffered so the next tile's scores overlap the
-//                     current softmax); O_tile = Z^T P' (M = 128 latent
-//                     features, N = 16 heads, K = 64 tokens).
-//   softmax (warps 8-11)
-//                     s = scale * (r (S_lat - mu w) + b + S_rope): the LayerNorm
-//                     is applied after the MMA, because
-//                     q^.LN(z) = r (q^ gamma).z - r mu sum(q^ gamma) + q^.beta;
-//                     online softmax with a running max per head; P' = p r
-//                     (bf16) is written as the B operand of the PV MMA; then,
-//                     one thread per latent feature, O = O alpha + O_tile.
+//   TMA (warp 3)      latent page [64 tok x d_c] (one 3-D box: 64-feature
+//                     columns x 64 rows) and RoPE-key page [64 x 64], both
+//                     128-byte swizzled.
+//   gate (warps 4-11; each quarter-warp owns two token rows, lane u the 16-byte
+//                     unit u of every 64-feature column of them)
+//                     the token ids (two tiles ahead) and the gate rows
+//                     g = G[id] (EG-MLA-A table, Section 5.2; one tile ahead)
+//                     from L2 into registers, every quarter-warp load reading
+//                     one whole 128-byte line; z = c (*) g rounded to bf16 and
+//                     written back in place, and the LayerNorm statistics
+//                     mu, r = 1/sqrt(var + eps) of z (Eq. 5 over d_c).
+//   MMA (warp 2)      transposed scores S^T = Q Z^T and S_rope^T = Q^R K^R^T
+//                     (M = 64 rows, N = 64 tokens, fp32 in TMEM, double-buffered)
+//                     and the latent output O += P' Z (M = 64 rows, N = d_c
+//                     features, K = 64 tokens), accumulated in TMEM over a
+//                     sequence segment.  The operand rows of heads 0-7 and 8-15
+//                     are placed so that their accumulator rows fall in TMEM lane
+//                     quadrants 0 and 1.
+//   softmax (warps 0 and 1, heads 0-7 and 8-15)
+//                     reads its eight head rows of S^T spread over the 32
+//                     threads (one head x 16 tokens each), s = scale * (r (S -
+//                     mu w) + b + S_rope) -- the LayerNorm applied after the MMA,
+//                     since q^.LN(z) = r (q^ gamma).z - r mu sum(q^ gamma) +
+//                     q^.beta --, an online softmax whose per-head maxima need no
+//                     exchange beyond the four threads of a head, and P' = p r
+//                     (bf16) as the A operand of the output MMA.
 //
-// At the end of each sequence segment the un-normalised latent output
-// gamma (*) (O - sum_j P'_j mu_j) + beta l, the running max m and the
-// denominator l = sum_j P'_j / r_j are written as this split's partial result.
+// With heads in the accumulator rows, the running max, its lazy rescaling of
+// O and the final read-out of a head all stay inside one softmax warp.  At the end of each
+// sequence segment the un-normalised latent output gamma (*) (O - sum_j P'_j
+// mu_j) + beta l, the running max m and the denominator l = sum_j P'_j / r_j are
+// written as this split's partial result.
 //
 // The queries are absorbed before this kernel (q^ = W_UK^T q^C, with gamma
 // folded in); W_UV is applied after the split merge.  Everything the kernel
@@ -47,63 +58,59 @@ namespace {
 
 constexpr int kHeads = 16;
 constexpr int kRope = 64;
-constexpr int kThreads = 384;  // warp 0 TMA, warp 1 MMA + TMEM owner, 2-3 spare, 4-7 gate, 8-11 softmax
+constexpr int kThreads = 384;
+constexpr int kSoftWarps = 2;    // warps 0 and 1: TMEM lane quadrants 0 and 1 hold heads 0-7 and 8-15
+constexpr int kMmaWarp = 2;
+constexpr int kTmaWarp = 3;
 constexpr int kGateWarp0 = 4;
-constexpr int kSoftWarp0 = 8;
+constexpr int kGateWarps = 8;
 constexpr uint32_t kSmemLimit = 232448;
-// registers per thread: 384 threads x 168 at launch; warps 0-3 give theirs up
-// to the gate and softmax warpgroups (128 x 56 + 256 x 224 = 384 x 168)
-constexpr int kProducerRegs = 56;
-constexpr int kConsumerRegs = 224;
 // a head's reference max moves only when a tile exceeds it by 2^8
 constexpr float kLazyLog2 = 8.f;
 
 template <int D_C, bool GATE>
 struct Cfg {
   static constexpr int NCH = D_C / 64;                  // 64-feature swizzle-atom columns
-  static constexpr int NMC = (D_C + 127) / 128;         // 128-feature M chunks of the PV MMA
+  static constexpr int UNITS = D_C / 8;                 // 16-byte units of a latent row
+  static constexpr int NU = UNITS / 4;                  // units per gate thread
   static constexpr uint32_t PCHUNK = kPage * 128;       // one atom column of a page: 8 KB
   static constexpr uint32_t KR_OFF = NCH * PCHUNK;
   static constexpr uint32_t SLOT = KR_OFF + PCHUNK;     // latent + RoPE key of one page
-  static constexpr uint32_t QB_LAT = kHeads * D_C * 2;
-  static constexpr uint32_t QB_ROPE = kHeads * kRope * 2;
-  static constexpr uint32_t QPREP = QB_LAT + QB_ROPE + 128;
+  static constexpr uint32_t QB_LAT = qprep_lat_bytes(D_C);
+  static constexpr uint32_t QB_ROPE = qprep_rope_bytes(kRope);
+  static constexpr uint32_t QPREP = qprep_bytes_tc(D_C, kRope);
+  // two query blocks (the next sequence's loads while this one is in use)
   static constexpr uint32_t QBUF = (QPREP + 127) / 128 * 128;
-  static constexpr uint32_t PBUF = kPage * kHeads * 2;
-  // gate rows of a page, gathered by TMA bulk copies: row stride padded by 16 B
-  // so that the gate threads' 16-byte reads of 8 consecutive rows hit 8 distinct
-  // bank groups; double-buffered
-  static constexpr uint32_t GSTRIDE = D_C * 2 + 16;
-  static constexpr uint32_t GBUF = (kPage * GSTRIDE + 127) / 128 * 128;
-  static constexpr int NGB = GATE ? 2 : 0;
-  static constexpr uint32_t GIDS = kPage * 4;           // token ids of a gathered page
-  static constexpr uint32_t STAT_BYTES = kPage * 8;     // per slot: (mu, r) per token
-  static constexpr uint32_t MISC = 2048;
-  static constexpr int NS_FIT =
-      (int)((kSmemLimit - 1024 - 2 * QBUF - PBUF - MISC - NGB * (GBUF + GIDS)) / (SLOT + STAT_BYTES));
+  // P' [16 heads x 64 tokens] in the layout of the query block (qop_offset)
+  static constexpr uint32_t PBUF = kPage / 8 * kQGroupBytes;
+  static constexpr uint32_t STAT_BYTES = 3 * kPage * 4;   // per slot: mu[64], r[64], 1/r[64]
+  static constexpr uint32_t MISC = 1024;
+  static constexpr int NS_FIT = (int)((kSmemLimit - 1024 - 2 * QBUF - 2 * PBUF - MISC) / (SLOT + STAT_BYTES));
   static constexpr int NS = NS_FIT > 6 ? 6 : NS_FIT;
   static constexpr uint32_t OFF_QBUF = NS * SLOT;
   static constexpr uint32_t OFF_PBUF = OFF_QBUF + 2 * QBUF;
-  static constexpr uint32_t OFF_GBUF = OFF_PBUF + PBUF;
-  static constexpr uint32_t OFF_GIDS = OFF_GBUF + NGB * GBUF;
-  static constexpr uint32_t OFF_STAT = OFF_GIDS + NGB * GIDS;
+  static constexpr uint32_t OFF_STAT = OFF_PBUF + 2 * PBUF;
   static constexpr uint32_t OFF_MISC = OFF_STAT + NS * STAT_BYTES;
   static constexpr uint32_t SMEM = OFF_MISC + MISC + 1024;
-  // TMEM columns: two score buffers of (latent 16 + RoPE 16) columns, then the
-  // latent-output accumulator (16 columns per 128-feature chunk), which stays
-  // in TMEM across the tiles of a sequence segment
-  static constexpr uint32_t S_COLS = 32;
+  // TMEM columns: two score buffers of (latent 64 + RoPE 64) token columns, then
+  // the latent output (d_c columns), rows = heads
+  static constexpr uint32_t S_COLS = 128;
   static constexpr uint32_t COL_S = 0, COL_O = 2 * S_COLS;
-  static constexpr uint32_t TMEM_COLS = 128;
-  static constexpr uint32_t PAGE_TX = NCH * PCHUNK + PCHUNK;
+  static constexpr uint32_t TMEM_COLS = 512;
+  static constexpr uint32_t PAGE_TX = SLOT;
   static_assert(NS >= 2, "the ring needs two page slots");
   static_assert(SMEM <= kSmemLimit, "shared memory");
-  static_assert(D_C % 64 == 0 && D_C >= 128, "d_c");
-  // first latent feature of PV M-chunk j; the last chunk is shifted back so that
-  // it ends at D_C (for D_C = 192 it overlaps the previous one by 64 features)
-  __host__ __device__ static constexpr int mc_start(int j) {
-    return (128 * j + 128 <= D_C) ? 128 * j : D_C - 128;
-  }
+  static_assert(D_C == 192 || D_C == 256, "latent widths of this kernel");
+  static_assert(COL_O + D_C <= TMEM_COLS, "tensor memory");
+  // The M = 64 MMAs read 64 operand rows (8 row groups 128 B apart in each of
+  // the two 512-byte K groups of a step), 16 of which are heads: a step reads
+  // up to 1536 bytes from its start (the other rows land in TMEM lanes nobody
+  // reads).  Every such read stays inside the allocation:
+  static constexpr uint32_t STEP_SPAN = kQGroupBytes + 8 * 128;
+  static_assert(OFF_QBUF + QBUF + QB_LAT + (kRope / 16 - 1) * 2 * kQGroupBytes + STEP_SPAN <= OFF_MISC,
+                "query over-read");
+  static_assert(OFF_PBUF + PBUF + (kPage / 16 - 1) * 2 * kQGroupBytes + STEP_SPAN <= OFF_MISC + MISC,
+                "weight over-read");
 };
 
 struct TcParams {
@@ -140,7 +147,7 @@ struct Tracer {
     n = 0;
     cap = p.trace_cap;
     if (p.trace != nullptr && static_cast<int>(blockIdx.x) < p.trace_ctas)
-      base = p.trace + (static_cast<size_t>(blockIdx.x) * 4 + role) * p.trace_cap * 2;
+      base = p.trace + (static_cast<size_t>(blockIdx.x) * kTraceRoles + role) * p.trace_cap * 2;
   }
   __device__ __forceinline__ void mark(int event, int tile) {
     if (base != nullptr && n < cap) {
@@ -151,14 +158,15 @@ struct Tracer {
   }
 };
 
-// shared-memory barrier block (inside MISC, after 1 KB of reduction scratch)
+// shared-memory barrier block (inside MISC)
 struct Bars {
   uint64_t full[6], empty[6], zready[6];
-  uint64_t gfull[2], gempty[2];
   uint64_t qfull[2], qempty[2];
-  uint64_t s_ready[2];
-  uint64_t sp_done, o_ready;
-  uint64_t red[2], sum;
+  uint64_t s_ready[2], pfree[2];
+  // weights of tile j ready: sp_done[j & 1] (the two softmax warps may be one
+  // tile apart, never two: tile j + 2's scores follow tile j's output MMA)
+  uint64_t sp_done[2];
+  uint64_t drain;
   uint32_t tmem_base;
   int abort;
 };
@@ -220,11 +228,36 @@ struct Walker {
   }
 };
 
-// mbarrier wait taken by a whole warp: every lane polls, then the warp agrees,
-// so that a timeout never splits the warp before a .sync.aligned instruction
+// Page of tile t through a 32-entry window of the block table held one entry per
+// lane (whole warp; the window moves when the tile leaves it).
+struct PageWindow {
+  int b = -1, base = 0, reg = -1;
+  __device__ __forceinline__ int page(const TcParams& p, const Tile& t, int lane) {
+    if (t.b != b || t.lp >= base + 32) {
+      b = t.b;
+      base = t.lp;
+      const int lp = t.lp + lane;
+      reg = lp < p.max_pages ? __ldg(p.block_table + static_cast<size_t>(t.b) * p.max_pages + lp) : -1;
+    }
+    return __shfl_sync(0xffffffffu, reg, t.lp - base);
+  }
+};
+
+// mbarrier wait taken by a whole warp: the warp first reconverges (a lane
+// still on a divergent path would otherwise only resume after the others'
+// suspended wait), every lane polls, then the warp agrees, so that a timeout
+// never splits the warp before a .sync.aligned instruction
 __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+  __syncwarp();
   const bool ok = mbar_wait(bar, parity, abort_flag);
   return __all_sync(0xffffffffu, ok);
+}
+
+// one arrival per warp: the warp barrier orders every lane's earlier writes
+// before lane 0's release arrival
+__device__ __forceinline__ void warp_arrive(uint32_t bar) {
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
 }
 
 __device__ __forceinline__ float2 unpack_bf16x2(uint32_t w) {
@@ -251,38 +284,6 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&z);
 }
 
-// Reduce 16 per-lane values over the 32 lanes of a warp; lane l ends with the
-// result for index (l >> 1) & 15.  Each step hands half of the remaining
-// values to the partner lane, so 16 shuffles replace 80.
-template <bool MAX>
-__device__ __forceinline__ float warp_reduce16(const float (&v)[16], int lane) {
-  auto op = [](float a, float b) { return MAX ? fmaxf(a, b) : a + b; };
-  float r8[8], r4[4], r2[2];
-  const bool u16 = lane & 16, u8 = lane & 8, u4 = lane & 4, u2 = lane & 2;
-#pragma unroll
-  for (int k = 0; k < 8; ++k) {
-    const float send = u16 ? v[k] : v[k + 8];
-    const float keep = u16 ? v[k + 8] : v[k];
-    r8[k] = op(keep, __shfl_xor_sync(0xffffffffu, send, 16));
-  }
-#pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    const float send = u8 ? r8[k] : r8[k + 4];
-    const float keep = u8 ? r8[k + 4] : r8[k];
-    r4[k] = op(keep, __shfl_xor_sync(0xffffffffu, send, 8));
-  }
-#pragma unroll
-  for (int k = 0; k < 2; ++k) {
-    const float send = u4 ? r4[k] : r4[k + 2];
-    const float keep = u4 ? r4[k + 2] : r4[k];
-    r2[k] = op(keep, __shfl_xor_sync(0xffffffffu, send, 4));
-  }
-  const float send = u2 ? r2[0] : r2[1];
-  const float keep = u2 ? r2[1] : r2[0];
-  const float r1 = op(keep, __shfl_xor_sync(0xffffffffu, send, 2));
-  return op(r1, __shfl_xor_sync(0xffffffffu, r1, 1));
-}
-
 template <int D_C, bool GATE, bool DUMP>
 __global__ void __launch_bounds__(kThreads, 1)
     decode_tc_kernel(const __grid_constant__ CUtensorMap cmap, const __grid_constant__ CUtensorMap krmap,
@@ -293,9 +294,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // __shared__ array so that every access through it stays a shared-memory access
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const uint32_t sbase = smem_u32(smem);
-  float* red_max = reinterpret_cast<float*>(smem + C::OFF_MISC);         // [2][4][16]
-  float* red_sum = red_max + 2 * 4 * 16;                                 // [4][32]
-  Bars& bars = *reinterpret_cast<Bars*>(smem + C::OFF_MISC + 1024);
+  Bars& bars = *reinterpret_cast<Bars*>(smem + C::OFF_MISC);
   volatile int* abort_flag = &bars.abort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -303,24 +302,24 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::NS; ++s) {
       mbar_init(smem_u32(&bars.full[s]), 1);
-      mbar_init(smem_u32(&bars.empty[s]), DUMP ? 128 : 1);
-      mbar_init(smem_u32(&bars.zready[s]), 128);
+      mbar_init(smem_u32(&bars.empty[s]), DUMP ? kGateWarps : 1);
+      mbar_init(smem_u32(&bars.zready[s]), kGateWarps);
     }
     for (int s = 0; s < 2; ++s) {
-      mbar_init(smem_u32(&bars.gfull[s]), 1);
-      mbar_init(smem_u32(&bars.gempty[s]), 128);
       mbar_init(smem_u32(&bars.qfull[s]), 1);
-      mbar_init(smem_u32(&bars.qempty[s]), 1 + 128);
-      mbar_init(smem_u32(&bars.s_ready[s]), 1);
-      mbar_init(smem_u32(&bars.red[s]), 128);
+      mbar_init(smem_u32(&bars.qempty[s]), 1 + kSoftWarps);
+      // the MMA commit plus a release arrival of the MMA warp after it saw the
+      // gate's zready (so that the statistics are visible to the softmax warps)
+      mbar_init(smem_u32(&bars.s_ready[s]), 2);
+      mbar_init(smem_u32(&bars.pfree[s]), 1);
     }
-    mbar_init(smem_u32(&bars.sp_done), 128);
-    mbar_init(smem_u32(&bars.o_ready), 1);
-    mbar_init(smem_u32(&bars.sum), 128);
+    mbar_init(smem_u32(&bars.sp_done[0]), kSoftWarps);
+    mbar_init(smem_u32(&bars.sp_done[1]), kSoftWarps);
+    mbar_init(smem_u32(&bars.drain), 1);
     bars.abort = 0;
     fence_mbar_init();
   }
-  if (warp == 1) {
+  if (warp == kMmaWarp) {
     tmem_alloc(smem_u32(&bars.tmem_base), C::TMEM_COLS);
     tmem_relinquish();
   }
@@ -329,8 +328,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = bars.tmem_base;
 
-  if (warp < kGateWarp0) regs_decrease<kProducerRegs>();
-  if (warp == 0) {
+  if (warp == kTmaWarp) {
     // ---------------------------------------------------------------- TMA producer
     // The whole warp walks the tiles; lane 0 waits and issues.  Block-table
     // entries are fetched 32 at a time (one per lane) so no page lookup sits on
@@ -342,23 +340,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint64_t pol_stream = policy_evict_first();
     Walker w;
     w.start(p.cu, p.seq_lens, p.batch);
+    PageWindow pw;
     Tile t;
     int it = 0, seg = -1;
     int last_it[6] = {-1, -1, -1, -1, -1, -1};
     int last_qseg[2] = {-1, -1};
-    int bt_b = -1, bt_base = 0, bt_reg = -1;
     Tracer tr;
     tr.init(p, 0);
     if (lane != 0) tr.base = nullptr;
     bool ok_loop = true;
     while (ok_loop && w.next(t)) {
-      if (t.b != bt_b || t.lp >= bt_base + 32) {
-        bt_b = t.b;
-        bt_base = t.lp;
-        const int lp = t.lp + lane;
-        bt_reg = lp < p.max_pages ? __ldg(p.block_table + static_cast<size_t>(t.b) * p.max_pages + lp) : -1;
-      }
-      const int pg = __shfl_sync(0xffffffffu, bt_reg, t.lp - bt_base);
+      const int pg = pw.page(p, t, lane);
       if (t.first) ++seg;
       const int slot = it % C::NS;
       if (lane == 0) {
@@ -381,11 +373,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!ok) report_status(p.status, kStatusOutOfRange);
           const uint32_t fb = smem_u32(&bars.full[slot]);
           mbar_arrive_expect_tx(fb, ok ? C::PAGE_TX : 0u);
+          tr.mark(3, it);
           if (ok) {
             const uint32_t dst = sbase + slot * C::SLOT;
             const int y = pg * kPage;
-#pragma unroll
-            for (int fc = 0; fc < C::NCH; ++fc) tma_load_2d(dst + fc * C::PCHUNK, &cmap, fc * 64, y, fb, pol_stream);
+            tma_load_3d(dst, &cmap, 0, y, 0, fb, pol_stream);
             tma_load_2d(dst + C::KR_OFF, &krmap, 0, y, fb, pol_stream);
           }
           tr.mark(2, it);
@@ -403,30 +395,35 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (last_qseg[s] >= 0) mbar_wait(smem_u32(&bars.qfull[s]), (last_qseg[s] >> 1) & 1, abort_flag);
     }
     __syncwarp();
-  } else if (warp == 1) {
+  } else if (warp == kMmaWarp) {
     // ---------------------------------------------------------------- MMA issuer
     // Converged warp; one elected lane issues.  Order: scores(i + 1) before
-    // PV(i), so the next tile's scores are ready when the softmax warps finish
+    // PV(i), so the next tile's scores are ready when the softmax warp finishes
     // tile i.  All loops are unrolled with compile-time accumulate flags.
     if (!DUMP) {
-      constexpr uint32_t IDESC_QK = idesc_bf16(64, 16, 0, 0);
-      constexpr uint32_t IDESC_PV = idesc_bf16(128, 16, 1, 1);
+      constexpr uint32_t IDESC_S = idesc_bf16(64, kPage, 0, 0);
+      constexpr uint32_t IDESC_PV = idesc_bf16(64, D_C, 0, 1);
       Walker w;
       w.start(p.cu, p.seq_lens, p.batch);
-      uint32_t last_bar = 0, last_par = 0;
       int seg = -1;
       Tracer tr;
       tr.init(p, 1);
       if (lane != 0) tr.base = nullptr;
-      const uint64_t qdesc0 = smem_desc(sbase + C::OFF_QBUF, 256, 128, kSwizzleNone);
-      const uint64_t zdesc_k = smem_desc(sbase, 16, 1024, kSwizzle128B);         // K-major view of a slot
-      const uint64_t zdesc_mn = smem_desc(sbase, C::PCHUNK, 1024, kSwizzle128B);  // MN-major view of a slot
-      const uint64_t pdesc = smem_desc(sbase + C::OFF_PBUF, 256, 128, kSwizzleNone);
+      // A operands: the query block and P' in 8x8 core matrices, K groups 512 B
+      // apart, row groups 128 B apart (heads 0-7 -> rows 0-7, heads 8-15 ->
+      // rows 16-23).  B operands: the page slot, 128-byte swizzled, read K-major
+      // (tokens x features) for the scores and MN-major (features along N,
+      // tokens along K) for the output.
+      const uint64_t qdesc0 = smem_desc(sbase + C::OFF_QBUF, kQGroupBytes, 128, kSwizzleNone);
+      const uint64_t pdesc0 = smem_desc(sbase + C::OFF_PBUF, kQGroupBytes, 128, kSwizzleNone);
+      constexpr uint32_t KSTEP = 2 * kQGroupBytes;   // bytes of 16 columns of an A operand
+      const uint64_t zdesc_k = smem_desc(sbase, 16, 1024, kSwizzle128B);
+      const uint64_t zdesc_mn = smem_desc(sbase, C::PCHUNK, 1024, kSwizzle128B);
       Tile cur, nxt;
       bool have = w.next(cur);
       bool ok = true;
       int it = 0;
-      // scores of tile j (t): S_lat = Z (q^ gamma)^T, S_rope = K^R (q^R)^T
+      // scores of tile j: S^T = (q^ gamma) Z^T, S_rope^T = q^R K^R^T
       auto scores = [&](const Tile& t, int j) -> bool {
         if (t.first) {
           ++seg;
@@ -436,426 +433,440 @@ __global__ void __launch_bounds__(kThreads, 1)
         tr.mark(0, j);
         if (!warp_wait(smem_u32(&bars.zready[slot]), (j / C::NS) & 1, abort_flag)) return false;
         tr.mark(1, j);
+        if (lane == 0) mbar_arrive(smem_u32(&bars.s_ready[j & 1]));
         tc_fence_after();
         if (elect_one()) {
-          const uint64_t za = zdesc_k + ((slot * C::SLOT) >> 4);
-          const uint64_t qb = qdesc0 + (((seg & 1) * C::QBUF) >> 4);
+          const uint64_t zb = zdesc_k + ((slot * C::SLOT) >> 4);
+          const uint64_t qa = qdesc0 + (((seg & 1) * C::QBUF) >> 4);
           const uint32_t ds = tmem + C::COL_S + (j & 1) * C::S_COLS;
 #pragma unroll
           for (int kk = 0; kk < D_C / 16; ++kk)
-            mma_bf16_ss(ds, za + (((kk >> 2) * C::PCHUNK + (kk & 3) * 32) >> 4), qb + ((kk * 512) >> 4), IDESC_QK,
+            mma_bf16_ss(ds, qa + ((kk * KSTEP) >> 4), zb + (((kk >> 2) * C::PCHUNK + (kk & 3) * 32) >> 4), IDESC_S,
                         kk > 0);
 #pragma unroll
           for (int kk = 0; kk < kRope / 16; ++kk)
-            mma_bf16_ss(ds + 16, za + ((C::KR_OFF + kk * 32) >> 4), qb + ((C::QB_LAT + kk * 512) >> 4), IDESC_QK,
+            mma_bf16_ss(ds + kPage, qa + ((C::QB_LAT + kk * KSTEP) >> 4), zb + ((C::KR_OFF + kk * 32) >> 4), IDESC_S,
                         kk > 0);
           mma_commit(smem_u32(&bars.s_ready[j & 1]));
           if (t.last) mma_commit(smem_u32(&bars.qempty[seg & 1]));
         }
         __syncwarp();
-        last_bar = smem_u32(&bars.s_ready[j & 1]);
-        last_par = (j >> 1) & 1;
         return true;
       };
       if (have) ok = scores(cur, 0);
       while (have && ok) {
         const bool have_next = w.next(nxt);
         if (have_next && !scores(nxt, it + 1)) break;
-        // latent output of tile it, accumulated in TMEM over the segment:
-        // O^T[feature, head] += Z^T P'
+        // latent output of tile it, accumulated in TMEM over the segment: O += P' Z
         tr.mark(2, it);
-        if (!warp_wait(smem_u32(&bars.sp_done), it & 1, abort_flag)) break;
+        if (!warp_wait(smem_u32(&bars.sp_done[it & 1]), (it >> 1) & 1, abort_flag)) break;
         tr.mark(3, it);
         tc_fence_after();
         if (elect_one()) {
           const int slot = it % C::NS;
-          const uint64_t za = zdesc_mn + ((slot * C::SLOT) >> 4);
+          const uint64_t zb = zdesc_mn + ((slot * C::SLOT) >> 4);
+          const uint64_t pa = pdesc0 + (((it & 1) * C::PBUF) >> 4);
           if (cur.first) {
 #pragma unroll
             for (int ks = 0; ks < kPage / 16; ++ks)
-#pragma unroll
-              for (int mc = 0; mc < C::NMC; ++mc)
-                mma_bf16_ss(tmem + C::COL_O + 16 * mc, za + (((C::mc_start(mc) / 64) * C::PCHUNK + ks * 2048) >> 4),
-                            pdesc + ((ks * 512) >> 4), IDESC_PV, ks > 0);
+              mma_bf16_ss(tmem + C::COL_O, pa + ((ks * KSTEP) >> 4), zb + ((ks * 2048) >> 4), IDESC_PV, ks > 0);
           } else {
 #pragma unroll
             for (int ks = 0; ks < kPage / 16; ++ks)
-#pragma unroll
-              for (int mc = 0; mc < C::NMC; ++mc)
-                mma_bf16_ss(tmem + C::COL_O + 16 * mc, za + (((C::mc_start(mc) / 64) * C::PCHUNK + ks * 2048) >> 4),
-                            pdesc + ((ks * 512) >> 4), IDESC_PV, 1);
+              mma_bf16_ss(tmem + C::COL_O, pa + ((ks * KSTEP) >> 4), zb + ((ks * 2048) >> 4), IDESC_PV, 1);
           }
-          mma_commit(smem_u32(&bars.o_ready));
           mma_commit(smem_u32(&bars.empty[slot]));
+          mma_commit(smem_u32(&bars.pfree[it & 1]));
         }
         __syncwarp();
-        last_bar = smem_u32(&bars.o_ready);
-        last_par = it & 1;
         cur = nxt;
         have = have_next;
         ++it;
       }
-      // drain: the last MMAs must finish before TMEM is released
-      if (last_bar != 0) mbar_wait(last_bar, last_par, abort_flag);
+      // drain: every MMA issued must finish before TMEM is released (one commit
+      // on a barrier of its own tracks all of them)
+      if (elect_one()) mma_commit(smem_u32(&bars.drain));
+      __syncwarp();
+      mbar_wait(smem_u32(&bars.drain), 0, abort_flag);
     }
     __syncwarp();
-  } else if (warp == 2) {
-    // ---------------------------------------------------------------- gate-row gather (TMA)
-    // For every page: its 64 token ids (two per lane), then one bulk copy of
-    // the gate row G[id] per valid token into a double-buffered row area.
-    if (GATE) {
-      const uint64_t pol_keep = policy_evict_last();
-      Walker w;
-      w.start(p.cu, p.seq_lens, p.batch);
-      Tile t;
-      int j = 0;
-      int bt_b = -1, bt_base = 0, bt_reg = -1;
-      int last_j[2] = {-1, -1};
-      while (w.next(t)) {
-        if (t.b != bt_b || t.lp >= bt_base + 32) {
-          bt_b = t.b;
-          bt_base = t.lp;
-          const int lp = t.lp + lane;
-          bt_reg = lp < p.max_pages ? __ldg(p.block_table + static_cast<size_t>(t.b) * p.max_pages + lp) : -1;
-        }
-        const int pg = __shfl_sync(0xffffffffu, bt_reg, t.lp - bt_base);
-        const int ntok = (pg >= 0 && pg < p.num_pages) ? t.ntok : 0;   // bad pages: reported by the producer
-        const int gb = j & 1;
-        int ids[2];
-#pragma unroll
-        for (int r = 0; r < 2; ++r) {
-          const int row = lane + 32 * r;
-          int id = row < ntok ? __ldg(p.id_pool + static_cast<size_t>(pg) * kPage + row) : 0;
-          if (row < ntok && (unsigned)id >= (unsigned)p.vocab) {
-            report_status(p.status, kStatusOutOfRange);
-            id = 0;
-          }
-          ids[r] = id;
-        }
-        if (!warp_wait(smem_u32(&bars.gempty[gb]), ((j >> 1) & 1) ^ 1, abort_flag)) break;
-        int32_t* gids = reinterpret_cast<int32_t*>(smem + C::OFF_GIDS + gb * C::GIDS);
-        gids[lane] = ids[0];
-        gids[lane + 32] = ids[1];
-        __syncwarp();
-        const uint32_t gbar = smem_u32(&bars.gfull[gb]);
-        if (lane == 0) mbar_arrive_expect_tx(gbar, static_cast<uint32_t>(ntok) * D_C * 2);
-        __syncwarp();
-        const uint32_t gdst = sbase + C::OFF_GBUF + gb * C::GBUF;
-#pragma unroll
-        for (int r = 0; r < 2; ++r) {
-          const int row = lane + 32 * r;
-          if (row < ntok)
-            bulk_load_hint(gdst + row * C::GSTRIDE, p.gate_table + static_cast<size_t>(ids[r]) * D_C, D_C * 2,
-                           gbar, pol_keep);
-        }
-        last_j[gb] = j;
-        ++j;
-      }
-      // drain: the copies this warp issued must land before the CTA exits
-      for (int b = 0; b < 2; ++b)
-        if (last_j[b] >= 0) mbar_wait(smem_u32(&bars.gfull[b]), (last_j[b] >> 1) & 1, abort_flag);
-    }
-    __syncwarp();
-  } else if (warp >= kGateWarp0 && warp < kGateWarp0 + 4) {
+  } else if (warp >= kGateWarp0) {
     // ---------------------------------------------------------------- gate: z = c (*) g, LN statistics
-    regs_increase<kConsumerRegs>();
+    // Quarter-warp k = 4 (warp - 4) + lane / 8 owns token rows 2k and 2k + 1;
+    // lane u = lane % 8 takes the 16-byte unit u of every 64-feature column of
+    // both rows.  Each quarter-warp access then covers one whole 128-byte line:
+    // of the gate table (a global load that reads whole lines costs the SM's
+    // load/store data path one wavefront per line, one that reads parts of many
+    // lines about one per lane) and of the swizzled page (eight distinct bank
+    // groups).  The gate rows come from L2 (the table stays there under an
+    // evict-last hint while the cache stream is evict-first): each tile issues
+    // the id loads of the tile two ahead and the gate-row loads of the next
+    // tile, so neither latency sits on the loop.
     const int gw = warp - kGateWarp0;
-    const int row = gw * 16 + (lane & 15);    // token row of the page
-    const int half = lane >> 4;               // 16-byte units 2k + half of every 128-byte chunk row
-    const int sw = row & 7;
+    const int u = lane & 7;
+    const int row0 = 2 * (gw * 4 + (lane >> 3));   // rows row0 and row0 + 1
+    const uint64_t pol_keep = policy_evict_last();
     Walker w;
     w.start(p.cu, p.seq_lens, p.batch);
+    PageWindow pw;
+    // ids of this thread's two rows of a tile (0 past the end of the page or for
+    // a bad page, which the producer reports)
+    auto load_ids = [&](const Tile& tt, int (&id)[2]) {
+      const int pg = pw.page(p, tt, lane);
+      const int n = (pg >= 0 && pg < p.num_pages) ? tt.ntok : 0;
+#pragma unroll
+      for (int rr = 0; rr < 2; ++rr)
+        id[rr] = row0 + rr < n ? __ldg(p.id_pool + static_cast<size_t>(pg) * kPage + row0 + rr) : 0;
+    };
+    auto load_g = [&](int (&id)[2], uint4 (&gv)[2][C::NCH]) {
+#pragma unroll
+      for (int rr = 0; rr < 2; ++rr) {
+        if ((unsigned)id[rr] >= (unsigned)p.vocab) {
+          report_status(p.status, kStatusOutOfRange);
+          id[rr] = 0;
+        }
+        const __nv_bfloat16* src = p.gate_table + static_cast<size_t>(id[rr]) * D_C + u * 8;
+#pragma unroll
+        for (int fc = 0; fc < C::NCH; ++fc) gv[rr][fc] = ldg_16_na_hint(src + fc * 64, pol_keep);
+      }
+    };
     Tracer tr;
     tr.init(p, 2);
     if (threadIdx.x != kGateWarp0 * 32) tr.base = nullptr;
-    Tile t;
+    Tile t, t1, t2;
+    bool have = w.next(t);
+    bool have1 = have && w.next(t1);
+    bool have2 = have1 && w.next(t2);
+    int id0[2] = {0, 0}, id1[2] = {0, 0}, id2[2] = {0, 0};   // ids of tiles j, j + 1, j + 2
+    uint4 gcur[2][C::NCH], gnext[2][C::NCH];
+    if (GATE) {
+      if (have) load_ids(t, id0);
+      if (have1) load_ids(t1, id1);
+      if (have) load_g(id0, gcur);
+    }
     int j = 0;
-    while (w.next(t)) {
+    while (have) {
       const int slot = j % C::NS;
-      const int gb = j & 1;
       tr.mark(0, j);
-      if (!warp_wait(smem_u32(&bars.full[slot]), (j / C::NS) & 1, abort_flag)) break;
-      if (GATE && !warp_wait(smem_u32(&bars.gfull[gb]), (j >> 1) & 1, abort_flag)) break;
-      tr.mark(1, j);
-      uint8_t* crow = smem + slot * C::SLOT + row * 128;
-      const uint8_t* grow = smem + C::OFF_GBUF + gb * C::GBUF + row * C::GSTRIDE;
-      const bool valid = row < t.ntok;
-      if (DUMP) {
-        if (valid && half == 0) {
-          const int id = reinterpret_cast<const int32_t*>(smem + C::OFF_GIDS + gb * C::GIDS)[row];
-          const size_t o = static_cast<size_t>(t.b) * p.dump_len + t.tok0 + row;
-          p.dump_ids[o] = id;
-          uint4* dc = reinterpret_cast<uint4*>(p.dump_c + o * D_C);
-          uint4* dg = reinterpret_cast<uint4*>(p.dump_g + o * D_C);
-          uint4* dk = reinterpret_cast<uint4*>(p.dump_kr + o * kRope);
-          for (int fc = 0; fc < C::NCH; ++fc)
-            for (int u = 0; u < 8; ++u) {
-              dc[fc * 8 + u] = *reinterpret_cast<const uint4*>(crow + fc * C::PCHUNK + ((u ^ sw) << 4));
-              dg[fc * 8 + u] = *reinterpret_cast<const uint4*>(grow + fc * 128 + u * 16);
-            }
-          for (int u = 0; u < 8; ++u)
-            dk[u] = *reinterpret_cast<const uint4*>(smem + slot * C::SLOT + C::KR_OFF + row * 128 + ((u ^ sw) << 4));
-        }
-        mbar_arrive(smem_u32(&bars.empty[slot]));
-        mbar_arrive(smem_u32(&bars.gempty[gb]));
-        ++j;
-        continue;
-      }
-      float2* stat = reinterpret_cast<float2*>(smem + C::OFF_STAT + slot * C::STAT_BYTES);
       if (GATE) {
-        // all shared-memory reads of this thread's units first (the in-place
-        // stores below would otherwise order every later load behind them)
-        uint4 cv[C::NCH * 4], gv[C::NCH * 4];
-#pragma unroll
-        for (int i = 0; i < C::NCH * 4; ++i) {
-          const int fc = i >> 2, u = 2 * (i & 3) + half;
-          cv[i] = *reinterpret_cast<const uint4*>(crow + fc * C::PCHUNK + ((u ^ sw) << 4));
-          gv[i] = *reinterpret_cast<const uint4*>(grow + fc * 128 + u * 16);
-        }
-        const bool full_page = t.ntok == kPage;   // uniform: no token masking needed
-        float2 s1 = make_float2(0.f, 0.f), s2 = make_float2(0.f, 0.f);
-        float2 a1 = make_float2(0.f, 0.f), a2 = make_float2(0.f, 0.f);
-#pragma unroll
-        for (int i = 0; i < C::NCH * 4; ++i) {
-          const int fc = i >> 2, u = 2 * (i & 3) + half;
-          uint4 z;
-          z.x = mul_bf16x2(cv[i].x, gv[i].x);
-          z.y = mul_bf16x2(cv[i].y, gv[i].y);
-          z.z = mul_bf16x2(cv[i].z, gv[i].z);
-          z.w = mul_bf16x2(cv[i].w, gv[i].w);
-          if (!full_page && !valid) z = make_uint4(0, 0, 0, 0);
-          const float2 f0 = unpack_bf16x2(z.x), f1 = unpack_bf16x2(z.y);
-          const float2 f2 = unpack_bf16x2(z.z), f3 = unpack_bf16x2(z.w);
-          s1 = __fadd2_rn(s1, f0);
-          a1 = __fadd2_rn(a1, f1);
-          s1 = __fadd2_rn(s1, f2);
-          a1 = __fadd2_rn(a1, f3);
-          s2 = __ffma2_rn(f0, f0, s2);
-          a2 = __ffma2_rn(f1, f1, a2);
-          s2 = __ffma2_rn(f2, f2, s2);
-          a2 = __ffma2_rn(f3, f3, a2);
-          *reinterpret_cast<uint4*>(crow + fc * C::PCHUNK + ((u ^ sw) << 4)) = z;
-        }
-        s1 = __fadd2_rn(s1, a1);
-        s2 = __fadd2_rn(s2, a2);
-        float sum1 = s1.x + s1.y, sum2 = s2.x + s2.y;
-        sum1 += __shfl_xor_sync(0xffffffffu, sum1, 16);
-        sum2 += __shfl_xor_sync(0xffffffffu, sum2, 16);
-        constexpr float inv_dc = 1.f / D_C;
-        const float mu = sum1 * inv_dc;
-        const float var = fmaxf(sum2 * inv_dc - mu * mu, 0.f);
-        if (half == 0) stat[row] = valid ? make_float2(mu, rsqrtf(var + p.eps)) : make_float2(0.f, 0.f);
-      } else if (!valid) {
-#pragma unroll
-        for (int fc = 0; fc < C::NCH; ++fc)
-#pragma unroll
-          for (int k = 0; k < 4; ++k)
-            *reinterpret_cast<uint4*>(crow + fc * C::PCHUNK + (2 * k + half) * 16) = make_uint4(0, 0, 0, 0);
+        // prefetch: ids of tile j + 2, gate rows of tile j + 1
+        if (have2) load_ids(t2, id2);
+        if (have1) load_g(id1, gnext);
       }
-      tr.mark(2, j);
-      fence_proxy_async_smem();
-      mbar_arrive(smem_u32(&bars.zready[slot]));
-      if (GATE) mbar_arrive(smem_u32(&bars.gempty[gb]));
+      if (!warp_wait(smem_u32(&bars.full[slot]), (j / C::NS) & 1, abort_flag)) break;
+      tr.mark(1, j);
+      uint8_t* cpage = smem + slot * C::SLOT;
+      if (DUMP) {
+#pragma unroll
+        for (int rr = 0; rr < 2; ++rr) {
+          const int row = row0 + rr;
+          if (row < t.ntok) {
+            const size_t o = static_cast<size_t>(t.b) * p.dump_len + t.tok0 + row;
+            uint4* dc = reinterpret_cast<uint4*>(p.dump_c + o * D_C);
+            uint4* dg = reinterpret_cast<uint4*>(p.dump_g + o * D_C);
+#pragma unroll
+            for (int fc = 0; fc < C::NCH; ++fc) {
+              dc[fc * 8 + u] =
+                  *reinterpret_cast<const uint4*>(cpage + fc * C::PCHUNK + row * 128 + ((u ^ (row & 7)) << 4));
+              dg[fc * 8 + u] = gcur[rr][fc];
+            }
+            reinterpret_cast<uint4*>(p.dump_kr + o * kRope)[u] =
+                *reinterpret_cast<const uint4*>(cpage + C::KR_OFF + row * 128 + ((u ^ (row & 7)) << 4));
+            if (u == 0) p.dump_ids[o] = id0[rr];
+          }
+        }
+        warp_arrive(smem_u32(&bars.empty[slot]));
+      } else {
+        const bool full_page = t.ntok == kPage;   // uniform: no token masking needed
+        if (GATE) {
+          float* st = reinterpret_cast<float*>(smem + C::OFF_STAT + slot * C::STAT_BYTES);
+          // all shared-memory reads of this thread's units first (the in-place
+          // stores below would otherwise order every later load behind them)
+          uint4 cv[2][C::NCH];
+#pragma unroll
+          for (int rr = 0; rr < 2; ++rr) {
+            const int row = row0 + rr;
+#pragma unroll
+            for (int fc = 0; fc < C::NCH; ++fc)
+              cv[rr][fc] =
+                  *reinterpret_cast<const uint4*>(cpage + fc * C::PCHUNK + row * 128 + ((u ^ (row & 7)) << 4));
+          }
+          tr.mark(5, j);
+          float sum1[2], sum2[2];
+#pragma unroll
+          for (int rr = 0; rr < 2; ++rr) {
+            const int row = row0 + rr;
+            const bool valid = row < t.ntok;
+            float2 s1 = make_float2(0.f, 0.f), s2 = make_float2(0.f, 0.f);
+            float2 a1 = make_float2(0.f, 0.f), a2 = make_float2(0.f, 0.f);
+#pragma unroll
+            for (int fc = 0; fc < C::NCH; ++fc) {
+              uint4 z;
+              z.x = mul_bf16x2(cv[rr][fc].x, gcur[rr][fc].x);
+              z.y = mul_bf16x2(cv[rr][fc].y, gcur[rr][fc].y);
+              z.z = mul_bf16x2(cv[rr][fc].z, gcur[rr][fc].z);
+              z.w = mul_bf16x2(cv[rr][fc].w, gcur[rr][fc].w);
+              if (!full_page && !valid) z = make_uint4(0, 0, 0, 0);
+              const float2 f0 = unpack_bf16x2(z.x), f1 = unpack_bf16x2(z.y);
+              const float2 f2 = unpack_bf16x2(z.z), f3 = unpack_bf16x2(z.w);
+              s1 = __fadd2_rn(s1, f0);
+              a1 = __fadd2_rn(a1, f1);
+              s1 = __fadd2_rn(s1, f2);
+              a1 = __fadd2_rn(a1, f3);
+              s2 = __ffma2_rn(f0, f0, s2);
+              a2 = __ffma2_rn(f1, f1, a2);
+              s2 = __ffma2_rn(f2, f2, s2);
+              a2 = __ffma2_rn(f3, f3, a2);
+              *reinterpret_cast<uint4*>(cpage + fc * C::PCHUNK + row * 128 + ((u ^ (row & 7)) << 4)) = z;
+            }
+            s1 = __fadd2_rn(s1, a1);
+            s2 = __fadd2_rn(s2, a2);
+            sum1[rr] = s1.x + s1.y;
+            sum2[rr] = s2.x + s2.y;
+          }
+          tr.mark(6, j);
+          // row sums over the eight lanes of the quarter-warp
+#pragma unroll
+          for (int o = 1; o < 8; o <<= 1) {
+#pragma unroll
+            for (int rr = 0; rr < 2; ++rr) {
+              sum1[rr] += __shfl_xor_sync(0xffffffffu, sum1[rr], o);
+              sum2[rr] += __shfl_xor_sync(0xffffffffu, sum2[rr], o);
+            }
+          }
+          if (u < 2) {
+            // lane 0 of the quarter-warp publishes row0, lane 1 row0 + 1
+            const int row = row0 + u;
+            const float a = u ? sum1[1] : sum1[0], b2 = u ? sum2[1] : sum2[0];
+            constexpr float inv_dc = 1.f / D_C;
+            const float mu = a * inv_dc;
+            const float var = fmaxf(b2 * inv_dc - mu * mu, 0.f);
+            const float r = rsqrtf(var + p.eps);
+            const bool valid = row < t.ntok;
+            st[row] = valid ? mu : 0.f;
+            st[kPage + row] = valid ? r : 0.f;
+            st[2 * kPage + row] = valid ? 1.f / r : 0.f;
+          }
+        } else if (!full_page) {
+#pragma unroll
+          for (int rr = 0; rr < 2; ++rr) {
+            const int row = row0 + rr;
+            if (row >= t.ntok) {
+#pragma unroll
+              for (int fc = 0; fc < C::NCH; ++fc)
+                *reinterpret_cast<uint4*>(cpage + fc * C::PCHUNK + row * 128 + (u << 4)) = make_uint4(0, 0, 0, 0);
+            }
+          }
+        }
+        tr.mark(2, j);
+        fence_proxy_async_smem();
+        warp_arrive(smem_u32(&bars.zready[slot]));
+      }
       tr.mark(3, j);
       ++j;
-    }
-  } else if (warp >= kSoftWarp0 && !DUMP) {
-    // ---------------------------------------------------------------- softmax, output read-out
-    regs_increase<kConsumerRegs>();
-    const int q4 = warp & 3;                   // TMEM lane quadrant of this warp
-    const int srow = q4 * 16 + lane;           // token row of the M=64 score accumulator (lane < 16)
-    const bool token_lane = lane < 16;
-    const int frow = q4 * 32 + lane;           // latent feature row of the PV accumulator
-    const uint32_t tl = tmem + (static_cast<uint32_t>(q4 * 32) << 16);
-    // Online softmax with a lazily updated reference max m_ref per head: the
-    // exponentials are taken against m_ref, which only moves (rescaling the
-    // TMEM accumulator, l and the mean correction) when a tile's max exceeds it
-    // by more than 2^kLazyLog2; otherwise the weights stay below 2^kLazyLog2.
-    float m_ref[16], l_part[16], bmu_part[16];
-    float gam[C::NMC], bet[C::NMC];
+      t = t1;
+      t1 = t2;
+      have = have1;
+      have1 = have2;
+      have2 = have2 && w.next(t2);
+      if (GATE) {
 #pragma unroll
-    for (int mc = 0; mc < C::NMC; ++mc) {
-      const int f = C::mc_start(mc) + frow;
-      gam[mc] = (GATE && p.gamma) ? p.gamma[f] : 1.f;
-      bet[mc] = (GATE && p.beta) ? p.beta[f] : 0.f;
+        for (int rr = 0; rr < 2; ++rr) {
+          id0[rr] = id1[rr];
+          id1[rr] = id2[rr];
+#pragma unroll
+          for (int fc = 0; fc < C::NCH; ++fc) gcur[rr][fc] = gnext[rr][fc];
+        }
+      }
     }
+  } else if (warp < kSoftWarps && !DUMP) {
+    // ---------------------------------------------------------------- softmax, output read-out
+    // Warp hw owns heads 8hw..8hw+7, whose rows of S^T and O sit in TMEM lanes
+    // 32hw..32hw+7.  Thread t owns head hd = 8hw + t/4 and, in every 8-token
+    // group k of a page, the tokens 8k + 2(t%4) and 8k + 2(t%4) + 1.  The
+    // 16-lane TMEM loads also return lanes 32hw+8..32hw+15 (rows no head uses),
+    // which are ignored.
+    const int hw = warp, hd = 8 * hw + (lane >> 2), qq = lane & 3;
+    const uint32_t tq = tmem + (static_cast<uint32_t>(32 * hw) << 16);
+    const float scale = p.scale_log2;
+    // Online softmax with a lazily updated reference max m_ref per head: the
+    // exponentials are taken against m_ref, which only moves (rescaling the TMEM
+    // accumulator, l and the mean correction) when a tile's max exceeds it by
+    // more than 2^kLazyLog2; otherwise the weights stay below 2^kLazyLog2.
+    float m_ref = 0.f, l_acc = 0.f, bmu_acc = 0.f, wq = 0.f, bsc = 0.f;
     Walker w;
     w.start(p.cu, p.seq_lens, p.batch);
     Tile t;
-    int it = 0, seg = -1, nseg_end = 0;
+    int it = 0, seg = -1;
     Tracer tr;
     tr.init(p, 3);
-    if (threadIdx.x != kSoftWarp0 * 32) tr.base = nullptr;
+    if (threadIdx.x != 0) tr.base = nullptr;
     while (w.next(t)) {
       if (t.first) {
         ++seg;
-#pragma unroll
-        for (int h = 0; h < 16; ++h) {
-          l_part[h] = 0.f;
-          bmu_part[h] = 0.f;
-        }
         if (!warp_wait(smem_u32(&bars.qfull[seg & 1]), (seg >> 1) & 1, abort_flag)) break;
+        if (GATE) {
+          // w_h = sum_f bf16(q^ gamma)_hf and b_h = q^_h . beta, after the operands
+          const float* sums = reinterpret_cast<const float*>(smem + C::OFF_QBUF + (seg & 1) * C::QBUF + C::QB_LAT +
+                                                             C::QB_ROPE);
+          wq = sums[hd];
+          bsc = sums[16 + hd] * scale;
+        }
+        warp_arrive(smem_u32(&bars.qempty[seg & 1]));
+        l_acc = 0.f;
+        bmu_acc = 0.f;
       }
       const int slot = it % C::NS;
       const int par = it & 1;
       tr.mark(0, it);
-      // the gate's statistics for this tile are published with its zready arrival
-      if (GATE && !warp_wait(smem_u32(&bars.zready[slot]), (it / C::NS) & 1, abort_flag)) break;
+      // Scores of this tile.  Their completion also implies (same issuing
+      // thread, earlier commit) that the output MMA two tiles back is done, so
+      // the weight buffer of this parity is free; and the MMA warp's release
+      // arrival on the same barrier orders the gate's statistics before it.
       if (!warp_wait(smem_u32(&bars.s_ready[par]), (it >> 1) & 1, abort_flag)) break;
       tr.mark(1, it);
       tc_fence_after();
-      float sl[16], sr[16], s[16];
-      tmem_ld16(tl + C::COL_S + par * C::S_COLS, sl);
-      tmem_ld16(tl + C::COL_S + par * C::S_COLS + 16, sr);
-      const bool valid = token_lane && srow < t.ntok;
-      float mu = 0.f, rstd = 1.f;
-      if (GATE && token_lane) {
-        const float2 st = reinterpret_cast<const float2*>(smem + C::OFF_STAT + slot * C::STAT_BYTES)[srow];
-        mu = st.x;
-        rstd = st.y;
-      }
-      const float4* sums4 = reinterpret_cast<const float4*>(smem + C::OFF_QBUF + (seg & 1) * C::QBUF + C::QB_LAT +
-                                                            C::QB_ROPE);
-      float wq[16], bq[16];
+      float sl[32], sr[32];
+      tmem_ld_16x256b_x8(tq + C::COL_S + par * C::S_COLS, sl);
+      tmem_ld_16x256b_x8(tq + C::COL_S + par * C::S_COLS + kPage, sr);
+      const float* st = reinterpret_cast<const float*>(smem + C::OFF_STAT + slot * C::STAT_BYTES);
+      float2 mu2[8], r2[8], ri2[8];
       if (GATE) {
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const float4 a = sums4[k], b = sums4[4 + k];
-          wq[4 * k] = a.x; wq[4 * k + 1] = a.y; wq[4 * k + 2] = a.z; wq[4 * k + 3] = a.w;
-          bq[4 * k] = b.x; bq[4 * k + 1] = b.y; bq[4 * k + 2] = b.z; bq[4 * k + 3] = b.w;
+        for (int k = 0; k < 8; ++k) {
+          mu2[k] = *reinterpret_cast<const float2*>(st + 8 * k + 2 * qq);
+          r2[k] = *reinterpret_cast<const float2*>(st + kPage + 8 * k + 2 * qq);
+          ri2[k] = *reinterpret_cast<const float2*>(st + 2 * kPage + 8 * k + 2 * qq);
         }
       }
       tmem_wait_ld();
-#pragma unroll
-      for (int h = 0; h < 16; ++h) {
-        const float lat = GATE ? rstd * (sl[h] - mu * wq[h]) + bq[h] : sl[h];
-        s[h] = valid ? (lat + sr[h]) * p.scale_log2 : -INFINITY;
-      }
-      const float wmax = warp_reduce16<true>(s, lane);
-      if ((lane & 1) == 0) red_max[(par * 16 + (lane >> 1)) * 4 + q4] = wmax;
-      mbar_arrive(smem_u32(&bars.red[par]));
-      if (!warp_wait(smem_u32(&bars.red[par]), (it >> 1) & 1, abort_flag)) break;
-      tr.mark(2, it);
-      // the previous tile's PV (same segment) must be complete before the
-      // weight buffer is rewritten or the accumulator rescaled
-      if (!t.first && !warp_wait(smem_u32(&bars.o_ready), (it - 1) & 1, abort_flag)) break;
-      tr.mark(5, it);
-      bool rescale = false;
-      float alpha[16];
-#pragma unroll
-      for (int h = 0; h < 16; ++h) {
-        const float4 rm = reinterpret_cast<const float4*>(red_max)[par * 16 + h];
-        const float tmax = fmaxf(fmaxf(rm.x, rm.y), fmaxf(rm.z, rm.w));
-        alpha[h] = 1.f;
-        if (t.first) {
-          m_ref[h] = tmax;
-        } else if (tmax > m_ref[h] + kLazyLog2) {
-          alpha[h] = exp2f(m_ref[h] - tmax);
-          m_ref[h] = tmax;
-          rescale = true;
-        }
-      }
-      if (rescale) {
-        // every thread saw the same maxima, so the branch is uniform
-        tc_fence_after();
-#pragma unroll
-        for (int mc = 0; mc < C::NMC; ++mc) {
-          float o[16];
-          tmem_ld16(tl + C::COL_O + 16 * mc, o);
-          tmem_wait_ld();
-#pragma unroll
-          for (int h = 0; h < 16; ++h) o[h] *= alpha[h];
-          tmem_st16(tl + C::COL_O + 16 * mc, o);
-        }
-        tmem_wait_st();
-#pragma unroll
-        for (int h = 0; h < 16; ++h) {
-          l_part[h] *= alpha[h];
-          bmu_part[h] *= alpha[h];
-        }
-      }
-      // The PV MMA sees the bf16-rounded weights P'; the denominator and the mean
-      // correction use the same rounded values (l = sum P'/r), so the rounding of
-      // P' cancels in o = (sum P' z - sum P' mu) / l instead of biasing it.
-      const float inv_r = GATE ? (valid ? 1.f / rstd : 0.f) : 1.f;
-#pragma unroll
-      for (int h = 0; h < 16; ++h) {
-        const float pr = ex2_approx(s[h] - m_ref[h]);
-        s[h] = GATE ? pr * rstd : pr;
-      }
-      uint32_t pw[8];
+      tr.mark(7, it);
+      // s[2k + e]: token 8k + 2 qq + e of head hd (log2 units)
+      float s[16];
+      const bool full_page = t.ntok == kPage;
 #pragma unroll
       for (int k = 0; k < 8; ++k) {
-        pw[k] = pack_bf16x2(s[2 * k], s[2 * k + 1]);
-        const float2 pq = unpack_bf16x2(pw[k]);
-        l_part[2 * k] = fmaf(pq.x, inv_r, l_part[2 * k]);
-        l_part[2 * k + 1] = fmaf(pq.y, inv_r, l_part[2 * k + 1]);
-        if (GATE) {
-          bmu_part[2 * k] = fmaf(pq.x, mu, bmu_part[2 * k]);
-          bmu_part[2 * k + 1] = fmaf(pq.y, mu, bmu_part[2 * k + 1]);
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const float lat = sl[4 * k + e], rope = sr[4 * k + e];
+          float v;
+          if (GATE) {
+            const float mu = e ? mu2[k].y : mu2[k].x;
+            const float rs = (e ? r2[k].y : r2[k].x) * scale;
+            v = fmaf(rs, fmaf(-mu, wq, lat), fmaf(rope, scale, bsc));
+          } else {
+            v = (lat + rope) * scale;
+          }
+          const bool valid = full_page || (8 * k + 2 * qq + e) < t.ntok;
+          s[2 * k + e] = valid ? v : -INFINITY;
         }
       }
-      // P'[token][head] as an MN-major B operand: 8x8 core matrices, token group
-      // stride 256 B, head group stride 128 B
-      if (token_lane) {
-        uint8_t* prow = smem + C::OFF_PBUF + (srow >> 3) * 256 + (srow & 7) * 16;
-        *reinterpret_cast<uint4*>(prow) = make_uint4(pw[0], pw[1], pw[2], pw[3]);
-        *reinterpret_cast<uint4*>(prow + 128) = make_uint4(pw[4], pw[5], pw[6], pw[7]);
+      tr.mark(8, it);
+      // tile max of the head: 16 tokens in-thread (a tree), then its four threads
+      float m8[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) m8[i] = fmaxf(s[i], s[i + 8]);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) m8[i] = fmaxf(m8[i], m8[i + 4]);
+      float mx = fmaxf(fmaxf(m8[0], m8[2]), fmaxf(m8[1], m8[3]));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+      float alpha = 1.f;
+      bool rescale = false;
+      if (t.first) {
+        m_ref = mx;
+      } else if (mx > m_ref + kLazyLog2) {
+        alpha = ex2_approx(m_ref - mx);
+        m_ref = mx;
+        rescale = true;
+      }
+      tr.mark(2, it);
+      if (__any_sync(0xffffffffu, rescale)) {
+        // The previous tile's output MMA must be complete before O is rescaled.
+        // Phase n of pfree[b] completes with output MMA 2n + b; the MMA two
+        // tiles before that is known complete (see above), so this buffer's
+        // phase count is at most one behind and the parity wait is exact.
+        if (!warp_wait(smem_u32(&bars.pfree[(it - 1) & 1]), ((it - 1) >> 1) & 1, abort_flag)) break;
+        tc_fence_after();
+#pragma unroll 1
+        for (int c = 0; c < D_C / 64; ++c) {
+          float o[32];
+          tmem_ld_16x256b_x8(tq + C::COL_O + 64 * c, o);
+          tmem_wait_ld();
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            o[4 * k] *= alpha;
+            o[4 * k + 1] *= alpha;
+          }
+          tmem_st_16x256b_x8(tq + C::COL_O + 64 * c, o);
+        }
+        tmem_wait_st();
+        l_acc *= alpha;
+        bmu_acc *= alpha;
+      }
+      tr.mark(5, it);
+      // The output MMA sees the bf16-rounded weights P'; the denominator and the
+      // mean correction use the same rounded values (l = sum P'/r), so the
+      // rounding of P' cancels in o = (sum P' z - sum P' mu) / l.
+      uint8_t* pbuf = smem + C::OFF_PBUF + par * C::PBUF + qop_offset(hd, 2 * qq);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const float r0 = GATE ? r2[k].x : 1.f, r1 = GATE ? r2[k].y : 1.f;
+        const float p0 = ex2_approx(s[2 * k] - m_ref) * r0;
+        const float p1 = ex2_approx(s[2 * k + 1] - m_ref) * r1;
+        const uint32_t pw = pack_bf16x2(p0, p1);
+        const float2 pq = unpack_bf16x2(pw);
+        if (GATE) {
+          l_acc = fmaf(pq.x, ri2[k].x, fmaf(pq.y, ri2[k].y, l_acc));
+          bmu_acc = fmaf(pq.x, mu2[k].x, fmaf(pq.y, mu2[k].y, bmu_acc));
+        } else {
+          l_acc += pq.x + pq.y;
+        }
+        *reinterpret_cast<uint32_t*>(pbuf + k * kQGroupBytes) = pw;
       }
       tr.mark(6, it);
       fence_proxy_async_smem();
       tc_fence_before();
-      tr.mark(7, it);
-      mbar_arrive(smem_u32(&bars.sp_done));
+      warp_arrive(smem_u32(&bars.sp_done[par]));
       tr.mark(3, it);
 
       if (t.last) {
-        mbar_arrive(smem_u32(&bars.qempty[seg & 1]));
-        // ---- segment end: reduce l and sum_j P'_j mu_j over the token rows
-        const float lw = warp_reduce16<false>(l_part, lane);
-        const float bw = GATE ? warp_reduce16<false>(bmu_part, lane) : 0.f;
-        if ((lane & 1) == 0) {
-          red_sum[q4 * 32 + (lane >> 1)] = lw;
-          red_sum[q4 * 32 + 16 + (lane >> 1)] = bw;
-        }
-        mbar_arrive(smem_u32(&bars.sum));
-        if (!warp_wait(smem_u32(&bars.sum), nseg_end & 1, abort_flag)) break;
-        ++nseg_end;
-        float lh[16], bh[16];
-#pragma unroll
-        for (int h = 0; h < 16; ++h) {
-          lh[h] = red_sum[h] + red_sum[32 + h] + red_sum[64 + h] + red_sum[96 + h];
-          bh[h] = red_sum[16 + h] + red_sum[48 + h] + red_sum[80 + h] + red_sum[112 + h];
-        }
-        // the segment's last PV, then the accumulated latent output
-        if (!warp_wait(smem_u32(&bars.o_ready), it & 1, abort_flag)) break;
+        // ---- segment end: l and sum_j P'_j mu_j over the four threads of the head
+        float lh = l_acc, bh = bmu_acc;
+        lh += __shfl_xor_sync(0xffffffffu, lh, 1);
+        bh += __shfl_xor_sync(0xffffffffu, bh, 1);
+        lh += __shfl_xor_sync(0xffffffffu, lh, 2);
+        bh += __shfl_xor_sync(0xffffffffu, bh, 2);
+        // the segment's last output MMA (the earlier ones complete before it;
+        // exact parity wait as for the rescale), then the accumulated output
+        if (!warp_wait(smem_u32(&bars.pfree[par]), (it >> 1) & 1, abort_flag)) break;
         tc_fence_after();
         const int slot_out = blockIdx.x + t.b;
-        float* po = p.part_o + static_cast<size_t>(slot_out) * kHeads * D_C;
-#pragma unroll
-        for (int mc = 0; mc < C::NMC; ++mc) {
-          float o[16];
-          tmem_ld16(tl + C::COL_O + 16 * mc, o);
+        float* po = p.part_o + (static_cast<size_t>(slot_out) * kHeads + hd) * D_C;
+#pragma unroll 1
+        for (int c = 0; c < D_C / 64; ++c) {
+          float o[32];
+          tmem_ld_16x256b_x8(tq + C::COL_O + 64 * c, o);
           tmem_wait_ld();
-          const int f = C::mc_start(mc) + frow;
-          if (mc == 0 || f >= 128 * mc) {
 #pragma unroll
-            for (int h = 0; h < 16; ++h)
-              po[h * D_C + f] = GATE ? fmaf(gam[mc], o[h] - bh[h], bet[mc] * lh[h]) : o[h];
+          for (int k = 0; k < 8; ++k) {
+            const int f = 64 * c + 8 * k + 2 * qq;
+            float2 v = make_float2(o[4 * k], o[4 * k + 1]);
+            if (GATE) {
+              float2 gm = make_float2(1.f, 1.f), bt = make_float2(0.f, 0.f);
+              if (p.gamma) gm = __ldg(reinterpret_cast<const float2*>(p.gamma + f));
+              if (p.beta) bt = __ldg(reinterpret_cast<const float2*>(p.beta + f));
+              v.x = fmaf(gm.x, v.x - bh, bt.x * lh);
+              v.y = fmaf(gm.y, v.y - bh, bt.y * lh);
+            }
+            *reinterpret_cast<float2*>(po + f) = v;
           }
         }
         tc_fence_before();
-        if (frow < 16) {
-          float mv = 0.f, lv = 0.f;
-#pragma unroll
-          for (int h = 0; h < 16; ++h)
-            if (h == frow) {
-              mv = m_ref[h];
-              lv = lh[h];
-            }
-          float* ml = p.part_ml + (static_cast<size_t>(slot_out) * kHeads + frow) * 2;
-          ml[0] = mv;
-          ml[1] = lv;
+        if (qq == 0) {
+          float* ml = p.part_ml + (static_cast<size_t>(slot_out) * kHeads + hd) * 2;
+          ml[0] = m_ref;
+          ml[1] = lh;
         }
         tr.mark(4, it);
       }
@@ -865,7 +876,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  if (warp == 1) tmem_dealloc(tmem, C::TMEM_COLS);
+  if (warp == kMmaWarp) tmem_dealloc(tmem, C::TMEM_COLS);
   if (threadIdx.x == 0 && bars.abort) report_status(p.status, kStatusTimeout);
 }
 
@@ -926,7 +937,7 @@ cudaError_t launch_decode_tc(const DecodeArgs& a, const CUtensorMap* maps, bool 
   } else {
     if (a.d_c == 192) return launch_one<192, false, false>(a, maps, st);
     if (a.d_c == 256) return launch_one<256, false, false>(a, maps, st);
-    if (a.d_c == 512) return launch_one<512, false, false>(a, maps, st);
+    if (a.d_c == 512) return launch_decode_wide(a, maps, st);
   }
   return cudaErrorInvalidValue;
 }
