@@ -145,7 +145,7 @@ size_t eg_mla_decode_workspace_size(const eg_mla_dims* dims, int32_t batch, int3
  * v^C = W_UV c~ (weight absorption).  A sequence with L_b = 0 gets u = 0.
  *
  *   q            [batch, num_heads, d_nope + d_rope] model dtype; RoPE already
- *                applied to the last d_rope entries
+ *                applied to the last d_rope entries; 16-byte aligned
  *   c_pool, krope_pool, id_pool: the paged cache (see eg_mla_append_latent);
  *                id_pool may be NULL for EG_MLA_GATE_NONE.  c_pool and
  *                krope_pool must be 16-byte aligned.
@@ -156,8 +156,9 @@ size_t eg_mla_decode_workspace_size(const eg_mla_dims* dims, int32_t batch, int3
  *                vocabulary entry (EG-MLA-A); ignored for EG_MLA_GATE_NONE
  *   ln_gamma, ln_beta  [d_c] fp32, may be NULL (gamma = 1, beta = 0)
  *   w_uk         [num_heads, d_nope, d_c] model dtype (the k_nope rows of the
- *                listing's wkv_b weight viewed per head)
- *   w_uv         [num_heads, d_v, d_c] model dtype (the v rows of wkv_b)
+ *                listing's wkv_b weight viewed per head), 16-byte aligned
+ *   w_uv         [num_heads, d_v, d_c] model dtype (the v rows of wkv_b),
+ *                16-byte aligned
  *   out          [batch, num_heads, d_v] model dtype, written
  *   num_splits   number of split-KV work units (0 = eg_mla_default_num_splits);
  *                the cache pages of all sequences are divided into this many

@@ -332,6 +332,8 @@ int eg_mla_decode(const eg_mla_dims* dims, const void* q, const void* c_pool, co
   if (rc != EG_MLA_OK) return rc;
   if (batch == 0) return EG_MLA_OK;
   if (q == nullptr || w_uk == nullptr || w_uv == nullptr || out == nullptr) return EG_MLA_ERR_INVALID_ARG;
+  // q, W_UK and W_UV rows are read in 16-byte pieces
+  if (!aligned(w_uv, 16) || !aligned(w_uk, 16) || !aligned(q, 16)) return EG_MLA_ERR_INVALID_ARG;
   a.q = q;
   a.ln_gamma = ln_gamma;
   a.ln_beta = ln_beta;

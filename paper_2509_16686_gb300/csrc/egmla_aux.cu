@@ -55,117 +55,118 @@ __global__ void append_latent_kernel(uint8_t* __restrict__ c_pool, uint8_t* __re
 }
 
 // ------------------------------------------------------------------ prologue
-// Exclusive prefix sum of pages per sequence: cu[b] = sum_{b'<b} ceil(L_b'/P).
+// Exclusive prefix sum of pages per sequence: cu[b] = sum_{b'<b} ceil(L_b'/P),
+// cu[batch] = total; a scan by the block's first warp, 32 sequences per pass.
 __device__ void page_prefix_sums(const int32_t* seq_lens, int batch, int page_size, int32_t* cu) {
-  if (threadIdx.x == 0) {
-    int32_t acc = 0;
-    for (int b = 0; b < batch; ++b) {
-      cu[b] = acc;
-      int L = seq_lens[b];
-      acc += L > 0 ? (L + page_size - 1) / page_size : 0;
+  if (threadIdx.x >= 32) return;
+  const int lane = threadIdx.x;
+  int32_t carry = 0;
+  for (int base = 0; base < batch; base += 32) {
+    const int b = base + lane;
+    const int L = b < batch ? seq_lens[b] : 0;
+    const int np = L > 0 ? (L + page_size - 1) / page_size : 0;
+    int incl = np;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int t = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += t;
     }
-    cu[batch] = acc;
+    if (b < batch) cu[b] = carry + incl - np;
+    carry += __shfl_sync(0xffffffffu, incl, 31);
   }
+  if (lane == 0) cu[batch] = carry;
 }
 
-__device__ __forceinline__ float block_sum_256(float v, float* red) {
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  __syncthreads();
-  if (lane == 0) red[w] = v;
-  __syncthreads();
-  float s = 0.f;
-  for (int i = 0; i < (int)(blockDim.x >> 5); ++i) s += red[i];
-  return s;
-}
+// Tensor-core path: block (head h, chunk of kSumFeatures latent features,
+// group of kPBatch sequences) computes q^_{b,h}[f] = sum_n W_UK,h[n][f] q^C_{b,h}[n]
+// in fp32 (thread: one feature, four sequences) from W_UK and q^C staged in
+// shared memory as bf16 (all 16-byte global loads of a thread are issued
+// before any is stored, so their latencies overlap), and stores (q^ (*) gamma)
+// rounded to bf16 in the prepared query block (qop_offset layout).  Its
+// per-chunk partials of w_h = sum_f bf16(q^ gamma)_f and b_h = q^_h . beta go to
+// the block's slots of the sums area.  Chunk-0 blocks also copy q^R.  The last
+// block computes the page prefix sums.
+constexpr int kPBatch = 32;
+constexpr int kPMaxNope = 256;
+constexpr int kPThreads = 256;
+constexpr int kPLoads = kPMaxNope * kSumFeatures * 2 / 16 / kPThreads;   // 16-byte pieces per thread and array
 
-// Tensor-core path: block (h, group of up to kQGroup sequences) computes
-// q^_{b,h} = W_UK,h^T q^C_{b,h} in fp32 (one latent feature per thread, W_UK,h
-// read once per group) and stores (q^ (*) gamma) as the bf16 B operand of the
-// score MMA, laid out in 8x8 core matrices (no swizzle, K-major): element
-// (head n, feature k) at byte (k/8)*256 + (n/8)*128 + (n%8)*16 + (k%8)*2.  q^R
-// goes to the same layout.  The per-head sums w_h = sum_f bf16(q^ gamma)_f and
-// b_h = q^_h . beta are the terms the LayerNorm contributes after the MMA.
-constexpr int kQGroup = 8;
-
-__global__ void __launch_bounds__(256)
-prologue_tc_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ w_uk,
-                   const float* __restrict__ gamma, const float* __restrict__ beta,
-                   const int32_t* __restrict__ seq_lens, int batch, int d_nope, int d_rope, int d_c,
-                   int page_size, uint8_t* __restrict__ qprep, size_t qstride, int32_t* __restrict__ cu) {
-  __shared__ float qn[kQGroup][256];
-  __shared__ float red[2][kQGroup][8];
-  const int H = 16;
-  const int ngroups = (batch + kQGroup - 1) / kQGroup;
-  if (blockIdx.x == static_cast<unsigned>(ngroups * H)) {
+__global__ void __launch_bounds__(kPThreads)
+    prologue_tc_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ w_uk,
+                       const float* __restrict__ gamma, const float* __restrict__ beta,
+                       const int32_t* __restrict__ seq_lens, int batch, int d_nope, int d_rope, int d_c,
+                       int page_size, uint8_t* __restrict__ qprep, size_t qstride, int32_t* __restrict__ cu) {
+  __shared__ __align__(16) __nv_bfloat16 ws[kPMaxNope][kSumFeatures];   // W_UK,h[n][f0 + f]
+  __shared__ __align__(16) __nv_bfloat16 qs[kPBatch][kPMaxNope];       // q^C_{b0 + j, h}[n]
+  constexpr int H = 16;
+  const int nchunk = d_c / kSumFeatures;
+  const int ngroups = (batch + kPBatch - 1) / kPBatch;
+  if (blockIdx.x == static_cast<unsigned>(H * nchunk * ngroups)) {
     page_prefix_sums(seq_lens, batch, page_size, cu);
     return;
   }
   if (q == nullptr) return;  // cache-read test entry: prefix sums only
-  const int h = blockIdx.x % H, b0 = (blockIdx.x / H) * kQGroup;
-  const int nb = min(kQGroup, batch - b0);
-  for (int i = threadIdx.x; i < kQGroup * d_nope; i += blockDim.x) {
-    const int j = i / d_nope, n = i % d_nope;
-    qn[j][n] = j < nb ? __bfloat162float(q[(static_cast<size_t>(b0 + j) * H + h) * (d_nope + d_rope) + n]) : 0.f;
+  const int h = blockIdx.x % H, fc = (blockIdx.x / H) % nchunk, bg = blockIdx.x / (H * nchunk);
+  const int b0 = bg * kPBatch, nb = min(kPBatch, batch - b0);
+  const int f0 = fc * kSumFeatures;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;   // feature f0 + lane; sequences b0 + 4 warp + i
+  const int qrow = d_nope + d_rope;
+  // W piece i: row n = i / 4, features 8 (i % 4) ..; q piece i: sequence j = i / (d_nope / 8), columns 8 (i % ..)
+  const int wpieces = d_nope * (kSumFeatures / 8), qpr = d_nope / 8, qpieces = kPBatch * qpr;
+  uint4 wv[kPLoads], qv[kPLoads];
+#pragma unroll
+  for (int k = 0; k < kPLoads; ++k) {
+    const int i = tid + k * kPThreads;
+    wv[k] = make_uint4(0, 0, 0, 0);
+    qv[k] = make_uint4(0, 0, 0, 0);
+    if (i < wpieces)
+      wv[k] = *reinterpret_cast<const uint4*>(w_uk + (static_cast<size_t>(h) * d_nope + i / 4) * d_c + f0 + 8 * (i % 4));
+    if (i < qpieces && i / qpr < nb)
+      qv[k] = *reinterpret_cast<const uint4*>(q + (static_cast<size_t>(b0 + i / qpr) * H + h) * qrow + 8 * (i % qpr));
+  }
+#pragma unroll
+  for (int k = 0; k < kPLoads; ++k) {
+    const int i = tid + k * kPThreads;
+    if (i < wpieces) *reinterpret_cast<uint4*>(&ws[i / 4][8 * (i % 4)]) = wv[k];
+    if (i < qpieces) *reinterpret_cast<uint4*>(&qs[i / qpr][8 * (i % qpr)]) = qv[k];
   }
   __syncthreads();
-  const __nv_bfloat16* w = w_uk + static_cast<size_t>(h) * d_nope * d_c;
-  float wpart[kQGroup], bpart[kQGroup];
-#pragma unroll
-  for (int j = 0; j < kQGroup; ++j) wpart[j] = bpart[j] = 0.f;
-  for (int f = threadIdx.x; f < d_c; f += blockDim.x) {
-    float acc[kQGroup];
-#pragma unroll
-    for (int j = 0; j < kQGroup; ++j) acc[j] = 0.f;
+  float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll 8
-    for (int n = 0; n < d_nope; ++n) {
-      const float wv = __bfloat162float(w[static_cast<size_t>(n) * d_c + f]);
+  for (int n = 0; n < d_nope; ++n) {
+    const float w = __bfloat162float(ws[n][lane]);
 #pragma unroll
-      for (int j = 0; j < kQGroup; ++j) acc[j] = fmaf(wv, qn[j][n], acc[j]);
-    }
-    const float gm = gamma ? gamma[f] : 1.f;
-    const float bt = beta ? beta[f] : 0.f;
-    const size_t off = qop_offset(h, f);
-#pragma unroll
-    for (int j = 0; j < kQGroup; ++j) {
-      if (j >= nb) break;
-      const __nv_bfloat16 bq = __float2bfloat16_rn(acc[j] * gm);
-      *reinterpret_cast<__nv_bfloat16*>(qprep + static_cast<size_t>(b0 + j) * qstride + off) = bq;
-      wpart[j] += __bfloat162float(bq);
-      bpart[j] = fmaf(acc[j], bt, bpart[j]);
-    }
+    for (int i = 0; i < 4; ++i) acc[i] = fmaf(w, __bfloat162float(qs[4 * warp + i][n]), acc[i]);
   }
-  for (int i = threadIdx.x; i < nb * d_rope; i += blockDim.x) {
-    const int j = i / d_rope, r = i % d_rope;
-    const size_t off = qprep_lat_bytes(d_c) + qop_offset(h, r);
-    *reinterpret_cast<__nv_bfloat16*>(qprep + static_cast<size_t>(b0 + j) * qstride + off) = q[(static_cast<size_t>(b0 + j) * H + h) * (d_nope + d_rope) + d_nope + r];
-  }
-  // per-sequence block sums of w and b
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int f = f0 + lane;
+  const float gm = gamma ? gamma[f] : 1.f;
+  const float bt = beta ? beta[f] : 0.f;
 #pragma unroll
-  for (int j = 0; j < kQGroup; ++j) {
-    float a = wpart[j], c = bpart[j];
+  for (int i = 0; i < 4; ++i) {
+    const int j = 4 * warp + i;
+    const __nv_bfloat16 bq = __float2bfloat16_rn(acc[i] * gm);
+    float wpart = __bfloat162float(bq), bpart = acc[i] * bt;
+#pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
-      a += __shfl_xor_sync(0xffffffffu, a, o);
-      c += __shfl_xor_sync(0xffffffffu, c, o);
+      wpart += __shfl_xor_sync(0xffffffffu, wpart, o);
+      bpart += __shfl_xor_sync(0xffffffffu, bpart, o);
     }
-    if (lane == 0) {
-      red[0][j][warp] = a;
-      red[1][j][warp] = c;
+    if (j < nb) {
+      uint8_t* qb = qprep + static_cast<size_t>(b0 + j) * qstride;
+      *reinterpret_cast<__nv_bfloat16*>(qb + qop_offset(h, f)) = bq;
+      if (lane == 0) {
+        float* sums = reinterpret_cast<float*>(qb + qprep_lat_bytes(d_c) + qprep_rope_bytes(d_rope));
+        sums[(fc * 2) * 16 + h] = wpart;
+        sums[(fc * 2 + 1) * 16 + h] = bpart;
+      }
     }
   }
-  __syncthreads();
-  if (threadIdx.x < nb) {
-    const int j = threadIdx.x;
-    float a = 0.f, c = 0.f;
-    for (int k = 0; k < (int)(blockDim.x >> 5); ++k) {
-      a += red[0][j][k];
-      c += red[1][j][k];
+  if (fc == 0) {
+    for (int i = tid; i < nb * d_rope; i += kPThreads) {
+      const int j = i / d_rope, r = i % d_rope;
+      *reinterpret_cast<__nv_bfloat16*>(qprep + static_cast<size_t>(b0 + j) * qstride + qprep_lat_bytes(d_c) +
+                                        qop_offset(h, r)) = q[(static_cast<size_t>(b0 + j) * H + h) * qrow + d_nope + r];
     }
-    float* sums = reinterpret_cast<float*>(qprep + static_cast<size_t>(b0 + j) * qstride + qprep_lat_bytes(d_c) +
-                                           qprep_rope_bytes(d_rope));
-    sums[h] = a;
-    sums[16 + h] = c;
   }
 }
 
@@ -214,76 +215,117 @@ __device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float v) { return
 // Block per (sequence b, head h), 256 threads.  The splits that covered b are
 // the CTAs c0..c1 of the page schedule; their partials sit in slots c + b.
 // M = max_s m_s; o = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s (m in log2
-// units); then u = W_UV,h o with two threads per output row.  A sequence of
-// length 0 gets u = 0.
+// units), one thread per latent feature with four independent accumulators
+// over the slots; then u = W_UV,h o with a warp per output row (lanes read
+// 16-byte pieces of the row, a shuffle tree adds them).  A sequence of length
+// 0 gets u = 0.
 constexpr int kCombineThreads = 256;
 constexpr int kMaxSlotsSmem = 512;
+constexpr int kCombineMaxDc = 512;
 
 template <typename T>
 __global__ void __launch_bounds__(kCombineThreads)
 combine_kernel(const int32_t* __restrict__ cu, const float* __restrict__ part_ml, const float* __restrict__ part_o,
                const T* __restrict__ w_uv, T* __restrict__ out, int batch, int H, int d_c, int d_v,
                int num_splits) {
-  extern __shared__ float olat[];  // [d_c]
+  __shared__ __align__(16) float olat[kCombineMaxDc];
   __shared__ float wts[kMaxSlotsSmem];
-  __shared__ float red[32];
+  __shared__ float red[kCombineThreads / 32];
   const int b = blockIdx.x / H, h = blockIdx.x % H;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  constexpr int kWarps = kCombineThreads / 32;
   const int total = cu[batch];
   const int chunk = split_chunk(total, num_splits);
   const int p0 = cu[b], p1 = cu[b + 1];
   const int c0 = p0 / chunk;
   const int n = p1 > p0 ? (p1 - 1) / chunk - c0 + 1 : 0;
   if (n == 0) {
-    for (int f = tid; f < d_c; f += blockDim.x) olat[f] = 0.f;
+    for (int f = tid; f < d_c; f += kCombineThreads) olat[f] = 0.f;
   } else {
-    // running max and denominator over the slots (n <= num_splits)
+    // running maxima and denominators of the slots (n <= num_splits)
     float mloc = -INFINITY;
-    for (int k = tid; k < n; k += blockDim.x) mloc = fmaxf(mloc, part_ml[(static_cast<size_t>(c0 + k + b) * H + h) * 2]);
+    for (int k = tid; k < n; k += kCombineThreads)
+      mloc = fmaxf(mloc, part_ml[(static_cast<size_t>(c0 + k + b) * H + h) * 2]);
+#pragma unroll
     for (int o = 16; o > 0; o >>= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, o));
     if (lane == 0) red[warp] = mloc;
     __syncthreads();
     float M = red[0];
-    for (int k = 1; k < (int)(blockDim.x >> 5); ++k) M = fmaxf(M, red[k]);
+#pragma unroll
+    for (int k = 1; k < kWarps; ++k) M = fmaxf(M, red[k]);
     __syncthreads();
     float lloc = 0.f;
-    for (int k = tid; k < n; k += blockDim.x) {
+    for (int k = tid; k < n; k += kCombineThreads) {
       const float* ml = part_ml + (static_cast<size_t>(c0 + k + b) * H + h) * 2;
       const float wk = exp2f(ml[0] - M);
       if (k < kMaxSlotsSmem) wts[k] = wk;
       lloc = fmaf(wk, ml[1], lloc);
     }
+#pragma unroll
     for (int o = 16; o > 0; o >>= 1) lloc += __shfl_xor_sync(0xffffffffu, lloc, o);
     if (lane == 0) red[warp] = lloc;
     __syncthreads();
     float L = 0.f;
-    for (int k = 0; k < (int)(blockDim.x >> 5); ++k) L += red[k];
+#pragma unroll
+    for (int k = 0; k < kWarps; ++k) L += red[k];
     const float invL = 1.f / L;
-    for (int f = tid; f < d_c; f += blockDim.x) {
-      float acc = 0.f;
-#pragma unroll 8
-      for (int k = 0; k < n; ++k) {
-        const size_t s = static_cast<size_t>(c0 + k + b) * H + h;
-        const float wk = k < kMaxSlotsSmem ? wts[k] : exp2f(part_ml[s * 2] - M);
-        acc = fmaf(wk, part_o[s * d_c + f], acc);
+    const size_t sstride = static_cast<size_t>(H) * d_c;
+    for (int f = tid; f < d_c; f += kCombineThreads) {
+      const float* po = part_o + (static_cast<size_t>(c0 + b) * H + h) * d_c + f;
+      float a[4] = {0.f, 0.f, 0.f, 0.f};
+      int k = 0;
+      for (; k + 4 <= n; k += 4) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float wk = k + i < kMaxSlotsSmem ? wts[k + i] : exp2f(part_ml[((c0 + k + i + b) * H + h) * 2] - M);
+          a[i] = fmaf(wk, po[(k + i) * sstride], a[i]);
+        }
       }
-      olat[f] = acc * invL;
+      for (; k < n; ++k) {
+        const float wk = k < kMaxSlotsSmem ? wts[k] : exp2f(part_ml[((c0 + k + b) * H + h) * 2] - M);
+        a[0] = fmaf(wk, po[k * sstride], a[0]);
+      }
+      olat[f] = ((a[0] + a[1]) + (a[2] + a[3])) * invL;
     }
   }
   __syncthreads();
-  // u[v] = sum_f W_UV[h][v][f] olat[f]: a thread pair per row v, halves of f
+  // u[v] = sum_f W_UV[h][v][f] olat[f]: lane l reads the 16-byte pieces l, l + 32, ... of row v;
+  // a warp takes 8 rows at a time and issues all their loads before the sums
+  constexpr int VEC = 16 / sizeof(T);
+  constexpr int kRows = 8;
   const T* wh = w_uv + static_cast<size_t>(h) * d_v * d_c;
-  const int half = tid & 1;
-  for (int base = 0; base < d_v; base += blockDim.x >> 1) {
-    const int v = base + (tid >> 1);
-    float acc = 0.f;
-    if (v < d_v) {
-      const T* row = wh + static_cast<size_t>(v) * d_c;
-#pragma unroll 8
-      for (int f = half; f < d_c; f += 2) acc = fmaf(to_f<T>(row[f]), olat[f], acc);
+  for (int v0 = warp * kRows; v0 < d_v; v0 += kWarps * kRows) {
+    float acc[kRows];
+#pragma unroll
+    for (int r = 0; r < kRows; ++r) acc[r] = 0.f;
+    for (int f = lane * VEC; f < d_c; f += 32 * VEC) {
+      uint4 raw[kRows];
+#pragma unroll
+      for (int r = 0; r < kRows; ++r)
+        raw[r] = v0 + r < d_v ? *reinterpret_cast<const uint4*>(wh + static_cast<size_t>(v0 + r) * d_c + f)
+                              : make_uint4(0, 0, 0, 0);
+      float o[VEC];
+#pragma unroll
+      for (int i = 0; i < VEC; ++i) o[i] = olat[f + i];
+#pragma unroll
+      for (int r = 0; r < kRows; ++r) {
+        const T* e = reinterpret_cast<const T*>(&raw[r]);
+#pragma unroll
+        for (int i = 0; i < VEC; ++i) acc[r] = fmaf(to_f<T>(e[i]), o[i], acc[r]);
+      }
     }
-    acc += __shfl_xor_sync(0xffffffffu, acc, 1);
-    if (half == 0 && v < d_v) out[(static_cast<size_t>(b) * H + h) * d_v + v] = from_f<T>(acc);
+#pragma unroll
+    for (int r = 0; r < kRows; ++r) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) acc[r] += __shfl_xor_sync(0xffffffffu, acc[r], o);
+    }
+    if (lane < kRows && v0 + lane < d_v) {
+      float mine = acc[0];
+#pragma unroll
+      for (int r = 1; r < kRows; ++r)
+        if (lane == r) mine = acc[r];
+      out[(static_cast<size_t>(b) * H + h) * d_v + v0 + lane] = from_f<T>(mine);
+    }
   }
 }
 
@@ -426,8 +468,8 @@ cudaError_t launch_prologue_tc(const DecodeArgs& a, cudaStream_t st) {
   // with the gate off the latent is used as cached: no LayerNorm affine to fold into q^
   const float* gamma = a.gate ? a.ln_gamma : nullptr;
   const float* beta = a.gate ? a.ln_beta : nullptr;
-  const int ngroups = (a.batch + kQGroup - 1) / kQGroup;
-  prologue_tc_kernel<<<ngroups * 16 + 1, 256, 0, st>>>(
+  const int ngroups = (a.batch + kPBatch - 1) / kPBatch;
+  prologue_tc_kernel<<<16 * (a.d_c / kSumFeatures) * ngroups + 1, 256, 0, st>>>(
       static_cast<const __nv_bfloat16*>(a.q), static_cast<const __nv_bfloat16*>(a.w_uk), gamma, beta,
       a.seq_lens, a.batch, a.d_nope, a.d_rope, a.d_c, a.page_size, ws + wl.off_qprep, wl.qprep_stride,
       reinterpret_cast<int32_t*>(ws + wl.off_cu));
@@ -460,17 +502,16 @@ cudaError_t launch_decode_f32(const DecodeArgs& a, cudaStream_t st) {
 cudaError_t launch_combine(const DecodeArgs& a, bool tc_path, cudaStream_t st) {
   const WorkspaceLayout wl = workspace_layout(a.batch, a.num_splits, a.H, a.d_c, a.d_rope, tc_path);
   uint8_t* ws = static_cast<uint8_t*>(a.workspace);
-  const size_t smem = static_cast<size_t>(a.d_c) * sizeof(float);
   const int32_t* cu = reinterpret_cast<const int32_t*>(ws + wl.off_cu);
   const float* ml = reinterpret_cast<const float*>(ws + wl.off_ml);
   const float* po = reinterpret_cast<const float*>(ws + wl.off_o);
   const int grid = a.batch * a.H;
   if (a.dtype == 0) {
-    combine_kernel<__nv_bfloat16><<<grid, kCombineThreads, smem, st>>>(
+    combine_kernel<__nv_bfloat16><<<grid, kCombineThreads, 0, st>>>(
         cu, ml, po, static_cast<const __nv_bfloat16*>(a.w_uv), static_cast<__nv_bfloat16*>(a.out), a.batch, a.H,
         a.d_c, a.d_v, a.num_splits);
   } else {
-    combine_kernel<float><<<grid, kCombineThreads, smem, st>>>(cu, ml, po, static_cast<const float*>(a.w_uv),
+    combine_kernel<float><<<grid, kCombineThreads, 0, st>>>(cu, ml, po, static_cast<const float*>(a.w_uv),
                                                                 static_cast<float*>(a.out), a.batch, a.H, a.d_c,
                                                                 a.d_v, a.num_splits);
   }

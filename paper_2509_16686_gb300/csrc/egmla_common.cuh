@@ -21,8 +21,10 @@ __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a -
 
 // Per-sequence prepared query block of the tensor-core path: q^ (*) gamma
 // [16 heads x d_c] and q^R [16 x d_rope] as bf16 MMA operands in 8x8 core
-// matrices, then per-head fp32 sums w_h = sum_f (q^ gamma)_hf and
-// b_h = q^_h . beta (16 + 16 floats, 128 bytes).  In every group of 8 columns
+// matrices, then, per chunk of kSumFeatures latent features, the per-head fp32
+// partial sums of w_h = sum_f bf16(q^ gamma)_hf and b_h = q^_h . beta
+// ([d_c / kSumFeatures][2][16] floats; the consumer adds the chunks in order,
+// so the result does not depend on launch order).  In every group of 8 columns
 // (512 bytes) heads 0-7 fill core-matrix row group 0 and heads 8-15 row group
 // 2.  Read as the A operand of an M = 64 MMA (row-group stride 128 B) the two
 // head halves land in TMEM lane quadrants 0 and 1; read as an N = 16 B operand
@@ -36,8 +38,12 @@ __host__ __device__ constexpr size_t qprep_lat_bytes(int d_c) { return static_ca
 __host__ __device__ constexpr size_t qprep_rope_bytes(int d_rope) {
   return static_cast<size_t>(d_rope / 8) * kQGroupBytes;
 }
+constexpr int kSumFeatures = 32;
+__host__ __device__ constexpr size_t qprep_sums_bytes(int d_c) {
+  return static_cast<size_t>(d_c / kSumFeatures) * 2 * 16 * 4;
+}
 __host__ __device__ constexpr size_t qprep_bytes_tc(int d_c, int d_rope) {
-  return qprep_lat_bytes(d_c) + qprep_rope_bytes(d_rope) + 128;
+  return qprep_lat_bytes(d_c) + qprep_rope_bytes(d_rope) + qprep_sums_bytes(d_c);
 }
 
 // fp32 path: q^ [H, d_c] and q^R [H, d_rope] in fp32.

@@ -706,11 +706,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         ++seg;
         if (!warp_wait(smem_u32(&bars.qfull[seg & 1]), (seg >> 1) & 1, abort_flag)) break;
         if (GATE) {
-          // w_h = sum_f bf16(q^ gamma)_hf and b_h = q^_h . beta, after the operands
+          // w_h = sum_f bf16(q^ gamma)_hf and b_h = q^_h . beta from their
+          // per-chunk partials after the operands, added in chunk order
           const float* sums = reinterpret_cast<const float*>(smem + C::OFF_QBUF + (seg & 1) * C::QBUF + C::QB_LAT +
                                                              C::QB_ROPE);
-          wq = sums[hd];
-          bsc = sums[16 + hd] * scale;
+          float wsum = 0.f, bsum = 0.f;
+#pragma unroll
+          for (int c = 0; c < D_C / kSumFeatures; ++c) {
+            wsum += sums[c * 32 + hd];
+            bsum += sums[c * 32 + 16 + hd];
+          }
+          wq = wsum;
+          bsc = bsum * scale;
         }
         warp_arrive(smem_u32(&bars.qempty[seg & 1]));
         l_acc = 0.f;

@@ -65,7 +65,7 @@ struct Cfg {
   static constexpr uint32_t SLOT = KR_OFF + PCHUNK;     // latent + RoPE key of one page
   static constexpr uint32_t QB_LAT = qprep_lat_bytes(D_C);
   static constexpr uint32_t QB_ROPE = qprep_rope_bytes(kRope);
-  static constexpr uint32_t QPREP = QB_LAT + QB_ROPE + 128;
+  static constexpr uint32_t QPREP = qprep_bytes_tc(D_C, kRope);
   static constexpr uint32_t QBUF = (QPREP + 127) / 128 * 128;
   static constexpr uint32_t PBUF = kPage * kHeads * 2;
   // gate rows of a page, gathered by TMA bulk copies: row stride padded by 16 B
