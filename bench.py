@@ -27,6 +27,7 @@ sets the aggregate.
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import math
 import os
@@ -230,6 +231,16 @@ def run_reference(args):
 
 
 # ----------------------------------------------------------------------------- GPU arm
+def kernel_source_sha(files):
+    h = hashlib.sha256()
+    for f in files:
+        path = os.path.join(ROOT, f)
+        if not os.path.exists(path):
+            return None
+        h.update(open(path, "rb").read())
+    return h.hexdigest()[:16]
+
+
 def main():
     args = parse()
     if args.impl == "reference":
@@ -330,8 +341,10 @@ def main():
     traffic = None
     tpath = os.path.join(ROOT, "profiles", "traffic.json")
     if os.path.exists(tpath):
-        tj = json.load(open(tpath)).get(args.workload)
-        if tj:
+        tall = json.load(open(tpath))
+        tj = tall.get(args.workload)
+        # counters taken on other kernel sources no longer describe this kernel
+        if tj and tall.get("source_sha") == kernel_source_sha(tall.get("source_files", [])):
             traffic = tj.get("dram_bytes_per_launch")
 
     # ---- end to end through the C ABI with host buffers
