@@ -16,13 +16,15 @@
 //                     one whole 128-byte line; z = c (*) g rounded to bf16 and
 //                     written back in place, and the LayerNorm statistics
 //                     mu, r = 1/sqrt(var + eps) of z (Eq. 5 over d_c).
-//   MMA (warp 2)      transposed scores S^T = Q Z^T and S_rope^T = Q^R K^R^T
-//                     (M = 64 rows, N = 64 tokens, fp32 in TMEM, double-buffered)
-//                     and the latent output O += P' Z (M = 64 rows, N = d_c
-//                     features, K = 64 tokens), accumulated in TMEM over a
-//                     sequence segment.  The operand rows of heads 0-7 and 8-15
+//   scores (warp 2)   transposed scores S^T = Q Z^T and S_rope^T = Q^R K^R^T on
+//                     tcgen05 (M = 64 rows, N = 64 tokens, fp32 in TMEM,
+//                     double-buffered).  The operand rows of heads 0-7 and 8-15
 //                     are placed so that their accumulator rows fall in TMEM lane
 //                     quadrants 0 and 1.
+//   output (warp 3, with the TMA loads) the latent output O += P' Z (M = 64
+//                     rows, N = d_c features, K = 64 tokens), accumulated in
+//                     TMEM over a sequence segment.  Issued by its own thread, so
+//                     that the scores of later tiles never queue behind it.
 //   softmax (warps 0 and 1, heads 0-7 and 8-15)
 //                     reads its eight head rows of S^T spread over the 32
 //                     threads (one head x 16 tokens each), s = scale * (r (S -
@@ -166,7 +168,8 @@ struct Bars {
   // weights of tile j ready: sp_done[j & 1] (the two softmax warps may be one
   // tile apart, never two: tile j + 2's scores follow tile j's output MMA)
   uint64_t sp_done[2];
-  uint64_t drain;
+  uint64_t sfree[2];           // the softmax warps have read score buffer b
+  uint64_t drain_s, drain_o;   // all MMAs of the score / output issuer done
   uint32_t tmem_base;
   int abort;
 };
@@ -315,7 +318,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(smem_u32(&bars.sp_done[0]), kSoftWarps);
     mbar_init(smem_u32(&bars.sp_done[1]), kSoftWarps);
-    mbar_init(smem_u32(&bars.drain), 1);
+    mbar_init(smem_u32(&bars.sfree[0]), kSoftWarps);
+    mbar_init(smem_u32(&bars.sfree[1]), kSoftWarps);
+    mbar_init(smem_u32(&bars.drain_s), 1);
+    mbar_init(smem_u32(&bars.drain_o), 1);
     bars.abort = 0;
     fence_mbar_init();
   }
@@ -328,43 +334,68 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = bars.tmem_base;
 
+  constexpr uint32_t KSTEP = 2 * kQGroupBytes;   // bytes of 16 columns of an A operand
   if (warp == kTmaWarp) {
-    // ---------------------------------------------------------------- TMA producer
-    // The whole warp walks the tiles; lane 0 waits and issues.  Block-table
-    // entries are fetched 32 at a time (one per lane) so no page lookup sits on
-    // the issue path.
+    // ---------------------------------------------------------------- TMA producer + output MMAs
+    // The whole warp walks the tiles; lane 0 waits and issues the copies.
+    // Before a page slot is reused the output MMA of the tile that held it is
+    // issued here (it is what frees the slot), as soon as that tile's weights
+    // are ready; the remaining ones after the last copy.
     if (lane == 0) {
       prefetch_tensormap(&cmap);
       prefetch_tensormap(&krmap);
     }
     const uint64_t pol_stream = policy_evict_first();
-    Walker w;
+    constexpr uint32_t IDESC_PV = idesc_bf16(64, D_C, 0, 1);
+    // A operand P' in 8x8 core matrices (K groups 512 B apart, row groups
+    // 128 B); B operand: the page slot read MN-major (features along N, tokens
+    // along K)
+    const uint64_t pdesc0 = smem_desc(sbase + C::OFF_PBUF, kQGroupBytes, 128, kSwizzleNone);
+    const uint64_t zdesc_mn = smem_desc(sbase, C::PCHUNK, 1024, kSwizzle128B);
+    Walker w, wo;
     w.start(p.cu, p.seq_lens, p.batch);
+    wo.start(p.cu, p.seq_lens, p.batch);
     PageWindow pw;
-    Tile t;
-    int it = 0, seg = -1;
+    Tile t, to;
+    int it = 0, io = 0;
     int last_it[6] = {-1, -1, -1, -1, -1, -1};
-    int last_qseg[2] = {-1, -1};
+    bool issued_o = false;
     Tracer tr;
     tr.init(p, 0);
     if (lane != 0) tr.base = nullptr;
     bool ok_loop = true;
+    // output MMA of the next tile in order (O += P' Z); false on a timeout
+    auto output = [&]() -> bool {
+      if (!wo.next(to)) return true;
+      if (!warp_wait(smem_u32(&bars.sp_done[io & 1]), (io >> 1) & 1, abort_flag)) return false;
+      tc_fence_after();
+      if (elect_one()) {
+        const int slot = io % C::NS;
+        const uint64_t zb = zdesc_mn + ((slot * C::SLOT) >> 4);
+        const uint64_t pa = pdesc0 + (((io & 1) * C::PBUF) >> 4);
+        if (to.first) {
+#pragma unroll
+          for (int ks = 0; ks < kPage / 16; ++ks)
+            mma_bf16_ss(tmem + C::COL_O, pa + ((ks * KSTEP) >> 4), zb + ((ks * 2048) >> 4), IDESC_PV, ks > 0);
+        } else {
+#pragma unroll
+          for (int ks = 0; ks < kPage / 16; ++ks)
+            mma_bf16_ss(tmem + C::COL_O, pa + ((ks * KSTEP) >> 4), zb + ((ks * 2048) >> 4), IDESC_PV, 1);
+        }
+        mma_commit(smem_u32(&bars.empty[slot]));
+        mma_commit(smem_u32(&bars.pfree[io & 1]));
+      }
+      __syncwarp();
+      issued_o = true;
+      ++io;
+      return true;
+    };
     while (ok_loop && w.next(t)) {
       const int pg = pw.page(p, t, lane);
-      if (t.first) ++seg;
       const int slot = it % C::NS;
+      // the tile that held this slot must have had its output MMA issued
+      if (!DUMP && it >= C::NS && !output()) break;
       if (lane == 0) {
-        if (t.first && !DUMP) {
-          const int qb = seg & 1;
-          if (mbar_wait(smem_u32(&bars.qempty[qb]), ((seg >> 1) & 1) ^ 1, abort_flag)) {
-            mbar_arrive_expect_tx(smem_u32(&bars.qfull[qb]), C::QPREP);
-            bulk_load(sbase + C::OFF_QBUF + qb * C::QBUF, p.qprep + static_cast<size_t>(t.b) * C::QPREP, C::QPREP,
-                      smem_u32(&bars.qfull[qb]));
-            last_qseg[qb] = seg;
-          } else {
-            ok_loop = false;
-          }
-        }
         tr.mark(0, it);
         if (ok_loop && !mbar_wait(smem_u32(&bars.empty[slot]), ((it / C::NS) & 1) ^ 1, abort_flag)) ok_loop = false;
         if (ok_loop) {
@@ -387,51 +418,93 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok_loop = __shfl_sync(0xffffffffu, ok_loop, 0);
       ++it;
     }
+    // the output MMAs of the last tiles
+    if (!DUMP && ok_loop)
+      while (io < it)
+        if (!output()) break;
+    if (!DUMP && issued_o) {
+      // every output MMA must finish before TMEM is released
+      if (elect_one()) mma_commit(smem_u32(&bars.drain_o));
+      __syncwarp();
+      mbar_wait(smem_u32(&bars.drain_o), 0, abort_flag);
+    }
     if (lane == 0) {
       // drain: every copy this thread issued must land before the CTA exits
       for (int s = 0; s < C::NS; ++s)
         if (last_it[s] >= 0) mbar_wait(smem_u32(&bars.full[s]), (last_it[s] / C::NS) & 1, abort_flag);
-      for (int s = 0; s < 2; ++s)
-        if (last_qseg[s] >= 0) mbar_wait(smem_u32(&bars.qfull[s]), (last_qseg[s] >> 1) & 1, abort_flag);
     }
     __syncwarp();
   } else if (warp == kMmaWarp) {
-    // ---------------------------------------------------------------- MMA issuer
-    // Converged warp; one elected lane issues.  Order: scores(i + 1) before
-    // PV(i), so the next tile's scores are ready when the softmax warp finishes
-    // tile i.  All loops are unrolled with compile-time accumulate flags.
+    // ---------------------------------------------------------------- score MMAs
+    // Converged warp; one elected lane issues.  Tile j's scores go out as soon
+    // as its gated page is ready and the softmax warps have read the score
+    // buffer two tiles back.  Loops are unrolled with compile-time accumulate
+    // flags.  This warp also loads the sequences' query blocks (double-
+    // buffered): the next segment's block as soon as its buffer is free (a
+    // non-blocking test after every tile), blocking only at a segment start.
     if (!DUMP) {
       constexpr uint32_t IDESC_S = idesc_bf16(64, kPage, 0, 0);
-      constexpr uint32_t IDESC_PV = idesc_bf16(64, D_C, 0, 1);
       Walker w;
       w.start(p.cu, p.seq_lens, p.batch);
       int seg = -1;
       Tracer tr;
       tr.init(p, 1);
       if (lane != 0) tr.base = nullptr;
-      // A operands: the query block and P' in 8x8 core matrices, K groups 512 B
-      // apart, row groups 128 B apart (heads 0-7 -> rows 0-7, heads 8-15 ->
-      // rows 16-23).  B operands: the page slot, 128-byte swizzled, read K-major
-      // (tokens x features) for the scores and MN-major (features along N,
-      // tokens along K) for the output.
+      // A operand: the query block in 8x8 core matrices, K groups 512 B apart,
+      // row groups 128 B apart (heads 0-7 -> rows 0-7, heads 8-15 -> rows
+      // 16-23).  B operand: the page slot, 128-byte swizzled, read K-major
+      // (tokens x features).
       const uint64_t qdesc0 = smem_desc(sbase + C::OFF_QBUF, kQGroupBytes, 128, kSwizzleNone);
-      const uint64_t pdesc0 = smem_desc(sbase + C::OFF_PBUF, kQGroupBytes, 128, kSwizzleNone);
-      constexpr uint32_t KSTEP = 2 * kQGroupBytes;   // bytes of 16 columns of an A operand
       const uint64_t zdesc_k = smem_desc(sbase, 16, 1024, kSwizzle128B);
-      const uint64_t zdesc_mn = smem_desc(sbase, C::PCHUNK, 1024, kSwizzle128B);
-      Tile cur, nxt;
-      bool have = w.next(cur);
-      bool ok = true;
-      int it = 0;
-      // scores of tile j: S^T = (q^ gamma) Z^T, S_rope^T = q^R K^R^T
-      auto scores = [&](const Tile& t, int j) -> bool {
+      // segment starts ahead of the tile loop: wq sits on the first tile of
+      // segment qn, the next one whose query block is to be loaded
+      Walker wq;
+      wq.start(p.cu, p.seq_lens, p.batch);
+      Tile tq;
+      bool q_more = wq.next(tq);
+      int qn = 0;
+      int last_q[2] = {-1, -1};
+      // 1: issued, 0: buffer still in use (non-blocking call), -1: timed out
+      auto load_query = [&](bool block) -> int {
+        const int qb = qn & 1;
+        if (qn >= 2) {
+          const uint32_t qe = smem_u32(&bars.qempty[qb]);
+          const uint32_t par = ((qn >> 1) & 1) ^ 1;
+          if (block) {
+            if (!warp_wait(qe, par, abort_flag)) return -1;
+          } else if (!__all_sync(0xffffffffu, mbar_test_now(qe, par))) {
+            return 0;
+          }
+        }
+        if (lane == 0) {
+          mbar_arrive_expect_tx(smem_u32(&bars.qfull[qb]), C::QPREP);
+          bulk_load(sbase + C::OFF_QBUF + qb * C::QBUF, p.qprep + static_cast<size_t>(tq.b) * C::QPREP, C::QPREP,
+                    smem_u32(&bars.qfull[qb]));
+        }
+        __syncwarp();
+        last_q[qb] = qn;
+        ++qn;
+        do {
+          q_more = wq.next(tq);
+        } while (q_more && !tq.first);
+        return 1;
+      };
+      Tile t;
+      int j = 0;
+      bool issued = false;
+      bool ok_q = true;
+      while (w.next(t)) {
         if (t.first) {
           ++seg;
-          if (!warp_wait(smem_u32(&bars.qfull[seg & 1]), (seg >> 1) & 1, abort_flag)) return false;
+          while (qn <= seg && (ok_q = load_query(true) > 0)) {
+          }
+          if (!ok_q) break;
+          if (!warp_wait(smem_u32(&bars.qfull[seg & 1]), (seg >> 1) & 1, abort_flag)) break;
         }
         const int slot = j % C::NS;
         tr.mark(0, j);
-        if (!warp_wait(smem_u32(&bars.zready[slot]), (j / C::NS) & 1, abort_flag)) return false;
+        if (!warp_wait(smem_u32(&bars.zready[slot]), (j / C::NS) & 1, abort_flag)) break;
+        if (j >= 2 && !warp_wait(smem_u32(&bars.sfree[j & 1]), ((j >> 1) & 1) ^ 1, abort_flag)) break;
         tr.mark(1, j);
         if (lane == 0) mbar_arrive(smem_u32(&bars.s_ready[j & 1]));
         tc_fence_after();
@@ -451,43 +524,23 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (t.last) mma_commit(smem_u32(&bars.qempty[seg & 1]));
         }
         __syncwarp();
-        return true;
-      };
-      if (have) ok = scores(cur, 0);
-      while (have && ok) {
-        const bool have_next = w.next(nxt);
-        if (have_next && !scores(nxt, it + 1)) break;
-        // latent output of tile it, accumulated in TMEM over the segment: O += P' Z
-        tr.mark(2, it);
-        if (!warp_wait(smem_u32(&bars.sp_done[it & 1]), (it >> 1) & 1, abort_flag)) break;
-        tr.mark(3, it);
-        tc_fence_after();
-        if (elect_one()) {
-          const int slot = it % C::NS;
-          const uint64_t zb = zdesc_mn + ((slot * C::SLOT) >> 4);
-          const uint64_t pa = pdesc0 + (((it & 1) * C::PBUF) >> 4);
-          if (cur.first) {
-#pragma unroll
-            for (int ks = 0; ks < kPage / 16; ++ks)
-              mma_bf16_ss(tmem + C::COL_O, pa + ((ks * KSTEP) >> 4), zb + ((ks * 2048) >> 4), IDESC_PV, ks > 0);
-          } else {
-#pragma unroll
-            for (int ks = 0; ks < kPage / 16; ++ks)
-              mma_bf16_ss(tmem + C::COL_O, pa + ((ks * KSTEP) >> 4), zb + ((ks * 2048) >> 4), IDESC_PV, 1);
-          }
-          mma_commit(smem_u32(&bars.empty[slot]));
-          mma_commit(smem_u32(&bars.pfree[it & 1]));
-        }
-        __syncwarp();
-        cur = nxt;
-        have = have_next;
-        ++it;
+        tr.mark(2, j);
+        issued = true;
+        ++j;
+        if (q_more && qn == seg + 1 && load_query(false) < 0) break;
       }
-      // drain: every MMA issued must finish before TMEM is released (one commit
-      // on a barrier of its own tracks all of them)
-      if (elect_one()) mma_commit(smem_u32(&bars.drain));
+      if (lane == 0) {
+        // drain: the query-block copies this warp issued must land before the CTA exits
+        for (int b = 0; b < 2; ++b)
+          if (last_q[b] >= 0) mbar_wait(smem_u32(&bars.qfull[b]), (last_q[b] >> 1) & 1, abort_flag);
+      }
       __syncwarp();
-      mbar_wait(smem_u32(&bars.drain), 0, abort_flag);
+      if (issued) {
+        // every score MMA must finish before TMEM is released
+        if (elect_one()) mma_commit(smem_u32(&bars.drain_s));
+        __syncwarp();
+        mbar_wait(smem_u32(&bars.drain_s), 0, abort_flag);
+      }
     }
     __syncwarp();
   } else if (warp >= kGateWarp0) {
@@ -726,10 +779,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int slot = it % C::NS;
       const int par = it & 1;
       tr.mark(0, it);
-      // Scores of this tile.  Their completion also implies (same issuing
-      // thread, earlier commit) that the output MMA two tiles back is done, so
-      // the weight buffer of this parity is free; and the MMA warp's release
-      // arrival on the same barrier orders the gate's statistics before it.
+      // Scores of this tile; the score warp's release arrival on the same
+      // barrier orders the gate's statistics before it.
       if (!warp_wait(smem_u32(&bars.s_ready[par]), (it >> 1) & 1, abort_flag)) break;
       tr.mark(1, it);
       tc_fence_after();
@@ -747,6 +798,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       tmem_wait_ld();
+      tc_fence_before();
+      warp_arrive(smem_u32(&bars.sfree[par]));   // score buffer read: tile it + 2 may overwrite it
       tr.mark(7, it);
       // s[2k + e]: token 8k + 2 qq + e of head hd (log2 units)
       float s[16];
@@ -790,9 +843,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       tr.mark(2, it);
       if (__any_sync(0xffffffffu, rescale)) {
         // The previous tile's output MMA must be complete before O is rescaled.
-        // Phase n of pfree[b] completes with output MMA 2n + b; the MMA two
-        // tiles before that is known complete (see above), so this buffer's
-        // phase count is at most one behind and the parity wait is exact.
+        // Phase n of pfree[b] completes with output MMA 2n + b; the wait below
+        // on every tile keeps each buffer's phase count at most one behind, so
+        // the parity wait is exact.
         if (!warp_wait(smem_u32(&bars.pfree[(it - 1) & 1]), ((it - 1) >> 1) & 1, abort_flag)) break;
         tc_fence_after();
 #pragma unroll 1
@@ -811,6 +864,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         l_acc *= alpha;
         bmu_acc *= alpha;
       }
+      // the weight buffer of this parity is free once the output MMA two tiles
+      // back has read it
+      if (!warp_wait(smem_u32(&bars.pfree[par]), ((it >> 1) & 1) ^ 1, abort_flag)) break;
       tr.mark(5, it);
       // The output MMA sees the bf16-rounded weights P'; the denominator and the
       // mean correction use the same rounded values (l = sum P'/r), so the
