@@ -54,6 +54,24 @@ __global__ void append_latent_kernel(uint8_t* __restrict__ c_pool, uint8_t* __re
   if (id_pool != nullptr && ids_new != nullptr && threadIdx.x == 0) id_pool[row] = ids_new[b];
 }
 
+// ------------------------------------------------------------------ helpers
+// eight bf16 (or four fp32) of a 16-byte piece as floats
+__device__ __forceinline__ void unpack16(const uint4& raw, float (&w)[8]) {
+  const __nv_bfloat162* e = reinterpret_cast<const __nv_bfloat162*>(&raw);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 f = __bfloat1622float2(e[i]);
+    w[2 * i] = f.x;
+    w[2 * i + 1] = f.y;
+  }
+}
+__device__ __forceinline__ void unpack16(const uint4& raw, float (&w)[4]) {
+  w[0] = __uint_as_float(raw.x);
+  w[1] = __uint_as_float(raw.y);
+  w[2] = __uint_as_float(raw.z);
+  w[3] = __uint_as_float(raw.w);
+}
+
 // ------------------------------------------------------------------ prologue
 // Exclusive prefix sum of pages per sequence: cu[b] = sum_{b'<b} ceil(L_b'/P),
 // cu[batch] = total; a scan by the block's first warp, 32 sequences per pass.
@@ -77,27 +95,34 @@ __device__ void page_prefix_sums(const int32_t* seq_lens, int batch, int page_si
   if (lane == 0) cu[batch] = carry;
 }
 
-// Tensor-core path: block (head h, chunk of kSumFeatures latent features,
-// group of kPBatch sequences) computes q^_{b,h}[f] = sum_n W_UK,h[n][f] q^C_{b,h}[n]
-// in fp32 (thread: one feature, four sequences) from W_UK and q^C staged in
-// shared memory as bf16 (all 16-byte global loads of a thread are issued
-// before any is stored, so their latencies overlap), and stores (q^ (*) gamma)
-// rounded to bf16 in the prepared query block (qop_offset layout).  Its
-// per-chunk partials of w_h = sum_f bf16(q^ gamma)_f and b_h = q^_h . beta go to
-// the block's slots of the sums area.  Chunk-0 blocks also copy q^R.  The last
-// block computes the page prefix sums.
+// Tensor-core path: block (head h, chunk of kSumFeatures = 32 latent features,
+// group of up to kPBatch sequences) computes q^_{b,h}[f] = sum_n W_UK,h[n][f] q^C_{b,h}[n]
+// in fp32 and stores (q^ (*) gamma) rounded to bf16 in the prepared query
+// block (qop_offset layout).  Its per-chunk partials of w_h = sum_f bf16(q^ gamma)_f
+// and b_h = q^_h . beta go to the block's slots of the sums area.  Chunk-0
+// blocks also copy q^R.  The last block computes the page prefix sums.
+//  - All 16-byte global loads of a thread are issued before any is stored
+//    (W_UK with an L2 evict-last hint: it stays in L2 across steps).
+//  - W_UK and q^C are staged row-major; a warp takes a quad of sequences and
+//    a part of the n range, reading per 8 n the lane's feature of 8 W rows
+//    and 8 n of each q^C row (one 16-byte broadcast per sequence) for 32
+//    FMAs.  With few sequences the spare warps split n further; the parts
+//    are added in shared memory.
 constexpr int kPBatch = 32;
 constexpr int kPMaxNope = 256;
 constexpr int kPThreads = 256;
 constexpr int kPLoads = kPMaxNope * kSumFeatures * 2 / 16 / kPThreads;   // 16-byte pieces per thread and array
 
-__global__ void __launch_bounds__(kPThreads)
-    prologue_tc_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ w_uk,
+// (no launch bound: with one, ptxas trims the kernel to 48 registers and spills)
+__global__ void prologue_tc_kernel(const __nv_bfloat16* __restrict__ q, const __nv_bfloat16* __restrict__ w_uk,
                        const float* __restrict__ gamma, const float* __restrict__ beta,
                        const int32_t* __restrict__ seq_lens, int batch, int d_nope, int d_rope, int d_c,
                        int page_size, uint8_t* __restrict__ qprep, size_t qstride, int32_t* __restrict__ cu) {
-  __shared__ __align__(16) __nv_bfloat16 ws[kPMaxNope][kSumFeatures];   // W_UK,h[n][f0 + f]
-  __shared__ __align__(16) __nv_bfloat16 qs[kPBatch][kPMaxNope];       // q^C_{b0 + j, h}[n]
+  __shared__ __align__(16) __nv_bfloat16 ws[kPMaxNope][kSumFeatures];  // W_UK,h[n][f0 + f]
+  __shared__ __align__(16) __nv_bfloat16 qs[kPBatch][kPMaxNope];      // q^C_{b0 + j, h}[n]
+  // partial sums [n part * 4 quads + j][f], written once every warp is done with ws
+  float (*red)[kSumFeatures] = reinterpret_cast<float (*)[kSumFeatures]>(&ws[0][0]);
+  static_assert(sizeof(ws) >= 32 * kSumFeatures * sizeof(float), "reduction buffer aliases ws");
   constexpr int H = 16;
   const int nchunk = d_c / kSumFeatures;
   const int ngroups = (batch + kPBatch - 1) / kPBatch;
@@ -109,10 +134,11 @@ __global__ void __launch_bounds__(kPThreads)
   const int h = blockIdx.x % H, fc = (blockIdx.x / H) % nchunk, bg = blockIdx.x / (H * nchunk);
   const int b0 = bg * kPBatch, nb = min(kPBatch, batch - b0);
   const int f0 = fc * kSumFeatures;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;   // feature f0 + lane; sequences b0 + 4 warp + i
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int qrow = d_nope + d_rope;
   // W piece i: row n = i / 4, features 8 (i % 4) ..; q piece i: sequence j = i / (d_nope / 8), columns 8 (i % ..)
   const int wpieces = d_nope * (kSumFeatures / 8), qpr = d_nope / 8, qpieces = kPBatch * qpr;
+  const uint64_t keep = policy_evict_last();
   uint4 wv[kPLoads], qv[kPLoads];
 #pragma unroll
   for (int k = 0; k < kPLoads; ++k) {
@@ -120,7 +146,7 @@ __global__ void __launch_bounds__(kPThreads)
     wv[k] = make_uint4(0, 0, 0, 0);
     qv[k] = make_uint4(0, 0, 0, 0);
     if (i < wpieces)
-      wv[k] = *reinterpret_cast<const uint4*>(w_uk + (static_cast<size_t>(h) * d_nope + i / 4) * d_c + f0 + 8 * (i % 4));
+      wv[k] = ldg_16_na_hint(w_uk + (static_cast<size_t>(h) * d_nope + i / 4) * d_c + f0 + 8 * (i % 4), keep);
     if (i < qpieces && i / qpr < nb)
       qv[k] = *reinterpret_cast<const uint4*>(q + (static_cast<size_t>(b0 + i / qpr) * H + h) * qrow + 8 * (i % qpr));
   }
@@ -131,34 +157,65 @@ __global__ void __launch_bounds__(kPThreads)
     if (i < qpieces) *reinterpret_cast<uint4*>(&qs[i / qpr][8 * (i % qpr)]) = qv[k];
   }
   __syncthreads();
+  // warp -> (sequence quad sq, n part kp); nq quads, ks parts of the n range
+  const int nq = (nb + 3) / 4, nblk = d_nope / 8;
+  int ks = 8 / nq;
+  ks = ks >= 8 ? 8 : ks >= 4 ? 4 : ks >= 2 ? 2 : 1;
+  while (nblk % ks) ks >>= 1;
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll 8
-  for (int n = 0; n < d_nope; ++n) {
-    const float w = __bfloat162float(ws[n][lane]);
+  const int sq = warp % nq, kp = warp / nq, bpk = nblk / ks;
+  if (warp < nq * ks) {
+    for (int blk = kp * bpk; blk < (kp + 1) * bpk; ++blk) {
+      float w[8];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) acc[i] = fmaf(w, __bfloat162float(qs[4 * warp + i][n]), acc[i]);
+      for (int e = 0; e < 8; ++e) w[e] = __bfloat162float(ws[blk * 8 + e][lane]);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        float x[8];
+        unpack16(*reinterpret_cast<const uint4*>(&qs[4 * sq + i][blk * 8]), x);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[i] = fmaf(w[e], x[e], acc[i]);
+      }
+    }
   }
   const int f = f0 + lane;
   const float gm = gamma ? gamma[f] : 1.f;
   const float bt = beta ? beta[f] : 0.f;
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int j = 4 * warp + i;
-    const __nv_bfloat16 bq = __float2bfloat16_rn(acc[i] * gm);
-    float wpart = __bfloat162float(bq), bpart = acc[i] * bt;
+  // q^ of sequence j (its 32 features over the warp's lanes) -> prepared query block
+  auto emit = [&](int j, float a) {
+    const __nv_bfloat16 bq = __float2bfloat16_rn(a * gm);
+    float wpart = __bfloat162float(bq), bpart = a * bt;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       wpart += __shfl_xor_sync(0xffffffffu, wpart, o);
       bpart += __shfl_xor_sync(0xffffffffu, bpart, o);
     }
-    if (j < nb) {
-      uint8_t* qb = qprep + static_cast<size_t>(b0 + j) * qstride;
-      *reinterpret_cast<__nv_bfloat16*>(qb + qop_offset(h, f)) = bq;
-      if (lane == 0) {
-        float* sums = reinterpret_cast<float*>(qb + qprep_lat_bytes(d_c) + qprep_rope_bytes(d_rope));
-        sums[(fc * 2) * 16 + h] = wpart;
-        sums[(fc * 2 + 1) * 16 + h] = bpart;
-      }
+    uint8_t* qb = qprep + static_cast<size_t>(b0 + j) * qstride;
+    *reinterpret_cast<__nv_bfloat16*>(qb + qop_offset(h, f)) = bq;
+    if (lane == 0) {
+      float* sums = reinterpret_cast<float*>(qb + qprep_lat_bytes(d_c) + qprep_rope_bytes(d_rope));
+      sums[(fc * 2) * 16 + h] = wpart;
+      sums[(fc * 2 + 1) * 16 + h] = bpart;
+    }
+  };
+  if (ks == 1) {
+    // each warp holds whole sums: emit from registers
+    if (warp < nq) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (4 * sq + i < nb) emit(4 * sq + i, acc[i]);
+    }
+  } else {
+    __syncthreads();   // every warp is done with ws, which red aliases
+    if (warp < nq * ks) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) red[kp * 4 * nq + 4 * sq + i][lane] = acc[i];
+    }
+    __syncthreads();
+    for (int j = warp; j < nb; j += kPThreads / 32) {
+      float a = 0.f;
+      for (int k = 0; k < ks; ++k) a += red[k * 4 * nq + j][lane];
+      emit(j, a);
     }
   }
   if (fc == 0) {
@@ -196,9 +253,6 @@ __global__ void prologue_f32_kernel(const float* __restrict__ q, const float* __
 }
 
 // ------------------------------------------------------------------ combine
-// Block (h, group of 8 sequences).  For each sequence: M = max_s m_s,
-// o = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s (m in log2 units), then
-// u = W_UV,h o.  Sequences of length 0 get u = 0.
 template <typename T>
 __device__ __forceinline__ float to_f(T v);
 template <>
@@ -215,15 +269,25 @@ __device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float v) { return
 // Block per (sequence b, head h), 256 threads.  The splits that covered b are
 // the CTAs c0..c1 of the page schedule; their partials sit in slots c + b.
 // M = max_s m_s; o = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s (m in log2
-// units), one thread per latent feature with four independent accumulators
-// over the slots; then u = W_UV,h o with a warp per output row (lanes read
-// 16-byte pieces of the row, a shuffle tree adds them).  A sequence of length
-// 0 gets u = 0.
+// units); then u = W_UV,h o.  A sequence of length 0 gets u = 0.  The kernel
+// is a chain of dependent loads, so it is laid out to keep that chain short:
+//  - thread k keeps the (m, l) of slot k that it loaded for the maximum and
+//    forms its weight 2^(m - M) from registers;
+//  - a thread per latent feature loads O of up to kCombineBurst slots into
+//    registers before it adds any of them (one round trip for that many
+//    splits);
+//  - a warp loads all kCombineRows of its W_UV,h rows (16-byte pieces, lane l
+//    the pieces l, l + 32, ..) before the sums, and a shuffle tree adds the
+//    lanes' parts of each row.
+// Two instantiations: <16, 24> (about 110 registers) for grids of up to about
+// two blocks per SM, where each block's latency is the step's; <8, 8> (about
+// half the registers, more resident blocks) for larger grids, where
+// occupancy hides the latency.
 constexpr int kCombineThreads = 256;
 constexpr int kMaxSlotsSmem = 512;
 constexpr int kCombineMaxDc = 512;
 
-template <typename T>
+template <typename T, int kCombineRows, int kCombineBurst>
 __global__ void __launch_bounds__(kCombineThreads)
 combine_kernel(const int32_t* __restrict__ cu, const float* __restrict__ part_ml, const float* __restrict__ part_o,
                const T* __restrict__ w_uv, T* __restrict__ out, int batch, int H, int d_c, int d_v,
@@ -242,10 +306,14 @@ combine_kernel(const int32_t* __restrict__ cu, const float* __restrict__ part_ml
   if (n == 0) {
     for (int f = tid; f < d_c; f += kCombineThreads) olat[f] = 0.f;
   } else {
-    // running maxima and denominators of the slots (n <= num_splits)
-    float mloc = -INFINITY;
-    for (int k = tid; k < n; k += kCombineThreads)
-      mloc = fmaxf(mloc, part_ml[(static_cast<size_t>(c0 + k + b) * H + h) * 2]);
+    const float* pml = part_ml + (static_cast<size_t>(c0 + b) * H + h) * 2;
+    const size_t mlstride = static_cast<size_t>(H) * 2;
+    // running maxima and denominators of the slots (n <= num_splits); thread
+    // tid keeps slot tid's pair
+    float2 mine = make_float2(-INFINITY, 0.f);
+    if (tid < n) mine = *reinterpret_cast<const float2*>(pml + tid * mlstride);
+    float mloc = mine.x;
+    for (int k = tid + kCombineThreads; k < n; k += kCombineThreads) mloc = fmaxf(mloc, pml[k * mlstride]);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, o));
     if (lane == 0) red[warp] = mloc;
@@ -255,11 +323,15 @@ combine_kernel(const int32_t* __restrict__ cu, const float* __restrict__ part_ml
     for (int k = 1; k < kWarps; ++k) M = fmaxf(M, red[k]);
     __syncthreads();
     float lloc = 0.f;
-    for (int k = tid; k < n; k += kCombineThreads) {
-      const float* ml = part_ml + (static_cast<size_t>(c0 + k + b) * H + h) * 2;
-      const float wk = exp2f(ml[0] - M);
+    if (tid < n) {
+      const float wk = exp2f(mine.x - M);
+      if (tid < kMaxSlotsSmem) wts[tid] = wk;
+      lloc = wk * mine.y;
+    }
+    for (int k = tid + kCombineThreads; k < n; k += kCombineThreads) {
+      const float wk = exp2f(pml[k * mlstride] - M);
       if (k < kMaxSlotsSmem) wts[k] = wk;
-      lloc = fmaf(wk, ml[1], lloc);
+      lloc = fmaf(wk, pml[k * mlstride + 1], lloc);
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) lloc += __shfl_xor_sync(0xffffffffu, lloc, o);
@@ -272,57 +344,60 @@ combine_kernel(const int32_t* __restrict__ cu, const float* __restrict__ part_ml
     const size_t sstride = static_cast<size_t>(H) * d_c;
     for (int f = tid; f < d_c; f += kCombineThreads) {
       const float* po = part_o + (static_cast<size_t>(c0 + b) * H + h) * d_c + f;
-      float a[4] = {0.f, 0.f, 0.f, 0.f};
-      int k = 0;
-      for (; k + 4 <= n; k += 4) {
+      float a0 = 0.f, a1 = 0.f;
+      for (int k0 = 0; k0 < n; k0 += kCombineBurst) {
+        float v[kCombineBurst];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const float wk = k + i < kMaxSlotsSmem ? wts[k + i] : exp2f(part_ml[((c0 + k + i + b) * H + h) * 2] - M);
-          a[i] = fmaf(wk, po[(k + i) * sstride], a[i]);
+        for (int i = 0; i < kCombineBurst; ++i) v[i] = k0 + i < n ? po[(k0 + i) * sstride] : 0.f;
+#pragma unroll
+        for (int i = 0; i < kCombineBurst; i += 2) {
+          const int k = k0 + i;
+          if (k < n) a0 = fmaf(k < kMaxSlotsSmem ? wts[k] : exp2f(pml[k * mlstride] - M), v[i], a0);
+          if (k + 1 < n) a1 = fmaf(k + 1 < kMaxSlotsSmem ? wts[k + 1] : exp2f(pml[(k + 1) * mlstride] - M), v[i + 1], a1);
         }
       }
-      for (; k < n; ++k) {
-        const float wk = k < kMaxSlotsSmem ? wts[k] : exp2f(part_ml[((c0 + k + b) * H + h) * 2] - M);
-        a[0] = fmaf(wk, po[k * sstride], a[0]);
-      }
-      olat[f] = ((a[0] + a[1]) + (a[2] + a[3])) * invL;
+      olat[f] = (a0 + a1) * invL;
     }
   }
   __syncthreads();
-  // u[v] = sum_f W_UV[h][v][f] olat[f]: lane l reads the 16-byte pieces l, l + 32, ... of row v;
-  // a warp takes 8 rows at a time and issues all their loads before the sums
+  // u[v] = sum_f W_UV[h][v][f] olat[f]
   constexpr int VEC = 16 / sizeof(T);
-  constexpr int kRows = 8;
   const T* wh = w_uv + static_cast<size_t>(h) * d_v * d_c;
-  for (int v0 = warp * kRows; v0 < d_v; v0 += kWarps * kRows) {
-    float acc[kRows];
+  for (int v0 = warp * kCombineRows; v0 < d_v; v0 += kWarps * kCombineRows) {
+    float acc[kCombineRows];
 #pragma unroll
-    for (int r = 0; r < kRows; ++r) acc[r] = 0.f;
+    for (int r = 0; r < kCombineRows; ++r) acc[r] = 0.f;
     for (int f = lane * VEC; f < d_c; f += 32 * VEC) {
-      uint4 raw[kRows];
+      uint4 raw[kCombineRows];
 #pragma unroll
-      for (int r = 0; r < kRows; ++r)
+      for (int r = 0; r < kCombineRows; ++r)
         raw[r] = v0 + r < d_v ? *reinterpret_cast<const uint4*>(wh + static_cast<size_t>(v0 + r) * d_c + f)
                               : make_uint4(0, 0, 0, 0);
       float o[VEC];
 #pragma unroll
-      for (int i = 0; i < VEC; ++i) o[i] = olat[f + i];
+      for (int i = 0; i < VEC; i += 4) {
+        const float4 q = *reinterpret_cast<const float4*>(olat + f + i);
+        o[i] = q.x;
+        o[i + 1] = q.y;
+        o[i + 2] = q.z;
+        o[i + 3] = q.w;
+      }
 #pragma unroll
-      for (int r = 0; r < kRows; ++r) {
+      for (int r = 0; r < kCombineRows; ++r) {
         const T* e = reinterpret_cast<const T*>(&raw[r]);
 #pragma unroll
         for (int i = 0; i < VEC; ++i) acc[r] = fmaf(to_f<T>(e[i]), o[i], acc[r]);
       }
     }
 #pragma unroll
-    for (int r = 0; r < kRows; ++r) {
+    for (int r = 0; r < kCombineRows; ++r) {
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) acc[r] += __shfl_xor_sync(0xffffffffu, acc[r], o);
     }
-    if (lane < kRows && v0 + lane < d_v) {
+    if (lane < kCombineRows && v0 + lane < d_v) {
       float mine = acc[0];
 #pragma unroll
-      for (int r = 1; r < kRows; ++r)
+      for (int r = 1; r < kCombineRows; ++r)
         if (lane == r) mine = acc[r];
       out[(static_cast<size_t>(b) * H + h) * d_v + v0 + lane] = from_f<T>(mine);
     }
@@ -499,22 +574,43 @@ cudaError_t launch_decode_f32(const DecodeArgs& a, cudaStream_t st) {
   return cudaGetLastError();
 }
 
+namespace {
+int device_sms() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+  if (cached[dev] == 0) {
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) sms = 1;
+    cached[dev] = sms;
+  }
+  return cached[dev];
+}
+
+template <typename T>
+void launch_combine_t(const DecodeArgs& a, const int32_t* cu, const float* ml, const float* po, cudaStream_t st) {
+  const int grid = a.batch * a.H;
+  const T* w = static_cast<const T*>(a.w_uv);
+  T* out = static_cast<T*>(a.out);
+  if (grid <= 2 * device_sms())
+    combine_kernel<T, 16, 24><<<grid, kCombineThreads, 0, st>>>(cu, ml, po, w, out, a.batch, a.H, a.d_c, a.d_v,
+                                                                a.num_splits);
+  else
+    combine_kernel<T, 8, 8><<<grid, kCombineThreads, 0, st>>>(cu, ml, po, w, out, a.batch, a.H, a.d_c, a.d_v,
+                                                              a.num_splits);
+}
+}  // namespace
+
 cudaError_t launch_combine(const DecodeArgs& a, bool tc_path, cudaStream_t st) {
   const WorkspaceLayout wl = workspace_layout(a.batch, a.num_splits, a.H, a.d_c, a.d_rope, tc_path);
   uint8_t* ws = static_cast<uint8_t*>(a.workspace);
   const int32_t* cu = reinterpret_cast<const int32_t*>(ws + wl.off_cu);
   const float* ml = reinterpret_cast<const float*>(ws + wl.off_ml);
   const float* po = reinterpret_cast<const float*>(ws + wl.off_o);
-  const int grid = a.batch * a.H;
-  if (a.dtype == 0) {
-    combine_kernel<__nv_bfloat16><<<grid, kCombineThreads, 0, st>>>(
-        cu, ml, po, static_cast<const __nv_bfloat16*>(a.w_uv), static_cast<__nv_bfloat16*>(a.out), a.batch, a.H,
-        a.d_c, a.d_v, a.num_splits);
-  } else {
-    combine_kernel<float><<<grid, kCombineThreads, 0, st>>>(cu, ml, po, static_cast<const float*>(a.w_uv),
-                                                                static_cast<float*>(a.out), a.batch, a.H, a.d_c,
-                                                                a.d_v, a.num_splits);
-  }
+  if (a.dtype == 0)
+    launch_combine_t<__nv_bfloat16>(a, cu, ml, po, st);
+  else
+    launch_combine_t<float>(a, cu, ml, po, st);
   return cudaGetLastError();
 }
 
