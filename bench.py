@@ -13,10 +13,12 @@ value: decode tokens/s (new tokens produced per second, all GPUs) with every
 input resident in HBM; the step is replayed from a CUDA graph over three
 rotating cache replicas (3 x 168 MB > L2), so the latent stream comes from HBM.
 e2e: the same metric through the C ABI from pinned HOST buffers, the per-step
-inputs copied in and the output copied back inside the timed region.
+inputs (packed in one buffer) copied in and the output copied back inside the
+timed region, calls issued eagerly from Python.
 roofline: the decode kernel's latent-cache bytes per launch divided by its own
-CUDA-event duration (a second pass of the same steps with per-launch events on
-the launching stream), against the measured HBM copy bandwidth.
+CUDA-event duration (events recorded around every decode launch inside a
+captured graph of the same steps, on the launching stream), against the
+measured HBM copy bandwidth.
 cpu_baseline / --impl reference: the fp64 oracle on the host cores on a bounded
 sample of the same workload, scaled to decode tokens/s.
 
@@ -264,11 +266,13 @@ def main():
     for _ in range(REPLICAS - 1):
         r = device.upload(case, num_splits=args.splits)
         dcs.append(r)
-    # all replicas share the weights, queries and outputs of the first
+    # all replicas share the weights, block table and workspace of the first;
+    # each keeps its own per-step inputs, packed in one device buffer (one
+    # host-to-device copy per end-to-end step), and its own output
     for r in dcs[1:]:
-        for name in ("q", "gate_table", "ln_gamma", "ln_beta", "w_uk", "w_uv", "out", "workspace", "status",
-                     "block_table", "seq_lens", "positions", "c_new", "kr_new", "ids_new"):
+        for name in ("gate_table", "ln_gamma", "ln_beta", "w_uk", "w_uv", "workspace", "status", "block_table"):
             setattr(r, name, getattr(dcs[0], name))
+    packed = [device.pack_step_inputs(r) for r in dcs]
     stream = torch.cuda.Stream()
     tokens_cached = int(case.seq_lens.astype(np.int64).sum())
     elem = 2 if d.dtype == "bf16" else 4
@@ -318,17 +322,21 @@ def main():
     ms_per_step = elapsed_ms / steps
     value = ws * B * steps / (elapsed_ms / 1e3)
 
-    # ---- the decode kernel alone: per-launch events on the launching stream
-    prof_steps = min(steps, 200)
+    # ---- the decode kernel alone: CUDA events around every decode launch,
+    # recorded as nodes of a captured graph of the same steps (so that each
+    # launch is timed as it runs in the step, without host launch gaps); the
+    # graph is replayed twice and the events hold the second replay
+    prof_steps = 10 * REPLICAS
     _lib.eg_mla_profile_begin(prof_steps)
-    torch.cuda.synchronize()
-    with torch.cuda.stream(stream):
-        # a spin kernel keeps the GPU busy while the host queues the steps, so the
-        # events bracket kernel execution rather than host launch gaps
-        torch.cuda._sleep(int(150e6))
+    pgraph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(pgraph, stream=stream):
         for i in range(prof_steps):
             dcs[i % REPLICAS].step(stream)
+    with torch.cuda.stream(stream):
+        pgraph.replay()
+        pgraph.replay()
     stream.synchronize()
+    del pgraph
     ms_sum, n_l = _lib.eg_mla_profile_end()
     k_ms = ms_sum / max(1, n_l)
     achieved = cache_bytes / (k_ms * 1e-3) / 1e9
@@ -347,24 +355,45 @@ def main():
         if tj and tall.get("source_sha") == kernel_source_sha(tall.get("source_files", [])):
             traffic = tj.get("dram_bytes_per_launch")
 
-    # ---- end to end through the C ABI with host buffers
+    # ---- end to end through the C ABI with host buffers.  Step i uses replica
+    # i % REPLICAS and runs on the compute stream (its two C calls bound once,
+    # see _lib.bind_step); a copy stream carries the input copy of step i + 1
+    # (issued first, so it overlaps step i) and the read-back of step i's
+    # output.  Events order each replica's buffers between uses.
     e2e_steps = args.e2e_steps or min(steps, 2000)
-    h_in = {k: getattr(dcs[0], k).cpu().pin_memory() for k in ("q", "c_new", "kr_new", "ids_new", "positions",
-                                                             "seq_lens")}
-    h_out = torch.empty(dcs[0].out.shape, dtype=dcs[0].out.dtype).pin_memory()
-    h2d = sum(t.numel() * t.element_size() for t in h_in.values())
-    d2h = h_out.numel() * h_out.element_size()
+    h_outs = [torch.empty(r.out.shape, dtype=r.out.dtype).pin_memory() for r in dcs]
+    h2d = packed[0][0].numel() * packed[0][0].element_size()
+    d2h = h_outs[0].numel() * h_outs[0].element_size()
+    steps_bound = [r.bind(stream) for r in dcs]
+    s_copy = torch.cuda.Stream()
+    ev_in = [torch.cuda.Event() for _ in dcs]
+    ev_comp = [torch.cuda.Event() for _ in dcs]
+    ev_out = [torch.cuda.Event() for _ in dcs]
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
-    with torch.cuda.stream(stream):
-        e0.record(stream)
+    e0.record(stream)
+    s_copy.wait_stream(stream)
+    with torch.cuda.stream(s_copy):
+        packed[0][1].copy_(packed[0][0], non_blocking=True)
+        ev_in[0].record(s_copy)
         for i in range(e2e_steps):
-            r = dcs[i % REPLICAS]
-            for k, t in h_in.items():
-                getattr(r, k).copy_(t, non_blocking=True)
-            r.step(stream)
-            h_out.copy_(r.out, non_blocking=True)
-        e1.record(stream)
+            k = i % REPLICAS
+            stream.wait_event(ev_in[k])
+            if i >= REPLICAS:
+                stream.wait_event(ev_out[k])      # step i - REPLICAS's output has been read back
+            steps_bound[k]()
+            ev_comp[k].record(stream)
+            if i + 1 < e2e_steps:
+                k1 = (i + 1) % REPLICAS
+                if i + 1 >= REPLICAS:
+                    s_copy.wait_event(ev_comp[k1])   # step i + 1 - REPLICAS has read these inputs
+                packed[k1][1].copy_(packed[k1][0], non_blocking=True)
+                ev_in[k1].record(s_copy)
+            s_copy.wait_event(ev_comp[k])
+            h_outs[k].copy_(dcs[k].out, non_blocking=True)
+            ev_out[k].record(s_copy)
+    stream.wait_stream(s_copy)
+    e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1)
     if dist:

@@ -255,8 +255,10 @@ int eg_mla_debug_gather(const eg_mla_dims* dims, const void* c_pool, const void*
  * eg_mla_decode call records a CUDA event pair around that kernel's launch on
  * its stream, for at most max_launches launches.  end synchronises on the
  * events, returns the summed kernel time in milliseconds and the number of
- * launches timed, releases the events and stops recording.  Host-side event
- * objects only; not for use while a stream is being captured into a graph.
+ * launches timed, releases the events and stops recording.  During stream
+ * capture the pair becomes event-record nodes of the graph
+ * (cudaEventRecordExternal): replay the graph, synchronise, then call end,
+ * which reads the last replay's timestamps.
  * Returns EG_MLA_ERR_CUDA if event creation fails, EG_MLA_ERR_INVALID_ARG for
  * max_launches <= 0 or null outputs.
  */

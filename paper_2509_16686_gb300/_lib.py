@@ -206,6 +206,39 @@ def eg_mla_decode_static(dims: EgMlaDims, q, c_pool, krope_pool, id_pool, block_
     _check(code, "eg_mla_decode_static")
 
 
+def bind_step(dims: EgMlaDims, c_pool, krope_pool, id_pool, c_new, krope_new, ids_new, positions, q, block_table,
+              seq_lens, max_seq_len, gate_table, ln_gamma, ln_beta, w_uk, w_uv, out, workspace, num_splits=0,
+              dev_status=None, stream=None):
+    """One decode step (eg_mla_append_latent, then eg_mla_decode) with every
+    argument converted once: returns a callable that issues both C calls on
+    `stream` with those pointers.  The tensors must stay alive and in place
+    while the callable is used; a caller that reruns the same step every token
+    saves the per-call argument marshalling."""
+    lib = load()
+    d = ctypes.byref(dims)
+    st = _stream(stream)
+    append_args = (d, _ptr(c_pool), _ptr(krope_pool), _ptr(id_pool), _ptr(c_new), _ptr(krope_new), _ptr(ids_new),
+                   _ptr(block_table), block_table.shape[1], _ptr(positions), positions.shape[0], c_pool.shape[0],
+                   _ptr(dev_status), st)
+    decode_args = (d, _ptr(q), _ptr(c_pool), _ptr(krope_pool), _ptr(id_pool), _ptr(block_table),
+                   block_table.shape[1], _ptr(seq_lens), int(max_seq_len), seq_lens.shape[0], c_pool.shape[0],
+                   _ptr(gate_table), _ptr(ln_gamma), _ptr(ln_beta), _ptr(w_uk), _ptr(w_uv), _ptr(out), num_splits,
+                   _ptr(workspace), workspace.numel() * workspace.element_size(), _ptr(dev_status), st)
+    append_fn, decode_fn = lib.eg_mla_append_latent, lib.eg_mla_decode
+
+    def step() -> None:
+        rc = append_fn(*append_args)
+        if rc != EG_MLA_OK:
+            raise EgMlaError(rc, "eg_mla_append_latent")
+        rc = decode_fn(*decode_args)
+        if rc != EG_MLA_OK:
+            raise EgMlaError(rc, "eg_mla_decode")
+
+    step.keepalive = (dims, c_pool, krope_pool, id_pool, c_new, krope_new, ids_new, positions, q, block_table,
+                      seq_lens, gate_table, ln_gamma, ln_beta, w_uk, w_uv, out, workspace, dev_status)
+    return step
+
+
 def eg_mla_debug_gather(dims: EgMlaDims, c_pool, krope_pool, id_pool, block_table, seq_lens, max_seq_len,
                         gate_table, c_out, kr_out, ids_out, g_out, workspace, num_splits=0,
                         dev_status=None, stream=None) -> None:

@@ -199,14 +199,24 @@ void apply_trace(DecodeArgs& a) {
   a.trace_cap = g_trace.cap;
 }
 
+// Records a profiling event on the launching stream; under stream capture it
+// becomes an event-record node of the graph (timestamped at each replay).
+void prof_record(cudaEvent_t e, cudaStream_t st) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(st, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusActive)
+    cudaEventRecordWithFlags(e, st, cudaEventRecordExternal);
+  else
+    cudaEventRecord(e, st);
+}
+
 void prof_mark(cudaStream_t st, bool before) {
   std::lock_guard<std::mutex> lk(g_prof.mu);
   if (!g_prof.active) return;
   const int pairs = static_cast<int>(g_prof.ev.size() / 2);
   if (before) {
-    if (g_prof.used < pairs) cudaEventRecord(g_prof.ev[2 * g_prof.used], st);
+    if (g_prof.used < pairs) prof_record(g_prof.ev[2 * g_prof.used], st);
   } else if (g_prof.used < pairs) {
-    cudaEventRecord(g_prof.ev[2 * g_prof.used + 1], st);
+    prof_record(g_prof.ev[2 * g_prof.used + 1], st);
     ++g_prof.used;
   }
 }

@@ -74,6 +74,13 @@ class DeviceCase:
         self.append(stream)
         return self.decode(stream)
 
+    def bind(self, stream=None):
+        """step() with its C-ABI arguments converted once (see _lib.bind_step)."""
+        return _lib.bind_step(self.dims, self.c_pool, self.kr_pool, self.id_pool, self.c_new, self.kr_new,
+                              self.ids_new, self.positions, self.q, self.block_table, self.seq_lens,
+                              self.max_seq_len, self.gate_table, self.ln_gamma, self.ln_beta, self.w_uk, self.w_uv,
+                              self.out, self.workspace, self.num_splits, self.status, stream)
+
     def read_status(self) -> int:
         return int(self.status.item())
 
@@ -114,6 +121,32 @@ def upload(case: Case, device="cuda", num_splits: int = 0) -> DeviceCase:
         max_seq_len=int(case.seq_lens.max()) if B else 0,
         num_splits=num_splits,
     )
+
+
+# inputs that change from one decode step to the next
+STEP_INPUTS = ("q", "c_new", "kr_new", "ids_new", "positions", "seq_lens")
+
+
+def pack_step_inputs(dc: DeviceCase, names=STEP_INPUTS):
+    """Move the per-step inputs of `dc` into one device buffer (each a view at a
+    256-byte aligned offset, so the C ABI's 16-byte alignment rules hold) and
+    return (pinned host buffer, device buffer) with the same bytes: a step's
+    host-to-device traffic is then a single copy instead of one per tensor."""
+    layout, off = [], 0
+    for n in names:
+        t = getattr(dc, n)
+        nbytes = t.numel() * t.element_size()
+        layout.append((n, off, nbytes))
+        off = (off + nbytes + 255) // 256 * 256
+    dev = torch.empty(off, dtype=torch.uint8, device=dc.q.device)
+    host = torch.zeros(off, dtype=torch.uint8).pin_memory()
+    for n, o, nbytes in layout:
+        t = getattr(dc, n).contiguous()
+        view = dev[o:o + nbytes].view(t.dtype).view(t.shape)
+        view.copy_(t)
+        host[o:o + nbytes].copy_(t.cpu().view(torch.uint8).reshape(-1))
+        setattr(dc, n, view)
+    return host, dev
 
 
 def output_f64(t: torch.Tensor) -> np.ndarray:
