@@ -356,12 +356,13 @@ int eg_mla_decode(const eg_mla_dims* dims, const void* q, const void* c_pool, co
     if (!encode_decode_maps(maps, dims, c_pool, krope_pool, num_pages)) return EG_MLA_ERR_CUDA;
     apply_trace(a);
     cudaError_t e = egmla::launch_prologue_tc(a, st);
+    bool fused = false;
     if (e == cudaSuccess) {
       prof_mark(st, true);
-      e = egmla::launch_decode_tc(a, maps, false, st);
+      e = egmla::launch_decode_tc(a, maps, false, st, &fused);
       prof_mark(st, false);
     }
-    if (e == cudaSuccess) e = egmla::launch_combine(a, true, st);
+    if (e == cudaSuccess && !fused) e = egmla::launch_combine(a, true, st);
     return to_status(e);
   }
   cudaError_t e = egmla::launch_decode_f32(a, st);
@@ -467,7 +468,7 @@ int eg_mla_debug_gather(const eg_mla_dims* dims, const void* c_pool, const void*
   if (!encode_decode_maps(maps, dims, c_pool, krope_pool, num_pages)) return EG_MLA_ERR_CUDA;
   a.q = nullptr;  // prologue computes the page prefix sums only
   cudaError_t e = egmla::launch_prologue_tc(a, st);
-  if (e == cudaSuccess) e = egmla::launch_decode_tc(a, maps, true, st);
+  if (e == cudaSuccess) e = egmla::launch_decode_tc(a, maps, true, st, nullptr);
   return to_status(e);
 }
 

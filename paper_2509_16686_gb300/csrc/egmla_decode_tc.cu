@@ -47,6 +47,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdint>
 
@@ -67,6 +68,8 @@ constexpr int kTmaWarp = 3;
 constexpr int kGateWarp0 = 4;
 constexpr int kGateWarps = 8;
 constexpr uint32_t kSmemLimit = 232448;
+// sequences per unit of the fused combine
+constexpr uint32_t kFusedMaxG = 16;
 // a head's reference max moves only when a tile exceeds it by 2^8
 constexpr float kLazyLog2 = 8.f;
 
@@ -113,6 +116,9 @@ struct Cfg {
                 "query over-read");
   static_assert(OFF_PBUF + PBUF + (kPage / 16 - 1) * 2 * kQGroupBytes + STEP_SPAN <= OFF_MISC + MISC,
                 "weight over-read");
+  // fused combine: W_UV,h (at most 256 rows) and up to kFusedMaxG merged
+  // latent rows reuse the page-slot area
+  static_assert(256u * D_C * 2 + kFusedMaxG * D_C * 4 + 128 <= OFF_QBUF, "fused combine area");
 };
 
 struct TcParams {
@@ -138,6 +144,13 @@ struct TcParams {
   // run of (tag, clock64) pairs; tag = event << 24 | tile
   unsigned long long* trace;
   int trace_ctas, trace_cap;
+  // fused split combine (cooperative launch only): W_UV, output, grid counter,
+  // and the (head, group of cmb_g sequences) units
+  const __nv_bfloat16* w_uv;
+  __nv_bfloat16* out;
+  uint32_t* grid_bar;
+  int d_v, cmb_groups, cmb_g;
+  int fuse;
 };
 
 // Trace recorder of one role of one CTA (a no-op unless tracing is on).
@@ -170,6 +183,7 @@ struct Bars {
   uint64_t sp_done[2];
   uint64_t sfree[2];           // the softmax warps have read score buffer b
   uint64_t drain_s, drain_o;   // all MMAs of the score / output issuer done
+  uint64_t wbar;               // W_UV rows of the fused combine landed
   uint32_t tmem_base;
   int abort;
 };
@@ -282,6 +296,190 @@ __device__ __forceinline__ float ex2_approx(float x) {
   return y;
 }
 
+// ---------------------------------------------------------------- fused split combine
+// Eight bf16 of a 16-byte piece as floats.
+__device__ __forceinline__ void bf16x8_to_float(const uint4& raw, float (&w)[8]) {
+  const __nv_bfloat162* e = reinterpret_cast<const __nv_bfloat162*>(&raw);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 f = __bfloat1622float2(e[i]);
+    w[2 * i] = f.x;
+    w[2 * i + 1] = f.y;
+  }
+}
+
+// Sums of eight rows whose parts are spread over the warp (v[r] = this lane's
+// part of row r): a transposing butterfly halves the rows a lane carries at
+// each of the xor-16, -8 and -4 exchanges, then two plain steps finish; lane
+// 4r + q (q < 4) ends with the sum of row r.
+__device__ __forceinline__ float reduce8_rows(const float (&v)[8], int lane) {
+  const bool b4 = (lane & 16) != 0, b3 = (lane & 8) != 0, b2 = (lane & 4) != 0;
+  float a[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float send = b4 ? v[i] : v[i + 4];
+    const float keep = b4 ? v[i + 4] : v[i];
+    a[i] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
+  }
+  float c[2];
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const float send = b3 ? a[i] : a[i + 2];
+    const float keep = b3 ? a[i + 2] : a[i];
+    c[i] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
+  }
+  const float send = b2 ? c[0] : c[1];
+  float s = (b2 ? c[1] : c[0]) + __shfl_xor_sync(0xffffffffu, send, 4);
+  s += __shfl_xor_sync(0xffffffffu, s, 2);
+  s += __shfl_xor_sync(0xffffffffu, s, 1);
+  return s;
+}
+
+// Split-KV combine inside the decode kernel (cooperative launch: every CTA is
+// resident, so a grid-wide wait cannot starve).  After its pages each CTA
+// arrives on a grid counter (zeroed by the prologue kernel of the same call)
+// and, once all have arrived, merges its units (head h, group of cmb_g
+// sequences): for each sequence b, over the splits s that covered it,
+//   o = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s,
+//   u_{b,h} = W_UV,h o
+// (a sequence of length 0 gets u = 0).  W_UV,h is bulk-copied into the free
+// page-slot area while the CTA waits for the others.  Merge: a warp per
+// (sequence, 32 features), lane k loading (m, l) of slot k0 + k and every lane
+// O of 32 slots at once (online rescaling across groups of 32).  u: a warp per
+// group of eight output rows (see below).
+template <int D_C>
+__device__ void fused_combine(const TcParams& p, uint8_t* smem, Bars& bars) {
+  constexpr int kWarps = kThreads / 32;
+  constexpr int NFB = D_C / 32;      // 32-feature blocks of a row
+  constexpr int LANES = D_C / 8;     // lanes holding 8 features each
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int G = p.cmb_g, units = kHeads * p.cmb_groups;
+  const uint32_t wbytes = static_cast<uint32_t>(p.d_v) * D_C * 2;
+  uint8_t* wsm = smem;                                                    // [d_v][D_C] bf16
+  float* olat = reinterpret_cast<float*>(smem + ((wbytes + 127u) & ~127u));   // [G][D_C]
+  const uint32_t wbar = smem_u32(&bars.wbar);
+  volatile int* abort_flag = &bars.abort;
+  auto issue_w = [&](int h) {
+    if (tid == 0) {
+      fence_proxy_async_smem();   // the slot area was last used through the generic proxy too
+      mbar_arrive_expect_tx(wbar, wbytes);
+      bulk_load_hint(smem_u32(wsm), p.w_uv + static_cast<size_t>(h) * p.d_v * D_C, wbytes, wbar,
+                     policy_evict_last());
+    }
+  };
+  int u = blockIdx.x;
+  if (u < units) issue_w(u % kHeads);
+  if (tid == 0) {
+    // this CTA's partials are stored (the kernel-end barrier ordered the other
+    // threads' stores before this thread): release them, then wait for all
+    __threadfence();
+    atomicAdd(p.grid_bar, 1u);
+    const uint64_t t0 = globaltimer();
+    while (ld_acquire_gpu(p.grid_bar) < gridDim.x) {
+      if (globaltimer() - t0 > kWaitLimitNs) {
+        report_status(p.status, kStatusTimeout);
+        *abort_flag = 1;
+        break;
+      }
+      __nanosleep(32);
+    }
+  }
+  __syncthreads();
+  int phase = 0;
+  for (; u < units; u += gridDim.x) {
+    const int h = u % kHeads, grp = u / kHeads;
+    const int b0 = grp * G, nb = min(G, p.batch - b0);
+    if (!*abort_flag) {
+      const int total = p.cu[p.batch];
+      const int chunk = split_chunk(total, gridDim.x);
+      for (int w = warp; w < nb * NFB; w += kWarps) {
+        const int j = w / NFB, f = (w % NFB) * 32 + lane, b = b0 + j;
+        const int q0 = p.cu[b], q1 = p.cu[b + 1];
+        const int c0 = q0 / chunk;
+        const int n = q1 > q0 ? (q1 - 1) / chunk - c0 + 1 : 0;
+        const float* po = p.part_o + (static_cast<size_t>(c0 + b) * kHeads + h) * D_C + f;
+        const float* pm = p.part_ml + (static_cast<size_t>(c0 + b) * kHeads + h) * 2;
+        float M = -INFINITY, L = 0.f, acc = 0.f;
+        for (int k0 = 0; k0 < n; k0 += 32) {
+          const int kn = min(32, n - k0);
+          float2 ml = make_float2(-INFINITY, 0.f);
+          if (lane < kn) ml = __ldcg(reinterpret_cast<const float2*>(pm + static_cast<size_t>(k0 + lane) * kHeads * 2));
+          float ov[32];
+#pragma unroll
+          for (int kk = 0; kk < 32; ++kk)
+            ov[kk] = kk < kn ? __ldcg(po + static_cast<size_t>(k0 + kk) * kHeads * D_C) : 0.f;
+          float mc = ml.x;
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) mc = fmaxf(mc, __shfl_xor_sync(0xffffffffu, mc, o));
+          const float Mn = fmaxf(M, mc);
+          const float sc = exp2f(M - Mn);   // 0 on the first group (M = -inf)
+          const float wk = lane < kn ? exp2f(ml.x - Mn) : 0.f;
+          float lw = wk * ml.y;
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) lw += __shfl_xor_sync(0xffffffffu, lw, o);
+          L = fmaf(L, sc, lw);
+          acc *= sc;
+#pragma unroll
+          for (int kk = 0; kk < 32; ++kk) acc = fmaf(__shfl_sync(0xffffffffu, wk, kk), ov[kk], acc);
+          M = Mn;
+        }
+        olat[j * D_C + f] = n > 0 ? acc / L : 0.f;
+      }
+    }
+    // the W_UV,h rows have landed: thread 0 waits on its own flag, so that the
+    // copy is waited for even after an abort (no copy may outlive the CTA)
+    if (tid == 0) {
+      volatile int own = 0;
+      if (!mbar_wait(wbar, phase, &own)) {
+        report_status(p.status, kStatusTimeout);
+        *abort_flag = 1;
+      }
+    }
+    phase ^= 1;
+    __syncthreads();
+    if (*abort_flag) return;
+    // u = W_UV,h o: a warp per group of 8 output rows (loaded once, lane l
+    // holding features 8l .. 8l + 7 of each), then for each sequence the eight
+    // row sums, reduced across the lanes by a transposing butterfly (9
+    // shuffles) after which lane 4r holds row r
+    const int nvg = (p.d_v + 7) / 8;
+    for (int g = warp; g < nvg; g += kWarps) {
+      uint4 wraw[8];
+#pragma unroll
+      for (int r = 0; r < 8; ++r) {
+        const int v = 8 * g + r;
+        wraw[r] = make_uint4(0, 0, 0, 0);
+        if (lane < LANES && v < p.d_v)
+          wraw[r] = *reinterpret_cast<const uint4*>(wsm + (static_cast<size_t>(v) * D_C + 8 * lane) * 2);
+      }
+      for (int j = 0; j < nb; ++j) {
+        float o8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        if (lane < LANES) {
+          const float4 x0 = *reinterpret_cast<const float4*>(olat + j * D_C + 8 * lane);
+          const float4 x1 = *reinterpret_cast<const float4*>(olat + j * D_C + 8 * lane + 4);
+          o8[0] = x0.x; o8[1] = x0.y; o8[2] = x0.z; o8[3] = x0.w;
+          o8[4] = x1.x; o8[5] = x1.y; o8[6] = x1.z; o8[7] = x1.w;
+        }
+        float part[8];
+#pragma unroll
+        for (int r = 0; r < 8; ++r) {
+          float wv[8];
+          bf16x8_to_float(wraw[r], wv);
+          part[r] = 0.f;
+#pragma unroll
+          for (int e = 0; e < 8; ++e) part[r] = fmaf(wv[e], o8[e], part[r]);
+        }
+        const float sum = reduce8_rows(part, lane);
+        const int v = 8 * g + (lane >> 2);
+        if ((lane & 3) == 0 && v < p.d_v)
+          p.out[(static_cast<size_t>(b0 + j) * kHeads + h) * p.d_v + v] = __float2bfloat16_rn(sum);
+      }
+    }
+    __syncthreads();   // W and olat are free for the next unit
+    if (u + static_cast<int>(gridDim.x) < units) issue_w((u + gridDim.x) % kHeads);
+  }
+}
+
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 z = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&z);
@@ -322,6 +520,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(smem_u32(&bars.sfree[1]), kSoftWarps);
     mbar_init(smem_u32(&bars.drain_s), 1);
     mbar_init(smem_u32(&bars.drain_o), 1);
+    mbar_init(smem_u32(&bars.wbar), 1);
     bars.abort = 0;
     fence_mbar_init();
   }
@@ -941,10 +1140,27 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   if (warp == kMmaWarp) tmem_dealloc(tmem, C::TMEM_COLS);
   if (threadIdx.x == 0 && bars.abort) report_status(p.status, kStatusTimeout);
+  if (!DUMP && p.fuse) fused_combine<D_C>(p, smem, bars);
+}
+
+// CTAs of `kern` that the current device holds at once (1 per SM here), cached per kernel
+template <typename K>
+int resident_ctas(K kern, uint32_t smem) {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  if (cached[dev] == 0) {
+    int per_sm = 0, sms = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return 0;
+    cached[dev] = std::max(0, per_sm) * sms;
+  }
+  return cached[dev];
 }
 
 template <int D_C, bool GATE, bool DUMP>
-cudaError_t launch_one(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_t st) {
+cudaError_t launch_one(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_t st, bool* fused) {
   using C = Cfg<D_C, GATE>;
   auto kern = decode_tc_kernel<D_C, GATE, DUMP>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
@@ -977,8 +1193,33 @@ cudaError_t launch_one(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_
   p.trace = static_cast<unsigned long long*>(a.trace);
   p.trace_ctas = a.trace_ctas;
   p.trace_cap = a.trace_cap;
-  kern<<<a.num_splits, kThreads, C::SMEM, st>>>(maps[0], maps[1], p);
-  return cudaGetLastError();
+  // The split combine runs inside this kernel when every CTA of the grid can
+  // be resident at once (a cooperative launch guarantees it, or fails).
+  p.w_uv = static_cast<const __nv_bfloat16*>(a.w_uv);
+  p.out = static_cast<__nv_bfloat16*>(a.out);
+  p.grid_bar = reinterpret_cast<uint32_t*>(ws + wl.off_bar);
+  p.d_v = a.d_v;
+  int groups = std::max(1, std::min(a.batch, a.num_splits / kHeads));
+  const int g = std::min(static_cast<int>(kFusedMaxG), (a.batch + groups - 1) / groups);
+  p.cmb_g = g;
+  p.cmb_groups = (a.batch + g - 1) / g;
+  p.fuse = !DUMP && a.batch > 0 && a.num_splits <= resident_ctas(kern, C::SMEM);
+  if (fused) *fused = p.fuse != 0;
+  if (!p.fuse) {
+    kern<<<a.num_splits, kThreads, C::SMEM, st>>>(maps[0], maps[1], p);
+    return cudaGetLastError();
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.num_splits);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = C::SMEM;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, maps[0], maps[1], p);
 }
 
 }  // namespace
@@ -988,18 +1229,20 @@ bool tc_supported(int d_c, int gate) {
   return d_c == 192 || d_c == 256 || d_c == 512;
 }
 
-cudaError_t launch_decode_tc(const DecodeArgs& a, const CUtensorMap* maps, bool dump, cudaStream_t st) {
+cudaError_t launch_decode_tc(const DecodeArgs& a, const CUtensorMap* maps, bool dump, cudaStream_t st,
+                             bool* fused) {
+  if (fused) *fused = false;
   if (dump) {
-    if (a.d_c == 192) return launch_one<192, true, true>(a, maps, st);
-    if (a.d_c == 256) return launch_one<256, true, true>(a, maps, st);
+    if (a.d_c == 192) return launch_one<192, true, true>(a, maps, st, nullptr);
+    if (a.d_c == 256) return launch_one<256, true, true>(a, maps, st, nullptr);
     return cudaErrorInvalidValue;
   }
   if (a.gate) {
-    if (a.d_c == 192) return launch_one<192, true, false>(a, maps, st);
-    if (a.d_c == 256) return launch_one<256, true, false>(a, maps, st);
+    if (a.d_c == 192) return launch_one<192, true, false>(a, maps, st, fused);
+    if (a.d_c == 256) return launch_one<256, true, false>(a, maps, st, fused);
   } else {
-    if (a.d_c == 192) return launch_one<192, false, false>(a, maps, st);
-    if (a.d_c == 256) return launch_one<256, false, false>(a, maps, st);
+    if (a.d_c == 192) return launch_one<192, false, false>(a, maps, st, fused);
+    if (a.d_c == 256) return launch_one<256, false, false>(a, maps, st, fused);
     if (a.d_c == 512) return launch_decode_wide(a, maps, st);
   }
   return cudaErrorInvalidValue;

@@ -67,8 +67,11 @@ cudaError_t launch_append(const AppendArgs& a, cudaStream_t st);
 cudaError_t launch_prologue_tc(const DecodeArgs& a, cudaStream_t st);
 cudaError_t launch_decode_f32(const DecodeArgs& a, cudaStream_t st);
 cudaError_t launch_combine(const DecodeArgs& a, bool tc_path, cudaStream_t st);
-// tensor-core split-KV kernel; `maps` = {c_pool map (3-D page box for d_c <= 256), kr_pool map}
-cudaError_t launch_decode_tc(const DecodeArgs& a, const CUtensorMap* maps, bool dump, cudaStream_t st);
+// tensor-core split-KV kernel; `maps` = {c_pool map (3-D page box for d_c <= 256), kr_pool map}.
+// *fused (may be null) is set when the split combine ran inside the kernel
+// (cooperative launch); otherwise launch_combine must follow.
+cudaError_t launch_decode_tc(const DecodeArgs& a, const CUtensorMap* maps, bool dump, cudaStream_t st,
+                             bool* fused);
 // d_c = 512 without the gate (output accumulated with latent features in TMEM lanes)
 cudaError_t launch_decode_wide(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_t st);
 // true if the bf16 tensor-core path has a kernel for these shapes
