@@ -1,17 +1,21 @@
 """Decode-step benchmark of libegmla on synthetic EG-MLA workloads.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c32k] [--impl reference]
+    python bench.py --sweep        (decode throughput vs context length)
 
 A step is one pass of the whole decode hot path for one batch: append of each
 sequence's new token to the paged latent cache, query absorption, the split-KV
-gated latent attention and the split merge with the W_UV up-projection.  The
-default workload is the 32K-context one (batch 8, 16 heads, d_c 256, RoPE 64,
-64-token pages permuted over a shared pool, vocabulary 32000), on which the
-roofline target of the hot path is stated.
+gated latent attention and the split merge with the W_UV up-projection (for
+layers24: that, for each of 24 attention layers in turn).  The default
+workload is the 32K-context one (batch 8, 16 heads, d_c 256, RoPE 64, 64-token
+pages permuted over a shared pool, vocabulary 32000), on which the roofline
+target of the hot path is stated.  --sweep prints one line per context length
+L = 1K .. 64K at batch 8 (d_c 256, contiguous pages).
 
 value: decode tokens/s (new tokens produced per second, all GPUs) with every
 input resident in HBM; the step is replayed from a CUDA graph over three
-rotating cache replicas (3 x 168 MB > L2), so the latent stream comes from HBM.
+rotating cache replicas (3 x 168 MB > L2; layers24: 24 distinct layer caches),
+so the latent stream comes from HBM.
 e2e: the same metric through the C ABI from pinned HOST buffers, the per-step
 inputs (packed in one buffer) copied in and the output copied back inside the
 timed region, calls issued eagerly from Python.
@@ -52,9 +56,12 @@ REPLICAS = 3
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--steps", type=int, default=None,
+                    help="timed steps (default 20000; 200 for layers24, 2000 per length for --sweep)")
     ap.add_argument("--warmup", type=int, default=30)
-    ap.add_argument("--workload", default="c32k", choices=["c32k", "c4k", "ragged", "ragged_mla"])
+    ap.add_argument("--workload", default="c32k", choices=["c32k", "c4k", "ragged", "ragged_mla", "layers24"])
+    ap.add_argument("--sweep", action="store_true",
+                    help="decode throughput vs context length: batch 8, d_c 256, L = 1K .. 64K, one line per L")
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--splits", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -74,10 +81,26 @@ def make_workload(name):
     elif name == "ragged":
         case = synth.case_ragged(keep_logical=False)
         desc = "ragged: batch 128, contexts log-uniform [128, 16384], 16 heads, d_c 192, vocab 50000, Zipf(1.1) ids"
-    else:
+    elif name == "ragged_mla":
         case = synth.case_ragged(gate=False, keep_logical=False)
         desc = "ragged_mla: plain-MLA baseline (gate off) at d_c 512 on the ragged lengths"
+    elif name == "layers24":
+        case = synth.case_layer(0)
+        desc = "layers24: decoder step over 24 attention layers (append + decode per layer on one stream), " \
+               "batch 64 x context 8192, 16 heads, d_c 256, d_rope 64, vocab 50000, contiguous pages; layer 0's " \
+               "seeded synthetic cache, ids, gate table, weights and inputs cloned into 24 distinct device copies"
+    else:
+        ctx = int(name[3:])
+        case = synth.case_c4k(batch=8, ctx=ctx, keep_logical=False)
+        desc = f"ctx{ctx}: batch 8 x context {ctx}, 16 heads, d_c 256, d_rope 64, vocab 32000, contiguous pages"
     return case, desc
+
+
+def layers_of(name):
+    return 24 if name == "layers24" else 1
+
+
+SWEEP_CTX = (1024, 2048, 4096, 8192, 16384, 32768, 65536)
 
 
 def dist_env():
@@ -216,7 +239,8 @@ def run_reference(args):
             times.append(dt)
         if time.perf_counter() - t_start > 170:
             break
-    t_token = statistics.mean(times) * H * (L / S)
+    n_layers = layers_of(args.workload)
+    t_token = statistics.mean(times) * H * (L / S) * n_layers
     rate = 1.0 / t_token
     line = {
         "impl": "reference", "metric": METRIC, "value": rate, "unit": UNIT, "n_gpus": args.gpus,
@@ -225,7 +249,7 @@ def run_reference(args):
         "config": {"workload": desc, "batch": case.batch, "ctx": L},
         "cpu_baseline": {"value": rate, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
                          "sample": f"per step one head of one sequence over its first {S} of {L} cached "
-                                   f"tokens, scaled x{H} heads x{L / S:.1f} context"},
+                                   f"tokens, scaled x{H} heads x{L / S:.1f} context x{n_layers} layer(s)"},
         "e2e": {"value": rate, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -243,57 +267,65 @@ def kernel_source_sha(files):
     return h.hexdigest()[:16]
 
 
-def main():
-    args = parse()
-    if args.impl == "reference":
-        return run_reference(args)
-    import torch
-    ws, rank, local = dist_env()
-    dist = None
-    if ws > 1:
-        import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+def run_gpu(args, workload, torch, dist, ws, rank):
+    """One bench line of `workload` (see the module docstring)."""
+    from paper_2509_16686_gb300 import _lib, device  # noqa: F401
     dev = torch.cuda.current_device()
-
-    from paper_2509_16686_gb300 import _lib, device, synth  # noqa: F401
-    from oracle import egmla_oracle as orc  # CPU-baseline leg only
-
-    case, desc = make_workload(args.workload)
+    case, desc = make_workload(workload)
     B = case.batch
     d = case.dims
-    dcs = [device.upload(case, num_splits=args.splits)]
-    for _ in range(REPLICAS - 1):
-        r = device.upload(case, num_splits=args.splits)
-        dcs.append(r)
-    # all replicas share the weights, block table and workspace of the first;
-    # each keeps its own per-step inputs, packed in one device buffer (one
-    # host-to-device copy per end-to-end step), and its own output
-    for r in dcs[1:]:
-        for name in ("gate_table", "ln_gamma", "ln_beta", "w_uk", "w_uv", "workspace", "status", "block_table"):
-            setattr(r, name, getattr(dcs[0], name))
-    packed = [device.pack_step_inputs(r) for r in dcs]
+    n_layers = layers_of(workload)
+    steps_arg = args.steps if args.steps is not None else (200 if n_layers > 1 else
+                                                          2000 if args.sweep else 20000)
+    # units: one append + decode each.  A step runs one group of units: one of
+    # REPLICAS rotating cache replicas (so consecutive steps stream different
+    # memory), or all layers of the decoder.
+    if n_layers > 1:
+        base = device.upload(case, num_splits=args.splits)
+        units = [base] + [device.clone_case(base) for _ in range(n_layers - 1)]
+        groups = [units]
+        l2_note = f"inputs larger than L2: {n_layers} layers' distinct caches"
+    else:
+        units = [device.upload(case, num_splits=args.splits) for _ in range(REPLICAS)]
+        # replicas share the weights, block table and workspace of the first
+        for r in units[1:]:
+            for name in ("gate_table", "ln_gamma", "ln_beta", "w_uk", "w_uv", "workspace", "status",
+                         "block_table"):
+                setattr(r, name, getattr(units[0], name))
+        groups = [[u] for u in units]
+        l2_note = f"inputs larger than L2: {REPLICAS} rotating cache replicas"
+    # each unit keeps its own per-step inputs, packed in one device buffer (one
+    # host-to-device copy per unit in the end-to-end run), and its own output
+    packed = [device.pack_step_inputs(u) for u in units]
     stream = torch.cuda.Stream()
     tokens_cached = int(case.seq_lens.astype(np.int64).sum())
     elem = 2 if d.dtype == "bf16" else 4
     id_bytes = 4 if d.gate else 0
-    cache_bytes = tokens_cached * ((d.d_c + d.d_rope) * elem + id_bytes)
-    splits = dcs[0].num_splits or _lib.eg_mla_default_num_splits()
-    launches_per_step = 4 if d.dtype == "bf16" else 3
+    cache_bytes = tokens_cached * ((d.d_c + d.d_rope) * elem + id_bytes)     # per unit (layer)
+    splits = units[0].num_splits or _lib.eg_mla_default_num_splits()
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    # append + prologue + decode, + the combine kernel unless the decode kernel
+    # runs fused (bf16, d_c 192/256, a grid of at most one CTA per SM)
+    fused = d.dtype == "bf16" and d.d_c in (192, 256) and splits <= sms
+    launches_per_step = n_layers * (3 if fused else 4)
 
-    # ---- warm-up, then capture one graph of REPLICAS steps (one per cache replica)
+    def run_group(g):
+        for u in g:
+            u.step(stream)
+
+    # ---- warm-up, then capture one graph of every group (one step each)
     with torch.cuda.stream(stream):
         for i in range(max(3, args.warmup)):
-            dcs[i % REPLICAS].step(stream)
+            run_group(groups[i % len(groups)])
     stream.synchronize()
-    assert dcs[0].read_status() == 0, "device status after warm-up"
+    assert units[0].read_status() == 0, "device status after warm-up"
     graph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(graph, stream=stream):
-        for r in dcs:
-            r.step(stream)
+        for g in groups:
+            run_group(g)
     torch.cuda.synchronize()
-    reps = max(1, math.ceil(args.steps / REPLICAS))
-    steps = reps * REPLICAS
+    reps = max(1, math.ceil(steps_arg / len(groups)))
+    steps = reps * len(groups)
     with torch.cuda.stream(stream):
         for _ in range(2):
             graph.replay()
@@ -318,7 +350,7 @@ def main():
         t = torch.tensor([elapsed_ms], device="cuda")
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         elapsed_ms = float(t.item())
-    assert dcs[0].read_status() == 0, "device status after timed region"
+    assert units[0].read_status() == 0, "device status after timed region"
     ms_per_step = elapsed_ms / steps
     value = ws * B * steps / (elapsed_ms / 1e3)
 
@@ -326,12 +358,12 @@ def main():
     # recorded as nodes of a captured graph of the same steps (so that each
     # launch is timed as it runs in the step, without host launch gaps); the
     # graph is replayed twice and the events hold the second replay
-    prof_steps = 10 * REPLICAS
-    _lib.eg_mla_profile_begin(prof_steps)
+    prof_groups = max(1, 10 // n_layers) * len(groups) if n_layers == 1 else 2
+    _lib.eg_mla_profile_begin(prof_groups * len(groups[0]))
     pgraph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(pgraph, stream=stream):
-        for i in range(prof_steps):
-            dcs[i % REPLICAS].step(stream)
+        for i in range(prof_groups):
+            run_group(groups[i % len(groups)])
     with torch.cuda.stream(stream):
         pgraph.replay()
         pgraph.replay()
@@ -350,48 +382,51 @@ def main():
     tpath = os.path.join(ROOT, "profiles", "traffic.json")
     if os.path.exists(tpath):
         tall = json.load(open(tpath))
-        tj = tall.get(args.workload)
-        # counters taken on other kernel sources no longer describe this kernel
+        tj = tall.get(workload)
         if tj and tall.get("source_sha") == kernel_source_sha(tall.get("source_files", [])):
             traffic = tj.get("dram_bytes_per_launch")
 
-    # ---- end to end through the C ABI with host buffers.  Step i uses replica
-    # i % REPLICAS and runs on the compute stream (its two C calls bound once,
-    # see _lib.bind_step); a copy stream carries the input copy of step i + 1
-    # (issued first, so it overlaps step i) and the read-back of step i's
-    # output.  Events order each replica's buffers between uses.
-    e2e_steps = args.e2e_steps or min(steps, 2000)
-    h_outs = [torch.empty(r.out.shape, dtype=r.out.dtype).pin_memory() for r in dcs]
-    h2d = packed[0][0].numel() * packed[0][0].element_size()
-    d2h = h_outs[0].numel() * h_outs[0].element_size()
-    steps_bound = [r.bind(stream) for r in dcs]
+    # ---- end to end through the C ABI with host buffers.  The units of the
+    # steps run in order on the compute stream (each unit's two C calls bound
+    # once, see _lib.bind_step); a copy stream carries the input copy of the
+    # next unit (issued first, so it overlaps this one) and the read-back of
+    # this unit's output.  Events order each unit's buffers between uses.
+    e2e_steps = args.e2e_steps or min(steps, 2000 if n_layers == 1 else 100)
+    pos = {id(u): k for k, u in enumerate(units)}
+    seq = [pos[id(u)] for s_ in range(e2e_steps) for u in groups[s_ % len(groups)]]
+    h_outs = [torch.empty(u.out.shape, dtype=u.out.dtype).pin_memory() for u in units]
+    h2d = sum(packed[k][0].numel() * packed[k][0].element_size() for k in seq[:len(seq) // e2e_steps])
+    d2h = sum(h_outs[k].numel() * h_outs[k].element_size() for k in seq[:len(seq) // e2e_steps])
+    steps_bound = [u.bind(stream) for u in units]
     s_copy = torch.cuda.Stream()
-    ev_in = [torch.cuda.Event() for _ in dcs]
-    ev_comp = [torch.cuda.Event() for _ in dcs]
-    ev_out = [torch.cuda.Event() for _ in dcs]
+    nu = len(units)
+    ev_in = [torch.cuda.Event() for _ in units]
+    ev_comp = [torch.cuda.Event() for _ in units]
+    ev_out = [torch.cuda.Event() for _ in units]
+    used = [False] * nu
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
     e0.record(stream)
     s_copy.wait_stream(stream)
     with torch.cuda.stream(s_copy):
-        packed[0][1].copy_(packed[0][0], non_blocking=True)
-        ev_in[0].record(s_copy)
-        for i in range(e2e_steps):
-            k = i % REPLICAS
+        packed[seq[0]][1].copy_(packed[seq[0]][0], non_blocking=True)
+        ev_in[seq[0]].record(s_copy)
+        for i, k in enumerate(seq):
             stream.wait_event(ev_in[k])
-            if i >= REPLICAS:
-                stream.wait_event(ev_out[k])      # step i - REPLICAS's output has been read back
+            if used[k]:
+                stream.wait_event(ev_out[k])          # this unit's last output has been read back
             steps_bound[k]()
             ev_comp[k].record(stream)
-            if i + 1 < e2e_steps:
-                k1 = (i + 1) % REPLICAS
-                if i + 1 >= REPLICAS:
-                    s_copy.wait_event(ev_comp[k1])   # step i + 1 - REPLICAS has read these inputs
+            if i + 1 < len(seq):
+                k1 = seq[i + 1]
+                if used[k1] or k1 == k:
+                    s_copy.wait_event(ev_comp[k1])    # the unit's last run has read its inputs
                 packed[k1][1].copy_(packed[k1][0], non_blocking=True)
                 ev_in[k1].record(s_copy)
             s_copy.wait_event(ev_comp[k])
-            h_outs[k].copy_(dcs[k].out, non_blocking=True)
+            h_outs[k].copy_(units[k].out, non_blocking=True)
             ev_out[k].record(s_copy)
+            used[k] = True
     stream.wait_stream(s_copy)
     e1.record(stream)
     torch.cuda.synchronize()
@@ -401,32 +436,53 @@ def main():
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         e2e_ms = float(t.item())
     e2e_value = ws * B * e2e_steps / (e2e_ms / 1e3)
+    assert units[0].read_status() == 0, "device status after end-to-end run"
 
-    # ---- CPU baseline (rank 0, N = 1 only)
+    # ---- CPU baseline (rank 0, N = 1 only); a decode token passes every layer
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         rate, sample, _ = oracle_sample_rate(case, budget_s=12.0)
+        if n_layers > 1:
+            rate /= n_layers
+            sample += f", one layer of {n_layers} (rate / {n_layers})"
         cpu = {"value": rate, "unit": UNIT, "cores": host_cores(), "kind": "oracle", "sample": sample}
 
-    if rank == 0:
-        line = {
-            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": steps, "warmup": args.warmup,
-            "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": d.dtype, "data": "synthetic",
-            "config": {"workload": desc, "batch": B, "ctx_tokens_cached": tokens_cached, "splits": splits,
-                       "page_size": d.page_size, "l2": f"inputs larger than L2: {REPLICAS} rotating cache "
-                       f"replicas of {cache_bytes / 1e6:.0f} MB", "graph": "step replayed from a CUDA graph"},
-            "kv_cache_gbs": cache_bytes * steps / (elapsed_ms / 1e3) / 1e9 * 1.0,
-            "kv_bytes_per_token": (d.d_c + d.d_rope) * elem + id_bytes,
-            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                         "frac": achieved / peak, "traffic": traffic, "kernel": "decode_tc_kernel",
-                         "kernel_ms": k_ms, "bytes_per_launch": cache_bytes, "peak_source": peak_src},
-            "cpu_baseline": cpu,
-            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-            "gpu_launches": steps * launches_per_step,
-            "clocks": clk.summary(),
-        }
-        print(json.dumps(line), flush=True)
+    return {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": steps, "warmup": args.warmup,
+        "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": d.dtype, "data": "synthetic",
+        "config": {"workload": desc, "batch": B, "layers": n_layers, "ctx_tokens_cached": tokens_cached,
+                   "splits": splits, "page_size": d.page_size,
+                   "l2": f"{l2_note} of {cache_bytes / 1e6:.0f} MB", "graph": "step replayed from a CUDA graph"},
+        "kv_cache_gbs": n_layers * cache_bytes * steps / (elapsed_ms / 1e3) / 1e9,
+        "kv_bytes_per_token": (d.d_c + d.d_rope) * elem + id_bytes,
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic, "kernel": "decode_tc_kernel",
+                     "kernel_ms": k_ms, "bytes_per_launch": cache_bytes, "peak_source": peak_src},
+        "cpu_baseline": cpu,
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": steps * launches_per_step,
+        "clocks": clk.summary(),
+    }
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    import torch
+    ws, rank, local = dist_env()
+    dist = None
+    if ws > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    workloads = [f"ctx{c}" for c in SWEEP_CTX] if args.sweep else [args.workload]
+    for wl in workloads:
+        line = run_gpu(args, wl, torch, dist, ws, rank)
+        if rank == 0:
+            print(json.dumps(line), flush=True)
+        torch.cuda.empty_cache()
     if dist:
         dist.barrier()
         dist.destroy_process_group()

@@ -123,6 +123,16 @@ def upload(case: Case, device="cuda", num_splits: int = 0) -> DeviceCase:
     )
 
 
+def clone_case(dc: DeviceCase, share=("workspace", "status")) -> DeviceCase:
+    """A copy of `dc` in distinct device memory (same values), sharing the
+    fields named in `share` (e.g. one workspace for units run in sequence)."""
+    fields = {}
+    for f in dataclasses.fields(dc):
+        v = getattr(dc, f.name)
+        fields[f.name] = v.clone() if isinstance(v, torch.Tensor) and f.name not in share else v
+    return DeviceCase(**fields)
+
+
 # inputs that change from one decode step to the next
 STEP_INPUTS = ("q", "c_new", "kr_new", "ids_new", "positions", "seq_lens")
 
