@@ -153,7 +153,9 @@ size_t eg_mla_decode_workspace_size(const eg_mla_dims* dims, int32_t batch, int3
  *   seq_lens     [batch] int32 (device), each <= max_seq_len
  *   max_seq_len  host-side upper bound of seq_lens (<= max_pages_per_seq*page_size)
  *   gate_table   [vocab, d_c] model dtype: G[i] = W^UE Emb(i) precomputed per
- *                vocabulary entry (EG-MLA-A); ignored for EG_MLA_GATE_NONE
+ *                vocabulary entry (EG-MLA-A); ignored for EG_MLA_GATE_NONE;
+ *                32-byte aligned for bf16 (read in 32-byte pieces), 16-byte
+ *                aligned for fp32
  *   ln_gamma, ln_beta  [d_c] fp32, may be NULL (gamma = 1, beta = 0)
  *   w_uk         [num_heads, d_nope, d_c] model dtype (the k_nope rows of the
  *                listing's wkv_b weight viewed per head), 16-byte aligned

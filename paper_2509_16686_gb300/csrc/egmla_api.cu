@@ -138,8 +138,10 @@ int fill_decode_args(DecodeArgs& a, const eg_mla_dims* d, const void* c_pool, co
     return EG_MLA_ERR_INVALID_ARG;
   if (d->gate_mode == EG_MLA_GATE_MUL_LN && (id_pool == nullptr || gate_table == nullptr))
     return EG_MLA_ERR_INVALID_ARG;
+  // the bf16 kernels read gate rows in 32-byte pieces
+  const size_t g_align = is_tc_path(d) ? 32 : 16;
   if (!aligned(c_pool, 16) || !aligned(krope_pool, 16) || (id_pool && !aligned(id_pool, 16)) ||
-      (gate_table && !aligned(gate_table, 16)))
+      (gate_table && d->gate_mode == EG_MLA_GATE_MUL_LN && !aligned(gate_table, g_align)))
     return EG_MLA_ERR_INVALID_ARG;
   int32_t splits = 0;
   rc = resolve_splits(num_splits, &splits);

@@ -744,43 +744,43 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else if (warp >= kGateWarp0) {
     // ---------------------------------------------------------------- gate: z = c (*) g, LN statistics
-    // Quarter-warp k = 4 (warp - 4) + lane / 8 owns token rows 2k and 2k + 1;
-    // lane u = lane % 8 takes the 16-byte unit u of every 64-feature column of
-    // both rows.  Each quarter-warp access then covers one whole 128-byte line:
-    // of the gate table (a global load that reads whole lines costs the SM's
-    // load/store data path one wavefront per line, one that reads parts of many
-    // lines about one per lane) and of the swizzled page (eight distinct bank
-    // groups).  The gate rows come from L2 (the table stays there under an
-    // evict-last hint while the cache stream is evict-first): each tile issues
-    // the id loads of the tile two ahead and the gate-row loads of the next
-    // tile, so neither latency sits on the loop.
+    // Quarter-warp k = 4 (warp - 4) + lane / 8 owns token rows 2k (lanes 0-3)
+    // and 2k + 1 (lanes 4-7); lane p = lane % 4 of a row takes the 16-byte
+    // units 2p and 2p + 1 of every 64-feature column.  The gate-row load of a
+    // column is then one 32-byte load per lane and a whole 128-byte line per
+    // row (the load/store data path pays per instruction and per line, so
+    // fewer, wider loads are cheaper), and a quarter-warp's shared-memory
+    // accesses to the swizzled page still hit eight distinct bank groups (the
+    // two rows differ in swizzle parity).  The gate rows come from L2 (the
+    // table stays there under an evict-last hint while the cache stream is
+    // evict-first): each tile issues the id loads of the tile two ahead and the
+    // gate-row loads of the next tile, so neither latency sits on the loop.
     const int gw = warp - kGateWarp0;
-    const int u = lane & 7;
-    const int row0 = 2 * (gw * 4 + (lane >> 3));   // rows row0 and row0 + 1
+    const int pp = lane & 3;
+    const int row = 2 * (gw * 4 + (lane >> 3)) + ((lane >> 2) & 1);
     const uint64_t pol_keep = policy_evict_last();
     Walker w;
     w.start(p.cu, p.seq_lens, p.batch);
     PageWindow pw;
-    // ids of this thread's two rows of a tile (0 past the end of the page or for
-    // a bad page, which the producer reports)
-    auto load_ids = [&](const Tile& tt, int (&id)[2]) {
+    // id of this thread's row of a tile (0 past the end of the page or for a
+    // bad page, which the producer reports)
+    auto load_id = [&](const Tile& tt) -> int {
       const int pg = pw.page(p, tt, lane);
       const int n = (pg >= 0 && pg < p.num_pages) ? tt.ntok : 0;
-#pragma unroll
-      for (int rr = 0; rr < 2; ++rr)
-        id[rr] = row0 + rr < n ? __ldg(p.id_pool + static_cast<size_t>(pg) * kPage + row0 + rr) : 0;
+      return row < n ? __ldg(p.id_pool + static_cast<size_t>(pg) * kPage + row) : 0;
     };
-    auto load_g = [&](int (&id)[2], uint4 (&gv)[2][C::NCH]) {
-#pragma unroll
-      for (int rr = 0; rr < 2; ++rr) {
-        if ((unsigned)id[rr] >= (unsigned)p.vocab) {
-          report_status(p.status, kStatusOutOfRange);
-          id[rr] = 0;
-        }
-        const __nv_bfloat16* src = p.gate_table + static_cast<size_t>(id[rr]) * D_C + u * 8;
-#pragma unroll
-        for (int fc = 0; fc < C::NCH; ++fc) gv[rr][fc] = ldg_16_na_hint(src + fc * 64, pol_keep);
+    auto load_g = [&](int& id, uint4 (&gv)[C::NCH][2]) {
+      if ((unsigned)id >= (unsigned)p.vocab) {
+        report_status(p.status, kStatusOutOfRange);
+        id = 0;
       }
+      const __nv_bfloat16* src = p.gate_table + static_cast<size_t>(id) * D_C + pp * 16;
+#pragma unroll
+      for (int fc = 0; fc < C::NCH; ++fc) ldg_32_na_hint(src + fc * 64, pol_keep, gv[fc][0], gv[fc][1]);
+    };
+    // shared-memory offset of unit (2 pp + h) of column fc of this thread's row
+    auto unit_off = [&](int fc, int h) -> uint32_t {
+      return fc * C::PCHUNK + row * 128 + (((2 * pp + h) ^ (row & 7)) << 4);
     };
     Tracer tr;
     tr.init(p, 2);
@@ -789,11 +789,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool have = w.next(t);
     bool have1 = have && w.next(t1);
     bool have2 = have1 && w.next(t2);
-    int id0[2] = {0, 0}, id1[2] = {0, 0}, id2[2] = {0, 0};   // ids of tiles j, j + 1, j + 2
-    uint4 gcur[2][C::NCH], gnext[2][C::NCH];
+    int id0 = 0, id1 = 0, id2 = 0;   // ids of tiles j, j + 1, j + 2
+    uint4 gcur[C::NCH][2], gnext[C::NCH][2];
     if (GATE) {
-      if (have) load_ids(t, id0);
-      if (have1) load_ids(t1, id1);
+      if (have) id0 = load_id(t);
+      if (have1) id1 = load_id(t1);
       if (have) load_g(id0, gcur);
     }
     int j = 0;
@@ -802,30 +802,30 @@ __global__ void __launch_bounds__(kThreads, 1)
       tr.mark(0, j);
       if (GATE) {
         // prefetch: ids of tile j + 2, gate rows of tile j + 1
-        if (have2) load_ids(t2, id2);
+        if (have2) id2 = load_id(t2);
         if (have1) load_g(id1, gnext);
       }
       if (!warp_wait(smem_u32(&bars.full[slot]), (j / C::NS) & 1, abort_flag)) break;
       tr.mark(1, j);
       uint8_t* cpage = smem + slot * C::SLOT;
       if (DUMP) {
+        if (row < t.ntok) {
+          const size_t o = static_cast<size_t>(t.b) * p.dump_len + t.tok0 + row;
+          uint4* dc = reinterpret_cast<uint4*>(p.dump_c + o * D_C);
+          uint4* dg = reinterpret_cast<uint4*>(p.dump_g + o * D_C);
 #pragma unroll
-        for (int rr = 0; rr < 2; ++rr) {
-          const int row = row0 + rr;
-          if (row < t.ntok) {
-            const size_t o = static_cast<size_t>(t.b) * p.dump_len + t.tok0 + row;
-            uint4* dc = reinterpret_cast<uint4*>(p.dump_c + o * D_C);
-            uint4* dg = reinterpret_cast<uint4*>(p.dump_g + o * D_C);
+          for (int fc = 0; fc < C::NCH; ++fc) {
 #pragma unroll
-            for (int fc = 0; fc < C::NCH; ++fc) {
-              dc[fc * 8 + u] =
-                  *reinterpret_cast<const uint4*>(cpage + fc * C::PCHUNK + row * 128 + ((u ^ (row & 7)) << 4));
-              dg[fc * 8 + u] = gcur[rr][fc];
+            for (int h = 0; h < 2; ++h) {
+              dc[fc * 8 + 2 * pp + h] = *reinterpret_cast<const uint4*>(cpage + unit_off(fc, h));
+              dg[fc * 8 + 2 * pp + h] = gcur[fc][h];
             }
-            reinterpret_cast<uint4*>(p.dump_kr + o * kRope)[u] =
-                *reinterpret_cast<const uint4*>(cpage + C::KR_OFF + row * 128 + ((u ^ (row & 7)) << 4));
-            if (u == 0) p.dump_ids[o] = id0[rr];
           }
+#pragma unroll
+          for (int h = 0; h < 2; ++h)
+            reinterpret_cast<uint4*>(p.dump_kr + o * kRope)[2 * pp + h] = *reinterpret_cast<const uint4*>(
+                cpage + C::KR_OFF + row * 128 + (((2 * pp + h) ^ (row & 7)) << 4));
+          if (pp == 0) p.dump_ids[o] = id0;
         }
         warp_arrive(smem_u32(&bars.empty[slot]));
       } else {
@@ -834,30 +834,24 @@ __global__ void __launch_bounds__(kThreads, 1)
           float* st = reinterpret_cast<float*>(smem + C::OFF_STAT + slot * C::STAT_BYTES);
           // all shared-memory reads of this thread's units first (the in-place
           // stores below would otherwise order every later load behind them)
-          uint4 cv[2][C::NCH];
+          uint4 cv[C::NCH][2];
 #pragma unroll
-          for (int rr = 0; rr < 2; ++rr) {
-            const int row = row0 + rr;
+          for (int fc = 0; fc < C::NCH; ++fc)
 #pragma unroll
-            for (int fc = 0; fc < C::NCH; ++fc)
-              cv[rr][fc] =
-                  *reinterpret_cast<const uint4*>(cpage + fc * C::PCHUNK + row * 128 + ((u ^ (row & 7)) << 4));
-          }
+            for (int h = 0; h < 2; ++h) cv[fc][h] = *reinterpret_cast<const uint4*>(cpage + unit_off(fc, h));
           tr.mark(5, j);
-          float sum1[2], sum2[2];
+          const bool valid = row < t.ntok;
+          float2 s1 = make_float2(0.f, 0.f), s2 = make_float2(0.f, 0.f);
+          float2 a1 = make_float2(0.f, 0.f), a2 = make_float2(0.f, 0.f);
 #pragma unroll
-          for (int rr = 0; rr < 2; ++rr) {
-            const int row = row0 + rr;
-            const bool valid = row < t.ntok;
-            float2 s1 = make_float2(0.f, 0.f), s2 = make_float2(0.f, 0.f);
-            float2 a1 = make_float2(0.f, 0.f), a2 = make_float2(0.f, 0.f);
+          for (int fc = 0; fc < C::NCH; ++fc) {
 #pragma unroll
-            for (int fc = 0; fc < C::NCH; ++fc) {
+            for (int h = 0; h < 2; ++h) {
               uint4 z;
-              z.x = mul_bf16x2(cv[rr][fc].x, gcur[rr][fc].x);
-              z.y = mul_bf16x2(cv[rr][fc].y, gcur[rr][fc].y);
-              z.z = mul_bf16x2(cv[rr][fc].z, gcur[rr][fc].z);
-              z.w = mul_bf16x2(cv[rr][fc].w, gcur[rr][fc].w);
+              z.x = mul_bf16x2(cv[fc][h].x, gcur[fc][h].x);
+              z.y = mul_bf16x2(cv[fc][h].y, gcur[fc][h].y);
+              z.z = mul_bf16x2(cv[fc][h].z, gcur[fc][h].z);
+              z.w = mul_bf16x2(cv[fc][h].w, gcur[fc][h].w);
               if (!full_page && !valid) z = make_uint4(0, 0, 0, 0);
               const float2 f0 = unpack_bf16x2(z.x), f1 = unpack_bf16x2(z.y);
               const float2 f2 = unpack_bf16x2(z.z), f3 = unpack_bf16x2(z.w);
@@ -869,45 +863,35 @@ __global__ void __launch_bounds__(kThreads, 1)
               a2 = __ffma2_rn(f1, f1, a2);
               s2 = __ffma2_rn(f2, f2, s2);
               a2 = __ffma2_rn(f3, f3, a2);
-              *reinterpret_cast<uint4*>(cpage + fc * C::PCHUNK + row * 128 + ((u ^ (row & 7)) << 4)) = z;
+              *reinterpret_cast<uint4*>(cpage + unit_off(fc, h)) = z;
             }
-            s1 = __fadd2_rn(s1, a1);
-            s2 = __fadd2_rn(s2, a2);
-            sum1[rr] = s1.x + s1.y;
-            sum2[rr] = s2.x + s2.y;
           }
+          s1 = __fadd2_rn(s1, a1);
+          s2 = __fadd2_rn(s2, a2);
+          float sum1 = s1.x + s1.y, sum2 = s2.x + s2.y;
           tr.mark(6, j);
-          // row sums over the eight lanes of the quarter-warp
+          // row sums over the four lanes of the row
 #pragma unroll
-          for (int o = 1; o < 8; o <<= 1) {
-#pragma unroll
-            for (int rr = 0; rr < 2; ++rr) {
-              sum1[rr] += __shfl_xor_sync(0xffffffffu, sum1[rr], o);
-              sum2[rr] += __shfl_xor_sync(0xffffffffu, sum2[rr], o);
-            }
+          for (int o = 1; o < 4; o <<= 1) {
+            sum1 += __shfl_xor_sync(0xffffffffu, sum1, o);
+            sum2 += __shfl_xor_sync(0xffffffffu, sum2, o);
           }
-          if (u < 2) {
-            // lane 0 of the quarter-warp publishes row0, lane 1 row0 + 1
-            const int row = row0 + u;
-            const float a = u ? sum1[1] : sum1[0], b2 = u ? sum2[1] : sum2[0];
+          if (pp == 0) {
             constexpr float inv_dc = 1.f / D_C;
-            const float mu = a * inv_dc;
-            const float var = fmaxf(b2 * inv_dc - mu * mu, 0.f);
+            const float mu = sum1 * inv_dc;
+            const float var = fmaxf(sum2 * inv_dc - mu * mu, 0.f);
             const float r = rsqrtf(var + p.eps);
-            const bool valid = row < t.ntok;
             st[row] = valid ? mu : 0.f;
             st[kPage + row] = valid ? r : 0.f;
             st[2 * kPage + row] = valid ? 1.f / r : 0.f;
           }
         } else if (!full_page) {
+          if (row >= t.ntok) {
 #pragma unroll
-          for (int rr = 0; rr < 2; ++rr) {
-            const int row = row0 + rr;
-            if (row >= t.ntok) {
+            for (int fc = 0; fc < C::NCH; ++fc)
 #pragma unroll
-              for (int fc = 0; fc < C::NCH; ++fc)
-                *reinterpret_cast<uint4*>(cpage + fc * C::PCHUNK + row * 128 + (u << 4)) = make_uint4(0, 0, 0, 0);
-            }
+              for (int h = 0; h < 2; ++h)
+                *reinterpret_cast<uint4*>(cpage + unit_off(fc, h)) = make_uint4(0, 0, 0, 0);
           }
         }
         tr.mark(2, j);
@@ -922,12 +906,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       have1 = have2;
       have2 = have2 && w.next(t2);
       if (GATE) {
+        id0 = id1;
+        id1 = id2;
 #pragma unroll
-        for (int rr = 0; rr < 2; ++rr) {
-          id0[rr] = id1[rr];
-          id1[rr] = id2[rr];
-#pragma unroll
-          for (int fc = 0; fc < C::NCH; ++fc) gcur[rr][fc] = gnext[rr][fc];
+        for (int fc = 0; fc < C::NCH; ++fc) {
+          gcur[fc][0] = gnext[fc][0];
+          gcur[fc][1] = gnext[fc][1];
         }
       }
     }

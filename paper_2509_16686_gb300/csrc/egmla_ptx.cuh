@@ -182,6 +182,14 @@ __device__ __forceinline__ uint4 ldg_16_na_hint(const void* p, uint64_t policy) 
   return v;
 }
 
+// 32-byte read-only global load (two 16-byte halves) that skips L1 allocation,
+// with an L2 eviction-priority hint; address 32-byte aligned
+__device__ __forceinline__ void ldg_32_na_hint(const void* p, uint64_t policy, uint4& lo, uint4& hi) {
+  asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.v8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8], %9;"
+               : "=r"(lo.x), "=r"(lo.y), "=r"(lo.z), "=r"(lo.w), "=r"(hi.x), "=r"(hi.y), "=r"(hi.z), "=r"(hi.w)
+               : "l"(reinterpret_cast<uint64_t>(p)), "l"(policy));
+}
+
 __device__ __forceinline__ uint64_t policy_evict_first() {
   uint64_t p;
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
