@@ -107,6 +107,29 @@ def gated_latent(c: np.ndarray, g: np.ndarray, gamma, beta, eps: float) -> np.nd
     return layer_norm(c * g, gamma, beta, eps)
 
 
+def gated_latent_no_norm(c: np.ndarray, g: np.ndarray) -> np.ndarray:
+    """Section 4.4 ablation "remove LayerNorm" (Table 'Ablation on Embedding
+    Gating'): Eq. 5 without its LayerNorm, c~ = c (*) g."""
+    return c * g
+
+
+def gated_latent_added(c: np.ndarray, g: np.ndarray, gamma, beta, eps: float) -> np.ndarray:
+    """Section 4.4 ablation "replace (*) with addition": c~ = LN(c + g)."""
+    return layer_norm(c + g, gamma, beta, eps)
+
+
+def gate_latents(c: np.ndarray, g: np.ndarray, gamma, beta, eps: float, op: str) -> np.ndarray:
+    """The gated latent of gate operation `op`: "mul_ln" (the method, Eq. 5),
+    "mul" or "add_ln" (the two ablations of Section 4.4)."""
+    if op == "mul_ln":
+        return gated_latent(c, g, gamma, beta, eps)
+    if op == "mul":
+        return gated_latent_no_norm(c, g)
+    if op == "add_ln":
+        return gated_latent_added(c, g, gamma, beta, eps)
+    raise ValueError(f"unknown gate operation {op!r}")
+
+
 # --------------------------------------------------------------------------
 # attention for one decode query (Appendix C Eqs. 11-13)
 # --------------------------------------------------------------------------
@@ -129,8 +152,8 @@ def _sequence_latents(case, b: int, gate: bool):
     if gate:
         ids = gather_sequence(id_pool, case.block_table, b, L, d.page_size).astype(np.int64)
         g = widen(case.gate_table, d.dtype)[ids] if L > 0 else np.zeros((0, d.d_c))
-        c_t = gated_latent(c, g, np.asarray(case.ln_gamma, np.float64),
-                           np.asarray(case.ln_beta, np.float64), d.ln_eps)
+        c_t = gate_latents(c, g, np.asarray(case.ln_gamma, np.float64), np.asarray(case.ln_beta, np.float64),
+                           d.ln_eps, getattr(d, "gate_op", "mul_ln"))
     else:
         c_t = c
     return c_t, kr

@@ -58,6 +58,9 @@ class Dims:
     vocab: int
     dtype: str          # "bf16" | "fp32"
     gate: bool = True   # False: plain MLA (gate and LayerNorm off)
+    # with the gate on: "mul_ln" c~ = LN(c (*) g) (the method), or the paper's
+    # ablations "mul" (LayerNorm removed) and "add_ln" ((*) replaced by +)
+    gate_op: str = "mul_ln"
     ln_eps: float = 1e-5
     softmax_scale: float = 0.0   # <= 0 means 1/sqrt(d_nope + d_rope)
 
@@ -248,9 +251,9 @@ def dims_tiny() -> Dims:
                 vocab=1000, dtype="fp32")
 
 
-def dims_bf16(d_c: int = 256, vocab: int = 32000, gate: bool = True) -> Dims:
+def dims_bf16(d_c: int = 256, vocab: int = 32000, gate: bool = True, gate_op: str = "mul_ln") -> Dims:
     return Dims(num_heads=16, d_nope=128, d_rope=64, d_v=128, d_c=d_c, page_size=PAGE_SIZE,
-                vocab=vocab, dtype="bf16", gate=gate)
+                vocab=vocab, dtype="bf16", gate=gate, gate_op=gate_op)
 
 
 def case_tiny(seed: int = 0, **kw) -> Case:

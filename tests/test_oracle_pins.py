@@ -32,9 +32,9 @@ def _rows(name):
 
 
 def small_case(seed=0, dtype="fp32", lens=(37, 64, 1, 130), H=3, dn=8, dr=4, dv=8, dc=16, V=50,
-               P=16, affine=True, gate=True, layout="permuted"):
+               P=16, affine=True, gate=True, layout="permuted", gate_op="mul_ln"):
     dims = synth.Dims(num_heads=H, d_nope=dn, d_rope=dr, d_v=dv, d_c=dc, page_size=P, vocab=V,
-                      dtype=dtype, gate=gate)
+                      dtype=dtype, gate=gate, gate_op=gate_op)
     return synth.make_case("small", dims, list(lens), seed=seed, affine_ln=affine, layout=layout,
                            extra_pages=3)
 
@@ -55,8 +55,14 @@ def torch_reference(case, gate=True):
         if gate:
             g = torch.from_numpy(orc.widen(case.gate_table, d.dtype))[torch.from_numpy(
                 case.logical_ids[b].astype(np.int64))]
-            c = F.layer_norm(c * g, (d.d_c,), weight=torch.from_numpy(case.ln_gamma.astype(np.float64)),
-                             bias=torch.from_numpy(case.ln_beta.astype(np.float64)), eps=d.ln_eps)
+            ln = dict(weight=torch.from_numpy(case.ln_gamma.astype(np.float64)),
+                      bias=torch.from_numpy(case.ln_beta.astype(np.float64)), eps=d.ln_eps)
+            if d.gate_op == "mul_ln":
+                c = F.layer_norm(c * g, (d.d_c,), **ln)
+            elif d.gate_op == "mul":          # ablation: LayerNorm removed
+                c = torch.mul(c, g)
+            else:                             # ablation: (*) replaced by +
+                c = F.layer_norm(torch.add(c, g), (d.d_c,), **ln)
         w_uk = torch.from_numpy(orc.widen(case.w_uk, d.dtype))   # [H, dn, dc]
         w_uv = torch.from_numpy(orc.widen(case.w_uv, d.dtype))
         k_nope = torch.einsum("hnc,lc->hln", w_uk, c)            # [H, L, dn]
@@ -345,6 +351,45 @@ def test_r0_matches_listing_form():
         q = torch.from_numpy(case.q[b].astype(np.float64))[None, :, None, :]
         y = F.scaled_dot_product_attention(q, k.transpose(0, 1)[None], v.transpose(0, 1)[None])
         np.testing.assert_allclose(got[b], y[0, :, 0].numpy(), rtol=1e-11, atol=1e-12)
+
+
+# ---------------------------------------------------------------------------
+# the ablation gate operations (Section 4.4, Table 'Ablation on Embedding Gating')
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("op", ["mul", "add_ln"])
+def test_ablation_gates_match_library_reference(op):
+    case = small_case(seed=21, lens=(37, 64, 1, 130), gate_op=op)
+    np.testing.assert_allclose(orc.decode_unabsorbed(case), torch_reference(case), rtol=1e-11, atol=1e-12)
+    np.testing.assert_allclose(orc.decode_absorbed(case), orc.decode_unabsorbed(case), rtol=1e-11, atol=1e-12)
+
+
+def test_gate_without_norm_of_ones_is_plain_mla():
+    # c (*) 1 = c: the "remove LayerNorm" gate with an all-ones table is MLA
+    case = small_case(seed=22, gate_op="mul")
+    case.gate_table[:] = 1.0
+    np.testing.assert_allclose(orc.decode_unabsorbed(case), orc.decode_unabsorbed(case, gate=False),
+                               rtol=1e-13, atol=1e-13)
+
+
+def test_added_gate_of_zeros_equals_multiplied_gate_of_ones():
+    # LN(c + 0) = LN(c (*) 1): both ablation-free readings reduce to LN(c)
+    a = small_case(seed=23, gate_op="add_ln")
+    b = small_case(seed=23, gate_op="mul_ln")
+    a.gate_table[:] = 0.0
+    b.gate_table[:] = 1.0
+    np.testing.assert_allclose(orc.decode_unabsorbed(a), orc.decode_unabsorbed(b), rtol=1e-13, atol=1e-13)
+
+
+def test_ablation_gates_on_hand_values():
+    # d_c = 4: c = (1, 2, 3, 4), g = (2, 1, 1, 0.5)
+    c, g = np.array([[1.0, 2.0, 3.0, 4.0]]), np.array([[2.0, 1.0, 1.0, 0.5]])
+    np.testing.assert_array_equal(orc.gated_latent_no_norm(c, g), [[2.0, 2.0, 3.0, 2.0]])
+    # c + g = (3, 3, 4, 4.5): mean 29/8, biased variance 27/64
+    got = orc.gated_latent_added(c, g, np.ones(4), np.zeros(4), 0.0)
+    want = (np.array([3.0, 3.0, 4.0, 4.5]) - 29 / 8) / math.sqrt(27 / 64)
+    np.testing.assert_allclose(got[0], want, rtol=1e-14)
+    # c = -g leaves nothing to normalise: LN(0) = beta
+    np.testing.assert_allclose(orc.gated_latent_added(-g, g, np.ones(4), np.full(4, 0.25), 1e-5), 0.25)
 
 
 # ---------------------------------------------------------------------------
