@@ -61,7 +61,9 @@ typedef enum { EG_MLA_BF16 = 0, EG_MLA_FP32 = 1 } eg_mla_dtype;
 
 typedef enum {
   EG_MLA_GATE_NONE = 0,    /* plain MLA: the latent is used as cached (baseline) */
-  EG_MLA_GATE_MUL_LN = 1   /* EG-MLA: c~ = LN(c (*) G[id]) with affine gamma/beta */
+  EG_MLA_GATE_MUL_LN = 1,  /* EG-MLA: c~ = LN(c (*) G[id]) with affine gamma/beta */
+  EG_MLA_GATE_MUL = 2,     /* ablation "remove LayerNorm" (Section 4.4): c~ = c (*) G[id] */
+  EG_MLA_GATE_ADD_LN = 3   /* ablation "replace (*) with addition" (Section 4.4): c~ = LN(c + G[id]) */
 } eg_mla_gate_mode;
 
 /* Shapes of one attention layer.  d_v = value head dim (= d_nope in the paper's
@@ -84,7 +86,7 @@ typedef struct {
 
 /* Supported shapes.
  *   bf16 (tensor-core path): num_heads 16, d_rope 64, page_size 64,
- *        d_c in {192, 256} with either gate mode, d_c 512 with EG_MLA_GATE_NONE;
+ *        d_c in {192, 256} with any gate mode, d_c 512 with EG_MLA_GATE_NONE;
  *        d_nope, d_v multiples of 8 up to 256.
  *   fp32: num_heads <= 16, d_c <= 512 and a multiple of 4, d_rope <= 64,
  *        d_nope, d_v <= 256, page_size 64.
@@ -138,7 +140,9 @@ size_t eg_mla_decode_workspace_size(const eg_mla_dims* dims, int32_t batch, int3
  *
  * For each sequence b and head h, with L_b = seq_lens[b] cached tokens
  * (including the one just appended) and c~_j = LN(c_j (*) G[id_j]) over d_c
- * (EG_MLA_GATE_MUL_LN) or c~_j = c_j (EG_MLA_GATE_NONE):
+ * (EG_MLA_GATE_MUL_LN), c_j (*) G[id_j] (EG_MLA_GATE_MUL), LN(c_j + G[id_j])
+ * (EG_MLA_GATE_ADD_LN) or c~_j = c_j (EG_MLA_GATE_NONE); gamma and beta apply
+ * only with a LayerNorm:
  *   s_j   = scale * (q^_h . c~_j + q^R_h . k^R_j),  q^_h = W_UK,h^T q^C_h   (Eqs. 11-13)
  *   u_b,h = W_UV,h sum_j softmax(s)_j c~_j                                    (Eq. 13, Eq. 6)
  * which equals the paper's per-head attention with k^C = W_UK c~ and

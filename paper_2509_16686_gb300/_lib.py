@@ -33,6 +33,9 @@ EG_MLA_BF16 = 0
 EG_MLA_FP32 = 1
 EG_MLA_GATE_NONE = 0
 EG_MLA_GATE_MUL_LN = 1
+EG_MLA_GATE_MUL = 2      # ablation: LayerNorm removed
+EG_MLA_GATE_ADD_LN = 3   # ablation: (*) replaced by +
+GATE_MODES = {"mul_ln": EG_MLA_GATE_MUL_LN, "mul": EG_MLA_GATE_MUL, "add_ln": EG_MLA_GATE_ADD_LN}
 
 EXPORTED = [
     "eg_mla_append_latent",
@@ -148,10 +151,12 @@ def _stream(stream) -> int:
 
 
 def make_dims(num_heads, d_nope, d_rope, d_v, d_c, vocab, dtype="bf16", gate=True, page_size=64,
-              softmax_scale=0.0, ln_eps=1e-5) -> EgMlaDims:
+              softmax_scale=0.0, ln_eps=1e-5, gate_op="mul_ln") -> EgMlaDims:
+    """gate False: plain MLA; gate True: gate operation `gate_op` ("mul_ln",
+    or the ablations "mul" and "add_ln")."""
     return EgMlaDims(num_heads, d_nope, d_rope, d_v, d_c, page_size, vocab,
                      EG_MLA_BF16 if dtype == "bf16" else EG_MLA_FP32,
-                     EG_MLA_GATE_MUL_LN if gate else EG_MLA_GATE_NONE, softmax_scale, ln_eps)
+                     GATE_MODES[gate_op] if gate else EG_MLA_GATE_NONE, softmax_scale, ln_eps)
 
 
 def eg_mla_default_num_splits() -> int:

@@ -30,7 +30,7 @@ int check_dims(const eg_mla_dims* d) {
   if (d->num_heads <= 0 || d->d_nope <= 0 || d->d_rope <= 0 || d->d_v <= 0 || d->d_c <= 0 ||
       d->page_size <= 0 || d->vocab <= 0)
     return EG_MLA_ERR_INVALID_ARG;
-  if (d->gate_mode != EG_MLA_GATE_NONE && d->gate_mode != EG_MLA_GATE_MUL_LN) return EG_MLA_ERR_INVALID_ARG;
+  if (d->gate_mode < EG_MLA_GATE_NONE || d->gate_mode > EG_MLA_GATE_ADD_LN) return EG_MLA_ERR_INVALID_ARG;
   if (d->page_size != egmla::kPage) return EG_MLA_ERR_UNSUPPORTED;
   if (d->dtype == EG_MLA_BF16) {
     if (d->num_heads != 16 || d->d_rope != 64) return EG_MLA_ERR_UNSUPPORTED;
@@ -136,12 +136,12 @@ int fill_decode_args(DecodeArgs& a, const eg_mla_dims* d, const void* c_pool, co
   if (static_cast<int64_t>(num_pages) * d->page_size > INT32_MAX) return EG_MLA_ERR_UNSUPPORTED;
   if (c_pool == nullptr || krope_pool == nullptr || block_table == nullptr || seq_lens == nullptr)
     return EG_MLA_ERR_INVALID_ARG;
-  if (d->gate_mode == EG_MLA_GATE_MUL_LN && (id_pool == nullptr || gate_table == nullptr))
+  if (d->gate_mode != EG_MLA_GATE_NONE && (id_pool == nullptr || gate_table == nullptr))
     return EG_MLA_ERR_INVALID_ARG;
   // the bf16 kernels read gate rows in 32-byte pieces
   const size_t g_align = is_tc_path(d) ? 32 : 16;
   if (!aligned(c_pool, 16) || !aligned(krope_pool, 16) || (id_pool && !aligned(id_pool, 16)) ||
-      (gate_table && d->gate_mode == EG_MLA_GATE_MUL_LN && !aligned(gate_table, g_align)))
+      (gate_table && d->gate_mode != EG_MLA_GATE_NONE && !aligned(gate_table, g_align)))
     return EG_MLA_ERR_INVALID_ARG;
   int32_t splits = 0;
   rc = resolve_splits(num_splits, &splits);
@@ -158,7 +158,9 @@ int fill_decode_args(DecodeArgs& a, const eg_mla_dims* d, const void* c_pool, co
   a.page_size = d->page_size;
   a.vocab = d->vocab;
   a.dtype = d->dtype;
-  a.gate = d->gate_mode == EG_MLA_GATE_MUL_LN ? 1 : 0;
+  a.gate = d->gate_mode != EG_MLA_GATE_NONE ? 1 : 0;
+  a.gate_add = d->gate_mode == EG_MLA_GATE_ADD_LN ? 1 : 0;
+  a.gate_ln = (d->gate_mode == EG_MLA_GATE_MUL_LN || d->gate_mode == EG_MLA_GATE_ADD_LN) ? 1 : 0;
   a.scale_log2 = resolve_scale(d) * 1.4426950408889634f;
   a.eps = d->ln_eps > 0.f ? d->ln_eps : 1e-5f;
   a.c_pool = c_pool;
@@ -281,7 +283,7 @@ int eg_mla_kv_bytes_per_token(const eg_mla_dims* dims, int32_t n_layers, int64_t
   if (dims == nullptr || bytes_out == nullptr || n_layers < 0) return EG_MLA_ERR_INVALID_ARG;
   if (dims->d_c <= 0 || dims->d_rope < 0) return EG_MLA_ERR_INVALID_ARG;
   const int64_t per_layer = static_cast<int64_t>(dims->d_c + dims->d_rope) * elem_bytes(dims) +
-                            (dims->gate_mode == EG_MLA_GATE_MUL_LN ? 4 : 0);
+                            (dims->gate_mode != EG_MLA_GATE_NONE ? 4 : 0);
   *bytes_out = per_layer * n_layers;
   return EG_MLA_OK;
 }
@@ -451,7 +453,7 @@ int eg_mla_debug_gather(const eg_mla_dims* dims, const void* c_pool, const void*
                         const void* gate_table, void* c_out, void* kr_out, int32_t* ids_out, void* g_out,
                         int32_t num_splits, void* workspace, size_t workspace_bytes, int32_t* dev_status,
                         void* stream) {
-  if (dims == nullptr || dims->dtype != EG_MLA_BF16 || dims->gate_mode != EG_MLA_GATE_MUL_LN ||
+  if (dims == nullptr || dims->dtype != EG_MLA_BF16 || dims->gate_mode == EG_MLA_GATE_NONE ||
       (dims->d_c != 192 && dims->d_c != 256))
     return EG_MLA_ERR_UNSUPPORTED;
   DecodeArgs a;

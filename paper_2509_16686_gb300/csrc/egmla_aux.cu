@@ -430,7 +430,8 @@ decode_f32_kernel(const float* __restrict__ c_pool, const float* __restrict__ kr
                   const float* __restrict__ gate_table, const float* __restrict__ gamma,
                   const float* __restrict__ beta, const uint8_t* __restrict__ qprep, size_t qstride,
                   const int32_t* __restrict__ cu, float* __restrict__ part_ml, float* __restrict__ part_o,
-                  int H, int d_c, int d_rope, int vocab, int gate, float scale_log2, float eps,
+                  int H, int d_c, int d_rope, int vocab, int gate, int gate_add, int gate_ln, float scale_log2,
+                  float eps,
                   int32_t* status) {
   extern __shared__ float sm[];
   float* qh = sm;                               // [H][d_c]
@@ -475,12 +476,15 @@ decode_f32_kernel(const float* __restrict__ c_pool, const float* __restrict__ kr
       float s1 = 0.f;
       for (int f = threadIdx.x; f < d_c; f += blockDim.x) {
         float z = c_pool[row * d_c + f];
-        if (gate) z *= gate_table[static_cast<size_t>(id) * d_c + f];
+        if (gate) {
+          const float g = gate_table[static_cast<size_t>(id) * d_c + f];
+          z = gate_add ? z + g : z * g;
+        }
         ct[f] = z;
         s1 += z;
       }
       for (int r = threadIdx.x; r < d_rope; r += blockDim.x) krs[r] = kr_pool[row * d_rope + r];
-      if (gate) {
+      if (gate && gate_ln) {
         const float mean = block_sum_128(s1, red, 0) / d_c;
         float s2 = 0.f;
         for (int f = threadIdx.x; f < d_c; f += blockDim.x) {
@@ -543,8 +547,8 @@ cudaError_t launch_prologue_tc(const DecodeArgs& a, cudaStream_t st) {
   const WorkspaceLayout wl = workspace_layout(a.batch, a.num_splits, 16, a.d_c, a.d_rope, true);
   uint8_t* ws = static_cast<uint8_t*>(a.workspace);
   // with the gate off the latent is used as cached: no LayerNorm affine to fold into q^
-  const float* gamma = a.gate ? a.ln_gamma : nullptr;
-  const float* beta = a.gate ? a.ln_beta : nullptr;
+  const float* gamma = a.gate && a.gate_ln ? a.ln_gamma : nullptr;
+  const float* beta = a.gate && a.gate_ln ? a.ln_beta : nullptr;
   const int ngroups = (a.batch + kPBatch - 1) / kPBatch;
   prologue_tc_kernel<<<16 * (a.d_c / kSumFeatures) * ngroups + 1, 256, 0, st>>>(
       static_cast<const __nv_bfloat16*>(a.q), static_cast<const __nv_bfloat16*>(a.w_uk), gamma, beta,
@@ -572,7 +576,7 @@ cudaError_t launch_decode_f32(const DecodeArgs& a, cudaStream_t st) {
       a.max_pages, a.seq_lens, a.batch, a.num_pages, static_cast<const float*>(a.gate_table), a.ln_gamma,
       a.ln_beta, ws + wl.off_qprep, wl.qprep_stride, reinterpret_cast<const int32_t*>(ws + wl.off_cu),
       reinterpret_cast<float*>(ws + wl.off_ml), reinterpret_cast<float*>(ws + wl.off_o), a.H, a.d_c, a.d_rope,
-      a.vocab, a.gate, a.scale_log2, a.eps, a.status);
+      a.vocab, a.gate, a.gate_add, a.gate_ln, a.scale_log2, a.eps, a.status);
   return cudaGetLastError();
 }
 

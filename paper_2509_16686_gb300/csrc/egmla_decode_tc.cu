@@ -485,10 +485,14 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&z);
 }
 
-template <int D_C, bool GATE, bool DUMP>
+// GM: gate mode (0 none, 1 LN(c (*) g), 2 c (*) g, 3 LN(c + g): eg_mla_gate_mode)
+template <int D_C, int GM, bool DUMP>
 __global__ void __launch_bounds__(kThreads, 1)
     decode_tc_kernel(const __grid_constant__ CUtensorMap cmap, const __grid_constant__ CUtensorMap krmap,
                      const TcParams p) {
+  constexpr bool GATE = GM != 0;
+  constexpr bool GATE_ADD = GM == 3;             // ablation: c + g
+  constexpr bool GATE_LN = GM == 1 || GM == 3;   // LayerNorm after the gate
   using C = Cfg<D_C, GATE>;
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte aligned base (128-byte swizzle atoms); derived by an offset from the
@@ -759,6 +763,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int pp = lane & 3;
     const int row = 2 * (gw * 4 + (lane >> 3)) + ((lane >> 2) & 1);
     const uint64_t pol_keep = policy_evict_last();
+    constexpr bool gate_ln = GATE_LN;
     Walker w;
     w.start(p.cu, p.seq_lens, p.batch);
     PageWindow pw;
@@ -841,49 +846,108 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int h = 0; h < 2; ++h) cv[fc][h] = *reinterpret_cast<const uint4*>(cpage + unit_off(fc, h));
           tr.mark(5, j);
           const bool valid = row < t.ntok;
-          float2 s1 = make_float2(0.f, 0.f), s2 = make_float2(0.f, 0.f);
-          float2 a1 = make_float2(0.f, 0.f), a2 = make_float2(0.f, 0.f);
+          if constexpr (GATE_ADD) {
+            // ablation LN(c + g): c + g is exact in fp32; the row is centred by its
+            // mean before the bf16 rounding (LN is shift-invariant), so the rounding
+            // error is relative to the spread LN keeps, not to the gate's offset
+            float2 s1 = make_float2(0.f, 0.f), s2 = make_float2(0.f, 0.f);
 #pragma unroll
-          for (int fc = 0; fc < C::NCH; ++fc) {
+            for (int fc = 0; fc < C::NCH; ++fc) {
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-              uint4 z;
-              z.x = mul_bf16x2(cv[fc][h].x, gcur[fc][h].x);
-              z.y = mul_bf16x2(cv[fc][h].y, gcur[fc][h].y);
-              z.z = mul_bf16x2(cv[fc][h].z, gcur[fc][h].z);
-              z.w = mul_bf16x2(cv[fc][h].w, gcur[fc][h].w);
-              if (!full_page && !valid) z = make_uint4(0, 0, 0, 0);
-              const float2 f0 = unpack_bf16x2(z.x), f1 = unpack_bf16x2(z.y);
-              const float2 f2 = unpack_bf16x2(z.z), f3 = unpack_bf16x2(z.w);
-              s1 = __fadd2_rn(s1, f0);
-              a1 = __fadd2_rn(a1, f1);
-              s1 = __fadd2_rn(s1, f2);
-              a1 = __fadd2_rn(a1, f3);
-              s2 = __ffma2_rn(f0, f0, s2);
-              a2 = __ffma2_rn(f1, f1, a2);
-              s2 = __ffma2_rn(f2, f2, s2);
-              a2 = __ffma2_rn(f3, f3, a2);
-              *reinterpret_cast<uint4*>(cpage + unit_off(fc, h)) = z;
+              for (int h = 0; h < 2; ++h) {
+                const uint32_t* cw = reinterpret_cast<const uint32_t*>(&cv[fc][h]);
+                const uint32_t* gw2 = reinterpret_cast<const uint32_t*>(&gcur[fc][h]);
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                  const float2 zf = __fadd2_rn(unpack_bf16x2(cw[k]), unpack_bf16x2(gw2[k]));
+                  s1 = __fadd2_rn(s1, zf);
+                  s2 = __ffma2_rn(zf, zf, s2);
+                }
+              }
             }
-          }
-          s1 = __fadd2_rn(s1, a1);
-          s2 = __fadd2_rn(s2, a2);
-          float sum1 = s1.x + s1.y, sum2 = s2.x + s2.y;
-          tr.mark(6, j);
-          // row sums over the four lanes of the row
+            float sum1 = s1.x + s1.y, sum2 = s2.x + s2.y;
 #pragma unroll
-          for (int o = 1; o < 4; o <<= 1) {
-            sum1 += __shfl_xor_sync(0xffffffffu, sum1, o);
-            sum2 += __shfl_xor_sync(0xffffffffu, sum2, o);
-          }
-          if (pp == 0) {
+            for (int o = 1; o < 4; o <<= 1) {
+              sum1 += __shfl_xor_sync(0xffffffffu, sum1, o);
+              sum2 += __shfl_xor_sync(0xffffffffu, sum2, o);
+            }
             constexpr float inv_dc = 1.f / D_C;
             const float mu = sum1 * inv_dc;
             const float var = fmaxf(sum2 * inv_dc - mu * mu, 0.f);
             const float r = rsqrtf(var + p.eps);
-            st[row] = valid ? mu : 0.f;
-            st[kPage + row] = valid ? r : 0.f;
-            st[2 * kPage + row] = valid ? 1.f / r : 0.f;
+            const float2 mu2v = make_float2(mu, mu);
+#pragma unroll
+            for (int fc = 0; fc < C::NCH; ++fc) {
+#pragma unroll
+              for (int h = 0; h < 2; ++h) {
+                const uint32_t* cw = reinterpret_cast<const uint32_t*>(&cv[fc][h]);
+                const uint32_t* gw2 = reinterpret_cast<const uint32_t*>(&gcur[fc][h]);
+                uint4 z;
+                uint32_t* zw = reinterpret_cast<uint32_t*>(&z);
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                  const float2 zf = __fadd2_rn(__fadd2_rn(unpack_bf16x2(cw[k]), unpack_bf16x2(gw2[k])),
+                                               make_float2(-mu2v.x, -mu2v.y));
+                  zw[k] = pack_bf16x2(zf.x, zf.y);
+                }
+                if (!full_page && !valid) z = make_uint4(0, 0, 0, 0);
+                *reinterpret_cast<uint4*>(cpage + unit_off(fc, h)) = z;
+              }
+            }
+            tr.mark(6, j);
+            if (pp == 0) {
+              st[row] = 0.f;   // the stored z is centred
+              st[kPage + row] = valid ? r : 0.f;
+              st[2 * kPage + row] = valid ? 1.f / r : 0.f;
+            }
+          } else {
+            float2 s1 = make_float2(0.f, 0.f), s2 = make_float2(0.f, 0.f);
+            float2 a1 = make_float2(0.f, 0.f), a2 = make_float2(0.f, 0.f);
+#pragma unroll
+            for (int fc = 0; fc < C::NCH; ++fc) {
+#pragma unroll
+              for (int h = 0; h < 2; ++h) {
+                uint4 z;
+                z.x = mul_bf16x2(cv[fc][h].x, gcur[fc][h].x);
+                z.y = mul_bf16x2(cv[fc][h].y, gcur[fc][h].y);
+                z.z = mul_bf16x2(cv[fc][h].z, gcur[fc][h].z);
+                z.w = mul_bf16x2(cv[fc][h].w, gcur[fc][h].w);
+                if (!full_page && !valid) z = make_uint4(0, 0, 0, 0);
+                const float2 f0 = unpack_bf16x2(z.x), f1 = unpack_bf16x2(z.y);
+                const float2 f2 = unpack_bf16x2(z.z), f3 = unpack_bf16x2(z.w);
+                s1 = __fadd2_rn(s1, f0);
+                a1 = __fadd2_rn(a1, f1);
+                s1 = __fadd2_rn(s1, f2);
+                a1 = __fadd2_rn(a1, f3);
+                s2 = __ffma2_rn(f0, f0, s2);
+                a2 = __ffma2_rn(f1, f1, a2);
+                s2 = __ffma2_rn(f2, f2, s2);
+                a2 = __ffma2_rn(f3, f3, a2);
+                *reinterpret_cast<uint4*>(cpage + unit_off(fc, h)) = z;
+              }
+            }
+            s1 = __fadd2_rn(s1, a1);
+            s2 = __fadd2_rn(s2, a2);
+            float sum1 = s1.x + s1.y, sum2 = s2.x + s2.y;
+            tr.mark(6, j);
+            // row sums over the four lanes of the row (without the LayerNorm
+            // ablation's norm: mu = 0, r = 1)
+            if (gate_ln) {
+#pragma unroll
+              for (int o = 1; o < 4; o <<= 1) {
+                sum1 += __shfl_xor_sync(0xffffffffu, sum1, o);
+                sum2 += __shfl_xor_sync(0xffffffffu, sum2, o);
+              }
+            }
+            if (pp == 0) {
+              constexpr float inv_dc = 1.f / D_C;
+              const float mu = gate_ln ? sum1 * inv_dc : 0.f;
+              const float var = fmaxf(sum2 * inv_dc - mu * mu, 0.f);
+              const float r = gate_ln ? rsqrtf(var + p.eps) : 1.f;
+              st[row] = valid ? mu : 0.f;
+              st[kPage + row] = valid ? r : 0.f;
+              st[2 * kPage + row] = valid ? 1.f / r : 0.f;
+            }
           }
         } else if (!full_page) {
           if (row >= t.ntok) {
@@ -1143,10 +1207,10 @@ int resident_ctas(K kern, uint32_t smem) {
   return cached[dev];
 }
 
-template <int D_C, bool GATE, bool DUMP>
+template <int D_C, int GM, bool DUMP>
 cudaError_t launch_one(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_t st, bool* fused) {
-  using C = Cfg<D_C, GATE>;
-  auto kern = decode_tc_kernel<D_C, GATE, DUMP>;
+  using C = Cfg<D_C, GM != 0>;
+  auto kern = decode_tc_kernel<D_C, GM, DUMP>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
   if (e != cudaSuccess) return e;
   const WorkspaceLayout wl = workspace_layout(a.batch, a.num_splits, kHeads, D_C, kRope, true);
@@ -1156,8 +1220,10 @@ cudaError_t launch_one(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_
   p.block_table = a.block_table;
   p.seq_lens = a.seq_lens;
   p.gate_table = static_cast<const __nv_bfloat16*>(a.gate_table);
-  p.gamma = a.ln_gamma;
-  p.beta = a.ln_beta;
+  // gamma and beta belong to the LayerNorm (none in the "remove LayerNorm" ablation)
+  p.gamma = a.gate_ln ? a.ln_gamma : nullptr;
+  p.beta = a.gate_ln ? a.ln_beta : nullptr;
+
   p.qprep = ws + wl.off_qprep;
   p.cu = reinterpret_cast<const int32_t*>(ws + wl.off_cu);
   p.part_ml = reinterpret_cast<float*>(ws + wl.off_ml);
@@ -1213,23 +1279,29 @@ bool tc_supported(int d_c, int gate) {
   return d_c == 192 || d_c == 256 || d_c == 512;
 }
 
+// d_c-dispatch of one gate mode
+template <int GM>
+cudaError_t launch_mode(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_t st, bool* fused) {
+  if (a.d_c == 192) return launch_one<192, GM, false>(a, maps, st, fused);
+  if (a.d_c == 256) return launch_one<256, GM, false>(a, maps, st, fused);
+  return cudaErrorInvalidValue;
+}
+
 cudaError_t launch_decode_tc(const DecodeArgs& a, const CUtensorMap* maps, bool dump, cudaStream_t st,
                              bool* fused) {
   if (fused) *fused = false;
-  if (dump) {
-    if (a.d_c == 192) return launch_one<192, true, true>(a, maps, st, nullptr);
-    if (a.d_c == 256) return launch_one<256, true, true>(a, maps, st, nullptr);
+  if (dump) {   // cache-read test entry: the raw page and gate rows
+    if (a.d_c == 192) return launch_one<192, 1, true>(a, maps, st, nullptr);
+    if (a.d_c == 256) return launch_one<256, 1, true>(a, maps, st, nullptr);
     return cudaErrorInvalidValue;
   }
-  if (a.gate) {
-    if (a.d_c == 192) return launch_one<192, true, false>(a, maps, st, fused);
-    if (a.d_c == 256) return launch_one<256, true, false>(a, maps, st, fused);
-  } else {
-    if (a.d_c == 192) return launch_one<192, false, false>(a, maps, st, fused);
-    if (a.d_c == 256) return launch_one<256, false, false>(a, maps, st, fused);
+  if (!a.gate) {
     if (a.d_c == 512) return launch_decode_wide(a, maps, st);
+    return launch_mode<0>(a, maps, st, fused);
   }
-  return cudaErrorInvalidValue;
+  if (a.gate_add) return launch_mode<3>(a, maps, st, fused);
+  if (a.gate_ln) return launch_mode<1>(a, maps, st, fused);
+  return launch_mode<2>(a, maps, st, fused);
 }
 
 }  // namespace egmla

@@ -31,7 +31,9 @@ struct DecodeArgs {
   // shapes
   int H, d_nope, d_rope, d_v, d_c, page_size, vocab;
   int dtype;  // 0 bf16, 1 fp32
-  int gate;   // 0 none, 1 mul+LN
+  int gate;      // 0 none, 1 gated (the three gate modes below)
+  int gate_add;  // gate by c + g (EG_MLA_GATE_ADD_LN) instead of c (*) g
+  int gate_ln;   // LayerNorm after the gate (EG_MLA_GATE_MUL_LN, EG_MLA_GATE_ADD_LN)
   float scale_log2;  // softmax scale * log2(e)
   float eps;
   // tensors

@@ -88,7 +88,8 @@ class DeviceCase:
 def dims_of(case: Case) -> _lib.EgMlaDims:
     d = case.dims
     return _lib.make_dims(d.num_heads, d.d_nope, d.d_rope, d.d_v, d.d_c, d.vocab, dtype=d.dtype, gate=d.gate,
-                          page_size=d.page_size, softmax_scale=d.softmax_scale, ln_eps=d.ln_eps)
+                          page_size=d.page_size, softmax_scale=d.softmax_scale, ln_eps=d.ln_eps,
+                          gate_op=getattr(d, "gate_op", "mul_ln"))
 
 
 def upload(case: Case, device="cuda", num_splits: int = 0) -> DeviceCase:

@@ -6,6 +6,8 @@ the token-id gate gather bit-exact.  Small cases are compared element by element
 in full; the full-size workloads are compared on sampled sequences (every head)
 in the same launch configuration the bench uses (default split count).
 """
+import dataclasses
+
 import numpy as np
 import pytest
 import torch
@@ -82,6 +84,29 @@ def test_bf16_small_matches_oracle(gpu_lib, d_c, lens):
     for splits in (1, 2, 7):
         _, got = run(case, splits)
         check_bf16(got, ref, f"d_c={d_c} lens={lens} splits={splits}", scaled_abs=min(lens) < 128)
+
+
+# --------------------------------------------------------------------------- gating ablations (Section 4.4)
+@pytest.mark.parametrize("op", ["mul", "add_ln"])
+@pytest.mark.parametrize("d_c", [256, 192])
+def test_bf16_ablation_gates_match_oracle(gpu_lib, op, d_c):
+    dims = synth.dims_bf16(d_c=d_c, vocab=3000, gate=True, gate_op=op)
+    case = synth.make_case("ablation", dims, [5, 64, 130, 700], seed=31, latent_scale=0.5, layout="permuted",
+                           affine_ln=True, extra_pages=5)
+    ref = orc.decode_unabsorbed(case)
+    for splits in (3, 0):
+        _, got = run(case, splits)
+        check_bf16(got, ref, f"{op} d_c={d_c} splits={splits}", scaled_abs=True)
+
+
+@pytest.mark.parametrize("op", ["mul", "add_ln"])
+def test_fp32_ablation_gates_match_oracle(gpu_lib, op):
+    dims = dataclasses.replace(synth.dims_tiny(), gate_op=op)
+    case = synth.make_case("f32-ablation", dims, [1, 63, 130], seed=32, affine_ln=True, layout="permuted",
+                           extra_pages=2)
+    for splits in (1, 3):
+        _, got = run(case, splits)
+        assert rel_l2(got, orc.decode_unabsorbed(case)) <= F32_REL_L2
 
 
 def test_bf16_mla_gate_off_matches_oracle(gpu_lib):
