@@ -141,6 +141,17 @@ def test_split_count_invariance(gpu_lib):
         assert np.abs(o - outs[0]).max() <= 4e-3
 
 
+def test_one_long_sequence_over_every_split(gpu_lib):
+    # batch 1 x 256 pages over the default one split per SM: every split holds
+    # a piece of the one sequence, so the split merge takes more than 32
+    # partials per (sequence, head) (its online rescaling across groups of 32)
+    case = small_bf16((16384,), seed=41)
+    ref = orc.decode_unabsorbed(case)
+    for splits in (0, 48):
+        _, got = run(case, splits)
+        check_bf16(got, ref, f"long sequence splits={splits}", scaled_abs=True)
+
+
 def test_page_pool_permutation_is_bit_stable(gpu_lib):
     case = small_bf16((300, 129))
     _, a = run(case, 3)
