@@ -76,8 +76,6 @@ constexpr float kLazyLog2 = 8.f;
 template <int D_C, bool GATE>
 struct Cfg {
   static constexpr int NCH = D_C / 64;                  // 64-feature swizzle-atom columns
-  static constexpr int UNITS = D_C / 8;                 // 16-byte units of a latent row
-  static constexpr int NU = UNITS / 4;                  // units per gate thread
   static constexpr uint32_t PCHUNK = kPage * 128;       // one atom column of a page: 8 KB
   static constexpr uint32_t KR_OFF = NCH * PCHUNK;
   static constexpr uint32_t SLOT = KR_OFF + PCHUNK;     // latent + RoPE key of one page
