@@ -110,6 +110,22 @@ def dist_env():
     return ws, rank, local
 
 
+def max_over_ranks(ms, dist, device):
+    """The slowest rank's time (every rank gets it); `ms` itself without a process group."""
+    if dist is None:
+        return ms
+    import torch
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(world_size, batch, steps, ms):
+    """Decode tokens/s of the whole job: every rank decodes `batch` sequences per
+    step (weak scaling), `steps` steps in `ms` milliseconds (the slowest rank's)."""
+    return world_size * batch * steps / (ms / 1e3)
+
+
 # ----------------------------------------------------------------------------- clocks
 class ClockSampler:
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -345,14 +361,10 @@ def run_gpu(args, workload, torch, dist, ws, rank):
         torch.cuda.synchronize()
         if dist:
             dist.barrier()
-    elapsed_ms = ev0.elapsed_time(ev1)
-    if dist:
-        t = torch.tensor([elapsed_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
+    elapsed_ms = max_over_ranks(ev0.elapsed_time(ev1), dist, "cuda")
     assert units[0].read_status() == 0, "device status after timed region"
     ms_per_step = elapsed_ms / steps
-    value = ws * B * steps / (elapsed_ms / 1e3)
+    value = whole_job_rate(ws, B, steps, elapsed_ms)
 
     # ---- the decode kernel alone: CUDA events around every decode launch,
     # recorded as nodes of a captured graph of the same steps (so that each
@@ -430,12 +442,8 @@ def run_gpu(args, workload, torch, dist, ws, rank):
     stream.wait_stream(s_copy)
     e1.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1)
-    if dist:
-        t = torch.tensor([e2e_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
-    e2e_value = ws * B * e2e_steps / (e2e_ms / 1e3)
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), dist, "cuda")
+    e2e_value = whole_job_rate(ws, B, e2e_steps, e2e_ms)
     assert units[0].read_status() == 0, "device status after end-to-end run"
 
     # ---- CPU baseline (rank 0, N = 1 only); a decode token passes every layer
