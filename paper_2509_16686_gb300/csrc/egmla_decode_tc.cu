@@ -88,12 +88,16 @@ struct Cfg {
   static constexpr uint32_t PBUF = kPage / 8 * kQGroupBytes;
   static constexpr uint32_t STAT_BYTES = 3 * kPage * 4;   // per slot: mu[64], r[64], 1/r[64]
   static constexpr uint32_t MISC = 1024;
-  static constexpr int NS_FIT = (int)((kSmemLimit - 1024 - 2 * QBUF - 2 * PBUF - MISC) / (SLOT + STAT_BYTES));
+  // LayerNorm gamma and beta of the segment read-out, one copy per softmax warp
+  static constexpr uint32_t GB_BYTES = 2 * D_C * 4;
+  static constexpr int NS_FIT =
+      (int)((kSmemLimit - 1024 - 2 * QBUF - 2 * PBUF - 2 * GB_BYTES - MISC) / (SLOT + STAT_BYTES));
   static constexpr int NS = NS_FIT > 6 ? 6 : NS_FIT;
   static constexpr uint32_t OFF_QBUF = NS * SLOT;
   static constexpr uint32_t OFF_PBUF = OFF_QBUF + 2 * QBUF;
   static constexpr uint32_t OFF_STAT = OFF_PBUF + 2 * PBUF;
-  static constexpr uint32_t OFF_MISC = OFF_STAT + NS * STAT_BYTES;
+  static constexpr uint32_t OFF_GB = OFF_STAT + NS * STAT_BYTES;
+  static constexpr uint32_t OFF_MISC = OFF_GB + 2 * GB_BYTES;
   static constexpr uint32_t SMEM = OFF_MISC + MISC + 1024;
   // TMEM columns: two score buffers of (latent 64 + RoPE 64) token columns, then
   // the latent output (d_c columns), rows = heads
@@ -151,25 +155,41 @@ struct TcParams {
   int fuse;
 };
 
-// Trace recorder of one role of one CTA (a no-op unless tracing is on).
-struct Tracer {
+// Trace recorder of one role of one CTA.  Only the trace instantiation of the
+// kernel records (ON); in the others every call compiles to nothing, since even
+// untaken trace stores in the loops cost registers and instruction-cache room.
+template <bool ON>
+struct TracerT {
   unsigned long long* base;
   int n, cap;
   __device__ void init(const TcParams& p, int role) {
     base = nullptr;
     n = 0;
     cap = p.trace_cap;
-    if (p.trace != nullptr && static_cast<int>(blockIdx.x) < p.trace_ctas)
+    if (ON && p.trace != nullptr && static_cast<int>(blockIdx.x) < p.trace_ctas)
       base = p.trace + (static_cast<size_t>(blockIdx.x) * kTraceRoles + role) * p.trace_cap * 2;
   }
   __device__ __forceinline__ void mark(int event, int tile) {
-    if (base != nullptr && n < cap) {
-      base[2 * n] = (static_cast<unsigned long long>(event) << 24) | static_cast<unsigned>(tile & 0xffffff);
+    if (ON && base != nullptr && n < cap) {
+      base[2 * n] = (static_cast<unsigned long long>(event) << 56) |
+                    (static_cast<unsigned long long>(tile & 0xffffff) << 32) |
+                    static_cast<uint32_t>(globaltimer());
       base[2 * n + 1] = clock64();
       ++n;
     }
   }
 };
+
+// Kernel phase `event` of this CTA into entry `event` of trace role 4 (thread 0;
+// stateless, so that nothing stays live across the kernel for it).
+template <bool ON>
+__device__ __forceinline__ void phase_mark(const TcParams& p, int event) {
+  if (ON && p.trace != nullptr && threadIdx.x == 0 && static_cast<int>(blockIdx.x) < p.trace_ctas && event < p.trace_cap) {
+    unsigned long long* e = p.trace + ((static_cast<size_t>(blockIdx.x) * kTraceRoles + 4) * p.trace_cap + event) * 2;
+    e[0] = (static_cast<unsigned long long>(event) << 56) | static_cast<uint32_t>(globaltimer());
+    e[1] = clock64();
+  }
+}
 
 // shared-memory barrier block (inside MISC)
 struct Bars {
@@ -484,10 +504,14 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 }
 
 // GM: gate mode (0 none, 1 LN(c (*) g), 2 c (*) g, 3 LN(c + g): eg_mla_gate_mode)
-template <int D_C, int GM, bool DUMP>
+// DBG: 0 the decode, 1 the cache-read dump (raw pages and gate rows, no
+// attention), 2 the decode with the pipeline trace
+template <int D_C, int GM, int DBG>
 __global__ void __launch_bounds__(kThreads, 1)
     decode_tc_kernel(const __grid_constant__ CUtensorMap cmap, const __grid_constant__ CUtensorMap krmap,
                      const TcParams p) {
+  constexpr bool DUMP = DBG == 1;
+  using Tracer = TracerT<DBG == 2>;
   constexpr bool GATE = GM != 0;
   constexpr bool GATE_ADD = GM == 3;             // ablation: c + g
   constexpr bool GATE_LN = GM == 1 || GM == 3;   // LayerNorm after the gate
@@ -501,6 +525,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int* abort_flag = &bars.abort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  phase_mark<DBG == 2>(p, 0);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::NS; ++s) {
@@ -533,6 +558,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  phase_mark<DBG == 2>(p, 1);
   const uint32_t tmem = bars.tmem_base;
 
   constexpr uint32_t KSTEP = 2 * kQGroupBytes;   // bytes of 16 columns of an A operand
@@ -992,6 +1018,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     // accumulator, l and the mean correction) when a tile's max exceeds it by
     // more than 2^kLazyLog2; otherwise the weights stay below 2^kLazyLog2.
     float m_ref = 0.f, l_acc = 0.f, bmu_acc = 0.f, wq = 0.f, bsc = 0.f;
+    // this warp's copy of gamma and beta (identity without a LayerNorm), so that
+    // the segment read-out waits on no global load
+    float* gb = reinterpret_cast<float*>(smem + C::OFF_GB + hw * C::GB_BYTES);
+    if (GATE) {
+      for (int f = lane; f < D_C; f += 32) {
+        gb[f] = p.gamma ? __ldg(p.gamma + f) : 1.f;
+        gb[D_C + f] = p.beta ? __ldg(p.beta + f) : 0.f;
+      }
+      __syncwarp();
+    }
     Walker w;
     w.start(p.cu, p.seq_lens, p.batch);
     Tile t;
@@ -1161,9 +1197,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int f = 64 * c + 8 * k + 2 * qq;
             float2 v = make_float2(o[4 * k], o[4 * k + 1]);
             if (GATE) {
-              float2 gm = make_float2(1.f, 1.f), bt = make_float2(0.f, 0.f);
-              if (p.gamma) gm = __ldg(reinterpret_cast<const float2*>(p.gamma + f));
-              if (p.beta) bt = __ldg(reinterpret_cast<const float2*>(p.beta + f));
+              const float2 gm = *reinterpret_cast<const float2*>(gb + f);
+              const float2 bt = *reinterpret_cast<const float2*>(gb + D_C + f);
               v.x = fmaf(gm.x, v.x - bh, bt.x * lh);
               v.y = fmaf(gm.y, v.y - bh, bt.y * lh);
             }
@@ -1184,9 +1219,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  phase_mark<DBG == 2>(p, 2);
   if (warp == kMmaWarp) tmem_dealloc(tmem, C::TMEM_COLS);
   if (threadIdx.x == 0 && bars.abort) report_status(p.status, kStatusTimeout);
   if (!DUMP && p.fuse) fused_combine<D_C>(p, smem, bars);
+  phase_mark<DBG == 2>(p, 3);
 }
 
 // CTAs of `kern` that the current device holds at once (1 per SM here), cached per kernel
@@ -1205,10 +1242,10 @@ int resident_ctas(K kern, uint32_t smem) {
   return cached[dev];
 }
 
-template <int D_C, int GM, bool DUMP>
+template <int D_C, int GM, int DBG>
 cudaError_t launch_one(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_t st, bool* fused) {
   using C = Cfg<D_C, GM != 0>;
-  auto kern = decode_tc_kernel<D_C, GM, DUMP>;
+  auto kern = decode_tc_kernel<D_C, GM, DBG>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
   if (e != cudaSuccess) return e;
   const WorkspaceLayout wl = workspace_layout(a.batch, a.num_splits, kHeads, D_C, kRope, true);
@@ -1251,7 +1288,7 @@ cudaError_t launch_one(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_
   const int g = std::min(static_cast<int>(kFusedMaxG), (a.batch + groups - 1) / groups);
   p.cmb_g = g;
   p.cmb_groups = (a.batch + g - 1) / g;
-  p.fuse = !DUMP && a.batch > 0 && a.num_splits <= resident_ctas(kern, C::SMEM);
+  p.fuse = DBG != 1 && a.batch > 0 && a.num_splits <= resident_ctas(kern, C::SMEM);
   if (fused) *fused = p.fuse != 0;
   if (!p.fuse) {
     kern<<<a.num_splits, kThreads, C::SMEM, st>>>(maps[0], maps[1], p);
@@ -1277,11 +1314,19 @@ bool tc_supported(int d_c, int gate) {
   return d_c == 192 || d_c == 256 || d_c == 512;
 }
 
-// d_c-dispatch of one gate mode
+// d_c-dispatch of one gate mode; the trace instantiation exists for the modes
+// none and mul_ln (the others run untraced)
 template <int GM>
 cudaError_t launch_mode(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_t st, bool* fused) {
-  if (a.d_c == 192) return launch_one<192, GM, false>(a, maps, st, fused);
-  if (a.d_c == 256) return launch_one<256, GM, false>(a, maps, st, fused);
+  if constexpr (GM <= 1) {
+    if (a.trace != nullptr) {
+      if (a.d_c == 192) return launch_one<192, GM, 2>(a, maps, st, fused);
+      if (a.d_c == 256) return launch_one<256, GM, 2>(a, maps, st, fused);
+      return cudaErrorInvalidValue;
+    }
+  }
+  if (a.d_c == 192) return launch_one<192, GM, 0>(a, maps, st, fused);
+  if (a.d_c == 256) return launch_one<256, GM, 0>(a, maps, st, fused);
   return cudaErrorInvalidValue;
 }
 
@@ -1289,8 +1334,8 @@ cudaError_t launch_decode_tc(const DecodeArgs& a, const CUtensorMap* maps, bool 
                              bool* fused) {
   if (fused) *fused = false;
   if (dump) {   // cache-read test entry: the raw page and gate rows
-    if (a.d_c == 192) return launch_one<192, 1, true>(a, maps, st, nullptr);
-    if (a.d_c == 256) return launch_one<256, 1, true>(a, maps, st, nullptr);
+    if (a.d_c == 192) return launch_one<192, 1, 1>(a, maps, st, nullptr);
+    if (a.d_c == 256) return launch_one<256, 1, 1>(a, maps, st, nullptr);
     return cudaErrorInvalidValue;
   }
   if (!a.gate) {

@@ -123,30 +123,6 @@ struct TcParams {
   int32_t* dump_ids;
   __nv_bfloat16* dump_g;
   int dump_len;
-  // optional event trace (eg_mla_debug_set_trace): per traced CTA and role a
-  // run of (tag, clock64) pairs; tag = event << 24 | tile
-  unsigned long long* trace;
-  int trace_ctas, trace_cap;
-};
-
-// Trace recorder of one role of one CTA (a no-op unless tracing is on).
-struct Tracer {
-  unsigned long long* base;
-  int n, cap;
-  __device__ void init(const TcParams& p, int role) {
-    base = nullptr;
-    n = 0;
-    cap = p.trace_cap;
-    if (p.trace != nullptr && static_cast<int>(blockIdx.x) < p.trace_ctas)
-      base = p.trace + (static_cast<size_t>(blockIdx.x) * kTraceRoles + role) * p.trace_cap * 2;
-  }
-  __device__ __forceinline__ void mark(int event, int tile) {
-    if (base != nullptr && n < cap) {
-      base[2 * n] = (static_cast<unsigned long long>(event) << 24) | static_cast<unsigned>(tile & 0xffffff);
-      base[2 * n + 1] = clock64();
-      ++n;
-    }
-  }
 };
 
 // shared-memory barrier block (inside MISC, after 1 KB of reduction scratch)
@@ -345,9 +321,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     int last_it[6] = {-1, -1, -1, -1, -1, -1};
     int last_qseg[2] = {-1, -1};
     int bt_b = -1, bt_base = 0, bt_reg = -1;
-    Tracer tr;
-    tr.init(p, 0);
-    if (lane != 0) tr.base = nullptr;
     bool ok_loop = true;
     while (ok_loop && w.next(t)) {
       if (t.b != bt_b || t.lp >= bt_base + 32) {
@@ -371,10 +344,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             ok_loop = false;
           }
         }
-        tr.mark(0, it);
         if (ok_loop && !mbar_wait(smem_u32(&bars.empty[slot]), ((it / C::NS) & 1) ^ 1, abort_flag)) ok_loop = false;
         if (ok_loop) {
-          tr.mark(1, it);
           const bool ok = pg >= 0 && pg < p.num_pages;
           if (!ok) report_status(p.status, kStatusOutOfRange);
           const uint32_t fb = smem_u32(&bars.full[slot]);
@@ -386,7 +357,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int fc = 0; fc < C::NCH; ++fc) tma_load_2d(dst + fc * C::PCHUNK, &cmap, fc * 64, y, fb, pol_stream);
             tma_load_2d(dst + C::KR_OFF, &krmap, 0, y, fb, pol_stream);
           }
-          tr.mark(2, it);
           last_it[slot] = it;
         }
       }
@@ -413,9 +383,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       w.start(p.cu, p.seq_lens, p.batch);
       uint32_t last_bar = 0, last_par = 0;
       int seg = -1;
-      Tracer tr;
-      tr.init(p, 1);
-      if (lane != 0) tr.base = nullptr;
       // the query block as an N = 16 B operand: K groups 512 B apart, head halves 256 B apart
       const uint64_t qdesc0 = smem_desc(sbase + C::OFF_QBUF, kQGroupBytes, 256, kSwizzleNone);
       const uint64_t zdesc_k = smem_desc(sbase, 16, 1024, kSwizzle128B);         // K-major view of a slot
@@ -432,9 +399,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!warp_wait(smem_u32(&bars.qfull[seg & 1]), (seg >> 1) & 1, abort_flag)) return false;
         }
         const int slot = j % C::NS;
-        tr.mark(0, j);
         if (!warp_wait(smem_u32(&bars.zready[slot]), (j / C::NS) & 1, abort_flag)) return false;
-        tr.mark(1, j);
         tc_fence_after();
         if (elect_one()) {
           const uint64_t za = zdesc_k + ((slot * C::SLOT) >> 4);
@@ -462,9 +427,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (have_next && !scores(nxt, it + 1)) break;
         // latent output of tile it, accumulated in TMEM over the segment:
         // O^T[feature, head] += Z^T P'
-        tr.mark(2, it);
         if (!warp_wait(smem_u32(&bars.sp_done), it & 1, abort_flag)) break;
-        tr.mark(3, it);
         tc_fence_after();
         if (elect_one()) {
           const int slot = it % C::NS;
@@ -534,11 +497,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       int j = 0;
       int last_j[2] = {-1, -1};
-      Tracer tr;
-      tr.init(p, 4);
-      if (lane != 0) tr.base = nullptr;
       while (have) {
-        tr.mark(0, j);
         // ids of the next tile, consumed one iteration later
         Tile nt;
         const bool have_next = w.next(nt);
@@ -556,7 +515,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         const int gb = j & 1;
         if (!warp_wait(smem_u32(&bars.gempty[gb]), ((j >> 1) & 1) ^ 1, abort_flag)) break;
-        tr.mark(1, j);
         int32_t* gids = reinterpret_cast<int32_t*>(smem + C::OFF_GIDS + gb * C::GIDS);
         gids[lane] = id0;
         gids[lane + 32] = id1;
@@ -570,7 +528,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         cp_async_mbar_arrive(gbar);
         __syncwarp();
         if (lane == 0) mbar_arrive(gbar);   // releases the ids written above
-        tr.mark(2, j);
         last_j[gb] = j;
         ++j;
         t = nt;
@@ -594,19 +551,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int sw = row & 7;
     Walker w;
     w.start(p.cu, p.seq_lens, p.batch);
-    Tracer tr;
-    tr.init(p, 2);
-    if (threadIdx.x != kGateWarp0 * 32) tr.base = nullptr;
     Tile t;
     int j = 0;
     while (w.next(t)) {
       const int slot = j % C::NS;
       const int gb = j & 1;
-      tr.mark(0, j);
       if (!warp_wait(smem_u32(&bars.full[slot]), (j / C::NS) & 1, abort_flag)) break;
-      tr.mark(4, j);
       if (GATE && !warp_wait(smem_u32(&bars.gfull[gb]), (j >> 1) & 1, abort_flag)) break;
-      tr.mark(1, j);
       uint8_t* crow = smem + slot * C::SLOT + row * 128;
       const uint8_t* grow = smem + C::OFF_GBUF + gb * C::GBUF + row * C::GSTRIDE;
       const bool valid = row < t.ntok;
@@ -682,11 +633,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int k = 0; k < 4; ++k)
             *reinterpret_cast<uint4*>(crow + fc * C::PCHUNK + (2 * k + half) * 16) = make_uint4(0, 0, 0, 0);
       }
-      tr.mark(2, j);
       fence_proxy_async_smem();
       mbar_arrive(smem_u32(&bars.zready[slot]));
       if (GATE) mbar_arrive(smem_u32(&bars.gempty[gb]));
-      tr.mark(3, j);
       ++j;
     }
   } else if (warp >= kSoftWarp0 && !DUMP) {
@@ -713,9 +662,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     w.start(p.cu, p.seq_lens, p.batch);
     Tile t;
     int it = 0, seg = -1, nseg_end = 0;
-    Tracer tr;
-    tr.init(p, 3);
-    if (threadIdx.x != kSoftWarp0 * 32) tr.base = nullptr;
     while (w.next(t)) {
       if (t.first) {
         ++seg;
@@ -728,11 +674,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       const int slot = it % C::NS;
       const int par = it & 1;
-      tr.mark(0, it);
       // the gate's statistics for this tile are published with its zready arrival
       if (GATE && !warp_wait(smem_u32(&bars.zready[slot]), (it / C::NS) & 1, abort_flag)) break;
       if (!warp_wait(smem_u32(&bars.s_ready[par]), (it >> 1) & 1, abort_flag)) break;
-      tr.mark(1, it);
       tc_fence_after();
       float sl[16], sr[16], s[16];
       tmem_ld16(tl + C::COL_S + par * C::S_COLS, sl);
@@ -765,11 +709,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       if ((lane & 1) == 0) red_max[(par * 16 + (lane >> 1)) * 4 + q4] = wmax;
       mbar_arrive(smem_u32(&bars.red[par]));
       if (!warp_wait(smem_u32(&bars.red[par]), (it >> 1) & 1, abort_flag)) break;
-      tr.mark(2, it);
       // the previous tile's PV (same segment) must be complete before the
       // weight buffer is rewritten or the accumulator rescaled
       if (!t.first && !warp_wait(smem_u32(&bars.o_ready), (it - 1) & 1, abort_flag)) break;
-      tr.mark(5, it);
       bool rescale = false;
       float alpha[16];
 #pragma unroll
@@ -832,12 +774,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         *reinterpret_cast<uint4*>(prow) = make_uint4(pw[0], pw[1], pw[2], pw[3]);
         *reinterpret_cast<uint4*>(prow + 128) = make_uint4(pw[4], pw[5], pw[6], pw[7]);
       }
-      tr.mark(6, it);
       fence_proxy_async_smem();
       tc_fence_before();
-      tr.mark(7, it);
       mbar_arrive(smem_u32(&bars.sp_done));
-      tr.mark(3, it);
 
       if (t.last) {
         mbar_arrive(smem_u32(&bars.qempty[seg & 1]));
@@ -887,7 +826,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           ml[0] = mv;
           ml[1] = lv;
         }
-        tr.mark(4, it);
       }
       ++it;
     }
@@ -930,9 +868,6 @@ cudaError_t launch_one(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_
   p.dump_ids = a.dump_ids;
   p.dump_g = static_cast<__nv_bfloat16*>(a.dump_g);
   p.dump_len = a.max_seq_len;
-  p.trace = static_cast<unsigned long long*>(a.trace);
-  p.trace_ctas = a.trace_ctas;
-  p.trace_cap = a.trace_cap;
   kern<<<a.num_splits, kThreads, C::SMEM, st>>>(maps[0], maps[1], p);
   return cudaGetLastError();
 }

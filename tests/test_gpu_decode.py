@@ -163,6 +163,28 @@ def test_page_pool_permutation_is_bit_stable(gpu_lib):
     assert a.tobytes() == b.tobytes()
 
 
+@pytest.mark.parametrize("d_c,gate", [(256, True), (192, False)])
+def test_traced_build_matches_untraced(gpu_lib, d_c, gate):
+    # the pipeline trace runs a separately compiled build of the decode kernel:
+    # same outputs bit for bit, and every traced CTA records its kernel phases
+    case = small_bf16((700, 65, 1), d_c=d_c, gate=gate)
+    _, plain = run(case, 4)   # 14 pages: every one of the 4 splits has work
+    ctas, roles, cap = 4, 5, 64
+    buf = torch.zeros(ctas * roles * cap * 2, dtype=torch.int64, device="cuda")
+    _lib.eg_mla_debug_set_trace(buf, ctas)
+    try:
+        _, traced = run(case, 4)
+    finally:
+        _lib.eg_mla_debug_set_trace(None)
+    assert plain.tobytes() == traced.tobytes()
+    t = buf.cpu().numpy().reshape(ctas, roles, cap, 2)
+    for c in range(ctas):
+        phases = t[c, 4, :4]
+        assert (phases[:, 1] != 0).all(), f"CTA {c}: kernel phases missing"
+        assert list((phases[:, 0].astype(np.uint64) >> np.uint64(56)).astype(int)) == [0, 1, 2, 3]
+        assert (t[c, 0, 0, 1] != 0), f"CTA {c}: no TMA record"
+
+
 # --------------------------------------------------------------------------- bit-exact pieces
 def test_append_is_bit_exact(gpu_lib):
     case = small_bf16((1, 64, 65, 200))
