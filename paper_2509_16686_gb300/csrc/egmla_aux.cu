@@ -73,8 +73,9 @@ __device__ __forceinline__ void unpack16(const uint4& raw, float (&w)[4]) {
 }
 
 // ------------------------------------------------------------------ prologue
-// Exclusive prefix sum of pages per sequence: cu[b] = sum_{b'<b} ceil(L_b'/P),
-// cu[batch] = total; a scan by the block's first warp, 32 sequences per pass.
+// Exclusive prefix sum of the schedule units per sequence (its pages plus
+// kSegCost when it has any): cu[b] = sum_{b'<b} units_b', cu[batch] = total; a
+// scan by the block's first warp, 32 sequences per pass.
 __device__ void page_prefix_sums(const int32_t* seq_lens, int batch, int page_size, int32_t* cu) {
   if (threadIdx.x >= 32) return;
   const int lane = threadIdx.x;
@@ -82,7 +83,7 @@ __device__ void page_prefix_sums(const int32_t* seq_lens, int batch, int page_si
   for (int base = 0; base < batch; base += 32) {
     const int b = base + lane;
     const int L = b < batch ? seq_lens[b] : 0;
-    const int np = L > 0 ? (L + page_size - 1) / page_size : 0;
+    const int np = L > 0 ? (L + page_size - 1) / page_size + kSegCost : 0;
     int incl = np;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -302,7 +303,7 @@ combine_kernel(const int32_t* __restrict__ cu, const float* __restrict__ part_ml
   constexpr int kWarps = kCombineThreads / 32;
   const int total = cu[batch];
   const int chunk = split_chunk(total, num_splits);
-  const int p0 = cu[b], p1 = cu[b + 1];
+  const int p0 = cu[b] + kSegCost, p1 = cu[b + 1];   // units of the sequence's pages
   const int c0 = p0 / chunk;
   const int n = p1 > p0 ? (p1 - 1) / chunk - c0 + 1 : 0;
   if (n == 0) {
@@ -452,8 +453,10 @@ decode_f32_kernel(const float* __restrict__ c_pool, const float* __restrict__ kr
   while (g < g1) {
     const int pend = min(g1, cu[b + 1]);
     const int L = seq_lens[b];
-    const int tok0 = (g - cu[b]) * kPage;
-    const int tok1 = min((pend - cu[b]) * kPage, L);
+    const int s = cu[b] + kSegCost;   // unit of the sequence's first page
+    const int tok0 = max(g - s, 0) * kPage;
+    const int tok1 = min((pend - s) * kPage, L);
+    if (tok1 <= tok0) break;   // the range ends inside the sequence's start cost
     const float* qsrc = reinterpret_cast<const float*>(qprep + static_cast<size_t>(b) * qstride);
     for (int i = threadIdx.x; i < H * (d_c + d_rope); i += blockDim.x) qh[i] = qsrc[i];
     for (int i = threadIdx.x; i < H * d_c; i += blockDim.x) acc[i] = 0.f;

@@ -78,7 +78,15 @@ __host__ __device__ inline WorkspaceLayout workspace_layout(int batch, int num_s
   return w;
 }
 
-// pages per split for the total page count
+// Split-KV schedule.  The splits share the work in units: one per cache page,
+// plus kSegCost for the start of every non-empty sequence (the per-sequence cost
+// of a split: loading the query block, reading out and storing the partial
+// output), so that splits that take in more sequences get fewer pages.  cu[b]
+// is the first unit of sequence b; its pages are units cu[b] + kSegCost + i,
+// i < ceil(L_b / page); split c owns units [c chunk, (c + 1) chunk).
+constexpr int kSegCost = 1;
+
+// units per split for the total unit count
 __host__ __device__ inline int split_chunk(int total_pages, int num_splits) {
   int c = (total_pages + num_splits - 1) / num_splits;
   return c < 1 ? 1 : c;

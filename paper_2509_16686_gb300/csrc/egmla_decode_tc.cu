@@ -233,11 +233,12 @@ struct Walker {
     enter(g0);
   }
   __device__ void enter(int g) {
-    const int base = __ldg(cu + b);
-    lp = g - base;
+    const int base = __ldg(cu + b) + kSegCost;   // unit of the sequence's first page
+    lp = max(g - base, 0);
     lp_end = min(g1, __ldg(cu + b + 1)) - base;
     L = __ldg(lens + b);
     first = true;
+    if (lp_end <= lp) done = true;   // the range ends inside the sequence's start cost
   }
   __device__ bool next(Tile& t) {
     if (done) return false;
@@ -250,7 +251,7 @@ struct Walker {
     lp += 1;
     t.last = lp >= lp_end;
     if (t.last) {
-      const int g = __ldg(cu + b) + lp_end;
+      const int g = __ldg(cu + b) + kSegCost + lp_end;
       if (g >= g1) {
         done = true;
       } else {
@@ -412,7 +413,7 @@ __device__ void fused_combine(const TcParams& p, uint8_t* smem, Bars& bars) {
       const int chunk = split_chunk(total, gridDim.x);
       for (int w = warp; w < nb * NFB; w += kWarps) {
         const int j = w / NFB, f = (w % NFB) * 32 + lane, b = b0 + j;
-        const int q0 = p.cu[b], q1 = p.cu[b + 1];
+        const int q0 = p.cu[b] + kSegCost, q1 = p.cu[b + 1];   // units of the sequence's pages
         const int c0 = q0 / chunk;
         const int n = q1 > q0 ? (q1 - 1) / chunk - c0 + 1 : 0;
         const float* po = p.part_o + (static_cast<size_t>(c0 + b) * kHeads + h) * D_C + f;

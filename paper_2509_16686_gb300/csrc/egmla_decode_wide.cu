@@ -164,11 +164,12 @@ struct Walker {
     enter(g0);
   }
   __device__ void enter(int g) {
-    const int base = __ldg(cu + b);
-    lp = g - base;
+    const int base = __ldg(cu + b) + kSegCost;   // unit of the sequence's first page
+    lp = max(g - base, 0);
     lp_end = min(g1, __ldg(cu + b + 1)) - base;
     L = __ldg(lens + b);
     first = true;
+    if (lp_end <= lp) done = true;   // the range ends inside the sequence's start cost
   }
   __device__ bool next(Tile& t) {
     if (done) return false;
@@ -181,7 +182,7 @@ struct Walker {
     lp += 1;
     t.last = lp >= lp_end;
     if (t.last) {
-      const int g = __ldg(cu + b) + lp_end;
+      const int g = __ldg(cu + b) + kSegCost + lp_end;
       if (g >= g1) {
         done = true;
       } else {
