@@ -119,7 +119,7 @@ __global__ void prologue_tc_kernel(const __nv_bfloat16* __restrict__ q, const __
                        const float* __restrict__ gamma, const float* __restrict__ beta,
                        const int32_t* __restrict__ seq_lens, int batch, int d_nope, int d_rope, int d_c,
                        int page_size, uint8_t* __restrict__ qprep, size_t qstride, int32_t* __restrict__ cu,
-                       uint32_t* __restrict__ grid_bar) {
+                       uint32_t* __restrict__ seq_done) {
   __shared__ __align__(16) __nv_bfloat16 ws[kPMaxNope][kSumFeatures];  // W_UK,h[n][f0 + f]
   __shared__ __align__(16) __nv_bfloat16 qs[kPBatch][kPMaxNope];      // q^C_{b0 + j, h}[n]
   // partial sums [n part * 4 quads + j][f], written once every warp is done with ws
@@ -129,7 +129,8 @@ __global__ void prologue_tc_kernel(const __nv_bfloat16* __restrict__ q, const __
   const int nchunk = d_c / kSumFeatures;
   const int ngroups = (batch + kPBatch - 1) / kPBatch;
   if (blockIdx.x == static_cast<unsigned>(H * nchunk * ngroups)) {
-    if (threadIdx.x == 0 && grid_bar != nullptr) *grid_bar = 0u;
+    if (seq_done != nullptr)
+      for (int i = threadIdx.x; i <= batch; i += blockDim.x) seq_done[i] = 0u;
     page_prefix_sums(seq_lens, batch, page_size, cu);
     return;
   }
@@ -556,7 +557,7 @@ cudaError_t launch_prologue_tc(const DecodeArgs& a, cudaStream_t st) {
   prologue_tc_kernel<<<16 * (a.d_c / kSumFeatures) * ngroups + 1, 256, 0, st>>>(
       static_cast<const __nv_bfloat16*>(a.q), static_cast<const __nv_bfloat16*>(a.w_uk), gamma, beta,
       a.seq_lens, a.batch, a.d_nope, a.d_rope, a.d_c, a.page_size, ws + wl.off_qprep, wl.qprep_stride,
-      reinterpret_cast<int32_t*>(ws + wl.off_cu), reinterpret_cast<uint32_t*>(ws + wl.off_bar));
+      reinterpret_cast<int32_t*>(ws + wl.off_cu), reinterpret_cast<uint32_t*>(ws + wl.off_done));
   return cudaGetLastError();
 }
 

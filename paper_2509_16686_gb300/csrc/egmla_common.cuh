@@ -52,7 +52,7 @@ __host__ __device__ inline size_t qprep_bytes_f32(int H, int d_c, int d_rope) {
 }
 
 struct WorkspaceLayout {
-  size_t off_cu, off_bar, off_qprep, off_ml, off_o, total;
+  size_t off_cu, off_done, off_qprep, off_ml, off_o, total;
   size_t qprep_stride;
   int num_slots;
 };
@@ -65,9 +65,10 @@ __host__ __device__ inline WorkspaceLayout workspace_layout(int batch, int num_s
   size_t off = 0;
   w.off_cu = off;
   off = align_up(off + static_cast<size_t>(batch + 1) * 4, 256);
-  // grid-barrier counter of the fused combine (zeroed by the prologue each call)
-  w.off_bar = off;
-  off = align_up(off + 4, 256);
+  // the fused combine's counters (zeroed by the prologue each call): [0] the
+  // CTAs done, [1 + b] the split partials of sequence b stored
+  w.off_done = off;
+  off = align_up(off + static_cast<size_t>(batch + 1) * 4, 256);
   w.off_qprep = off;
   off = align_up(off + static_cast<size_t>(batch) * w.qprep_stride, 256);
   w.off_ml = off;

@@ -150,7 +150,7 @@ struct TcParams {
   // and the (head, group of cmb_g sequences) units
   const __nv_bfloat16* w_uv;
   __nv_bfloat16* out;
-  uint32_t* grid_bar;
+  uint32_t* seq_done;   // [0] CTAs done, [1 + b] split partials of sequence b stored
   int d_v, cmb_groups, cmb_g;
   int fuse;
 };
@@ -355,10 +355,13 @@ __device__ __forceinline__ float reduce8_rows(const float (&v)[8], int lane) {
 }
 
 // Split-KV combine inside the decode kernel (cooperative launch: every CTA is
-// resident, so a grid-wide wait cannot starve).  After its pages each CTA
-// arrives on a grid counter (zeroed by the prologue kernel of the same call)
-// and, once all have arrived, merges its units (head h, group of cmb_g
-// sequences): for each sequence b, over the splits s that covered it,
+// resident, so a wait on other CTAs cannot starve).  A CTA merges its units
+// (head h, group of cmb_g sequences) once their split partials are stored:
+// with one sequence per unit (small batches) as soon as the softmax warps of
+// the splits that covered that sequence have counted their halves on its
+// counter, otherwise after every CTA has arrived on a grid counter (both
+// counters zeroed by the prologue kernel of the same call).  For each sequence
+// b, over the splits s that covered it,
 //   o = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s,
 //   u_{b,h} = W_UV,h o
 // (a sequence of length 0 gets u = 0).  W_UV,h is bulk-copied into the free
@@ -388,13 +391,21 @@ __device__ void fused_combine(const TcParams& p, uint8_t* smem, Bars& bars) {
   };
   int u = blockIdx.x;
   if (u < units) issue_w(u % kHeads);
-  if (tid == 0) {
-    // this CTA's partials are stored (the kernel-end barrier ordered the other
-    // threads' stores before this thread): release them, then wait for all
+  const int total = p.cu[p.batch];
+  const int chunk = split_chunk(total, gridDim.x);
+  // splits that covered sequence b
+  auto splits_of = [&](int b) -> int {
+    const int q0 = p.cu[b] + kSegCost, q1 = p.cu[b + 1];   // units of the sequence's pages
+    return q1 > q0 ? (q1 - 1) / chunk - q0 / chunk + 1 : 0;
+  };
+  if (G > 1 && tid == 0) {
+    // units of several sequences wait for the whole grid: this CTA's partials
+    // are stored (the kernel-end barrier ordered the other threads' stores
+    // before this thread): release them, then wait for all
     __threadfence();
-    atomicAdd(p.grid_bar, 1u);
+    atomicAdd(p.seq_done, 1u);
     const uint64_t t0 = globaltimer();
-    while (ld_acquire_gpu(p.grid_bar) < gridDim.x) {
+    while (ld_acquire_gpu(p.seq_done) < gridDim.x) {
       if (globaltimer() - t0 > kWaitLimitNs) {
         report_status(p.status, kStatusTimeout);
         *abort_flag = 1;
@@ -403,14 +414,26 @@ __device__ void fused_combine(const TcParams& p, uint8_t* smem, Bars& bars) {
       __nanosleep(32);
     }
   }
-  __syncthreads();
   int phase = 0;
   for (; u < units; u += gridDim.x) {
     const int h = u % kHeads, grp = u / kHeads;
     const int b0 = grp * G, nb = min(G, p.batch - b0);
+    if (G == 1 && tid == 0 && !*abort_flag) {
+      // a unit of one sequence: both halves of every split partial of it stored
+      const uint32_t want = 2u * static_cast<uint32_t>(splits_of(b0));
+      const uint64_t t0 = globaltimer();
+      while (ld_acquire_gpu(p.seq_done + 1 + b0) < want) {
+        if (*abort_flag) break;
+        if (globaltimer() - t0 > kWaitLimitNs) {
+          report_status(p.status, kStatusTimeout);
+          *abort_flag = 1;
+          break;
+        }
+        __nanosleep(32);
+      }
+    }
+    __syncthreads();
     if (!*abort_flag) {
-      const int total = p.cu[p.batch];
-      const int chunk = split_chunk(total, gridDim.x);
       for (int w = warp; w < nb * NFB; w += kWarps) {
         const int j = w / NFB, f = (w % NFB) * 32 + lane, b = b0 + j;
         const int q0 = p.cu[b] + kSegCost, q1 = p.cu[b + 1];   // units of the sequence's pages
@@ -1212,6 +1235,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           ml[0] = m_ref;
           ml[1] = lh;
         }
+        if (p.fuse && p.cmb_g == 1) {
+          // one sequence per combine unit: release this warp's half of the
+          // partial to the wait on its sequence (the warp barrier orders every
+          // lane's stores before lane 0's fence)
+          __syncwarp();
+          if (lane == 0) {
+            __threadfence();
+            atomicAdd(p.seq_done + 1 + t.b, 1u);
+          }
+        }
+
         tr.mark(4, it);
       }
       ++it;
@@ -1283,7 +1317,7 @@ cudaError_t launch_one(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_
   // be resident at once (a cooperative launch guarantees it, or fails).
   p.w_uv = static_cast<const __nv_bfloat16*>(a.w_uv);
   p.out = static_cast<__nv_bfloat16*>(a.out);
-  p.grid_bar = reinterpret_cast<uint32_t*>(ws + wl.off_bar);
+  p.seq_done = reinterpret_cast<uint32_t*>(ws + wl.off_done);
   p.d_v = a.d_v;
   int groups = std::max(1, std::min(a.batch, a.num_splits / kHeads));
   const int g = std::min(static_cast<int>(kFusedMaxG), (a.batch + groups - 1) / groups);
