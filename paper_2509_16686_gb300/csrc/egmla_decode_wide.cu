@@ -45,7 +45,7 @@ namespace {
 
 constexpr int kHeads = 16;
 constexpr int kRope = 64;
-constexpr int kThreads = 384;  // warp 0 TMA, warp 1 MMA + TMEM owner, 2-3 spare, 4-7 gate, 8-11 softmax
+constexpr int kThreads = 384;  // warp 0 TMA, warp 1 MMA + TMEM owner, 2-3 spare, 4-7 zero fill, 8-11 softmax
 constexpr int kGateWarp0 = 4;
 constexpr int kSoftWarp0 = 8;
 constexpr uint32_t kSmemLimit = 232448;
@@ -56,7 +56,7 @@ constexpr int kConsumerRegs = 224;
 // a head's reference max moves only when a tile exceeds it by 2^8
 constexpr float kLazyLog2 = 8.f;
 
-template <int D_C, bool GATE>
+template <int D_C>
 struct Cfg {
   static constexpr int NCH = D_C / 64;                  // 64-feature swizzle-atom columns
   static constexpr int NMC = (D_C + 127) / 128;         // 128-feature M chunks of the PV MMA
@@ -64,28 +64,15 @@ struct Cfg {
   static constexpr uint32_t KR_OFF = NCH * PCHUNK;
   static constexpr uint32_t SLOT = KR_OFF + PCHUNK;     // latent + RoPE key of one page
   static constexpr uint32_t QB_LAT = qprep_lat_bytes(D_C);
-  static constexpr uint32_t QB_ROPE = qprep_rope_bytes(kRope);
   static constexpr uint32_t QPREP = qprep_bytes_tc(D_C, kRope);
   static constexpr uint32_t QBUF = (QPREP + 127) / 128 * 128;
   static constexpr uint32_t PBUF = kPage * kHeads * 2;
-  // gate rows of a page, gathered by TMA bulk copies: row stride padded by 16 B
-  // so that the gate threads' 16-byte reads of 8 consecutive rows hit 8 distinct
-  // bank groups; double-buffered
-  static constexpr uint32_t GSTRIDE = D_C * 2 + 16;
-  static constexpr uint32_t GBUF = (kPage * GSTRIDE + 127) / 128 * 128;
-  static constexpr int NGB = GATE ? 2 : 0;
-  static constexpr uint32_t GIDS = kPage * 4;           // token ids of a gathered page
-  static constexpr uint32_t STAT_BYTES = kPage * 8;     // per slot: (mu, r) per token
   static constexpr uint32_t MISC = 2048;
-  static constexpr int NS_FIT =
-      (int)((kSmemLimit - 1024 - 2 * QBUF - PBUF - MISC - NGB * (GBUF + GIDS)) / (SLOT + STAT_BYTES));
+  static constexpr int NS_FIT = (int)((kSmemLimit - 1024 - 2 * QBUF - PBUF - MISC) / SLOT);
   static constexpr int NS = NS_FIT > 6 ? 6 : NS_FIT;
   static constexpr uint32_t OFF_QBUF = NS * SLOT;
   static constexpr uint32_t OFF_PBUF = OFF_QBUF + 2 * QBUF;
-  static constexpr uint32_t OFF_GBUF = OFF_PBUF + PBUF;
-  static constexpr uint32_t OFF_GIDS = OFF_GBUF + NGB * GBUF;
-  static constexpr uint32_t OFF_STAT = OFF_GIDS + NGB * GIDS;
-  static constexpr uint32_t OFF_MISC = OFF_STAT + NS * STAT_BYTES;
+  static constexpr uint32_t OFF_MISC = OFF_PBUF + PBUF;
   static constexpr uint32_t SMEM = OFF_MISC + MISC + 1024;
   // TMEM columns: two score buffers of (latent 16 + RoPE 16) columns, then the
   // latent-output accumulator (16 columns per 128-feature chunk), which stays
@@ -105,30 +92,20 @@ struct Cfg {
 };
 
 struct TcParams {
-  const int32_t* id_pool;
   const int32_t* block_table;
   const int32_t* seq_lens;
-  const __nv_bfloat16* gate_table;
-  const float* gamma;
-  const float* beta;
   const uint8_t* qprep;
   const int32_t* cu;
   float* part_ml;
   float* part_o;
   int32_t* status;
-  int batch, max_pages, num_pages, vocab;
-  float scale_log2, eps;
-  __nv_bfloat16* dump_c;
-  __nv_bfloat16* dump_kr;
-  int32_t* dump_ids;
-  __nv_bfloat16* dump_g;
-  int dump_len;
+  int batch, max_pages, num_pages;
+  float scale_log2;
 };
 
 // shared-memory barrier block (inside MISC, after 1 KB of reduction scratch)
 struct Bars {
   uint64_t full[6], empty[6], zready[6];
-  uint64_t gfull[2], gempty[2];
   uint64_t qfull[2], qempty[2];
   uint64_t s_ready[2];
   uint64_t sp_done, o_ready;
@@ -206,13 +183,6 @@ __device__ __forceinline__ float2 unpack_bf16x2(uint32_t w) {
   return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
 }
 
-__device__ __forceinline__ uint32_t mul_bf16x2(uint32_t a, uint32_t b) {
-  __nv_bfloat162 x = *reinterpret_cast<__nv_bfloat162*>(&a);
-  __nv_bfloat162 y = *reinterpret_cast<__nv_bfloat162*>(&b);
-  __nv_bfloat162 z = __hmul2(x, y);
-  return *reinterpret_cast<uint32_t*>(&z);
-}
-
 // 2^x with the hardware approximation (max 2 ulp; the weights are rounded to
 // bf16 right after, and -inf gives 0)
 __device__ __forceinline__ float ex2_approx(float x) {
@@ -258,11 +228,11 @@ __device__ __forceinline__ float warp_reduce16(const float (&v)[16], int lane) {
   return op(r1, __shfl_xor_sync(0xffffffffu, r1, 1));
 }
 
-template <int D_C, bool GATE, bool DUMP>
+template <int D_C>
 __global__ void __launch_bounds__(kThreads, 1)
     decode_tc_kernel(const __grid_constant__ CUtensorMap cmap, const __grid_constant__ CUtensorMap krmap,
                      const TcParams p) {
-  using C = Cfg<D_C, GATE>;
+  using C = Cfg<D_C>;
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte aligned base (128-byte swizzle atoms); derived by an offset from the
   // __shared__ array so that every access through it stays a shared-memory access
@@ -278,12 +248,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::NS; ++s) {
       mbar_init(smem_u32(&bars.full[s]), 1);
-      mbar_init(smem_u32(&bars.empty[s]), DUMP ? 128 : 1);
+      mbar_init(smem_u32(&bars.empty[s]), 1);
       mbar_init(smem_u32(&bars.zready[s]), 128);
     }
     for (int s = 0; s < 2; ++s) {
-      mbar_init(smem_u32(&bars.gfull[s]), 33);   // 32 cp.async arrivals + the ids
-      mbar_init(smem_u32(&bars.gempty[s]), 128);
       mbar_init(smem_u32(&bars.qfull[s]), 1);
       mbar_init(smem_u32(&bars.qempty[s]), 1 + 128);
       mbar_init(smem_u32(&bars.s_ready[s]), 1);
@@ -334,7 +302,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (t.first) ++seg;
       const int slot = it % C::NS;
       if (lane == 0) {
-        if (t.first && !DUMP) {
+        if (t.first) {
           const int qb = seg & 1;
           if (mbar_wait(smem_u32(&bars.qempty[qb]), ((seg >> 1) & 1) ^ 1, abort_flag)) {
             mbar_arrive_expect_tx(smem_u32(&bars.qfull[qb]), C::QPREP);
@@ -377,7 +345,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Converged warp; one elected lane issues.  Order: scores(i + 1) before
     // PV(i), so the next tile's scores are ready when the softmax warps finish
     // tile i.  All loops are unrolled with compile-time accumulate flags.
-    if (!DUMP) {
+    {
       constexpr uint32_t IDESC_QK = idesc_bf16(64, 16, 0, 0);
       constexpr uint32_t IDESC_PV = idesc_bf16(128, 16, 1, 1);
       Walker w;
@@ -462,172 +430,21 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (last_bar != 0) mbar_wait(last_bar, last_par, abort_flag);
     }
     __syncwarp();
-  } else if (warp == 2) {
-    // ---------------------------------------------------------------- gate-row gather
-    // For every page: its 64 token ids (two per lane, loaded one page ahead so
-    // the load latency is off this loop), then the gate rows G[id] copied with
-    // 16-byte cp.async, one row per warp instruction, into a double-buffered row
-    // area.  Per-row bulk copies cost the copy engine ~60 cycles each; cp.async
-    // keeps the gather under the latent stream.  Each lane's async arrival fires
-    // once its copies have landed; lane 0 adds one release arrival after the ids.
-    if constexpr (GATE) {
-      constexpr int kUnits = D_C * 2 / 16;   // 16-byte units of a gate row
-      static_assert(kUnits <= 32, "one row per warp instruction");
-      const uint64_t pol_keep = policy_evict_last();
-      Walker w;
-      w.start(p.cu, p.seq_lens, p.batch);
-      int bt_b = -1, bt_base = 0, bt_reg = -1;
-      // page of tile t through a 32-entry window of the block table (one entry per lane)
-      auto page_of = [&](const Tile& t) -> int {
-        if (t.b != bt_b || t.lp >= bt_base + 32) {
-          bt_b = t.b;
-          bt_base = t.lp;
-          const int lp = t.lp + lane;
-          bt_reg = lp < p.max_pages ? __ldg(p.block_table + static_cast<size_t>(t.b) * p.max_pages + lp) : -1;
-        }
-        return __shfl_sync(0xffffffffu, bt_reg, t.lp - bt_base);
-      };
-      Tile t;
-      bool have = w.next(t);
-      int ntok = 0, id0 = 0, id1 = 0;
-      if (have) {
-        const int pg = page_of(t);
-        ntok = (pg >= 0 && pg < p.num_pages) ? t.ntok : 0;   // bad pages: reported by the producer
-        if (lane < ntok) id0 = __ldg(p.id_pool + static_cast<size_t>(pg) * kPage + lane);
-        if (lane + 32 < ntok) id1 = __ldg(p.id_pool + static_cast<size_t>(pg) * kPage + lane + 32);
-      }
-      int j = 0;
-      int last_j[2] = {-1, -1};
-      while (have) {
-        // ids of the next tile, consumed one iteration later
-        Tile nt;
-        const bool have_next = w.next(nt);
-        int n_ntok = 0, n_id0 = 0, n_id1 = 0;
-        if (have_next) {
-          const int pg = page_of(nt);
-          n_ntok = (pg >= 0 && pg < p.num_pages) ? nt.ntok : 0;
-          if (lane < n_ntok) n_id0 = __ldg(p.id_pool + static_cast<size_t>(pg) * kPage + lane);
-          if (lane + 32 < n_ntok) n_id1 = __ldg(p.id_pool + static_cast<size_t>(pg) * kPage + lane + 32);
-        }
-        if ((lane < ntok && (unsigned)id0 >= (unsigned)p.vocab) || (lane + 32 < ntok && (unsigned)id1 >= (unsigned)p.vocab)) {
-          report_status(p.status, kStatusOutOfRange);
-          if ((unsigned)id0 >= (unsigned)p.vocab) id0 = 0;
-          if ((unsigned)id1 >= (unsigned)p.vocab) id1 = 0;
-        }
-        const int gb = j & 1;
-        if (!warp_wait(smem_u32(&bars.gempty[gb]), ((j >> 1) & 1) ^ 1, abort_flag)) break;
-        int32_t* gids = reinterpret_cast<int32_t*>(smem + C::OFF_GIDS + gb * C::GIDS);
-        gids[lane] = id0;
-        gids[lane + 32] = id1;
-        const uint32_t gbar = smem_u32(&bars.gfull[gb]);
-        const uint32_t gdst = sbase + C::OFF_GBUF + gb * C::GBUF + lane * 16;
-        const __nv_bfloat16* gsrc = p.gate_table + lane * 8;
-        for (int r = 0; r < ntok; ++r) {
-          const int id = __shfl_sync(0xffffffffu, r < 32 ? id0 : id1, r & 31);
-          if (lane < kUnits) cp_async_16_hint(gdst + r * C::GSTRIDE, gsrc + static_cast<size_t>(id) * D_C, pol_keep);
-        }
-        cp_async_mbar_arrive(gbar);
-        __syncwarp();
-        if (lane == 0) mbar_arrive(gbar);   // releases the ids written above
-        last_j[gb] = j;
-        ++j;
-        t = nt;
-        have = have_next;
-        ntok = n_ntok;
-        id0 = n_id0;
-        id1 = n_id1;
-      }
-      // drain: the copies this warp issued must land before the CTA exits
-      cp_async_wait_all();
-      for (int b = 0; b < 2; ++b)
-        if (last_j[b] >= 0) mbar_wait(smem_u32(&bars.gfull[b]), (last_j[b] >> 1) & 1, abort_flag);
-    }
-    __syncwarp();
   } else if (warp >= kGateWarp0 && warp < kGateWarp0 + 4) {
-    // ---------------------------------------------------------------- gate: z = c (*) g, LN statistics
+    // ---------------------------------------------------------------- zero fill of rows past a partial page
     regs_increase<kConsumerRegs>();
     const int gw = warp - kGateWarp0;
     const int row = gw * 16 + (lane & 15);    // token row of the page
     const int half = lane >> 4;               // 16-byte units 2k + half of every 128-byte chunk row
-    const int sw = row & 7;
     Walker w;
     w.start(p.cu, p.seq_lens, p.batch);
     Tile t;
     int j = 0;
     while (w.next(t)) {
       const int slot = j % C::NS;
-      const int gb = j & 1;
       if (!warp_wait(smem_u32(&bars.full[slot]), (j / C::NS) & 1, abort_flag)) break;
-      if (GATE && !warp_wait(smem_u32(&bars.gfull[gb]), (j >> 1) & 1, abort_flag)) break;
       uint8_t* crow = smem + slot * C::SLOT + row * 128;
-      const uint8_t* grow = smem + C::OFF_GBUF + gb * C::GBUF + row * C::GSTRIDE;
-      const bool valid = row < t.ntok;
-      if (DUMP) {
-        if (valid && half == 0) {
-          const int id = reinterpret_cast<const int32_t*>(smem + C::OFF_GIDS + gb * C::GIDS)[row];
-          const size_t o = static_cast<size_t>(t.b) * p.dump_len + t.tok0 + row;
-          p.dump_ids[o] = id;
-          uint4* dc = reinterpret_cast<uint4*>(p.dump_c + o * D_C);
-          uint4* dg = reinterpret_cast<uint4*>(p.dump_g + o * D_C);
-          uint4* dk = reinterpret_cast<uint4*>(p.dump_kr + o * kRope);
-          for (int fc = 0; fc < C::NCH; ++fc)
-            for (int u = 0; u < 8; ++u) {
-              dc[fc * 8 + u] = *reinterpret_cast<const uint4*>(crow + fc * C::PCHUNK + ((u ^ sw) << 4));
-              dg[fc * 8 + u] = *reinterpret_cast<const uint4*>(grow + fc * 128 + u * 16);
-            }
-          for (int u = 0; u < 8; ++u)
-            dk[u] = *reinterpret_cast<const uint4*>(smem + slot * C::SLOT + C::KR_OFF + row * 128 + ((u ^ sw) << 4));
-        }
-        mbar_arrive(smem_u32(&bars.empty[slot]));
-        mbar_arrive(smem_u32(&bars.gempty[gb]));
-        ++j;
-        continue;
-      }
-      float2* stat = reinterpret_cast<float2*>(smem + C::OFF_STAT + slot * C::STAT_BYTES);
-      if (GATE) {
-        // all shared-memory reads of this thread's units first (the in-place
-        // stores below would otherwise order every later load behind them)
-        uint4 cv[C::NCH * 4], gv[C::NCH * 4];
-#pragma unroll
-        for (int i = 0; i < C::NCH * 4; ++i) {
-          const int fc = i >> 2, u = 2 * (i & 3) + half;
-          cv[i] = *reinterpret_cast<const uint4*>(crow + fc * C::PCHUNK + ((u ^ sw) << 4));
-          gv[i] = *reinterpret_cast<const uint4*>(grow + fc * 128 + u * 16);
-        }
-        const bool full_page = t.ntok == kPage;   // uniform: no token masking needed
-        float2 s1 = make_float2(0.f, 0.f), s2 = make_float2(0.f, 0.f);
-        float2 a1 = make_float2(0.f, 0.f), a2 = make_float2(0.f, 0.f);
-#pragma unroll
-        for (int i = 0; i < C::NCH * 4; ++i) {
-          const int fc = i >> 2, u = 2 * (i & 3) + half;
-          uint4 z;
-          z.x = mul_bf16x2(cv[i].x, gv[i].x);
-          z.y = mul_bf16x2(cv[i].y, gv[i].y);
-          z.z = mul_bf16x2(cv[i].z, gv[i].z);
-          z.w = mul_bf16x2(cv[i].w, gv[i].w);
-          if (!full_page && !valid) z = make_uint4(0, 0, 0, 0);
-          const float2 f0 = unpack_bf16x2(z.x), f1 = unpack_bf16x2(z.y);
-          const float2 f2 = unpack_bf16x2(z.z), f3 = unpack_bf16x2(z.w);
-          s1 = __fadd2_rn(s1, f0);
-          a1 = __fadd2_rn(a1, f1);
-          s1 = __fadd2_rn(s1, f2);
-          a1 = __fadd2_rn(a1, f3);
-          s2 = __ffma2_rn(f0, f0, s2);
-          a2 = __ffma2_rn(f1, f1, a2);
-          s2 = __ffma2_rn(f2, f2, s2);
-          a2 = __ffma2_rn(f3, f3, a2);
-          *reinterpret_cast<uint4*>(crow + fc * C::PCHUNK + ((u ^ sw) << 4)) = z;
-        }
-        s1 = __fadd2_rn(s1, a1);
-        s2 = __fadd2_rn(s2, a2);
-        float sum1 = s1.x + s1.y, sum2 = s2.x + s2.y;
-        sum1 += __shfl_xor_sync(0xffffffffu, sum1, 16);
-        sum2 += __shfl_xor_sync(0xffffffffu, sum2, 16);
-        constexpr float inv_dc = 1.f / D_C;
-        const float mu = sum1 * inv_dc;
-        const float var = fmaxf(sum2 * inv_dc - mu * mu, 0.f);
-        if (half == 0) stat[row] = valid ? make_float2(mu, rsqrtf(var + p.eps)) : make_float2(0.f, 0.f);
-      } else if (!valid) {
+      if (row >= t.ntok) {
 #pragma unroll
         for (int fc = 0; fc < C::NCH; ++fc)
 #pragma unroll
@@ -636,10 +453,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       fence_proxy_async_smem();
       mbar_arrive(smem_u32(&bars.zready[slot]));
-      if (GATE) mbar_arrive(smem_u32(&bars.gempty[gb]));
       ++j;
     }
-  } else if (warp >= kSoftWarp0 && !DUMP) {
+  } else if (warp >= kSoftWarp0) {
     // ---------------------------------------------------------------- softmax, output read-out
     regs_increase<kConsumerRegs>();
     const int q4 = warp & 3;                   // TMEM lane quadrant of this warp
@@ -649,16 +465,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tl = tmem + (static_cast<uint32_t>(q4 * 32) << 16);
     // Online softmax with a lazily updated reference max m_ref per head: the
     // exponentials are taken against m_ref, which only moves (rescaling the
-    // TMEM accumulator, l and the mean correction) when a tile's max exceeds it
-    // by more than 2^kLazyLog2; otherwise the weights stay below 2^kLazyLog2.
-    float m_ref[16], l_part[16], bmu_part[16];
-    float gam[C::NMC], bet[C::NMC];
-#pragma unroll
-    for (int mc = 0; mc < C::NMC; ++mc) {
-      const int f = C::mc_start(mc) + frow;
-      gam[mc] = (GATE && p.gamma) ? p.gamma[f] : 1.f;
-      bet[mc] = (GATE && p.beta) ? p.beta[f] : 0.f;
-    }
+    // TMEM accumulator and l) when a tile's max exceeds it by more than
+    // 2^kLazyLog2; otherwise the weights stay below 2^kLazyLog2.
+    float m_ref[16], l_part[16];
     Walker w;
     w.start(p.cu, p.seq_lens, p.batch);
     Tile t;
@@ -667,45 +476,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (t.first) {
         ++seg;
 #pragma unroll
-        for (int h = 0; h < 16; ++h) {
-          l_part[h] = 0.f;
-          bmu_part[h] = 0.f;
-        }
+        for (int h = 0; h < 16; ++h) l_part[h] = 0.f;
         if (!warp_wait(smem_u32(&bars.qfull[seg & 1]), (seg >> 1) & 1, abort_flag)) break;
       }
       const int slot = it % C::NS;
       const int par = it & 1;
-      // the gate's statistics for this tile are published with its zready arrival
-      if (GATE && !warp_wait(smem_u32(&bars.zready[slot]), (it / C::NS) & 1, abort_flag)) break;
       if (!warp_wait(smem_u32(&bars.s_ready[par]), (it >> 1) & 1, abort_flag)) break;
       tc_fence_after();
       float sl[16], sr[16], s[16];
       tmem_ld16(tl + C::COL_S + par * C::S_COLS, sl);
       tmem_ld16(tl + C::COL_S + par * C::S_COLS + 16, sr);
       const bool valid = token_lane && srow < t.ntok;
-      float mu = 0.f, rstd = 1.f;
-      if (GATE && token_lane) {
-        const float2 st = reinterpret_cast<const float2*>(smem + C::OFF_STAT + slot * C::STAT_BYTES)[srow];
-        mu = st.x;
-        rstd = st.y;
-      }
-      const float4* sums4 = reinterpret_cast<const float4*>(smem + C::OFF_QBUF + (seg & 1) * C::QBUF + C::QB_LAT +
-                                                            C::QB_ROPE);
-      float wq[16], bq[16];
-      if (GATE) {
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const float4 a = sums4[k], b = sums4[4 + k];
-          wq[4 * k] = a.x; wq[4 * k + 1] = a.y; wq[4 * k + 2] = a.z; wq[4 * k + 3] = a.w;
-          bq[4 * k] = b.x; bq[4 * k + 1] = b.y; bq[4 * k + 2] = b.z; bq[4 * k + 3] = b.w;
-        }
-      }
       tmem_wait_ld();
 #pragma unroll
-      for (int h = 0; h < 16; ++h) {
-        const float lat = GATE ? rstd * (sl[h] - mu * wq[h]) + bq[h] : sl[h];
-        s[h] = valid ? (lat + sr[h]) * p.scale_log2 : -INFINITY;
-      }
+      for (int h = 0; h < 16; ++h) s[h] = valid ? (sl[h] + sr[h]) * p.scale_log2 : -INFINITY;
       const float wmax = warp_reduce16<true>(s, lane);
       if ((lane & 1) == 0) red_max[(par * 16 + (lane >> 1)) * 4 + q4] = wmax;
       mbar_arrive(smem_u32(&bars.red[par]));
@@ -742,31 +526,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tmem_wait_st();
 #pragma unroll
-        for (int h = 0; h < 16; ++h) {
-          l_part[h] *= alpha[h];
-          bmu_part[h] *= alpha[h];
-        }
+        for (int h = 0; h < 16; ++h) l_part[h] *= alpha[h];
       }
-      // The PV MMA sees the bf16-rounded weights P'; the denominator and the mean
-      // correction use the same rounded values (l = sum P'/r), so the rounding of
-      // P' cancels in o = (sum P' z - sum P' mu) / l instead of biasing it.
-      const float inv_r = GATE ? (valid ? 1.f / rstd : 0.f) : 1.f;
+      // The PV MMA sees the bf16-rounded weights P'; the denominator sums the
+      // same rounded values, so their rounding cancels in o = sum P' z / l.
 #pragma unroll
-      for (int h = 0; h < 16; ++h) {
-        const float pr = ex2_approx(s[h] - m_ref[h]);
-        s[h] = GATE ? pr * rstd : pr;
-      }
+      for (int h = 0; h < 16; ++h) s[h] = ex2_approx(s[h] - m_ref[h]);
       uint32_t pw[8];
 #pragma unroll
       for (int k = 0; k < 8; ++k) {
         pw[k] = pack_bf16x2(s[2 * k], s[2 * k + 1]);
         const float2 pq = unpack_bf16x2(pw[k]);
-        l_part[2 * k] = fmaf(pq.x, inv_r, l_part[2 * k]);
-        l_part[2 * k + 1] = fmaf(pq.y, inv_r, l_part[2 * k + 1]);
-        if (GATE) {
-          bmu_part[2 * k] = fmaf(pq.x, mu, bmu_part[2 * k]);
-          bmu_part[2 * k + 1] = fmaf(pq.y, mu, bmu_part[2 * k + 1]);
-        }
+        l_part[2 * k] += pq.x;
+        l_part[2 * k + 1] += pq.y;
       }
       // P'[token][head] as an MN-major B operand: 8x8 core matrices, token group
       // stride 256 B, head group stride 128 B
@@ -781,22 +553,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 
       if (t.last) {
         mbar_arrive(smem_u32(&bars.qempty[seg & 1]));
-        // ---- segment end: reduce l and sum_j P'_j mu_j over the token rows
+        // ---- segment end: reduce l over the token rows
         const float lw = warp_reduce16<false>(l_part, lane);
-        const float bw = GATE ? warp_reduce16<false>(bmu_part, lane) : 0.f;
-        if ((lane & 1) == 0) {
-          red_sum[q4 * 32 + (lane >> 1)] = lw;
-          red_sum[q4 * 32 + 16 + (lane >> 1)] = bw;
-        }
+        if ((lane & 1) == 0) red_sum[q4 * 32 + (lane >> 1)] = lw;
         mbar_arrive(smem_u32(&bars.sum));
         if (!warp_wait(smem_u32(&bars.sum), nseg_end & 1, abort_flag)) break;
         ++nseg_end;
-        float lh[16], bh[16];
+        float lh[16];
 #pragma unroll
-        for (int h = 0; h < 16; ++h) {
-          lh[h] = red_sum[h] + red_sum[32 + h] + red_sum[64 + h] + red_sum[96 + h];
-          bh[h] = red_sum[16 + h] + red_sum[48 + h] + red_sum[80 + h] + red_sum[112 + h];
-        }
+        for (int h = 0; h < 16; ++h) lh[h] = red_sum[h] + red_sum[32 + h] + red_sum[64 + h] + red_sum[96 + h];
         // the segment's last PV, then the accumulated latent output
         if (!warp_wait(smem_u32(&bars.o_ready), it & 1, abort_flag)) break;
         tc_fence_after();
@@ -811,7 +576,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (mc == 0 || f >= 128 * mc) {
 #pragma unroll
             for (int h = 0; h < 16; ++h)
-              po[h * D_C + f] = GATE ? fmaf(gam[mc], o[h] - bh[h], bet[mc] * lh[h]) : o[h];
+              po[h * D_C + f] = o[h];
           }
         }
         tc_fence_before();
@@ -838,21 +603,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0 && bars.abort) report_status(p.status, kStatusTimeout);
 }
 
-template <int D_C, bool GATE, bool DUMP>
+template <int D_C>
 cudaError_t launch_one(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_t st) {
-  using C = Cfg<D_C, GATE>;
-  auto kern = decode_tc_kernel<D_C, GATE, DUMP>;
+  using C = Cfg<D_C>;
+  auto kern = decode_tc_kernel<D_C>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
   if (e != cudaSuccess) return e;
   const WorkspaceLayout wl = workspace_layout(a.batch, a.num_splits, kHeads, D_C, kRope, true);
   uint8_t* ws = static_cast<uint8_t*>(a.workspace);
   TcParams p;
-  p.id_pool = a.id_pool;
   p.block_table = a.block_table;
   p.seq_lens = a.seq_lens;
-  p.gate_table = static_cast<const __nv_bfloat16*>(a.gate_table);
-  p.gamma = a.ln_gamma;
-  p.beta = a.ln_beta;
   p.qprep = ws + wl.off_qprep;
   p.cu = reinterpret_cast<const int32_t*>(ws + wl.off_cu);
   p.part_ml = reinterpret_cast<float*>(ws + wl.off_ml);
@@ -861,14 +622,7 @@ cudaError_t launch_one(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_
   p.batch = a.batch;
   p.max_pages = a.max_pages;
   p.num_pages = a.num_pages;
-  p.vocab = a.vocab;
   p.scale_log2 = a.scale_log2;
-  p.eps = a.eps;
-  p.dump_c = static_cast<__nv_bfloat16*>(a.dump_c);
-  p.dump_kr = static_cast<__nv_bfloat16*>(a.dump_kr);
-  p.dump_ids = a.dump_ids;
-  p.dump_g = static_cast<__nv_bfloat16*>(a.dump_g);
-  p.dump_len = a.max_seq_len;
   kern<<<a.num_splits, kThreads, C::SMEM, st>>>(maps[0], maps[1], p);
   return cudaGetLastError();
 }
@@ -876,7 +630,7 @@ cudaError_t launch_one(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_
 }  // namespace
 
 cudaError_t launch_decode_wide(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_t st) {
-  if (a.d_c == 512 && !a.gate) return launch_one<512, false, false>(a, maps, st);
+  if (a.d_c == 512 && !a.gate) return launch_one<512>(a, maps, st);
   return cudaErrorInvalidValue;
 }
 
