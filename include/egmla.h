@@ -161,9 +161,10 @@ size_t eg_mla_decode_workspace_size(const eg_mla_dims* dims, int32_t batch, int3
  *                32-byte aligned for bf16 (read in 32-byte pieces), 16-byte
  *                aligned for fp32
  *   ln_gamma, ln_beta  [d_c] fp32, may be NULL (gamma = 1, beta = 0)
- *   w_uk         [num_heads, d_nope, d_c] model dtype (the k_nope rows of the
- *                listing's wkv_b weight viewed per head), 16-byte aligned
- *   w_uv         [num_heads, d_v, d_c] model dtype (the v rows of wkv_b),
+ *   w_uk         [num_heads, d_nope, d_c] model dtype (the key rows of the
+ *                joint key/value up-projection W^UKV, Appendix C Eq. 2,
+ *                viewed per head), 16-byte aligned
+ *   w_uv         [num_heads, d_v, d_c] model dtype (its value rows),
  *                16-byte aligned
  *   out          [batch, num_heads, d_v] model dtype, written
  *   num_splits   number of split-KV work units (0 = eg_mla_default_num_splits);

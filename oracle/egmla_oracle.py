@@ -249,7 +249,8 @@ def decode_r0(case, w_ukv_full: Optional[np.ndarray] = None, gate_r0: Optional[n
     kv~ = LN_{H(d_n+d_v)}((W^UKV c) (*) g) over all heads at once, split per head
     into k^C, v^C (Eq. 6), then Eqs. 11-13.  ``gate_r0`` [V, H(d_n+d_v)] is the
     precomputed gate in that space and must be given.  W^UKV defaults to stacking
-    W_UK,h and W_UV,h per head, the row order of the listing's wkv_b.
+    W_UK,h and W_UV,h per head (keys, then values, head by head, the row order
+    of the joint up-projection in Appendix E).
     Returns [B, H, d_v]."""
     d = case.dims
     B, H, dn, dv = case.batch, d.num_heads, d.d_nope, d.d_v
