@@ -339,11 +339,11 @@ def test_r0_matches_listing_form():
     gate_r0 = rng.normal(1.0, 0.2, size=(d.vocab, width))
     got = orc.decode_r0(case, gate_r0=gate_r0)
     w_uk, w_uv = orc.widen(case.w_uk, d.dtype), orc.widen(case.w_uv, d.dtype)
-    wkv_b = torch.from_numpy(np.concatenate([w_uk, w_uv], axis=1).reshape(width, d.d_c))
+    w_ukv = torch.from_numpy(np.concatenate([w_uk, w_uv], axis=1).reshape(width, d.d_c))
     for b in range(case.batch):
         L = int(case.seq_lens[b])
         c = torch.from_numpy(case.logical_c[b].astype(np.float64))
-        kv = F.linear(c, wkv_b) * torch.from_numpy(gate_r0)[torch.from_numpy(case.logical_ids[b].astype(np.int64))]
+        kv = F.linear(c, w_ukv) * torch.from_numpy(gate_r0)[torch.from_numpy(case.logical_ids[b].astype(np.int64))]
         kv = F.layer_norm(kv, (width,), eps=d.ln_eps).view(L, d.num_heads, d.d_nope + d.d_v)
         k_nope, v = kv[..., :d.d_nope], kv[..., d.d_nope:]
         kr = torch.from_numpy(case.logical_kr[b].astype(np.float64))
