@@ -288,3 +288,26 @@ def test_workload_layers_full_size_sampled(gpu_lib):
     for layer in (0, 23):
         case = synth.case_layer(layer)
         sampled_check(case, [3, 60])
+
+
+def growing_rope_case(d_c, gate, lens=(3000, 700, 1280), seed=23):
+    """RoPE keys whose scale grows along the sequence (sigma = 1 + 0.02 j at
+    position j): the tile maxima of the scores keep rising, so the online
+    softmax's reference max moves every few tiles of every split."""
+    case = small_bf16(lens, d_c=d_c, gate=gate, seed=seed)
+    kr = synth.bf16_bits_to_f32(case.kr_pool).copy()
+    for b, L in enumerate(case.seq_lens):
+        for lp in range((int(L) + 63) // 64):
+            pos = lp * 64 + np.arange(64)
+            kr[case.block_table[b, lp]] *= (1.0 + 0.02 * pos)[:, None]
+    case.kr_pool = synth.f32_to_bf16_bits(kr)
+    return case
+
+
+@pytest.mark.parametrize("d_c,gate", [(256, True), (192, True), (256, False)])
+def test_rising_scores_move_the_reference_max(gpu_lib, d_c, gate):
+    case = growing_rope_case(d_c, gate)
+    ref = orc.decode_unabsorbed(case)
+    for splits in (1, 3, 0):
+        _, got = run(case, splits)
+        check_bf16(got, ref, f"rising scores d_c={d_c} gate={gate} splits={splits}", scaled_abs=True)
