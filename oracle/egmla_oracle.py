@@ -22,12 +22,16 @@ as ``decode_r0`` for documentation.
 
 Parity status: every function here is pinned by the tests in
 ``tests/test_oracle_pins.py`` (library routines, closed forms, invariants, the
-paper's printed cache sizes).  ``decode_r0`` is pinned only against a PyTorch
+paper's printed cache sizes).  The attention-layer step (``layer_step``,
+``layer_decode``) is pinned by decoding a sequence one token at a time against
+one causal forward pass over the whole sequence written from the listing, and
+its RoPE, RMSNorm and bf16 storage against the corresponding torch routines.  ``decode_r0`` is pinned only against a PyTorch
 re-expression of the paper's listing on tiny inputs (parity unpinned beyond
 that: the paper prints no numeric example).
 """
 from __future__ import annotations
 
+import dataclasses
 import math
 from typing import Iterable, Optional
 
@@ -278,6 +282,88 @@ def decode_r0(case, w_ukv_full: Optional[np.ndarray] = None, gate_r0: Optional[n
             p = softmax((k @ widen(case.q[b, h], d.dtype)) * d.scale())
             out[b, h] = p @ v
     return out
+
+
+# --------------------------------------------------------------------------
+# one decode step through a whole attention layer (Appendix C, Appendix E)
+# --------------------------------------------------------------------------
+def to_bf16_bits(x: np.ndarray) -> np.ndarray:
+    """The bf16 value a model of dtype bf16 stores for x: float64 -> float32 ->
+    bf16, each step rounded to nearest, ties to even (NaN kept as a quiet NaN)."""
+    f = np.ascontiguousarray(np.asarray(x, dtype=np.float64).astype(np.float32))
+    u = f.view(np.uint32).astype(np.uint64)
+    r = ((u + 0x7FFF + ((u >> 16) & 1)) >> 16).astype(np.uint16)
+    nan = np.isnan(f)
+    if nan.any():
+        r[nan] = np.uint16(0x7FC0)
+    return r
+
+
+def store(x: np.ndarray, dtype: str) -> np.ndarray:
+    """A float64 result kept in the model dtype (bf16 bits, or float64 for fp32
+    workloads, whose values the oracle keeps exactly)."""
+    return to_bf16_bits(x) if dtype == "bf16" else np.asarray(x, dtype=np.float64)
+
+
+def rope(x: np.ndarray, pos, theta: float) -> np.ndarray:
+    """Rotary position embedding as the listing applies it (apply_rotary_emb with
+    freqs_cis): consecutive pairs (x_2i, x_2i+1) of the last axis rotated by the
+    angle pos * theta^(-2i/d).  ``pos`` broadcasts against x.shape[:-1]."""
+    x = np.asarray(x, dtype=np.float64)
+    d = x.shape[-1]
+    freq = theta ** (-2.0 * np.arange(d // 2) / d)
+    ang = np.asarray(pos, dtype=np.float64)[..., None] * freq
+    c, s = np.cos(ang), np.sin(ang)
+    x0, x1 = x[..., 0::2], x[..., 1::2]
+    out = np.empty(np.broadcast_shapes(x.shape, ang.shape[:-1] + (d,)), dtype=np.float64)
+    out[..., 0::2] = x0 * c - x1 * s
+    out[..., 1::2] = x0 * s + x1 * c
+    return out
+
+
+def rms_norm(x: np.ndarray, w: np.ndarray, eps: float) -> np.ndarray:
+    """x / sqrt(mean(x^2) + eps) * w over the last axis (the listing's kv_norm)."""
+    x = np.asarray(x, dtype=np.float64)
+    return x / np.sqrt((x * x).mean(axis=-1, keepdims=True) + eps) * np.asarray(w, dtype=np.float64)
+
+
+def layer_step(lc):
+    """The decode-step inputs of the attention (Appendix C with q-LoRA rank 0, as
+    every model of Appendix A): q = W^Q x split per head into [q^C ; q^R] with
+    q^R rotated (Eqs. 8-9), [c^KV ; k^R] = W^{DKV,KR} x (Eqs. 1 and 10) with k^R
+    rotated and c^KV passed through the listing's kv_norm (RMSNorm) before it is
+    cached.  The rotation position of a sequence's new token is L_b - 1.
+    Returns the decode case of this step: the cache plus (q, c_new, kr_new) as
+    the model stores them."""
+    case = lc.case
+    d = case.dims
+    H, dn, dr, dc = d.num_heads, d.d_nope, d.d_rope, d.d_c
+    B = case.batch
+    pos = case.positions().astype(np.float64)
+    x = widen(lc.x, d.dtype)
+    q = (x @ widen(lc.w_q, d.dtype).T).reshape(B, H, dn + dr)
+    q[..., dn:] = rope(q[..., dn:], pos[:, None], lc.rope_theta)
+    kv = x @ widen(lc.w_kv_a, d.dtype).T
+    c = rms_norm(kv[:, :dc], widen(lc.kv_norm_w, d.dtype), lc.rms_eps)
+    kr = rope(kv[:, dc:], pos, lc.rope_theta)
+    return dataclasses.replace(case, q=store(q, d.dtype), c_new=store(c, d.dtype), kr_new=store(kr, d.dtype))
+
+
+def layer_decode(lc, batches: Optional[Iterable[int]] = None) -> np.ndarray:
+    """o_t = W^O [u_t,1 ; ... ; u_t,n_h] (Eq. 14) with u the attention output of
+    ``decode_unabsorbed`` over the cache after this step's append, kept in the
+    model dtype as the layer stores it.  Returns [B, E] float64 (rows of
+    unselected batches NaN)."""
+    step = layer_step(lc)
+    d = step.dims
+    u = decode_unabsorbed(step, batches=batches)
+    B = step.batch
+    y = np.full((B, lc.n_embd), np.nan)
+    bs = range(B) if batches is None else list(batches)
+    w_o = widen(lc.w_o, d.dtype)
+    for b in bs:
+        y[b] = w_o @ widen(store(u[b], d.dtype), d.dtype).reshape(-1)
+    return y
 
 
 # --------------------------------------------------------------------------

@@ -296,3 +296,47 @@ def case_layer(layer: int, seed: int = 4, batch: int = 64, ctx: int = 8192, **kw
 
 
 N_LAYERS = 24
+
+
+# --------------------------------------------------------------------------
+# one full attention layer of a decode step
+# --------------------------------------------------------------------------
+F32_EPS = float(np.finfo(np.float32).eps)
+
+
+@dataclasses.dataclass
+class LayerCase:
+    """Inputs of one decode step through a whole EG-MLA attention layer.
+
+    ``case`` holds the cache (its first ``seq_lens[b]-1`` tokens), the gate
+    table, LayerNorm and absorbed weights; its ``q``/``c_new``/``kr_new`` are
+    not used: the layer derives them from the hidden state ``x``.  Weights have
+    the PyTorch Linear layout [out, in] in the model dtype.
+    """
+    case: Case
+    n_embd: int
+    x: np.ndarray           # [B, E]
+    w_q: np.ndarray         # [H (d_nope + d_rope), E]
+    w_kv_a: np.ndarray      # [d_c + d_rope, E]
+    kv_norm_w: np.ndarray   # [d_c]
+    w_o: np.ndarray         # [E, H d_v]
+    rope_theta: float = 10000.0
+    rms_eps: float = F32_EPS
+
+
+def make_layer_case(case: Case, n_embd: int, *, seed: int, rope_theta: float = 10000.0,
+                    rms_eps: float = F32_EPS) -> LayerCase:
+    """Hidden state N(0, 1) and projection weights N(0, fan_in^-1/2); the
+    RMSNorm weight N(1, 0.1)."""
+    rng = np.random.default_rng(seed)
+    d, dt = case.dims, case.dims.dtype
+    H, dn, dr, dv, dc, E = d.num_heads, d.d_nope, d.d_rope, d.d_v, d.d_c, n_embd
+    B = case.batch
+    return LayerCase(
+        case=case, n_embd=E,
+        x=_store(_normal(rng, (B, E), 1.0), dt),
+        w_q=_store(_normal(rng, (H * (dn + dr), E), 1.0 / math.sqrt(E)), dt),
+        w_kv_a=_store(_normal(rng, (dc + dr, E), 1.0 / math.sqrt(E)), dt),
+        kv_norm_w=_store(_normal(rng, (dc,), 0.1, mean=1.0), dt),
+        w_o=_store(_normal(rng, (E, H * dv), 1.0 / math.sqrt(H * dv)), dt),
+        rope_theta=rope_theta, rms_eps=rms_eps)

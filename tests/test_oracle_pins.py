@@ -438,3 +438,110 @@ def test_planted_scale_and_rope_mistakes_are_caught(monkeypatch):
     case._oracle_appended = None
     assert rel_err(orc.decode_unabsorbed(case), ref) > 1e-6
     case.kr_pool[:] = saved
+
+
+# --------------------------------------------------------------------------- one attention layer
+def _rope_listing(x, pos, theta):
+    """The listing's apply_rotary_emb: pairs viewed as complex numbers, multiplied
+    by freqs_cis = polar(1, pos * theta^(-2i/d))."""
+    d = x.shape[-1]
+    freq = theta ** (-torch.arange(0, d, 2, dtype=torch.float64) / d)
+    ang = pos[..., None] * freq
+    xc = torch.view_as_complex(x.reshape(*x.shape[:-1], d // 2, 2).contiguous())
+    return torch.view_as_real(xc * torch.polar(torch.ones_like(ang), ang)).reshape(x.shape)
+
+
+def test_rope_matches_the_listing_complex_rotation():
+    rng = np.random.default_rng(5)
+    x = rng.standard_normal((3, 4, 64))
+    pos = rng.integers(0, 40000, size=(3, 1)).astype(np.float64)
+    got = orc.rope(x, pos, 10000.0)
+    ref = _rope_listing(torch.from_numpy(x), torch.from_numpy(pos), 10000.0).numpy()
+    assert np.abs(got - ref).max() <= 1e-9 * max(1.0, np.abs(ref).max())
+
+
+def test_rope_scores_depend_only_on_relative_position():
+    rng = np.random.default_rng(6)
+    q, k = rng.standard_normal(64), rng.standard_normal(64)
+    s = [float(orc.rope(q, m, 10000.0) @ orc.rope(k, n, 10000.0)) for m, n in ((5, 2), (105, 102), (8005, 8002))]
+    assert abs(s[0] - s[1]) <= 1e-9 and abs(s[0] - s[2]) <= 1e-9
+    assert abs(s[0] - float(orc.rope(q, 6, 10000.0) @ orc.rope(k, 2, 10000.0))) > 1e-6
+    assert abs(np.linalg.norm(orc.rope(q, 12345, 10000.0)) - np.linalg.norm(q)) <= 1e-12
+
+
+def test_rms_norm_matches_torch():
+    rng = np.random.default_rng(7)
+    x, w = rng.standard_normal((5, 256)) * 3.0, rng.standard_normal(256)
+    ref = F.rms_norm(torch.from_numpy(x), (256,), torch.from_numpy(w), synth.F32_EPS).numpy()
+    assert np.abs(orc.rms_norm(x, w, synth.F32_EPS) - ref).max() <= 1e-12
+
+
+def test_bf16_store_matches_torch_rounding():
+    rng = np.random.default_rng(8)
+    f = np.concatenate([rng.standard_normal(20000) * 10.0 ** rng.integers(-30, 30, 20000),
+                        np.array([0.0, -0.0, 1.0, 1.00390625, 1.01171875, 3.0e38, -3.0e38, 1e-40, np.inf, -np.inf])])
+    f32 = f.astype(np.float32)
+    ref = torch.from_numpy(f32).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(orc.to_bf16_bits(f32), ref)
+
+
+def _tiny_layer_model(seed=9):
+    dims = synth.Dims(num_heads=2, d_nope=8, d_rope=4, d_v=8, d_c=16, page_size=4, vocab=50, dtype="fp32")
+    rng = np.random.default_rng(seed)
+    E, T = 32, 7
+    H, dn, dr, dv, dc = 2, 8, 4, 8, 16
+    w = dict(
+        w_q=rng.standard_normal((H * (dn + dr), E)) / math.sqrt(E),
+        w_kv_a=rng.standard_normal((dc + dr, E)) / math.sqrt(E),
+        kv_norm_w=1.0 + 0.1 * rng.standard_normal(dc),
+        w_o=rng.standard_normal((E, H * dv)) / math.sqrt(H * dv),
+        gate_table=1.0 + 0.1 * rng.standard_normal((dims.vocab, dc)),
+        ln_gamma=1.0 + 0.1 * rng.standard_normal(dc), ln_beta=0.1 * rng.standard_normal(dc),
+        w_uk=rng.standard_normal((H, dn, dc)) / math.sqrt(dc), w_uv=rng.standard_normal((H, dv, dc)) / math.sqrt(dc))
+    xs = rng.standard_normal((T, E))
+    ids = rng.integers(0, dims.vocab, size=T).astype(np.int32)
+    return dims, w, xs, ids
+
+
+def test_layer_steps_match_the_full_sequence_causal_forward():
+    """Decoding T tokens one step at a time through the layer oracle (append,
+    then attend) gives, at every step, the output of one causal forward pass over
+    the whole sequence written from the listing with the gate in latent space
+    (torch float64: complex-rotation RoPE, rms_norm, layer_norm, SDPA)."""
+    dims, w, xs, ids = _tiny_layer_model()
+    T, E = xs.shape
+    H, dn, dr, dv, dc, P = dims.num_heads, dims.d_nope, dims.d_rope, dims.d_v, dims.d_c, dims.page_size
+    pages = (T + P - 1) // P
+    c_pool = np.full((pages, P, dc), np.nan)
+    kr_pool = np.full((pages, P, dr), np.nan)
+    id_pool = np.full((pages, P), -7, dtype=np.int32)
+    ys = []
+    for t in range(T):
+        case = synth.Case(name="steps", dims=dims, seed=0, c_pool=c_pool, kr_pool=kr_pool, id_pool=id_pool,
+                          block_table=np.arange(pages, dtype=np.int32)[None, :],
+                          seq_lens=np.array([t + 1], dtype=np.int32), c_new=np.zeros((1, dc)),
+                          kr_new=np.zeros((1, dr)), ids_new=ids[t:t + 1], q=np.zeros((1, H, dn + dr)),
+                          gate_table=w["gate_table"], ln_gamma=w["ln_gamma"], ln_beta=w["ln_beta"],
+                          w_uk=w["w_uk"], w_uv=w["w_uv"])
+        lc = synth.LayerCase(case=case, n_embd=E, x=xs[t:t + 1], w_q=w["w_q"], w_kv_a=w["w_kv_a"],
+                             kv_norm_w=w["kv_norm_w"], w_o=w["w_o"])
+        ys.append(orc.layer_decode(lc)[0])
+        c_pool, kr_pool, id_pool = orc.appended_pools(orc.layer_step(lc))
+
+    tt = {k: torch.from_numpy(np.asarray(v, dtype=np.float64)) for k, v in w.items()}
+    X = torch.from_numpy(xs)
+    pos = torch.arange(T, dtype=torch.float64)
+    q = (X @ tt["w_q"].T).view(T, H, dn + dr)
+    q_nope, q_pe = q[..., :dn], _rope_listing(q[..., dn:], pos[:, None], 10000.0)
+    kv = X @ tt["w_kv_a"].T
+    c, k_pe = kv[:, :dc], _rope_listing(kv[:, dc:], pos, 10000.0)
+    c = F.rms_norm(c, (dc,), tt["kv_norm_w"], synth.F32_EPS)
+    ct = F.layer_norm(c * tt["gate_table"][torch.from_numpy(ids).long()], (dc,), tt["ln_gamma"], tt["ln_beta"],
+                      dims.ln_eps)
+    k_nope = torch.einsum("tc,hnc->htn", ct, tt["w_uk"])
+    v = torch.einsum("tc,hvc->htv", ct, tt["w_uv"])
+    k = torch.cat([k_nope, k_pe[None].expand(H, T, dr)], dim=-1)
+    qh = torch.cat([q_nope, q_pe], dim=-1).transpose(0, 1)
+    u = F.scaled_dot_product_attention(qh[None], k[None], v[None], is_causal=True)[0]
+    y_ref = (u.transpose(0, 1).reshape(T, H * dv) @ tt["w_o"].T).numpy()
+    assert np.abs(np.stack(ys) - y_ref).max() <= 1e-10
