@@ -228,6 +228,79 @@ int eg_mla_decode_static(const eg_mla_dims* dims, const void* q, const void* c_p
                          int32_t num_splits, int32_t* dev_status, void* stream);
 
 /*
+ * One decode step through a whole EG-MLA attention layer (Appendix C Eqs. 1,
+ * 8-14 with the q-LoRA rank 0 of every model in Appendix A; the listing of
+ * Appendix E for kv_norm and the rotary embedding).  For every sequence b:
+ *
+ *   q      = W^Q x_b                    [H (d_nope + d_rope)], split per head
+ *                                        into [q^C ; q^R]   (Eqs. 8-9, 11)
+ *   [c ; k] = W^{DKV,KR} x_b            [d_c + d_rope]      (Eqs. 1, 10)
+ *   c^KV   = RMSNorm(c) * kv_norm_w     (the listing's kv_norm; what the cache keeps)
+ *   q^R, k^R rotated at position L_b - 1: pair (2i, 2i + 1) by the angle
+ *            pos * theta^(-2i / d_rope) (the listing's apply_rotary_emb)
+ *   append (c^KV, k^R, id) to the cache; u = eg_mla_decode(q, cache)  (Eqs. 2-13)
+ *   y_b    = W^O [u_b,1 ; ... ; u_b,H]  [n_embd]             (Eq. 14)
+ *
+ * bf16 only.  q, c^KV, k^R and u are rounded to bf16 once, from fp32, where
+ * the layer stores them; y is written in bf16.
+ */
+typedef struct {
+  int32_t n_embd;     /* model width E (a multiple of 8) */
+  float rope_theta;   /* rotary base; <= 0 selects 10000 */
+  float rms_eps;      /* kv_norm epsilon; <= 0 selects 2^-23 (the fp32 machine epsilon) */
+} eg_mla_layer_dims;
+
+/* Device pointers of one layer's weights, each 16-byte aligned, in the
+ * PyTorch Linear layout [out, in] of the model dtype (bf16) unless stated. */
+typedef struct {
+  const void* w_q;          /* [H (d_nope + d_rope), E] */
+  const void* w_kv_a;       /* [d_c + d_rope, E] */
+  const void* kv_norm_w;    /* [d_c] */
+  const void* w_o;          /* [E, H d_v] */
+  const void* gate_table;   /* [vocab, d_c]  as for eg_mla_decode */
+  const float* ln_gamma;    /* [d_c] fp32 or NULL, as for eg_mla_decode */
+  const float* ln_beta;     /* [d_c] fp32 or NULL */
+  const void* w_uk;         /* [H, d_nope, d_c] */
+  const void* w_uv;         /* [H, d_v, d_c] */
+} eg_mla_layer_weights;
+
+/* Workspace bytes eg_mla_layer_decode needs (0 on invalid arguments): the
+ * projections' outputs, the decode workspace of eg_mla_decode and a 4 MiB
+ * cuBLAS workspace. */
+size_t eg_mla_layer_workspace_size(const eg_mla_dims* dims, const eg_mla_layer_dims* layer,
+                                   int32_t batch, int32_t num_splits);
+
+/*
+ * eg_mla_layer_decode - the step above for `batch` sequences, on `stream`.
+ *
+ *   x          [batch, E] bf16 hidden states of the new tokens
+ *   ids_new    [batch] int32 token ids of the new tokens (their gate rows)
+ *   positions  [batch] int32 = seq_lens[b] - 1: the new token's slot and its
+ *              rotation position
+ *   c_pool, krope_pool, id_pool, block_table, max_pages_per_seq, seq_lens,
+ *   max_seq_len, num_pages, num_splits, dev_status: as for
+ *              eg_mla_append_latent and eg_mla_decode (seq_lens include the
+ *              new token, so every sequence has L_b >= 1)
+ *   y          [batch, E] bf16 output, caller-owned
+ *   workspace  >= eg_mla_layer_workspace_size(...) bytes, 256-byte aligned
+ *
+ * The projections are plain GEMMs run by cuBLAS on a cuBLAS handle this
+ * library creates once per device, at the first call on that device (make
+ * that first call before any stream capture); every later call allocates
+ * nothing and is capturable.  Calls on one device share that handle: issue
+ * them from one host thread at a time.  Host-side argument errors return a
+ * negative status and launch nothing; device errors go to *dev_status as for
+ * eg_mla_decode.
+ */
+int eg_mla_layer_decode(const eg_mla_dims* dims, const eg_mla_layer_dims* layer,
+                        const eg_mla_layer_weights* weights, const void* x, const int32_t* ids_new,
+                        const int32_t* positions, void* c_pool, void* krope_pool, int32_t* id_pool,
+                        const int32_t* block_table, int32_t max_pages_per_seq, const int32_t* seq_lens,
+                        int32_t max_seq_len, int32_t batch, int32_t num_pages, void* y,
+                        int32_t num_splits, void* workspace, size_t workspace_bytes,
+                        int32_t* dev_status, void* stream);
+
+/*
  * eg_mla_kv_bytes_per_token - bytes the paged cache keeps per token over
  * n_layers layers: (d_c + d_rope) elements of the model dtype per layer
  * (Table 5 with d_c the cached latent width), plus a 4-byte token id per

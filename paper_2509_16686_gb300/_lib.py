@@ -49,6 +49,8 @@ EXPORTED = [
     "eg_mla_profile_begin",
     "eg_mla_profile_end",
     "eg_mla_debug_set_trace",
+    "eg_mla_layer_workspace_size",
+    "eg_mla_layer_decode",
 ]
 
 
@@ -103,6 +105,11 @@ def _declare(lib: ctypes.CDLL) -> None:
     lib.eg_mla_profile_end.restype = ctypes.c_int
     lib.eg_mla_debug_set_trace.argtypes = [P, ctypes.c_int64, I32]
     lib.eg_mla_debug_set_trace.restype = ctypes.c_int
+    LD, LW = ctypes.POINTER(EgMlaLayerDims), ctypes.POINTER(EgMlaLayerWeights)
+    lib.eg_mla_layer_workspace_size.argtypes = [D, LD, I32, I32]
+    lib.eg_mla_layer_workspace_size.restype = SZ
+    lib.eg_mla_layer_decode.argtypes = [D, LD, LW, P, P, P, P, P, P, P, I32, P, I32, I32, I32, P, I32, P, SZ, P, P]
+    lib.eg_mla_layer_decode.restype = ctypes.c_int
 
 
 def library_path() -> str:
@@ -132,6 +139,18 @@ def status_string(code: int) -> str:
 def _check(code: int, where: str) -> None:
     if code != EG_MLA_OK:
         raise EgMlaError(code, where)
+
+class EgMlaLayerDims(ctypes.Structure):
+    _fields_ = [
+        ("n_embd", ctypes.c_int32),
+        ("rope_theta", ctypes.c_float),
+        ("rms_eps", ctypes.c_float),
+    ]
+
+
+class EgMlaLayerWeights(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in ("w_q", "w_kv_a", "kv_norm_w", "w_o", "gate_table", "ln_gamma",
+                                                "ln_beta", "w_uk", "w_uv")]
 
 
 def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
@@ -209,6 +228,34 @@ def eg_mla_decode_static(dims: EgMlaDims, q, c_pool, krope_pool, id_pool, block_
         _ptr(gate_table), _ptr(ln_gamma), _ptr(ln_beta), _ptr(w_uk), _ptr(w_uv), _ptr(out), num_splits,
         _ptr(dev_status), _stream(stream))
     _check(code, "eg_mla_decode_static")
+
+
+def make_layer_dims(n_embd: int, rope_theta: float = 10000.0, rms_eps: float = 0.0) -> EgMlaLayerDims:
+    return EgMlaLayerDims(n_embd, rope_theta, rms_eps)
+
+
+def make_layer_weights(w_q, w_kv_a, kv_norm_w, w_o, gate_table, ln_gamma, ln_beta, w_uk, w_uv) -> EgMlaLayerWeights:
+    return EgMlaLayerWeights(*[_ptr(t) for t in (w_q, w_kv_a, kv_norm_w, w_o, gate_table, ln_gamma, ln_beta,
+                                                 w_uk, w_uv)])
+
+
+def eg_mla_layer_workspace_size(dims: EgMlaDims, layer: EgMlaLayerDims, batch: int, num_splits: int = 0) -> int:
+    n = load().eg_mla_layer_workspace_size(ctypes.byref(dims), ctypes.byref(layer), batch, num_splits)
+    if n == 0:
+        raise EgMlaError(EG_MLA_ERR_UNSUPPORTED, "eg_mla_layer_workspace_size")
+    return int(n)
+
+
+def eg_mla_layer_decode(dims: EgMlaDims, layer: EgMlaLayerDims, weights: EgMlaLayerWeights, x, ids_new, positions,
+                        c_pool, krope_pool, id_pool, block_table, seq_lens, max_seq_len, y, workspace,
+                        num_splits=0, dev_status=None, stream=None) -> None:
+    """One decode step through a whole attention layer (see include/egmla.h)."""
+    code = load().eg_mla_layer_decode(
+        ctypes.byref(dims), ctypes.byref(layer), ctypes.byref(weights), _ptr(x), _ptr(ids_new), _ptr(positions),
+        _ptr(c_pool), _ptr(krope_pool), _ptr(id_pool), _ptr(block_table), block_table.shape[1], _ptr(seq_lens),
+        int(max_seq_len), seq_lens.shape[0], c_pool.shape[0], _ptr(y), num_splits, _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _ptr(dev_status), _stream(stream))
+    _check(code, "eg_mla_layer_decode")
 
 
 def bind_step(dims: EgMlaDims, c_pool, krope_pool, id_pool, c_new, krope_new, ids_new, positions, q, block_table,

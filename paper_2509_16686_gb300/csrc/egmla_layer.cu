@@ -1,0 +1,204 @@
+// egmla_layer.cu - one decode step through a whole EG-MLA attention layer:
+// the query and latent projections, the latent's RMSNorm and the rotary
+// embedding of q^R and k^R (one fused kernel), the cache append and the
+// gated latent attention of egmla_api.cu, and the output projection.  The
+// three projections are plain GEMMs and run in cuBLAS; everything between
+// them runs in this library's kernels.  See include/egmla.h for the contract.
+#include <cublas_v2.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+#include <mutex>
+
+#include "../../include/egmla.h"
+
+namespace {
+
+constexpr size_t kCublasWorkspace = size_t(4) << 20;
+constexpr int kMaxDevices = 64;
+constexpr int kQkvThreads = 256;
+
+size_t up256(size_t x) { return (x + 255) / 256 * 256; }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+struct LayerWorkspace {
+  size_t off_cublas, off_q32, off_kv32, off_q, off_c, off_kr, off_u, off_dec, dec_bytes, total;
+};
+
+// carve of the layer workspace (every piece 256-byte aligned); dec_bytes = 0 on
+// invalid decode arguments
+LayerWorkspace layer_workspace(const eg_mla_dims* d, int32_t n_embd, int32_t batch, int32_t num_splits) {
+  LayerWorkspace w{};
+  const size_t B = static_cast<size_t>(batch > 0 ? batch : 0);
+  const size_t nq = static_cast<size_t>(d->num_heads) * (d->d_nope + d->d_rope);
+  const size_t nkv = static_cast<size_t>(d->d_c + d->d_rope);
+  (void)n_embd;
+  size_t off = 0;
+  w.off_cublas = off;
+  off += kCublasWorkspace;
+  w.off_q32 = off;
+  off = up256(off + B * nq * 4);
+  w.off_kv32 = off;
+  off = up256(off + B * nkv * 4);
+  w.off_q = off;
+  off = up256(off + B * nq * 2);
+  w.off_c = off;
+  off = up256(off + B * d->d_c * 2);
+  w.off_kr = off;
+  off = up256(off + B * d->d_rope * 2);
+  w.off_u = off;
+  off = up256(off + B * d->num_heads * d->d_v * 2);
+  w.off_dec = off;
+  w.dec_bytes = eg_mla_decode_workspace_size(d, batch, num_splits);
+  w.total = up256(off + w.dec_bytes);
+  return w;
+}
+
+// One cuBLAS handle per device, created at the first call with that device
+// current, and a lock that keeps one host thread at a time on it.
+struct Handles {
+  std::mutex mu;
+  cublasHandle_t h[kMaxDevices] = {};
+};
+Handles g_handles;
+
+// The new token's kv_norm and rotary embedding (one CTA per sequence):
+//   c^KV = c / sqrt(mean(c^2) + eps) * w,  k^R and every head's q^R rotated,
+//   pair (2i, 2i + 1) by the angle pos * theta^(-2i / d_rope).
+// Inputs are the fp32 GEMM outputs; each result is rounded to bf16 once.  The
+// angle and its sine and cosine are taken in double precision, so positions
+// in the tens of thousands keep full fp32 accuracy in the rotation.
+__global__ void __launch_bounds__(kQkvThreads) layer_qkv_kernel(
+    const float* __restrict__ q32, const float* __restrict__ kv32, const int32_t* __restrict__ positions,
+    const __nv_bfloat16* __restrict__ kv_norm_w, int H, int dn, int dr, int dc, double theta, float eps,
+    __nv_bfloat16* __restrict__ q_out, __nv_bfloat16* __restrict__ c_out, __nv_bfloat16* __restrict__ kr_out) {
+  __shared__ float red[kQkvThreads / 32];
+  const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int dq = dn + dr;
+  const float* kv = kv32 + static_cast<size_t>(b) * (dc + dr);
+  const float* q = q32 + static_cast<size_t>(b) * H * dq;
+  __nv_bfloat16* qo = q_out + static_cast<size_t>(b) * H * dq;
+
+  // kv_norm: the mean of c^2 over d_c (warp sums, then the warps' sums in order)
+  float ss = 0.f;
+  for (int f = tid; f < dc; f += blockDim.x) ss = fmaf(kv[f], kv[f], ss);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  if (lane == 0) red[warp] = ss;
+  __syncthreads();
+  float tot = 0.f;
+  for (int i = 0; i < static_cast<int>(blockDim.x / 32); ++i) tot += red[i];
+  const float r = 1.f / sqrtf(tot / static_cast<float>(dc) + eps);
+  for (int f = tid; f < dc; f += blockDim.x)
+    c_out[static_cast<size_t>(b) * dc + f] = __float2bfloat16_rn(kv[f] * r * __bfloat162float(kv_norm_w[f]));
+
+  // q^C of every head, rounded
+  for (int e = tid; e < H * dq; e += blockDim.x)
+    if (e % dq < dn) qo[e] = __float2bfloat16_rn(q[e]);
+
+  // rotary embedding: thread i owns pair i of k^R and of every head's q^R
+  const double pos = static_cast<double>(positions[b]);
+  for (int i = tid; i < dr / 2; i += blockDim.x) {
+    double sd, cd;
+    sincos(pos * pow(theta, -2.0 * i / dr), &sd, &cd);
+    const float sn = static_cast<float>(sd), cs = static_cast<float>(cd);
+    const float k0 = kv[dc + 2 * i], k1 = kv[dc + 2 * i + 1];
+    kr_out[static_cast<size_t>(b) * dr + 2 * i] = __float2bfloat16_rn(k0 * cs - k1 * sn);
+    kr_out[static_cast<size_t>(b) * dr + 2 * i + 1] = __float2bfloat16_rn(k0 * sn + k1 * cs);
+    for (int h = 0; h < H; ++h) {
+      const float x0 = q[h * dq + dn + 2 * i], x1 = q[h * dq + dn + 2 * i + 1];
+      qo[h * dq + dn + 2 * i] = __float2bfloat16_rn(x0 * cs - x1 * sn);
+      qo[h * dq + dn + 2 * i + 1] = __float2bfloat16_rn(x0 * sn + x1 * cs);
+    }
+  }
+}
+
+// C[m, n] (column-major, ld m) = A^T B with A [k, m] and B [k, n] column-major,
+// i.e. row-major out[n][m] = in[n][:] . W[m][:] for a Linear weight W [m, k]
+cublasStatus_t linear(cublasHandle_t h, int m, int n, int k, const void* w, const void* in, void* out,
+                      cudaDataType_t out_type) {
+  const float one = 1.f, zero = 0.f;
+  return cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, m, n, k, &one, w, CUDA_R_16BF, k, in, CUDA_R_16BF, k, &zero, out,
+                      out_type, m, CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT);
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t eg_mla_layer_workspace_size(const eg_mla_dims* dims, const eg_mla_layer_dims* layer, int32_t batch,
+                                   int32_t num_splits) {
+  if (dims == nullptr || layer == nullptr || batch < 0 || layer->n_embd <= 0) return 0;
+  if (dims->dtype != EG_MLA_BF16) return 0;
+  const LayerWorkspace w = layer_workspace(dims, layer->n_embd, batch, num_splits);
+  return w.dec_bytes == 0 ? 0 : w.total;
+}
+
+int eg_mla_layer_decode(const eg_mla_dims* dims, const eg_mla_layer_dims* layer, const eg_mla_layer_weights* wt,
+                        const void* x, const int32_t* ids_new, const int32_t* positions, void* c_pool,
+                        void* krope_pool, int32_t* id_pool, const int32_t* block_table, int32_t max_pages_per_seq,
+                        const int32_t* seq_lens, int32_t max_seq_len, int32_t batch, int32_t num_pages, void* y,
+                        int32_t num_splits, void* workspace, size_t workspace_bytes, int32_t* dev_status,
+                        void* stream) {
+  if (dims == nullptr || layer == nullptr || wt == nullptr) return EG_MLA_ERR_INVALID_ARG;
+  if (dims->dtype != EG_MLA_BF16) return EG_MLA_ERR_UNSUPPORTED;
+  if (batch < 0 || num_splits < 0 || layer->n_embd <= 0) return EG_MLA_ERR_INVALID_ARG;
+  if (layer->n_embd % 8 || dims->d_rope % 2) return EG_MLA_ERR_UNSUPPORTED;
+  if (batch == 0) return EG_MLA_OK;
+  if (!x || !positions || !y || !workspace || !wt->w_q || !wt->w_kv_a || !wt->kv_norm_w || !wt->w_o)
+    return EG_MLA_ERR_INVALID_ARG;
+  if (!aligned16(x) || !aligned16(y) || !aligned16(wt->w_q) || !aligned16(wt->w_kv_a) || !aligned16(wt->w_o))
+    return EG_MLA_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255) != 0) return EG_MLA_ERR_INVALID_ARG;
+  const LayerWorkspace ws = layer_workspace(dims, layer->n_embd, batch, num_splits);
+  if (ws.dec_bytes == 0) return EG_MLA_ERR_INVALID_ARG;
+  if (workspace_bytes < ws.total) return EG_MLA_ERR_WORKSPACE;
+  uint8_t* base = static_cast<uint8_t*>(workspace);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int H = dims->num_heads, E = layer->n_embd;
+  const int nq = H * (dims->d_nope + dims->d_rope), nkv = dims->d_c + dims->d_rope, nu = H * dims->d_v;
+  const double theta = layer->rope_theta > 0.f ? static_cast<double>(layer->rope_theta) : 10000.0;
+  const float eps = layer->rms_eps > 0.f ? layer->rms_eps : 1.1920928955078125e-07f;
+  void* q32 = base + ws.off_q32;
+  void* kv32 = base + ws.off_kv32;
+  auto* qb = reinterpret_cast<__nv_bfloat16*>(base + ws.off_q);
+  auto* cb = reinterpret_cast<__nv_bfloat16*>(base + ws.off_c);
+  auto* krb = reinterpret_cast<__nv_bfloat16*>(base + ws.off_kr);
+  void* ub = base + ws.off_u;
+
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return EG_MLA_ERR_CUDA;
+  std::lock_guard<std::mutex> lk(g_handles.mu);
+  cublasHandle_t& h = g_handles.h[dev];
+  if (h == nullptr && cublasCreate(&h) != CUBLAS_STATUS_SUCCESS) {
+    h = nullptr;
+    return EG_MLA_ERR_CUDA;
+  }
+  if (cublasSetStream(h, st) != CUBLAS_STATUS_SUCCESS ||
+      cublasSetWorkspace(h, base + ws.off_cublas, kCublasWorkspace) != CUBLAS_STATUS_SUCCESS)
+    return EG_MLA_ERR_CUDA;
+  // Eqs. 8-9 and 1, 10: the query and the latent + RoPE-key projections (fp32 out)
+  if (linear(h, nq, batch, E, wt->w_q, x, q32, CUDA_R_32F) != CUBLAS_STATUS_SUCCESS ||
+      linear(h, nkv, batch, E, wt->w_kv_a, x, kv32, CUDA_R_32F) != CUBLAS_STATUS_SUCCESS)
+    return EG_MLA_ERR_CUDA;
+  layer_qkv_kernel<<<batch, kQkvThreads, 0, st>>>(
+      static_cast<const float*>(q32), static_cast<const float*>(kv32), positions,
+      static_cast<const __nv_bfloat16*>(wt->kv_norm_w), H, dims->d_nope, dims->d_rope, dims->d_c, theta, eps, qb, cb,
+      krb);
+  if (cudaGetLastError() != cudaSuccess) return EG_MLA_ERR_CUDA;
+  int rc = eg_mla_append_latent(dims, c_pool, krope_pool, id_pool, cb, krb, ids_new, block_table, max_pages_per_seq,
+                                positions, batch, num_pages, dev_status, stream);
+  if (rc != EG_MLA_OK) return rc;
+  rc = eg_mla_decode(dims, qb, c_pool, krope_pool, id_pool, block_table, max_pages_per_seq, seq_lens, max_seq_len,
+                     batch, num_pages, wt->gate_table, wt->ln_gamma, wt->ln_beta, wt->w_uk, wt->w_uv, ub, num_splits,
+                     base + ws.off_dec, ws.dec_bytes, dev_status, stream);
+  if (rc != EG_MLA_OK) return rc;
+  // Eq. 14: the output projection of the heads' concatenated outputs
+  if (linear(h, E, batch, nu, wt->w_o, ub, y, CUDA_R_16BF) != CUBLAS_STATUS_SUCCESS) return EG_MLA_ERR_CUDA;
+  return EG_MLA_OK;
+}
+
+}  // extern "C"

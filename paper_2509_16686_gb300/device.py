@@ -162,3 +162,47 @@ def pack_step_inputs(dc: DeviceCase, names=STEP_INPUTS):
 
 def output_f64(t: torch.Tensor) -> np.ndarray:
     return t.detach().float().cpu().numpy().astype(np.float64)
+
+
+@dataclasses.dataclass
+class DeviceLayer:
+    """One attention layer's decode step on the device: the cache and decode
+    inputs of ``dc`` plus the hidden state, the projection weights, the output
+    and the layer workspace."""
+    dc: DeviceCase
+    layer_dims: _lib.EgMlaLayerDims
+    x: torch.Tensor
+    w_q: torch.Tensor
+    w_kv_a: torch.Tensor
+    kv_norm_w: torch.Tensor
+    w_o: torch.Tensor
+    y: torch.Tensor
+    workspace: torch.Tensor
+
+    def weights(self) -> _lib.EgMlaLayerWeights:
+        dc = self.dc
+        return _lib.make_layer_weights(self.w_q, self.w_kv_a, self.kv_norm_w, self.w_o, dc.gate_table, dc.ln_gamma,
+                                       dc.ln_beta, dc.w_uk, dc.w_uv)
+
+    def step(self, stream=None) -> torch.Tensor:
+        """x -> y: projections, kv_norm and RoPE, append, decode, output projection."""
+        dc = self.dc
+        _lib.eg_mla_layer_decode(dc.dims, self.layer_dims, self.weights(), self.x, dc.ids_new, dc.positions,
+                                 dc.c_pool, dc.kr_pool, dc.id_pool, dc.block_table, dc.seq_lens, dc.max_seq_len,
+                                 self.y, self.workspace, dc.num_splits, dc.status, stream)
+        return self.y
+
+
+def upload_layer(lc, device="cuda", num_splits: int = 0) -> DeviceLayer:
+    """A synth.LayerCase on the device (bf16)."""
+    dc = upload(lc.case, device=device, num_splits=num_splits)
+    dt = lc.case.dims.dtype
+    ld = _lib.make_layer_dims(lc.n_embd, lc.rope_theta, lc.rms_eps)
+    ws = _lib.eg_mla_layer_workspace_size(dc.dims, ld, dc.batch, num_splits)
+    return DeviceLayer(
+        dc=dc, layer_dims=ld,
+        x=to_device_array(lc.x, dt, device), w_q=to_device_array(lc.w_q, dt, device),
+        w_kv_a=to_device_array(lc.w_kv_a, dt, device), kv_norm_w=to_device_array(lc.kv_norm_w, dt, device),
+        w_o=to_device_array(lc.w_o, dt, device),
+        y=torch.empty((dc.batch, lc.n_embd), dtype=torch.bfloat16, device=device),
+        workspace=torch.empty(ws, dtype=torch.uint8, device=device))
