@@ -2,6 +2,7 @@
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c32k] [--impl reference]
     python bench.py --sweep        (decode throughput vs context length)
+    python bench.py --workload layers24_full   (24 whole attention layers per step)
 
 A step is one pass of the whole decode hot path for one batch: append of each
 sequence's new token to the paged latent cache, query absorption, the split-KV
@@ -59,7 +60,8 @@ def parse():
     ap.add_argument("--steps", type=int, default=None,
                     help="timed steps (default 20000; 200 for layers24, 2000 per length for --sweep)")
     ap.add_argument("--warmup", type=int, default=30)
-    ap.add_argument("--workload", default="c32k", choices=["c32k", "c4k", "ragged", "ragged_mla", "layers24"])
+    ap.add_argument("--workload", default="c32k",
+                    choices=["c32k", "c4k", "ragged", "ragged_mla", "layers24", "layers24_full"])
     ap.add_argument("--sweep", action="store_true",
                     help="decode throughput vs context length: batch 8, d_c 256, L = 1K .. 64K, one line per L")
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
@@ -84,6 +86,13 @@ def make_workload(name):
     elif name == "ragged_mla":
         case = synth.case_ragged(gate=False, keep_logical=False)
         desc = "ragged_mla: plain-MLA baseline (gate off) at d_c 512 on the ragged lengths"
+    elif name == "layers24_full":
+        case = synth.case_layer(0)
+        desc = "layers24_full: decoder step over 24 full attention layers (hidden 2048: W^Q and W^DKV,KR " \
+               "projections in cuBLAS, fused kv_norm + RoPE, append, gated latent attention, W^O in cuBLAS; " \
+               "each layer's output is the next layer's input), batch 64 x context 8192, 16 heads, d_c 256, " \
+               "d_rope 64, vocab 50000, contiguous pages; layer 0's seeded synthetic cache, ids, gate table and " \
+               "weights cloned into 24 distinct device copies"
     elif name == "layers24":
         case = synth.case_layer(0)
         desc = "layers24: decoder step over 24 attention layers (append + decode per layer on one stream), " \
@@ -97,7 +106,7 @@ def make_workload(name):
 
 
 def layers_of(name):
-    return 24 if name == "layers24" else 1
+    return 24 if name.startswith("layers24") else 1
 
 
 SWEEP_CTX = (1024, 2048, 4096, 8192, 16384, 32768, 65536)
@@ -283,8 +292,144 @@ def kernel_source_sha(files):
     return h.hexdigest()[:16]
 
 
+def run_gpu_full_layers(args, workload, torch, dist, ws, rank):
+    """The 24-layer decoder step through whole attention layers (eg_mla_layer_decode
+    per layer, each layer's output the next one's input)."""
+    from oracle import egmla_oracle as orc
+    from paper_2509_16686_gb300 import _lib, device, synth
+    dev = torch.cuda.current_device()
+    case, desc = make_workload(workload)
+    lc = synth.make_layer_case(case, 2048, seed=5)
+    n_layers = layers_of(workload)
+    B, d = case.batch, case.dims
+    base = device.upload_layer(lc, num_splits=args.splits)
+    layers = [base] + [device.clone_layer(base) for _ in range(n_layers - 1)]
+    for k in range(1, n_layers):
+        layers[k].x = layers[k - 1].y          # the residual stream is left out: attention layers only
+        for name in ("ids_new", "positions", "seq_lens"):   # one step's token ids and lengths, shared
+            setattr(layers[k].dc, name, getattr(base.dc, name))
+    steps_arg = args.steps if args.steps is not None else 200
+    stream = torch.cuda.Stream()
+    tokens_cached = int(case.seq_lens.astype(np.int64).sum())
+    cache_bytes = tokens_cached * ((d.d_c + d.d_rope) * 2 + 4)
+    splits = base.dc.num_splits or _lib.eg_mla_default_num_splits()
+
+    def run_step():
+        for layer in layers:
+            layer.step(stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, args.warmup)):
+            run_step()
+    stream.synchronize()
+    assert base.dc.read_status() == 0, "device status after warm-up"
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        run_step()
+    with torch.cuda.stream(stream):
+        graph.replay()
+        graph.replay()
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(nvsmi_id(torch, dev)) as clk:
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize()
+        with torch.cuda.stream(stream):
+            ev0.record(stream)
+            for _ in range(steps_arg):
+                graph.replay()
+            ev1.record(stream)
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+    elapsed_ms = max_over_ranks(ev0.elapsed_time(ev1), dist, "cuda")
+    assert base.dc.read_status() == 0, "device status after timed region"
+    value = whole_job_rate(ws, B, steps_arg, elapsed_ms)
+
+    # the decode kernel alone, as in run_gpu: events around its launches in a captured step
+    _lib.eg_mla_profile_begin(2 * n_layers)
+    pgraph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(pgraph, stream=stream):
+        run_step()
+        run_step()
+    with torch.cuda.stream(stream):
+        pgraph.replay()
+        pgraph.replay()
+    stream.synchronize()
+    del pgraph
+    ms_sum, n_l = _lib.eg_mla_profile_end()
+    k_ms = ms_sum / max(1, n_l)
+    achieved = cache_bytes / (k_ms * 1e-3) / 1e9
+    peaks_path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(peaks_path):
+        peak, peak_src = float(json.load(open(peaks_path))["hbm_gbs"]), "measured"
+    else:
+        peak, peak_src = 6800.0, "fallback"
+
+    # end to end through the C ABI from pinned host buffers: every step copies in
+    # the new tokens' hidden states, ids and positions and reads back the last
+    # layer's output
+    x0 = base.x.clone()
+    base.x = x0
+    ins = [x0, base.dc.ids_new, base.dc.positions, base.dc.seq_lens]
+    h_ins = [t.cpu().pin_memory() for t in ins]
+    h_out = torch.empty(layers[-1].y.shape, dtype=layers[-1].y.dtype).pin_memory()
+    e2e_steps = args.e2e_steps or min(steps_arg, 100)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(e2e_steps):
+            for dst, src in zip(ins, h_ins):
+                dst.copy_(src, non_blocking=True)
+            run_step()
+            h_out.copy_(layers[-1].y, non_blocking=True)
+        e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), dist, "cuda")
+    assert base.dc.read_status() == 0, "device status after end-to-end run"
+    h2d = sum(t.numel() * t.element_size() for t in h_ins)
+    d2h = h_out.numel() * h_out.element_size()
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        t0 = time.perf_counter()
+        done = 0
+        while done < B and (done == 0 or time.perf_counter() - t0 < 12.0):
+            orc.layer_decode(lc, batches=[done])
+            done += 1
+        dt = time.perf_counter() - t0
+        cpu = {"value": done / dt / n_layers, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
+               "sample": f"the layer oracle on {done} sequence(s) of one layer at full context, {dt:.1f} s "
+                         f"(rate / {n_layers} layers)"}
+    return {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": steps_arg, "warmup": args.warmup,
+        "ms_per_step": elapsed_ms / steps_arg, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": desc, "batch": B, "layers": n_layers, "n_embd": 2048,
+                   "ctx_tokens_cached": tokens_cached, "splits": splits, "page_size": d.page_size,
+                   "l2": f"inputs larger than L2: {n_layers} layers' distinct caches of {cache_bytes / 1e6:.0f} MB "
+                         f"and weights", "graph": "step replayed from a CUDA graph"},
+        "kv_cache_gbs": n_layers * cache_bytes * steps_arg / (elapsed_ms / 1e3) / 1e9,
+        "kv_bytes_per_token": (d.d_c + d.d_rope) * 2 + 4,
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                     "traffic": None, "kernel": "decode_tc_kernel", "kernel_ms": k_ms,
+                     "bytes_per_launch": cache_bytes, "peak_source": peak_src},
+        "cpu_baseline": cpu,
+        "e2e": {"value": whole_job_rate(ws, B, e2e_steps, e2e_ms), "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        # this library's kernels per layer: kv_norm + RoPE, append, query absorption,
+        # decode (the three projection GEMMs are cuBLAS kernels, not counted)
+        "gpu_launches": steps_arg * n_layers * 4,
+        "clocks": clk.summary(),
+    }
+
+
 def run_gpu(args, workload, torch, dist, ws, rank):
     """One bench line of `workload` (see the module docstring)."""
+    if workload == "layers24_full":
+        return run_gpu_full_layers(args, workload, torch, dist, ws, rank)
     from paper_2509_16686_gb300 import _lib, device  # noqa: F401
     dev = torch.cuda.current_device()
     case, desc = make_workload(workload)

@@ -253,8 +253,8 @@ typedef struct {
 /* Device pointers of one layer's weights, each 16-byte aligned, in the
  * PyTorch Linear layout [out, in] of the model dtype (bf16) unless stated. */
 typedef struct {
-  const void* w_q;          /* [H (d_nope + d_rope), E] */
-  const void* w_kv_a;       /* [d_c + d_rope, E] */
+  const void* w_qkv_a;      /* [H (d_nope + d_rope) + d_c + d_rope, E]: the rows of
+                               W^Q, then those of W^{DKV,KR} (one projection GEMM) */
   const void* kv_norm_w;    /* [d_c] */
   const void* w_o;          /* [E, H d_v] */
   const void* gate_table;   /* [vocab, d_c]  as for eg_mla_decode */

@@ -149,8 +149,8 @@ class EgMlaLayerDims(ctypes.Structure):
 
 
 class EgMlaLayerWeights(ctypes.Structure):
-    _fields_ = [(n, ctypes.c_void_p) for n in ("w_q", "w_kv_a", "kv_norm_w", "w_o", "gate_table", "ln_gamma",
-                                                "ln_beta", "w_uk", "w_uv")]
+    _fields_ = [(n, ctypes.c_void_p) for n in ("w_qkv_a", "kv_norm_w", "w_o", "gate_table", "ln_gamma", "ln_beta",
+                                                "w_uk", "w_uv")]
 
 
 def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
@@ -234,9 +234,9 @@ def make_layer_dims(n_embd: int, rope_theta: float = 10000.0, rms_eps: float = 0
     return EgMlaLayerDims(n_embd, rope_theta, rms_eps)
 
 
-def make_layer_weights(w_q, w_kv_a, kv_norm_w, w_o, gate_table, ln_gamma, ln_beta, w_uk, w_uv) -> EgMlaLayerWeights:
-    return EgMlaLayerWeights(*[_ptr(t) for t in (w_q, w_kv_a, kv_norm_w, w_o, gate_table, ln_gamma, ln_beta,
-                                                 w_uk, w_uv)])
+def make_layer_weights(w_qkv_a, kv_norm_w, w_o, gate_table, ln_gamma, ln_beta, w_uk, w_uv) -> EgMlaLayerWeights:
+    """w_qkv_a: the rows of W^Q stacked on those of W^{DKV,KR} ([nq + d_c + d_rope, E])."""
+    return EgMlaLayerWeights(*[_ptr(t) for t in (w_qkv_a, kv_norm_w, w_o, gate_table, ln_gamma, ln_beta, w_uk, w_uv)])
 
 
 def eg_mla_layer_workspace_size(dims: EgMlaDims, layer: EgMlaLayerDims, batch: int, num_splits: int = 0) -> int:

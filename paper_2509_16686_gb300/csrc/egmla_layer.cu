@@ -25,7 +25,7 @@ size_t up256(size_t x) { return (x + 255) / 256 * 256; }
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
 struct LayerWorkspace {
-  size_t off_cublas, off_q32, off_kv32, off_q, off_c, off_kr, off_u, off_dec, dec_bytes, total;
+  size_t off_cublas, off_qkv32, off_q, off_c, off_kr, off_u, off_dec, dec_bytes, total;
 };
 
 // carve of the layer workspace (every piece 256-byte aligned); dec_bytes = 0 on
@@ -39,10 +39,8 @@ LayerWorkspace layer_workspace(const eg_mla_dims* d, int32_t n_embd, int32_t bat
   size_t off = 0;
   w.off_cublas = off;
   off += kCublasWorkspace;
-  w.off_q32 = off;
-  off = up256(off + B * nq * 4);
-  w.off_kv32 = off;
-  off = up256(off + B * nkv * 4);
+  w.off_qkv32 = off;
+  off = up256(off + B * (nq + nkv) * 4);
   w.off_q = off;
   off = up256(off + B * nq * 2);
   w.off_c = off;
@@ -69,50 +67,63 @@ Handles g_handles;
 //   c^KV = c / sqrt(mean(c^2) + eps) * w,  k^R and every head's q^R rotated,
 //   pair (2i, 2i + 1) by the angle pos * theta^(-2i / d_rope).
 // Inputs are the fp32 GEMM outputs; each result is rounded to bf16 once.  The
-// angle and its sine and cosine are taken in double precision, so positions
-// in the tens of thousands keep full fp32 accuracy in the rotation.
+// d_rope / 2 angles are formed and reduced to [-pi, pi] in double precision
+// (the frequencies theta^(-2i/d_rope) come from the host in double), so that
+// positions in the tens of thousands keep full fp32 accuracy in the rotation;
+// sine and cosine of the reduced angle are taken in fp32, once per sequence,
+// and shared through shared memory.  The rotations of the heads' q^R and of
+// k^R are spread over all threads.
+constexpr int kMaxRopePairs = 64;
+
+struct RopeFreqs {
+  double f[kMaxRopePairs];
+};
+
 __global__ void __launch_bounds__(kQkvThreads) layer_qkv_kernel(
-    const float* __restrict__ q32, const float* __restrict__ kv32, const int32_t* __restrict__ positions,
-    const __nv_bfloat16* __restrict__ kv_norm_w, int H, int dn, int dr, int dc, double theta, float eps,
+    const float* __restrict__ qkv32, const int32_t* __restrict__ positions,
+    const __nv_bfloat16* __restrict__ kv_norm_w, int H, int dn, int dr, int dc, const RopeFreqs freqs, float eps,
     __nv_bfloat16* __restrict__ q_out, __nv_bfloat16* __restrict__ c_out, __nv_bfloat16* __restrict__ kr_out) {
   __shared__ float red[kQkvThreads / 32];
+  __shared__ float cs_s[kMaxRopePairs], sn_s[kMaxRopePairs];
   const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int dq = dn + dr;
-  const float* kv = kv32 + static_cast<size_t>(b) * (dc + dr);
-  const float* q = q32 + static_cast<size_t>(b) * H * dq;
+  const int dq = dn + dr, np = dr / 2;
+  const float* q = qkv32 + static_cast<size_t>(b) * (H * dq + dc + dr);   // [q (H dq) | c (dc) | k^R (dr)]
+  const float* kv = q + H * dq;
   __nv_bfloat16* qo = q_out + static_cast<size_t>(b) * H * dq;
 
+  if (tid < np) {
+    constexpr double kTwoPi = 6.283185307179586, kInvTwoPi = 0.15915494309189535;
+    const double ang = static_cast<double>(positions[b]) * freqs.f[tid];
+    const double red_ang = fma(-rint(ang * kInvTwoPi), kTwoPi, ang);
+    float sn, cs;
+    sincosf(static_cast<float>(red_ang), &sn, &cs);
+    sn_s[tid] = sn;
+    cs_s[tid] = cs;
+  }
   // kv_norm: the mean of c^2 over d_c (warp sums, then the warps' sums in order)
   float ss = 0.f;
   for (int f = tid; f < dc; f += blockDim.x) ss = fmaf(kv[f], kv[f], ss);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
   if (lane == 0) red[warp] = ss;
+  // q^C of every head, rounded
+  for (int e = tid; e < H * dq; e += blockDim.x)
+    if (e % dq < dn) qo[e] = __float2bfloat16_rn(q[e]);
   __syncthreads();
   float tot = 0.f;
   for (int i = 0; i < static_cast<int>(blockDim.x / 32); ++i) tot += red[i];
   const float r = 1.f / sqrtf(tot / static_cast<float>(dc) + eps);
   for (int f = tid; f < dc; f += blockDim.x)
     c_out[static_cast<size_t>(b) * dc + f] = __float2bfloat16_rn(kv[f] * r * __bfloat162float(kv_norm_w[f]));
-
-  // q^C of every head, rounded
-  for (int e = tid; e < H * dq; e += blockDim.x)
-    if (e % dq < dn) qo[e] = __float2bfloat16_rn(q[e]);
-
-  // rotary embedding: thread i owns pair i of k^R and of every head's q^R
-  const double pos = static_cast<double>(positions[b]);
-  for (int i = tid; i < dr / 2; i += blockDim.x) {
-    double sd, cd;
-    sincos(pos * pow(theta, -2.0 * i / dr), &sd, &cd);
-    const float sn = static_cast<float>(sd), cs = static_cast<float>(cd);
-    const float k0 = kv[dc + 2 * i], k1 = kv[dc + 2 * i + 1];
-    kr_out[static_cast<size_t>(b) * dr + 2 * i] = __float2bfloat16_rn(k0 * cs - k1 * sn);
-    kr_out[static_cast<size_t>(b) * dr + 2 * i + 1] = __float2bfloat16_rn(k0 * sn + k1 * cs);
-    for (int h = 0; h < H; ++h) {
-      const float x0 = q[h * dq + dn + 2 * i], x1 = q[h * dq + dn + 2 * i + 1];
-      qo[h * dq + dn + 2 * i] = __float2bfloat16_rn(x0 * cs - x1 * sn);
-      qo[h * dq + dn + 2 * i + 1] = __float2bfloat16_rn(x0 * sn + x1 * cs);
-    }
+  // rotations: item (h, i) for h < H is pair i of head h's q^R, h = H is k^R
+  for (int it = tid; it < (H + 1) * np; it += blockDim.x) {
+    const int h = it / np, i = it % np;
+    const float cs = cs_s[i], sn = sn_s[i];
+    const float* src = h < H ? q + h * dq + dn : kv + dc;
+    __nv_bfloat16* dst = h < H ? qo + h * dq + dn : kr_out + static_cast<size_t>(b) * dr;
+    const float x0 = src[2 * i], x1 = src[2 * i + 1];
+    dst[2 * i] = __float2bfloat16_rn(x0 * cs - x1 * sn);
+    dst[2 * i + 1] = __float2bfloat16_rn(x0 * sn + x1 * cs);
   }
 }
 
@@ -146,12 +157,11 @@ int eg_mla_layer_decode(const eg_mla_dims* dims, const eg_mla_layer_dims* layer,
   if (dims == nullptr || layer == nullptr || wt == nullptr) return EG_MLA_ERR_INVALID_ARG;
   if (dims->dtype != EG_MLA_BF16) return EG_MLA_ERR_UNSUPPORTED;
   if (batch < 0 || num_splits < 0 || layer->n_embd <= 0) return EG_MLA_ERR_INVALID_ARG;
-  if (layer->n_embd % 8 || dims->d_rope % 2) return EG_MLA_ERR_UNSUPPORTED;
+  if (layer->n_embd % 8 || dims->d_rope % 2 || dims->d_rope > 2 * kMaxRopePairs) return EG_MLA_ERR_UNSUPPORTED;
   if (batch == 0) return EG_MLA_OK;
-  if (!x || !positions || !y || !workspace || !wt->w_q || !wt->w_kv_a || !wt->kv_norm_w || !wt->w_o)
+  if (!x || !positions || !y || !workspace || !wt->w_qkv_a || !wt->kv_norm_w || !wt->w_o)
     return EG_MLA_ERR_INVALID_ARG;
-  if (!aligned16(x) || !aligned16(y) || !aligned16(wt->w_q) || !aligned16(wt->w_kv_a) || !aligned16(wt->w_o))
-    return EG_MLA_ERR_INVALID_ARG;
+  if (!aligned16(x) || !aligned16(y) || !aligned16(wt->w_qkv_a) || !aligned16(wt->w_o)) return EG_MLA_ERR_INVALID_ARG;
   if ((reinterpret_cast<uintptr_t>(workspace) & 255) != 0) return EG_MLA_ERR_INVALID_ARG;
   const LayerWorkspace ws = layer_workspace(dims, layer->n_embd, batch, num_splits);
   if (ws.dec_bytes == 0) return EG_MLA_ERR_INVALID_ARG;
@@ -161,9 +171,10 @@ int eg_mla_layer_decode(const eg_mla_dims* dims, const eg_mla_layer_dims* layer,
   const int H = dims->num_heads, E = layer->n_embd;
   const int nq = H * (dims->d_nope + dims->d_rope), nkv = dims->d_c + dims->d_rope, nu = H * dims->d_v;
   const double theta = layer->rope_theta > 0.f ? static_cast<double>(layer->rope_theta) : 10000.0;
+  RopeFreqs freqs{};
+  for (int i = 0; i < dims->d_rope / 2; ++i) freqs.f[i] = std::pow(theta, -2.0 * i / dims->d_rope);
   const float eps = layer->rms_eps > 0.f ? layer->rms_eps : 1.1920928955078125e-07f;
-  void* q32 = base + ws.off_q32;
-  void* kv32 = base + ws.off_kv32;
+  void* qkv32 = base + ws.off_qkv32;
   auto* qb = reinterpret_cast<__nv_bfloat16*>(base + ws.off_q);
   auto* cb = reinterpret_cast<__nv_bfloat16*>(base + ws.off_c);
   auto* krb = reinterpret_cast<__nv_bfloat16*>(base + ws.off_kr);
@@ -180,13 +191,13 @@ int eg_mla_layer_decode(const eg_mla_dims* dims, const eg_mla_layer_dims* layer,
   if (cublasSetStream(h, st) != CUBLAS_STATUS_SUCCESS ||
       cublasSetWorkspace(h, base + ws.off_cublas, kCublasWorkspace) != CUBLAS_STATUS_SUCCESS)
     return EG_MLA_ERR_CUDA;
-  // Eqs. 8-9 and 1, 10: the query and the latent + RoPE-key projections (fp32 out)
-  if (linear(h, nq, batch, E, wt->w_q, x, q32, CUDA_R_32F) != CUBLAS_STATUS_SUCCESS ||
-      linear(h, nkv, batch, E, wt->w_kv_a, x, kv32, CUDA_R_32F) != CUBLAS_STATUS_SUCCESS)
+  // Eqs. 8-9 and 1, 10: the query and the latent + RoPE-key projections, one
+  // GEMM over the stacked weight (fp32 out)
+  if (linear(h, nq + nkv, batch, E, wt->w_qkv_a, x, qkv32, CUDA_R_32F) != CUBLAS_STATUS_SUCCESS)
     return EG_MLA_ERR_CUDA;
   layer_qkv_kernel<<<batch, kQkvThreads, 0, st>>>(
-      static_cast<const float*>(q32), static_cast<const float*>(kv32), positions,
-      static_cast<const __nv_bfloat16*>(wt->kv_norm_w), H, dims->d_nope, dims->d_rope, dims->d_c, theta, eps, qb, cb,
+      static_cast<const float*>(qkv32), positions,
+      static_cast<const __nv_bfloat16*>(wt->kv_norm_w), H, dims->d_nope, dims->d_rope, dims->d_c, freqs, eps, qb, cb,
       krb);
   if (cudaGetLastError() != cudaSuccess) return EG_MLA_ERR_CUDA;
   int rc = eg_mla_append_latent(dims, c_pool, krope_pool, id_pool, cb, krb, ids_new, block_table, max_pages_per_seq,

@@ -172,8 +172,7 @@ class DeviceLayer:
     dc: DeviceCase
     layer_dims: _lib.EgMlaLayerDims
     x: torch.Tensor
-    w_q: torch.Tensor
-    w_kv_a: torch.Tensor
+    w_qkv_a: torch.Tensor       # [W^Q ; W^{DKV,KR}] stacked by rows
     kv_norm_w: torch.Tensor
     w_o: torch.Tensor
     y: torch.Tensor
@@ -181,7 +180,7 @@ class DeviceLayer:
 
     def weights(self) -> _lib.EgMlaLayerWeights:
         dc = self.dc
-        return _lib.make_layer_weights(self.w_q, self.w_kv_a, self.kv_norm_w, self.w_o, dc.gate_table, dc.ln_gamma,
+        return _lib.make_layer_weights(self.w_qkv_a, self.kv_norm_w, self.w_o, dc.gate_table, dc.ln_gamma,
                                        dc.ln_beta, dc.w_uk, dc.w_uv)
 
     def step(self, stream=None) -> torch.Tensor:
@@ -201,8 +200,18 @@ def upload_layer(lc, device="cuda", num_splits: int = 0) -> DeviceLayer:
     ws = _lib.eg_mla_layer_workspace_size(dc.dims, ld, dc.batch, num_splits)
     return DeviceLayer(
         dc=dc, layer_dims=ld,
-        x=to_device_array(lc.x, dt, device), w_q=to_device_array(lc.w_q, dt, device),
-        w_kv_a=to_device_array(lc.w_kv_a, dt, device), kv_norm_w=to_device_array(lc.kv_norm_w, dt, device),
+        x=to_device_array(lc.x, dt, device),
+        w_qkv_a=to_device_array(np.concatenate([lc.w_q, lc.w_kv_a], axis=0), dt, device),
+        kv_norm_w=to_device_array(lc.kv_norm_w, dt, device),
         w_o=to_device_array(lc.w_o, dt, device),
         y=torch.empty((dc.batch, lc.n_embd), dtype=torch.bfloat16, device=device),
         workspace=torch.empty(ws, dtype=torch.uint8, device=device))
+
+
+def clone_layer(dl: DeviceLayer) -> DeviceLayer:
+    """Another layer of the same shape: its own cache and weights (same values),
+    its own output; the decode and layer workspaces and the status word shared
+    (layers run one after another on one stream)."""
+    return DeviceLayer(dc=clone_case(dl.dc), layer_dims=dl.layer_dims, x=dl.x.clone(), w_qkv_a=dl.w_qkv_a.clone(),
+                       kv_norm_w=dl.kv_norm_w.clone(), w_o=dl.w_o.clone(),
+                       y=torch.empty_like(dl.y), workspace=dl.workspace)
