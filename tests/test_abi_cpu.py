@@ -110,3 +110,35 @@ def test_library_has_no_oracle_dependency():
             if f.endswith((".py", ".cu", ".cuh", ".h")):
                 text = open(os.path.join(dirpath, f)).read()
                 assert "import oracle" not in text and "from oracle" not in text, f
+
+
+def test_layer_workspace_size():
+    d = _lib.make_dims(16, 128, 64, 128, 256, 32000)
+    ld = _lib.make_layer_dims(2048)
+    n = _lib.eg_mla_layer_workspace_size(d, ld, 64, 152)
+    dec = _lib.eg_mla_decode_workspace_size(d, 64, 152)
+    # the decode workspace, a 4 MiB cuBLAS workspace, the fp32 projections and bf16 q, c, k^R, u
+    assert n >= dec + (4 << 20) + 64 * (16 * 192 + 320) * 4 + 64 * (16 * 192 + 256 + 64 + 16 * 128) * 2
+    assert n % 256 == 0
+    f32 = _lib.make_dims(4, 32, 16, 32, 64, 1000, dtype="fp32")
+    assert _lib.load().eg_mla_layer_workspace_size(ctypes.byref(f32), ctypes.byref(ld), 4, 8) == 0
+    assert _lib.load().eg_mla_layer_workspace_size(ctypes.byref(d), None, 4, 8) == 0
+
+
+def test_layer_decode_rejects_before_launch(lib):
+    d = _lib.make_dims(16, 128, 64, 128, 256, 32000)
+    ld = _lib.make_layer_dims(2048)
+    fake = 0x10000  # 256-byte aligned, never dereferenced: validation fails first
+    w = _lib.EgMlaLayerWeights(*([fake] * 8))
+    P = ctypes.c_void_p
+
+    def call(dims=d, layer=ld, weights=w, x=fake, batch=4, ws_bytes=1 << 20):
+        return lib.eg_mla_layer_decode(ctypes.byref(dims), ctypes.byref(layer), ctypes.byref(weights), P(x),
+                                       P(fake), P(fake), P(fake), P(fake), P(fake), P(fake), 4, P(fake), 256, batch,
+                                       8, P(fake), 152, P(fake), ws_bytes, None, None)
+    assert call(dims=_lib.make_dims(4, 32, 16, 32, 64, 1000, dtype="fp32")) == _lib.EG_MLA_ERR_UNSUPPORTED
+    assert call(layer=_lib.make_layer_dims(2044)) == _lib.EG_MLA_ERR_UNSUPPORTED
+    assert call(x=0) == _lib.EG_MLA_ERR_INVALID_ARG
+    assert call(x=fake + 8) == _lib.EG_MLA_ERR_INVALID_ARG              # 16-byte alignment
+    assert call(ws_bytes=1 << 20) == _lib.EG_MLA_ERR_WORKSPACE         # far below the layer's workspace
+    assert call(batch=0) == _lib.EG_MLA_OK                              # nothing to do, nothing launched
