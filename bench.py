@@ -68,6 +68,9 @@ def parse():
     ap.add_argument("--splits", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=0)
+    ap.add_argument("--lgz", type=int, default=1,
+                    help="layers24_full: layer group size (consecutive layers share one latent cache and its "
+                         "KV projection, Appendix H)")
     return ap.parse_args()
 
 
@@ -305,8 +308,20 @@ def run_gpu_full_layers(args, workload, torch, dist, ws, rank):
     lc = synth.make_layer_case(case, 2048, seed=5)
     n_layers = layers_of(workload)
     B, d = case.batch, case.dims
+    lgz = max(1, args.lgz)
+    if n_layers % lgz:
+        raise SystemExit(f"--lgz {lgz} does not divide {n_layers} layers")
     base = device.upload_layer(lc, num_splits=args.splits)
-    layers = [base] + [device.clone_layer(base) for _ in range(n_layers - 1)]
+    layers = [base]
+    for k in range(1, n_layers):
+        if k % lgz:
+            # a later layer of a layer group: the group's cache and first-half KV projection
+            layer = device.clone_layer(layers[k - k % lgz], share=("workspace", "status", "c_pool", "kr_pool",
+                                                                   "id_pool", "block_table"))
+            layer.layer_dims = _lib.make_layer_dims(lc.n_embd, lc.rope_theta, lc.rms_eps, share_kv=True)
+        else:
+            layer = device.clone_layer(base)
+        layers.append(layer)
     for k in range(1, n_layers):
         layers[k].x = layers[k - 1].y          # the residual stream is left out: attention layers only
         for name in ("ids_new", "positions", "seq_lens"):   # one step's token ids and lengths, shared
@@ -410,21 +425,24 @@ def run_gpu_full_layers(args, workload, torch, dist, ws, rank):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": steps_arg, "warmup": args.warmup,
         "ms_per_step": elapsed_ms / steps_arg, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": desc, "batch": B, "layers": n_layers, "n_embd": 2048,
+        "config": {"workload": desc + (f"; layer groups of {lgz} sharing one cache" if lgz > 1 else ""),
+                   "batch": B, "layers": n_layers, "n_embd": 2048, "lgz": lgz,
                    "ctx_tokens_cached": tokens_cached, "splits": splits, "page_size": d.page_size,
                    "l2": f"inputs larger than L2: {n_layers} layers' distinct caches of {cache_bytes / 1e6:.0f} MB "
                          f"and weights", "graph": "step replayed from a CUDA graph"},
         "kv_cache_gbs": n_layers * cache_bytes * steps_arg / (elapsed_ms / 1e3) / 1e9,
         "kv_bytes_per_token": (d.d_c + d.d_rope) * 2 + 4,
+        "kv_bytes_per_token_model": n_layers // lgz * ((d.d_c + d.d_rope) * 2 + 4),
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                      "traffic": None, "kernel": "decode_tc_kernel", "kernel_ms": k_ms,
                      "bytes_per_launch": cache_bytes, "peak_source": peak_src},
         "cpu_baseline": cpu,
         "e2e": {"value": whole_job_rate(ws, B, e2e_steps, e2e_ms), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
-        # this library's kernels per layer: kv_norm + RoPE, append, query absorption,
-        # decode (the three projection GEMMs are cuBLAS kernels, not counted)
-        "gpu_launches": steps_arg * n_layers * 4,
+        # this library's kernels per layer: kv_norm + RoPE, append (first layer of
+        # a group only), query absorption, decode (the projection GEMMs are cuBLAS
+        # kernels, not counted)
+        "gpu_launches": steps_arg * (n_layers * 3 + n_layers // lgz),
         "clocks": clk.summary(),
     }
 

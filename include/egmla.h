@@ -248,6 +248,14 @@ typedef struct {
   int32_t n_embd;     /* model width E (a multiple of 8) */
   float rope_theta;   /* rotary base; <= 0 selects 10000 */
   float rms_eps;      /* kv_norm epsilon; <= 0 selects 2^-23 (the fp32 machine epsilon) */
+  int32_t share_kv;   /* nonzero: a later layer of a layer group (Section 5 inter-layer
+                         sharing, Appendix H "layer group size"): the group shares the
+                         first half of the KV projection, W^{DKV,KR}, and its activations,
+                         so the group's first layer already projected, normalised, rotated
+                         and appended this step's c^KV, k^R and id to the cache the group
+                         shares.  This layer projects only its q (only the W^Q rows of
+                         w_qkv_a are read), appends nothing and attends over the shared
+                         cache with its own W_UK, W_UV, gate table and LayerNorm */
 } eg_mla_layer_dims;
 
 /* Device pointers of one layer's weights, each 16-byte aligned, in the

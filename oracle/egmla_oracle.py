@@ -327,14 +327,19 @@ def rms_norm(x: np.ndarray, w: np.ndarray, eps: float) -> np.ndarray:
     return x / np.sqrt((x * x).mean(axis=-1, keepdims=True) + eps) * np.asarray(w, dtype=np.float64)
 
 
-def layer_step(lc):
+def layer_step(lc, kv_from=None):
     """The decode-step inputs of the attention (Appendix C with q-LoRA rank 0, as
     every model of Appendix A): q = W^Q x split per head into [q^C ; q^R] with
     q^R rotated (Eqs. 8-9), [c^KV ; k^R] = W^{DKV,KR} x (Eqs. 1 and 10) with k^R
     rotated and c^KV passed through the listing's kv_norm (RMSNorm) before it is
     cached.  The rotation position of a sequence's new token is L_b - 1.
     Returns the decode case of this step: the cache plus (q, c_new, kr_new) as
-    the model stores them."""
+    the model stores them.
+
+    kv_from: for a later layer of a layer group (Section 5 inter-layer sharing,
+    Appendix H), the group's first layer: the group shares W^{DKV,KR} and its
+    activations, so this step's c^KV, k^R and id are that layer's and only q is
+    this layer's own (its cache, gate table and up-projections are lc.case's)."""
     case = lc.case
     d = case.dims
     H, dn, dr, dc = d.num_heads, d.d_nope, d.d_rope, d.d_c
@@ -346,15 +351,19 @@ def layer_step(lc):
     kv = x @ widen(lc.w_kv_a, d.dtype).T
     c = rms_norm(kv[:, :dc], widen(lc.kv_norm_w, d.dtype), lc.rms_eps)
     kr = rope(kv[:, dc:], pos, lc.rope_theta)
+    if kv_from is not None:
+        first = layer_step(kv_from)
+        return dataclasses.replace(case, q=store(q, d.dtype), c_new=first.c_new, kr_new=first.kr_new,
+                                   ids_new=first.ids_new)
     return dataclasses.replace(case, q=store(q, d.dtype), c_new=store(c, d.dtype), kr_new=store(kr, d.dtype))
 
 
-def layer_decode(lc, batches: Optional[Iterable[int]] = None) -> np.ndarray:
+def layer_decode(lc, batches: Optional[Iterable[int]] = None, kv_from=None) -> np.ndarray:
     """o_t = W^O [u_t,1 ; ... ; u_t,n_h] (Eq. 14) with u the attention output of
     ``decode_unabsorbed`` over the cache after this step's append, kept in the
     model dtype as the layer stores it.  Returns [B, E] float64 (rows of
-    unselected batches NaN)."""
-    step = layer_step(lc)
+    unselected batches NaN).  kv_from: as for layer_step."""
+    step = layer_step(lc, kv_from)
     d = step.dims
     u = decode_unabsorbed(step, batches=batches)
     B = step.batch

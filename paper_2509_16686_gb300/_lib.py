@@ -145,6 +145,7 @@ class EgMlaLayerDims(ctypes.Structure):
         ("n_embd", ctypes.c_int32),
         ("rope_theta", ctypes.c_float),
         ("rms_eps", ctypes.c_float),
+        ("share_kv", ctypes.c_int32),
     ]
 
 
@@ -230,8 +231,11 @@ def eg_mla_decode_static(dims: EgMlaDims, q, c_pool, krope_pool, id_pool, block_
     _check(code, "eg_mla_decode_static")
 
 
-def make_layer_dims(n_embd: int, rope_theta: float = 10000.0, rms_eps: float = 0.0) -> EgMlaLayerDims:
-    return EgMlaLayerDims(n_embd, rope_theta, rms_eps)
+def make_layer_dims(n_embd: int, rope_theta: float = 10000.0, rms_eps: float = 0.0,
+                    share_kv: bool = False) -> EgMlaLayerDims:
+    """share_kv: a later layer of a layer group (its group's first layer projects
+    and appends the shared c^KV, k^R; this one attends over the shared cache)."""
+    return EgMlaLayerDims(n_embd, rope_theta, rms_eps, 1 if share_kv else 0)
 
 
 def make_layer_weights(w_qkv_a, kv_norm_w, w_o, gate_table, ln_gamma, ln_beta, w_uk, w_uv) -> EgMlaLayerWeights:

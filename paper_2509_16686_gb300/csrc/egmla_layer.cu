@@ -82,7 +82,8 @@ struct RopeFreqs {
 __global__ void __launch_bounds__(kQkvThreads) layer_qkv_kernel(
     const float* __restrict__ qkv32, const int32_t* __restrict__ positions,
     const __nv_bfloat16* __restrict__ kv_norm_w, int H, int dn, int dr, int dc, const RopeFreqs freqs, float eps,
-    __nv_bfloat16* __restrict__ q_out, __nv_bfloat16* __restrict__ c_out, __nv_bfloat16* __restrict__ kr_out) {
+    int do_kv, __nv_bfloat16* __restrict__ q_out, __nv_bfloat16* __restrict__ c_out,
+    __nv_bfloat16* __restrict__ kr_out) {
   __shared__ float red[kQkvThreads / 32];
   __shared__ float cs_s[kMaxRopePairs], sn_s[kMaxRopePairs];
   const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -102,7 +103,8 @@ __global__ void __launch_bounds__(kQkvThreads) layer_qkv_kernel(
   }
   // kv_norm: the mean of c^2 over d_c (warp sums, then the warps' sums in order)
   float ss = 0.f;
-  for (int f = tid; f < dc; f += blockDim.x) ss = fmaf(kv[f], kv[f], ss);
+  if (do_kv)
+    for (int f = tid; f < dc; f += blockDim.x) ss = fmaf(kv[f], kv[f], ss);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
   if (lane == 0) red[warp] = ss;
@@ -113,10 +115,11 @@ __global__ void __launch_bounds__(kQkvThreads) layer_qkv_kernel(
   float tot = 0.f;
   for (int i = 0; i < static_cast<int>(blockDim.x / 32); ++i) tot += red[i];
   const float r = 1.f / sqrtf(tot / static_cast<float>(dc) + eps);
-  for (int f = tid; f < dc; f += blockDim.x)
-    c_out[static_cast<size_t>(b) * dc + f] = __float2bfloat16_rn(kv[f] * r * __bfloat162float(kv_norm_w[f]));
+  if (do_kv)
+    for (int f = tid; f < dc; f += blockDim.x)
+      c_out[static_cast<size_t>(b) * dc + f] = __float2bfloat16_rn(kv[f] * r * __bfloat162float(kv_norm_w[f]));
   // rotations: item (h, i) for h < H is pair i of head h's q^R, h = H is k^R
-  for (int it = tid; it < (H + 1) * np; it += blockDim.x) {
+  for (int it = tid; it < (H + (do_kv ? 1 : 0)) * np; it += blockDim.x) {
     const int h = it / np, i = it % np;
     const float cs = cs_s[i], sn = sn_s[i];
     const float* src = h < H ? q + h * dq + dn : kv + dc;
@@ -129,11 +132,12 @@ __global__ void __launch_bounds__(kQkvThreads) layer_qkv_kernel(
 
 // C[m, n] (column-major, ld m) = A^T B with A [k, m] and B [k, n] column-major,
 // i.e. row-major out[n][m] = in[n][:] . W[m][:] for a Linear weight W [m, k]
+// (ldc >= m: the output row stride in elements)
 cublasStatus_t linear(cublasHandle_t h, int m, int n, int k, const void* w, const void* in, void* out,
-                      cudaDataType_t out_type) {
+                      cudaDataType_t out_type, int ldc) {
   const float one = 1.f, zero = 0.f;
   return cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, m, n, k, &one, w, CUDA_R_16BF, k, in, CUDA_R_16BF, k, &zero, out,
-                      out_type, m, CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT);
+                      out_type, ldc, CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT);
 }
 
 }  // namespace
@@ -159,7 +163,7 @@ int eg_mla_layer_decode(const eg_mla_dims* dims, const eg_mla_layer_dims* layer,
   if (batch < 0 || num_splits < 0 || layer->n_embd <= 0) return EG_MLA_ERR_INVALID_ARG;
   if (layer->n_embd % 8 || dims->d_rope % 2 || dims->d_rope > 2 * kMaxRopePairs) return EG_MLA_ERR_UNSUPPORTED;
   if (batch == 0) return EG_MLA_OK;
-  if (!x || !positions || !y || !workspace || !wt->w_qkv_a || !wt->kv_norm_w || !wt->w_o)
+  if (!x || !positions || !y || !workspace || !wt->w_qkv_a || (layer->share_kv == 0 && !wt->kv_norm_w) || !wt->w_o)
     return EG_MLA_ERR_INVALID_ARG;
   if (!aligned16(x) || !aligned16(y) || !aligned16(wt->w_qkv_a) || !aligned16(wt->w_o)) return EG_MLA_ERR_INVALID_ARG;
   if ((reinterpret_cast<uintptr_t>(workspace) & 255) != 0) return EG_MLA_ERR_INVALID_ARG;
@@ -192,23 +196,28 @@ int eg_mla_layer_decode(const eg_mla_dims* dims, const eg_mla_layer_dims* layer,
       cublasSetWorkspace(h, base + ws.off_cublas, kCublasWorkspace) != CUBLAS_STATUS_SUCCESS)
     return EG_MLA_ERR_CUDA;
   // Eqs. 8-9 and 1, 10: the query and the latent + RoPE-key projections, one
-  // GEMM over the stacked weight (fp32 out)
-  if (linear(h, nq + nkv, batch, E, wt->w_qkv_a, x, qkv32, CUDA_R_32F) != CUBLAS_STATUS_SUCCESS)
+  // GEMM over the stacked weight (fp32 out); a later layer of a layer group
+  // projects only its query
+  const bool do_kv = layer->share_kv == 0;
+  if (linear(h, do_kv ? nq + nkv : nq, batch, E, wt->w_qkv_a, x, qkv32, CUDA_R_32F, nq + nkv) !=
+      CUBLAS_STATUS_SUCCESS)
     return EG_MLA_ERR_CUDA;
   layer_qkv_kernel<<<batch, kQkvThreads, 0, st>>>(
       static_cast<const float*>(qkv32), positions,
-      static_cast<const __nv_bfloat16*>(wt->kv_norm_w), H, dims->d_nope, dims->d_rope, dims->d_c, freqs, eps, qb, cb,
-      krb);
+      static_cast<const __nv_bfloat16*>(wt->kv_norm_w), H, dims->d_nope, dims->d_rope, dims->d_c, freqs, eps,
+      do_kv ? 1 : 0, qb, cb, krb);
   if (cudaGetLastError() != cudaSuccess) return EG_MLA_ERR_CUDA;
-  int rc = eg_mla_append_latent(dims, c_pool, krope_pool, id_pool, cb, krb, ids_new, block_table, max_pages_per_seq,
-                                positions, batch, num_pages, dev_status, stream);
+  int rc = EG_MLA_OK;
+  if (do_kv)
+    rc = eg_mla_append_latent(dims, c_pool, krope_pool, id_pool, cb, krb, ids_new, block_table, max_pages_per_seq,
+                              positions, batch, num_pages, dev_status, stream);
   if (rc != EG_MLA_OK) return rc;
   rc = eg_mla_decode(dims, qb, c_pool, krope_pool, id_pool, block_table, max_pages_per_seq, seq_lens, max_seq_len,
                      batch, num_pages, wt->gate_table, wt->ln_gamma, wt->ln_beta, wt->w_uk, wt->w_uv, ub, num_splits,
                      base + ws.off_dec, ws.dec_bytes, dev_status, stream);
   if (rc != EG_MLA_OK) return rc;
   // Eq. 14: the output projection of the heads' concatenated outputs
-  if (linear(h, E, batch, nu, wt->w_o, ub, y, CUDA_R_16BF) != CUBLAS_STATUS_SUCCESS) return EG_MLA_ERR_CUDA;
+  if (linear(h, E, batch, nu, wt->w_o, ub, y, CUDA_R_16BF, E) != CUBLAS_STATUS_SUCCESS) return EG_MLA_ERR_CUDA;
   return EG_MLA_OK;
 }
 

@@ -208,10 +208,12 @@ def upload_layer(lc, device="cuda", num_splits: int = 0) -> DeviceLayer:
         workspace=torch.empty(ws, dtype=torch.uint8, device=device))
 
 
-def clone_layer(dl: DeviceLayer) -> DeviceLayer:
+def clone_layer(dl: DeviceLayer, share=("workspace", "status")) -> DeviceLayer:
     """Another layer of the same shape: its own cache and weights (same values),
     its own output; the decode and layer workspaces and the status word shared
-    (layers run one after another on one stream)."""
-    return DeviceLayer(dc=clone_case(dl.dc), layer_dims=dl.layer_dims, x=dl.x.clone(), w_qkv_a=dl.w_qkv_a.clone(),
+    (layers run one after another on one stream), and whatever else of the
+    cache ``share`` names (a layer group shares its pools and block table)."""
+    return DeviceLayer(dc=clone_case(dl.dc, share=share), layer_dims=dl.layer_dims, x=dl.x.clone(),
+                       w_qkv_a=dl.w_qkv_a.clone(),
                        kv_norm_w=dl.kv_norm_w.clone(), w_o=dl.w_o.clone(),
                        y=torch.empty_like(dl.y), workspace=dl.workspace)

@@ -19,7 +19,7 @@ import pytest
 import torch
 
 from oracle import egmla_oracle as orc
-from paper_2509_16686_gb300 import device, synth
+from paper_2509_16686_gb300 import _lib, device, synth
 
 pytestmark = pytest.mark.gpu
 
@@ -85,3 +85,32 @@ def test_layer_step_24_layer_model_shape_sampled(gpu_lib):
     sample = [0, 37, 63]
     ref = orc.layer_decode(lc, batches=sample)
     check_bf16(got[sample], ref[sample], "layer 2048 sampled")
+
+
+def test_layer_group_shares_one_cache(gpu_lib):
+    """Two layers of one layer group (Appendix H): the first projects, rotates and
+    appends the shared c^KV, k^R; the second (share_kv) projects only its query
+    and attends over the same cache with its own up-projections, gate table and
+    output projection."""
+    import dataclasses
+    case_a = synth.make_case("group", synth.dims_bf16(vocab=3000), [300, 65, 1], seed=41, latent_scale=0.5,
+                             layout="permuted", affine_ln=True)
+    other = synth.make_case("group-b", synth.dims_bf16(vocab=3000), [300, 65, 1], seed=42, latent_scale=0.5,
+                            layout="permuted", affine_ln=True)
+    case_b = dataclasses.replace(case_a, gate_table=other.gate_table, ln_gamma=other.ln_gamma,
+                                 ln_beta=other.ln_beta, w_uk=other.w_uk, w_uv=other.w_uv)
+    lc_a = synth.make_layer_case(case_a, 256, seed=43)
+    lc_b = synth.make_layer_case(case_b, 256, seed=44)
+    dl_a = device.upload_layer(lc_a)
+    dl_b = device.upload_layer(lc_b)
+    for name in ("c_pool", "kr_pool", "id_pool", "block_table", "seq_lens", "positions", "ids_new"):
+        setattr(dl_b.dc, name, getattr(dl_a.dc, name))
+    dl_b.layer_dims = _lib.make_layer_dims(256, share_kv=True)
+    dl_a.step()
+    dl_b.step()
+    torch.cuda.synchronize()
+    assert dl_a.dc.read_status() == 0 and dl_b.dc.read_status() == 0
+    check_bf16(device.output_f64(dl_a.y), orc.layer_decode(lc_a), "group first layer")
+    check_bf16(device.output_f64(dl_b.y), orc.layer_decode(lc_b, kv_from=lc_a), "group second layer")
+    # the cache holds the first layer's token once; a second append would have been the same row
+    check_appended_rows(dl_a, lc_a)

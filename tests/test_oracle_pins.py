@@ -545,3 +545,18 @@ def test_layer_steps_match_the_full_sequence_causal_forward():
     u = F.scaled_dot_product_attention(qh[None], k[None], v[None], is_causal=True)[0]
     y_ref = (u.transpose(0, 1).reshape(T, H * dv) @ tt["w_o"].T).numpy()
     assert np.abs(np.stack(ys) - y_ref).max() <= 1e-10
+
+
+def test_layer_group_sharing_reuses_what_the_layer_would_compute():
+    """A later layer of a layer group takes c^KV, k^R and the id from the group's
+    first layer (Appendix H).  When both layers have the same first-half weights
+    and input, that is exactly what the later layer would have computed itself;
+    with a different input it is not."""
+    import dataclasses
+    case = synth.make_case("grp", synth.dims_bf16(vocab=500), [70, 3], seed=51, latent_scale=0.5)
+    lc_a = synth.make_layer_case(case, 64, seed=52)
+    lc_b = dataclasses.replace(synth.make_layer_case(case, 64, seed=53), x=lc_a.x, w_kv_a=lc_a.w_kv_a,
+                               kv_norm_w=lc_a.kv_norm_w)
+    assert np.array_equal(orc.layer_decode(lc_b, kv_from=lc_a), orc.layer_decode(lc_b))
+    lc_c = dataclasses.replace(lc_b, x=synth.make_layer_case(case, 64, seed=54).x)
+    assert not np.allclose(orc.layer_decode(lc_c, kv_from=lc_a), orc.layer_decode(lc_c))
