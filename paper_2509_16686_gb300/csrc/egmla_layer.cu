@@ -30,12 +30,11 @@ struct LayerWorkspace {
 
 // carve of the layer workspace (every piece 256-byte aligned); dec_bytes = 0 on
 // invalid decode arguments
-LayerWorkspace layer_workspace(const eg_mla_dims* d, int32_t n_embd, int32_t batch, int32_t num_splits) {
+LayerWorkspace layer_workspace(const eg_mla_dims* d, int32_t batch, int32_t num_splits) {
   LayerWorkspace w{};
   const size_t B = static_cast<size_t>(batch > 0 ? batch : 0);
   const size_t nq = static_cast<size_t>(d->num_heads) * (d->d_nope + d->d_rope);
   const size_t nkv = static_cast<size_t>(d->d_c + d->d_rope);
-  (void)n_embd;
   size_t off = 0;
   w.off_cublas = off;
   off += kCublasWorkspace;
@@ -148,7 +147,7 @@ size_t eg_mla_layer_workspace_size(const eg_mla_dims* dims, const eg_mla_layer_d
                                    int32_t num_splits) {
   if (dims == nullptr || layer == nullptr || batch < 0 || layer->n_embd <= 0) return 0;
   if (dims->dtype != EG_MLA_BF16) return 0;
-  const LayerWorkspace w = layer_workspace(dims, layer->n_embd, batch, num_splits);
+  const LayerWorkspace w = layer_workspace(dims, batch, num_splits);
   return w.dec_bytes == 0 ? 0 : w.total;
 }
 
@@ -167,7 +166,7 @@ int eg_mla_layer_decode(const eg_mla_dims* dims, const eg_mla_layer_dims* layer,
     return EG_MLA_ERR_INVALID_ARG;
   if (!aligned16(x) || !aligned16(y) || !aligned16(wt->w_qkv_a) || !aligned16(wt->w_o)) return EG_MLA_ERR_INVALID_ARG;
   if ((reinterpret_cast<uintptr_t>(workspace) & 255) != 0) return EG_MLA_ERR_INVALID_ARG;
-  const LayerWorkspace ws = layer_workspace(dims, layer->n_embd, batch, num_splits);
+  const LayerWorkspace ws = layer_workspace(dims, batch, num_splits);
   if (ws.dec_bytes == 0) return EG_MLA_ERR_INVALID_ARG;
   if (workspace_bytes < ws.total) return EG_MLA_ERR_WORKSPACE;
   uint8_t* base = static_cast<uint8_t*>(workspace);
