@@ -503,11 +503,9 @@ def _tiny_layer_model(seed=9):
     return dims, w, xs, ids
 
 
-def test_layer_steps_match_the_full_sequence_causal_forward():
-    """Decoding T tokens one step at a time through the layer oracle (append,
-    then attend) gives, at every step, the output of one causal forward pass over
-    the whole sequence written from the listing with the gate in latent space
-    (torch float64: complex-rotation RoPE, rms_norm, layer_norm, SDPA)."""
+def _layer_steps_deviation():
+    """Largest difference between the layer oracle decoding a tiny sequence one
+    token at a time and one causal forward pass over the whole sequence."""
     dims, w, xs, ids = _tiny_layer_model()
     T, E = xs.shape
     H, dn, dr, dv, dc, P = dims.num_heads, dims.d_nope, dims.d_rope, dims.d_v, dims.d_c, dims.page_size
@@ -544,7 +542,42 @@ def test_layer_steps_match_the_full_sequence_causal_forward():
     qh = torch.cat([q_nope, q_pe], dim=-1).transpose(0, 1)
     u = F.scaled_dot_product_attention(qh[None], k[None], v[None], is_causal=True)[0]
     y_ref = (u.transpose(0, 1).reshape(T, H * dv) @ tt["w_o"].T).numpy()
-    assert np.abs(np.stack(ys) - y_ref).max() <= 1e-10
+    return float(np.abs(np.stack(ys) - y_ref).max())
+
+
+def test_layer_steps_match_the_full_sequence_causal_forward():
+    """Decoding T tokens one step at a time through the layer oracle (append,
+    then attend) gives, at every step, the output of one causal forward pass over
+    the whole sequence written from the listing with the gate in latent space
+    (torch float64: complex-rotation RoPE, rms_norm, layer_norm, SDPA)."""
+    assert _layer_steps_deviation() <= 1e-10
+
+
+def _rope_rotate_half(x, pos, theta):
+    # the other common convention: pairs (i, i + d/2) instead of (2i, 2i + 1)
+    x = np.asarray(x, dtype=np.float64)
+    d = x.shape[-1]
+    ang = np.asarray(pos, dtype=np.float64)[..., None] * theta ** (-2.0 * np.arange(d // 2) / d)
+    a, b = x[..., :d // 2], x[..., d // 2:]
+    return np.concatenate([a * np.cos(ang) - b * np.sin(ang), a * np.sin(ang) + b * np.cos(ang)], axis=-1)
+
+
+@pytest.mark.parametrize("mistake", ["key_position_plus_one", "no_kv_norm", "rotate_half"])
+def test_layer_pin_catches_planted_mistakes(monkeypatch, mistake):
+    """Each planted mistake moves the decoded outputs away from the full-sequence
+    forward.  (Shifting every position by the same offset is not a mistake the
+    outputs can show: rotary scores depend only on relative position.  An
+    offset between the new token's query and its appended key is one.)"""
+    good_rope = orc.rope
+    if mistake == "key_position_plus_one":
+        # q^R has a head axis ([B, H, d_r]); k^R does not ([B, d_r])
+        monkeypatch.setattr(orc, "rope", lambda x, pos, theta: good_rope(
+            x, np.asarray(pos) + (0.0 if np.ndim(x) == 3 else 1.0), theta))
+    elif mistake == "no_kv_norm":
+        monkeypatch.setattr(orc, "rms_norm", lambda x, w, eps: np.asarray(x, dtype=np.float64))
+    else:
+        monkeypatch.setattr(orc, "rope", _rope_rotate_half)
+    assert _layer_steps_deviation() > 1e-3
 
 
 def test_layer_group_sharing_reuses_what_the_layer_would_compute():
