@@ -295,8 +295,9 @@ size_t eg_mla_layer_workspace_size(const eg_mla_dims* dims, const eg_mla_layer_d
  * The projections are plain GEMMs run by cuBLAS on a cuBLAS handle this
  * library creates once per device, at the first call on that device (make
  * that first call before any stream capture); every later call allocates
- * nothing and is capturable.  Calls on one device share that handle: issue
- * them from one host thread at a time.  Host-side argument errors return a
+ * nothing and is capturable.  Calls on one device share that handle; the
+ * library holds a lock while a call sets the handle's stream and workspace
+ * and issues its work.  Host-side argument errors return a
  * negative status and launch nothing; device errors go to *dev_status as for
  * eg_mla_decode.
  */

@@ -1,9 +1,10 @@
 // egmla_layer.cu - one decode step through a whole EG-MLA attention layer:
 // the query and latent projections, the latent's RMSNorm and the rotary
 // embedding of q^R and k^R (one fused kernel), the cache append and the
-// gated latent attention of egmla_api.cu, and the output projection.  The
-// three projections are plain GEMMs and run in cuBLAS; everything between
-// them runs in this library's kernels.  See include/egmla.h for the contract.
+// gated latent attention of egmla_api.cu, and the output projection.  The two
+// projection GEMMs (the stacked query/latent weight, and W^O) are plain GEMMs
+// and run in cuBLAS; everything between them runs in this library's kernels.
+// See include/egmla.h for the contract.
 #include <cublas_v2.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
