@@ -244,7 +244,7 @@ def run_reference(args):
     from oracle import egmla_oracle as orc
     H = case.dims.num_heads
     L = int(case.seq_lens[0])
-    n_steps = max(1, args.steps) + max(0, args.warmup)
+    n_steps = max(1, args.steps if args.steps is not None else 10) + max(0, args.warmup)
     probe = dataclasses.replace(case, seq_lens=case.seq_lens[:1].copy(), block_table=case.block_table[:1],
                                 q=case.q[:1], c_new=case.c_new[:1], kr_new=case.kr_new[:1],
                                 ids_new=case.ids_new[:1])
