@@ -353,6 +353,59 @@ def test_r0_matches_listing_form():
         np.testing.assert_allclose(got[b], y[0, :, 0].numpy(), rtol=1e-11, atol=1e-12)
 
 
+def _r0_gate(case, seed=12):
+    d = case.dims
+    return np.random.default_rng(seed).normal(1.0, 0.2, size=(d.vocab, d.num_heads * (d.d_nope + d.d_v)))
+
+
+def test_r0_single_token_closed_form():
+    """One cached token: every head's output is that token's normalised value
+    part, LN((W^UKV c) (*) g) restricted to the head's d_v values."""
+    case = small_case(seed=13, lens=(1, 1), H=2, dn=4, dr=4, dv=4, dc=8, V=20)
+    d = case.dims
+    g = _r0_gate(case)
+    got = orc.decode_r0(case, gate_r0=g)
+    w = np.concatenate([orc.widen(case.w_uk, d.dtype), orc.widen(case.w_uv, d.dtype)], axis=1).reshape(-1, d.d_c)
+    for b in range(case.batch):
+        c = orc.widen(case.c_new[b], d.dtype)
+        kv = (w @ c) * g[int(case.ids_new[b])]
+        kv = ((kv - kv.mean()) / np.sqrt(kv.var() + d.ln_eps)).reshape(d.num_heads, d.d_nope + d.d_v)
+        np.testing.assert_allclose(got[b], kv[:, d.d_nope:], rtol=1e-12, atol=1e-12)
+
+
+def test_r0_position_permutation_invariance():
+    case = small_case(seed=14, lens=(40,), H=2, dn=4, dr=4, dv=4, dc=8, V=20, layout="contiguous")
+    g = _r0_gate(case)
+    ref = orc.decode_r0(case, gate_r0=g)
+    # swap the first 39 cached tokens in a random order (the new token stays last)
+    perm = np.random.default_rng(15).permutation(39)
+    flat = lambda a: a.reshape(-1, *a.shape[2:])
+    c, kr, ids = flat(case.c_pool).copy(), flat(case.kr_pool).copy(), flat(case.id_pool).copy()
+    c[:39], kr[:39], ids[:39] = c[perm], kr[perm], ids[perm]
+    case.c_pool, case.kr_pool, case.id_pool = (c.reshape(case.c_pool.shape), kr.reshape(case.kr_pool.shape),
+                                               ids.reshape(case.id_pool.shape))
+    case._oracle_appended = None
+    np.testing.assert_allclose(orc.decode_r0(case, gate_r0=g), ref, rtol=1e-12, atol=1e-12)
+
+
+def test_r0_reduces_to_r1_when_the_up_projection_is_the_identity():
+    """With d_c = H (d_n + d_v) and W^UKV = I, gating after the up-projection
+    (the paper-literal R0) and gating the latent (R1) are the same computation:
+    the LayerNorm runs over the same vector and W_UK,h, W_UV,h select the head's
+    key and value parts."""
+    H, dn, dv = 2, 4, 4
+    width = H * (dn + dv)
+    case = small_case(seed=16, lens=(23, 1, 40), H=H, dn=dn, dr=4, dv=dv, dc=width, V=20)
+    eye = np.eye(width).reshape(H, dn + dv, width)
+    case.w_uk = eye[:, :dn, :].astype(np.float32)
+    case.w_uv = eye[:, dn:, :].astype(np.float32)
+    g = _r0_gate(case)
+    case.gate_table = g.astype(np.float32)
+    g32 = case.gate_table.astype(np.float64)     # the table both forms read
+    got_r0 = orc.decode_r0(case, gate_r0=g32, ln_gamma_r0=case.ln_gamma, ln_beta_r0=case.ln_beta)
+    np.testing.assert_allclose(got_r0, orc.decode_unabsorbed(case), rtol=1e-11, atol=1e-12)
+
+
 # ---------------------------------------------------------------------------
 # the ablation gate operations (Section 4.4, Table 'Ablation on Embedding Gating')
 # ---------------------------------------------------------------------------
