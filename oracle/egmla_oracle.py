@@ -25,9 +25,11 @@ Parity status: every function here is pinned by the tests in
 paper's printed cache sizes).  The attention-layer step (``layer_step``,
 ``layer_decode``) is pinned by decoding a sequence one token at a time against
 one causal forward pass over the whole sequence written from the listing, and
-its RoPE, RMSNorm and bf16 storage against the corresponding torch routines.  ``decode_r0`` is pinned only against a PyTorch
-re-expression of the paper's listing on tiny inputs (parity unpinned beyond
-that: the paper prints no numeric example).
+its RoPE, RMSNorm and bf16 storage against the corresponding torch routines.
+``decode_r0`` (no GPU path; the paper prints no numeric example of it) is
+pinned against a PyTorch re-expression of the paper's listing, a single-token
+closed form, invariance under permuting cached positions, and its reduction to
+the latent-gated form when the joint up-projection is the identity.
 """
 from __future__ import annotations
 
