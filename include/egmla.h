@@ -16,13 +16,18 @@
  *     RoPE key with scale 1/sqrt(d_h + d_h^R), an online softmax with split-KV
  *     partials is merged by log-sum-exp, and the latent-space output is
  *     up-projected through W_UV,h.  It returns the per-head outputs u_{t,i}.
+ *   - eg_mla_layer_decode runs the same step from the layer's hidden state:
+ *     the query and latent projections (Eqs. 1, 8-10), the latent's RMSNorm
+ *     and the rotary embedding, the append and the decode above, and the
+ *     output projection (Eq. 14).
  *
  * Conventions shared by every call:
  *   - Every pointer argument except `dims`, `bytes_out` and `out_splits` is a
  *     DEVICE pointer to caller-owned memory.  The library never allocates,
- *     frees or keeps device memory between calls; the one device buffer it
- *     owns is the fixed static scratch array of eg_mla_decode_static, which
- *     is part of the loaded module.
+ *     frees or keeps device memory between calls; the device memory it owns
+ *     is the fixed static scratch array of eg_mla_decode_static, which is
+ *     part of the loaded module, and the cuBLAS handle eg_mla_layer_decode
+ *     creates at its first call on each device.
  *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
  *     stream).  Calls are asynchronous on that stream and never synchronise
  *     the host.
