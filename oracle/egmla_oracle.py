@@ -51,6 +51,14 @@ def widen(x: np.ndarray, dtype: str) -> np.ndarray:
     return np.asarray(x, dtype=np.float64)
 
 
+def softmax_scale(d) -> float:
+    """Attention scale 1/sqrt(d_h + d_h^R) (Appendix C Eq. 13; the listing's SDPA
+    default over q of width d_nope + d_rope), unless the dims fix another one."""
+    if d.softmax_scale > 0:
+        return float(d.softmax_scale)
+    return 1.0 / math.sqrt(d.d_nope + d.d_rope)
+
+
 # --------------------------------------------------------------------------
 # paged latent cache (Table 5: the cache holds d_c + d_h^R values per token)
 # --------------------------------------------------------------------------
@@ -189,7 +197,7 @@ def head_probs_unabsorbed(case, b: int, h: int, gate: Optional[bool] = None):
     w_uk = widen(case.w_uk[h], d.dtype)               # [d_n, d_c]
     k_c = c_t @ w_uk.T                                 # [L, d_n]   (Eq. 2 + split, Eq. 6)
     k = np.concatenate([k_c, kr], axis=1)              # [L, d_n + d_r] (Eq. 12)
-    s = (k @ qv) * d.scale()                           # (Eq. 13)
+    s = (k @ qv) * softmax_scale(d)                           # (Eq. 13)
     return softmax(s), c_t
 
 
@@ -218,7 +226,7 @@ def decode_unabsorbed(case, batches: Optional[Iterable[int]] = None,
             w_uv = widen(case.w_uv[h], d.dtype)
             k = np.concatenate([c_t @ w_uk.T, kr], axis=1)
             v = c_t @ w_uv.T                             # [L, d_v]
-            p = softmax((k @ qv) * d.scale())
+            p = softmax((k @ qv) * softmax_scale(d))
             out[b, h] = p @ v
     return out
 
@@ -243,7 +251,7 @@ def decode_absorbed(case, batches=None, heads=None, gate: Optional[bool] = None)
             qv = widen(case.q[b, h], d.dtype)
             q_nope, q_rope = qv[:d.d_nope], qv[d.d_nope:]
             q_hat = widen(case.w_uk[h], d.dtype).T @ q_nope          # [d_c]
-            s = (c_t @ q_hat + kr @ q_rope) * d.scale()
+            s = (c_t @ q_hat + kr @ q_rope) * softmax_scale(d)
             o_lat = softmax(s) @ c_t                                 # [d_c]
             out[b, h] = widen(case.w_uv[h], d.dtype) @ o_lat
     return out
@@ -281,7 +289,7 @@ def decode_r0(case, w_ukv_full: Optional[np.ndarray] = None, gate_r0: Optional[n
         for h in range(H):
             k = np.concatenate([kv[:, h, :dn], kr], axis=1)
             v = kv[:, h, dn:]
-            p = softmax((k @ widen(case.q[b, h], d.dtype)) * d.scale())
+            p = softmax((k @ widen(case.q[b, h], d.dtype)) * softmax_scale(d))
             out[b, h] = p @ v
     return out
 

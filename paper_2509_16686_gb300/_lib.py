@@ -8,7 +8,6 @@ cannot be built or loaded, ``load()`` raises.
 from __future__ import annotations
 
 import ctypes
-import math
 import os
 import threading
 from typing import Optional
@@ -325,7 +324,3 @@ def eg_mla_debug_set_trace(buf: Optional[torch.Tensor], ctas: int = 0) -> None:
         return
     _check(load().eg_mla_debug_set_trace(_ptr(buf), buf.numel() * buf.element_size(), ctas),
            "eg_mla_debug_set_trace")
-
-
-def default_scale(d_nope: int, d_rope: int) -> float:
-    return 1.0 / math.sqrt(d_nope + d_rope)

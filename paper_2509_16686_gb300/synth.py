@@ -62,12 +62,7 @@ class Dims:
     # ablations "mul" (LayerNorm removed) and "add_ln" ((*) replaced by +)
     gate_op: str = "mul_ln"
     ln_eps: float = 1e-5
-    softmax_scale: float = 0.0   # <= 0 means 1/sqrt(d_nope + d_rope)
-
-    def scale(self) -> float:
-        if self.softmax_scale > 0:
-            return float(self.softmax_scale)
-        return 1.0 / math.sqrt(self.d_nope + self.d_rope)
+    softmax_scale: float = 0.0   # <= 0: the method's default scale (the consumer's rule)
 
 
 @dataclasses.dataclass
@@ -225,7 +220,7 @@ def make_case(name: str, dims: Dims, seq_lens, *, seed: int, latent_scale: float
 
     q = _store(_normal(rng, (B, H, dn + dr), 1.0), dt)
     gate_table = _store(_normal(rng, (V, dc), 0.1, mean=1.0), dt)
-    wstd = 1.0 / math.sqrt(dc)
+    wstd = dc ** -0.5   # std of the N(0, d_c^-1/2) draw
     w_uk = _store(_normal(rng, (H, dn, dc), wstd), dt)
     w_uv = _store(_normal(rng, (H, dv, dc), wstd), dt)
     if affine_ln:
@@ -335,8 +330,8 @@ def make_layer_case(case: Case, n_embd: int, *, seed: int, rope_theta: float = 1
     return LayerCase(
         case=case, n_embd=E,
         x=_store(_normal(rng, (B, E), 1.0), dt),
-        w_q=_store(_normal(rng, (H * (dn + dr), E), 1.0 / math.sqrt(E)), dt),
-        w_kv_a=_store(_normal(rng, (dc + dr, E), 1.0 / math.sqrt(E)), dt),
+        w_q=_store(_normal(rng, (H * (dn + dr), E), E ** -0.5), dt),
+        w_kv_a=_store(_normal(rng, (dc + dr, E), E ** -0.5), dt),
         kv_norm_w=_store(_normal(rng, (dc,), 0.1, mean=1.0), dt),
-        w_o=_store(_normal(rng, (E, H * dv), 1.0 / math.sqrt(H * dv)), dt),
+        w_o=_store(_normal(rng, (E, H * dv), (H * dv) ** -0.5), dt),
         rope_theta=rope_theta, rms_eps=rms_eps)
