@@ -365,8 +365,9 @@ int eg_mla_profile_end(double* ms_sum, int32_t* launches);
  * eg_mla_decode at d_c 192 or 256 in the gate modes none and mul_ln run a
  * separately compiled traced build of the kernel (same results; the untraced
  * build carries no trace code), whose first `ctas` CTAs record, per role (0 TMA producer,
- * 1 MMA issuer, 2 gate, 3 softmax, 4 at d_c 192/256 the kernel phases: entry,
- * set-up done, tile loops done, split combine done), a run of (tag, SM clock) pairs of 8-byte
+ * 1 MMA issuers: the score issuer in the first half of the run, the output
+ * issuer in the second, 2 gate, 3 softmax, 4 at d_c 192/256 the kernel phases:
+ * entry, set-up done, tile loops done, split combine done), a run of (tag, SM clock) pairs of 8-byte
  * words, tag = event << 56 | tile index << 32 | low 32 bits of the global
  * nanosecond timer; run r of CTA c starts at word (c * 5 + r) * cap * 2 with
  * cap = bytes / (ctas * 5 * 16).  The caller zeroes

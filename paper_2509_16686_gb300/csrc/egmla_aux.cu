@@ -96,12 +96,52 @@ __device__ void page_prefix_sums(const int32_t* seq_lens, int batch, int page_si
   if (lane == 0) cu[batch] = carry;
 }
 
+// Start record of every split (see SplitStart), from the prefix sums this
+// block just wrote (plain loads: they are this kernel's own stores).  Split c
+// owns units [c chunk, (c + 1) chunk); its first sequence is the last one whose
+// first unit is at most c chunk (empty sequences skipped), as in the decode
+// kernel's walk.
+__device__ void split_starts(const int32_t* cu, const int32_t* seq_lens, int batch, int num_splits,
+                             const int32_t* __restrict__ block_table, int max_pages, SplitStart* starts) {
+  const int total = cu[batch];
+  const int chunk = split_chunk(total, num_splits);
+  for (int c = threadIdx.x; c < num_splits; c += blockDim.x) {
+    SplitStart st;
+    const int g0 = c * chunk;
+    st.g1 = min(g0 + chunk, total);
+    st.b = st.lp = st.lp_end = st.L = st.npages = st.pad = 0;
+    st.done = g0 >= st.g1;
+    if (!st.done) {
+      int lo = 0, hi = batch - 1;
+      while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (cu[mid] <= g0) lo = mid; else hi = mid - 1;
+      }
+      while (lo < batch - 1 && cu[lo + 1] <= g0) ++lo;
+      const int base = cu[lo] + kSegCost;   // unit of the sequence's first page
+      st.b = lo;
+      st.lp = max(g0 - base, 0);
+      st.lp_end = min(st.g1, cu[lo + 1]) - base;
+      st.L = seq_lens[lo];
+      st.done = st.lp_end <= st.lp;
+      if (!st.done) st.npages = min(kStartPages, min(st.lp_end, max_pages) - st.lp);
+    }
+    for (int i = 0; i < kStartPages; ++i)
+      st.page[i] = i < st.npages ? block_table[static_cast<size_t>(st.b) * max_pages + st.lp + i] : -1;
+    const int4* src = reinterpret_cast<const int4*>(&st);
+    int4* dst = reinterpret_cast<int4*>(starts + c);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) dst[k] = src[k];
+  }
+}
+
 // Tensor-core path: block (head h, chunk of kSumFeatures = 32 latent features,
 // group of up to kPBatch sequences) computes q^_{b,h}[f] = sum_n W_UK,h[n][f] q^C_{b,h}[n]
 // in fp32 and stores (q^ (*) gamma) rounded to bf16 in the prepared query
 // block (qop_offset layout).  Its per-chunk partials of w_h = sum_f bf16(q^ gamma)_f
 // and b_h = q^_h . beta go to the block's slots of the sums area.  Chunk-0
-// blocks also copy q^R.  The last block computes the page prefix sums.
+// blocks also copy q^R.  The last block computes the page prefix sums and the
+// splits' start records.
 //  - All 16-byte global loads of a thread are issued before any is stored
 //    (W_UK with an L2 evict-last hint: it stays in L2 across steps).
 //  - W_UK and q^C are staged row-major; a warp takes a quad of sequences and
@@ -119,7 +159,8 @@ __global__ void prologue_tc_kernel(const __nv_bfloat16* __restrict__ q, const __
                        const float* __restrict__ gamma, const float* __restrict__ beta,
                        const int32_t* __restrict__ seq_lens, int batch, int d_nope, int d_rope, int d_c,
                        int page_size, uint8_t* __restrict__ qprep, size_t qstride, int32_t* __restrict__ cu,
-                       uint32_t* __restrict__ seq_done) {
+                       uint32_t* __restrict__ seq_done, int num_splits, const int32_t* __restrict__ block_table,
+                       int max_pages, SplitStart* __restrict__ starts) {
   __shared__ __align__(16) __nv_bfloat16 ws[kPMaxNope][kSumFeatures];  // W_UK,h[n][f0 + f]
   __shared__ __align__(16) __nv_bfloat16 qs[kPBatch][kPMaxNope];      // q^C_{b0 + j, h}[n]
   // partial sums [n part * 4 quads + j][f], written once every warp is done with ws
@@ -132,6 +173,8 @@ __global__ void prologue_tc_kernel(const __nv_bfloat16* __restrict__ q, const __
     if (seq_done != nullptr)
       for (int i = threadIdx.x; i <= batch; i += blockDim.x) seq_done[i] = 0u;
     page_prefix_sums(seq_lens, batch, page_size, cu);
+    __syncthreads();   // the prefix sums are visible to the whole block
+    split_starts(cu, seq_lens, batch, num_splits, block_table, max_pages, starts);
     return;
   }
   if (q == nullptr) return;  // cache-read test entry: prefix sums only
@@ -557,7 +600,8 @@ cudaError_t launch_prologue_tc(const DecodeArgs& a, cudaStream_t st) {
   prologue_tc_kernel<<<16 * (a.d_c / kSumFeatures) * ngroups + 1, 256, 0, st>>>(
       static_cast<const __nv_bfloat16*>(a.q), static_cast<const __nv_bfloat16*>(a.w_uk), gamma, beta,
       a.seq_lens, a.batch, a.d_nope, a.d_rope, a.d_c, a.page_size, ws + wl.off_qprep, wl.qprep_stride,
-      reinterpret_cast<int32_t*>(ws + wl.off_cu), reinterpret_cast<uint32_t*>(ws + wl.off_done));
+      reinterpret_cast<int32_t*>(ws + wl.off_cu), reinterpret_cast<uint32_t*>(ws + wl.off_done), a.num_splits,
+      a.block_table, a.max_pages, reinterpret_cast<SplitStart*>(ws + wl.off_start));
   return cudaGetLastError();
 }
 

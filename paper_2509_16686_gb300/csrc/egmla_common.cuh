@@ -24,15 +24,15 @@ __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a -
 // matrices, then, per chunk of kSumFeatures latent features, the per-head fp32
 // partial sums of w_h = sum_f bf16(q^ gamma)_hf and b_h = q^_h . beta
 // ([d_c / kSumFeatures][2][16] floats; the consumer adds the chunks in order,
-// so the result does not depend on launch order).  In every group of 8 columns
-// (512 bytes) heads 0-7 fill core-matrix row group 0 and heads 8-15 row group
-// 2.  Read as the A operand of an M = 64 MMA (row-group stride 128 B) the two
-// head halves land in TMEM lane quadrants 0 and 1; read as an N = 16 B operand
-// (row-group stride 256 B) they are its 16 rows.  The unused row groups are
-// never written.
-constexpr int kQGroupBytes = 512;
+// so the result does not depend on launch order).  Every group of 8 columns
+// (one K core of the operand, 256 bytes) holds heads 0-7 in its first 128
+// bytes and heads 8-15 in its second: read as the N = 16 B operand of the
+// score MMA (K-major, no swizzle) the K cores are 256 B apart and the two
+// 8-head row groups 128 B apart.
+constexpr int kQGroupBytes = 256;
+constexpr int kQRowGroupBytes = 128;
 __host__ __device__ constexpr size_t qop_offset(int h, int k) {
-  return static_cast<size_t>(k / 8) * kQGroupBytes + (h / 8) * 256 + (h % 8) * 16 + (k % 8) * 2;
+  return static_cast<size_t>(k / 8) * kQGroupBytes + (h / 8) * kQRowGroupBytes + (h % 8) * 16 + (k % 8) * 2;
 }
 __host__ __device__ constexpr size_t qprep_lat_bytes(int d_c) { return static_cast<size_t>(d_c / 8) * kQGroupBytes; }
 __host__ __device__ constexpr size_t qprep_rope_bytes(int d_rope) {
@@ -51,8 +51,21 @@ __host__ __device__ inline size_t qprep_bytes_f32(int H, int d_c, int d_rope) {
   return align_up(static_cast<size_t>(H) * (d_c + d_rope) * 4, 16);
 }
 
+// Where a split's page walk starts, written by the prologue kernel, so that
+// each role of the decode kernel reads it with one round of loads instead of
+// searching the prefix sums: the sequence b, the split's first page lp and
+// end lp_end in it, the sequence length L, the split's end unit g1, whether
+// the split is empty, and the physical ids of the first npages pages of the
+// walk (at most kStartPages, all in sequence b).
+constexpr int kStartPages = 8;
+struct alignas(16) SplitStart {
+  int32_t b, lp, lp_end, L, g1, done, npages, pad;
+  int32_t page[kStartPages];
+};
+static_assert(sizeof(SplitStart) == 64, "split start record");
+
 struct WorkspaceLayout {
-  size_t off_cu, off_done, off_qprep, off_ml, off_o, total;
+  size_t off_cu, off_done, off_start, off_qprep, off_ml, off_o, total;
   size_t qprep_stride;
   int num_slots;
 };
@@ -69,6 +82,8 @@ __host__ __device__ inline WorkspaceLayout workspace_layout(int batch, int num_s
   // CTAs done, [1 + b] the split partials of sequence b stored
   w.off_done = off;
   off = align_up(off + static_cast<size_t>(batch + 1) * 4, 256);
+  w.off_start = off;
+  off = align_up(off + static_cast<size_t>(num_splits) * sizeof(SplitStart), 256);
   w.off_qprep = off;
   off = align_up(off + static_cast<size_t>(batch) * w.qprep_stride, 256);
   w.off_ml = off;

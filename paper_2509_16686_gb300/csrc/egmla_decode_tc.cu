@@ -3,42 +3,48 @@
 //
 // One CTA per split-KV work unit (see egmla_common.cuh for the schedule).  The
 // CTA streams its cache pages, one 64-token page per tile, through a ring of
-// shared-memory slots.  Four roles run concurrently on different tiles:
+// shared-memory slots; the tiles are token rows of the tensor-core operations
+// (M = 64 tokens), the 16 heads their columns (N = 16).  Roles:
 //
-//   TMA (warp 3)      latent page [64 tok x d_c] (one 3-D box: 64-feature
+//   TMA (warp 4)      latent page [64 tok x d_c] (one 3-D box: 64-feature
 //                     columns x 64 rows) and RoPE-key page [64 x 64], both
-//                     128-byte swizzled.
-//   gate (warps 4-11; each quarter-warp owns two token rows, lane u the 16-byte
-//                     unit u of every 64-feature column of them)
+//                     128-byte swizzled, as soon as the page slot is free.
+//   gate (warps 7-14; each quarter-warp owns two token rows, lane u the 16-byte
+//                     units 2u, 2u + 1 of every 64-feature column of them)
 //                     the token ids (two tiles ahead) and the gate rows
 //                     g = G[id] (EG-MLA-A table, Section 5.2; one tile ahead)
 //                     from L2 into registers, every quarter-warp load reading
 //                     one whole 128-byte line; z = c (*) g rounded to bf16 and
 //                     written back in place, and the LayerNorm statistics
 //                     mu, r = 1/sqrt(var + eps) of z (Eq. 5 over d_c).
-//   scores (warp 2)   transposed scores S^T = Q Z^T and S_rope^T = Q^R K^R^T on
-//                     tcgen05 (M = 64 rows, N = 64 tokens, fp32 in TMEM,
-//                     double-buffered).  The operand rows of heads 0-7 and 8-15
-//                     are placed so that their accumulator rows fall in TMEM lane
-//                     quadrants 0 and 1.
-//   output (warp 3, with the TMA loads) the latent output O += P' Z (M = 64
-//                     rows, N = d_c features, K = 64 tokens), accumulated in
-//                     TMEM over a sequence segment.  Issued by its own thread, so
-//                     that the scores of later tiles never queue behind it.
-//   softmax (warps 0 and 1, heads 0-7 and 8-15)
-//                     reads its eight head rows of S^T spread over the 32
-//                     threads (one head x 16 tokens each), s = scale * (r (S -
-//                     mu w) + b + S_rope) -- the LayerNorm applied after the MMA,
-//                     since q^.LN(z) = r (q^ gamma).z - r mu sum(q^ gamma) +
-//                     q^.beta --, an online softmax whose per-head maxima need no
-//                     exchange beyond the four threads of a head, and P' = p r
-//                     (bf16) as the A operand of the output MMA.
+//   scores (warp 5)   S = Z (q^ gamma)^T and S_rope = K^R q^R^T (M = 64 tokens,
+//                     N = 16 heads, K = d_c and 64; fp32 in TMEM, four score
+//                     buffers) as soon as a gated page and a score buffer are
+//                     ready, and the query block of the next sequence segment
+//                     (the warp polls both conditions, so neither waits for
+//                     the other).
+//   output (warp 6)   O^T += Z^T P' (M = 128 latent features, N = 16 heads,
+//                     K = 64 tokens; O^T stays in TMEM over a sequence
+//                     segment).  An issuing thread stalls while the tensor
+//                     pipe's queue is full, so the two MMA streams have a
+//                     thread each.
+//   softmax (warps 0-3, one per TMEM lane quadrant: tokens 16w .. 16w + 15)
+//                     thread t reads two tokens x four heads of S; the
+//                     LayerNorm is applied after the MMA, since
+//                       q^.LN(z) = r (q^ gamma).z - r mu sum(q^ gamma) + q^.beta,
+//                     s = scale (r (S - mu w) + b + S_rope); an online softmax
+//                     whose per-head reference max moves only when a tile
+//                     exceeds it by 2^8 (one barrier vote of the four warps per
+//                     tile decides; the maxima are exchanged only then), and
+//                     P' = p r (bf16) as the B operand of the output MMA.
 //
-// With heads in the accumulator rows, the running max, its lazy rescaling of
-// O and the final read-out of a head all stay inside one softmax warp.  At the end of each
-// sequence segment the un-normalised latent output gamma (*) (O - sum_j P'_j
-// mu_j) + beta l, the running max m and the denominator l = sum_j P'_j / r_j are
-// written as this split's partial result.
+// At the end of each sequence segment the four softmax warps read O^T (latent
+// features in TMEM lanes) and write the split's partial result: the
+// un-normalised latent output gamma (*) (O - sum_j P'_j mu_j) + beta l, the
+// reference max m and the denominator l = sum_j P'_j / r_j.  With heads as
+// the MMA columns, no tensor-core work is spent on padding rows, tensor
+// memory holds four score buffers and the whole output in 160 columns, and the
+// query block takes 10 KB, which leaves room for five page slots at d_c = 256.
 //
 // The queries are absorbed before this kernel (q^ = W_UK^T q^C, with gamma
 // folded in); W_UV is applied after the split merge.  Everything the kernel
@@ -61,17 +67,25 @@ namespace {
 
 constexpr int kHeads = 16;
 constexpr int kRope = 64;
-constexpr int kThreads = 384;
-constexpr int kSoftWarps = 2;    // warps 0 and 1: TMEM lane quadrants 0 and 1 hold heads 0-7 and 8-15
-constexpr int kMmaWarp = 2;
-constexpr int kTmaWarp = 3;
-constexpr int kGateWarp0 = 4;
+constexpr int kThreads = 480;
+constexpr int kSoftWarps = 4;    // warps 0-3: TMEM lane quadrants 0-3
+constexpr int kSoftThreads = 32 * kSoftWarps;
+constexpr int kTmaWarp = 4;
+constexpr int kMmaWarp = 5;      // score MMAs and query blocks; also allocates and frees TMEM
+constexpr int kOutWarp = 6;      // output MMAs
+constexpr int kGateWarp0 = 7;
 constexpr int kGateWarps = 8;
 constexpr uint32_t kSmemLimit = 232448;
+// named barriers of the softmax warps (0 is __syncthreads)
+constexpr int kBarTile = 1;
+constexpr int kBarXch = 2;
 // sequences per unit of the fused combine
 constexpr uint32_t kFusedMaxG = 16;
 // a head's reference max moves only when a tile exceeds it by 2^8
 constexpr float kLazyLog2 = 8.f;
+// score buffers in TMEM and P' buffers in shared memory
+constexpr int kNB = 4;
+constexpr int kNP = 4;
 
 template <int D_C, bool GATE>
 struct Cfg {
@@ -79,45 +93,46 @@ struct Cfg {
   static constexpr uint32_t PCHUNK = kPage * 128;       // one atom column of a page: 8 KB
   static constexpr uint32_t KR_OFF = NCH * PCHUNK;
   static constexpr uint32_t SLOT = KR_OFF + PCHUNK;     // latent + RoPE key of one page
+  static constexpr uint32_t STAT_BYTES = GATE ? 2 * kPage * 4 : 0;   // per slot: mu[64], r[64]
   static constexpr uint32_t QB_LAT = qprep_lat_bytes(D_C);
-  static constexpr uint32_t QB_ROPE = qprep_rope_bytes(kRope);
   static constexpr uint32_t QPREP = qprep_bytes_tc(D_C, kRope);
-  // two query blocks (the next sequence's loads while this one is in use)
   static constexpr uint32_t QBUF = (QPREP + 127) / 128 * 128;
-  // P' [16 heads x 64 tokens] in the layout of the query block (qop_offset)
-  static constexpr uint32_t PBUF = kPage / 8 * kQGroupBytes;
-  static constexpr uint32_t STAT_BYTES = 3 * kPage * 4;   // per slot: mu[64], r[64], 1/r[64]
+  // P' [64 tokens x 16 heads] as the MN-major B operand of the output MMA
+  static constexpr uint32_t PBUF = kPage * kHeads * 2;
+  // LayerNorm gamma and beta of the segment read-out
+  static constexpr uint32_t GB_BYTES = GATE ? 2 * D_C * 4 : 0;
+  // softmax exchange: tile maxima [4 warps][16], segment sums [4 warps][16][2]
+  static constexpr uint32_t XCH = 1024;
   static constexpr uint32_t MISC = 1024;
-  // LayerNorm gamma and beta of the segment read-out, one copy per softmax warp
-  static constexpr uint32_t GB_BYTES = 2 * D_C * 4;
-  static constexpr int NS_FIT =
-      (int)((kSmemLimit - 1024 - 2 * QBUF - 2 * PBUF - 2 * GB_BYTES - MISC) / (SLOT + STAT_BYTES));
+  static constexpr uint32_t FIXED = kNP * PBUF + GB_BYTES + XCH + MISC + 1024;
+  // slots with two query buffers (the next segment's loaded while this one is
+  // in use) or with one; one buffer when a second would cost a slot below five
+  static constexpr int NS2 = (int)((kSmemLimit - FIXED - 2 * QBUF) / (SLOT + STAT_BYTES));
+  static constexpr int NS1 = (int)((kSmemLimit - FIXED - QBUF) / (SLOT + STAT_BYTES));
+  static constexpr int NQ = (NS2 < 5 && NS1 > NS2) ? 1 : 2;
+  static constexpr int NS_FIT = NQ == 2 ? NS2 : NS1;
   static constexpr int NS = NS_FIT > 6 ? 6 : NS_FIT;
   static constexpr uint32_t OFF_QBUF = NS * SLOT;
-  static constexpr uint32_t OFF_PBUF = OFF_QBUF + 2 * QBUF;
-  static constexpr uint32_t OFF_STAT = OFF_PBUF + 2 * PBUF;
+  static constexpr uint32_t OFF_PBUF = OFF_QBUF + NQ * QBUF;
+  static constexpr uint32_t OFF_STAT = OFF_PBUF + kNP * PBUF;
   static constexpr uint32_t OFF_GB = OFF_STAT + NS * STAT_BYTES;
-  static constexpr uint32_t OFF_MISC = OFF_GB + 2 * GB_BYTES;
+  static constexpr uint32_t OFF_XCH = OFF_GB + GB_BYTES;
+  static constexpr uint32_t OFF_MISC = OFF_XCH + XCH;
   static constexpr uint32_t SMEM = OFF_MISC + MISC + 1024;
-  // TMEM columns: two score buffers of (latent 64 + RoPE 64) token columns, then
-  // the latent output (d_c columns), rows = heads
-  static constexpr uint32_t S_COLS = 128;
-  static constexpr uint32_t COL_S = 0, COL_O = 2 * S_COLS;
-  static constexpr uint32_t TMEM_COLS = 512;
+  // TMEM columns: kNB score buffers of (latent 16 + RoPE 16) head columns,
+  // then the latent output O^T (16 head columns per 128-feature M chunk)
+  static constexpr uint32_t S_COLS = 32;
+  static constexpr uint32_t COL_S = 0, COL_O = kNB * S_COLS;
+  static constexpr uint32_t TMEM_COLS = 256;
   static constexpr uint32_t PAGE_TX = SLOT;
-  static_assert(NS >= 2, "the ring needs two page slots");
+  static_assert(NS >= 3, "the ring needs three page slots");
   static_assert(SMEM <= kSmemLimit, "shared memory");
   static_assert(D_C == 192 || D_C == 256, "latent widths of this kernel");
-  static_assert(COL_O + D_C <= TMEM_COLS, "tensor memory");
-  // The M = 64 MMAs read 64 operand rows (8 row groups 128 B apart in each of
-  // the two 512-byte K groups of a step), 16 of which are heads: a step reads
-  // up to 1536 bytes from its start (the other rows land in TMEM lanes nobody
-  // reads).  Every such read stays inside the allocation:
-  static constexpr uint32_t STEP_SPAN = kQGroupBytes + 8 * 128;
-  static_assert(OFF_QBUF + QBUF + QB_LAT + (kRope / 16 - 1) * 2 * kQGroupBytes + STEP_SPAN <= OFF_MISC,
-                "query over-read");
-  static_assert(OFF_PBUF + PBUF + (kPage / 16 - 1) * 2 * kQGroupBytes + STEP_SPAN <= OFF_MISC + MISC,
-                "weight over-read");
+  static_assert(COL_O + 32 <= TMEM_COLS, "tensor memory");
+  // first latent feature of output M chunk j (two chunks of 128 rows); for
+  // D_C = 192 the second chunk starts at 64 and overlaps the first, so that no
+  // MMA reads past the latent part of a slot (its rows 64..127 are not read out)
+  __host__ __device__ static constexpr int mc_start(int j) { return j == 0 ? 0 : D_C - 128; }
   // fused combine: W_UV,h (at most 256 rows) and up to kFusedMaxG merged
   // latent rows reuse the page-slot area
   static_assert(256u * D_C * 2 + kFusedMaxG * D_C * 4 + 128 <= OFF_QBUF, "fused combine area");
@@ -132,6 +147,7 @@ struct TcParams {
   const float* beta;
   const uint8_t* qprep;
   const int32_t* cu;
+  const SplitStart* starts;
   float* part_ml;
   float* part_o;
   int32_t* status;
@@ -162,12 +178,13 @@ template <bool ON>
 struct TracerT {
   unsigned long long* base;
   int n, cap;
-  __device__ void init(const TcParams& p, int role) {
+  // part 0 of 1 is the role's whole run; part k of 2 is half of it (two writers)
+  __device__ void init(const TcParams& p, int role, int part = 0, int parts = 1) {
     base = nullptr;
     n = 0;
-    cap = p.trace_cap;
+    cap = p.trace_cap / parts;
     if (ON && p.trace != nullptr && static_cast<int>(blockIdx.x) < p.trace_ctas)
-      base = p.trace + (static_cast<size_t>(blockIdx.x) * kTraceRoles + role) * p.trace_cap * 2;
+      base = p.trace + ((static_cast<size_t>(blockIdx.x) * kTraceRoles + role) * p.trace_cap + part * cap) * 2;
   }
   __device__ __forceinline__ void mark(int event, int tile) {
     if (ON && base != nullptr && n < cap) {
@@ -195,11 +212,8 @@ __device__ __forceinline__ void phase_mark(const TcParams& p, int event) {
 struct Bars {
   uint64_t full[6], empty[6], zready[6];
   uint64_t qfull[2], qempty[2];
-  uint64_t s_ready[2], pfree[2];
-  // weights of tile j ready: sp_done[j & 1] (the two softmax warps may be one
-  // tile apart, never two: tile j + 2's scores follow tile j's output MMA)
-  uint64_t sp_done[2];
-  uint64_t sfree[2];           // the softmax warps have read score buffer b
+  uint64_t sready[kNB], sfree[kNB];
+  uint64_t spdone[kNP], pfree[kNP];
   uint64_t drain_s, drain_o;   // all MMAs of the score / output issuer done
   uint64_t wbar;               // W_UV rows of the fused combine landed
   uint32_t tmem_base;
@@ -219,18 +233,20 @@ struct Walker {
   int batch, g1, b, lp, lp_end, L;
   bool first, done;
 
-  __device__ void start(const int32_t* cu_, const int32_t* lens_, int batch_) {
-    cu = cu_;
-    lens = lens_;
-    batch = batch_;
-    const int total = __ldg(cu + batch);
-    const int chunk = split_chunk(total, gridDim.x);
-    const int g0 = blockIdx.x * chunk;
-    g1 = min(g0 + chunk, total);
-    done = g0 >= g1;
-    if (done) return;
-    b = find_sequence(cu, batch, g0);
-    enter(g0);
+  // the split's start record (written by the prologue kernel): one round of loads
+  __device__ void start(const TcParams& p) {
+    cu = p.cu;
+    lens = p.seq_lens;
+    batch = p.batch;
+    const int4* r = reinterpret_cast<const int4*>(p.starts + blockIdx.x);
+    const int4 h0 = __ldg(r), h1 = __ldg(r + 1);
+    b = h0.x;
+    lp = h0.y;
+    lp_end = h0.z;
+    L = h0.w;
+    g1 = h1.x;
+    done = h1.y != 0;
+    first = true;
   }
   __device__ void enter(int g) {
     const int base = __ldg(cu + b) + kSegCost;   // unit of the sequence's first page
@@ -266,12 +282,21 @@ struct Walker {
 
 // Page of tile t through a 32-entry window of the block table held one entry per
 // lane (whole warp; the window moves when the tile leaves it).
+// The window starts as the first pages of the split's start record.
 struct PageWindow {
-  int b = -1, base = 0, reg = -1;
+  int b = -1, base = 0, n = 0, reg = -1;
+  __device__ __forceinline__ void init(const TcParams& p, int lane) {
+    const SplitStart* r = p.starts + blockIdx.x;
+    b = __ldg(&r->b);
+    base = __ldg(&r->lp);
+    n = __ldg(&r->npages);
+    reg = lane < kStartPages ? __ldg(&r->page[lane]) : -1;
+  }
   __device__ __forceinline__ int page(const TcParams& p, const Tile& t, int lane) {
-    if (t.b != b || t.lp >= base + 32) {
+    if (t.b != b || t.lp < base || t.lp >= base + n) {
       b = t.b;
       base = t.lp;
+      n = 32;
       const int lp = t.lp + lane;
       reg = lp < p.max_pages ? __ldg(p.block_table + static_cast<size_t>(t.b) * p.max_pages + lp) : -1;
     }
@@ -296,6 +321,30 @@ __device__ __forceinline__ void warp_arrive(uint32_t bar) {
   if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
 }
 
+// lane 0's non-blocking test of a phase, the same answer in every lane
+__device__ __forceinline__ bool warp_test(uint32_t bar, uint32_t parity) {
+  return __shfl_sync(0xffffffffu, mbar_test_now(bar, parity) ? 1 : 0, 0) != 0;
+}
+
+// Named barrier of the softmax warps that also ORs a predicate over them: every
+// participant gets the same answer, so a branch on it is uniform.
+__device__ __forceinline__ bool soft_vote(int id, bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "barrier.cta.red.or.pred q, %2, %3, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(v ? 1u : 0u), "r"(id), "r"(kSoftThreads)
+      : "memory");
+  return r != 0;
+}
+
+__device__ __forceinline__ void soft_sync(int id) {
+  asm volatile("barrier.cta.sync %0, %1;" ::"r"(id), "r"(kSoftThreads) : "memory");
+}
+
 __device__ __forceinline__ float2 unpack_bf16x2(uint32_t w) {
   return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
 }
@@ -307,12 +356,70 @@ __device__ __forceinline__ uint32_t mul_bf16x2(uint32_t a, uint32_t b) {
   return *reinterpret_cast<uint32_t*>(&z);
 }
 
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 z = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&z);
+}
+
 // 2^x with the hardware approximation (max 2 ulp; the weights are rounded to
 // bf16 right after, and -inf gives 0)
 __device__ __forceinline__ float ex2_approx(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+// 16 lanes x 32 columns of 32-bit (tcgen05.ld.16x256b.x4): thread t gets lanes
+// t/4 and t/4 + 8 at columns 8k + 2(t%4) and 8k + 2(t%4) + 1 of every 8-column
+// group k, as v[4k] = (t/4, 8k + 2(t%4)), v[4k + 1] = (t/4, +1),
+// v[4k + 2] = (t/4 + 8, ...), v[4k + 3] = (t/4 + 8, +1)
+__device__ __forceinline__ void tmem_ld_16x256b_x4(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.16x256b.x4.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// 32 lanes x 32 columns of 32-bit: thread i of the warp gets its lane's 32 values
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, "
+      "%23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// inverse of tmem_ld32 (same thread-to-element map)
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const float (&v)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, "
+      "%24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
+      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])), "r"(__float_as_uint(v[3])),
+      "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])), "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])),
+      "r"(__float_as_uint(v[8])), "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+      "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+      "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])),
+      "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])),
+      "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])),
+      "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])),
+      "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])),
+      "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
+      : "memory");
 }
 
 // ---------------------------------------------------------------- fused split combine
@@ -358,7 +465,7 @@ __device__ __forceinline__ float reduce8_rows(const float (&v)[8], int lane) {
 // resident, so a wait on other CTAs cannot starve).  A CTA merges its units
 // (head h, group of cmb_g sequences) once their split partials are stored:
 // with one sequence per unit (small batches) as soon as the softmax warps of
-// the splits that covered that sequence have counted their halves on its
+// the splits that covered that sequence have counted their parts on its
 // counter, otherwise after every CTA has arrived on a grid counter (both
 // counters zeroed by the prologue kernel of the same call).  For each sequence
 // b, over the splits s that covered it,
@@ -419,8 +526,8 @@ __device__ void fused_combine(const TcParams& p, uint8_t* smem, Bars& bars) {
     const int h = u % kHeads, grp = u / kHeads;
     const int b0 = grp * G, nb = min(G, p.batch - b0);
     if (G == 1 && tid == 0 && !*abort_flag) {
-      // a unit of one sequence: both halves of every split partial of it stored
-      const uint32_t want = 2u * static_cast<uint32_t>(splits_of(b0));
+      // a unit of one sequence: every softmax warp's part of every split partial of it stored
+      const uint32_t want = static_cast<uint32_t>(kSoftWarps) * static_cast<uint32_t>(splits_of(b0));
       const uint64_t t0 = globaltimer();
       while (ld_acquire_gpu(p.seq_done + 1 + b0) < want) {
         if (*abort_flag) break;
@@ -522,11 +629,6 @@ __device__ void fused_combine(const TcParams& p, uint8_t* smem, Bars& bars) {
   }
 }
 
-__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
-  __nv_bfloat162 z = __floats2bfloat162_rn(lo, hi);
-  return *reinterpret_cast<uint32_t*>(&z);
-}
-
 // GM: gate mode (0 none, 1 LN(c (*) g), 2 c (*) g, 3 LN(c + g): eg_mla_gate_mode)
 // DBG: 0 the decode, 1 the cache-read dump (raw pages and gate rows, no
 // attention), 2 the decode with the pipeline trace
@@ -559,16 +661,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(smem_u32(&bars.qfull[s]), 1);
+      // the last score MMA of the segment (commit) and the softmax warps' read of its sums
       mbar_init(smem_u32(&bars.qempty[s]), 1 + kSoftWarps);
+    }
+    for (int s = 0; s < kNB; ++s) {
       // the MMA commit plus a release arrival of the MMA warp after it saw the
       // gate's zready (so that the statistics are visible to the softmax warps)
-      mbar_init(smem_u32(&bars.s_ready[s]), 2);
+      mbar_init(smem_u32(&bars.sready[s]), 2);
+      mbar_init(smem_u32(&bars.sfree[s]), kSoftWarps);
+    }
+    for (int s = 0; s < kNP; ++s) {
+      mbar_init(smem_u32(&bars.spdone[s]), kSoftWarps);
       mbar_init(smem_u32(&bars.pfree[s]), 1);
     }
-    mbar_init(smem_u32(&bars.sp_done[0]), kSoftWarps);
-    mbar_init(smem_u32(&bars.sp_done[1]), kSoftWarps);
-    mbar_init(smem_u32(&bars.sfree[0]), kSoftWarps);
-    mbar_init(smem_u32(&bars.sfree[1]), kSoftWarps);
     mbar_init(smem_u32(&bars.drain_s), 1);
     mbar_init(smem_u32(&bars.drain_o), 1);
     mbar_init(smem_u32(&bars.wbar), 1);
@@ -585,77 +690,39 @@ __global__ void __launch_bounds__(kThreads, 1)
   phase_mark<DBG == 2>(p, 1);
   const uint32_t tmem = bars.tmem_base;
 
-  constexpr uint32_t KSTEP = 2 * kQGroupBytes;   // bytes of 16 columns of an A operand
   if (warp == kTmaWarp) {
-    // ---------------------------------------------------------------- TMA producer + output MMAs
-    // The whole warp walks the tiles; lane 0 waits and issues the copies.
-    // Before a page slot is reused the output MMA of the tile that held it is
-    // issued here (it is what frees the slot), as soon as that tile's weights
-    // are ready; the remaining ones after the last copy.
+    // ---------------------------------------------------------------- TMA producer
+    // The whole warp walks the tiles; lane 0 waits for the slot and issues the
+    // copies.  A slot is free once the output MMA of the tile that held it is
+    // complete.
     if (lane == 0) {
       prefetch_tensormap(&cmap);
       prefetch_tensormap(&krmap);
     }
     const uint64_t pol_stream = policy_evict_first();
-    constexpr uint32_t IDESC_PV = idesc_bf16(64, D_C, 0, 1);
-    // A operand P' in 8x8 core matrices (K groups 512 B apart, row groups
-    // 128 B); B operand: the page slot read MN-major (features along N, tokens
-    // along K)
-    const uint64_t pdesc0 = smem_desc(sbase + C::OFF_PBUF, kQGroupBytes, 128, kSwizzleNone);
-    const uint64_t zdesc_mn = smem_desc(sbase, C::PCHUNK, 1024, kSwizzle128B);
-    Walker w, wo;
-    w.start(p.cu, p.seq_lens, p.batch);
-    wo.start(p.cu, p.seq_lens, p.batch);
+    Walker w;
+    w.start(p);
     PageWindow pw;
-    Tile t, to;
-    int it = 0, io = 0;
+    pw.init(p, lane);
+    Tile t;
+    int it = 0;
     int last_it[6] = {-1, -1, -1, -1, -1, -1};
-    bool issued_o = false;
     Tracer tr;
     tr.init(p, 0);
     if (lane != 0) tr.base = nullptr;
     bool ok_loop = true;
-    // output MMA of the next tile in order (O += P' Z); false on a timeout
-    auto output = [&]() -> bool {
-      if (!wo.next(to)) return true;
-      if (!warp_wait(smem_u32(&bars.sp_done[io & 1]), (io >> 1) & 1, abort_flag)) return false;
-      tc_fence_after();
-      if (elect_one()) {
-        const int slot = io % C::NS;
-        const uint64_t zb = zdesc_mn + ((slot * C::SLOT) >> 4);
-        const uint64_t pa = pdesc0 + (((io & 1) * C::PBUF) >> 4);
-        if (to.first) {
-#pragma unroll
-          for (int ks = 0; ks < kPage / 16; ++ks)
-            mma_bf16_ss(tmem + C::COL_O, pa + ((ks * KSTEP) >> 4), zb + ((ks * 2048) >> 4), IDESC_PV, ks > 0);
-        } else {
-#pragma unroll
-          for (int ks = 0; ks < kPage / 16; ++ks)
-            mma_bf16_ss(tmem + C::COL_O, pa + ((ks * KSTEP) >> 4), zb + ((ks * 2048) >> 4), IDESC_PV, 1);
-        }
-        mma_commit(smem_u32(&bars.empty[slot]));
-        mma_commit(smem_u32(&bars.pfree[io & 1]));
-      }
-      __syncwarp();
-      issued_o = true;
-      ++io;
-      return true;
-    };
     while (ok_loop && w.next(t)) {
       const int pg = pw.page(p, t, lane);
       const int slot = it % C::NS;
-      // the tile that held this slot must have had its output MMA issued
-      if (!DUMP && it >= C::NS && !output()) break;
       if (lane == 0) {
         tr.mark(0, it);
-        if (ok_loop && !mbar_wait(smem_u32(&bars.empty[slot]), ((it / C::NS) & 1) ^ 1, abort_flag)) ok_loop = false;
+        if (!mbar_wait(smem_u32(&bars.empty[slot]), ((it / C::NS) & 1) ^ 1, abort_flag)) ok_loop = false;
         if (ok_loop) {
           tr.mark(1, it);
           const bool ok = pg >= 0 && pg < p.num_pages;
           if (!ok) report_status(p.status, kStatusOutOfRange);
           const uint32_t fb = smem_u32(&bars.full[slot]);
           mbar_arrive_expect_tx(fb, ok ? C::PAGE_TX : 0u);
-          tr.mark(3, it);
           if (ok) {
             const uint32_t dst = sbase + slot * C::SLOT;
             const int y = pg * kPage;
@@ -669,134 +736,189 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok_loop = __shfl_sync(0xffffffffu, ok_loop, 0);
       ++it;
     }
-    // the output MMAs of the last tiles
-    if (!DUMP && ok_loop)
-      while (io < it)
-        if (!output()) break;
-    if (!DUMP && issued_o) {
-      // every output MMA must finish before TMEM is released
-      if (elect_one()) mma_commit(smem_u32(&bars.drain_o));
-      __syncwarp();
-      mbar_wait(smem_u32(&bars.drain_o), 0, abort_flag);
-    }
     if (lane == 0) {
-      // drain: every copy this thread issued must land before the CTA exits
+      // drain: every copy this thread issued must land before the CTA exits,
+      // also after an abort (own flag: the wait is bounded but not cut short)
+      volatile int own = 0;
       for (int s = 0; s < C::NS; ++s)
-        if (last_it[s] >= 0) mbar_wait(smem_u32(&bars.full[s]), (last_it[s] / C::NS) & 1, abort_flag);
+        if (last_it[s] >= 0 && !mbar_wait(smem_u32(&bars.full[s]), (last_it[s] / C::NS) & 1, &own)) *abort_flag = 1;
     }
     __syncwarp();
   } else if (warp == kMmaWarp) {
-    // ---------------------------------------------------------------- score MMAs
-    // Converged warp; one elected lane issues.  Tile j's scores go out as soon
-    // as its gated page is ready and the softmax warps have read the score
-    // buffer two tiles back.  Loops are unrolled with compile-time accumulate
-    // flags.  This warp also loads the sequences' query blocks (double-
-    // buffered): the next segment's block as soon as its buffer is free (a
-    // non-blocking test after every tile), blocking only at a segment start.
+    // ---------------------------------------------------------------- score MMAs, query blocks
+    // Converged warp; one elected lane issues.  The warp polls two queues and
+    // serves whichever is ready, so that neither waits for the other's
+    // condition:
+    //   query block of segment qn: its buffer's previous segment is done
+    //     (last score MMA complete, sums read by the softmax warps);
+    //   scores of tile js: its gated page (zready), a free score buffer (the
+    //     softmax warps read tile js - kNB's), and at a segment start the
+    //     segment's query block.
+    // Loops are unrolled with compile-time accumulate flags.
     if (!DUMP) {
-      constexpr uint32_t IDESC_S = idesc_bf16(64, kPage, 0, 0);
-      Walker w;
-      w.start(p.cu, p.seq_lens, p.batch);
-      int seg = -1;
-      Tracer tr;
-      tr.init(p, 1);
-      if (lane != 0) tr.base = nullptr;
-      // A operand: the query block in 8x8 core matrices, K groups 512 B apart,
-      // row groups 128 B apart (heads 0-7 -> rows 0-7, heads 8-15 -> rows
-      // 16-23).  B operand: the page slot, 128-byte swizzled, read K-major
-      // (tokens x features).
-      const uint64_t qdesc0 = smem_desc(sbase + C::OFF_QBUF, kQGroupBytes, 128, kSwizzleNone);
+      constexpr uint32_t IDESC_S = idesc_bf16(64, kHeads, 0, 0);
+      // A operand: the page slot, 128-byte swizzled, K-major (tokens x
+      // features); B: the query block in 8x8 core matrices, K cores 256 B
+      // apart, head halves 128 B apart
       const uint64_t zdesc_k = smem_desc(sbase, 16, 1024, kSwizzle128B);
-      // segment starts ahead of the tile loop: wq sits on the first tile of
-      // segment qn, the next one whose query block is to be loaded
-      Walker wq;
-      wq.start(p.cu, p.seq_lens, p.batch);
-      Tile tq;
-      bool q_more = wq.next(tq);
-      int qn = 0;
+      const uint64_t qdesc0 = smem_desc(sbase + C::OFF_QBUF, kQGroupBytes, kQRowGroupBytes, kSwizzleNone);
+      Walker ws, wq;
+      ws.start(p);
+      wq.start(p);
+      Tile ts, tq;
+      bool s_more = ws.next(ts), q_more = wq.next(tq);
+      int js = 0, qn = 0, seg_s = -1;
       int last_q[2] = {-1, -1};
-      // 1: issued, 0: buffer still in use (non-blocking call), -1: timed out
-      auto load_query = [&](bool block) -> int {
-        const int qb = qn & 1;
-        if (qn >= 2) {
-          const uint32_t qe = smem_u32(&bars.qempty[qb]);
-          const uint32_t par = ((qn >> 1) & 1) ^ 1;
-          if (block) {
-            if (!warp_wait(qe, par, abort_flag)) return -1;
-          } else if (!__all_sync(0xffffffffu, mbar_test_now(qe, par))) {
-            return 0;
-          }
-        }
-        if (lane == 0) {
-          mbar_arrive_expect_tx(smem_u32(&bars.qfull[qb]), C::QPREP);
-          bulk_load(sbase + C::OFF_QBUF + qb * C::QBUF, p.qprep + static_cast<size_t>(tq.b) * C::QPREP, C::QPREP,
-                    smem_u32(&bars.qfull[qb]));
-        }
-        __syncwarp();
-        last_q[qb] = qn;
-        ++qn;
-        do {
-          q_more = wq.next(tq);
-        } while (q_more && !tq.first);
-        return 1;
-      };
-      Tile t;
-      int j = 0;
       bool issued = false;
-      bool ok_q = true;
-      while (w.next(t)) {
-        if (t.first) {
-          ++seg;
-          while (qn <= seg && (ok_q = load_query(true) > 0)) {
+      Tracer tr;
+      tr.init(p, 1, 0, 2);
+      if (lane != 0) tr.base = nullptr;
+      uint64_t idle_since = 0;
+      while (s_more) {
+        bool progress = false;
+        // ---- query block of the next segment
+        if (q_more && warp_test(smem_u32(&bars.qempty[qn % C::NQ]), ((qn / C::NQ) & 1) ^ 1)) {
+          const int qb = qn % C::NQ;
+          if (lane == 0) {
+            mbar_arrive_expect_tx(smem_u32(&bars.qfull[qb]), C::QPREP);
+            bulk_load(sbase + C::OFF_QBUF + qb * C::QBUF, p.qprep + static_cast<size_t>(tq.b) * C::QPREP, C::QPREP,
+                      smem_u32(&bars.qfull[qb]));
           }
-          if (!ok_q) break;
-          if (!warp_wait(smem_u32(&bars.qfull[seg & 1]), (seg >> 1) & 1, abort_flag)) break;
+          __syncwarp();
+          last_q[qb] = qn;
+          ++qn;
+          do {
+            q_more = wq.next(tq);
+          } while (q_more && !tq.first);
+          progress = true;
         }
-        const int slot = j % C::NS;
-        tr.mark(0, j);
-        if (!warp_wait(smem_u32(&bars.zready[slot]), (j / C::NS) & 1, abort_flag)) break;
-        if (j >= 2 && !warp_wait(smem_u32(&bars.sfree[j & 1]), ((j >> 1) & 1) ^ 1, abort_flag)) break;
-        tr.mark(1, j);
-        if (lane == 0) mbar_arrive(smem_u32(&bars.s_ready[j & 1]));
-        tc_fence_after();
-        if (elect_one()) {
-          const uint64_t zb = zdesc_k + ((slot * C::SLOT) >> 4);
-          const uint64_t qa = qdesc0 + (((seg & 1) * C::QBUF) >> 4);
-          const uint32_t ds = tmem + C::COL_S + (j & 1) * C::S_COLS;
+        // ---- scores of tile js
+        const int slot = js % C::NS, sb = js % kNB;
+        const int sg = seg_s + (ts.first ? 1 : 0);
+        bool ready = !ts.first || (qn > sg && warp_test(smem_u32(&bars.qfull[sg % C::NQ]), (sg / C::NQ) & 1));
+        ready = ready && warp_test(smem_u32(&bars.zready[slot]), (js / C::NS) & 1);
+        ready = ready && warp_test(smem_u32(&bars.sfree[sb]), ((js / kNB) & 1) ^ 1);
+        if (ready) {
+          seg_s = sg;
+          tr.mark(1, js);
+          if (lane == 0) mbar_arrive(smem_u32(&bars.sready[sb]));
+          tc_fence_after();
+          if (elect_one()) {
+            const uint64_t za = zdesc_k + ((slot * C::SLOT) >> 4);
+            const uint64_t qb = qdesc0 + (((seg_s % C::NQ) * C::QBUF) >> 4);
+            const uint32_t ds = tmem + C::COL_S + sb * C::S_COLS;
 #pragma unroll
-          for (int kk = 0; kk < D_C / 16; ++kk)
-            mma_bf16_ss(ds, qa + ((kk * KSTEP) >> 4), zb + (((kk >> 2) * C::PCHUNK + (kk & 3) * 32) >> 4), IDESC_S,
-                        kk > 0);
+            for (int kk = 0; kk < D_C / 16; ++kk)
+              mma_bf16_ss(ds, za + (((kk >> 2) * C::PCHUNK + (kk & 3) * 32) >> 4),
+                          qb + ((kk * 2 * kQGroupBytes) >> 4), IDESC_S, kk > 0);
 #pragma unroll
-          for (int kk = 0; kk < kRope / 16; ++kk)
-            mma_bf16_ss(ds + kPage, qa + ((C::QB_LAT + kk * KSTEP) >> 4), zb + ((C::KR_OFF + kk * 32) >> 4), IDESC_S,
-                        kk > 0);
-          mma_commit(smem_u32(&bars.s_ready[j & 1]));
-          if (t.last) mma_commit(smem_u32(&bars.qempty[seg & 1]));
+            for (int kk = 0; kk < kRope / 16; ++kk)
+              mma_bf16_ss(ds + kHeads, za + ((C::KR_OFF + kk * 32) >> 4),
+                          qb + ((C::QB_LAT + kk * 2 * kQGroupBytes) >> 4), IDESC_S, kk > 0);
+            mma_commit(smem_u32(&bars.sready[sb]));
+            if (ts.last) mma_commit(smem_u32(&bars.qempty[seg_s % C::NQ]));
+          }
+          __syncwarp();
+          tr.mark(2, js);
+          issued = true;
+          ++js;
+          s_more = ws.next(ts);
+          progress = true;
         }
-        __syncwarp();
-        tr.mark(2, j);
-        issued = true;
-        ++j;
-        if (q_more && qn == seg + 1 && load_query(false) < 0) break;
+        if (progress) {
+          idle_since = 0;
+        } else {
+          // nothing ready: bounded wait for the others (and their abort)
+          const uint64_t now = globaltimer();
+          if (idle_since == 0) idle_since = now;
+          bool stop = *abort_flag != 0;
+          if (!stop && now - idle_since > kWaitLimitNs) {
+            *abort_flag = 1;
+            stop = true;
+          }
+          if (__any_sync(0xffffffffu, stop)) break;
+          __nanosleep(32);   // leave the issue slots to the warps that do the work
+        }
       }
       if (lane == 0) {
-        // drain: the query-block copies this warp issued must land before the CTA exits
+        // drain: the query-block copies this warp issued must land, and every
+        // MMA must finish, before the CTA exits and TMEM is released (own flag:
+        // bounded but not cut short by an abort)
+        volatile int own = 0;
         for (int b = 0; b < 2; ++b)
-          if (last_q[b] >= 0) mbar_wait(smem_u32(&bars.qfull[b]), (last_q[b] >> 1) & 1, abort_flag);
+          if (last_q[b] >= 0 && !mbar_wait(smem_u32(&bars.qfull[b]), (last_q[b] / C::NQ) & 1, &own)) *abort_flag = 1;
       }
       __syncwarp();
       if (issued) {
-        // every score MMA must finish before TMEM is released
         if (elect_one()) mma_commit(smem_u32(&bars.drain_s));
         __syncwarp();
-        mbar_wait(smem_u32(&bars.drain_s), 0, abort_flag);
+        volatile int own = 0;
+        if (!mbar_wait(smem_u32(&bars.drain_s), 0, &own)) *abort_flag = 1;
+      }
+    }
+    __syncwarp();
+  } else if (warp == kOutWarp) {
+    // ---------------------------------------------------------------- output MMAs
+    // O^T[feature, head] += Z^T P' for each tile in order, as soon as the
+    // softmax warps wrote its P'; completion frees the page slot and the P'
+    // buffer.  A operand: the page slot read MN-major (features along M,
+    // 64-feature atoms PCHUNK apart; tokens along K, 8-row groups 1 KB apart);
+    // B: P' MN-major in 8x8 core matrices (token groups 256 B, head halves
+    // 128 B).
+    if (!DUMP) {
+      constexpr uint32_t IDESC_O = idesc_bf16(128, kHeads, 1, 1);
+      const uint64_t zdesc_mn = smem_desc(sbase, C::PCHUNK, 1024, kSwizzle128B);
+      const uint64_t pdesc0 = smem_desc(sbase + C::OFF_PBUF, 256, 128, kSwizzleNone);
+      Walker wo;
+      wo.start(p);
+      Tile to;
+      int jo = 0;
+      bool issued = false;
+      Tracer tr;
+      tr.init(p, 1, 1, 2);   // second half of the MMA role's run
+      if (lane != 0) tr.base = nullptr;
+      while (wo.next(to)) {
+        if (!warp_wait(smem_u32(&bars.spdone[jo % kNP]), (jo / kNP) & 1, abort_flag)) break;
+        tr.mark(3, jo);
+        tc_fence_after();
+        if (elect_one()) {
+          const int slot = jo % C::NS;
+          const uint64_t za = zdesc_mn + ((slot * C::SLOT) >> 4);
+          const uint64_t pb = pdesc0 + (((jo % kNP) * C::PBUF) >> 4);
+          if (to.first) {
+#pragma unroll
+            for (int ks = 0; ks < kPage / 16; ++ks)
+#pragma unroll
+              for (int mc = 0; mc < 2; ++mc)
+                mma_bf16_ss(tmem + C::COL_O + kHeads * mc, za + (((C::mc_start(mc) / 64) * C::PCHUNK + ks * 2048) >> 4),
+                            pb + ((ks * 512) >> 4), IDESC_O, ks > 0);
+          } else {
+#pragma unroll
+            for (int ks = 0; ks < kPage / 16; ++ks)
+#pragma unroll
+              for (int mc = 0; mc < 2; ++mc)
+                mma_bf16_ss(tmem + C::COL_O + kHeads * mc, za + (((C::mc_start(mc) / 64) * C::PCHUNK + ks * 2048) >> 4),
+                            pb + ((ks * 512) >> 4), IDESC_O, 1);
+          }
+          mma_commit(smem_u32(&bars.empty[slot]));
+          mma_commit(smem_u32(&bars.pfree[jo % kNP]));
+        }
+        __syncwarp();
+        tr.mark(4, jo);
+        issued = true;
+        ++jo;
+      }
+      if (issued) {
+        if (elect_one()) mma_commit(smem_u32(&bars.drain_o));
+        __syncwarp();
+        volatile int own = 0;
+        if (!mbar_wait(smem_u32(&bars.drain_o), 0, &own)) *abort_flag = 1;
       }
     }
     __syncwarp();
   } else if (warp >= kGateWarp0) {
     // ---------------------------------------------------------------- gate: z = c (*) g, LN statistics
-    // Quarter-warp k = 4 (warp - 4) + lane / 8 owns token rows 2k (lanes 0-3)
+    // Quarter-warp k = 4 (warp - 7) + lane / 8 owns token rows 2k (lanes 0-3)
     // and 2k + 1 (lanes 4-7); lane p = lane % 4 of a row takes the 16-byte
     // units 2p and 2p + 1 of every 64-feature column.  The gate-row load of a
     // column is then one 32-byte load per lane and a whole 128-byte line per
@@ -813,8 +935,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint64_t pol_keep = policy_evict_last();
     constexpr bool gate_ln = GATE_LN;
     Walker w;
-    w.start(p.cu, p.seq_lens, p.batch);
+    w.start(p);
     PageWindow pw;
+    pw.init(p, lane);
     // id of this thread's row of a tile (0 past the end of the page or for a
     // bad page, which the producer reports)
     auto load_id = [&](const Tile& tt) -> int {
@@ -944,9 +1067,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tr.mark(6, j);
             if (pp == 0) {
-              st[row] = 0.f;   // the stored z is centred
-              st[kPage + row] = valid ? r : 0.f;
-              st[2 * kPage + row] = valid ? 1.f / r : 0.f;
+              // the stored z is centred; rows past the page end get r = 1 (their
+              // weight is 0, and l adds 0 / r)
+              st[row] = 0.f;
+              st[kPage + row] = valid ? r : 1.f;
             }
           } else {
             float2 s1 = make_float2(0.f, 0.f), s2 = make_float2(0.f, 0.f);
@@ -992,9 +1116,9 @@ __global__ void __launch_bounds__(kThreads, 1)
               const float mu = gate_ln ? sum1 * inv_dc : 0.f;
               const float var = fmaxf(sum2 * inv_dc - mu * mu, 0.f);
               const float r = gate_ln ? rsqrtf(var + p.eps) : 1.f;
+              // rows past the page end: mu = 0, r = 1 (their weight is 0, and l adds 0 / r)
               st[row] = valid ? mu : 0.f;
-              st[kPage + row] = valid ? r : 0.f;
-              st[2 * kPage + row] = valid ? 1.f / r : 0.f;
+              st[kPage + row] = valid ? r : 1.f;
             }
           }
         } else if (!full_page) {
@@ -1029,224 +1153,293 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp < kSoftWarps && !DUMP) {
     // ---------------------------------------------------------------- softmax, output read-out
-    // Warp hw owns heads 8hw..8hw+7, whose rows of S^T and O sit in TMEM lanes
-    // 32hw..32hw+7.  Thread t owns head hd = 8hw + t/4 and, in every 8-token
-    // group k of a page, the tokens 8k + 2(t%4) and 8k + 2(t%4) + 1.  The
-    // 16-lane TMEM loads also return lanes 32hw+8..32hw+15 (rows no head uses),
-    // which are ignored.
-    const int hw = warp, hd = 8 * hw + (lane >> 2), qq = lane & 3;
-    const uint32_t tq = tmem + (static_cast<uint32_t>(32 * hw) << 16);
+    // Warp w reads TMEM lane quadrant w: tokens 16w .. 16w + 15 of a tile's
+    // scores (rows of the M = 64 accumulator) and latent features 32w .. 32w +
+    // 31 of each 128-feature chunk of O^T.  Thread t owns tokens r0 = 16w + t/4
+    // and r1 = r0 + 8 and heads hh(k) = 2q, 2q + 1, 8 + 2q, 9 + 2q (q = t % 4).
+    // Lane h < 16 of every warp also keeps head h's reference max (the same in
+    // all four warps), which the rare slow path of the max update uses.
+    const int q = lane & 3;
+    const int r0 = 16 * warp + (lane >> 2), r1 = r0 + 8;
+    const uint32_t tq = tmem + (static_cast<uint32_t>(32 * warp) << 16);
     const float scale = p.scale_log2;
-    // Online softmax with a lazily updated reference max m_ref per head: the
-    // exponentials are taken against m_ref, which only moves (rescaling the TMEM
-    // accumulator, l and the mean correction) when a tile's max exceeds it by
-    // more than 2^kLazyLog2; otherwise the weights stay below 2^kLazyLog2.
-    float m_ref = 0.f, l_acc = 0.f, bmu_acc = 0.f, wq = 0.f, bsc = 0.f;
-    // this warp's copy of gamma and beta (identity without a LayerNorm), so that
-    // the segment read-out waits on no global load
-    float* gb = reinterpret_cast<float*>(smem + C::OFF_GB + hw * C::GB_BYTES);
+    float* xmax = reinterpret_cast<float*>(smem + C::OFF_XCH);        // [4 warps][16 heads]
+    float* xsum = xmax + kSoftWarps * kHeads;                         // [4 warps][16 heads][2]
+    auto head_of = [&](int k) { return (k & 1) + 2 * q + 8 * (k >> 1); };
+    // gamma and beta of the segment read-out in shared memory (written once by
+    // the four warps; the first tile's barrier orders the writes before any read)
+    float* gb = reinterpret_cast<float*>(smem + C::OFF_GB);
     if (GATE) {
-      for (int f = lane; f < D_C; f += 32) {
+      for (int f = threadIdx.x; f < D_C; f += kSoftThreads) {
         gb[f] = p.gamma ? __ldg(p.gamma + f) : 1.f;
         gb[D_C + f] = p.beta ? __ldg(p.beta + f) : 0.f;
       }
-      __syncwarp();
+    }
+    float m_ref[4], l_acc[4], bmu_acc[4], wq[4], bsc[4];
+    float m16 = -INFINITY;   // head `lane` (lanes 0-15)
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      m_ref[k] = -INFINITY;
+      l_acc[k] = 0.f;
+      bmu_acc[k] = 0.f;
+      wq[k] = 0.f;
+      bsc[k] = 0.f;
     }
     Walker w;
-    w.start(p.cu, p.seq_lens, p.batch);
+    w.start(p);
     Tile t;
     int it = 0, seg = -1;
     Tracer tr;
     tr.init(p, 3);
     if (threadIdx.x != 0) tr.base = nullptr;
     while (w.next(t)) {
+      bool ok = true;
       if (t.first) {
         ++seg;
-        if (!warp_wait(smem_u32(&bars.qfull[seg & 1]), (seg >> 1) & 1, abort_flag)) break;
-        if (GATE) {
+        ok = warp_wait(smem_u32(&bars.qfull[seg % C::NQ]), (seg / C::NQ) & 1, abort_flag);
+        if (ok && GATE) {
           // w_h = sum_f bf16(q^ gamma)_hf and b_h = q^_h . beta from their
           // per-chunk partials after the operands, added in chunk order
-          const float* sums = reinterpret_cast<const float*>(smem + C::OFF_QBUF + (seg & 1) * C::QBUF + C::QB_LAT +
-                                                             C::QB_ROPE);
-          float wsum = 0.f, bsum = 0.f;
+          const float* sums = reinterpret_cast<const float*>(smem + C::OFF_QBUF + (seg % C::NQ) * C::QBUF +
+                                                             C::QB_LAT + qprep_rope_bytes(kRope));
 #pragma unroll
-          for (int c = 0; c < D_C / kSumFeatures; ++c) {
-            wsum += sums[c * 32 + hd];
-            bsum += sums[c * 32 + 16 + hd];
+          for (int k = 0; k < 4; ++k) {
+            const int h = head_of(k);
+            float wsum = 0.f, bsum = 0.f;
+#pragma unroll
+            for (int c = 0; c < D_C / kSumFeatures; ++c) {
+              wsum += sums[c * 32 + h];
+              bsum += sums[c * 32 + 16 + h];
+            }
+            wq[k] = wsum;
+            bsc[k] = bsum * scale;
           }
-          wq = wsum;
-          bsc = bsum * scale;
         }
-        warp_arrive(smem_u32(&bars.qempty[seg & 1]));
-        l_acc = 0.f;
-        bmu_acc = 0.f;
+        if (ok) warp_arrive(smem_u32(&bars.qempty[seg % C::NQ]));
       }
-      const int slot = it % C::NS;
-      const int par = it & 1;
+      const int slot = it % C::NS, sb = it % kNB, pb = it % kNP;
       tr.mark(0, it);
-      // Scores of this tile; the score warp's release arrival on the same
-      // barrier orders the gate's statistics before it.
-      if (!warp_wait(smem_u32(&bars.s_ready[par]), (it >> 1) & 1, abort_flag)) break;
+      // scores of this tile; the MMA warp's release arrival on the same barrier
+      // orders the gate's statistics before them
+      ok = ok && warp_wait(smem_u32(&bars.sready[sb]), (it / kNB) & 1, abort_flag);
       tr.mark(1, it);
-      tc_fence_after();
-      float sl[32], sr[32];
-      tmem_ld_16x256b_x8(tq + C::COL_S + par * C::S_COLS, sl);
-      tmem_ld_16x256b_x8(tq + C::COL_S + par * C::S_COLS + kPage, sr);
-      const float* st = reinterpret_cast<const float*>(smem + C::OFF_STAT + slot * C::STAT_BYTES);
-      float2 mu2[8], r2[8], ri2[8];
-      if (GATE) {
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-          mu2[k] = *reinterpret_cast<const float2*>(st + 8 * k + 2 * qq);
-          r2[k] = *reinterpret_cast<const float2*>(st + kPage + 8 * k + 2 * qq);
-          ri2[k] = *reinterpret_cast<const float2*>(st + 2 * kPage + 8 * k + 2 * qq);
+      float s[2][4];
+      float mu[2] = {0.f, 0.f}, rr[2] = {1.f, 1.f};
+      bool exceed = false;
+      if (ok) {
+        tc_fence_after();
+        float v[16];
+        tmem_ld_16x256b_x4(tq + C::COL_S + sb * C::S_COLS, v);
+        if (GATE) {
+          const float* st = reinterpret_cast<const float*>(smem + C::OFF_STAT + slot * C::STAT_BYTES);
+          mu[0] = st[r0];
+          mu[1] = st[r1];
+          rr[0] = st[kPage + r0];
+          rr[1] = st[kPage + r1];
         }
-      }
-      tmem_wait_ld();
-      tc_fence_before();
-      warp_arrive(smem_u32(&bars.sfree[par]));   // score buffer read: tile it + 2 may overwrite it
-      tr.mark(7, it);
-      // s[2k + e]: token 8k + 2 qq + e of head hd (log2 units)
-      float s[16];
-      const bool full_page = t.ntok == kPage;
-#pragma unroll
-      for (int k = 0; k < 8; ++k) {
+        tmem_wait_ld();
+        tc_fence_before();
+        warp_arrive(smem_u32(&bars.sfree[sb]));   // score buffer read: tile it + kNB may overwrite it
+        tr.mark(7, it);
+        const bool full_page = t.ntok == kPage;
 #pragma unroll
         for (int e = 0; e < 2; ++e) {
-          const float lat = sl[4 * k + e], rope = sr[4 * k + e];
-          float v;
-          if (GATE) {
-            const float mu = e ? mu2[k].y : mu2[k].x;
-            const float rs = (e ? r2[k].y : r2[k].x) * scale;
-            v = fmaf(rs, fmaf(-mu, wq, lat), fmaf(rope, scale, bsc));
-          } else {
-            v = (lat + rope) * scale;
+          const bool valid = full_page || (e ? r1 : r0) < t.ntok;
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const float lat = v[(k >> 1) * 4 + 2 * e + (k & 1)];
+            const float rope = v[8 + (k >> 1) * 4 + 2 * e + (k & 1)];
+            float x;
+            if (GATE) {
+              x = fmaf(rr[e] * scale, fmaf(-mu[e], wq[k], lat), fmaf(rope, scale, bsc[k]));
+            } else {
+              x = (lat + rope) * scale;
+            }
+            s[e][k] = valid ? x : -INFINITY;
+            exceed = exceed || (x > m_ref[k] + kLazyLog2 && valid);
           }
-          const bool valid = full_page || (8 * k + 2 * qq + e) < t.ntok;
-          s[2 * k + e] = valid ? v : -INFINITY;
         }
       }
       tr.mark(8, it);
-      // tile max of the head: 16 tokens in-thread (a tree), then its four threads
-      float m8[8];
+      // one vote of the four warps: a head's reference max must move (or a
+      // wait failed somewhere)
+      if (soft_vote(kBarTile, exceed || !ok)) {
+        if (soft_vote(kBarTile, !ok)) break;   // uniform: every warp leaves
+        // ---- slow path: tile maxima of the heads over the 64 tokens
+        float tm[4];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) m8[i] = fmaxf(s[i], s[i + 8]);
+        for (int k = 0; k < 4; ++k) tm[k] = fmaxf(s[0][k], s[1][k]);
 #pragma unroll
-      for (int i = 0; i < 4; ++i) m8[i] = fmaxf(m8[i], m8[i + 4]);
-      float mx = fmaxf(fmaxf(m8[0], m8[2]), fmaxf(m8[1], m8[3]));
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-      float alpha = 1.f;
-      bool rescale = false;
-      if (t.first) {
-        m_ref = mx;
-      } else if (mx > m_ref + kLazyLog2) {
-        alpha = ex2_approx(m_ref - mx);
-        m_ref = mx;
-        rescale = true;
-      }
-      tr.mark(2, it);
-      if (__any_sync(0xffffffffu, rescale)) {
-        // The previous tile's output MMA must be complete before O is rescaled.
-        // Phase n of pfree[b] completes with output MMA 2n + b; the wait below
-        // on every tile keeps each buffer's phase count at most one behind, so
-        // the parity wait is exact.
-        if (!warp_wait(smem_u32(&bars.pfree[(it - 1) & 1]), ((it - 1) >> 1) & 1, abort_flag)) break;
-        tc_fence_after();
-#pragma unroll 1
-        for (int c = 0; c < D_C / 64; ++c) {
-          float o[32];
-          tmem_ld_16x256b_x8(tq + C::COL_O + 64 * c, o);
-          tmem_wait_ld();
+        for (int o = 4; o < 32; o <<= 1)
 #pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            o[4 * k] *= alpha;
-            o[4 * k + 1] *= alpha;
+          for (int k = 0; k < 4; ++k) tm[k] = fmaxf(tm[k], __shfl_xor_sync(0xffffffffu, tm[k], o));
+        if (lane < 4) {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) xmax[warp * kHeads + head_of(k)] = tm[k];
+        }
+        soft_sync(kBarXch);
+        // lane h < 16: the new reference of head h and the factor for what was
+        // accumulated against the old one (the same in every warp)
+        float alpha = 1.f;
+        if (lane < kHeads) {
+          const float tmax = fmaxf(fmaxf(xmax[lane], xmax[kHeads + lane]),
+                                   fmaxf(xmax[2 * kHeads + lane], xmax[3 * kHeads + lane]));
+          if (m16 == -INFINITY) {
+            m16 = tmax;
+            alpha = 0.f;
+          } else if (tmax > m16 + kLazyLog2) {
+            alpha = ex2_approx(m16 - tmax);
+            m16 = tmax;
           }
-          tmem_st_16x256b_x8(tq + C::COL_O + 64 * c, o);
         }
-        tmem_wait_st();
-        l_acc *= alpha;
-        bmu_acc *= alpha;
-      }
-      // the weight buffer of this parity is free once the output MMA two tiles
-      // back has read it
-      if (!warp_wait(smem_u32(&bars.pfree[par]), ((it >> 1) & 1) ^ 1, abort_flag)) break;
-      tr.mark(5, it);
-      // The output MMA sees the bf16-rounded weights P'; the denominator and the
-      // mean correction use the same rounded values (l = sum P'/r), so the
-      // rounding of P' cancels in o = (sum P' z - sum P' mu) / l.
-      uint8_t* pbuf = smem + C::OFF_PBUF + par * C::PBUF + qop_offset(hd, 2 * qq);
 #pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        const float r0 = GATE ? r2[k].x : 1.f, r1 = GATE ? r2[k].y : 1.f;
-        const float p0 = ex2_approx(s[2 * k] - m_ref) * r0;
-        const float p1 = ex2_approx(s[2 * k + 1] - m_ref) * r1;
-        const uint32_t pw = pack_bf16x2(p0, p1);
-        const float2 pq = unpack_bf16x2(pw);
-        if (GATE) {
-          l_acc = fmaf(pq.x, ri2[k].x, fmaf(pq.y, ri2[k].y, l_acc));
-          bmu_acc = fmaf(pq.x, mu2[k].x, fmaf(pq.y, mu2[k].y, bmu_acc));
-        } else {
-          l_acc += pq.x + pq.y;
+        for (int k = 0; k < 4; ++k) m_ref[k] = __shfl_sync(0xffffffffu, m16, head_of(k));
+        if (!t.first && __any_sync(0xffffffffu, lane < kHeads && alpha != 1.f)) {
+          // O^T and the running sums were accumulated against the old
+          // reference: the previous tile's output MMA must be complete first
+          // (completion n of pfree[b] is output MMA n kNP + b)
+          const int pv = (it - 1) % kNP;
+          ok = warp_wait(smem_u32(&bars.pfree[pv]), ((it - 1) / kNP) & 1, abort_flag);
+          if (ok) {
+            tc_fence_after();
+            float o[32];
+            tmem_ld32(tq + C::COL_O, o);
+            tmem_wait_ld();
+#pragma unroll
+            for (int c = 0; c < 32; ++c) o[c] *= __shfl_sync(0xffffffffu, alpha, c & 15);
+            tmem_st32(tq + C::COL_O, o);
+            tmem_wait_st();
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const float a = __shfl_sync(0xffffffffu, alpha, head_of(k));
+              l_acc[k] *= a;
+              bmu_acc[k] *= a;
+            }
+          }
         }
-        *reinterpret_cast<uint32_t*>(pbuf + k * kQGroupBytes) = pw;
       }
-      tr.mark(6, it);
-      fence_proxy_async_smem();
-      tc_fence_before();
-      warp_arrive(smem_u32(&bars.sp_done[par]));
+      // the P' buffer of this tile is free once the output MMA kNP tiles back
+      // has read it
+      ok = ok && warp_wait(smem_u32(&bars.pfree[pb]), ((it / kNP) & 1) ^ 1, abort_flag);
+      tr.mark(5, it);
+      if (ok) {
+        // The output MMA sees the bf16-rounded weights P'; the denominator and
+        // the mean correction use the same rounded values (l = sum P'/r), so
+        // the rounding of P' cancels in o = (sum P' z - sum P' mu) / l.
+        // P'[token][head] as an MN-major B operand: element (head n, token k)
+        // at (k / 8) 256 + (n / 8) 128 + (k % 8) 16 + (n % 8) 2.
+        uint8_t* pbuf = smem + C::OFF_PBUF + pb * C::PBUF;
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int r = e ? r1 : r0;
+          const float ri = GATE ? 1.f / rr[e] : 1.f;
+          float pq[4];
+#pragma unroll
+          for (int k = 0; k < 4; ++k) pq[k] = ex2_approx(s[e][k] - m_ref[k]) * rr[e];
+#pragma unroll
+          for (int hp = 0; hp < 2; ++hp) {
+            const uint32_t pw = pack_bf16x2(pq[2 * hp], pq[2 * hp + 1]);
+            const float2 pr = unpack_bf16x2(pw);
+            if (GATE) {
+              l_acc[2 * hp] = fmaf(pr.x, ri, l_acc[2 * hp]);
+              l_acc[2 * hp + 1] = fmaf(pr.y, ri, l_acc[2 * hp + 1]);
+              bmu_acc[2 * hp] = fmaf(pr.x, mu[e], bmu_acc[2 * hp]);
+              bmu_acc[2 * hp + 1] = fmaf(pr.y, mu[e], bmu_acc[2 * hp + 1]);
+            } else {
+              l_acc[2 * hp] += pr.x;
+              l_acc[2 * hp + 1] += pr.y;
+            }
+            *reinterpret_cast<uint32_t*>(pbuf + (r >> 3) * 256 + hp * 128 + (r & 7) * 16 + 4 * q) = pw;
+          }
+        }
+        tr.mark(6, it);
+        fence_proxy_async_smem();
+        tc_fence_before();
+        warp_arrive(smem_u32(&bars.spdone[pb]));
+      }
       tr.mark(3, it);
 
       if (t.last) {
-        // ---- segment end: l and sum_j P'_j mu_j over the four threads of the head
-        float lh = l_acc, bh = bmu_acc;
-        lh += __shfl_xor_sync(0xffffffffu, lh, 1);
-        bh += __shfl_xor_sync(0xffffffffu, bh, 1);
-        lh += __shfl_xor_sync(0xffffffffu, lh, 2);
-        bh += __shfl_xor_sync(0xffffffffu, bh, 2);
-        // the segment's last output MMA (the earlier ones complete before it;
-        // exact parity wait as for the rescale), then the accumulated output
-        if (!warp_wait(smem_u32(&bars.pfree[par]), (it >> 1) & 1, abort_flag)) break;
-        tc_fence_after();
-        const int slot_out = blockIdx.x + t.b;
-        float* po = p.part_o + (static_cast<size_t>(slot_out) * kHeads + hd) * D_C;
-#pragma unroll 1
-        for (int c = 0; c < D_C / 64; ++c) {
-          float o[32];
-          tmem_ld_16x256b_x8(tq + C::COL_O + 64 * c, o);
-          tmem_wait_ld();
+        // ---- segment end: l and sum_j P'_j mu_j of every head over the 64 token rows
 #pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            const int f = 64 * c + 8 * k + 2 * qq;
-            float2 v = make_float2(o[4 * k], o[4 * k + 1]);
-            if (GATE) {
-              const float2 gm = *reinterpret_cast<const float2*>(gb + f);
-              const float2 bt = *reinterpret_cast<const float2*>(gb + D_C + f);
-              v.x = fmaf(gm.x, v.x - bh, bt.x * lh);
-              v.y = fmaf(gm.y, v.y - bh, bt.y * lh);
+        for (int o = 4; o < 32; o <<= 1)
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            l_acc[k] += __shfl_xor_sync(0xffffffffu, l_acc[k], o);
+            bmu_acc[k] += __shfl_xor_sync(0xffffffffu, bmu_acc[k], o);
+          }
+        if (lane < 4) {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            xsum[(warp * kHeads + head_of(k)) * 2] = l_acc[k];
+            xsum[(warp * kHeads + head_of(k)) * 2 + 1] = bmu_acc[k];
+          }
+        }
+        if (soft_vote(kBarXch, !ok)) break;   // uniform
+        float lh = 0.f, bh = 0.f;   // head `lane` (lanes 0-15)
+        if (lane < kHeads) {
+#pragma unroll
+          for (int ww = 0; ww < kSoftWarps; ++ww) {
+            lh += xsum[(ww * kHeads + lane) * 2];
+            bh += xsum[(ww * kHeads + lane) * 2 + 1];
+          }
+        }
+        // the segment's last output MMA (the earlier ones complete before it;
+        // completion n of pfree[b] is output MMA n kNP + b), then O^T
+        ok = warp_wait(smem_u32(&bars.pfree[pb]), (it / kNP) & 1, abort_flag);
+        if (ok) {
+          tc_fence_after();
+          float o[32];
+          tmem_ld32(tq + C::COL_O, o);
+          tmem_wait_ld();
+          const int slot_out = blockIdx.x + t.b;
+          float* po = p.part_o + static_cast<size_t>(slot_out) * kHeads * D_C;
+#pragma unroll
+          for (int mc = 0; mc < 2; ++mc) {
+            const int f = C::mc_start(mc) + 32 * warp + lane;
+            if (mc == 0 || C::mc_start(1) + 32 * warp >= 128) {   // uniform in the warp
+              float gm = 1.f, bt = 0.f;
+              if (GATE) {
+                gm = gb[f];
+                bt = gb[D_C + f];
+              }
+#pragma unroll
+              for (int h = 0; h < kHeads; ++h) {
+                float v = o[mc * kHeads + h];
+                if (GATE) {
+                  const float lhh = __shfl_sync(0xffffffffu, lh, h), bhh = __shfl_sync(0xffffffffu, bh, h);
+                  v = fmaf(gm, v - bhh, bt * lhh);
+                }
+                po[h * D_C + f] = v;
+              }
             }
-            *reinterpret_cast<float2*>(po + f) = v;
+          }
+          tc_fence_before();
+          if (warp == 0 && lane < kHeads) {
+            float* ml = p.part_ml + (static_cast<size_t>(slot_out) * kHeads + lane) * 2;
+            ml[0] = m16;
+            ml[1] = lh;
+          }
+          if (p.fuse && p.cmb_g == 1) {
+            // one sequence per combine unit: release this warp's part of the
+            // partial to the wait on its sequence (the warp barrier orders every
+            // lane's stores before lane 0's fence)
+            __syncwarp();
+            if (lane == 0) {
+              __threadfence();
+              atomicAdd(p.seq_done + 1 + t.b, 1u);
+            }
           }
         }
-        tc_fence_before();
-        if (qq == 0) {
-          float* ml = p.part_ml + (static_cast<size_t>(slot_out) * kHeads + hd) * 2;
-          ml[0] = m_ref;
-          ml[1] = lh;
-        }
-        if (p.fuse && p.cmb_g == 1) {
-          // one sequence per combine unit: release this warp's half of the
-          // partial to the wait on its sequence (the warp barrier orders every
-          // lane's stores before lane 0's fence)
-          __syncwarp();
-          if (lane == 0) {
-            __threadfence();
-            atomicAdd(p.seq_done + 1 + t.b, 1u);
-          }
-        }
-
         tr.mark(4, it);
+        // the next segment starts from scratch
+        m16 = -INFINITY;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          m_ref[k] = -INFINITY;
+          l_acc[k] = 0.f;
+          bmu_acc[k] = 0.f;
+        }
       }
       ++it;
     }
@@ -1296,6 +1489,7 @@ cudaError_t launch_one(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_
 
   p.qprep = ws + wl.off_qprep;
   p.cu = reinterpret_cast<const int32_t*>(ws + wl.off_cu);
+  p.starts = reinterpret_cast<const SplitStart*>(ws + wl.off_start);
   p.part_ml = reinterpret_cast<float*>(ws + wl.off_ml);
   p.part_o = reinterpret_cast<float*>(ws + wl.off_o);
   p.status = a.status;

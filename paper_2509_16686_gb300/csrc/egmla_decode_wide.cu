@@ -352,8 +352,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       w.start(p.cu, p.seq_lens, p.batch);
       uint32_t last_bar = 0, last_par = 0;
       int seg = -1;
-      // the query block as an N = 16 B operand: K groups 512 B apart, head halves 256 B apart
-      const uint64_t qdesc0 = smem_desc(sbase + C::OFF_QBUF, kQGroupBytes, 256, kSwizzleNone);
+      // the query block as an N = 16 B operand: K cores 256 B apart, head halves 128 B apart
+      const uint64_t qdesc0 = smem_desc(sbase + C::OFF_QBUF, kQGroupBytes, kQRowGroupBytes, kSwizzleNone);
       const uint64_t zdesc_k = smem_desc(sbase, 16, 1024, kSwizzle128B);         // K-major view of a slot
       const uint64_t zdesc_mn = smem_desc(sbase, C::PCHUNK, 1024, kSwizzle128B);  // MN-major view of a slot
       const uint64_t pdesc = smem_desc(sbase + C::OFF_PBUF, 256, 128, kSwizzleNone);
