@@ -284,6 +284,17 @@ size_t eg_mla_layer_workspace_size(const eg_mla_dims* dims, const eg_mla_layer_d
                                    int32_t batch, int32_t num_splits);
 
 /*
+ * eg_mla_layer_attn_offset - byte offset, within the workspace of an
+ * eg_mla_layer_decode call with these arguments, of the step's attention
+ * output u [batch, num_heads, d_v] (bf16, Eq. 13), which the call leaves there
+ * after it completes (the input of the output projection, Eq. 14): a testing
+ * and debugging aid.  Returns 0 on invalid arguments (a valid offset is never
+ * 0: the cuBLAS workspace comes first).
+ */
+size_t eg_mla_layer_attn_offset(const eg_mla_dims* dims, const eg_mla_layer_dims* layer, int32_t batch,
+                                int32_t num_splits);
+
+/*
  * eg_mla_layer_decode - the step above for `batch` sequences, on `stream`.
  *
  *   x          [batch, E] bf16 hidden states of the new tokens
@@ -368,12 +379,29 @@ int eg_mla_profile_end(double* ms_sum, int32_t* launches);
  * 1 MMA issuers: the score issuer in the first half of the run, the output
  * issuer in the second, 2 gate, 3 softmax, 4 at d_c 192/256 the kernel phases:
  * entry, set-up done, tile loops done, split combine done), a run of (tag, SM clock) pairs of 8-byte
- * words, tag = event << 56 | tile index << 32 | low 32 bits of the global
- * nanosecond timer; run r of CTA c starts at word (c * 5 + r) * cap * 2 with
- * cap = bytes / (ctas * 5 * 16).  The caller zeroes
+ * words, tag = event << 56 | tile index << 32, whose low 32 bits hold, in the
+ * kernel phases only, the low 32 bits of the global nanosecond timer (which
+ * maps each CTA's clock to time); run r of CTA c starts at word
+ * (c * 5 + r) * cap * 2 with cap = bytes / (ctas * 5 * 16).  The caller zeroes
  * the buffer; unused entries stay zero.  NULL or bytes <= 0 turns tracing off.
  */
 int eg_mla_debug_set_trace(void* dev_buf, int64_t bytes, int32_t ctas);
+
+/*
+ * eg_mla_debug_set_fault - test entry for the failure path of the split-KV
+ * decode kernel (d_c 192 and 256, bf16).  With cta >= 0, later eg_mla_decode
+ * calls withhold one page copy: CTA `cta` skips the copy of its tile `tile`
+ * (0-based in its walk) and its arrival, and every pipeline wait of those
+ * launches gives up after wait_limit_ns (1 us .. 2 s) instead of the default
+ * 2 s.  The wait on the withheld page then runs out: the kernel records
+ * EG_MLA_ERR_TIMEOUT in *dev_status, every role leaves its loop, the copies
+ * and MMAs already issued are waited for, TMEM is freed and the kernel
+ * returns; the rest of the grid reports the same status when its split merge
+ * waits for the missing partial.  No fault, trap or hang is involved, and the
+ * device stays usable.  cta < 0 restores normal operation.  Returns
+ * EG_MLA_ERR_INVALID_ARG for a negative tile or a limit out of range.
+ */
+int eg_mla_debug_set_fault(int32_t cta, int32_t tile, int64_t wait_limit_ns);
 
 #ifdef __cplusplus
 }

@@ -48,7 +48,9 @@ EXPORTED = [
     "eg_mla_profile_begin",
     "eg_mla_profile_end",
     "eg_mla_debug_set_trace",
+    "eg_mla_debug_set_fault",
     "eg_mla_layer_workspace_size",
+    "eg_mla_layer_attn_offset",
     "eg_mla_layer_decode",
 ]
 
@@ -104,9 +106,13 @@ def _declare(lib: ctypes.CDLL) -> None:
     lib.eg_mla_profile_end.restype = ctypes.c_int
     lib.eg_mla_debug_set_trace.argtypes = [P, ctypes.c_int64, I32]
     lib.eg_mla_debug_set_trace.restype = ctypes.c_int
+    lib.eg_mla_debug_set_fault.argtypes = [I32, I32, ctypes.c_int64]
+    lib.eg_mla_debug_set_fault.restype = ctypes.c_int
     LD, LW = ctypes.POINTER(EgMlaLayerDims), ctypes.POINTER(EgMlaLayerWeights)
     lib.eg_mla_layer_workspace_size.argtypes = [D, LD, I32, I32]
     lib.eg_mla_layer_workspace_size.restype = SZ
+    lib.eg_mla_layer_attn_offset.argtypes = [D, LD, I32, I32]
+    lib.eg_mla_layer_attn_offset.restype = SZ
     lib.eg_mla_layer_decode.argtypes = [D, LD, LW, P, P, P, P, P, P, P, I32, P, I32, I32, I32, P, I32, P, SZ, P, P]
     lib.eg_mla_layer_decode.restype = ctypes.c_int
 
@@ -249,6 +255,13 @@ def eg_mla_layer_workspace_size(dims: EgMlaDims, layer: EgMlaLayerDims, batch: i
     return int(n)
 
 
+def eg_mla_layer_attn_offset(dims: EgMlaDims, layer: EgMlaLayerDims, batch: int, num_splits: int = 0) -> int:
+    n = load().eg_mla_layer_attn_offset(ctypes.byref(dims), ctypes.byref(layer), batch, num_splits)
+    if n == 0:
+        raise EgMlaError(EG_MLA_ERR_UNSUPPORTED, "eg_mla_layer_attn_offset")
+    return int(n)
+
+
 def eg_mla_layer_decode(dims: EgMlaDims, layer: EgMlaLayerDims, weights: EgMlaLayerWeights, x, ids_new, positions,
                         c_pool, krope_pool, id_pool, block_table, seq_lens, max_seq_len, y, workspace,
                         num_splits=0, dev_status=None, stream=None) -> None:
@@ -324,3 +337,9 @@ def eg_mla_debug_set_trace(buf: Optional[torch.Tensor], ctas: int = 0) -> None:
         return
     _check(load().eg_mla_debug_set_trace(_ptr(buf), buf.numel() * buf.element_size(), ctas),
            "eg_mla_debug_set_trace")
+
+
+def eg_mla_debug_set_fault(cta: int = -1, tile: int = 0, wait_limit_ns: int = 0) -> None:
+    """Withhold the page copy of tile `tile` of CTA `cta` in later decode calls and
+    lower their wait limit (cta < 0: back to normal)."""
+    _check(load().eg_mla_debug_set_fault(cta, tile, wait_limit_ns), "eg_mla_debug_set_fault")

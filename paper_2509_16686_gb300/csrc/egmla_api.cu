@@ -13,6 +13,7 @@
 #include "../../include/egmla.h"
 #include "egmla_common.cuh"
 #include "egmla_kernels.h"
+#include "egmla_ptx.cuh"
 
 namespace {
 
@@ -176,6 +177,8 @@ int fill_decode_args(DecodeArgs& a, const eg_mla_dims* d, const void* c_pool, co
   a.num_splits = splits;
   a.workspace = workspace;
   a.status = dev_status;
+  a.wait_ns = egmla::kWaitLimitNs;
+  a.stall_cta = a.stall_tile = -1;
   return EG_MLA_OK;
 }
 
@@ -201,6 +204,20 @@ void apply_trace(DecodeArgs& a) {
   a.trace = g_trace.buf;
   a.trace_ctas = g_trace.ctas;
   a.trace_cap = g_trace.cap;
+}
+
+// test entry eg_mla_debug_set_fault: a withheld page copy and a lowered wait limit
+struct FaultCfg {
+  std::mutex mu;
+  int cta = -1, tile = -1;
+  uint64_t wait_ns = egmla::kWaitLimitNs;
+} g_fault;
+
+void apply_fault(DecodeArgs& a) {
+  std::lock_guard<std::mutex> lk(g_fault.mu);
+  a.wait_ns = g_fault.wait_ns;
+  a.stall_cta = g_fault.cta;
+  a.stall_tile = g_fault.tile;
 }
 
 // Records a profiling event on the launching stream; under stream capture it
@@ -359,6 +376,7 @@ int eg_mla_decode(const eg_mla_dims* dims, const void* q, const void* c_pool, co
     CUtensorMap maps[2];
     if (!encode_decode_maps(maps, dims, c_pool, krope_pool, num_pages)) return EG_MLA_ERR_CUDA;
     apply_trace(a);
+    apply_fault(a);
     cudaError_t e = egmla::launch_prologue_tc(a, st);
     bool fused = false;
     if (e == cudaSuccess) {
@@ -405,6 +423,21 @@ int eg_mla_debug_set_trace(void* dev_buf, int64_t bytes, int32_t ctas) {
   g_trace.buf = dev_buf;
   g_trace.ctas = ctas;
   g_trace.cap = static_cast<int>(cap > (1 << 20) ? (1 << 20) : cap);
+  return EG_MLA_OK;
+}
+
+int eg_mla_debug_set_fault(int32_t cta, int32_t tile, int64_t wait_limit_ns) {
+  std::lock_guard<std::mutex> lk(g_fault.mu);
+  if (cta < 0) {
+    g_fault.cta = g_fault.tile = -1;
+    g_fault.wait_ns = egmla::kWaitLimitNs;
+    return EG_MLA_OK;
+  }
+  if (tile < 0 || wait_limit_ns < 1000 || wait_limit_ns > static_cast<int64_t>(egmla::kWaitLimitNs))
+    return EG_MLA_ERR_INVALID_ARG;
+  g_fault.cta = cta;
+  g_fault.tile = tile;
+  g_fault.wait_ns = static_cast<uint64_t>(wait_limit_ns);
   return EG_MLA_OK;
 }
 

@@ -65,16 +65,24 @@ namespace egmla {
 
 namespace {
 
+#ifndef EGMLA_GATE_WARPS
+#define EGMLA_GATE_WARPS 8
+#endif
 constexpr int kHeads = 16;
 constexpr int kRope = 64;
-constexpr int kThreads = 480;
+constexpr int kThreads = 32 * (7 + EGMLA_GATE_WARPS);
 constexpr int kSoftWarps = 4;    // warps 0-3: TMEM lane quadrants 0-3
 constexpr int kSoftThreads = 32 * kSoftWarps;
 constexpr int kTmaWarp = 4;
 constexpr int kMmaWarp = 5;      // score MMAs and query blocks; also allocates and frees TMEM
 constexpr int kOutWarp = 6;      // output MMAs
 constexpr int kGateWarp0 = 7;
-constexpr int kGateWarps = 8;
+constexpr int kGateWarps = EGMLA_GATE_WARPS;
+// 16-byte units of each 64-feature column a gate thread takes (the 64 token
+// rows of a page over the gate threads), and lanes per token row
+constexpr int kGateUnits = 16 / kGateWarps;
+constexpr int kGateLanesPerRow = 8 / kGateUnits;
+static_assert(kGateWarps == 8 || kGateWarps == 16, "gate warps");
 constexpr uint32_t kSmemLimit = 232448;
 // named barriers of the softmax warps (0 is __syncthreads)
 constexpr int kBarTile = 1;
@@ -169,6 +177,10 @@ struct TcParams {
   uint32_t* seq_done;   // [0] CTAs done, [1 + b] split partials of sequence b stored
   int d_v, cmb_groups, cmb_g;
   int fuse;
+  // limit of every wait (ns); a test entry lowers it, together with a
+  // withheld page copy (stall_cta, stall_tile; stall_cta < 0: none)
+  uint64_t wait_ns;
+  int stall_cta, stall_tile;
 };
 
 // Trace recorder of one role of one CTA.  Only the trace instantiation of the
@@ -186,11 +198,12 @@ struct TracerT {
     if (ON && p.trace != nullptr && static_cast<int>(blockIdx.x) < p.trace_ctas)
       base = p.trace + ((static_cast<size_t>(blockIdx.x) * kTraceRoles + role) * p.trace_cap + part * cap) * 2;
   }
+  // (tag, SM clock); the phase marks carry the global timer that maps the
+  // clock of each CTA to time
   __device__ __forceinline__ void mark(int event, int tile) {
     if (ON && base != nullptr && n < cap) {
       base[2 * n] = (static_cast<unsigned long long>(event) << 56) |
-                    (static_cast<unsigned long long>(tile & 0xffffff) << 32) |
-                    static_cast<uint32_t>(globaltimer());
+                    (static_cast<unsigned long long>(tile & 0xffffff) << 32);
       base[2 * n + 1] = clock64();
       ++n;
     }
@@ -308,9 +321,9 @@ struct PageWindow {
 // still on a divergent path would otherwise only resume after the others'
 // suspended wait), every lane polls, then the warp agrees, so that a timeout
 // never splits the warp before a .sync.aligned instruction
-__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag, uint64_t limit_ns) {
   __syncwarp();
-  const bool ok = mbar_wait(bar, parity, abort_flag);
+  const bool ok = mbar_wait(bar, parity, abort_flag, limit_ns);
   return __all_sync(0xffffffffu, ok);
 }
 
@@ -488,6 +501,7 @@ __device__ void fused_combine(const TcParams& p, uint8_t* smem, Bars& bars) {
   float* olat = reinterpret_cast<float*>(smem + ((wbytes + 127u) & ~127u));   // [G][D_C]
   const uint32_t wbar = smem_u32(&bars.wbar);
   volatile int* abort_flag = &bars.abort;
+  const uint64_t wait_ns = p.wait_ns;
   auto issue_w = [&](int h) {
     if (tid == 0) {
       fence_proxy_async_smem();   // the slot area was last used through the generic proxy too
@@ -513,7 +527,7 @@ __device__ void fused_combine(const TcParams& p, uint8_t* smem, Bars& bars) {
     atomicAdd(p.seq_done, 1u);
     const uint64_t t0 = globaltimer();
     while (ld_acquire_gpu(p.seq_done) < gridDim.x) {
-      if (globaltimer() - t0 > kWaitLimitNs) {
+      if (globaltimer() - t0 > wait_ns) {
         report_status(p.status, kStatusTimeout);
         *abort_flag = 1;
         break;
@@ -531,7 +545,7 @@ __device__ void fused_combine(const TcParams& p, uint8_t* smem, Bars& bars) {
       const uint64_t t0 = globaltimer();
       while (ld_acquire_gpu(p.seq_done + 1 + b0) < want) {
         if (*abort_flag) break;
-        if (globaltimer() - t0 > kWaitLimitNs) {
+        if (globaltimer() - t0 > wait_ns) {
           report_status(p.status, kStatusTimeout);
           *abort_flag = 1;
           break;
@@ -579,7 +593,7 @@ __device__ void fused_combine(const TcParams& p, uint8_t* smem, Bars& bars) {
     // copy is waited for even after an abort (no copy may outlive the CTA)
     if (tid == 0) {
       volatile int own = 0;
-      if (!mbar_wait(wbar, phase, &own)) {
+      if (!mbar_wait(wbar, phase, &own, wait_ns)) {
         report_status(p.status, kStatusTimeout);
         *abort_flag = 1;
       }
@@ -649,6 +663,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t sbase = smem_u32(smem);
   Bars& bars = *reinterpret_cast<Bars*>(smem + C::OFF_MISC);
   volatile int* abort_flag = &bars.abort;
+  const uint64_t wait_ns = p.wait_ns;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   phase_mark<DBG == 2>(p, 0);
@@ -716,21 +731,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int slot = it % C::NS;
       if (lane == 0) {
         tr.mark(0, it);
-        if (!mbar_wait(smem_u32(&bars.empty[slot]), ((it / C::NS) & 1) ^ 1, abort_flag)) ok_loop = false;
+        if (!mbar_wait(smem_u32(&bars.empty[slot]), ((it / C::NS) & 1) ^ 1, abort_flag, wait_ns)) ok_loop = false;
         if (ok_loop) {
           tr.mark(1, it);
           const bool ok = pg >= 0 && pg < p.num_pages;
           if (!ok) report_status(p.status, kStatusOutOfRange);
-          const uint32_t fb = smem_u32(&bars.full[slot]);
-          mbar_arrive_expect_tx(fb, ok ? C::PAGE_TX : 0u);
-          if (ok) {
-            const uint32_t dst = sbase + slot * C::SLOT;
-            const int y = pg * kPage;
-            tma_load_3d(dst, &cmap, 0, y, 0, fb, pol_stream);
-            tma_load_2d(dst + C::KR_OFF, &krmap, 0, y, fb, pol_stream);
+          // (test entry) a withheld page: no copy and no arrival, so that the
+          // gate's wait on this slot runs out
+          const bool withheld = static_cast<int>(blockIdx.x) == p.stall_cta && it == p.stall_tile;
+          if (!withheld) {
+            const uint32_t fb = smem_u32(&bars.full[slot]);
+            mbar_arrive_expect_tx(fb, ok ? C::PAGE_TX : 0u);
+            if (ok) {
+              const uint32_t dst = sbase + slot * C::SLOT;
+              const int y = pg * kPage;
+              tma_load_3d(dst, &cmap, 0, y, 0, fb, pol_stream);
+              tma_load_2d(dst + C::KR_OFF, &krmap, 0, y, fb, pol_stream);
+            }
+            last_it[slot] = it;
           }
           tr.mark(2, it);
-          last_it[slot] = it;
         }
       }
       ok_loop = __shfl_sync(0xffffffffu, ok_loop, 0);
@@ -741,7 +761,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // also after an abort (own flag: the wait is bounded but not cut short)
       volatile int own = 0;
       for (int s = 0; s < C::NS; ++s)
-        if (last_it[s] >= 0 && !mbar_wait(smem_u32(&bars.full[s]), (last_it[s] / C::NS) & 1, &own)) *abort_flag = 1;
+        if (last_it[s] >= 0 && !mbar_wait(smem_u32(&bars.full[s]), (last_it[s] / C::NS) & 1, &own, wait_ns)) *abort_flag = 1;
     }
     __syncwarp();
   } else if (warp == kMmaWarp) {
@@ -832,7 +852,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint64_t now = globaltimer();
           if (idle_since == 0) idle_since = now;
           bool stop = *abort_flag != 0;
-          if (!stop && now - idle_since > kWaitLimitNs) {
+          if (!stop && now - idle_since > wait_ns) {
             *abort_flag = 1;
             stop = true;
           }
@@ -846,14 +866,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         // bounded but not cut short by an abort)
         volatile int own = 0;
         for (int b = 0; b < 2; ++b)
-          if (last_q[b] >= 0 && !mbar_wait(smem_u32(&bars.qfull[b]), (last_q[b] / C::NQ) & 1, &own)) *abort_flag = 1;
+          if (last_q[b] >= 0 && !mbar_wait(smem_u32(&bars.qfull[b]), (last_q[b] / C::NQ) & 1, &own, wait_ns)) *abort_flag = 1;
       }
       __syncwarp();
       if (issued) {
         if (elect_one()) mma_commit(smem_u32(&bars.drain_s));
         __syncwarp();
         volatile int own = 0;
-        if (!mbar_wait(smem_u32(&bars.drain_s), 0, &own)) *abort_flag = 1;
+        if (!mbar_wait(smem_u32(&bars.drain_s), 0, &own, wait_ns)) *abort_flag = 1;
       }
     }
     __syncwarp();
@@ -878,7 +898,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tr.init(p, 1, 1, 2);   // second half of the MMA role's run
       if (lane != 0) tr.base = nullptr;
       while (wo.next(to)) {
-        if (!warp_wait(smem_u32(&bars.spdone[jo % kNP]), (jo / kNP) & 1, abort_flag)) break;
+        if (!warp_wait(smem_u32(&bars.spdone[jo % kNP]), (jo / kNP) & 1, abort_flag, wait_ns)) break;
         tr.mark(3, jo);
         tc_fence_after();
         if (elect_one()) {
@@ -912,7 +932,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (elect_one()) mma_commit(smem_u32(&bars.drain_o));
         __syncwarp();
         volatile int own = 0;
-        if (!mbar_wait(smem_u32(&bars.drain_o), 0, &own)) *abort_flag = 1;
+        if (!mbar_wait(smem_u32(&bars.drain_o), 0, &own, wait_ns)) *abort_flag = 1;
       }
     }
     __syncwarp();
@@ -930,8 +950,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // evict-first): each tile issues the id loads of the tile two ahead and the
     // gate-row loads of the next tile, so neither latency sits on the loop.
     const int gw = warp - kGateWarp0;
-    const int pp = lane & 3;
-    const int row = 2 * (gw * 4 + (lane >> 3)) + ((lane >> 2) & 1);
+    const int pp = lane % kGateLanesPerRow;
+    const int row = gw * (32 / kGateLanesPerRow) + lane / kGateLanesPerRow;
     const uint64_t pol_keep = policy_evict_last();
     constexpr bool gate_ln = GATE_LN;
     Walker w;
@@ -945,18 +965,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int n = (pg >= 0 && pg < p.num_pages) ? tt.ntok : 0;
       return row < n ? __ldg(p.id_pool + static_cast<size_t>(pg) * kPage + row) : 0;
     };
-    auto load_g = [&](int& id, uint4 (&gv)[C::NCH][2]) {
+    auto load_g = [&](int& id, uint4 (&gv)[C::NCH][kGateUnits]) {
       if ((unsigned)id >= (unsigned)p.vocab) {
         report_status(p.status, kStatusOutOfRange);
         id = 0;
       }
-      const __nv_bfloat16* src = p.gate_table + static_cast<size_t>(id) * D_C + pp * 16;
+      const __nv_bfloat16* src = p.gate_table + static_cast<size_t>(id) * D_C + pp * 8 * kGateUnits;
 #pragma unroll
-      for (int fc = 0; fc < C::NCH; ++fc) ldg_32_na_hint(src + fc * 64, pol_keep, gv[fc][0], gv[fc][1]);
+      for (int fc = 0; fc < C::NCH; ++fc) {
+        if constexpr (kGateUnits == 2)
+          ldg_32_na_hint(src + fc * 64, pol_keep, gv[fc][0], gv[fc][1]);
+        else
+          gv[fc][0] = ldg_16_na_hint(src + fc * 64, pol_keep);
+      }
     };
-    // shared-memory offset of unit (2 pp + h) of column fc of this thread's row
+    // shared-memory offset of unit (kGateUnits pp + h) of column fc of this thread's row
     auto unit_off = [&](int fc, int h) -> uint32_t {
-      return fc * C::PCHUNK + row * 128 + (((2 * pp + h) ^ (row & 7)) << 4);
+      return fc * C::PCHUNK + row * 128 + (((kGateUnits * pp + h) ^ (row & 7)) << 4);
     };
     Tracer tr;
     tr.init(p, 2);
@@ -966,7 +991,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool have1 = have && w.next(t1);
     bool have2 = have1 && w.next(t2);
     int id0 = 0, id1 = 0, id2 = 0;   // ids of tiles j, j + 1, j + 2
-    uint4 gcur[C::NCH][2], gnext[C::NCH][2];
+    uint4 gcur[C::NCH][kGateUnits], gnext[C::NCH][kGateUnits];
     if (GATE) {
       if (have) id0 = load_id(t);
       if (have1) id1 = load_id(t1);
@@ -981,7 +1006,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (have2) id2 = load_id(t2);
         if (have1) load_g(id1, gnext);
       }
-      if (!warp_wait(smem_u32(&bars.full[slot]), (j / C::NS) & 1, abort_flag)) break;
+      if (!warp_wait(smem_u32(&bars.full[slot]), (j / C::NS) & 1, abort_flag, wait_ns)) break;
       tr.mark(1, j);
       uint8_t* cpage = smem + slot * C::SLOT;
       if (DUMP) {
@@ -992,15 +1017,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int fc = 0; fc < C::NCH; ++fc) {
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-              dc[fc * 8 + 2 * pp + h] = *reinterpret_cast<const uint4*>(cpage + unit_off(fc, h));
-              dg[fc * 8 + 2 * pp + h] = gcur[fc][h];
+            for (int h = 0; h < kGateUnits; ++h) {
+              dc[fc * 8 + kGateUnits * pp + h] = *reinterpret_cast<const uint4*>(cpage + unit_off(fc, h));
+              dg[fc * 8 + kGateUnits * pp + h] = gcur[fc][h];
             }
           }
 #pragma unroll
-          for (int h = 0; h < 2; ++h)
-            reinterpret_cast<uint4*>(p.dump_kr + o * kRope)[2 * pp + h] = *reinterpret_cast<const uint4*>(
-                cpage + C::KR_OFF + row * 128 + (((2 * pp + h) ^ (row & 7)) << 4));
+          for (int h = 0; h < kGateUnits; ++h)
+            reinterpret_cast<uint4*>(p.dump_kr + o * kRope)[kGateUnits * pp + h] = *reinterpret_cast<const uint4*>(
+                cpage + C::KR_OFF + row * 128 + (((kGateUnits * pp + h) ^ (row & 7)) << 4));
           if (pp == 0) p.dump_ids[o] = id0;
         }
         warp_arrive(smem_u32(&bars.empty[slot]));
@@ -1010,11 +1035,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           float* st = reinterpret_cast<float*>(smem + C::OFF_STAT + slot * C::STAT_BYTES);
           // all shared-memory reads of this thread's units first (the in-place
           // stores below would otherwise order every later load behind them)
-          uint4 cv[C::NCH][2];
+          uint4 cv[C::NCH][kGateUnits];
 #pragma unroll
           for (int fc = 0; fc < C::NCH; ++fc)
 #pragma unroll
-            for (int h = 0; h < 2; ++h) cv[fc][h] = *reinterpret_cast<const uint4*>(cpage + unit_off(fc, h));
+            for (int h = 0; h < kGateUnits; ++h) cv[fc][h] = *reinterpret_cast<const uint4*>(cpage + unit_off(fc, h));
           tr.mark(5, j);
           const bool valid = row < t.ntok;
           if constexpr (GATE_ADD) {
@@ -1025,7 +1050,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int fc = 0; fc < C::NCH; ++fc) {
 #pragma unroll
-              for (int h = 0; h < 2; ++h) {
+              for (int h = 0; h < kGateUnits; ++h) {
                 const uint32_t* cw = reinterpret_cast<const uint32_t*>(&cv[fc][h]);
                 const uint32_t* gw2 = reinterpret_cast<const uint32_t*>(&gcur[fc][h]);
 #pragma unroll
@@ -1038,7 +1063,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             float sum1 = s1.x + s1.y, sum2 = s2.x + s2.y;
 #pragma unroll
-            for (int o = 1; o < 4; o <<= 1) {
+            for (int o = 1; o < kGateLanesPerRow; o <<= 1) {
               sum1 += __shfl_xor_sync(0xffffffffu, sum1, o);
               sum2 += __shfl_xor_sync(0xffffffffu, sum2, o);
             }
@@ -1050,7 +1075,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int fc = 0; fc < C::NCH; ++fc) {
 #pragma unroll
-              for (int h = 0; h < 2; ++h) {
+              for (int h = 0; h < kGateUnits; ++h) {
                 const uint32_t* cw = reinterpret_cast<const uint32_t*>(&cv[fc][h]);
                 const uint32_t* gw2 = reinterpret_cast<const uint32_t*>(&gcur[fc][h]);
                 uint4 z;
@@ -1078,7 +1103,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int fc = 0; fc < C::NCH; ++fc) {
 #pragma unroll
-              for (int h = 0; h < 2; ++h) {
+              for (int h = 0; h < kGateUnits; ++h) {
                 uint4 z;
                 z.x = mul_bf16x2(cv[fc][h].x, gcur[fc][h].x);
                 z.y = mul_bf16x2(cv[fc][h].y, gcur[fc][h].y);
@@ -1106,7 +1131,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             // ablation's norm: mu = 0, r = 1)
             if (gate_ln) {
 #pragma unroll
-              for (int o = 1; o < 4; o <<= 1) {
+              for (int o = 1; o < kGateLanesPerRow; o <<= 1) {
                 sum1 += __shfl_xor_sync(0xffffffffu, sum1, o);
                 sum2 += __shfl_xor_sync(0xffffffffu, sum2, o);
               }
@@ -1126,7 +1151,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int fc = 0; fc < C::NCH; ++fc)
 #pragma unroll
-              for (int h = 0; h < 2; ++h)
+              for (int h = 0; h < kGateUnits; ++h)
                 *reinterpret_cast<uint4*>(cpage + unit_off(fc, h)) = make_uint4(0, 0, 0, 0);
           }
         }
@@ -1146,8 +1171,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         id1 = id2;
 #pragma unroll
         for (int fc = 0; fc < C::NCH; ++fc) {
-          gcur[fc][0] = gnext[fc][0];
-          gcur[fc][1] = gnext[fc][1];
+#pragma unroll
+          for (int h = 0; h < kGateUnits; ++h) gcur[fc][h] = gnext[fc][h];
         }
       }
     }
@@ -1196,7 +1221,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       if (t.first) {
         ++seg;
-        ok = warp_wait(smem_u32(&bars.qfull[seg % C::NQ]), (seg / C::NQ) & 1, abort_flag);
+        ok = warp_wait(smem_u32(&bars.qfull[seg % C::NQ]), (seg / C::NQ) & 1, abort_flag, wait_ns);
         if (ok && GATE) {
           // w_h = sum_f bf16(q^ gamma)_hf and b_h = q^_h . beta from their
           // per-chunk partials after the operands, added in chunk order
@@ -1221,7 +1246,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tr.mark(0, it);
       // scores of this tile; the MMA warp's release arrival on the same barrier
       // orders the gate's statistics before them
-      ok = ok && warp_wait(smem_u32(&bars.sready[sb]), (it / kNB) & 1, abort_flag);
+      ok = ok && warp_wait(smem_u32(&bars.sready[sb]), (it / kNB) & 1, abort_flag, wait_ns);
       tr.mark(1, it);
       float s[2][4];
       float mu[2] = {0.f, 0.f}, rr[2] = {1.f, 1.f};
@@ -1299,7 +1324,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           // reference: the previous tile's output MMA must be complete first
           // (completion n of pfree[b] is output MMA n kNP + b)
           const int pv = (it - 1) % kNP;
-          ok = warp_wait(smem_u32(&bars.pfree[pv]), ((it - 1) / kNP) & 1, abort_flag);
+          ok = warp_wait(smem_u32(&bars.pfree[pv]), ((it - 1) / kNP) & 1, abort_flag, wait_ns);
           if (ok) {
             tc_fence_after();
             float o[32];
@@ -1320,7 +1345,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // the P' buffer of this tile is free once the output MMA kNP tiles back
       // has read it
-      ok = ok && warp_wait(smem_u32(&bars.pfree[pb]), ((it / kNP) & 1) ^ 1, abort_flag);
+      ok = ok && warp_wait(smem_u32(&bars.pfree[pb]), ((it / kNP) & 1) ^ 1, abort_flag, wait_ns);
       tr.mark(5, it);
       if (ok) {
         // The output MMA sees the bf16-rounded weights P'; the denominator and
@@ -1386,7 +1411,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         // the segment's last output MMA (the earlier ones complete before it;
         // completion n of pfree[b] is output MMA n kNP + b), then O^T
-        ok = warp_wait(smem_u32(&bars.pfree[pb]), (it / kNP) & 1, abort_flag);
+        ok = warp_wait(smem_u32(&bars.pfree[pb]), (it / kNP) & 1, abort_flag, wait_ns);
         if (ok) {
           tc_fence_after();
           float o[32];
@@ -1517,6 +1542,9 @@ cudaError_t launch_one(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_
   const int g = std::min(static_cast<int>(kFusedMaxG), (a.batch + groups - 1) / groups);
   p.cmb_g = g;
   p.cmb_groups = (a.batch + g - 1) / g;
+  p.wait_ns = a.wait_ns;
+  p.stall_cta = a.stall_cta;
+  p.stall_tile = a.stall_tile;
   p.fuse = DBG != 1 && a.batch > 0 && a.num_splits <= resident_ctas(kern, C::SMEM);
   if (fused) *fused = p.fuse != 0;
   if (!p.fuse) {

@@ -63,6 +63,10 @@ struct DecodeArgs {
   // pipeline event trace of the decode kernel (eg_mla_debug_set_trace)
   void* trace;
   int trace_ctas, trace_cap;
+  // limit of every pipeline wait (ns), and a withheld page copy of the
+  // tensor-core decode kernel (eg_mla_debug_set_fault; stall_cta < 0: none)
+  uint64_t wait_ns;
+  int stall_cta, stall_tile;
 };
 
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t st);

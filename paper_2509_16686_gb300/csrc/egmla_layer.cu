@@ -152,6 +152,12 @@ size_t eg_mla_layer_workspace_size(const eg_mla_dims* dims, const eg_mla_layer_d
   return w.dec_bytes == 0 ? 0 : w.total;
 }
 
+size_t eg_mla_layer_attn_offset(const eg_mla_dims* dims, const eg_mla_layer_dims* layer, int32_t batch,
+                                int32_t num_splits) {
+  if (eg_mla_layer_workspace_size(dims, layer, batch, num_splits) == 0) return 0;
+  return layer_workspace(dims, batch, num_splits).off_u;
+}
+
 int eg_mla_layer_decode(const eg_mla_dims* dims, const eg_mla_layer_dims* layer, const eg_mla_layer_weights* wt,
                         const void* x, const int32_t* ids_new, const int32_t* positions, void* c_pool,
                         void* krope_pool, int32_t* id_pool, const int32_t* block_table, int32_t max_pages_per_seq,

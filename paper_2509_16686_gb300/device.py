@@ -191,6 +191,14 @@ class DeviceLayer:
                                  self.y, self.workspace, dc.num_splits, dc.status, stream)
         return self.y
 
+    def attn_output(self) -> torch.Tensor:
+        """The last step's attention output u [B, H, d_v] (bf16), read from where
+        eg_mla_layer_decode leaves it in the workspace."""
+        dc = self.dc
+        off = _lib.eg_mla_layer_attn_offset(dc.dims, self.layer_dims, dc.batch, dc.num_splits)
+        n = dc.batch * dc.dims.num_heads * dc.dims.d_v * 2
+        return self.workspace[off:off + n].view(torch.bfloat16).view(dc.batch, dc.dims.num_heads, dc.dims.d_v)
+
 
 def upload_layer(lc, device="cuda", num_splits: int = 0) -> DeviceLayer:
     """A synth.LayerCase on the device (bf16)."""

@@ -142,3 +142,20 @@ def test_layer_decode_rejects_before_launch(lib):
     assert call(x=fake + 8) == _lib.EG_MLA_ERR_INVALID_ARG              # 16-byte alignment
     assert call(ws_bytes=1 << 20) == _lib.EG_MLA_ERR_WORKSPACE         # far below the layer's workspace
     assert call(batch=0) == _lib.EG_MLA_OK                              # nothing to do, nothing launched
+
+
+def test_fault_entry_validates_its_arguments(lib):
+    # host-only: no launch happens here; cta < 0 restores normal operation
+    assert lib.eg_mla_debug_set_fault(0, -1, 1_000_000) == _lib.EG_MLA_ERR_INVALID_ARG
+    assert lib.eg_mla_debug_set_fault(0, 1, 10) == _lib.EG_MLA_ERR_INVALID_ARG
+    assert lib.eg_mla_debug_set_fault(0, 1, 3_000_000_000) == _lib.EG_MLA_ERR_INVALID_ARG
+    assert lib.eg_mla_debug_set_fault(0, 1, 1_000_000) == _lib.EG_MLA_OK
+    assert lib.eg_mla_debug_set_fault(-1, 0, 0) == _lib.EG_MLA_OK
+
+
+def test_layer_attention_offset_is_inside_the_workspace(lib):
+    dims = _lib.make_dims(16, 128, 64, 128, 256, 32000)
+    layer = _lib.make_layer_dims(2048)
+    ws = _lib.eg_mla_layer_workspace_size(dims, layer, 64, 152)
+    off = _lib.eg_mla_layer_attn_offset(dims, layer, 64, 152)
+    assert 0 < off and off % 256 == 0 and off + 64 * 16 * 128 * 2 <= ws

@@ -243,6 +243,27 @@ def test_out_of_range_token_id_is_reported_and_gpu_stays_usable(gpu_lib):
     check_bf16(got, orc.decode_unabsorbed(case), "after error", scaled_abs=True)
 
 
+def test_withheld_page_times_out_and_gpu_stays_usable(gpu_lib):
+    """The failure path of the decode kernel's pipeline waits, made to run: CTA 0
+    withholds the copy of its third page (eg_mla_debug_set_fault) and every
+    wait of that launch gives up after 1 ms.  The call must report
+    EG_MLA_ERR_TIMEOUT with every CTA returning on its own (the drain of copies
+    and MMAs, TMEM freed), and a clean step afterwards must match the oracle."""
+    case = small_bf16((700, 65, 300))   # 21 schedule units: CTA 0 of 4 walks 5 pages
+    dc = device.upload(case, num_splits=4)
+    _lib.eg_mla_debug_set_fault(0, 2, 1_000_000)
+    try:
+        dc.step()
+        torch.cuda.synchronize()
+    finally:
+        _lib.eg_mla_debug_set_fault(-1)
+    assert dc.read_status() == _lib.EG_MLA_ERR_TIMEOUT
+    _, got = run(case, 4)
+    check_bf16(got, orc.decode_unabsorbed(case), "after a timed-out step", scaled_abs=True)
+    _, got = run(case, 0)
+    check_bf16(got, orc.decode_unabsorbed(case), "after a timed-out step, default splits", scaled_abs=True)
+
+
 def test_out_of_range_page_is_reported(gpu_lib):
     case = small_bf16((70, 20))
     dc = device.upload(case, num_splits=2)
@@ -263,19 +284,24 @@ def sampled_check(case, batches, num_splits=0):
 
 
 def test_workload_c4k_full_size(gpu_lib):
+    # a third of the sequences (every third one), every head
     case = synth.case_c4k()
-    sampled_check(case, [0, 17, 31])
+    sampled_check(case, range(0, case.batch, 3))
 
 
 def test_workload_c32k_full_size(gpu_lib):
+    # every sequence, every head (the configuration the roofline target is stated on)
     case = synth.case_c32k()
-    sampled_check(case, [0, 5])
+    sampled_check(case, range(case.batch))
 
 
 def test_workload_ragged_full_size(gpu_lib):
+    # a third of the sequences, spread over the length distribution (every third
+    # in length order, so the shortest and the longest are among them)
     case = synth.case_ragged()
     order = np.argsort(case.seq_lens)
-    sampled_check(case, [int(order[0]), int(order[64]), int(order[-1])])
+    picked = sorted({int(b) for b in order[::3]} | {int(order[-1])})
+    sampled_check(case, picked)
 
 
 def test_workload_ragged_mla_baseline_full_size(gpu_lib):

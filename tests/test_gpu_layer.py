@@ -2,17 +2,22 @@
 (eg_mla_layer_decode: projections, kv_norm and RoPE, append, gated latent
 attention, output projection) against the fp64 layer oracle, through the C ABI.
 
-Bounds, derived from the arithmetic.  The attention output u inside the layer
-carries the decode's bf16 error (rel-L2 <= 5e-3, the hot path's bound), and the
-output y = W^O u sums the 2048 errors of u through a random weight row of unit
-norm: each element's error is close to normal with standard deviation
-rel-L2(u) * rms(y), and y itself is rounded to bf16.  So the layer output is
-held to rel-L2 <= 5e-3 and, per element, |dy| <= 5 * 5e-3 * rms(y_ref) +
-2^-8 |y_ref| (five standard deviations over ~10^4 outputs, plus one bf16
-rounding).  The appended cache row (c^KV after kv_norm, the rotated k^R) is
-within two bf16 units in the last place of the oracle's stored value (the
-projections are summed in a different order on the GPU, which can move a
-rounding by one unit).
+Bounds, each fixed in advance by the arithmetic that produces the checked value:
+  - the attention output u inside the layer (read where the call leaves it,
+    eg_mla_layer_attn_offset) is held to the hot path's bf16 bound against the
+    oracle's u of the same step: max-abs <= 1e-2 (per element 1e-2 max(1, |u|)
+    for sequences shorter than the workloads' shortest context, as in the
+    decode tests) and rel-L2 <= 5e-3;
+  - the output y = W^O u is compared with W^O applied in fp64 to the GPU's own
+    u: what remains is the projection's fp32 accumulation over K = H d_v terms
+    (at most K 2^-24 sum_i |w_i u_i|) and the bf16 rounding of y (at most
+    2^-8 |y|);
+  - y against the oracle's y: rel-L2 <= 5e-3 (the decode's bound carried
+    through a linear map);
+  - the appended cache row (c^KV after kv_norm, the rotated k^R) lies within
+    two bf16 units in the last place of the oracle's stored value (the
+    projections are summed in a different order on the GPU, which can move a
+    rounding by one unit).
 """
 import numpy as np
 import pytest
@@ -23,16 +28,38 @@ from paper_2509_16686_gb300 import _lib, device, synth
 
 pytestmark = pytest.mark.gpu
 
+BF16_MAX_ABS = 1e-2
 BF16_REL_L2 = 5e-3
 
 
-def check_bf16(got, ref, where):
+def rel_l2(got, ref):
+    return float(np.linalg.norm(got - ref) / max(np.linalg.norm(ref), 1e-30))
+
+
+def check_u(got, ref, where, scaled_abs):
+    """The hot path's bf16 bound on the attention output."""
     assert np.isfinite(got).all(), where
     diff = np.abs(got - ref)
-    rel = float(np.linalg.norm(got - ref) / max(np.linalg.norm(ref), 1e-30))
-    bound = 5 * BF16_REL_L2 * float(np.sqrt(np.mean(ref * ref))) + 2.0 ** -8 * np.abs(ref)
-    worst = float((diff / bound).max())
-    assert worst <= 1.0 and rel <= BF16_REL_L2, f"{where}: max_abs={diff.max():.3e} (x{worst:.2f} of bound) rel_l2={rel:.3e}"
+    bound = BF16_MAX_ABS * np.maximum(1.0, np.abs(ref)) if scaled_abs else BF16_MAX_ABS
+    rel = rel_l2(got, ref)
+    assert (diff <= bound).all() and rel <= BF16_REL_L2, f"{where} u: max_abs={diff.max():.3e} rel_l2={rel:.3e}"
+
+
+def check_y(dl, lc, got_y, ref_y, where, batches=None):
+    """y against W^O applied in fp64 to the GPU's u (rounding bound), and against
+    the oracle's y (rel-L2)."""
+    assert np.isfinite(got_y).all(), where
+    u = device.output_f64(dl.attn_output()).reshape(dl.dc.batch, -1)
+    w_o = orc.widen(lc.w_o, "bf16")
+    bs = list(range(dl.dc.batch)) if batches is None else list(batches)
+    y_u = u[bs] @ w_o.T
+    acc = np.abs(u[bs]) @ np.abs(w_o).T
+    k = w_o.shape[1]
+    bound = 2.0 ** -8 * np.abs(y_u) + k * 2.0 ** -24 * acc
+    diff = np.abs(got_y[bs] - y_u)
+    assert (diff <= bound).all(), f"{where} y vs W^O u: worst {float((diff / bound).max()):.2f} of the bound"
+    rel = rel_l2(got_y[bs], ref_y[bs])
+    assert rel <= BF16_REL_L2, f"{where} y vs oracle: rel_l2={rel:.3e}"
 
 
 def run_layer(lc, splits=0):
@@ -62,9 +89,12 @@ def test_layer_step_matches_oracle(gpu_lib, d_c, gate):
                            seed=31, latent_scale=0.5, layout="permuted", affine_ln=True, extra_pages=3)
     lc = synth.make_layer_case(case, 256, seed=32)
     ref = orc.layer_decode(lc)
+    u_ref = orc.decode_unabsorbed(orc.layer_step(lc))
     for splits in (0, 3):
         dl, got = run_layer(lc, splits)
-        check_bf16(got, ref, f"layer d_c={d_c} gate={gate} splits={splits}")
+        where = f"layer d_c={d_c} gate={gate} splits={splits}"
+        check_u(device.output_f64(dl.attn_output()), u_ref, where, scaled_abs=True)
+        check_y(dl, lc, got, ref, where)
     check_appended_rows(dl, lc)
 
 
@@ -74,17 +104,21 @@ def test_layer_step_long_positions(gpu_lib):
                            layout="permuted")
     lc = synth.make_layer_case(case, 512, seed=34)
     dl, got = run_layer(lc)
-    check_bf16(got, orc.layer_decode(lc), "layer long positions")
+    check_u(device.output_f64(dl.attn_output()), orc.decode_unabsorbed(orc.layer_step(lc)), "long positions",
+            scaled_abs=False)
+    check_y(dl, lc, got, orc.layer_decode(lc), "layer long positions")
     check_appended_rows(dl, lc)
 
 
 def test_layer_step_24_layer_model_shape_sampled(gpu_lib):
     # one layer of the 24-layer workload's shape: hidden 2048, batch 64 x 8192
     lc = synth.make_layer_case(synth.case_layer(0), 2048, seed=35)
-    _, got = run_layer(lc)
-    sample = [0, 37, 63]
-    ref = orc.layer_decode(lc, batches=sample)
-    check_bf16(got[sample], ref[sample], "layer 2048 sampled")
+    dl, got = run_layer(lc)
+    sample = [0, 21, 37, 50, 63]
+    step = orc.layer_step(lc)
+    u_ref = orc.decode_unabsorbed(step, batches=sample)
+    check_u(device.output_f64(dl.attn_output())[sample], u_ref[sample], "layer 2048 sampled", scaled_abs=False)
+    check_y(dl, lc, got, orc.layer_decode(lc, batches=sample), "layer 2048 sampled", batches=sample)
 
 
 def test_layer_group_shares_one_cache(gpu_lib):
@@ -110,7 +144,51 @@ def test_layer_group_shares_one_cache(gpu_lib):
     dl_b.step()
     torch.cuda.synchronize()
     assert dl_a.dc.read_status() == 0 and dl_b.dc.read_status() == 0
-    check_bf16(device.output_f64(dl_a.y), orc.layer_decode(lc_a), "group first layer")
-    check_bf16(device.output_f64(dl_b.y), orc.layer_decode(lc_b, kv_from=lc_a), "group second layer")
+    check_u(device.output_f64(dl_a.attn_output()), orc.decode_unabsorbed(orc.layer_step(lc_a)), "group first layer",
+            scaled_abs=True)
+    check_y(dl_a, lc_a, device.output_f64(dl_a.y), orc.layer_decode(lc_a), "group first layer")
+    # the second layer's u: its own step over the cache the first layer wrote
+    check_u(device.output_f64(dl_b.attn_output()), orc.decode_unabsorbed(orc.layer_step(lc_b, kv_from=lc_a)),
+            "group second layer", scaled_abs=True)
+    check_y(dl_b, lc_b, device.output_f64(dl_b.y), orc.layer_decode(lc_b, kv_from=lc_a), "group second layer")
     # the cache holds the first layer's token once; a second append would have been the same row
     check_appended_rows(dl_a, lc_a)
+
+
+def test_24_layer_chain_matches_chained_oracle(gpu_lib):
+    """The 24-layer decoder step as the bench runs it (each layer's output y the
+    next layer's input x), with 24 independently seeded layers (cache, gate
+    table, weights), at a reduced batch and context.  Every layer is held to
+    the layer bounds against the oracle applied to that layer's actual input
+    (the GPU's y of the layer before, as stored in bf16); the chain's last
+    output is compared with the oracle run through all 24 layers from the same
+    first input, where each layer can add at most its own bound: rel-L2 <= 24 x
+    5e-3 (reported, with the measured value, in the assertion message)."""
+    import dataclasses
+    n_layers, batch, ctx = 24, 4, 300
+    lcs = []
+    for k in range(n_layers):
+        case = synth.case_layer(k, batch=batch, ctx=ctx, layout="permuted", extra_pages=2)
+        lcs.append(synth.make_layer_case(case, 2048, seed=5000 + k))
+    dls = [device.upload_layer(lc) for lc in lcs]
+    for k in range(1, n_layers):
+        dls[k].x = dls[k - 1].y
+    for dl in dls:
+        dl.step()
+    torch.cuda.synchronize()
+    for k, dl in enumerate(dls):
+        assert dl.dc.read_status() == 0, k
+    x_oracle = lcs[0].x
+    for k, (lc, dl) in enumerate(zip(lcs, dls)):
+        # layer k on its actual input
+        x_gpu = device.bf16_tensor_to_bits(dl.x)
+        lc_k = dataclasses.replace(lc, x=x_gpu)
+        got = device.output_f64(dl.y)
+        check_u(device.output_f64(dl.attn_output()), orc.decode_unabsorbed(orc.layer_step(lc_k)), f"chain layer {k}",
+                scaled_abs=False)
+        check_y(dl, lc_k, got, orc.layer_decode(lc_k), f"chain layer {k}")
+        # the oracle's own chain, each y stored in the model dtype as the layer stores it
+        y_oracle = orc.layer_decode(dataclasses.replace(lc, x=x_oracle))
+        x_oracle = orc.store(y_oracle, "bf16")
+    rel = rel_l2(got, y_oracle)
+    assert rel <= n_layers * BF16_REL_L2, f"24-layer chain: rel_l2={rel:.3e}"
