@@ -36,14 +36,29 @@ from __future__ import annotations
 import argparse
 import hashlib
 import json
-import math
 import os
 import statistics
 import subprocess
 import sys
 import time
 
-import numpy as np
+
+def host_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+# The fp64 oracle's matrix products run in the BLAS numpy loads; its thread
+# count is pinned here, before numpy is imported, so that the CPU baseline can
+# state the threads it used (an explicit setting by the caller is kept).
+BLAS_ENV = ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS")
+for _v in BLAS_ENV:
+    os.environ.setdefault(_v, str(host_cores()))
+BLAS_THREADS = int(os.environ["OPENBLAS_NUM_THREADS"])
+
+import numpy as np  # noqa: E402
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
@@ -68,6 +83,10 @@ def parse():
     ap.add_argument("--splits", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=0)
+    ap.add_argument("--oracle-probe", default=None, help=argparse.SUPPRESS)
+    ap.add_argument("--oracle-budget", type=float, default=4.0, help=argparse.SUPPRESS)
+    ap.add_argument("--no-mla-baseline", action="store_true",
+                    help="skip the gate-off (plain MLA) measurement of the same workload")
     ap.add_argument("--lgz", type=int, default=1,
                     help="layers24_full: layer group size (consecutive layers share one latent cache and its "
                          "KV projection, Appendix H)")
@@ -224,11 +243,41 @@ def oracle_sample_rate(case, budget_s):
     return rate, sample, dt
 
 
-def host_cores():
-    try:
-        return len(os.sched_getaffinity(0))
-    except AttributeError:
-        return os.cpu_count() or 1
+def oracle_rate_subprocess(workload, threads, budget_s):
+    """The oracle's decode tokens/s on `workload` in a child process whose BLAS
+    runs `threads` threads (the single-thread times of the baseline)."""
+    env = dict(os.environ)
+    for v in BLAS_ENV:
+        env[v] = str(threads)
+    r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-probe", workload,
+                        "--oracle-budget", str(budget_s)], capture_output=True, text=True, env=env, timeout=600)
+    if r.returncode != 0:
+        return {"error": r.stderr.strip().splitlines()[-1:] if r.stderr else "failed"}
+    return json.loads(r.stdout.strip().splitlines()[-1])
+
+
+def oracle_probe(workload, budget_s):
+    """(child process) one bounded oracle sample of a workload, as JSON."""
+    from paper_2509_16686_gb300 import synth
+    case = synth.case_tiny() if workload == "tiny" else make_workload(workload)[0]
+    rate, sample, dt = oracle_sample_rate(case, budget_s)
+    print(json.dumps({"value": rate, "sample": sample, "seconds": dt, "threads": BLAS_THREADS}))
+    return 0
+
+
+def cpu_baseline_line(case, budget_s, n_layers=1):
+    """cpu_baseline: the oracle on this process's BLAS threads over a bounded
+    sample of the workload, plus single-thread rates on the tiny fp32 and the
+    4K workloads."""
+    rate, sample, _ = oracle_sample_rate(case, budget_s)
+    if n_layers > 1:
+        rate /= n_layers
+        sample += f", one layer of {n_layers} (rate / {n_layers})"
+    single = {w: oracle_rate_subprocess(w, 1, 4.0) for w in ("tiny", "c4k")}
+    return {"value": rate, "unit": UNIT, "cores": BLAS_THREADS, "threads": BLAS_THREADS, "host_cores": host_cores(),
+            "kind": "oracle", "sample": sample,
+            "single_thread": {w: {"value": v.get("value"), "unit": UNIT, "sample": v.get("sample")}
+                              for w, v in single.items()}}
 
 
 def run_reference(args):
@@ -268,14 +317,17 @@ def run_reference(args):
         if time.perf_counter() - t_start > 170:
             break
     n_layers = layers_of(args.workload)
-    t_token = statistics.mean(times) * H * (L / S) * n_layers
+    t_step = statistics.mean(times)
+    t_token = t_step * H * (L / S) * n_layers
     rate = 1.0 / t_token
     line = {
         "impl": "reference", "metric": METRIC, "value": rate, "unit": UNIT, "n_gpus": args.gpus,
-        "steps": len(times), "warmup": args.warmup, "ms_per_step": t_token * 1e3, "higher_is_better": True,
+        "steps": len(times), "warmup": args.warmup, "ms_per_step": t_step * 1e3,
+        "ms_per_decode_token_scaled": t_token * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": desc, "batch": case.batch, "ctx": L},
-        "cpu_baseline": {"value": rate, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
+        "cpu_baseline": {"value": rate, "unit": UNIT, "cores": BLAS_THREADS, "threads": BLAS_THREADS,
+                         "host_cores": host_cores(), "kind": "oracle",
                          "sample": f"per step one head of one sequence over its first {S} of {L} cached "
                                    f"tokens, scaled x{H} heads x{L / S:.1f} context x{n_layers} layer(s)"
                                    + ("; a whole layer's projections add under 0.2 % to the oracle's "
@@ -418,7 +470,8 @@ def run_gpu_full_layers(args, workload, torch, dist, ws, rank):
             orc.layer_decode(lc, batches=[done])
             done += 1
         dt = time.perf_counter() - t0
-        cpu = {"value": done / dt / n_layers, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
+        cpu = {"value": done / dt / n_layers, "unit": UNIT, "cores": BLAS_THREADS, "threads": BLAS_THREADS,
+               "host_cores": host_cores(), "kind": "oracle",
                "sample": f"the layer oracle on {done} sequence(s) of one layer at full context, {dt:.1f} s "
                          f"(rate / {n_layers} layers)"}
     return {
@@ -445,6 +498,63 @@ def run_gpu_full_layers(args, workload, torch, dist, ws, rank):
         "gpu_launches": steps_arg * (n_layers * 3 + n_layers // lgz),
         "clocks": clk.summary(),
     }
+
+
+def mla_baseline(case, torch, stream, peak, steps=600):
+    """The same workload with the gate off (plain MLA over the same cached
+    latents; the kernel's gate stage and the ids drop out): decode tokens/s of
+    the step (graph over three cache replicas), the decode kernel's CUDA-event
+    time, its roofline fraction and the cache bytes per token."""
+    import dataclasses
+    from paper_2509_16686_gb300 import _lib, device
+    d = dataclasses.replace(case.dims, gate=False)
+    mcase = dataclasses.replace(case, dims=d, name=case.name + "-mla")
+    units = [device.upload(mcase) for _ in range(REPLICAS)]
+    for r in units[1:]:
+        for name in ("w_uk", "w_uv", "workspace", "status", "block_table"):
+            setattr(r, name, getattr(units[0], name))
+    with torch.cuda.stream(stream):
+        for i in range(6):
+            units[i % REPLICAS].step(stream)
+    stream.synchronize()
+    assert units[0].read_status() == 0, "device status (MLA baseline)"
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        for u in units:
+            u.step(stream)
+    reps = max(1, steps // REPLICAS)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        graph.replay()
+        e0.record(stream)
+        for _ in range(reps):
+            graph.replay()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    ms_step = e0.elapsed_time(e1) / (reps * REPLICAS)
+    _lib.eg_mla_profile_begin(3 * REPLICAS)
+    pgraph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(pgraph, stream=stream):
+        for _ in range(3):
+            for u in units:
+                u.step(stream)
+    with torch.cuda.stream(stream):
+        pgraph.replay()
+        pgraph.replay()
+    stream.synchronize()
+    del pgraph
+    ms_sum, n_l = _lib.eg_mla_profile_end()
+    assert units[0].read_status() == 0, "device status (MLA baseline)"
+    k_ms = ms_sum / max(1, n_l)
+    tokens = int(case.seq_lens.astype(np.int64).sum())
+    kvb = (d.d_c + d.d_rope) * (2 if d.dtype == "bf16" else 4)
+    achieved = tokens * kvb / (k_ms * 1e-3) / 1e9
+    del units, graph
+    torch.cuda.empty_cache()
+    return {"what": "the same workload with the gate off (plain MLA over the same latent cache)",
+            "value": case.batch / (ms_step * 1e-3), "unit": UNIT, "ms_per_step": ms_step, "steps": reps * REPLICAS,
+            "decode_kernel_ms": k_ms, "kv_bytes_per_token": kvb,
+            "roofline": {"achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak}}
 
 
 def run_gpu(args, workload, torch, dist, ws, rank):
@@ -501,16 +611,26 @@ def run_gpu(args, workload, torch, dist, ws, rank):
             run_group(groups[i % len(groups)])
     stream.synchronize()
     assert units[0].read_status() == 0, "device status after warm-up"
+    # one graph of a step over every group in turn, replayed whole, and one
+    # graph per group for the remainder, so that exactly `steps_arg` steps run
     graph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(graph, stream=stream):
         for g in groups:
             run_group(g)
+    tail_graphs = []
+    for g in groups[:steps_arg % len(groups)]:
+        tg = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(tg, stream=stream):
+            run_group(g)
+        tail_graphs.append(tg)
     torch.cuda.synchronize()
-    reps = max(1, math.ceil(steps_arg / len(groups)))
-    steps = reps * len(groups)
+    reps = steps_arg // len(groups)
+    steps = reps * len(groups) + len(tail_graphs)
     with torch.cuda.stream(stream):
         for _ in range(2):
             graph.replay()
+        for tg in tail_graphs:
+            tg.replay()
     torch.cuda.synchronize()
 
     # ---- timed region: `steps` steps, barrier + sync on both sides
@@ -523,6 +643,8 @@ def run_gpu(args, workload, torch, dist, ws, rank):
             ev0.record(stream)
             for _ in range(reps):
                 graph.replay()
+            for tg in tail_graphs:
+                tg.replay()
             ev1.record(stream)
         torch.cuda.synchronize()
         if dist:
@@ -612,14 +734,15 @@ def run_gpu(args, workload, torch, dist, ws, rank):
     e2e_value = whole_job_rate(ws, B, e2e_steps, e2e_ms)
     assert units[0].read_status() == 0, "device status after end-to-end run"
 
+    # ---- the gate-off (plain MLA) result of the same workload, beside the gated one
+    mla = None
+    if n_layers == 1 and d.gate and d.dtype == "bf16" and not args.no_mla_baseline and not args.sweep:
+        mla = mla_baseline(case, torch, stream, peak)
+
     # ---- CPU baseline (rank 0, N = 1 only); a decode token passes every layer
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        rate, sample, _ = oracle_sample_rate(case, budget_s=12.0)
-        if n_layers > 1:
-            rate /= n_layers
-            sample += f", one layer of {n_layers} (rate / {n_layers})"
-        cpu = {"value": rate, "unit": UNIT, "cores": host_cores(), "kind": "oracle", "sample": sample}
+        cpu = cpu_baseline_line(case, 12.0, n_layers)
 
     return {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": steps, "warmup": args.warmup,
@@ -637,11 +760,14 @@ def run_gpu(args, workload, torch, dist, ws, rank):
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": steps * launches_per_step,
         "clocks": clk.summary(),
+        "mla_baseline": mla,
     }
 
 
 def main():
     args = parse()
+    if args.oracle_probe:
+        return oracle_probe(args.oracle_probe, args.oracle_budget)
     if args.impl == "reference":
         return run_reference(args)
     import torch

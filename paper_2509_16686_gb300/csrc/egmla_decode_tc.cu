@@ -133,6 +133,7 @@ struct Cfg {
   static constexpr uint32_t COL_S = 0, COL_O = kNB * S_COLS;
   static constexpr uint32_t TMEM_COLS = 256;
   static constexpr uint32_t PAGE_TX = SLOT;
+  static constexpr uint32_t ID_TX = GATE ? kPage * 4 : 0;   // the page's token ids
   static_assert(NS >= 3, "the ring needs three page slots");
   static_assert(SMEM <= kSmemLimit, "shared memory");
   static_assert(D_C == 192 || D_C == 256, "latent widths of this kernel");
@@ -741,18 +742,29 @@ __global__ void __launch_bounds__(kThreads, 1)
           const bool withheld = static_cast<int>(blockIdx.x) == p.stall_cta && it == p.stall_tile;
           if (!withheld) {
             const uint32_t fb = smem_u32(&bars.full[slot]);
-            mbar_arrive_expect_tx(fb, ok ? C::PAGE_TX : 0u);
+            mbar_arrive_expect_tx(fb, ok ? C::PAGE_TX + C::ID_TX : 0u);
             if (ok) {
               const uint32_t dst = sbase + slot * C::SLOT;
               const int y = pg * kPage;
               tma_load_3d(dst, &cmap, 0, y, 0, fb, pol_stream);
               tma_load_2d(dst + C::KR_OFF, &krmap, 0, y, fb, pol_stream);
+              // the page's token ids, into the half of the slot's statistics that
+              // holds r once the gate has read them
+              if (C::ID_TX)
+                bulk_load_hint(sbase + C::OFF_STAT + slot * C::STAT_BYTES + kPage * 4,
+                               p.id_pool + static_cast<size_t>(pg) * kPage, C::ID_TX, fb, pol_stream);
             }
             last_it[slot] = it;
           }
           tr.mark(2, it);
         }
       }
+      // The first page alone: every CTA asks for one page, and the rest only
+      // once it has landed, so that the first pages of all CTAs land early
+      // (one page per SM) instead of in a burst of all their slots.
+      if (it == 0 && lane == 0 && ok_loop && last_it[0] == 0 &&
+          !mbar_wait(smem_u32(&bars.full[0]), 0, abort_flag, wait_ns))
+        ok_loop = false;
       ok_loop = __shfl_sync(0xffffffffu, ok_loop, 0);
       ++it;
     }
@@ -947,8 +959,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     // accesses to the swizzled page still hit eight distinct bank groups (the
     // two rows differ in swizzle parity).  The gate rows come from L2 (the
     // table stays there under an evict-last hint while the cache stream is
-    // evict-first): each tile issues the id loads of the tile two ahead and the
-    // gate-row loads of the next tile, so neither latency sits on the loop.
+    // evict-first).  The token ids come with the page (the producer copies them
+    // into the slot), so the gate rows of the next tile are requested as soon
+    // as its page has landed, while this tile is processed; no load sits on a
+    // chain of dependent global accesses.
     const int gw = warp - kGateWarp0;
     const int pp = lane % kGateLanesPerRow;
     const int row = gw * (32 / kGateLanesPerRow) + lane / kGateLanesPerRow;
@@ -956,16 +970,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     constexpr bool gate_ln = GATE_LN;
     Walker w;
     w.start(p);
-    PageWindow pw;
-    pw.init(p, lane);
-    // id of this thread's row of a tile (0 past the end of the page or for a
-    // bad page, which the producer reports)
-    auto load_id = [&](const Tile& tt) -> int {
-      const int pg = pw.page(p, tt, lane);
-      const int n = (pg >= 0 && pg < p.num_pages) ? tt.ntok : 0;
-      return row < n ? __ldg(p.id_pool + static_cast<size_t>(pg) * kPage + row) : 0;
+    // id of this thread's row of tile jj, from the slot that holds its page (0
+    // past the end of the page)
+    auto slot_id = [&](int jj, const Tile& tt) -> int {
+      const int32_t* ids = reinterpret_cast<const int32_t*>(smem + C::OFF_STAT + (jj % C::NS) * C::STAT_BYTES + kPage * 4);
+      return row < tt.ntok ? ids[row] : 0;
     };
-    auto load_g = [&](int& id, uint4 (&gv)[C::NCH][kGateUnits]) {
+    auto load_g = [&](int id, uint4 (&gv)[C::NCH][kGateUnits]) {
       if ((unsigned)id >= (unsigned)p.vocab) {
         report_status(p.status, kStatusOutOfRange);
         id = 0;
@@ -986,28 +997,35 @@ __global__ void __launch_bounds__(kThreads, 1)
     Tracer tr;
     tr.init(p, 2);
     if (threadIdx.x != kGateWarp0 * 32) tr.base = nullptr;
-    Tile t, t1, t2;
+    Tile t, t1;
     bool have = w.next(t);
     bool have1 = have && w.next(t1);
-    bool have2 = have1 && w.next(t2);
-    int id0 = 0, id1 = 0, id2 = 0;   // ids of tiles j, j + 1, j + 2
     uint4 gcur[C::NCH][kGateUnits], gnext[C::NCH][kGateUnits];
-    if (GATE) {
-      if (have) id0 = load_id(t);
-      if (have1) id1 = load_id(t1);
-      if (have) load_g(id0, gcur);
+    int id0 = 0;
+    if (GATE && have) {
+      // the first tile's rows: its page must land first
+      if (warp_wait(smem_u32(&bars.full[0]), 0, abort_flag, wait_ns)) {
+        id0 = slot_id(0, t);
+        load_g(id0, gcur);
+      } else {
+        have = false;
+      }
     }
     int j = 0;
     while (have) {
       const int slot = j % C::NS;
       tr.mark(0, j);
-      if (GATE) {
-        // prefetch: ids of tile j + 2, gate rows of tile j + 1
-        if (have2) id2 = load_id(t2);
-        if (have1) load_g(id1, gnext);
+      // the next tile's gate rows now if its page has landed, otherwise after this tile
+      bool next_issued = false;
+      int id_next = 0;
+      if (GATE && have1 && warp_test(smem_u32(&bars.full[(j + 1) % C::NS]), ((j + 1) / C::NS) & 1)) {
+        id_next = slot_id(j + 1, t1);
+        load_g(id_next, gnext);
+        next_issued = true;
       }
       if (!warp_wait(smem_u32(&bars.full[slot]), (j / C::NS) & 1, abort_flag, wait_ns)) break;
       tr.mark(1, j);
+      if (DUMP) id0 = slot_id(j, t);
       uint8_t* cpage = smem + slot * C::SLOT;
       if (DUMP) {
         if (row < t.ntok) {
@@ -1160,15 +1178,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         warp_arrive(smem_u32(&bars.zready[slot]));
       }
       tr.mark(3, j);
+      if (GATE && have1 && !next_issued) {
+        // the next page landed only now
+        if (!warp_wait(smem_u32(&bars.full[(j + 1) % C::NS]), ((j + 1) / C::NS) & 1, abort_flag, wait_ns)) break;
+        id_next = slot_id(j + 1, t1);
+        load_g(id_next, gnext);
+      }
       ++j;
       t = t1;
-      t1 = t2;
       have = have1;
-      have1 = have2;
-      have2 = have2 && w.next(t2);
+      have1 = have1 && w.next(t1);
       if (GATE) {
-        id0 = id1;
-        id1 = id2;
 #pragma unroll
         for (int fc = 0; fc < C::NCH; ++fc) {
 #pragma unroll
