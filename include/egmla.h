@@ -210,11 +210,13 @@ int eg_mla_decode(const eg_mla_dims* dims, const void* q, const void* c_pool,
  *     exceeds EG_MLA_STATIC_SCRATCH_BYTES the call returns
  *     EG_MLA_ERR_SCRATCH_LIMIT and launches nothing; use eg_mla_decode with a
  *     workspace, or fewer splits, instead.  The limit covers, for example,
- *     batch 128 at d_c = 512 with 152 splits (about 12 MB).
+ *     batch 128 at d_c = 512 with 301 splits (16,754,944 bytes).
  *   - Start-up: the first call on each device, with that device current,
  *     looks up the array's device address (cudaGetSymbolAddress) and caches
- *     it; make that first call before any stream capture begins.  A failed
- *     lookup returns EG_MLA_ERR_CUDA.
+ *     it with the id of the current context; make that first call before any
+ *     stream capture begins.  After cudaDeviceReset the next call sees a new
+ *     context id and looks the address up again (the same rule applies to
+ *     that call).  A failed lookup returns EG_MLA_ERR_CUDA.
  *   - Zeroing: no part of the scratch needs to start at zero (every word the
  *     kernels read from it is written earlier in the same call), so the call
  *     runs no clearing pass.  *dev_status is the caller's, zeroed by the

@@ -255,23 +255,59 @@ static __device__ __align__(256) unsigned char g_static_scratch[EG_MLA_STATIC_SC
 
 constexpr int kMaxDevices = 64;
 
-// device address of g_static_scratch, looked up once per device with that
-// device current (the lookup may load the module, so the first call belongs
-// before any stream capture)
+// device address of g_static_scratch, looked up with the device current and
+// cached together with the id of the context it belongs to: a context made
+// after cudaDeviceReset gets a new id (and possibly a new address), so the
+// first call in it looks the address up again.  A lookup may load the module,
+// so the first call in each context belongs before any stream capture.
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+
 struct StaticScratch {
   std::mutex mu;
   void* ptr[kMaxDevices] = {};
+  unsigned long long ctx_id[kMaxDevices] = {};
+  CtxGetCurrentFn get_current = nullptr;
+  CtxGetIdFn get_id = nullptr;
+  bool resolved = false;
 } g_static;
+
+template <typename Fn>
+Fn driver_fn(const char* name) {
+  void* p = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion(name, &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+      q != cudaDriverEntryPointSuccess)
+    return nullptr;
+  return reinterpret_cast<Fn>(p);
+}
 
 int static_scratch(void** out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return EG_MLA_ERR_CUDA;
   if (dev < 0 || dev >= kMaxDevices) return EG_MLA_ERR_UNSUPPORTED;
   std::lock_guard<std::mutex> lk(g_static.mu);
-  if (g_static.ptr[dev] == nullptr) {
+  if (!g_static.resolved) {
+    g_static.get_current = driver_fn<CtxGetCurrentFn>("cuCtxGetCurrent");
+    g_static.get_id = driver_fn<CtxGetIdFn>("cuCtxGetId");
+    g_static.resolved = true;
+  }
+  if (g_static.get_current == nullptr || g_static.get_id == nullptr) return EG_MLA_ERR_CUDA;
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (g_static.get_current(&ctx) != CUDA_SUCCESS) return EG_MLA_ERR_CUDA;
+  if (ctx == nullptr) {
+    // no context on this thread yet: have the runtime make the device's
+    // primary context current
+    if (cudaFree(nullptr) != cudaSuccess || g_static.get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr)
+      return EG_MLA_ERR_CUDA;
+  }
+  if (g_static.get_id(ctx, &id) != CUDA_SUCCESS) return EG_MLA_ERR_CUDA;
+  if (g_static.ptr[dev] == nullptr || g_static.ctx_id[dev] != id) {
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || p == nullptr) return EG_MLA_ERR_CUDA;
     g_static.ptr[dev] = p;
+    g_static.ctx_id[dev] = id;
   }
   *out = g_static.ptr[dev];
   return EG_MLA_OK;

@@ -976,12 +976,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int32_t* ids = reinterpret_cast<const int32_t*>(smem + C::OFF_STAT + (jj % C::NS) * C::STAT_BYTES + kPage * 4);
       return row < tt.ntok ? ids[row] : 0;
     };
-    auto load_g = [&](int id, uint4 (&gv)[C::NCH][kGateUnits]) {
+    // this thread's part of the gate row of token id (row 0, reported, for an
+    // id outside the vocabulary)
+    auto g_row = [&](int id) -> const __nv_bfloat16* {
       if ((unsigned)id >= (unsigned)p.vocab) {
         report_status(p.status, kStatusOutOfRange);
         id = 0;
       }
-      const __nv_bfloat16* src = p.gate_table + static_cast<size_t>(id) * D_C + pp * 8 * kGateUnits;
+      return p.gate_table + static_cast<size_t>(id) * D_C + pp * 8 * kGateUnits;
+    };
+    auto load_g = [&](int id, uint4 (&gv)[C::NCH][kGateUnits]) {
+      const __nv_bfloat16* src = g_row(id);
 #pragma unroll
       for (int fc = 0; fc < C::NCH; ++fc) {
         if constexpr (kGateUnits == 2)
@@ -1015,14 +1020,23 @@ __global__ void __launch_bounds__(kThreads, 1)
     while (have) {
       const int slot = j % C::NS;
       tr.mark(0, j);
-      // the next tile's gate rows now if its page has landed, otherwise after this tile
+      // The next tile's gate rows: if its page has landed, requested column by
+      // column between this tile's shared-memory stores (spreading the loads
+      // over the tile instead of one burst), otherwise after this tile.
       bool next_issued = false;
-      int id_next = 0;
+      const __nv_bfloat16* gsrc_next = p.gate_table;
       if (GATE && have1 && warp_test(smem_u32(&bars.full[(j + 1) % C::NS]), ((j + 1) / C::NS) & 1)) {
-        id_next = slot_id(j + 1, t1);
-        load_g(id_next, gnext);
+        gsrc_next = g_row(slot_id(j + 1, t1));
         next_issued = true;
       }
+      auto load_next_column = [&](int fc) {
+        if (next_issued) {
+          if constexpr (kGateUnits == 2)
+            ldg_32_na_hint(gsrc_next + fc * 64, pol_keep, gnext[fc][0], gnext[fc][1]);
+          else
+            gnext[fc][0] = ldg_16_na_hint(gsrc_next + fc * 64, pol_keep);
+        }
+      };
       if (!warp_wait(smem_u32(&bars.full[slot]), (j / C::NS) & 1, abort_flag, wait_ns)) break;
       tr.mark(1, j);
       if (DUMP) id0 = slot_id(j, t);
@@ -1046,6 +1060,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 cpage + C::KR_OFF + row * 128 + (((kGateUnits * pp + h) ^ (row & 7)) << 4));
           if (pp == 0) p.dump_ids[o] = id0;
         }
+#pragma unroll
+        for (int fc = 0; fc < C::NCH; ++fc) load_next_column(fc);
         warp_arrive(smem_u32(&bars.empty[slot]));
       } else {
         const bool full_page = t.ntok == kPage;   // uniform: no token masking needed
@@ -1107,6 +1123,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (!full_page && !valid) z = make_uint4(0, 0, 0, 0);
                 *reinterpret_cast<uint4*>(cpage + unit_off(fc, h)) = z;
               }
+              load_next_column(fc);
             }
             tr.mark(6, j);
             if (pp == 0) {
@@ -1140,6 +1157,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 a2 = __ffma2_rn(f3, f3, a2);
                 *reinterpret_cast<uint4*>(cpage + unit_off(fc, h)) = z;
               }
+              load_next_column(fc);
             }
             s1 = __fadd2_rn(s1, a1);
             s2 = __fadd2_rn(s2, a2);
@@ -1181,8 +1199,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (GATE && have1 && !next_issued) {
         // the next page landed only now
         if (!warp_wait(smem_u32(&bars.full[(j + 1) % C::NS]), ((j + 1) / C::NS) & 1, abort_flag, wait_ns)) break;
-        id_next = slot_id(j + 1, t1);
-        load_g(id_next, gnext);
+        load_g(slot_id(j + 1, t1), gnext);
       }
       ++j;
       t = t1;
