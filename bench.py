@@ -492,10 +492,10 @@ def run_gpu_full_layers(args, workload, torch, dist, ws, rank):
         "cpu_baseline": cpu,
         "e2e": {"value": whole_job_rate(ws, B, e2e_steps, e2e_ms), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
-        # this library's kernels per layer: kv_norm + RoPE, append (first layer of
-        # a group only), query absorption, decode (the projection GEMMs are cuBLAS
-        # kernels, not counted)
-        "gpu_launches": steps_arg * (n_layers * 3 + n_layers // lgz),
+        # this library's kernels per layer: kv_norm + RoPE, query absorption
+        # (with the append in its grid in the first layer of a group), decode
+        # (the projection GEMMs are cuBLAS kernels, not counted)
+        "gpu_launches": steps_arg * n_layers * 3,
         "clocks": clk.summary(),
     }
 
@@ -596,10 +596,11 @@ def run_gpu(args, workload, torch, dist, ws, rank):
     cache_bytes = tokens_cached * ((d.d_c + d.d_rope) * elem + id_bytes)     # per unit (layer)
     splits = units[0].num_splits or _lib.eg_mla_default_num_splits()
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
-    # append + prologue + decode, + the combine kernel unless the decode kernel
-    # runs fused (bf16, d_c 192/256, a grid of at most one CTA per SM)
+    # bf16: query absorption (with the append in its grid) + decode, + the
+    # combine kernel unless the decode kernel runs fused (d_c 192/256, a grid
+    # of at most one CTA per SM); fp32: append + decode + combine
     fused = d.dtype == "bf16" and d.d_c in (192, 256) and splits <= sms
-    launches_per_step = n_layers * (3 if fused else 4)
+    launches_per_step = n_layers * ((2 if fused else 3) if d.dtype == "bf16" else 3)
 
     def run_group(g):
         for u in g:

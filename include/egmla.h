@@ -189,6 +189,33 @@ int eg_mla_decode(const eg_mla_dims* dims, const void* q, const void* c_pool,
                   int32_t num_splits, void* workspace, size_t workspace_bytes,
                   int32_t* dev_status, void* stream);
 
+/*
+ * eg_mla_step - one decode step: eg_mla_append_latent, then eg_mla_decode, in
+ * one call (the method's decode step: the new token is cached, Appendix C
+ * Eq. 1 and Eq. 10, and attends over the cache including itself, Eq. 13).
+ *
+ * Arguments: the union of the two calls', with the same meaning, layout,
+ * ownership and alignment rules (c_new, krope_new, ids_new and positions as
+ * for eg_mla_append_latent; seq_lens must already count the new token).
+ * Results: bit-identical to eg_mla_append_latent followed by eg_mla_decode on
+ * the same stream with the same arguments.  Every argument of both parts is
+ * checked before anything is launched; host errors return the same codes as
+ * the two calls, device errors go to *dev_status.
+ *
+ * On the bf16 path the append runs inside the grid of the query-absorption
+ * kernel (which reads no pool), one launch fewer per step; the split-KV
+ * kernel starts its setup while that kernel finishes and waits for its
+ * completion before it reads the cache.
+ */
+int eg_mla_step(const eg_mla_dims* dims, void* c_pool, void* krope_pool, int32_t* id_pool,
+                const void* c_new, const void* krope_new, const int32_t* ids_new,
+                const int32_t* positions, const void* q, const int32_t* block_table,
+                int32_t max_pages_per_seq, const int32_t* seq_lens, int32_t max_seq_len,
+                int32_t batch, int32_t num_pages, const void* gate_table,
+                const float* ln_gamma, const float* ln_beta, const void* w_uk,
+                const void* w_uv, void* out, int32_t num_splits, void* workspace,
+                size_t workspace_bytes, int32_t* dev_status, void* stream);
+
 /* Size of the static device scratch array behind eg_mla_decode_static. */
 #define EG_MLA_STATIC_SCRATCH_BYTES ((size_t)16 << 20)
 

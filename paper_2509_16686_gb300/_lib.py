@@ -42,6 +42,7 @@ EXPORTED = [
     "eg_mla_decode_workspace_size",
     "eg_mla_decode",
     "eg_mla_decode_static",
+    "eg_mla_step",
     "eg_mla_kv_bytes_per_token",
     "eg_mla_status_string",
     "eg_mla_debug_gather",
@@ -94,6 +95,9 @@ def _declare(lib: ctypes.CDLL) -> None:
     lib.eg_mla_decode.restype = ctypes.c_int
     lib.eg_mla_decode_static.argtypes = [D, P, P, P, P, P, I32, P, I32, I32, I32, P, P, P, P, P, P, I32, P, P]
     lib.eg_mla_decode_static.restype = ctypes.c_int
+    lib.eg_mla_step.argtypes = [D, P, P, P, P, P, P, P, P, P, I32, P, I32, I32, I32, P, P, P, P, P, P, I32, P, SZ,
+                                P, P]
+    lib.eg_mla_step.restype = ctypes.c_int
     lib.eg_mla_kv_bytes_per_token.argtypes = [D, I32, ctypes.POINTER(ctypes.c_int64)]
     lib.eg_mla_kv_bytes_per_token.restype = ctypes.c_int
     lib.eg_mla_status_string.argtypes = [ctypes.c_int]
@@ -224,6 +228,26 @@ def eg_mla_decode(dims: EgMlaDims, q, c_pool, krope_pool, id_pool, block_table, 
     _check(code, "eg_mla_decode")
 
 
+def _step_args(dims, c_pool, krope_pool, id_pool, c_new, krope_new, ids_new, positions, q, block_table, seq_lens,
+               max_seq_len, gate_table, ln_gamma, ln_beta, w_uk, w_uv, out, workspace, num_splits, dev_status,
+               stream):
+    return (ctypes.byref(dims), _ptr(c_pool), _ptr(krope_pool), _ptr(id_pool), _ptr(c_new), _ptr(krope_new),
+            _ptr(ids_new), _ptr(positions), _ptr(q), _ptr(block_table), block_table.shape[1], _ptr(seq_lens),
+            int(max_seq_len), seq_lens.shape[0], c_pool.shape[0], _ptr(gate_table), _ptr(ln_gamma), _ptr(ln_beta),
+            _ptr(w_uk), _ptr(w_uv), _ptr(out), num_splits, _ptr(workspace),
+            workspace.numel() * workspace.element_size(), _ptr(dev_status), _stream(stream))
+
+
+def eg_mla_step(dims: EgMlaDims, c_pool, krope_pool, id_pool, c_new, krope_new, ids_new, positions, q, block_table,
+                seq_lens, max_seq_len, gate_table, ln_gamma, ln_beta, w_uk, w_uv, out, workspace, num_splits=0,
+                dev_status=None, stream=None) -> None:
+    """eg_mla_append_latent followed by eg_mla_decode, as one C call."""
+    _check(load().eg_mla_step(*_step_args(dims, c_pool, krope_pool, id_pool, c_new, krope_new, ids_new, positions,
+                                          q, block_table, seq_lens, max_seq_len, gate_table, ln_gamma, ln_beta,
+                                          w_uk, w_uv, out, workspace, num_splits, dev_status, stream)),
+           "eg_mla_step")
+
+
 def eg_mla_decode_static(dims: EgMlaDims, q, c_pool, krope_pool, id_pool, block_table, seq_lens, max_seq_len,
                          gate_table, ln_gamma, ln_beta, w_uk, w_uv, out, num_splits=0,
                          dev_status=None, stream=None) -> None:
@@ -277,30 +301,20 @@ def eg_mla_layer_decode(dims: EgMlaDims, layer: EgMlaLayerDims, weights: EgMlaLa
 def bind_step(dims: EgMlaDims, c_pool, krope_pool, id_pool, c_new, krope_new, ids_new, positions, q, block_table,
               seq_lens, max_seq_len, gate_table, ln_gamma, ln_beta, w_uk, w_uv, out, workspace, num_splits=0,
               dev_status=None, stream=None):
-    """One decode step (eg_mla_append_latent, then eg_mla_decode) with every
-    argument converted once: returns a callable that issues both C calls on
-    `stream` with those pointers.  The tensors must stay alive and in place
-    while the callable is used; a caller that reruns the same step every token
-    saves the per-call argument marshalling."""
-    lib = load()
-    d = ctypes.byref(dims)
-    st = _stream(stream)
-    append_args = (d, _ptr(c_pool), _ptr(krope_pool), _ptr(id_pool), _ptr(c_new), _ptr(krope_new), _ptr(ids_new),
-                   _ptr(block_table), block_table.shape[1], _ptr(positions), positions.shape[0], c_pool.shape[0],
-                   _ptr(dev_status), st)
-    decode_args = (d, _ptr(q), _ptr(c_pool), _ptr(krope_pool), _ptr(id_pool), _ptr(block_table),
-                   block_table.shape[1], _ptr(seq_lens), int(max_seq_len), seq_lens.shape[0], c_pool.shape[0],
-                   _ptr(gate_table), _ptr(ln_gamma), _ptr(ln_beta), _ptr(w_uk), _ptr(w_uv), _ptr(out), num_splits,
-                   _ptr(workspace), workspace.numel() * workspace.element_size(), _ptr(dev_status), st)
-    append_fn, decode_fn = lib.eg_mla_append_latent, lib.eg_mla_decode
+    """One decode step (eg_mla_step: append, then decode) with every argument
+    converted once: returns a callable that issues the C call on `stream` with
+    those pointers.  The tensors must stay alive and in place while the
+    callable is used; a caller that reruns the same step every token saves the
+    per-call argument marshalling."""
+    fn = load().eg_mla_step
+    args = _step_args(dims, c_pool, krope_pool, id_pool, c_new, krope_new, ids_new, positions, q, block_table,
+                      seq_lens, max_seq_len, gate_table, ln_gamma, ln_beta, w_uk, w_uv, out, workspace, num_splits,
+                      dev_status, stream)
 
     def step() -> None:
-        rc = append_fn(*append_args)
+        rc = fn(*args)
         if rc != EG_MLA_OK:
-            raise EgMlaError(rc, "eg_mla_append_latent")
-        rc = decode_fn(*decode_args)
-        if rc != EG_MLA_OK:
-            raise EgMlaError(rc, "eg_mla_decode")
+            raise EgMlaError(rc, "eg_mla_step")
 
     step.keepalive = (dims, c_pool, krope_pool, id_pool, c_new, krope_new, ids_new, positions, q, block_table,
                       seq_lens, gate_table, ln_gamma, ln_beta, w_uk, w_uv, out, workspace, dev_status)

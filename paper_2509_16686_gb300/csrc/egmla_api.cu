@@ -313,6 +313,85 @@ int static_scratch(void** out) {
   return EG_MLA_OK;
 }
 
+// argument checks and launch record of one append (eg_mla_append_latent)
+int fill_append_args(egmla::AppendArgs& a, const eg_mla_dims* dims, void* c_pool, void* krope_pool,
+                     int32_t* id_pool, const void* c_new, const void* krope_new, const int32_t* ids_new,
+                     const int32_t* block_table, int32_t max_pages_per_seq, const int32_t* positions,
+                     int32_t batch, int32_t num_pages, int32_t* dev_status) {
+  int rc = check_dims(dims);
+  if (rc != EG_MLA_OK) return rc;
+  if (batch < 0 || num_pages <= 0 || max_pages_per_seq <= 0) return EG_MLA_ERR_INVALID_ARG;
+  std::memset(&a, 0, sizeof(a));
+  if (batch == 0) return EG_MLA_OK;
+  if (!c_pool || !krope_pool || !c_new || !krope_new || !block_table || !positions) return EG_MLA_ERR_INVALID_ARG;
+  const int eb = elem_bytes(dims);
+  const int crb = dims->d_c * eb, krb = dims->d_rope * eb;
+  if (crb % 16 || krb % 16) return EG_MLA_ERR_UNSUPPORTED;
+  if (!aligned(c_pool, 16) || !aligned(krope_pool, 16) || !aligned(c_new, 16) || !aligned(krope_new, 16))
+    return EG_MLA_ERR_INVALID_ARG;
+  a.c_pool = c_pool;
+  a.kr_pool = krope_pool;
+  a.id_pool = id_pool;
+  a.c_new = c_new;
+  a.kr_new = krope_new;
+  a.ids_new = ids_new;
+  a.block_table = block_table;
+  a.max_pages = max_pages_per_seq;
+  a.positions = positions;
+  a.batch = batch;
+  a.num_pages = num_pages;
+  a.page_size = dims->page_size;
+  a.c_row_bytes = crb;
+  a.kr_row_bytes = krb;
+  a.status = dev_status;
+  return EG_MLA_OK;
+}
+
+// eg_mla_decode, preceded by the append of `app` when it is non-null (in the
+// query-absorption kernel's grid on the tensor-core path; as its own launch
+// otherwise).  Every argument is checked before anything is launched.
+int decode_impl(const eg_mla_dims* dims, const void* q, const void* c_pool, const void* krope_pool,
+                const int32_t* id_pool, const int32_t* block_table, int32_t max_pages_per_seq,
+                const int32_t* seq_lens, int32_t max_seq_len, int32_t batch, int32_t num_pages,
+                const void* gate_table, const float* ln_gamma, const float* ln_beta, const void* w_uk,
+                const void* w_uv, void* out, int32_t num_splits, void* workspace, size_t workspace_bytes,
+                int32_t* dev_status, const egmla::AppendArgs* app, cudaStream_t st) {
+  DecodeArgs a;
+  int rc = fill_decode_args(a, dims, c_pool, krope_pool, id_pool, block_table, max_pages_per_seq, seq_lens,
+                            max_seq_len, batch, num_pages, gate_table, num_splits, workspace, workspace_bytes,
+                            dev_status);
+  if (rc != EG_MLA_OK) return rc;
+  if (batch == 0) return EG_MLA_OK;
+  if (q == nullptr || w_uk == nullptr || w_uv == nullptr || out == nullptr) return EG_MLA_ERR_INVALID_ARG;
+  // q, W_UK and W_UV rows are read in 16-byte pieces
+  if (!aligned(w_uv, 16) || !aligned(w_uk, 16) || !aligned(q, 16)) return EG_MLA_ERR_INVALID_ARG;
+  a.q = q;
+  a.ln_gamma = ln_gamma;
+  a.ln_beta = ln_beta;
+  a.w_uk = w_uk;
+  a.w_uv = w_uv;
+  a.out = out;
+  if (is_tc_path(dims)) {
+    CUtensorMap maps[2];
+    if (!encode_decode_maps(maps, dims, c_pool, krope_pool, num_pages)) return EG_MLA_ERR_CUDA;
+    apply_trace(a);
+    apply_fault(a);
+    cudaError_t e = egmla::launch_prologue_tc(a, app, st);
+    bool fused = false;
+    if (e == cudaSuccess) {
+      prof_mark(st, true);
+      e = egmla::launch_decode_tc(a, maps, false, st, &fused);
+      prof_mark(st, false);
+    }
+    if (e == cudaSuccess && !fused) e = egmla::launch_combine(a, true, st);
+    return to_status(e);
+  }
+  cudaError_t e = app != nullptr ? egmla::launch_append(*app, st) : cudaSuccess;
+  if (e == cudaSuccess) e = egmla::launch_decode_f32(a, st);
+  if (e == cudaSuccess) e = egmla::launch_combine(a, false, st);
+  return to_status(e);
+}
+
 }  // namespace
 
 extern "C" {
@@ -357,32 +436,10 @@ int eg_mla_append_latent(const eg_mla_dims* dims, void* c_pool, void* krope_pool
                          const void* c_new, const void* krope_new, const int32_t* ids_new,
                          const int32_t* block_table, int32_t max_pages_per_seq, const int32_t* positions,
                          int32_t batch, int32_t num_pages, int32_t* dev_status, void* stream) {
-  int rc = check_dims(dims);
-  if (rc != EG_MLA_OK) return rc;
-  if (batch < 0 || num_pages <= 0 || max_pages_per_seq <= 0) return EG_MLA_ERR_INVALID_ARG;
-  if (batch == 0) return EG_MLA_OK;
-  if (!c_pool || !krope_pool || !c_new || !krope_new || !block_table || !positions) return EG_MLA_ERR_INVALID_ARG;
-  const int eb = elem_bytes(dims);
-  const int crb = dims->d_c * eb, krb = dims->d_rope * eb;
-  if (crb % 16 || krb % 16) return EG_MLA_ERR_UNSUPPORTED;
-  if (!aligned(c_pool, 16) || !aligned(krope_pool, 16) || !aligned(c_new, 16) || !aligned(krope_new, 16))
-    return EG_MLA_ERR_INVALID_ARG;
   egmla::AppendArgs a;
-  a.c_pool = c_pool;
-  a.kr_pool = krope_pool;
-  a.id_pool = id_pool;
-  a.c_new = c_new;
-  a.kr_new = krope_new;
-  a.ids_new = ids_new;
-  a.block_table = block_table;
-  a.max_pages = max_pages_per_seq;
-  a.positions = positions;
-  a.batch = batch;
-  a.num_pages = num_pages;
-  a.page_size = dims->page_size;
-  a.c_row_bytes = crb;
-  a.kr_row_bytes = krb;
-  a.status = dev_status;
+  const int rc = fill_append_args(a, dims, c_pool, krope_pool, id_pool, c_new, krope_new, ids_new, block_table,
+                                  max_pages_per_seq, positions, batch, num_pages, dev_status);
+  if (rc != EG_MLA_OK || batch == 0) return rc;
   return to_status(egmla::launch_append(a, static_cast<cudaStream_t>(stream)));
 }
 
@@ -392,40 +449,24 @@ int eg_mla_decode(const eg_mla_dims* dims, const void* q, const void* c_pool, co
                   const void* gate_table, const float* ln_gamma, const float* ln_beta, const void* w_uk,
                   const void* w_uv, void* out, int32_t num_splits, void* workspace, size_t workspace_bytes,
                   int32_t* dev_status, void* stream) {
-  DecodeArgs a;
-  int rc = fill_decode_args(a, dims, c_pool, krope_pool, id_pool, block_table, max_pages_per_seq, seq_lens,
-                            max_seq_len, batch, num_pages, gate_table, num_splits, workspace, workspace_bytes,
-                            dev_status);
+  return decode_impl(dims, q, c_pool, krope_pool, id_pool, block_table, max_pages_per_seq, seq_lens, max_seq_len,
+                     batch, num_pages, gate_table, ln_gamma, ln_beta, w_uk, w_uv, out, num_splits, workspace,
+                     workspace_bytes, dev_status, nullptr, static_cast<cudaStream_t>(stream));
+}
+
+int eg_mla_step(const eg_mla_dims* dims, void* c_pool, void* krope_pool, int32_t* id_pool, const void* c_new,
+                const void* krope_new, const int32_t* ids_new, const int32_t* positions, const void* q,
+                const int32_t* block_table, int32_t max_pages_per_seq, const int32_t* seq_lens,
+                int32_t max_seq_len, int32_t batch, int32_t num_pages, const void* gate_table,
+                const float* ln_gamma, const float* ln_beta, const void* w_uk, const void* w_uv, void* out,
+                int32_t num_splits, void* workspace, size_t workspace_bytes, int32_t* dev_status, void* stream) {
+  egmla::AppendArgs app;
+  const int rc = fill_append_args(app, dims, c_pool, krope_pool, id_pool, c_new, krope_new, ids_new, block_table,
+                                  max_pages_per_seq, positions, batch, num_pages, dev_status);
   if (rc != EG_MLA_OK) return rc;
-  if (batch == 0) return EG_MLA_OK;
-  if (q == nullptr || w_uk == nullptr || w_uv == nullptr || out == nullptr) return EG_MLA_ERR_INVALID_ARG;
-  // q, W_UK and W_UV rows are read in 16-byte pieces
-  if (!aligned(w_uv, 16) || !aligned(w_uk, 16) || !aligned(q, 16)) return EG_MLA_ERR_INVALID_ARG;
-  a.q = q;
-  a.ln_gamma = ln_gamma;
-  a.ln_beta = ln_beta;
-  a.w_uk = w_uk;
-  a.w_uv = w_uv;
-  a.out = out;
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
-  if (is_tc_path(dims)) {
-    CUtensorMap maps[2];
-    if (!encode_decode_maps(maps, dims, c_pool, krope_pool, num_pages)) return EG_MLA_ERR_CUDA;
-    apply_trace(a);
-    apply_fault(a);
-    cudaError_t e = egmla::launch_prologue_tc(a, st);
-    bool fused = false;
-    if (e == cudaSuccess) {
-      prof_mark(st, true);
-      e = egmla::launch_decode_tc(a, maps, false, st, &fused);
-      prof_mark(st, false);
-    }
-    if (e == cudaSuccess && !fused) e = egmla::launch_combine(a, true, st);
-    return to_status(e);
-  }
-  cudaError_t e = egmla::launch_decode_f32(a, st);
-  if (e == cudaSuccess) e = egmla::launch_combine(a, false, st);
-  return to_status(e);
+  return decode_impl(dims, q, c_pool, krope_pool, id_pool, block_table, max_pages_per_seq, seq_lens, max_seq_len,
+                     batch, num_pages, gate_table, ln_gamma, ln_beta, w_uk, w_uv, out, num_splits, workspace,
+                     workspace_bytes, dev_status, &app, static_cast<cudaStream_t>(stream));
 }
 
 int eg_mla_decode_static(const eg_mla_dims* dims, const void* q, const void* c_pool, const void* krope_pool,
@@ -540,7 +581,7 @@ int eg_mla_debug_gather(const eg_mla_dims* dims, const void* c_pool, const void*
   CUtensorMap maps[2];
   if (!encode_decode_maps(maps, dims, c_pool, krope_pool, num_pages)) return EG_MLA_ERR_CUDA;
   a.q = nullptr;  // prologue computes the page prefix sums only
-  cudaError_t e = egmla::launch_prologue_tc(a, st);
+  cudaError_t e = egmla::launch_prologue_tc(a, nullptr, st);
   if (e == cudaSuccess) e = egmla::launch_decode_tc(a, maps, true, st, nullptr);
   return to_status(e);
 }

@@ -12,6 +12,7 @@
 
 #include <cmath>
 #include <cstdint>
+#include <cstring>
 
 #include "egmla_common.cuh"
 #include "egmla_kernels.h"
@@ -20,39 +21,36 @@
 namespace egmla {
 
 // ------------------------------------------------------------------ append
-// One block per sequence; the row copies are 16-byte vectors when the row
-// byte counts allow it (they do for every supported shape).
-__global__ void append_latent_kernel(uint8_t* __restrict__ c_pool, uint8_t* __restrict__ kr_pool,
-                                     int32_t* __restrict__ id_pool, const uint8_t* __restrict__ c_new,
-                                     const uint8_t* __restrict__ kr_new,
-                                     const int32_t* __restrict__ ids_new,
-                                     const int32_t* __restrict__ block_table, int max_pages,
-                                     const int32_t* __restrict__ positions, int num_pages, int page_size,
-                                     int c_row_bytes, int kr_row_bytes, int32_t* status) {
-  const int b = blockIdx.x;
-  const int pos = positions[b];
+// The new token's rows of sequence b, copied by the calling block; the row
+// copies are 16-byte vectors (the row byte counts allow it for every
+// supported shape).
+__device__ void append_row(const AppendArgs& a, int b) {
+  const int pos = a.positions[b];
   if (pos < 0) return;
-  const int lp = pos / page_size;
-  if (lp >= max_pages) {
-    if (threadIdx.x == 0) report_status(status, kStatusOutOfRange);
+  const int lp = pos / a.page_size;
+  if (lp >= a.max_pages) {
+    if (threadIdx.x == 0) report_status(a.status, kStatusOutOfRange);
     return;
   }
-  const int page = block_table[static_cast<size_t>(b) * max_pages + lp];
-  if (page < 0 || page >= num_pages) {
-    if (threadIdx.x == 0) report_status(status, kStatusOutOfRange);
+  const int page = a.block_table[static_cast<size_t>(b) * a.max_pages + lp];
+  if (page < 0 || page >= a.num_pages) {
+    if (threadIdx.x == 0) report_status(a.status, kStatusOutOfRange);
     return;
   }
-  const size_t row = static_cast<size_t>(page) * page_size + pos % page_size;
-  uint8_t* cd = c_pool + row * c_row_bytes;
-  const uint8_t* cs = c_new + static_cast<size_t>(b) * c_row_bytes;
-  for (int i = threadIdx.x; i < c_row_bytes / 16; i += blockDim.x)
-    reinterpret_cast<uint4*>(cd)[i] = reinterpret_cast<const uint4*>(cs)[i];
-  uint8_t* kd = kr_pool + row * kr_row_bytes;
-  const uint8_t* ks = kr_new + static_cast<size_t>(b) * kr_row_bytes;
-  for (int i = threadIdx.x; i < kr_row_bytes / 16; i += blockDim.x)
-    reinterpret_cast<uint4*>(kd)[i] = reinterpret_cast<const uint4*>(ks)[i];
-  if (id_pool != nullptr && ids_new != nullptr && threadIdx.x == 0) id_pool[row] = ids_new[b];
+  const size_t row = static_cast<size_t>(page) * a.page_size + pos % a.page_size;
+  uint4* cd = reinterpret_cast<uint4*>(static_cast<uint8_t*>(a.c_pool) + row * a.c_row_bytes);
+  const uint4* cs = reinterpret_cast<const uint4*>(static_cast<const uint8_t*>(a.c_new) +
+                                                   static_cast<size_t>(b) * a.c_row_bytes);
+  for (int i = threadIdx.x; i < a.c_row_bytes / 16; i += blockDim.x) cd[i] = cs[i];
+  uint4* kd = reinterpret_cast<uint4*>(static_cast<uint8_t*>(a.kr_pool) + row * a.kr_row_bytes);
+  const uint4* ks = reinterpret_cast<const uint4*>(static_cast<const uint8_t*>(a.kr_new) +
+                                                   static_cast<size_t>(b) * a.kr_row_bytes);
+  for (int i = threadIdx.x; i < a.kr_row_bytes / 16; i += blockDim.x) kd[i] = ks[i];
+  if (a.id_pool != nullptr && a.ids_new != nullptr && threadIdx.x == 0) a.id_pool[row] = a.ids_new[b];
 }
+
+// one block per sequence
+__global__ void append_latent_kernel(const AppendArgs a) { append_row(a, blockIdx.x); }
 
 // ------------------------------------------------------------------ helpers
 // eight bf16 (or four fp32) of a 16-byte piece as floats
@@ -160,7 +158,7 @@ __global__ void prologue_tc_kernel(const __nv_bfloat16* __restrict__ q, const __
                        const int32_t* __restrict__ seq_lens, int batch, int d_nope, int d_rope, int d_c,
                        int page_size, uint8_t* __restrict__ qprep, size_t qstride, int32_t* __restrict__ cu,
                        uint32_t* __restrict__ seq_done, int num_splits, const int32_t* __restrict__ block_table,
-                       int max_pages, SplitStart* __restrict__ starts) {
+                       int max_pages, SplitStart* __restrict__ starts, const AppendArgs app) {
   __shared__ __align__(16) __nv_bfloat16 ws[kPMaxNope][kSumFeatures];  // W_UK,h[n][f0 + f]
   __shared__ __align__(16) __nv_bfloat16 qs[kPBatch][kPMaxNope];      // q^C_{b0 + j, h}[n]
   // partial sums [n part * 4 quads + j][f], written once every warp is done with ws
@@ -169,6 +167,15 @@ __global__ void prologue_tc_kernel(const __nv_bfloat16* __restrict__ q, const __
   constexpr int H = 16;
   const int nchunk = d_c / kSumFeatures;
   const int ngroups = (batch + kPBatch - 1) / kPBatch;
+  // the decode kernel after this one may begin its setup (it waits for this
+  // kernel's completion before it reads anything written here)
+  grid_launch_dependents();
+  if (blockIdx.x > static_cast<unsigned>(H * nchunk * ngroups)) {
+    // blocks after the schedule block: the new token of one sequence (a step
+    // that appends before it attends); no block of this kernel reads the pools
+    append_row(app, blockIdx.x - (H * nchunk * ngroups + 1));
+    return;
+  }
   if (blockIdx.x == static_cast<unsigned>(H * nchunk * ngroups)) {
     if (seq_done != nullptr)
       for (int i = threadIdx.x; i <= batch; i += blockDim.x) seq_done[i] = 0u;
@@ -583,25 +590,25 @@ decode_f32_kernel(const float* __restrict__ c_pool, const float* __restrict__ kr
 // ------------------------------------------------------------------ launchers
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t st) {
   if (a.batch == 0) return cudaSuccess;
-  append_latent_kernel<<<a.batch, 64, 0, st>>>(
-      static_cast<uint8_t*>(a.c_pool), static_cast<uint8_t*>(a.kr_pool), a.id_pool,
-      static_cast<const uint8_t*>(a.c_new), static_cast<const uint8_t*>(a.kr_new), a.ids_new, a.block_table,
-      a.max_pages, a.positions, a.num_pages, a.page_size, a.c_row_bytes, a.kr_row_bytes, a.status);
+  append_latent_kernel<<<a.batch, 64, 0, st>>>(a);
   return cudaGetLastError();
 }
 
-cudaError_t launch_prologue_tc(const DecodeArgs& a, cudaStream_t st) {
+cudaError_t launch_prologue_tc(const DecodeArgs& a, const AppendArgs* app, cudaStream_t st) {
   const WorkspaceLayout wl = workspace_layout(a.batch, a.num_splits, 16, a.d_c, a.d_rope, true);
   uint8_t* ws = static_cast<uint8_t*>(a.workspace);
   // with the gate off the latent is used as cached: no LayerNorm affine to fold into q^
   const float* gamma = a.gate && a.gate_ln ? a.ln_gamma : nullptr;
   const float* beta = a.gate && a.gate_ln ? a.ln_beta : nullptr;
   const int ngroups = (a.batch + kPBatch - 1) / kPBatch;
-  prologue_tc_kernel<<<16 * (a.d_c / kSumFeatures) * ngroups + 1, 256, 0, st>>>(
+  AppendArgs none;
+  std::memset(&none, 0, sizeof(none));
+  const AppendArgs& ap = app != nullptr ? *app : none;
+  prologue_tc_kernel<<<16 * (a.d_c / kSumFeatures) * ngroups + 1 + ap.batch, 256, 0, st>>>(
       static_cast<const __nv_bfloat16*>(a.q), static_cast<const __nv_bfloat16*>(a.w_uk), gamma, beta,
       a.seq_lens, a.batch, a.d_nope, a.d_rope, a.d_c, a.page_size, ws + wl.off_qprep, wl.qprep_stride,
       reinterpret_cast<int32_t*>(ws + wl.off_cu), reinterpret_cast<uint32_t*>(ws + wl.off_done), a.num_splits,
-      a.block_table, a.max_pages, reinterpret_cast<SplitStart*>(ws + wl.off_start));
+      a.block_table, a.max_pages, reinterpret_cast<SplitStart*>(ws + wl.off_start), ap);
   return cudaGetLastError();
 }
 

@@ -89,6 +89,8 @@ constexpr int kBarTile = 1;
 constexpr int kBarXch = 2;
 // sequences per unit of the fused combine
 constexpr uint32_t kFusedMaxG = 16;
+// W_UV,h rows per warp in the fused combine (the fused path needs d_v <= 9 x warps)
+constexpr int kCombineRowsPerWarp = 9;
 // a head's reference max moves only when a tile exceeds it by 2^8
 constexpr float kLazyLog2 = 8.f;
 // score buffers in TMEM and P' buffers in shared memory
@@ -142,9 +144,8 @@ struct Cfg {
   // D_C = 192 the second chunk starts at 64 and overlaps the first, so that no
   // MMA reads past the latent part of a slot (its rows 64..127 are not read out)
   __host__ __device__ static constexpr int mc_start(int j) { return j == 0 ? 0 : D_C - 128; }
-  // fused combine: W_UV,h (at most 256 rows) and up to kFusedMaxG merged
-  // latent rows reuse the page-slot area
-  static_assert(256u * D_C * 2 + kFusedMaxG * D_C * 4 + 128 <= OFF_QBUF, "fused combine area");
+  // fused combine: up to kFusedMaxG merged latent rows reuse the page-slot area
+  static_assert(kFusedMaxG * D_C * 4 <= OFF_QBUF, "fused combine area");
 };
 
 struct TcParams {
@@ -229,7 +230,6 @@ struct Bars {
   uint64_t sready[kNB], sfree[kNB];
   uint64_t spdone[kNP], pfree[kNP];
   uint64_t drain_s, drain_o;   // all MMAs of the score / output issuer done
-  uint64_t wbar;               // W_UV rows of the fused combine landed
   uint32_t tmem_base;
   int abort;
 };
@@ -485,34 +485,27 @@ __device__ __forceinline__ float reduce8_rows(const float (&v)[8], int lane) {
 // b, over the splits s that covered it,
 //   o = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s,
 //   u_{b,h} = W_UV,h o
-// (a sequence of length 0 gets u = 0).  W_UV,h is bulk-copied into the free
-// page-slot area while the CTA waits for the others.  Merge: a warp per
-// (sequence, 32 features), lane k loading (m, l) of slot k0 + k and every lane
-// O of 32 slots at once (online rescaling across groups of 32).  u: a warp per
-// group of eight output rows (see below).
-template <int D_C>
+// (a sequence of length 0 gets u = 0).  Each warp loads its nine rows of
+// W_UV,h (lane l holding features 8l .. 8l + 7) from global memory into
+// registers before it waits, so that the loads overlap the wait.  Merge: a
+// warp per (sequence, 32 features), lane k loading (m, l) of slot k0 + k and
+// every lane O of 32 slots at once (online rescaling across groups of 32),
+// into shared memory.  u: per sequence, the warp's first eight row sums
+// reduced across the lanes by a transposing butterfly (9 shuffles, after
+// which lane 4r holds row r) and the ninth by a plain warp sum.
+template <int D_C, bool TRACE>
 __device__ void fused_combine(const TcParams& p, uint8_t* smem, Bars& bars) {
   constexpr int kWarps = kThreads / 32;
   constexpr int NFB = D_C / 32;      // 32-feature blocks of a row
   constexpr int LANES = D_C / 8;     // lanes holding 8 features each
+  constexpr int kRows = kCombineRowsPerWarp;   // output rows of W_UV,h per warp
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int G = p.cmb_g, units = kHeads * p.cmb_groups;
-  const uint32_t wbytes = static_cast<uint32_t>(p.d_v) * D_C * 2;
-  uint8_t* wsm = smem;                                                    // [d_v][D_C] bf16
-  float* olat = reinterpret_cast<float*>(smem + ((wbytes + 127u) & ~127u));   // [G][D_C]
-  const uint32_t wbar = smem_u32(&bars.wbar);
+  float* olat = reinterpret_cast<float*>(smem);   // [G][D_C], in the free page-slot area
   volatile int* abort_flag = &bars.abort;
   const uint64_t wait_ns = p.wait_ns;
-  auto issue_w = [&](int h) {
-    if (tid == 0) {
-      fence_proxy_async_smem();   // the slot area was last used through the generic proxy too
-      mbar_arrive_expect_tx(wbar, wbytes);
-      bulk_load_hint(smem_u32(wsm), p.w_uv + static_cast<size_t>(h) * p.d_v * D_C, wbytes, wbar,
-                     policy_evict_last());
-    }
-  };
-  int u = blockIdx.x;
-  if (u < units) issue_w(u % kHeads);
+  const uint64_t keep = policy_evict_last();
+  const int v0 = warp * kRows;   // this warp's first output row
   const int total = p.cu[p.batch];
   const int chunk = split_chunk(total, gridDim.x);
   // splits that covered sequence b
@@ -536,10 +529,18 @@ __device__ void fused_combine(const TcParams& p, uint8_t* smem, Bars& bars) {
       __nanosleep(32);
     }
   }
-  int phase = 0;
-  for (; u < units; u += gridDim.x) {
+  for (int u = blockIdx.x; u < units; u += gridDim.x) {
     const int h = u % kHeads, grp = u / kHeads;
     const int b0 = grp * G, nb = min(G, p.batch - b0);
+    // this warp's W_UV,h rows, requested before the wait
+    uint4 wraw[kRows];
+#pragma unroll
+    for (int r = 0; r < kRows; ++r) {
+      const int v = v0 + r;
+      wraw[r] = make_uint4(0, 0, 0, 0);
+      if (lane < LANES && v < p.d_v)
+        wraw[r] = ldg_16_na_hint(p.w_uv + (static_cast<size_t>(h) * p.d_v + v) * D_C + 8 * lane, keep);
+    }
     if (G == 1 && tid == 0 && !*abort_flag) {
       // a unit of one sequence: every softmax warp's part of every split partial of it stored
       const uint32_t want = static_cast<uint32_t>(kSoftWarps) * static_cast<uint32_t>(splits_of(b0));
@@ -555,67 +556,48 @@ __device__ void fused_combine(const TcParams& p, uint8_t* smem, Bars& bars) {
       }
     }
     __syncthreads();
-    if (!*abort_flag) {
-      for (int w = warp; w < nb * NFB; w += kWarps) {
-        const int j = w / NFB, f = (w % NFB) * 32 + lane, b = b0 + j;
-        const int q0 = p.cu[b] + kSegCost, q1 = p.cu[b + 1];   // units of the sequence's pages
-        const int c0 = q0 / chunk;
-        const int n = q1 > q0 ? (q1 - 1) / chunk - c0 + 1 : 0;
-        const float* po = p.part_o + (static_cast<size_t>(c0 + b) * kHeads + h) * D_C + f;
-        const float* pm = p.part_ml + (static_cast<size_t>(c0 + b) * kHeads + h) * 2;
-        float M = -INFINITY, L = 0.f, acc = 0.f;
-        for (int k0 = 0; k0 < n; k0 += 32) {
-          const int kn = min(32, n - k0);
-          float2 ml = make_float2(-INFINITY, 0.f);
-          if (lane < kn) ml = __ldcg(reinterpret_cast<const float2*>(pm + static_cast<size_t>(k0 + lane) * kHeads * 2));
-          float ov[32];
-#pragma unroll
-          for (int kk = 0; kk < 32; ++kk)
-            ov[kk] = kk < kn ? __ldcg(po + static_cast<size_t>(k0 + kk) * kHeads * D_C) : 0.f;
-          float mc = ml.x;
-#pragma unroll
-          for (int o = 16; o > 0; o >>= 1) mc = fmaxf(mc, __shfl_xor_sync(0xffffffffu, mc, o));
-          const float Mn = fmaxf(M, mc);
-          const float sc = exp2f(M - Mn);   // 0 on the first group (M = -inf)
-          const float wk = lane < kn ? exp2f(ml.x - Mn) : 0.f;
-          float lw = wk * ml.y;
-#pragma unroll
-          for (int o = 16; o > 0; o >>= 1) lw += __shfl_xor_sync(0xffffffffu, lw, o);
-          L = fmaf(L, sc, lw);
-          acc *= sc;
-#pragma unroll
-          for (int kk = 0; kk < 32; ++kk) acc = fmaf(__shfl_sync(0xffffffffu, wk, kk), ov[kk], acc);
-          M = Mn;
-        }
-        olat[j * D_C + f] = n > 0 ? acc / L : 0.f;
-      }
-    }
-    // the W_UV,h rows have landed: thread 0 waits on its own flag, so that the
-    // copy is waited for even after an abort (no copy may outlive the CTA)
-    if (tid == 0) {
-      volatile int own = 0;
-      if (!mbar_wait(wbar, phase, &own, wait_ns)) {
-        report_status(p.status, kStatusTimeout);
-        *abort_flag = 1;
-      }
-    }
-    phase ^= 1;
-    __syncthreads();
+    if (u == static_cast<int>(blockIdx.x)) phase_mark<TRACE>(p, 4);
     if (*abort_flag) return;
-    // u = W_UV,h o: a warp per group of 8 output rows (loaded once, lane l
-    // holding features 8l .. 8l + 7 of each), then for each sequence the eight
-    // row sums, reduced across the lanes by a transposing butterfly (9
-    // shuffles) after which lane 4r holds row r
-    const int nvg = (p.d_v + 7) / 8;
-    for (int g = warp; g < nvg; g += kWarps) {
-      uint4 wraw[8];
+    for (int w = warp; w < nb * NFB; w += kWarps) {
+      const int j = w / NFB, f = (w % NFB) * 32 + lane, b = b0 + j;
+      const int q0 = p.cu[b] + kSegCost, q1 = p.cu[b + 1];   // units of the sequence's pages
+      const int c0 = q0 / chunk;
+      const int n = q1 > q0 ? (q1 - 1) / chunk - c0 + 1 : 0;
+      const float* po = p.part_o + (static_cast<size_t>(c0 + b) * kHeads + h) * D_C + f;
+      const float* pm = p.part_ml + (static_cast<size_t>(c0 + b) * kHeads + h) * 2;
+      float M = -INFINITY, L = 0.f, acc = 0.f;
+      for (int k0 = 0; k0 < n; k0 += 32) {
+        const int kn = min(32, n - k0);
+        float2 ml = make_float2(-INFINITY, 0.f);
+        if (lane < kn) ml = __ldcg(reinterpret_cast<const float2*>(pm + static_cast<size_t>(k0 + lane) * kHeads * 2));
+        float ov[32];
 #pragma unroll
-      for (int r = 0; r < 8; ++r) {
-        const int v = 8 * g + r;
-        wraw[r] = make_uint4(0, 0, 0, 0);
-        if (lane < LANES && v < p.d_v)
-          wraw[r] = *reinterpret_cast<const uint4*>(wsm + (static_cast<size_t>(v) * D_C + 8 * lane) * 2);
+        for (int kk = 0; kk < 32; ++kk)
+          ov[kk] = kk < kn ? __ldcg(po + static_cast<size_t>(k0 + kk) * kHeads * D_C) : 0.f;
+        float mc = ml.x;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) mc = fmaxf(mc, __shfl_xor_sync(0xffffffffu, mc, o));
+        const float Mn = fmaxf(M, mc);
+        const float sc = exp2f(M - Mn);   // 0 on the first group (M = -inf)
+        const float wk = lane < kn ? exp2f(ml.x - Mn) : 0.f;
+        float lw = wk * ml.y;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) lw += __shfl_xor_sync(0xffffffffu, lw, o);
+        L = fmaf(L, sc, lw);
+        // four independent sums over the slots (zero weight past kn)
+        float a4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int kk = 0; kk < 32; ++kk) a4[kk & 3] = fmaf(__shfl_sync(0xffffffffu, wk, kk), ov[kk], a4[kk & 3]);
+        acc = fmaf(acc, sc, (a4[0] + a4[1]) + (a4[2] + a4[3]));
+        M = Mn;
       }
+      olat[j * D_C + f] = n > 0 ? acc / L : 0.f;
+    }
+    __syncthreads();
+    if (u == static_cast<int>(blockIdx.x)) phase_mark<TRACE>(p, 5);
+    // u = W_UV,h o from the registers loaded above: rows v0 .. v0 + 7 by the
+    // butterfly, the ninth by a plain reduction
+    if (v0 < p.d_v) {   // uniform in the warp
       for (int j = 0; j < nb; ++j) {
         float o8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
         if (lane < LANES) {
@@ -624,23 +606,27 @@ __device__ void fused_combine(const TcParams& p, uint8_t* smem, Bars& bars) {
           o8[0] = x0.x; o8[1] = x0.y; o8[2] = x0.z; o8[3] = x0.w;
           o8[4] = x1.x; o8[5] = x1.y; o8[6] = x1.z; o8[7] = x1.w;
         }
-        float part[8];
+        float part[kRows];
 #pragma unroll
-        for (int r = 0; r < 8; ++r) {
+        for (int r = 0; r < kRows; ++r) {
           float wv[8];
           bf16x8_to_float(wraw[r], wv);
           part[r] = 0.f;
 #pragma unroll
           for (int e = 0; e < 8; ++e) part[r] = fmaf(wv[e], o8[e], part[r]);
         }
-        const float sum = reduce8_rows(part, lane);
-        const int v = 8 * g + (lane >> 2);
-        if ((lane & 3) == 0 && v < p.d_v)
-          p.out[(static_cast<size_t>(b0 + j) * kHeads + h) * p.d_v + v] = __float2bfloat16_rn(sum);
+        const float sum = reduce8_rows(reinterpret_cast<const float (&)[8]>(part), lane);
+        float last = part[8];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) last += __shfl_xor_sync(0xffffffffu, last, o);
+        __nv_bfloat16* orow = p.out + (static_cast<size_t>(b0 + j) * kHeads + h) * p.d_v;
+        const int v = v0 + (lane >> 2);
+        if ((lane & 3) == 0 && v < p.d_v) orow[v] = __float2bfloat16_rn(sum);
+        if (lane == 0 && v0 + 8 < p.d_v) orow[v0 + 8] = __float2bfloat16_rn(last);
       }
     }
-    __syncthreads();   // W and olat are free for the next unit
-    if (u + static_cast<int>(gridDim.x) < units) issue_w((u + gridDim.x) % kHeads);
+    __syncthreads();   // olat is free for the next unit
+    if (u == static_cast<int>(blockIdx.x)) phase_mark<TRACE>(p, 6);
   }
 }
 
@@ -692,7 +678,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(smem_u32(&bars.drain_s), 1);
     mbar_init(smem_u32(&bars.drain_o), 1);
-    mbar_init(smem_u32(&bars.wbar), 1);
     bars.abort = 0;
     fence_mbar_init();
   }
@@ -700,21 +685,25 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_alloc(smem_u32(&bars.tmem_base), C::TMEM_COLS);
     tmem_relinquish();
   }
+  if (warp == kTmaWarp && lane == 0) {
+    prefetch_tensormap(&cmap);
+    prefetch_tensormap(&krmap);
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   phase_mark<DBG == 2>(p, 1);
   const uint32_t tmem = bars.tmem_base;
+  // Everything above touches only this CTA's shared and tensor memory; what
+  // follows reads the query-absorption kernel's outputs (prepared queries,
+  // split schedule, zeroed counters) and the cache it may have appended to.
+  grid_dependency_wait();
 
   if (warp == kTmaWarp) {
     // ---------------------------------------------------------------- TMA producer
     // The whole warp walks the tiles; lane 0 waits for the slot and issues the
     // copies.  A slot is free once the output MMA of the tile that held it is
     // complete.
-    if (lane == 0) {
-      prefetch_tensormap(&cmap);
-      prefetch_tensormap(&krmap);
-    }
     const uint64_t pol_stream = policy_evict_first();
     Walker w;
     w.start(p);
@@ -826,9 +815,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         // ---- scores of tile js
         const int slot = js % C::NS, sb = js % kNB;
+        const uint32_t zpar = (js / C::NS) & 1;
         const int sg = seg_s + (ts.first ? 1 : 0);
         bool ready = !ts.first || (qn > sg && warp_test(smem_u32(&bars.qfull[sg % C::NQ]), (sg / C::NQ) & 1));
-        ready = ready && warp_test(smem_u32(&bars.zready[slot]), (js / C::NS) & 1);
+        ready = ready && warp_test(smem_u32(&bars.zready[slot]), zpar);
         ready = ready && warp_test(smem_u32(&bars.sfree[sb]), ((js / kNB) & 1) ^ 1);
         if (ready) {
           seg_s = sg;
@@ -1512,7 +1502,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   phase_mark<DBG == 2>(p, 2);
   if (warp == kMmaWarp) tmem_dealloc(tmem, C::TMEM_COLS);
   if (threadIdx.x == 0 && bars.abort) report_status(p.status, kStatusTimeout);
-  if (!DUMP && p.fuse) fused_combine<D_C>(p, smem, bars);
+  if (!DUMP && p.fuse) fused_combine<D_C, DBG == 2>(p, smem, bars);
   phase_mark<DBG == 2>(p, 3);
 }
 
@@ -1582,22 +1572,30 @@ cudaError_t launch_one(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_
   p.wait_ns = a.wait_ns;
   p.stall_cta = a.stall_cta;
   p.stall_tile = a.stall_tile;
-  p.fuse = DBG != 1 && a.batch > 0 && a.num_splits <= resident_ctas(kern, C::SMEM);
+  // (the fused combine holds kCombineRowsPerWarp rows of W_UV,h per warp)
+  p.fuse = DBG != 1 && a.batch > 0 && a.d_v <= kCombineRowsPerWarp * (kThreads / 32) &&
+           a.num_splits <= resident_ctas(kern, C::SMEM);
   if (fused) *fused = p.fuse != 0;
-  if (!p.fuse) {
-    kern<<<a.num_splits, kThreads, C::SMEM, st>>>(maps[0], maps[1], p);
-    return cudaGetLastError();
-  }
+  // The kernel may start while the query-absorption kernel before it on the
+  // stream still runs (programmatic stream serialisation): its setup then
+  // overlaps that kernel's tail, and grid_dependency_wait orders the rest.
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(a.num_splits);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = C::SMEM;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeCooperative;
-  attr[0].val.cooperative = 1;
+  cudaLaunchAttribute attr[2];
+  int na = 0;
+  if (p.fuse) {
+    attr[na].id = cudaLaunchAttributeCooperative;
+    attr[na].val.cooperative = 1;
+    ++na;
+  }
+  attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[na].val.programmaticStreamSerializationAllowed = 1;
+  ++na;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = na;
   return cudaLaunchKernelEx(&cfg, kern, maps[0], maps[1], p);
 }
 

@@ -70,7 +70,9 @@ struct DecodeArgs {
 };
 
 cudaError_t launch_append(const AppendArgs& a, cudaStream_t st);
-cudaError_t launch_prologue_tc(const DecodeArgs& a, cudaStream_t st);
+// query absorption and split schedule; with `app` non-null its blocks also
+// append the new token of every sequence (the pools are read by no block of it)
+cudaError_t launch_prologue_tc(const DecodeArgs& a, const AppendArgs* app, cudaStream_t st);
 cudaError_t launch_decode_f32(const DecodeArgs& a, cudaStream_t st);
 cudaError_t launch_combine(const DecodeArgs& a, bool tc_path, cudaStream_t st);
 // tensor-core split-KV kernel; `maps` = {c_pool map (3-D page box for d_c <= 256), kr_pool map}.

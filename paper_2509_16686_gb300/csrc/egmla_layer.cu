@@ -213,14 +213,15 @@ int eg_mla_layer_decode(const eg_mla_dims* dims, const eg_mla_layer_dims* layer,
       static_cast<const __nv_bfloat16*>(wt->kv_norm_w), H, dims->d_nope, dims->d_rope, dims->d_c, freqs, eps,
       do_kv ? 1 : 0, qb, cb, krb);
   if (cudaGetLastError() != cudaSuccess) return EG_MLA_ERR_CUDA;
-  int rc = EG_MLA_OK;
-  if (do_kv)
-    rc = eg_mla_append_latent(dims, c_pool, krope_pool, id_pool, cb, krb, ids_new, block_table, max_pages_per_seq,
-                              positions, batch, num_pages, dev_status, stream);
-  if (rc != EG_MLA_OK) return rc;
-  rc = eg_mla_decode(dims, qb, c_pool, krope_pool, id_pool, block_table, max_pages_per_seq, seq_lens, max_seq_len,
-                     batch, num_pages, wt->gate_table, wt->ln_gamma, wt->ln_beta, wt->w_uk, wt->w_uv, ub, num_splits,
-                     base + ws.off_dec, ws.dec_bytes, dev_status, stream);
+  // the append (first layer of a group) and the decode as one step
+  const int rc = do_kv ? eg_mla_step(dims, c_pool, krope_pool, id_pool, cb, krb, ids_new, positions, qb, block_table,
+                                     max_pages_per_seq, seq_lens, max_seq_len, batch, num_pages, wt->gate_table,
+                                     wt->ln_gamma, wt->ln_beta, wt->w_uk, wt->w_uv, ub, num_splits, base + ws.off_dec,
+                                     ws.dec_bytes, dev_status, stream)
+                       : eg_mla_decode(dims, qb, c_pool, krope_pool, id_pool, block_table, max_pages_per_seq,
+                                       seq_lens, max_seq_len, batch, num_pages, wt->gate_table, wt->ln_gamma,
+                                       wt->ln_beta, wt->w_uk, wt->w_uv, ub, num_splits, base + ws.off_dec,
+                                       ws.dec_bytes, dev_status, stream);
   if (rc != EG_MLA_OK) return rc;
   // Eq. 14: the output projection of the heads' concatenated outputs
   if (linear(h, E, batch, nu, wt->w_o, ub, y, CUDA_R_16BF, E) != CUBLAS_STATUS_SUCCESS) return EG_MLA_ERR_CUDA;

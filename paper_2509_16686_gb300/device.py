@@ -69,10 +69,15 @@ class DeviceCase:
                            self.w_uk, self.w_uv, o, self.workspace, self.num_splits, self.status, stream)
         return o
 
-    def step(self, stream=None) -> torch.Tensor:
-        """One decode step: append the new token, then attend over the cache."""
-        self.append(stream)
-        return self.decode(stream)
+    def step(self, stream=None, out: Optional[torch.Tensor] = None) -> torch.Tensor:
+        """One decode step (eg_mla_step): append the new token, then attend over
+        the cache."""
+        o = self.out if out is None else out
+        _lib.eg_mla_step(self.dims, self.c_pool, self.kr_pool, self.id_pool, self.c_new, self.kr_new, self.ids_new,
+                         self.positions, self.q, self.block_table, self.seq_lens, self.max_seq_len, self.gate_table,
+                         self.ln_gamma, self.ln_beta, self.w_uk, self.w_uv, o, self.workspace, self.num_splits,
+                         self.status, stream)
+        return o
 
     def bind(self, stream=None):
         """step() with its C-ABI arguments converted once (see _lib.bind_step)."""

@@ -198,6 +198,36 @@ def test_append_is_bit_exact(gpu_lib):
     assert dc.id_pool.cpu().numpy().tobytes() == id_pool.tobytes()
 
 
+def raw_bytes(t):
+    return t.contiguous().view(torch.uint8).cpu().numpy().tobytes()
+
+
+@pytest.mark.parametrize("kind,splits", [("gate256", 5), ("gate192", 0), ("gate256", 400), ("mla512", 7),
+                                         ("fp32", 3)])
+def test_step_equals_append_then_decode(gpu_lib, kind, splits):
+    """eg_mla_step (the append inside the query-absorption grid on the bf16
+    path, the split-KV kernel launched to overlap its setup with it) leaves the
+    cache and the output bit-identical to eg_mla_append_latent followed by
+    eg_mla_decode; 400 splits take the unfused path (separate combine)."""
+    if kind == "fp32":
+        case = synth.case_tiny()
+    else:
+        d_c = {"gate256": 256, "gate192": 192, "mla512": 512}[kind]
+        case = small_bf16((1, 63, 64, 65, 129, 700), d_c=d_c, gate=kind != "mla512")
+    two = device.upload(case, num_splits=splits)
+    two.append()
+    two.decode()
+    one = device.upload(case, num_splits=splits)
+    one.step()
+    torch.cuda.synchronize()
+    assert two.read_status() == 0 and one.read_status() == 0
+    for name in ("c_pool", "kr_pool", "id_pool", "out"):
+        if getattr(two, name) is not None:
+            assert raw_bytes(getattr(one, name)) == raw_bytes(getattr(two, name)), name
+    if kind != "fp32":
+        check_bf16(device.output_f64(one.out), orc.decode_unabsorbed(case), f"step {kind}", scaled_abs=True)
+
+
 @pytest.mark.parametrize("d_c", [256, 192])
 def test_cache_read_and_gate_gather_are_bit_exact(gpu_lib, d_c):
     case = small_bf16((1, 63, 64, 65, 129, 250), d_c=d_c)
