@@ -111,7 +111,7 @@ def make_workload(name):
     elif name == "layers24_full":
         case = synth.case_layer(0)
         desc = "layers24_full: decoder step over 24 full attention layers (hidden 2048: W^Q and W^DKV,KR " \
-               "projections in cuBLAS, fused kv_norm + RoPE, append, gated latent attention, W^O in cuBLAS; " \
+               "projections in this library's tcgen05 GEMM, fused kv_norm + RoPE, append, gated latent attention, W^O; " \
                "each layer's output is the next layer's input), batch 64 x context 8192, 16 heads, d_c 256, " \
                "d_rope 64, vocab 50000, contiguous pages; layer 0's seeded synthetic cache, ids, gate table and " \
                "weights cloned into 24 distinct device copies"
@@ -149,6 +149,31 @@ def max_over_ranks(ms, dist, device):
     t = torch.tensor([ms], dtype=torch.float64, device=device)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def algorithmic_bytes(case, cache_bytes):
+    """Bytes one decode launch must move at least: the latent-cache stream
+    (c^KV, k^R and the token id of every cached token), each distinct gate row
+    G[id] once (the ids of the cached tokens after the step's append), and
+    W_UV of every head.  Queries, outputs, split partials and LayerNorm
+    parameters (under 1 % here) are left out."""
+    d = case.dims
+    elem = 2 if d.dtype == "bf16" else 4
+    gate_rows = 0
+    if d.gate:
+        P = d.page_size
+        ids = []
+        for b in range(case.batch):
+            L = int(case.seq_lens[b])
+            if L == 0:
+                continue
+            pages = case.block_table[b, :(L + P - 1) // P]
+            ids.append(case.id_pool[pages].reshape(-1)[:L - 1])
+            ids.append(case.ids_new[b:b + 1])
+        gate_rows = int(np.unique(np.concatenate(ids)).size) * d.d_c * elem if ids else 0
+    w_uv = d.num_heads * d.d_v * d.d_c * elem
+    return {"cache": int(cache_bytes), "gate_rows_unique": gate_rows, "w_uv": w_uv,
+            "total": int(cache_bytes) + gate_rows + w_uv}
 
 
 def whole_job_rate(world_size, batch, steps, ms):
@@ -382,6 +407,7 @@ def run_gpu_full_layers(args, workload, torch, dist, ws, rank):
     stream = torch.cuda.Stream()
     tokens_cached = int(case.seq_lens.astype(np.int64).sum())
     cache_bytes = tokens_cached * ((d.d_c + d.d_rope) * 2 + 4)
+    algo = algorithmic_bytes(case, cache_bytes)
     splits = base.dc.num_splits or _lib.eg_mla_default_num_splits()
 
     def run_step():
@@ -430,12 +456,13 @@ def run_gpu_full_layers(args, workload, torch, dist, ws, rank):
     del pgraph
     ms_sum, n_l = _lib.eg_mla_profile_end()
     k_ms = ms_sum / max(1, n_l)
-    achieved = cache_bytes / (k_ms * 1e-3) / 1e9
+    achieved = algo["total"] / (k_ms * 1e-3) / 1e9
     peaks_path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(peaks_path):
         peak, peak_src = float(json.load(open(peaks_path))["hbm_gbs"]), "measured"
     else:
         peak, peak_src = 6800.0, "fallback"
+    gemm = projection_gemm_timing(layers, torch, stream, peak)
 
     # end to end through the C ABI from pinned host buffers: every step copies in
     # the new tokens' hidden states, ids and positions and reads back the last
@@ -488,16 +515,63 @@ def run_gpu_full_layers(args, workload, torch, dist, ws, rank):
         "kv_bytes_per_token_model": n_layers // lgz * ((d.d_c + d.d_rope) * 2 + 4),
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                      "traffic": None, "kernel": "decode_tc_kernel", "kernel_ms": k_ms,
-                     "bytes_per_launch": cache_bytes, "peak_source": peak_src},
+                     "bytes_per_launch": algo["total"], "bytes_breakdown": algo, "peak_source": peak_src},
+        "projection_gemm": gemm,
         "cpu_baseline": cpu,
         "e2e": {"value": whole_job_rate(ws, B, e2e_steps, e2e_ms), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
-        # this library's kernels per layer: kv_norm + RoPE, query absorption
-        # (with the append in its grid in the first layer of a group), decode
-        # (the projection GEMMs are cuBLAS kernels, not counted)
-        "gpu_launches": steps_arg * n_layers * 3,
+        # this library's kernels per layer: the query/latent projection,
+        # kv_norm + RoPE, query absorption (with the append in its grid in the
+        # first layer of a group), decode, the output projection
+        "gpu_launches": steps_arg * n_layers * 5,
         "clocks": clk.summary(),
     }
+
+
+def projection_gemm_timing(layers, torch, stream, peak, rounds=4):
+    """The layer's two projection GEMMs alone (eg_mla_debug_linear on each
+    layer's own weights and inputs, every layer in turn, so that the weights
+    stream from HBM: 24 layers x 22 MB > L2): mean time per launch between
+    CUDA events on the launching stream, and the weight bytes per launch over
+    it (the batch rows and outputs are under 1 % of those bytes).  The launches
+    run back to back from a captured graph, each allowed to start streaming
+    its weights while the one before it finishes, as in the step."""
+    from paper_2509_16686_gb300 import _lib
+    res = {}
+    for name in ("w_qkv_a", "w_o"):
+        ops = []
+        for layer in layers:
+            w = getattr(layer, name)
+            if name == "w_qkv_a":
+                x, out = layer.x, torch.empty((layer.x.shape[0], w.shape[0]), dtype=torch.float32, device="cuda")
+            else:
+                u = layer.attn_output().reshape(layer.x.shape[0], -1)
+                x, out = u, torch.empty((u.shape[0], w.shape[0]), dtype=torch.bfloat16, device="cuda")
+            ops.append((w, x, out))
+        with torch.cuda.stream(stream):
+            for w, x, out in ops:
+                _lib.eg_mla_debug_linear(w, x, out, stream=stream)
+        stream.synchronize()
+        # replayed from a captured graph, so that host launch costs drop out
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            for w, x, out in ops:
+                _lib.eg_mla_debug_linear(w, x, out, stream=stream)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            graph.replay()
+            e0.record(stream)
+            for _ in range(rounds):
+                graph.replay()
+            e1.record(stream)
+        stream.synchronize()
+        del graph
+        ms = e0.elapsed_time(e1) / (rounds * len(ops))
+        wbytes = ops[0][0].numel() * ops[0][0].element_size()
+        gbs = wbytes / (ms * 1e-3) / 1e9
+        res[name] = {"shape": [int(ops[0][0].shape[0]), int(ops[0][0].shape[1]), int(ops[0][1].shape[0])],
+                     "kernel_ms": ms, "weight_bytes": wbytes, "achieved_gbs": gbs, "frac": gbs / peak}
+    return res
 
 
 def mla_baseline(case, torch, stream, peak, steps=600):
@@ -548,13 +622,15 @@ def mla_baseline(case, torch, stream, peak, steps=600):
     k_ms = ms_sum / max(1, n_l)
     tokens = int(case.seq_lens.astype(np.int64).sum())
     kvb = (d.d_c + d.d_rope) * (2 if d.dtype == "bf16" else 4)
-    achieved = tokens * kvb / (k_ms * 1e-3) / 1e9
+    algo = algorithmic_bytes(mcase, tokens * kvb)
+    achieved = algo["total"] / (k_ms * 1e-3) / 1e9
     del units, graph
     torch.cuda.empty_cache()
     return {"what": "the same workload with the gate off (plain MLA over the same latent cache)",
             "value": case.batch / (ms_step * 1e-3), "unit": UNIT, "ms_per_step": ms_step, "steps": reps * REPLICAS,
             "decode_kernel_ms": k_ms, "kv_bytes_per_token": kvb,
-            "roofline": {"achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak}}
+            "roofline": {"achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                         "bytes_per_launch": algo["total"], "bytes_breakdown": algo}}
 
 
 def run_gpu(args, workload, torch, dist, ws, rank):
@@ -594,6 +670,9 @@ def run_gpu(args, workload, torch, dist, ws, rank):
     elem = 2 if d.dtype == "bf16" else 4
     id_bytes = 4 if d.gate else 0
     cache_bytes = tokens_cached * ((d.d_c + d.d_rope) * elem + id_bytes)     # per unit (layer)
+    # algorithmic bytes of one decode launch: the cache stream, each distinct
+    # gate row once, and W_UV of every head
+    algo = algorithmic_bytes(case, cache_bytes)
     splits = units[0].num_splits or _lib.eg_mla_default_num_splits()
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     # bf16: query absorption (with the append in its grid) + decode, + the
@@ -672,7 +751,7 @@ def run_gpu(args, workload, torch, dist, ws, rank):
     del pgraph
     ms_sum, n_l = _lib.eg_mla_profile_end()
     k_ms = ms_sum / max(1, n_l)
-    achieved = cache_bytes / (k_ms * 1e-3) / 1e9
+    achieved = algo["total"] / (k_ms * 1e-3) / 1e9
     peaks_path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(peaks_path):
         peak = float(json.load(open(peaks_path))["hbm_gbs"])
@@ -756,7 +835,9 @@ def run_gpu(args, workload, torch, dist, ws, rank):
         "kv_bytes_per_token": (d.d_c + d.d_rope) * elem + id_bytes,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic, "kernel": "decode_tc_kernel",
-                     "kernel_ms": k_ms, "bytes_per_launch": cache_bytes, "peak_source": peak_src},
+                     "kernel_ms": k_ms, "bytes_per_launch": algo["total"], "bytes_breakdown": algo,
+                     "frac_cache_stream_only": cache_bytes / (k_ms * 1e-3) / 1e9 / peak,
+                     "peak_source": peak_src},
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": steps * launches_per_step,

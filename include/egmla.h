@@ -26,8 +26,7 @@
  *     DEVICE pointer to caller-owned memory.  The library never allocates,
  *     frees or keeps device memory between calls; the device memory it owns
  *     is the fixed static scratch array of eg_mla_decode_static, which is
- *     part of the loaded module, and the cuBLAS handle eg_mla_layer_decode
- *     creates at its first call on each device.
+ *     part of the loaded module.
  *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
  *     stream).  Calls are asynchronous on that stream and never synchronise
  *     the host.
@@ -307,8 +306,7 @@ typedef struct {
 } eg_mla_layer_weights;
 
 /* Workspace bytes eg_mla_layer_decode needs (0 on invalid arguments): the
- * projections' outputs, the decode workspace of eg_mla_decode and a 4 MiB
- * cuBLAS workspace. */
+ * projections' outputs, u and the decode workspace of eg_mla_decode. */
 size_t eg_mla_layer_workspace_size(const eg_mla_dims* dims, const eg_mla_layer_dims* layer,
                                    int32_t batch, int32_t num_splits);
 
@@ -317,8 +315,8 @@ size_t eg_mla_layer_workspace_size(const eg_mla_dims* dims, const eg_mla_layer_d
  * eg_mla_layer_decode call with these arguments, of the step's attention
  * output u [batch, num_heads, d_v] (bf16, Eq. 13), which the call leaves there
  * after it completes (the input of the output projection, Eq. 14): a testing
- * and debugging aid.  Returns 0 on invalid arguments (a valid offset is never
- * 0: the cuBLAS workspace comes first).
+ * and debugging aid.  Returns 0 on invalid arguments (a valid offset for
+ * batch >= 1 is never 0: the projections' outputs come first).
  */
 size_t eg_mla_layer_attn_offset(const eg_mla_dims* dims, const eg_mla_layer_dims* layer, int32_t batch,
                                 int32_t num_splits);
@@ -337,14 +335,14 @@ size_t eg_mla_layer_attn_offset(const eg_mla_dims* dims, const eg_mla_layer_dims
  *   y          [batch, E] bf16 output, caller-owned
  *   workspace  >= eg_mla_layer_workspace_size(...) bytes, 256-byte aligned
  *
- * The projections are plain GEMMs run by cuBLAS on a cuBLAS handle this
- * library creates once per device, at the first call on that device (make
- * that first call before any stream capture); every later call allocates
- * nothing and is capturable.  Calls on one device share that handle; the
- * library holds a lock while a call sets the handle's stream and workspace
- * and issues its work.  Host-side argument errors return a
- * negative status and launch nothing; device errors go to *dev_status as for
- * eg_mla_decode.
+ The projections run in this library's weight-streaming tcgen05 GEMM
+ * (fp32 accumulation, the reduction dimension split over the CTAs of a
+ * thread-block cluster and summed in rank order, so results do not depend on
+ * timing).  The call allocates nothing.  The first call with a given shape
+ * runs a host-side occupancy query for the GEMM's cluster size (cached
+ * afterwards); make it before any stream capture.  Host-side argument errors
+ * return a negative status and launch nothing; device errors go to
+ * *dev_status as for eg_mla_decode.
  */
 int eg_mla_layer_decode(const eg_mla_dims* dims, const eg_mla_layer_dims* layer,
                         const eg_mla_layer_weights* weights, const void* x, const int32_t* ids_new,
@@ -398,6 +396,36 @@ int eg_mla_debug_gather(const eg_mla_dims* dims, const void* c_pool, const void*
  */
 int eg_mla_profile_begin(int32_t max_launches);
 int eg_mla_profile_end(double* ms_sum, int32_t* launches);
+
+/*
+ * eg_mla_debug_linear - the projection GEMM of eg_mla_layer_decode on its own
+ * (a testing aid): out[b][n] = sum_j x[b][j] w[n][j] for b < batch,
+ * n < n_out (Eq. 14 and the projections of Appendix C Eqs. 1, 8-10 are of
+ * this form).
+ *
+ *   w     [n_out, k] bf16 row-major, 16-byte aligned
+ *   x     [batch, k] bf16 row-major, 16-byte aligned; k % 8 == 0
+ *   out   [batch, ldo] fp32 (out_f32 != 0) or bf16, ldo >= n_out; columns
+ *         n_out .. ldo - 1 are left untouched
+ * fp32 accumulation; the sum over k is split over the CTAs of a cluster and
+ * added in rank order.  Returns EG_MLA_ERR_INVALID_ARG for bad sizes, strides
+ * or alignment, EG_MLA_ERR_CUDA if the launch fails; a timed-out pipeline
+ * wait is reported in *dev_status (may be NULL) as EG_MLA_ERR_TIMEOUT.
+ */
+int eg_mla_debug_linear(const void* w, int32_t n_out, int32_t k, const void* x, int32_t batch, void* out,
+                        int32_t ldo, int32_t out_f32, int32_t* dev_status, void* stream);
+
+/*
+ * eg_mla_debug_linear_plan - the launch shape eg_mla_debug_linear (and the
+ * projections of eg_mla_layer_decode) use for these sizes on the current
+ * device: *cluster CTAs split the reduction dimension of each 128-row tile,
+ * *stages shared-memory stages, and *max_clusters clusters of that size the
+ * device holds at once (host-side queries; no launch).  Returns
+ * EG_MLA_ERR_INVALID_ARG for bad sizes or null outputs, EG_MLA_ERR_CUDA if a
+ * query fails.
+ */
+int eg_mla_debug_linear_plan(int32_t n_out, int32_t k, int32_t batch, int32_t* cluster, int32_t* stages,
+                             int32_t* max_clusters);
 
 /*
  * eg_mla_debug_set_trace - pipeline event trace of the split-KV decode kernel

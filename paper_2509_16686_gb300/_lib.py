@@ -46,6 +46,8 @@ EXPORTED = [
     "eg_mla_kv_bytes_per_token",
     "eg_mla_status_string",
     "eg_mla_debug_gather",
+    "eg_mla_debug_linear",
+    "eg_mla_debug_linear_plan",
     "eg_mla_profile_begin",
     "eg_mla_profile_end",
     "eg_mla_debug_set_trace",
@@ -98,6 +100,11 @@ def _declare(lib: ctypes.CDLL) -> None:
     lib.eg_mla_step.argtypes = [D, P, P, P, P, P, P, P, P, P, I32, P, I32, I32, I32, P, P, P, P, P, P, I32, P, SZ,
                                 P, P]
     lib.eg_mla_step.restype = ctypes.c_int
+    lib.eg_mla_debug_linear.argtypes = [P, I32, I32, P, I32, P, I32, I32, P, P]
+    lib.eg_mla_debug_linear.restype = ctypes.c_int
+    lib.eg_mla_debug_linear_plan.argtypes = [I32, I32, I32, ctypes.POINTER(I32), ctypes.POINTER(I32),
+                                             ctypes.POINTER(I32)]
+    lib.eg_mla_debug_linear_plan.restype = ctypes.c_int
     lib.eg_mla_kv_bytes_per_token.argtypes = [D, I32, ctypes.POINTER(ctypes.c_int64)]
     lib.eg_mla_kv_bytes_per_token.restype = ctypes.c_int
     lib.eg_mla_status_string.argtypes = [ctypes.c_int]
@@ -319,6 +326,23 @@ def bind_step(dims: EgMlaDims, c_pool, krope_pool, id_pool, c_new, krope_new, id
     step.keepalive = (dims, c_pool, krope_pool, id_pool, c_new, krope_new, ids_new, positions, q, block_table,
                       seq_lens, gate_table, ln_gamma, ln_beta, w_uk, w_uv, out, workspace, dev_status)
     return step
+
+
+def eg_mla_debug_linear(w, x, out, dev_status=None, stream=None) -> None:
+    """out[:, :n_out] = x @ w.T through the layer's projection GEMM (w [n_out, k],
+    x [batch, k] bf16; out fp32 or bf16 with out.shape[1] >= n_out)."""
+    n_out, k = w.shape
+    _check(load().eg_mla_debug_linear(_ptr(w), n_out, k, _ptr(x), x.shape[0], _ptr(out), out.shape[1],
+                                      1 if out.dtype == torch.float32 else 0, _ptr(dev_status), _stream(stream)),
+           "eg_mla_debug_linear")
+
+
+def eg_mla_debug_linear_plan(n_out: int, k: int, batch: int) -> dict:
+    """The projection GEMM's launch shape for these sizes (no launch)."""
+    c, st, m = ctypes.c_int32(0), ctypes.c_int32(0), ctypes.c_int32(0)
+    _check(load().eg_mla_debug_linear_plan(n_out, k, batch, ctypes.byref(c), ctypes.byref(st), ctypes.byref(m)),
+           "eg_mla_debug_linear_plan")
+    return {"cluster": int(c.value), "stages": int(st.value), "max_clusters": int(m.value)}
 
 
 def eg_mla_debug_gather(dims: EgMlaDims, c_pool, krope_pool, id_pool, block_table, seq_lens, max_seq_len,

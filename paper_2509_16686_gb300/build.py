@@ -19,7 +19,8 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libegmla.so")
 
-SOURCES = ["egmla_api.cu", "egmla_aux.cu", "egmla_decode_tc.cu", "egmla_decode_wide.cu", "egmla_layer.cu"]
+SOURCES = ["egmla_api.cu", "egmla_aux.cu", "egmla_decode_tc.cu", "egmla_decode_wide.cu", "egmla_layer.cu",
+           "egmla_linear.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -63,11 +64,11 @@ def build(force: bool = False, verbose_ptxas: bool = False) -> str:
     with cf.ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
         objs = list(ex.map(lambda s: _compile(s, extra), SOURCES))
     tmp = LIB + ".tmp"
-    # cuBLAS (the layer's projection GEMMs) from this toolkit, found at run time
-    # through an rpath to its library directory
+    # the CUDA runtime of this toolkit, found at run time through an rpath to
+    # its library directory
     libdir = os.path.join(os.path.dirname(os.path.dirname(os.path.realpath(nvcc()))), "lib64")
     rpath = ["-Xlinker", f"-rpath={libdir}"] if os.path.isdir(libdir) else []
-    cmd = [nvcc(), *ARCH, "-shared", "-cudart", "shared", "-o", tmp, *objs, "-lcublas", *rpath]
+    cmd = [nvcc(), *ARCH, "-shared", "-cudart", "shared", "-o", tmp, *objs, *rpath]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")

@@ -488,6 +488,28 @@ int eg_mla_decode_static(const eg_mla_dims* dims, const void* q, const void* c_p
                        EG_MLA_STATIC_SCRATCH_BYTES, dev_status, stream);
 }
 
+int eg_mla_debug_linear(const void* w, int32_t n_out, int32_t k, const void* x, int32_t batch, void* out,
+                        int32_t ldo, int32_t out_f32, int32_t* dev_status, void* stream) {
+  if (n_out <= 0 || k <= 0 || batch < 0 || ldo < n_out || k % 8 != 0) return EG_MLA_ERR_INVALID_ARG;
+  if (batch == 0) return EG_MLA_OK;
+  if (!w || !x || !out || !aligned(w, 16) || !aligned(x, 16) || !aligned(out, out_f32 ? 4 : 2))
+    return EG_MLA_ERR_INVALID_ARG;
+  return to_status(egmla::launch_linear_tc(w, n_out, k, x, batch, out, ldo, out_f32 != 0, dev_status,
+                                           static_cast<cudaStream_t>(stream)));
+}
+
+int eg_mla_debug_linear_plan(int32_t n_out, int32_t k, int32_t batch, int32_t* cluster, int32_t* stages,
+                             int32_t* max_clusters) {
+  if (!cluster || !stages || !max_clusters || n_out <= 0 || k <= 0 || batch <= 0 || k % 8 != 0)
+    return EG_MLA_ERR_INVALID_ARG;
+  int c = 0, s = 0, m = 0;
+  const cudaError_t e = egmla::linear_tc_plan(n_out, k, batch, &c, &s, &m);
+  *cluster = c;
+  *stages = s;
+  *max_clusters = m;
+  return to_status(e);
+}
+
 int eg_mla_debug_set_trace(void* dev_buf, int64_t bytes, int32_t ctas) {
   std::lock_guard<std::mutex> lk(g_trace.mu);
   if (dev_buf == nullptr || bytes <= 0 || ctas <= 0) {

@@ -654,6 +654,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   phase_mark<DBG == 2>(p, 0);
+  // a kernel launched after this one with programmatic stream serialisation
+  // (the layer's output projection) may take each SM this kernel leaves
+  grid_launch_dependents();
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::NS; ++s) {

@@ -84,5 +84,15 @@ cudaError_t launch_decode_tc(const DecodeArgs& a, const CUtensorMap* maps, bool 
 cudaError_t launch_decode_wide(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_t st);
 // true if the bf16 tensor-core path has a kernel for these shapes
 bool tc_supported(int d_c, int gate);
+// out[b][n] = sum_k x[b][k] W[n][k] for b < batch, n < n_out: W [n_out, k] and
+// x [batch, k] bf16 row-major (16-byte aligned, k % 8 == 0), out fp32 or
+// bf16 with row stride ldo elements (egmla_linear.cu).  Launched with
+// programmatic stream serialisation: the weight copies may start while the
+// kernel before it on the stream still runs.
+cudaError_t launch_linear_tc(const void* w, int n_out, int k, const void* x, int batch, void* out, int ldo,
+                             bool out_f32, int32_t* status, cudaStream_t st);
+// the launch shape launch_linear_tc picks: cluster size (CTAs splitting k),
+// ring stages, and the clusters of that size the device holds at once
+cudaError_t linear_tc_plan(int n_out, int k, int batch, int* cluster, int* stages, int* max_clusters);
 
 }  // namespace egmla

@@ -2,10 +2,9 @@
 // the query and latent projections, the latent's RMSNorm and the rotary
 // embedding of q^R and k^R (one fused kernel), the cache append and the
 // gated latent attention of egmla_api.cu, and the output projection.  The two
-// projection GEMMs (the stacked query/latent weight, and W^O) are plain GEMMs
-// and run in cuBLAS; everything between them runs in this library's kernels.
-// See include/egmla.h for the contract.
-#include <cublas_v2.h>
+// projection GEMMs (the stacked query/latent weight, and W^O) run in the
+// weight-streaming tcgen05 kernel of egmla_linear.cu.  See include/egmla.h
+// for the contract.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -14,11 +13,10 @@
 #include <mutex>
 
 #include "../../include/egmla.h"
+#include "egmla_kernels.h"
 
 namespace {
 
-constexpr size_t kCublasWorkspace = size_t(4) << 20;
-constexpr int kMaxDevices = 64;
 constexpr int kQkvThreads = 256;
 
 size_t up256(size_t x) { return (x + 255) / 256 * 256; }
@@ -26,7 +24,7 @@ size_t up256(size_t x) { return (x + 255) / 256 * 256; }
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
 struct LayerWorkspace {
-  size_t off_cublas, off_qkv32, off_q, off_c, off_kr, off_u, off_dec, dec_bytes, total;
+  size_t off_qkv32, off_q, off_c, off_kr, off_u, off_dec, dec_bytes, total;
 };
 
 // carve of the layer workspace (every piece 256-byte aligned); dec_bytes = 0 on
@@ -37,8 +35,6 @@ LayerWorkspace layer_workspace(const eg_mla_dims* d, int32_t batch, int32_t num_
   const size_t nq = static_cast<size_t>(d->num_heads) * (d->d_nope + d->d_rope);
   const size_t nkv = static_cast<size_t>(d->d_c + d->d_rope);
   size_t off = 0;
-  w.off_cublas = off;
-  off += kCublasWorkspace;
   w.off_qkv32 = off;
   off = up256(off + B * (nq + nkv) * 4);
   w.off_q = off;
@@ -54,14 +50,6 @@ LayerWorkspace layer_workspace(const eg_mla_dims* d, int32_t batch, int32_t num_
   w.total = up256(off + w.dec_bytes);
   return w;
 }
-
-// One cuBLAS handle per device, created at the first call with that device
-// current, and a lock that keeps one host thread at a time on it.
-struct Handles {
-  std::mutex mu;
-  cublasHandle_t h[kMaxDevices] = {};
-};
-Handles g_handles;
 
 // The new token's kv_norm and rotary embedding (one CTA per sequence):
 //   c^KV = c / sqrt(mean(c^2) + eps) * w,  k^R and every head's q^R rotated,
@@ -130,16 +118,6 @@ __global__ void __launch_bounds__(kQkvThreads) layer_qkv_kernel(
   }
 }
 
-// C[m, n] (column-major, ld m) = A^T B with A [k, m] and B [k, n] column-major,
-// i.e. row-major out[n][m] = in[n][:] . W[m][:] for a Linear weight W [m, k]
-// (ldc >= m: the output row stride in elements)
-cublasStatus_t linear(cublasHandle_t h, int m, int n, int k, const void* w, const void* in, void* out,
-                      cudaDataType_t out_type, int ldc) {
-  const float one = 1.f, zero = 0.f;
-  return cublasGemmEx(h, CUBLAS_OP_T, CUBLAS_OP_N, m, n, k, &one, w, CUDA_R_16BF, k, in, CUDA_R_16BF, k, &zero, out,
-                      out_type, ldc, CUBLAS_COMPUTE_32F, CUBLAS_GEMM_DEFAULT);
-}
-
 }  // namespace
 
 extern "C" {
@@ -190,23 +168,11 @@ int eg_mla_layer_decode(const eg_mla_dims* dims, const eg_mla_layer_dims* layer,
   auto* krb = reinterpret_cast<__nv_bfloat16*>(base + ws.off_kr);
   void* ub = base + ws.off_u;
 
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return EG_MLA_ERR_CUDA;
-  std::lock_guard<std::mutex> lk(g_handles.mu);
-  cublasHandle_t& h = g_handles.h[dev];
-  if (h == nullptr && cublasCreate(&h) != CUBLAS_STATUS_SUCCESS) {
-    h = nullptr;
-    return EG_MLA_ERR_CUDA;
-  }
-  if (cublasSetStream(h, st) != CUBLAS_STATUS_SUCCESS ||
-      cublasSetWorkspace(h, base + ws.off_cublas, kCublasWorkspace) != CUBLAS_STATUS_SUCCESS)
-    return EG_MLA_ERR_CUDA;
-  // Eqs. 8-9 and 1, 10: the query and the latent + RoPE-key projections, one
-  // GEMM over the stacked weight (fp32 out); a later layer of a layer group
-  // projects only its query
+  // the query and latent projections, fp32 out (a later layer of a layer
+  // group projects only its query)
   const bool do_kv = layer->share_kv == 0;
-  if (linear(h, do_kv ? nq + nkv : nq, batch, E, wt->w_qkv_a, x, qkv32, CUDA_R_32F, nq + nkv) !=
-      CUBLAS_STATUS_SUCCESS)
+  if (egmla::launch_linear_tc(wt->w_qkv_a, do_kv ? nq + nkv : nq, E, x, batch, qkv32, nq + nkv, true, dev_status,
+                              st) != cudaSuccess)
     return EG_MLA_ERR_CUDA;
   layer_qkv_kernel<<<batch, kQkvThreads, 0, st>>>(
       static_cast<const float*>(qkv32), positions,
@@ -224,7 +190,8 @@ int eg_mla_layer_decode(const eg_mla_dims* dims, const eg_mla_layer_dims* layer,
                                        ws.dec_bytes, dev_status, stream);
   if (rc != EG_MLA_OK) return rc;
   // Eq. 14: the output projection of the heads' concatenated outputs
-  if (linear(h, E, batch, nu, wt->w_o, ub, y, CUDA_R_16BF, E) != CUBLAS_STATUS_SUCCESS) return EG_MLA_ERR_CUDA;
+  if (egmla::launch_linear_tc(wt->w_o, E, nu, ub, batch, y, E, false, dev_status, st) != cudaSuccess)
+    return EG_MLA_ERR_CUDA;
   return EG_MLA_OK;
 }
 

@@ -192,3 +192,35 @@ def test_24_layer_chain_matches_chained_oracle(gpu_lib):
         x_oracle = orc.store(y_oracle, "bf16")
     rel = rel_l2(got, y_oracle)
     assert rel <= n_layers * BF16_REL_L2, f"24-layer chain: rel_l2={rel:.3e}"
+
+
+@pytest.mark.parametrize("n_out,k,batch,out_f32", [(3392, 2048, 64, True), (2048, 2048, 64, False),
+                                                   (300, 136, 5, True), (128, 64, 16, False),
+                                                   (1000, 520, 300, True), (3072, 2048, 1, True)])
+def test_projection_gemm_matches_fp64(gpu_lib, n_out, k, batch, out_f32):
+    """The layer's projection GEMM (eg_mla_debug_linear) against the product
+    in fp64 of the same bf16 operands: the fp32 accumulation over k terms can
+    move the sum by at most k 2^-24 sum_j |w_nj x_bj| (plus 2^-8 |out| for a
+    bf16 result).  Shapes cover the layer's two projections, ragged tiles
+    (n_out and k off the 128 and 64 multiples), a batch padded to 16, a batch
+    beyond one launch's 256 rows, and one row; columns past n_out stay
+    untouched."""
+    rng = np.random.default_rng(n_out * 7 + k + batch)
+    w = torch.from_numpy(rng.standard_normal((n_out, k)).astype(np.float32) * 0.05).to(torch.bfloat16).cuda()
+    x = torch.from_numpy(rng.standard_normal((batch, k)).astype(np.float32)).to(torch.bfloat16).cuda()
+    ldo = n_out + 8
+    out = torch.full((batch, ldo), 7.0, dtype=torch.float32 if out_f32 else torch.bfloat16, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    _lib.eg_mla_debug_linear(w, x, out, status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    wf = w.double().cpu().numpy()
+    xf = x.double().cpu().numpy()
+    ref = xf @ wf.T
+    got = out.double().cpu().numpy()
+    bound = k * 2.0 ** -24 * (np.abs(xf) @ np.abs(wf).T)
+    if not out_f32:
+        bound = bound + 2.0 ** -8 * np.abs(ref)
+    diff = np.abs(got[:, :n_out] - ref)
+    assert (diff <= bound + 1e-30).all(), f"worst {float((diff / (bound + 1e-30)).max()):.2f} of the bound"
+    assert (got[:, n_out:] == 7.0).all()
