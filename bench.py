@@ -82,6 +82,8 @@ def parse():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--splits", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="layers of the layers24 / layers24_full workloads (default 24; fewer for a profiling run)")
     ap.add_argument("--e2e-steps", type=int, default=0)
     ap.add_argument("--oracle-probe", default=None, help=argparse.SUPPRESS)
     ap.add_argument("--oracle-budget", type=float, default=4.0, help=argparse.SUPPRESS)
@@ -110,16 +112,17 @@ def make_workload(name):
         desc = "ragged_mla: plain-MLA baseline (gate off) at d_c 512 on the ragged lengths"
     elif name == "layers24_full":
         case = synth.case_layer(0)
-        desc = "layers24_full: decoder step over 24 full attention layers (hidden 2048: W^Q and W^DKV,KR " \
+        desc = f"layers24_full: decoder step over {layers_of(name)} full attention layers (hidden 2048: W^Q and W^DKV,KR " \
                "projections in this library's tcgen05 GEMM, fused kv_norm + RoPE, append, gated latent attention, W^O; " \
                "each layer's output is the next layer's input), batch 64 x context 8192, 16 heads, d_c 256, " \
                "d_rope 64, vocab 50000, contiguous pages; layer 0's seeded synthetic cache, ids, gate table and " \
-               "weights cloned into 24 distinct device copies"
+               f"weights cloned into {layers_of(name)} distinct device copies"
     elif name == "layers24":
         case = synth.case_layer(0)
-        desc = "layers24: decoder step over 24 attention layers (append + decode per layer on one stream), " \
+        desc = f"layers24: decoder step over {layers_of(name)} attention layers (append + decode per layer on one stream), " \
                "batch 64 x context 8192, 16 heads, d_c 256, d_rope 64, vocab 50000, contiguous pages; layer 0's " \
-               "seeded synthetic cache, ids, gate table, weights and inputs cloned into 24 distinct device copies"
+               f"seeded synthetic cache, ids, gate table, weights and inputs cloned into {layers_of(name)} distinct " \
+               "device copies"
     else:
         ctx = int(name[3:])
         case = synth.case_c4k(batch=8, ctx=ctx, keep_logical=False)
@@ -127,8 +130,13 @@ def make_workload(name):
     return case, desc
 
 
+LAYERS_OVERRIDE = None   # --layers: fewer layers for a profiling run of the layer workloads
+
+
 def layers_of(name):
-    return 24 if name.startswith("layers24") else 1
+    if not name.startswith("layers24"):
+        return 1
+    return LAYERS_OVERRIDE or 24
 
 
 SWEEP_CTX = (1024, 2048, 4096, 8192, 16384, 32768, 65536)
@@ -847,7 +855,10 @@ def run_gpu(args, workload, torch, dist, ws, rank):
 
 
 def main():
+    global LAYERS_OVERRIDE
     args = parse()
+    if args.layers:
+        LAYERS_OVERRIDE = args.layers
     if args.oracle_probe:
         return oracle_probe(args.oracle_probe, args.oracle_budget)
     if args.impl == "reference":
