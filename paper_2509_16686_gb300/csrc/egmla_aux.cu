@@ -320,141 +320,145 @@ __device__ __forceinline__ float from_f<float>(float v) { return v; }
 template <>
 __device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
 
-// Block per (sequence b, head h), 256 threads.  The splits that covered b are
-// the CTAs c0..c1 of the page schedule; their partials sit in slots c + b.
-// M = max_s m_s; o = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M) l_s (m in log2
-// units); then u = W_UV,h o.  A sequence of length 0 gets u = 0.  The kernel
-// is a chain of dependent loads, so it is laid out to keep that chain short:
-//  - thread k keeps the (m, l) of slot k that it loaded for the maximum and
-//    forms its weight 2^(m - M) from registers;
-//  - a thread per latent feature loads O of up to kCombineBurst slots into
-//    registers before it adds any of them (one round trip for that many
-//    splits);
-//  - a warp loads all kCombineRows of its W_UV,h rows (16-byte pieces, lane l
-//    the pieces l, l + 32, ..) before the sums, and a shuffle tree adds the
-//    lanes' parts of each row.
-// Two instantiations: <16, 24> (about 110 registers) for grids of up to about
-// two blocks per SM, where each block's latency is the step's; <8, 8> (about
-// half the registers, more resident blocks) for larger grids, where
-// occupancy hides the latency.
+// Block per (head h, group of kCombineGroup sequences), 256 threads: the
+// sequences of a group share one pass over W_UV,h.  The splits that covered
+// sequence b are the CTAs c0..c1 of the page schedule; their partials sit in
+// slots c + b.  M = max_s m_s; o = sum_s 2^(m_s - M) O_s / sum_s 2^(m_s - M)
+// l_s (m in log2 units); then u = W_UV,h o.  A sequence of length 0 gets
+// u = 0.
+//  - merge: warp j takes sequence b0 + j: lane k holds slot k's (m, l) of
+//    each group of 32 slots, and every lane the O values of its features
+//    (f = lane + 32 i) for one slot at a time, the slot's weight broadcast
+//    from the lane that holds it;
+//  - u: warp w takes groups of four W_UV,h rows; a lane loads its 16-byte
+//    pieces of the four rows once and multiplies them into all the group's
+//    merged vectors (shared memory), then the 32 sums (sequence, row) are
+//    reduced across the lanes by a transposing butterfly (31 shuffles), after
+//    which lane t holds sequence t / 4, row t % 4.
 constexpr int kCombineThreads = 256;
-constexpr int kMaxSlotsSmem = 512;
+constexpr int kCombineGroup = 8;        // sequences per block (one warp each in the merge)
 constexpr int kCombineMaxDc = 512;
+constexpr int kCombineFeat = kCombineMaxDc / 32;   // features per lane in the merge, at most
 
-template <typename T, int kCombineRows, int kCombineBurst>
+// v[i] (i < 32) summed over the warp; lane t returns the sum of v[t]
+__device__ __forceinline__ float reduce32_transpose(float (&v)[32], int lane) {
+#pragma unroll
+  for (int o = 16, len = 32; o > 0; o >>= 1, len >>= 1) {
+    const bool up = (lane & o) != 0;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      if (i < len / 2) {
+        const float keep = up ? v[i + len / 2] : v[i];
+        const float send = up ? v[i] : v[i + len / 2];
+        v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+      }
+    }
+  }
+  return v[0];
+}
+
+template <typename T>
 __global__ void __launch_bounds__(kCombineThreads)
 combine_kernel(const int32_t* __restrict__ cu, const float* __restrict__ part_ml, const float* __restrict__ part_o,
                const T* __restrict__ w_uv, T* __restrict__ out, int batch, int H, int d_c, int d_v,
                int num_splits) {
-  __shared__ __align__(16) float olat[kCombineMaxDc];
-  __shared__ float wts[kMaxSlotsSmem];
-  __shared__ float red[kCombineThreads / 32];
-  const int b = blockIdx.x / H, h = blockIdx.x % H;
+  __shared__ __align__(16) float olat[kCombineGroup][kCombineMaxDc];
+  const int h = blockIdx.x % H, b0 = (blockIdx.x / H) * kCombineGroup;
+  const int nb = min(kCombineGroup, batch - b0);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   constexpr int kWarps = kCombineThreads / 32;
   const int total = cu[batch];
   const int chunk = split_chunk(total, num_splits);
-  const int p0 = cu[b] + kSegCost, p1 = cu[b + 1];   // units of the sequence's pages
-  const int c0 = p0 / chunk;
-  const int n = p1 > p0 ? (p1 - 1) / chunk - c0 + 1 : 0;
-  if (n == 0) {
-    for (int f = tid; f < d_c; f += kCombineThreads) olat[f] = 0.f;
-  } else {
-    const float* pml = part_ml + (static_cast<size_t>(c0 + b) * H + h) * 2;
-    const size_t mlstride = static_cast<size_t>(H) * 2;
-    // running maxima and denominators of the slots (n <= num_splits); thread
-    // tid keeps slot tid's pair
-    float2 mine = make_float2(-INFINITY, 0.f);
-    if (tid < n) mine = *reinterpret_cast<const float2*>(pml + tid * mlstride);
-    float mloc = mine.x;
-    for (int k = tid + kCombineThreads; k < n; k += kCombineThreads) mloc = fmaxf(mloc, pml[k * mlstride]);
+  if (warp < nb) {
+    const int b = b0 + warp;
+    const int p0 = cu[b] + kSegCost, p1 = cu[b + 1];   // units of the sequence's pages
+    const int c0 = p0 / chunk;
+    const int n = p1 > p0 ? (p1 - 1) / chunk - c0 + 1 : 0;
+    float* ol = olat[warp];
+    if (n == 0) {
+      for (int f = lane; f < d_c; f += 32) ol[f] = 0.f;
+    } else {
+      const size_t mlstride = static_cast<size_t>(H) * 2, sstride = static_cast<size_t>(H) * d_c;
+      const float* pml = part_ml + (static_cast<size_t>(c0 + b) * H + h) * 2;
+      const float* po = part_o + (static_cast<size_t>(c0 + b) * H + h) * d_c;
+      float M = -INFINITY;
+      for (int k = lane; k < n; k += 32) M = fmaxf(M, pml[k * mlstride]);
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, o));
-    if (lane == 0) red[warp] = mloc;
-    __syncthreads();
-    float M = red[0];
+      for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+      float acc[kCombineFeat];
 #pragma unroll
-    for (int k = 1; k < kWarps; ++k) M = fmaxf(M, red[k]);
-    __syncthreads();
-    float lloc = 0.f;
-    if (tid < n) {
-      const float wk = exp2f(mine.x - M);
-      if (tid < kMaxSlotsSmem) wts[tid] = wk;
-      lloc = wk * mine.y;
-    }
-    for (int k = tid + kCombineThreads; k < n; k += kCombineThreads) {
-      const float wk = exp2f(pml[k * mlstride] - M);
-      if (k < kMaxSlotsSmem) wts[k] = wk;
-      lloc = fmaf(wk, pml[k * mlstride + 1], lloc);
-    }
+      for (int i = 0; i < kCombineFeat; ++i) acc[i] = 0.f;
+      float lsum = 0.f;
+      for (int k0 = 0; k0 < n; k0 += 32) {
+        const int kn = min(32, n - k0);
+        float wk = 0.f;
+        if (lane < kn) {
+          const float2 ml = *reinterpret_cast<const float2*>(pml + (k0 + lane) * mlstride);
+          wk = exp2f(ml.x - M);
+          lsum = fmaf(wk, ml.y, lsum);
+        }
+#pragma unroll 2
+        for (int kk = 0; kk < kn; ++kk) {
+          const float w = __shfl_sync(0xffffffffu, wk, kk);
+          const float* ps = po + (k0 + kk) * sstride;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) lloc += __shfl_xor_sync(0xffffffffu, lloc, o);
-    if (lane == 0) red[warp] = lloc;
-    __syncthreads();
-    float L = 0.f;
-#pragma unroll
-    for (int k = 0; k < kWarps; ++k) L += red[k];
-    const float invL = 1.f / L;
-    const size_t sstride = static_cast<size_t>(H) * d_c;
-    for (int f = tid; f < d_c; f += kCombineThreads) {
-      const float* po = part_o + (static_cast<size_t>(c0 + b) * H + h) * d_c + f;
-      float a0 = 0.f, a1 = 0.f;
-      for (int k0 = 0; k0 < n; k0 += kCombineBurst) {
-        float v[kCombineBurst];
-#pragma unroll
-        for (int i = 0; i < kCombineBurst; ++i) v[i] = k0 + i < n ? po[(k0 + i) * sstride] : 0.f;
-#pragma unroll
-        for (int i = 0; i < kCombineBurst; i += 2) {
-          const int k = k0 + i;
-          if (k < n) a0 = fmaf(k < kMaxSlotsSmem ? wts[k] : exp2f(pml[k * mlstride] - M), v[i], a0);
-          if (k + 1 < n) a1 = fmaf(k + 1 < kMaxSlotsSmem ? wts[k + 1] : exp2f(pml[(k + 1) * mlstride] - M), v[i + 1], a1);
+          for (int i = 0; i < kCombineFeat; ++i) {
+            const int f = lane + 32 * i;
+            if (f < d_c) acc[i] = fmaf(w, ps[f], acc[i]);
+          }
         }
       }
-      olat[f] = (a0 + a1) * invL;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, o);
+      const float invL = 1.f / lsum;
+#pragma unroll
+      for (int i = 0; i < kCombineFeat; ++i) {
+        const int f = lane + 32 * i;
+        if (f < d_c) ol[f] = acc[i] * invL;
+      }
     }
   }
   __syncthreads();
-  // u[v] = sum_f W_UV[h][v][f] olat[f]
+  // u[j][v] = sum_f W_UV[h][v][f] olat[j][f]
   constexpr int VEC = 16 / sizeof(T);
+  const int npieces = d_c / VEC;   // d_c is a multiple of VEC for both element types
   const T* wh = w_uv + static_cast<size_t>(h) * d_v * d_c;
-  for (int v0 = warp * kCombineRows; v0 < d_v; v0 += kWarps * kCombineRows) {
-    float acc[kCombineRows];
+  for (int v0 = 4 * warp; v0 < d_v; v0 += 4 * kWarps) {
+    float acc[32];
 #pragma unroll
-    for (int r = 0; r < kCombineRows; ++r) acc[r] = 0.f;
-    for (int f = lane * VEC; f < d_c; f += 32 * VEC) {
-      uint4 raw[kCombineRows];
+    for (int i = 0; i < 32; ++i) acc[i] = 0.f;
+    for (int pc = lane; pc < npieces; pc += 32) {
+      float wf[4][VEC];
 #pragma unroll
-      for (int r = 0; r < kCombineRows; ++r)
-        raw[r] = v0 + r < d_v ? *reinterpret_cast<const uint4*>(wh + static_cast<size_t>(v0 + r) * d_c + f)
-                              : make_uint4(0, 0, 0, 0);
-      float o[VEC];
+      for (int r = 0; r < 4; ++r) {
+        uint4 raw = make_uint4(0, 0, 0, 0);
+        if (v0 + r < d_v) raw = *reinterpret_cast<const uint4*>(wh + static_cast<size_t>(v0 + r) * d_c + pc * VEC);
+        const T* e = reinterpret_cast<const T*>(&raw);
 #pragma unroll
-      for (int i = 0; i < VEC; i += 4) {
-        const float4 q = *reinterpret_cast<const float4*>(olat + f + i);
-        o[i] = q.x;
-        o[i + 1] = q.y;
-        o[i + 2] = q.z;
-        o[i + 3] = q.w;
+        for (int i = 0; i < VEC; ++i) wf[r][i] = to_f<T>(e[i]);
       }
 #pragma unroll
-      for (int r = 0; r < kCombineRows; ++r) {
-        const T* e = reinterpret_cast<const T*>(&raw[r]);
+      for (int j = 0; j < kCombineGroup; ++j) {
+        if (j < nb) {
+          float o[VEC];
 #pragma unroll
-        for (int i = 0; i < VEC; ++i) acc[r] = fmaf(to_f<T>(e[i]), o[i], acc[r]);
+          for (int i = 0; i < VEC; i += 4) {
+            const float4 q = *reinterpret_cast<const float4*>(&olat[j][pc * VEC + i]);
+            o[i] = q.x;
+            o[i + 1] = q.y;
+            o[i + 2] = q.z;
+            o[i + 3] = q.w;
+          }
+#pragma unroll
+          for (int r = 0; r < 4; ++r)
+#pragma unroll
+            for (int i = 0; i < VEC; ++i) acc[4 * j + r] = fmaf(wf[r][i], o[i], acc[4 * j + r]);
+        }
       }
     }
-#pragma unroll
-    for (int r = 0; r < kCombineRows; ++r) {
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) acc[r] += __shfl_xor_sync(0xffffffffu, acc[r], o);
-    }
-    if (lane < kCombineRows && v0 + lane < d_v) {
-      float mine = acc[0];
-#pragma unroll
-      for (int r = 1; r < kCombineRows; ++r)
-        if (lane == r) mine = acc[r];
-      out[(static_cast<size_t>(b) * H + h) * d_v + v0 + lane] = from_f<T>(mine);
-    }
+    const float sum = reduce32_transpose(acc, lane);
+    const int j = lane >> 2, v = v0 + (lane & 3);
+    if (j < nb && v < d_v) out[(static_cast<size_t>(b0 + j) * H + h) * d_v + v] = from_f<T>(sum);
   }
 }
 
@@ -636,29 +640,12 @@ cudaError_t launch_decode_f32(const DecodeArgs& a, cudaStream_t st) {
 }
 
 namespace {
-int device_sms() {
-  static int cached[64] = {0};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
-  if (cached[dev] == 0) {
-    int sms = 0;
-    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) sms = 1;
-    cached[dev] = sms;
-  }
-  return cached[dev];
-}
-
 template <typename T>
 void launch_combine_t(const DecodeArgs& a, const int32_t* cu, const float* ml, const float* po, cudaStream_t st) {
-  const int grid = a.batch * a.H;
-  const T* w = static_cast<const T*>(a.w_uv);
-  T* out = static_cast<T*>(a.out);
-  if (grid <= 2 * device_sms())
-    combine_kernel<T, 16, 24><<<grid, kCombineThreads, 0, st>>>(cu, ml, po, w, out, a.batch, a.H, a.d_c, a.d_v,
-                                                                a.num_splits);
-  else
-    combine_kernel<T, 8, 8><<<grid, kCombineThreads, 0, st>>>(cu, ml, po, w, out, a.batch, a.H, a.d_c, a.d_v,
-                                                              a.num_splits);
+  const int grid = a.H * ((a.batch + kCombineGroup - 1) / kCombineGroup);
+  combine_kernel<T><<<grid, kCombineThreads, 0, st>>>(cu, ml, po, static_cast<const T*>(a.w_uv),
+                                                      static_cast<T*>(a.out), a.batch, a.H, a.d_c, a.d_v,
+                                                      a.num_splits);
 }
 }  // namespace
 
