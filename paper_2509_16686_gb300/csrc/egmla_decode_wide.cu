@@ -271,6 +271,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = bars.tmem_base;
+  // Everything above touches only this CTA's shared and tensor memory; what
+  // follows reads the query-absorption kernel's outputs and the cache it may
+  // have appended to (launched with programmatic stream serialisation).
+  grid_dependency_wait();
 
   if (warp < kGateWarp0) regs_decrease<kProducerRegs>();
   if (warp == 0) {
@@ -623,8 +627,18 @@ cudaError_t launch_one(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_
   p.max_pages = a.max_pages;
   p.num_pages = a.num_pages;
   p.scale_log2 = a.scale_log2;
-  kern<<<a.num_splits, kThreads, C::SMEM, st>>>(maps[0], maps[1], p);
-  return cudaGetLastError();
+  // set-up overlaps the query-absorption kernel before it on the stream
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.num_splits);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = C::SMEM;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, maps[0], maps[1], p);
 }
 
 }  // namespace
