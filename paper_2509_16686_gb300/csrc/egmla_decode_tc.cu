@@ -821,8 +821,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t zpar = (js / C::NS) & 1;
         const int sg = seg_s + (ts.first ? 1 : 0);
         bool ready = !ts.first || (qn > sg && warp_test(smem_u32(&bars.qfull[sg % C::NQ]), (sg / C::NQ) & 1));
-        ready = ready && warp_test(smem_u32(&bars.zready[slot]), zpar);
         ready = ready && warp_test(smem_u32(&bars.sfree[sb]), ((js / kNB) & 1) ^ 1);
+        if (ready && !(q_more && warp_test(smem_u32(&bars.qempty[qn % C::NQ]), ((qn / C::NQ) & 1) ^ 1))) {
+          // nothing else to serve: sleep in hardware until the gate warps
+          // release the slot (the gate waits on nothing this warp does)
+          ready = warp_wait(smem_u32(&bars.zready[slot]), zpar, abort_flag, wait_ns);
+          if (!ready) break;   // uniform: the wait ran out or another role aborted
+        } else {
+          ready = ready && warp_test(smem_u32(&bars.zready[slot]), zpar);
+        }
         if (ready) {
           seg_s = sg;
           tr.mark(1, js);
