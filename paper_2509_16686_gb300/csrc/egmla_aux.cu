@@ -1,9 +1,11 @@
 // egmla_aux.cu - the small kernels around the tensor-core decode kernel:
 //   append_latent_kernel   cache write of the new token (bit-exact copy)
-//   prologue_*_kernel      per-step query absorption q^ = W_UK,h^T q^C and the
-//                          page prefix sums the split-KV schedule needs
-//   combine_*_kernel       log-sum-exp merge of the split partials and the
-//                          W_UV,h up-projection of the latent output
+//   prologue_*_kernel      per-step query absorption q^ = W_UK,h^T q^C, the
+//                          page prefix sums and split start records of the
+//                          split-KV schedule, and (in eg_mla_step) the append
+//   combine_kernel         log-sum-exp merge of the split partials and the
+//                          W_UV,h up-projection of the latent output, for the
+//                          launches whose decode kernel does not fuse it
 //   decode_f32_kernel      the fp32 specialisation of the split-KV decode
 //                          (exact fp32 arithmetic on CUDA cores; bf16 runs on
 //                          tcgen05 in egmla_decode_tc.cu)

@@ -1,9 +1,11 @@
 // egmla_common.cuh - launch-independent pieces shared by the decode kernels:
 // the workspace layout and the split-KV work schedule.
 //
-// Split-KV schedule.  The cache pages of all sequences are numbered globally in
-// sequence order (prefix sums cu_pages[b] = sum_{b'<b} ceil(L_b'/P)) and cut
-// into `num_splits` equal contiguous ranges of `chunk` pages, one per CTA.  A
+// Split-KV schedule.  The work is counted in units: the cache pages of every
+// sequence plus kSegCost per non-empty sequence (what a split pays to take in
+// a sequence).  The units of all sequences are numbered globally in sequence
+// order (prefix sums cu[b]) and cut into `num_splits` equal contiguous ranges
+// of `chunk` units, one per CTA.  A
 // CTA may therefore cover the tail of one sequence and the head of the next;
 // it emits one partial result (running max m, denominator l, un-normalised
 // latent output) per sequence it touches.  Partial slot of (CTA c, sequence b)

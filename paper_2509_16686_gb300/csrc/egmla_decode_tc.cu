@@ -8,21 +8,27 @@
 //
 //   TMA (warp 4)      latent page [64 tok x d_c] (one 3-D box: 64-feature
 //                     columns x 64 rows) and RoPE-key page [64 x 64], both
-//                     128-byte swizzled, as soon as the page slot is free.
+//                     128-byte swizzled, and the page's token ids (a bulk copy
+//                     into the slot's statistics area), as soon as the page
+//                     slot is free; a CTA's first page is requested alone.
+//                     The split's start comes from a record the
+//                     query-absorption kernel wrote.
 //   gate (warps 7-14; each quarter-warp owns two token rows, lane u the 16-byte
 //                     units 2u, 2u + 1 of every 64-feature column of them)
-//                     the token ids (two tiles ahead) and the gate rows
-//                     g = G[id] (EG-MLA-A table, Section 5.2; one tile ahead)
-//                     from L2 into registers, every quarter-warp load reading
-//                     one whole 128-byte line; z = c (*) g rounded to bf16 and
-//                     written back in place, and the LayerNorm statistics
-//                     mu, r = 1/sqrt(var + eps) of z (Eq. 5 over d_c).
+//                     the gate rows g = G[id] (EG-MLA-A table, Section 5.2)
+//                     of the next tile into registers, requested column by
+//                     column between this tile's stores as soon as the next
+//                     page (and so its ids) has landed, every quarter-warp
+//                     load reading one whole 128-byte line from L2; z = c (*) g
+//                     rounded to bf16 and written back in place, and the
+//                     LayerNorm statistics mu, r = 1/sqrt(var + eps) of z
+//                     (Eq. 5 over d_c).
 //   scores (warp 5)   S = Z (q^ gamma)^T and S_rope = K^R q^R^T (M = 64 tokens,
 //                     N = 16 heads, K = d_c and 64; fp32 in TMEM, four score
 //                     buffers) as soon as a gated page and a score buffer are
-//                     ready, and the query block of the next sequence segment
-//                     (the warp polls both conditions, so neither waits for
-//                     the other).
+//                     ready, and the query block of the next sequence segment;
+//                     with no query block to load the warp sleeps in hardware
+//                     on the gate's barrier.
 //   output (warp 6)   O^T += Z^T P' (M = 128 latent features, N = 16 heads,
 //                     K = 64 tokens; O^T stays in TMEM over a sequence
 //                     segment).  An issuing thread stalls while the tensor
@@ -47,9 +53,11 @@
 // query block takes 10 KB, which leaves room for five page slots at d_c = 256.
 //
 // The queries are absorbed before this kernel (q^ = W_UK^T q^C, with gamma
-// folded in); W_UV is applied after the split merge.  Everything the kernel
-// waits on has a time limit: on expiry it records EG_MLA_ERR_TIMEOUT, drains
-// its own copies and MMAs, frees TMEM and exits.
+// folded in); the kernel may start while that kernel runs (programmatic
+// stream serialisation) and waits for it after its set-up.  The split merge
+// and W_UV run at its end when the grid is cooperative (fused_combine).
+// Everything the kernel waits on has a time limit: on expiry it records
+// EG_MLA_ERR_TIMEOUT, drains its own copies and MMAs, frees TMEM and exits.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
