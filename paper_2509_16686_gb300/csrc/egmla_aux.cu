@@ -96,8 +96,48 @@ __device__ void page_prefix_sums(const int32_t* seq_lens, int batch, int page_si
   if (lane == 0) cu[batch] = carry;
 }
 
+// The same prefix sums by a whole block of 256 threads (a warp scan per 256
+// sequences, the warps' totals through shared memory), written to global
+// memory and to the block's shared copy cu_s (batch + 1 entries); one load
+// round trip per 256 sequences.
+__device__ void page_prefix_sums_block(const int32_t* seq_lens, int batch, int page_size, int32_t* cu,
+                                       int32_t* cu_s, int32_t* wsum) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x / 32;
+  int32_t carry = 0;
+  for (int base = 0; base < batch; base += blockDim.x) {
+    const int b = base + tid;
+    const int L = b < batch ? seq_lens[b] : 0;
+    const int np = L > 0 ? (L + page_size - 1) / page_size + kSegCost : 0;
+    int incl = np;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int t = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += t;
+    }
+    if (lane == 31) wsum[warp] = incl;
+    __syncthreads();
+    int before = 0, total = 0;
+    for (int w = 0; w < nw; ++w) {
+      const int v = wsum[w];
+      before += w < warp ? v : 0;
+      total += v;
+    }
+    if (b < batch) {
+      const int32_t e = carry + before + incl - np;
+      cu[b] = e;
+      cu_s[b] = e;
+    }
+    carry += total;
+    __syncthreads();   // wsum is rewritten by the next pass
+  }
+  if (tid == 0) {
+    cu[batch] = carry;
+    cu_s[batch] = carry;
+  }
+}
+
 // Start record of every split (see SplitStart), from the prefix sums this
-// block just wrote (plain loads: they are this kernel's own stores).  Split c
+// block just wrote (its shared copy).  Split c
 // owns units [c chunk, (c + 1) chunk); its first sequence is the last one whose
 // first unit is at most c chunk (empty sequences skipped), as in the decode
 // kernel's walk.
@@ -140,7 +180,7 @@ __device__ void split_starts(const int32_t* cu, const int32_t* seq_lens, int bat
 // in fp32 and stores (q^ (*) gamma) rounded to bf16 in the prepared query
 // block (qop_offset layout).  Its per-chunk partials of w_h = sum_f bf16(q^ gamma)_f
 // and b_h = q^_h . beta go to the block's slots of the sums area.  Chunk-0
-// blocks also copy q^R.  The last block computes the page prefix sums and the
+// blocks also copy q^R.  Block 0 computes the page prefix sums and the
 // splits' start records.
 //  - All 16-byte global loads of a thread are issued before any is stored
 //    (W_UK with an L2 evict-last hint: it stays in L2 across steps).
@@ -172,22 +212,38 @@ __global__ void prologue_tc_kernel(const __nv_bfloat16* __restrict__ q, const __
   // the decode kernel after this one may begin its setup (it waits for this
   // kernel's completion before it reads anything written here)
   grid_launch_dependents();
-  if (blockIdx.x > static_cast<unsigned>(H * nchunk * ngroups)) {
+  // block 0: the schedule (dispatched first, so that it never waits for a
+  // second wave of the grid); blocks 1 .. A: the absorption items; then the
+  // append blocks
+  const int nabs = H * nchunk * ngroups;
+  if (blockIdx.x > static_cast<unsigned>(nabs)) {
     // blocks after the schedule block: the new token of one sequence (a step
     // that appends before it attends); no block of this kernel reads the pools
-    append_row(app, blockIdx.x - (H * nchunk * ngroups + 1));
+    append_row(app, blockIdx.x - (nabs + 1));
     return;
   }
-  if (blockIdx.x == static_cast<unsigned>(H * nchunk * ngroups)) {
+  if (blockIdx.x == 0) {
     if (seq_done != nullptr)
       for (int i = threadIdx.x; i <= batch; i += blockDim.x) seq_done[i] = 0u;
-    page_prefix_sums(seq_lens, batch, page_size, cu);
-    __syncthreads();   // the prefix sums are visible to the whole block
-    split_starts(cu, seq_lens, batch, num_splits, block_table, max_pages, starts);
+    // the prefix sums in shared memory too (the W_UK staging area is idle in
+    // this block), so that the splits' searches read them there
+    int32_t* cu_s = reinterpret_cast<int32_t*>(&ws[0][0]);
+    int32_t* wsum = reinterpret_cast<int32_t*>(&qs[0][0]);
+    constexpr int kCuSmem = static_cast<int>(sizeof(ws) / sizeof(int32_t));
+    if (batch + 1 <= kCuSmem) {
+      page_prefix_sums_block(seq_lens, batch, page_size, cu, cu_s, wsum);
+      __syncthreads();   // the prefix sums are visible to the whole block
+      split_starts(cu_s, seq_lens, batch, num_splits, block_table, max_pages, starts);
+    } else {
+      page_prefix_sums(seq_lens, batch, page_size, cu);
+      __syncthreads();
+      split_starts(cu, seq_lens, batch, num_splits, block_table, max_pages, starts);
+    }
     return;
   }
   if (q == nullptr) return;  // cache-read test entry: prefix sums only
-  const int h = blockIdx.x % H, fc = (blockIdx.x / H) % nchunk, bg = blockIdx.x / (H * nchunk);
+  const int item = static_cast<int>(blockIdx.x) - 1;
+  const int h = item % H, fc = (item / H) % nchunk, bg = item / (H * nchunk);
   const int b0 = bg * kPBatch, nb = min(kPBatch, batch - b0);
   const int f0 = fc * kSumFeatures;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
