@@ -76,7 +76,7 @@ def parse():
                     help="timed steps (default 20000; 200 for layers24, 2000 per length for --sweep)")
     ap.add_argument("--warmup", type=int, default=30)
     ap.add_argument("--workload", default="c32k",
-                    choices=["c32k", "c4k", "ragged", "ragged_mla", "layers24", "layers24_full"])
+                    choices=["c32k", "c4k", "ragged", "ragged_mla", "layers24", "layers24_full", "r0"])
     ap.add_argument("--sweep", action="store_true",
                     help="decode throughput vs context length: batch 8, d_c 256, L = 1K .. 64K, one line per L")
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
@@ -641,8 +641,91 @@ def mla_baseline(case, torch, stream, peak, steps=600):
                          "bytes_per_launch": algo["total"], "bytes_breakdown": algo}}
 
 
+def run_gpu_r0(args, workload, torch, dist, ws, rank):
+    """The paper-literal (R0) gated decode, eg_mla_decode_r0, on the 4K-context
+    shapes at batch 8 (d_c 256, vocabulary 32000): the up-projection of every
+    cached row through W^UKV on tcgen05, the gate and LayerNorm over the 4096
+    features of all heads, per-head attention.  Reported against the bf16
+    tensor peak: the up-projection's FLOPs (2 x 4096 x d_c per cached token)
+    over the whole call's time, a lower bound for the projection kernel."""
+    from paper_2509_16686_gb300 import _lib, device, synth
+    dev = torch.cuda.current_device()
+    case = synth.case_c4k(batch=8, ctx=4096, keep_logical=False)
+    r0 = synth.make_r0_inputs(case, seed=61)
+    d = case.dims
+    units = []
+    for _ in range(REPLICAS):
+        dc = device.upload(case)
+        dc.append()
+        units.append(dc)
+    w_ukv = device.to_device_array(r0.w_ukv, "bf16", "cuda")
+    gate = device.to_device_array(r0.gate_r0, "bf16", "cuda")
+    gamma, beta = torch.from_numpy(r0.gamma).cuda(), torch.from_numpy(r0.beta).cuda()
+    wsb = torch.empty(_lib.eg_mla_decode_r0_workspace_size(units[0].dims, case.num_pages), dtype=torch.uint8,
+                      device="cuda")
+    out = torch.empty((case.batch, 16, 128), dtype=torch.bfloat16, device="cuda")
+    stream = torch.cuda.Stream()
+
+    def call(u):
+        _lib.eg_mla_decode_r0(u.dims, u.q, u.c_pool, u.kr_pool, u.id_pool, u.block_table, u.seq_lens, w_ukv, gate,
+                              gamma, beta, out, wsb, u.status, stream)
+
+    with torch.cuda.stream(stream):
+        for i in range(max(3, args.warmup)):
+            call(units[i % REPLICAS])
+    stream.synchronize()
+    assert units[0].read_status() == 0, "device status (R0)"
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        for u in units:
+            call(u)
+    steps = args.steps if args.steps is not None else 60
+    reps = max(1, steps // REPLICAS)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(nvsmi_id(torch, dev)) as clk:
+        with torch.cuda.stream(stream):
+            graph.replay()
+            e0.record(stream)
+            for _ in range(reps):
+                graph.replay()
+            e1.record(stream)
+        torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / (reps * REPLICAS)
+    assert units[0].read_status() == 0, "device status (R0)"
+    tokens = int(case.seq_lens.astype(np.int64).sum())
+    width = d.num_heads * (d.d_nope + d.d_v)
+    flops = 2.0 * tokens * width * d.d_c
+    peaks_path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(peaks_path):
+        peak, src = float(json.load(open(peaks_path))["bf16_tflops"]), "measured"
+    else:
+        peak, src = 1900.0, "fallback"
+    achieved = flops / (ms * 1e-3) / 1e12
+    return {
+        "metric": METRIC, "value": case.batch / (ms * 1e-3), "unit": UNIT, "n_gpus": ws,
+        "steps": reps * REPLICAS, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": "r0: the paper-literal gate placement (gate and LayerNorm over the 4096 "
+                               "up-projected key/value features of all heads), batch 8 x context 4096, 16 heads, "
+                               "d_c 256, vocabulary 32000; seeded synthetic W^UKV (the case's W_UK, W_UV), "
+                               "R0 gate table N(1, 0.1), gamma N(1, 0.1), beta N(0, 0.1)",
+                   "batch": case.batch, "ctx_tokens_cached": tokens,
+                   "l2": f"{REPLICAS} rotating cache replicas; the gated projections of the pool "
+                         f"({case.num_pages * 64 * width * 2 / 1e6:.0f} MB) are written and read every step"},
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "traffic": None, "kernel": "r0_project_kernel (+ r0_attend_kernel)",
+                     "flops_per_launch": flops, "peak_source": src,
+                     "note": "up-projection FLOPs over the whole call (both kernels): a lower bound for the "
+                             "projection kernel's tensor rate"},
+        "gpu_launches": 2 * reps * REPLICAS,
+        "clocks": clk.summary(),
+    }
+
+
 def run_gpu(args, workload, torch, dist, ws, rank):
     """One bench line of `workload` (see the module docstring)."""
+    if workload == "r0":
+        return run_gpu_r0(args, workload, torch, dist, ws, rank)
     if workload == "layers24_full":
         return run_gpu_full_layers(args, workload, torch, dist, ws, rank)
     from paper_2509_16686_gb300 import _lib, device  # noqa: F401

@@ -398,6 +398,44 @@ int eg_mla_profile_begin(int32_t max_launches);
 int eg_mla_profile_end(double* ms_sum, int32_t* launches);
 
 /*
+ * eg_mla_decode_r0 - decode with the paper-literal gate placement (R0): the
+ * gate and the LayerNorm act on the up-projected keys and values of all heads
+ * at once (Section 3 Eq. 5 applied after Eq. 2, as the Appendix E listing
+ * does), kv~_j = LN_{H(d_n + d_v)}((W^UKV c_j) (*) G_R0[id_j]), split per head
+ * into k^C_j, v^C_j (Eq. 6); then u_h = sum_j softmax_j(s_j) v^C_j,h with
+ * s_j = ([k^C_j,h ; k^R_j] . q_h) / sqrt(d_n + d_r) (Eqs. 11-13, without
+ * weight absorption: the gate in this space cannot be folded into q).
+ *
+ * Supported: bf16, 16 heads, d_nope = d_v = 128, d_rope = 64, d_c in
+ * {192, 256} (EG_MLA_ERR_UNSUPPORTED otherwise).  dims->gate_mode is ignored;
+ * dims->ln_eps is the LayerNorm's epsilon (<= 0: 1e-5).
+ *
+ *   q, c_pool, krope_pool, id_pool, block_table, max_pages_per_seq,
+ *   seq_lens, batch, num_pages: as for eg_mla_decode (the cache after the
+ *              step's append; seq_lens include the new token)
+ *   w_ukv      [16 * 256, d_c] bf16: per head h its 128 key rows (W_UK,h),
+ *              then its 128 value rows (W_UV,h), the row order of the joint
+ *              up-projection in Appendix E
+ *   gate_r0    [vocab, 4096] bf16: the gate in that space per token id
+ *   ln_gamma_r0, ln_beta_r0  [4096] fp32, may be NULL (1, 0)
+ *   out        [batch, 16, 128] bf16
+ *   workspace  >= eg_mla_decode_r0_workspace_size(dims, num_pages) bytes,
+ *              256-byte aligned: the gated projections of every pool row
+ *              (4096 bf16 each) and their LayerNorm statistics
+ *
+ * Device errors: a page id outside [0, num_pages) or a token id outside
+ * [0, vocab) of a cached token is reported as EG_MLA_ERR_OUT_OF_RANGE (the
+ * gate then uses row 0); a timed-out pipeline wait as EG_MLA_ERR_TIMEOUT.
+ * All 16-byte-read arguments must be 16-byte aligned.
+ */
+size_t eg_mla_decode_r0_workspace_size(const eg_mla_dims* dims, int32_t num_pages);
+int eg_mla_decode_r0(const eg_mla_dims* dims, const void* q, const void* c_pool, const void* krope_pool,
+                     const int32_t* id_pool, const int32_t* block_table, int32_t max_pages_per_seq,
+                     const int32_t* seq_lens, int32_t batch, int32_t num_pages, const void* w_ukv,
+                     const void* gate_r0, const float* ln_gamma_r0, const float* ln_beta_r0, void* out,
+                     void* workspace, size_t workspace_bytes, int32_t* dev_status, void* stream);
+
+/*
  * eg_mla_debug_linear - the projection GEMM of eg_mla_layer_decode on its own
  * (a testing aid): out[b][n] = sum_j x[b][j] w[n][j] for b < batch,
  * n < n_out (Eq. 14 and the projections of Appendix C Eqs. 1, 8-10 are of

@@ -43,6 +43,8 @@ EXPORTED = [
     "eg_mla_decode",
     "eg_mla_decode_static",
     "eg_mla_step",
+    "eg_mla_decode_r0_workspace_size",
+    "eg_mla_decode_r0",
     "eg_mla_kv_bytes_per_token",
     "eg_mla_status_string",
     "eg_mla_debug_gather",
@@ -100,6 +102,10 @@ def _declare(lib: ctypes.CDLL) -> None:
     lib.eg_mla_step.argtypes = [D, P, P, P, P, P, P, P, P, P, I32, P, I32, I32, I32, P, P, P, P, P, P, I32, P, SZ,
                                 P, P]
     lib.eg_mla_step.restype = ctypes.c_int
+    lib.eg_mla_decode_r0_workspace_size.argtypes = [D, I32]
+    lib.eg_mla_decode_r0_workspace_size.restype = SZ
+    lib.eg_mla_decode_r0.argtypes = [D, P, P, P, P, P, I32, P, I32, I32, P, P, P, P, P, P, SZ, P, P]
+    lib.eg_mla_decode_r0.restype = ctypes.c_int
     lib.eg_mla_debug_linear.argtypes = [P, I32, I32, P, I32, P, I32, I32, P, P]
     lib.eg_mla_debug_linear.restype = ctypes.c_int
     lib.eg_mla_debug_linear_plan.argtypes = [I32, I32, I32, ctypes.POINTER(I32), ctypes.POINTER(I32),
@@ -326,6 +332,24 @@ def bind_step(dims: EgMlaDims, c_pool, krope_pool, id_pool, c_new, krope_new, id
     step.keepalive = (dims, c_pool, krope_pool, id_pool, c_new, krope_new, ids_new, positions, q, block_table,
                       seq_lens, gate_table, ln_gamma, ln_beta, w_uk, w_uv, out, workspace, dev_status)
     return step
+
+
+def eg_mla_decode_r0_workspace_size(dims: EgMlaDims, num_pages: int) -> int:
+    n = load().eg_mla_decode_r0_workspace_size(ctypes.byref(dims), num_pages)
+    if n == 0:
+        raise EgMlaError(EG_MLA_ERR_UNSUPPORTED, "eg_mla_decode_r0_workspace_size")
+    return int(n)
+
+
+def eg_mla_decode_r0(dims: EgMlaDims, q, c_pool, krope_pool, id_pool, block_table, seq_lens, w_ukv, gate_r0,
+                     ln_gamma, ln_beta, out, workspace, dev_status=None, stream=None) -> None:
+    """Paper-literal (R0) gated decode: see include/egmla.h."""
+    code = load().eg_mla_decode_r0(
+        ctypes.byref(dims), _ptr(q), _ptr(c_pool), _ptr(krope_pool), _ptr(id_pool), _ptr(block_table),
+        block_table.shape[1], _ptr(seq_lens), seq_lens.shape[0], c_pool.shape[0], _ptr(w_ukv), _ptr(gate_r0),
+        _ptr(ln_gamma), _ptr(ln_beta), _ptr(out), _ptr(workspace), workspace.numel() * workspace.element_size(),
+        _ptr(dev_status), _stream(stream))
+    _check(code, "eg_mla_decode_r0")
 
 
 def eg_mla_debug_linear(w, x, out, dev_status=None, stream=None) -> None:

@@ -488,6 +488,56 @@ int eg_mla_decode_static(const eg_mla_dims* dims, const void* q, const void* c_p
                        EG_MLA_STATIC_SCRATCH_BYTES, dev_status, stream);
 }
 
+size_t eg_mla_decode_r0_workspace_size(const eg_mla_dims* dims, int32_t num_pages) {
+  if (check_dims(dims) != EG_MLA_OK || num_pages <= 0) return 0;
+  if (dims->dtype != EG_MLA_BF16 || dims->d_nope != 128 || dims->d_v != 128 || (dims->d_c != 192 && dims->d_c != 256))
+    return 0;
+  return egmla::r0_workspace_bytes(num_pages);
+}
+
+int eg_mla_decode_r0(const eg_mla_dims* dims, const void* q, const void* c_pool, const void* krope_pool,
+                     const int32_t* id_pool, const int32_t* block_table, int32_t max_pages_per_seq,
+                     const int32_t* seq_lens, int32_t batch, int32_t num_pages, const void* w_ukv,
+                     const void* gate_r0, const float* ln_gamma_r0, const float* ln_beta_r0, void* out,
+                     void* workspace, size_t workspace_bytes, int32_t* dev_status, void* stream) {
+  int rc = check_dims(dims);
+  if (rc != EG_MLA_OK) return rc;
+  if (dims->dtype != EG_MLA_BF16 || dims->d_nope != 128 || dims->d_v != 128 || (dims->d_c != 192 && dims->d_c != 256))
+    return EG_MLA_ERR_UNSUPPORTED;
+  if (batch < 0 || num_pages <= 0 || max_pages_per_seq <= 0) return EG_MLA_ERR_INVALID_ARG;
+  if (batch == 0) return EG_MLA_OK;
+  if (!q || !c_pool || !krope_pool || !id_pool || !block_table || !seq_lens || !w_ukv || !gate_r0 || !out)
+    return EG_MLA_ERR_INVALID_ARG;
+  if (!aligned(q, 16) || !aligned(c_pool, 16) || !aligned(krope_pool, 16) || !aligned(w_ukv, 16) ||
+      !aligned(gate_r0, 16) || !aligned(out, 16))
+    return EG_MLA_ERR_INVALID_ARG;
+  if (static_cast<int64_t>(num_pages) * dims->page_size > INT32_MAX) return EG_MLA_ERR_UNSUPPORTED;
+  if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < egmla::r0_workspace_bytes(num_pages))
+    return EG_MLA_ERR_WORKSPACE;
+  egmla::R0Args a;
+  a.q = q;
+  a.c_pool = c_pool;
+  a.kr_pool = krope_pool;
+  a.id_pool = id_pool;
+  a.block_table = block_table;
+  a.seq_lens = seq_lens;
+  a.w_ukv = w_ukv;
+  a.gate_r0 = gate_r0;
+  a.ln_gamma = ln_gamma_r0;
+  a.ln_beta = ln_beta_r0;
+  a.out = out;
+  a.workspace = workspace;
+  a.status = dev_status;
+  a.d_c = dims->d_c;
+  a.vocab = dims->vocab;
+  a.batch = batch;
+  a.max_pages = max_pages_per_seq;
+  a.num_pages = num_pages;
+  a.eps = dims->ln_eps > 0.f ? dims->ln_eps : 1e-5f;
+  a.scale_log2 = resolve_scale(dims) * 1.4426950408889634f;
+  return to_status(egmla::launch_decode_r0(a, static_cast<cudaStream_t>(stream)));
+}
+
 int eg_mla_debug_linear(const void* w, int32_t n_out, int32_t k, const void* x, int32_t batch, void* out,
                         int32_t ldo, int32_t out_f32, int32_t* dev_status, void* stream) {
   if (n_out <= 0 || k <= 0 || batch < 0 || ldo < n_out || k % 8 != 0) return EG_MLA_ERR_INVALID_ARG;

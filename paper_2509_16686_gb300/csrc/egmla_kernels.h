@@ -84,6 +84,28 @@ cudaError_t launch_decode_tc(const DecodeArgs& a, const CUtensorMap* maps, bool 
 cudaError_t launch_decode_wide(const DecodeArgs& a, const CUtensorMap* maps, cudaStream_t st);
 // true if the bf16 tensor-core path has a kernel for these shapes
 bool tc_supported(int d_c, int gate);
+
+// R0 decode (egmla_r0.cu): bf16, 16 heads, d_n = d_v = 128, d_r = 64,
+// d_c in {192, 256}
+struct R0Args {
+  const void* q;
+  const void* c_pool;
+  const void* kr_pool;
+  const int32_t* id_pool;
+  const int32_t* block_table;
+  const int32_t* seq_lens;
+  const void* w_ukv;     // [16 * 256, d_c]: per head its 128 key rows, then its 128 value rows
+  const void* gate_r0;   // [vocab, 4096]
+  const float* ln_gamma;
+  const float* ln_beta;
+  void* out;
+  void* workspace;
+  int32_t* status;
+  int d_c, vocab, batch, max_pages, num_pages;
+  float eps, scale_log2;
+};
+size_t r0_workspace_bytes(int num_pages);
+cudaError_t launch_decode_r0(const R0Args& a, cudaStream_t st);
 // out[b][n] = sum_k x[b][k] W[n][k] for b < batch, n < n_out: W [n_out, k] and
 // x [batch, k] bf16 row-major (16-byte aligned, k % 8 == 0), out fp32 or
 // bf16 with row stride ldo elements (egmla_linear.cu).  Launched with

@@ -319,6 +319,32 @@ class LayerCase:
     rms_eps: float = F32_EPS
 
 
+@dataclasses.dataclass
+class R0Inputs:
+    """The extra inputs of the paper-literal (R0) gate placement: the joint
+    up-projection W^UKV (per head its key rows W_UK,h, then its value rows
+    W_UV,h: the case's own weights in the row order of Appendix E), a gate
+    table in that H (d_n + d_v)-wide space, and its LayerNorm's gamma, beta."""
+    w_ukv: np.ndarray      # [H (d_n + d_v), d_c] model dtype bits
+    gate_r0: np.ndarray    # [V, H (d_n + d_v)] model dtype bits
+    gamma: np.ndarray      # [H (d_n + d_v)] float32
+    beta: np.ndarray       # [H (d_n + d_v)] float32
+
+
+def make_r0_inputs(case: Case, *, seed: int, affine: bool = True) -> R0Inputs:
+    """Seeded R0 inputs for `case`: gate table N(1, 0.1) like the latent gate
+    table, gamma N(1, 0.1) and beta N(0, 0.1) (or 1 and 0)."""
+    d = case.dims
+    rng = np.random.default_rng(seed)
+    width = d.num_heads * (d.d_nope + d.d_v)
+    w_ukv = np.concatenate([case.w_uk, case.w_uv], axis=1).reshape(width, d.d_c)
+    gate = _store(_normal(rng, (d.vocab, width), 0.1, mean=1.0), d.dtype)
+    gamma = _normal(rng, (width,), 0.1, mean=1.0) if affine else np.ones(width, np.float32)
+    beta = _normal(rng, (width,), 0.1) if affine else np.zeros(width, np.float32)
+    return R0Inputs(w_ukv=np.ascontiguousarray(w_ukv), gate_r0=gate, gamma=np.asarray(gamma, np.float32),
+                    beta=np.asarray(beta, np.float32))
+
+
 def make_layer_case(case: Case, n_embd: int, *, seed: int, rope_theta: float = 10000.0,
                     rms_eps: float = F32_EPS) -> LayerCase:
     """Hidden state N(0, 1) and projection weights N(0, fan_in^-1/2); the
