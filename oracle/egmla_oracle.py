@@ -26,8 +26,12 @@ paper's printed cache sizes).  The attention-layer step (``layer_step``,
 ``layer_decode``) is pinned by decoding a sequence one token at a time against
 one causal forward pass over the whole sequence written from the listing, and
 its RoPE, RMSNorm and bf16 storage against the corresponding torch routines.
-``decode_r0`` (no GPU path; the paper prints no numeric example of it) is
-pinned against a PyTorch re-expression of the paper's listing, a single-token
+``prefill`` (every position of a prompt at once) is pinned row by row against
+``decode_unabsorbed`` on the cache holding the prompt up to that row, against
+torch's causal scaled_dot_product_attention where the projections are
+identities, by a one-token closed form, the causal running mean at q = 0, and
+causality and prompt-independence invariants.  ``decode_r0`` (the paper
+prints no numeric example of it) is pinned against a PyTorch re-expression of the paper's listing, a single-token
 closed form, invariance under permuting cached positions, and its reduction to
 the latent-gated form when the joint up-projection is the identity.
 """
@@ -292,6 +296,77 @@ def decode_r0(case, w_ukv_full: Optional[np.ndarray] = None, gate_r0: Optional[n
             p = softmax((k @ widen(case.q[b, h], d.dtype)) * softmax_scale(d))
             out[b, h] = p @ v
     return out
+
+
+# --------------------------------------------------------------------------
+# prompt processing (prefill): causal attention over every prompt position
+# --------------------------------------------------------------------------
+def prefill_latents(pc, b: int):
+    """(c~ [L, d_c], k^R [L, d_r]) of prompt b: its packed rows, gated as the
+    decode path gates cached rows (Eq. 5 in latent space, or the ablations)."""
+    d = pc.dims
+    s0, s1 = int(pc.cu_seqlens[b]), int(pc.cu_seqlens[b + 1])
+    c = widen(pc.c[s0:s1], d.dtype)
+    kr = widen(pc.kr[s0:s1], d.dtype)
+    if d.gate and s1 > s0:
+        g = widen(pc.gate_table, d.dtype)[pc.ids[s0:s1].astype(np.int64)]
+        c = gate_latents(c, g, np.asarray(pc.ln_gamma, np.float64), np.asarray(pc.ln_beta, np.float64),
+                         d.ln_eps, getattr(d, "gate_op", "mul_ln"))
+    return c, kr
+
+
+def future_positions(L: int) -> np.ndarray:
+    """[L, L] mask of the (query t, key j) pairs with j > t: the keys a query
+    of a prompt does not see (the sum of Eq. 13 stops at the query's own
+    position, which it includes)."""
+    return np.triu(np.ones((L, L), dtype=bool), k=1)
+
+
+def prefill(pc, batches: Optional[Iterable[int]] = None, heads: Optional[Iterable[int]] = None) -> np.ndarray:
+    """u_{t,i} = sum_{j <= t} softmax_j(q_{t,i} . k_{j,i} / sqrt(d_h + d_h^R)) v_{j,i}
+    for every position t of every prompt (Eq. 13, whose sum runs over the
+    positions up to the query's own), with k_{j,i} = [W_UK,i c~_j ; k^R_j] and
+    v_{j,i} = W_UV,i c~_j (Eqs. 2, 6, 12) up-projected from the gated latent:
+    the unabsorbed per-head form of the Appendix E listing applied to a whole
+    prompt at once, the causal mask written as a full score matrix with the
+    entries above the diagonal removed.  Returns [T, H, d_v] float64 (rows of
+    unselected prompts or heads NaN)."""
+    d = pc.dims
+    T, H = pc.total_tokens, d.num_heads
+    out = np.full((T, H, d.d_v), np.nan)
+    bs = range(pc.batch) if batches is None else list(batches)
+    hs = range(H) if heads is None else list(heads)
+    for b in bs:
+        s0, s1 = int(pc.cu_seqlens[b]), int(pc.cu_seqlens[b + 1])
+        L = s1 - s0
+        if L == 0:
+            continue
+        c_t, kr = prefill_latents(pc, b)
+        future = future_positions(L)
+        for h in hs:
+            k = np.concatenate([c_t @ widen(pc.w_uk[h], d.dtype).T, kr], axis=1)   # [L, d_n + d_r]
+            v = c_t @ widen(pc.w_uv[h], d.dtype).T                                   # [L, d_v]
+            q = widen(pc.q[s0:s1, h], d.dtype)                                      # [L, d_n + d_r]
+            s = (q @ k.T) * softmax_scale(d)
+            s[future] = -np.inf
+            out[s0:s1, h] = softmax(s) @ v
+    return out
+
+
+def prefill_pools(pc):
+    """The paged cache after the prompts are written into it: token t of
+    prompt b goes to logical position t through the block table (the decode
+    steps that follow read it there).  Returns new arrays."""
+    c_pool, kr_pool, id_pool = pc.c_pool.copy(), pc.kr_pool.copy(), pc.id_pool.copy()
+    P = pc.dims.page_size
+    for b in range(pc.batch):
+        s0, s1 = int(pc.cu_seqlens[b]), int(pc.cu_seqlens[b + 1])
+        for t in range(s1 - s0):
+            page, slot = paged_position(pc.block_table, b, t, P)
+            c_pool[page, slot] = pc.c[s0 + t]
+            kr_pool[page, slot] = pc.kr[s0 + t]
+            id_pool[page, slot] = pc.ids[s0 + t]
+    return c_pool, kr_pool, id_pool
 
 
 # --------------------------------------------------------------------------

@@ -361,3 +361,114 @@ def make_layer_case(case: Case, n_embd: int, *, seed: int, rope_theta: float = 1
         kv_norm_w=_store(_normal(rng, (dc,), 0.1, mean=1.0), dt),
         w_o=_store(_normal(rng, (E, H * dv), (H * dv) ** -0.5), dt),
         rope_theta=rope_theta, rms_eps=rms_eps)
+
+
+# --------------------------------------------------------------------------
+# prompt processing (prefill): prompts packed one after another
+# --------------------------------------------------------------------------
+@dataclasses.dataclass
+class PrefillCase:
+    """One prefill call: B prompts packed token after token (prompt b holds
+    rows ``cu_seqlens[b] .. cu_seqlens[b+1]-1`` of every per-token array), the
+    layer's gate table, LayerNorm and up-projections, and an empty paged cache
+    (NaN latents, out-of-range ids) that the call fills with the prompts.
+    Arrays of the model dtype are stored as in ``Case``."""
+    name: str
+    dims: Dims
+    seed: int
+    seq_lens: np.ndarray      # [B] int32
+    cu_seqlens: np.ndarray    # [B + 1] int32
+    q: np.ndarray             # [T, H, d_nope + d_rope], RoPE already applied
+    c: np.ndarray             # [T, d_c]
+    kr: np.ndarray            # [T, d_r]
+    ids: np.ndarray           # [T] int32
+    gate_table: np.ndarray    # [V, d_c]
+    ln_gamma: np.ndarray      # [d_c] float32
+    ln_beta: np.ndarray       # [d_c] float32
+    w_uk: np.ndarray          # [H, d_nope, d_c]
+    w_uv: np.ndarray          # [H, d_v, d_c]
+    c_pool: np.ndarray        # [num_pages, P, d_c]
+    kr_pool: np.ndarray       # [num_pages, P, d_r]
+    id_pool: np.ndarray       # [num_pages, P] int32
+    block_table: np.ndarray   # [B, max_pages] int32
+
+    @property
+    def batch(self) -> int:
+        return int(self.seq_lens.shape[0])
+
+    @property
+    def total_tokens(self) -> int:
+        return int(self.cu_seqlens[-1])
+
+    @property
+    def num_pages(self) -> int:
+        return int(self.c_pool.shape[0])
+
+    @property
+    def max_pages(self) -> int:
+        return int(self.block_table.shape[1])
+
+
+def make_prefill_case(name: str, dims: Dims, seq_lens, *, seed: int, latent_scale: float = 0.5,
+                      id_dist: str = "uniform", affine_ln: bool = False, extra_pages: int = 0,
+                      q_zero: bool = False) -> PrefillCase:
+    """Seeded prompts with the value distributions of the decode workloads; the
+    cache pages of all prompts are shuffled over one pool (plus ``extra_pages``
+    unused ones)."""
+    rng = np.random.default_rng(seed)
+    P = dims.page_size
+    seq_lens = np.asarray(seq_lens, dtype=np.int32)
+    B = seq_lens.shape[0]
+    cu = np.zeros(B + 1, dtype=np.int32)
+    cu[1:] = np.cumsum(seq_lens)
+    T = int(cu[-1])
+    npg = [(int(L) + P - 1) // P for L in seq_lens]
+    max_pages = max(max(npg) if npg else 1, 1)
+    num_pages = max(int(sum(npg)) + int(extra_pages), 1)
+    perm = rng.permutation(num_pages).astype(np.int32)
+    block_table = np.full((B, max_pages), perm[-1], dtype=np.int32)
+    k = 0
+    for b in range(B):
+        block_table[b, :npg[b]] = perm[k:k + npg[b]]
+        k += npg[b]
+
+    dt = dims.dtype
+    H, dn, dr, dv, dc, V = dims.num_heads, dims.d_nope, dims.d_rope, dims.d_v, dims.d_c, dims.vocab
+    c = _store(_normal(rng, (T, dc), latent_scale), dt)
+    kr = _store(_normal(rng, (T, dr), 1.0), dt)
+    ids = zipf_ids(rng, T, V) if id_dist == "zipf" else rng.integers(0, V, size=T, dtype=np.int64).astype(np.int32)
+    q = _normal(rng, (T, H, dn + dr), 1.0)
+    if q_zero:
+        q[:] = 0.0
+    q = _store(q, dt)
+    gate_table = _store(_normal(rng, (V, dc), 0.1, mean=1.0), dt)
+    wstd = dc ** -0.5
+    w_uk = _store(_normal(rng, (H, dn, dc), wstd), dt)
+    w_uv = _store(_normal(rng, (H, dv, dc), wstd), dt)
+    if affine_ln:
+        ln_gamma = _normal(rng, (dc,), 0.1, mean=1.0)
+        ln_beta = _normal(rng, (dc,), 0.1)
+    else:
+        ln_gamma = np.ones((dc,), dtype=np.float32)
+        ln_beta = np.zeros((dc,), dtype=np.float32)
+    c_pool = np.full((num_pages, P, dc), _nan_fill(dt), dtype=np.uint16 if dt == "bf16" else np.float32)
+    kr_pool = np.full((num_pages, P, dr), _nan_fill(dt), dtype=c_pool.dtype)
+    id_pool = np.full((num_pages, P), -7, dtype=np.int32)
+    return PrefillCase(name=name, dims=dims, seed=seed, seq_lens=seq_lens, cu_seqlens=cu, q=q, c=c, kr=kr,
+                       ids=ids.astype(np.int32), gate_table=gate_table, ln_gamma=np.asarray(ln_gamma, np.float32),
+                       ln_beta=np.asarray(ln_beta, np.float32), w_uk=w_uk, w_uv=w_uv, c_pool=c_pool,
+                       kr_pool=kr_pool, id_pool=id_pool, block_table=block_table)
+
+
+def case_prefill(seed: int = 5, batch: int = 8, prompt: int = 4096, **kw) -> PrefillCase:
+    """bf16, 8 prompts of 4096 tokens, 16 heads, d_c 256, vocab 32000 (the
+    shapes of the 4K decode workload)."""
+    return make_prefill_case("prefill", dims_bf16(), [prompt] * batch, seed=seed, **kw)
+
+
+def case_prefill_ragged(seed: int = 6, batch: int = 16, lo: int = 128, hi: int = 4096, **kw) -> PrefillCase:
+    """bf16, 16 prompts with log-uniform lengths in [128, 4096], d_c 192,
+    vocab 50000, Zipf(1.1) ids (the shapes of the ragged decode workload)."""
+    lens = log_uniform_lengths(np.random.default_rng(seed + 1000), batch, lo, hi)
+    kw.setdefault("id_dist", "zipf")
+    return make_prefill_case("prefill_ragged", dims_bf16(d_c=192, vocab=50000), lens, seed=seed, **kw)
