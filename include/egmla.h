@@ -436,6 +436,58 @@ int eg_mla_decode_r0(const eg_mla_dims* dims, const void* q, const void* c_pool,
                      void* workspace, size_t workspace_bytes, int32_t* dev_status, void* stream);
 
 /*
+ * eg_mla_prefill - prompt processing: causal attention of every prompt
+ * position over the prompt up to and including itself, and the prompt written
+ * into the paged latent cache for the decode steps that follow.
+ *
+ * For prompt b (packed rows cu_seqlens[b] .. cu_seqlens[b+1] - 1), position t
+ * and head h, with c~_j the gated latent of position j as in eg_mla_decode
+ * (the gate mode's form of Section 3 Eq. 5 in latent space):
+ *   k_j,h = [W_UK,h c~_j ; k^R_j],  v_j,h = W_UV,h c~_j        (Eqs. 2, 6, 12)
+ *   u_t,h = sum_{j <= t} softmax_j(q_t,h . k_j,h * scale) v_j,h  (Eq. 13)
+ * computed without weight absorption (the per-head keys and values are
+ * materialised once per token; Appendix E's form).  The new tokens' raw c,
+ * k^R and id are written to logical positions 0 .. L_b - 1 of prompt b.
+ *
+ * Supported: bf16, d_nope = d_v = 128, d_rope = 64, d_c a multiple of 64 up
+ * to 512, any number of heads, any gate mode, page size 64
+ * (EG_MLA_ERR_UNSUPPORTED otherwise).
+ *
+ *   q            [total_tokens, num_heads, d_nope + d_rope] bf16, RoPE already
+ *                applied to the last d_rope entries of every row
+ *   c_new        [total_tokens, d_c] bf16: each prompt token's c^KV (Eq. 1)
+ *   krope_new    [total_tokens, d_rope] bf16: its rotated k^R (Eq. 10)
+ *   ids_new      [total_tokens] int32 token ids (may be NULL with
+ *                EG_MLA_GATE_NONE)
+ *   cu_seqlens   [batch + 1] int32 on the device: cu_seqlens[0] = 0,
+ *                non-decreasing, cu_seqlens[batch] = total_tokens
+ *   max_seq_len  host-side bound of every prompt length (1 .. total_tokens)
+ *   gate_table, ln_gamma, ln_beta, w_uk, w_uv: as for eg_mla_decode
+ *   out          [total_tokens, num_heads, d_v] bf16, written
+ *   c_pool, krope_pool, id_pool, block_table, max_pages_per_seq, num_pages:
+ *                the paged cache as for eg_mla_append_latent; c_pool NULL
+ *                skips the cache write (the other four are then ignored);
+ *                id_pool may be NULL with EG_MLA_GATE_NONE
+ *   workspace    >= eg_mla_prefill_workspace_size(dims, total_tokens) bytes,
+ *                256-byte aligned: c~ of every token (d_c bf16) and its
+ *                per-head keys and values (num_heads * 256 bf16)
+ * All tensor arguments read or written in 16-byte pieces must be 16-byte
+ * aligned.  Host errors return at once (nothing launched).  Device errors go
+ * to *dev_status (may be NULL): a token id outside [0, vocab) (the gate then
+ * uses row 0), a page id outside [0, num_pages), a prompt past
+ * max_pages_per_seq pages, cu_seqlens inconsistent with total_tokens, or a
+ * prompt longer than max_seq_len (its rows past the bound are not computed)
+ * as EG_MLA_ERR_OUT_OF_RANGE; a timed-out pipeline wait as EG_MLA_ERR_TIMEOUT.
+ */
+size_t eg_mla_prefill_workspace_size(const eg_mla_dims* dims, int32_t total_tokens);
+int eg_mla_prefill(const eg_mla_dims* dims, const void* q, const void* c_new, const void* krope_new,
+                   const int32_t* ids_new, const int32_t* cu_seqlens, int32_t batch, int32_t total_tokens,
+                   int32_t max_seq_len, const void* gate_table, const float* ln_gamma, const float* ln_beta,
+                   const void* w_uk, const void* w_uv, void* out, void* c_pool, void* krope_pool,
+                   int32_t* id_pool, const int32_t* block_table, int32_t max_pages_per_seq, int32_t num_pages,
+                   void* workspace, size_t workspace_bytes, int32_t* dev_status, void* stream);
+
+/*
  * eg_mla_debug_linear - the projection GEMM of eg_mla_layer_decode on its own
  * (a testing aid): out[b][n] = sum_j x[b][j] w[n][j] for b < batch,
  * n < n_out (Eq. 14 and the projections of Appendix C Eqs. 1, 8-10 are of

@@ -45,6 +45,8 @@ EXPORTED = [
     "eg_mla_step",
     "eg_mla_decode_r0_workspace_size",
     "eg_mla_decode_r0",
+    "eg_mla_prefill_workspace_size",
+    "eg_mla_prefill",
     "eg_mla_kv_bytes_per_token",
     "eg_mla_status_string",
     "eg_mla_debug_gather",
@@ -106,6 +108,11 @@ def _declare(lib: ctypes.CDLL) -> None:
     lib.eg_mla_decode_r0_workspace_size.restype = SZ
     lib.eg_mla_decode_r0.argtypes = [D, P, P, P, P, P, I32, P, I32, I32, P, P, P, P, P, P, SZ, P, P]
     lib.eg_mla_decode_r0.restype = ctypes.c_int
+    lib.eg_mla_prefill_workspace_size.argtypes = [D, I32]
+    lib.eg_mla_prefill_workspace_size.restype = SZ
+    lib.eg_mla_prefill.argtypes = [D, P, P, P, P, P, I32, I32, I32, P, P, P, P, P, P, P, P, P, P, I32, I32,
+                                   P, SZ, P, P]
+    lib.eg_mla_prefill.restype = ctypes.c_int
     lib.eg_mla_debug_linear.argtypes = [P, I32, I32, P, I32, P, I32, I32, P, P]
     lib.eg_mla_debug_linear.restype = ctypes.c_int
     lib.eg_mla_debug_linear_plan.argtypes = [I32, I32, I32, ctypes.POINTER(I32), ctypes.POINTER(I32),
@@ -350,6 +357,28 @@ def eg_mla_decode_r0(dims: EgMlaDims, q, c_pool, krope_pool, id_pool, block_tabl
         _ptr(ln_gamma), _ptr(ln_beta), _ptr(out), _ptr(workspace), workspace.numel() * workspace.element_size(),
         _ptr(dev_status), _stream(stream))
     _check(code, "eg_mla_decode_r0")
+
+
+def eg_mla_prefill_workspace_size(dims: EgMlaDims, total_tokens: int) -> int:
+    n = load().eg_mla_prefill_workspace_size(ctypes.byref(dims), int(total_tokens))
+    if n == 0 and total_tokens > 0:
+        raise EgMlaError(EG_MLA_ERR_UNSUPPORTED, "eg_mla_prefill_workspace_size")
+    return int(n)
+
+
+def eg_mla_prefill(dims: EgMlaDims, q, c_new, krope_new, ids_new, cu_seqlens, max_seq_len, gate_table,
+                   ln_gamma, ln_beta, w_uk, w_uv, out, workspace, c_pool=None, krope_pool=None, id_pool=None,
+                   block_table=None, dev_status=None, stream=None) -> None:
+    """Prompt processing (causal attention over packed prompts, cache write):
+    see include/egmla.h.  Sizes are taken from the tensors: batch =
+    len(cu_seqlens) - 1, total_tokens = q.shape[0]."""
+    code = load().eg_mla_prefill(
+        ctypes.byref(dims), _ptr(q), _ptr(c_new), _ptr(krope_new), _ptr(ids_new), _ptr(cu_seqlens),
+        cu_seqlens.shape[0] - 1, q.shape[0], int(max_seq_len), _ptr(gate_table), _ptr(ln_gamma), _ptr(ln_beta),
+        _ptr(w_uk), _ptr(w_uv), _ptr(out), _ptr(c_pool), _ptr(krope_pool), _ptr(id_pool), _ptr(block_table),
+        block_table.shape[1] if block_table is not None else 0, c_pool.shape[0] if c_pool is not None else 0,
+        _ptr(workspace), workspace.numel() * workspace.element_size(), _ptr(dev_status), _stream(stream))
+    _check(code, "eg_mla_prefill")
 
 
 def eg_mla_debug_linear(w, x, out, dev_status=None, stream=None) -> None:

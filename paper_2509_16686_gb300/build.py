@@ -20,7 +20,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libegmla.so")
 
 SOURCES = ["egmla_api.cu", "egmla_aux.cu", "egmla_decode_tc.cu", "egmla_decode_wide.cu", "egmla_layer.cu",
-           "egmla_linear.cu", "egmla_r0.cu"]
+           "egmla_linear.cu", "egmla_prefill.cu", "egmla_r0.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -394,6 +394,20 @@ int decode_impl(const eg_mla_dims* dims, const void* q, const void* c_pool, cons
 
 }  // namespace
 
+namespace {
+// shapes the prefill kernels cover; EG_MLA_OK or the error code
+int check_prefill_dims(const eg_mla_dims* d) {
+  if (d == nullptr) return EG_MLA_ERR_INVALID_ARG;
+  if (d->num_heads <= 0 || d->d_nope <= 0 || d->d_rope <= 0 || d->d_v <= 0 || d->d_c <= 0 ||
+      d->page_size <= 0 || d->vocab <= 0)
+    return EG_MLA_ERR_INVALID_ARG;
+  if (d->gate_mode < EG_MLA_GATE_NONE || d->gate_mode > EG_MLA_GATE_ADD_LN) return EG_MLA_ERR_INVALID_ARG;
+  if (d->dtype != EG_MLA_BF16 || d->page_size != egmla::kPage) return EG_MLA_ERR_UNSUPPORTED;
+  if (!egmla::prefill_supported(d->d_nope, d->d_rope, d->d_v, d->d_c)) return EG_MLA_ERR_UNSUPPORTED;
+  return EG_MLA_OK;
+}
+}  // namespace
+
 extern "C" {
 
 const char* eg_mla_status_string(int status) {
@@ -536,6 +550,74 @@ int eg_mla_decode_r0(const eg_mla_dims* dims, const void* q, const void* c_pool,
   a.eps = dims->ln_eps > 0.f ? dims->ln_eps : 1e-5f;
   a.scale_log2 = resolve_scale(dims) * 1.4426950408889634f;
   return to_status(egmla::launch_decode_r0(a, static_cast<cudaStream_t>(stream)));
+}
+
+size_t eg_mla_prefill_workspace_size(const eg_mla_dims* dims, int32_t total_tokens) {
+  if (check_prefill_dims(dims) != EG_MLA_OK || total_tokens < 0) return 0;
+  return egmla::prefill_workspace_bytes(total_tokens, dims->num_heads, dims->d_c);
+}
+
+int eg_mla_prefill(const eg_mla_dims* dims, const void* q, const void* c_new, const void* krope_new,
+                   const int32_t* ids_new, const int32_t* cu_seqlens, int32_t batch, int32_t total_tokens,
+                   int32_t max_seq_len, const void* gate_table, const float* ln_gamma, const float* ln_beta,
+                   const void* w_uk, const void* w_uv, void* out, void* c_pool, void* krope_pool,
+                   int32_t* id_pool, const int32_t* block_table, int32_t max_pages_per_seq, int32_t num_pages,
+                   void* workspace, size_t workspace_bytes, int32_t* dev_status, void* stream) {
+  int rc = check_prefill_dims(dims);
+  if (rc != EG_MLA_OK) return rc;
+  if (batch < 0 || total_tokens < 0 || max_seq_len < 0) return EG_MLA_ERR_INVALID_ARG;
+  if (batch == 0 || total_tokens == 0) return EG_MLA_OK;
+  if (max_seq_len == 0 || max_seq_len > total_tokens) return EG_MLA_ERR_INVALID_ARG;
+  const bool gated = dims->gate_mode != EG_MLA_GATE_NONE;
+  if (!q || !c_new || !krope_new || !cu_seqlens || !w_uk || !w_uv || !out) return EG_MLA_ERR_INVALID_ARG;
+  if (gated && (!ids_new || !gate_table)) return EG_MLA_ERR_INVALID_ARG;
+  if (!aligned(q, 16) || !aligned(c_new, 16) || !aligned(krope_new, 16) || !aligned(w_uk, 16) ||
+      !aligned(w_uv, 16) || !aligned(out, 16) || (gated && !aligned(gate_table, 16)))
+    return EG_MLA_ERR_INVALID_ARG;
+  if (c_pool != nullptr) {
+    if (!krope_pool || !block_table || (gated && !id_pool) || max_pages_per_seq <= 0 || num_pages <= 0)
+      return EG_MLA_ERR_INVALID_ARG;
+    if (!aligned(c_pool, 16) || !aligned(krope_pool, 16)) return EG_MLA_ERR_INVALID_ARG;
+    if (static_cast<int64_t>(num_pages) * dims->page_size > INT32_MAX) return EG_MLA_ERR_UNSUPPORTED;
+  }
+  const int64_t qtiles = (static_cast<int64_t>(max_seq_len) + 127) / 128;
+  if (static_cast<int64_t>(batch) * dims->num_heads * qtiles > INT32_MAX) return EG_MLA_ERR_UNSUPPORTED;
+  if (workspace == nullptr || !aligned(workspace, 256) ||
+      workspace_bytes < egmla::prefill_workspace_bytes(total_tokens, dims->num_heads, dims->d_c))
+    return EG_MLA_ERR_WORKSPACE;
+  egmla::PrefillArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.q = q;
+  a.c = c_new;
+  a.kr = krope_new;
+  a.ids = ids_new;
+  a.cu_seqlens = cu_seqlens;
+  a.gate_table = gate_table;
+  a.ln_gamma = ln_gamma;
+  a.ln_beta = ln_beta;
+  a.w_uk = w_uk;
+  a.w_uv = w_uv;
+  a.out = out;
+  a.c_pool = c_pool;
+  a.kr_pool = c_pool ? krope_pool : nullptr;
+  a.id_pool = c_pool ? id_pool : nullptr;
+  a.block_table = block_table;
+  a.workspace = workspace;
+  a.status = dev_status;
+  a.H = dims->num_heads;
+  a.d_c = dims->d_c;
+  a.vocab = dims->vocab;
+  a.batch = batch;
+  a.total = total_tokens;
+  a.max_seq_len = max_seq_len;
+  a.max_pages = max_pages_per_seq;
+  a.num_pages = num_pages;
+  a.gate = gated ? 1 : 0;
+  a.gate_add = dims->gate_mode == EG_MLA_GATE_ADD_LN ? 1 : 0;
+  a.gate_ln = (dims->gate_mode == EG_MLA_GATE_MUL_LN || dims->gate_mode == EG_MLA_GATE_ADD_LN) ? 1 : 0;
+  a.eps = dims->ln_eps > 0.f ? dims->ln_eps : 1e-5f;
+  a.scale_log2 = resolve_scale(dims) * 1.4426950408889634f;
+  return to_status(egmla::launch_prefill(a, static_cast<cudaStream_t>(stream)));
 }
 
 int eg_mla_debug_linear(const void* w, int32_t n_out, int32_t k, const void* x, int32_t batch, void* out,

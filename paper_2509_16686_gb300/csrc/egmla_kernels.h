@@ -106,6 +106,35 @@ struct R0Args {
 };
 size_t r0_workspace_bytes(int num_pages);
 cudaError_t launch_decode_r0(const R0Args& a, cudaStream_t st);
+// Prefill (egmla_prefill.cu): bf16, d_n = d_v = 128, d_r = 64, d_c a
+// multiple of 64 up to 512, any head count.  Prompts packed row after row
+// (cu_seqlens [batch + 1] on the device); the pool pointers may be null (no
+// cache write).
+struct PrefillArgs {
+  const void* q;            // [total, H, d_n + d_r]
+  const void* c;            // [total, d_c]
+  const void* kr;           // [total, d_r]
+  const int32_t* ids;       // [total]
+  const int32_t* cu_seqlens;
+  const void* gate_table;
+  const float* ln_gamma;
+  const float* ln_beta;
+  const void* w_uk;
+  const void* w_uv;
+  void* out;                // [total, H, d_v]
+  void* c_pool;
+  void* kr_pool;
+  int32_t* id_pool;
+  const int32_t* block_table;
+  void* workspace;
+  int32_t* status;
+  int H, d_c, vocab, batch, total, max_seq_len, max_pages, num_pages;
+  int gate, gate_add, gate_ln;
+  float eps, scale_log2;
+};
+size_t prefill_workspace_bytes(int total_tokens, int H, int d_c);
+bool prefill_supported(int d_nope, int d_rope, int d_v, int d_c);
+cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st);
 // out[b][n] = sum_k x[b][k] W[n][k] for b < batch, n < n_out: W [n_out, k] and
 // x [batch, k] bf16 row-major (16-byte aligned, k % 8 == 0), out fp32 or
 // bf16 with row stride ldo elements (egmla_linear.cu).  Launched with

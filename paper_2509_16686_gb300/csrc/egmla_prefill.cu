@@ -1,0 +1,826 @@
+// egmla_prefill.cu - prompt processing (prefill): every position t of a prompt
+// attends causally to positions 0..t of the same prompt (Appendix C Eq. 13,
+// whose sum stops at the query's own position), and the prompt is written into
+// the paged latent cache for the decode steps that follow.
+//
+// Prefill is compute-bound (every query meets every earlier key), so it runs
+// in the unabsorbed per-head form of the Appendix E listing, which needs
+// 2 (d_n + d_r + d_v) = 640 flops per (query, key, head) instead of the
+// absorbed form's 2 (d_c + d_r + d_c) = 1152:
+//   prefill_gate_kernel  one warp per prompt token: c~ = LN(c (*) G[id]) (or the
+//                        gate mode's variant; Section 3 Eq. 5 in latent space),
+//                        rounded to bf16, and the raw c, k^R and id written to
+//                        the token's cache slot through the block table.
+//   prefill_kv_kernel    (tcgen05) [k^C_h ; v^C_h] = [W_UK,h ; W_UV,h] c~ for
+//                        128 tokens per CTA and every head h (Eqs. 2 and 6): M =
+//                        128 tokens, N = 256 (d_n key rows, then d_v value
+//                        rows), K = d_c, two TMEM accumulators so the epilogue
+//                        of head h overlaps the MMAs of head h + 1.
+//   prefill_attn_kernel  (tcgen05) flash attention: one CTA per (prompt, head,
+//                        128-query tile), walking the key tiles 0..qt of the
+//                        same prompt.  S = Q K^T (M = 128 queries, N = 128
+//                        keys, K = d_n + d_r, the RoPE part read from the
+//                        shared k^R rows) into one of two TMEM score buffers;
+//                        one softmax thread per query row (its TMEM lane) turns
+//                        S into P in bf16 in shared memory; O += P V (M = 128
+//                        queries, N = d_v, K = 128 keys, V read MN-major) in a
+//                        third TMEM buffer.  Scores of tile j + 1 are computed
+//                        while the softmax threads work on tile j.
+//
+// Warp roles of prefill_attn_kernel: warp 0 loads Q once and the key tiles
+// (two stages), warp 1 issues the MMAs, warps 2-5 run the softmax (warp w
+// owns TMEM lane quadrant w % 4) and the epilogue, warp 6 loads the value
+// tiles (one stage, refilled when the PV MMA that read it completes).
+//
+// Online softmax with a lazily moved reference: a row keeps the reference
+// maximum m of its exponentials until a tile's maximum exceeds it by more than
+// 2^8 (in log2 units 8); only then is O rescaled in TMEM.  Until then every
+// exponential is at most 2^8, exact enough in fp32 and bf16.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <mutex>
+
+#include "egmla_common.cuh"
+#include "egmla_kernels.h"
+#include "egmla_ptx.cuh"
+
+namespace egmla {
+namespace {
+
+constexpr int kPfRows = 128;                                // tokens per tile (the MMAs' M)
+constexpr int kPfChunk = 64;                                // elements per 128-byte swizzle row
+constexpr uint32_t kPfAtom = kPfRows * kPfChunk * 2;        // 16 KB: 128 rows x 64 bf16
+constexpr int kPfDn = 128, kPfDr = 64, kPfDv = 128;
+constexpr int kPfDqk = kPfDn + kPfDr;                       // 192: three 64-element chunks
+
+__device__ __forceinline__ float pf_ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+__device__ __forceinline__ bool pf_warp_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                             uint64_t limit_ns) {
+  __syncwarp();
+  const bool ok = mbar_wait(bar, parity, abort_flag, limit_ns);
+  return __all_sync(0xffffffffu, ok);
+}
+
+// prompt b of packed row t: the largest b with cu[b] <= t (empty prompts,
+// whose start equals the next one's, are passed over)
+__device__ __forceinline__ int prompt_of_row(const int32_t* cu, int batch, int t) {
+  int lo = 0, hi = batch - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (__ldg(cu + mid) <= t) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+// ============================================================================ 1. gate, LayerNorm, cache write
+struct PfGateParams {
+  const __nv_bfloat16* c;      // [T, d_c]
+  const __nv_bfloat16* kr;     // [T, d_r]
+  const int32_t* ids;          // [T] (null with the gate off)
+  const int32_t* cu;           // [batch + 1]
+  const __nv_bfloat16* gate_table;   // [vocab, d_c]
+  const float* gamma;                // [d_c] or null
+  const float* beta;
+  __nv_bfloat16* ctil;         // [T, d_c]
+  __nv_bfloat16* c_pool;       // null: no cache write
+  __nv_bfloat16* kr_pool;
+  int32_t* id_pool;
+  const int32_t* block_table;
+  int batch, total, d_c, d_r, vocab, max_pages, num_pages;
+  int gate, gate_add, gate_ln;
+  float eps;
+  int32_t* status;
+};
+
+constexpr int kGateWarps = 8;
+
+__global__ void __launch_bounds__(32 * kGateWarps) prefill_gate_kernel(const PfGateParams p) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int t = blockIdx.x * kGateWarps + warp;
+  if (t >= p.total) return;
+  const int b = prompt_of_row(p.cu, p.batch, t);
+  const int pos = t - __ldg(p.cu + b);
+  const int nu = p.d_c / 8;   // 16-byte units of a row (at most 64: two per lane)
+  bool bad = false;
+  int id = p.ids ? __ldg(p.ids + t) : 0;
+  if (p.gate && static_cast<unsigned>(id) >= static_cast<unsigned>(p.vocab)) {
+    bad = true;
+    id = 0;
+  }
+  uint4 craw[2];
+  float z[2][8];
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const int u = lane + 32 * i;
+    craw[i] = make_uint4(0u, 0u, 0u, 0u);
+    if (u < nu) craw[i] = __ldg(reinterpret_cast<const uint4*>(p.c + static_cast<size_t>(t) * p.d_c) + u);
+    const __nv_bfloat162* c2 = reinterpret_cast<const __nv_bfloat162*>(&craw[i]);
+    uint4 graw = make_uint4(0u, 0u, 0u, 0u);
+    if (p.gate && u < nu) graw = __ldg(reinterpret_cast<const uint4*>(p.gate_table + static_cast<size_t>(id) * p.d_c) + u);
+    const __nv_bfloat162* g2 = reinterpret_cast<const __nv_bfloat162*>(&graw);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float2 cf = __bfloat1622float2(c2[e]);
+      float2 v = cf;
+      if (p.gate) {
+        const float2 gf = __bfloat1622float2(g2[e]);
+        v = p.gate_add ? make_float2(cf.x + gf.x, cf.y + gf.y) : make_float2(cf.x * gf.x, cf.y * gf.y);
+      }
+      z[i][2 * e] = u < nu ? v.x : 0.f;
+      z[i][2 * e + 1] = u < nu ? v.y : 0.f;
+    }
+  }
+  if (p.gate && p.gate_ln) {
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < 2; ++i)
+#pragma unroll
+      for (int e = 0; e < 8; ++e) s += z[i][e];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    const float mu = s / p.d_c;
+    float q = 0.f;
+#pragma unroll
+    for (int i = 0; i < 2; ++i)
+      if (lane + 32 * i < nu)
+#pragma unroll
+        for (int e = 0; e < 8; ++e) q = fmaf(z[i][e] - mu, z[i][e] - mu, q);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
+    const float r = rsqrtf(q / p.d_c + p.eps);
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int u = lane + 32 * i;
+      if (u >= nu) continue;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        const float gm = p.gamma ? __ldg(p.gamma + 8 * u + e) : 1.f;
+        const float bt = p.beta ? __ldg(p.beta + 8 * u + e) : 0.f;
+        z[i][e] = fmaf((z[i][e] - mu) * r, gm, bt);
+      }
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const int u = lane + 32 * i;
+    if (u >= nu) continue;
+    uint4 o;
+    o.x = pack_bf16x2(z[i][0], z[i][1]);
+    o.y = pack_bf16x2(z[i][2], z[i][3]);
+    o.z = pack_bf16x2(z[i][4], z[i][5]);
+    o.w = pack_bf16x2(z[i][6], z[i][7]);
+    reinterpret_cast<uint4*>(p.ctil + static_cast<size_t>(t) * p.d_c)[u] = o;
+  }
+  if (p.c_pool) {
+    const int lp = pos / kPage;
+    const int page = lp < p.max_pages ? __ldg(p.block_table + static_cast<size_t>(b) * p.max_pages + lp) : -1;
+    if (page < 0 || page >= p.num_pages) {
+      bad = true;
+    } else {
+      const size_t slot = static_cast<size_t>(page) * kPage + pos % kPage;
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        const int u = lane + 32 * i;
+        if (u < nu) reinterpret_cast<uint4*>(p.c_pool + slot * p.d_c)[u] = craw[i];
+      }
+      if (lane < p.d_r / 8)
+        reinterpret_cast<uint4*>(p.kr_pool + slot * p.d_r)[lane] =
+            __ldg(reinterpret_cast<const uint4*>(p.kr + static_cast<size_t>(t) * p.d_r) + lane);
+      if (lane == 0 && p.id_pool && p.ids) p.id_pool[slot] = __ldg(p.ids + t);
+    }
+  }
+  if (bad && lane == 0) report_status(p.status, kStatusOutOfRange);
+}
+
+// ============================================================================ 2. key/value up-projection
+constexpr int kKvFeat = kPfDn + kPfDv;                      // 256 output features per head
+constexpr uint32_t kKvBBytes = kKvFeat * kPfChunk * 2;      // 32 KB: one K chunk of a head's rows
+constexpr int kKvStages = 3;
+constexpr int kKvEpiWarps = 8;                              // two per lane quadrant: key / value half
+constexpr int kKvThreads = 32 * (2 + kKvEpiWarps);          // warp 0 TMA, warp 1 MMA
+
+struct KvBars {
+  uint64_t afull;
+  uint64_t bfull[kKvStages], bempty[kKvStages];
+  uint64_t dfull[2], dfree[2];
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort;
+};
+
+struct KvParams {
+  __nv_bfloat16* kv;   // [T, H, 256]
+  int total, H, nkc;
+  uint64_t wait_ns;
+  int32_t* status;
+};
+
+__global__ void __launch_bounds__(kKvThreads, 1)
+    prefill_kv_kernel(const __grid_constant__ CUtensorMap cmap, const __grid_constant__ CUtensorMap wkmap,
+                      const __grid_constant__ CUtensorMap wvmap, const KvParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t b_off = static_cast<uint32_t>(p.nkc) * kPfAtom;
+  KvBars& bars = *reinterpret_cast<KvBars*>(smem + b_off + kKvStages * kKvBBytes);
+  volatile int* abort_flag = &bars.abort;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int row0 = blockIdx.x * kPfRows;
+  const int nsteps = p.H * p.nkc;
+
+  if (tid == 0) {
+    mbar_init(smem_u32(&bars.afull), 1);
+    for (int s = 0; s < kKvStages; ++s) {
+      mbar_init(smem_u32(&bars.bfull[s]), 1);
+      mbar_init(smem_u32(&bars.bempty[s]), 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(smem_u32(&bars.dfull[s]), 1);
+      mbar_init(smem_u32(&bars.dfree[s]), kKvEpiWarps);
+    }
+    mbar_init(smem_u32(&bars.drain), 1);
+    bars.abort = 0;
+    fence_mbar_init();
+    prefetch_tensormap(&cmap);
+    prefetch_tensormap(&wkmap);
+    prefetch_tensormap(&wvmap);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&bars.tmem_base), 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bars.tmem_base;
+
+  if (warp == 0) {
+    if (elect_one()) {
+      const uint64_t pol_stream = policy_evict_first(), pol_keep = policy_evict_last();
+      mbar_arrive_expect_tx(smem_u32(&bars.afull), static_cast<uint32_t>(p.nkc) * kPfAtom);
+      for (int kc = 0; kc < p.nkc; ++kc)
+        tma_load_2d(sbase + kc * kPfAtom, &cmap, kc * kPfChunk, row0, smem_u32(&bars.afull), pol_stream);
+      int issued = 0;
+      for (int i = 0; i < nsteps; ++i) {
+        const int s = i % kKvStages;
+        if (i >= kKvStages &&
+            !mbar_wait(smem_u32(&bars.bempty[s]), ((i / kKvStages) & 1) ^ 1, abort_flag, p.wait_ns))
+          break;
+        const int h = i / p.nkc, kc = i % p.nkc;
+        const uint32_t dst = sbase + b_off + s * kKvBBytes;
+        mbar_arrive_expect_tx(smem_u32(&bars.bfull[s]), kKvBBytes);
+        tma_load_2d(dst, &wkmap, kc * kPfChunk, h * kPfDn, smem_u32(&bars.bfull[s]), pol_keep);
+        tma_load_2d(dst + kKvBBytes / 2, &wvmap, kc * kPfChunk, h * kPfDv, smem_u32(&bars.bfull[s]), pol_keep);
+        issued = i + 1;
+      }
+      // every copy issued lands before the CTA can leave
+      volatile int own = 0;
+      if (!mbar_wait(smem_u32(&bars.afull), 0, &own, p.wait_ns)) *abort_flag = 1;
+      for (int i = issued > kKvStages ? issued - kKvStages : 0; i < issued; ++i)
+        if (!mbar_wait(smem_u32(&bars.bfull[i % kKvStages]), (i / kKvStages) & 1, &own, p.wait_ns))
+          *abort_flag = 1;
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    constexpr uint32_t idesc = idesc_bf16(kPfRows, kKvFeat, 0, 0);
+    bool ok = pf_warp_wait(smem_u32(&bars.afull), 0, abort_flag, p.wait_ns);
+    bool issued = false;
+    for (int h = 0; ok && h < p.H; ++h) {
+      const int db = h & 1;
+      if (h >= 2) ok = pf_warp_wait(smem_u32(&bars.dfree[db]), ((h - 2) >> 1) & 1, abort_flag, p.wait_ns);
+      for (int kc = 0; ok && kc < p.nkc; ++kc) {
+        const int i = h * p.nkc + kc, s = i % kKvStages;
+        ok = pf_warp_wait(smem_u32(&bars.bfull[s]), (i / kKvStages) & 1, abort_flag, p.wait_ns);
+        if (!ok) break;
+        tc_fence_after();
+        if (elect_one()) {
+          const uint64_t ad = smem_desc(sbase + kc * kPfAtom, 16, 1024, kSwizzle128B);
+          const uint64_t bd = smem_desc(sbase + b_off + s * kKvBBytes, 16, 1024, kSwizzle128B);
+#pragma unroll
+          for (int kk = 0; kk < kPfChunk / 16; ++kk)
+            mma_bf16_ss(tmem + db * kKvFeat, ad + ((kk * 32) >> 4), bd + ((kk * 32) >> 4), idesc,
+                        (kc > 0 || kk > 0) ? 1u : 0u);
+          mma_commit(smem_u32(&bars.bempty[s]));
+          if (kc == p.nkc - 1) mma_commit(smem_u32(&bars.dfull[db]));
+        }
+        __syncwarp();
+        issued = true;
+      }
+    }
+    if (issued) {
+      if (elect_one()) mma_commit(smem_u32(&bars.drain));
+      __syncwarp();
+      volatile int own = 0;
+      if (!mbar_wait(smem_u32(&bars.drain), 0, &own, p.wait_ns)) *abort_flag = 1;
+    }
+    __syncwarp();
+  } else {
+    // token row r = TMEM lane r; warps 2-5 store the key half (columns 0-127)
+    // of every head, warps 6-9 the value half
+    const int quad = warp & 3, half = (warp - 2) / 4;
+    const int r = 32 * quad + lane, row = row0 + r;
+    const bool live = row < p.total;
+    __nv_bfloat16* dst_row = p.kv + static_cast<size_t>(live ? row : 0) * p.H * kKvFeat + half * kPfDn;
+    bool ok = true;
+    for (int h = 0; h < p.H; ++h) {
+      const int db = h & 1;
+      ok = ok && pf_warp_wait(smem_u32(&bars.dfull[db]), (h >> 1) & 1, abort_flag, p.wait_ns);
+      if (!ok) break;
+      tc_fence_after();
+#pragma unroll
+      for (int c0 = 0; c0 < kPfDn; c0 += 32) {
+        float v[32];
+        const uint32_t ta = tmem + (static_cast<uint32_t>(32 * quad) << 16) + db * kKvFeat + half * kPfDn + c0;
+        tmem_ld16(ta, *reinterpret_cast<float(*)[16]>(&v[0]));
+        tmem_ld16(ta + 16, *reinterpret_cast<float(*)[16]>(&v[16]));
+        tmem_wait_ld();
+        if (live) {
+          uint4* d = reinterpret_cast<uint4*>(dst_row + static_cast<size_t>(h) * kKvFeat + c0);
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            d[q] = make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+                              pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&bars.dfree[db]));
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, 512);
+  if (tid == 0 && bars.abort) report_status(p.status, kStatusTimeout);
+}
+
+// ============================================================================ 3. causal flash attention
+constexpr int kAttnKStages = 2;
+constexpr uint32_t kAttnQBytes = 3 * kPfAtom;               // 48 KB: Q [128 x 192]
+constexpr uint32_t kAttnKBytes = 3 * kPfAtom;               // 48 KB: k^C [128 x 128] + k^R [128 x 64]
+constexpr uint32_t kAttnVBytes = 2 * kPfAtom;               // 32 KB: V [128 keys x 128]
+constexpr uint32_t kAttnPBytes = 2 * kPfAtom;               // 32 KB: P [128 queries x 128 keys]
+constexpr uint32_t kOffQ = 0;
+constexpr uint32_t kOffK = kOffQ + kAttnQBytes;
+constexpr uint32_t kOffV = kOffK + kAttnKStages * kAttnKBytes;
+constexpr uint32_t kOffP = kOffV + kAttnVBytes;
+constexpr uint32_t kOffBars = kOffP + kAttnPBytes;
+constexpr int kAttnVWarp = 6;
+constexpr int kAttnThreads = 32 * 7;
+constexpr uint32_t kColO = 2 * kPfRows;                     // TMEM: S0 at 0, S1 at 128, O at 256
+constexpr float kRescaleLog2 = 8.f;
+
+struct AttnBars {
+  uint64_t qfull;
+  uint64_t kfull[kAttnKStages], kempty[kAttnKStages];
+  uint64_t vfull;
+  uint64_t sfull[2], sfree[2];
+  uint64_t pfull, pvdone;
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort;
+};
+constexpr uint32_t kAttnSmem = kOffBars + sizeof(AttnBars) + 1024;
+
+struct AttnParams {
+  const int32_t* cu;
+  __nv_bfloat16* out;   // [T, H, d_v]
+  int batch, H, qtiles, total;
+  float scale_log2;
+  uint64_t wait_ns;
+  int32_t* status;
+};
+
+__global__ void __launch_bounds__(kAttnThreads, 1)
+    prefill_attn_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kvmap,
+                        const __grid_constant__ CUtensorMap krmap, const AttnParams p) {
+  // heaviest query tiles of a (prompt, head) first; the tiles of one (prompt,
+  // head) are neighbours in launch order, so its keys stay in L2 while read
+  const int group = blockIdx.x / p.qtiles;
+  const int qt = p.qtiles - 1 - blockIdx.x % p.qtiles;
+  const int b = group / p.H, h = group % p.H;
+  const int start = __ldg(p.cu + b);
+  const int L = __ldg(p.cu + b + 1) - start;
+  const int q0 = qt * kPfRows;
+  // prompt offsets that do not fit the packed rows, or a prompt longer than
+  // the host bound the grid was sized for: report, compute nothing past it
+  if (start < 0 || L < 0 || start > p.total - L || (qt == p.qtiles - 1 && L > p.qtiles * kPfRows)) {
+    if (threadIdx.x == 0) report_status(p.status, kStatusOutOfRange);
+    if (start < 0 || L < 0 || start > p.total - L) return;
+  }
+  if (q0 >= L) return;
+  const int nkt = qt + 1;   // key tiles 0..qt; the last one is the diagonal tile
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  const uint32_t sbase = smem_u32(smem);
+  AttnBars& bars = *reinterpret_cast<AttnBars*>(smem + kOffBars);
+  volatile int* abort_flag = &bars.abort;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+  if (tid == 0) {
+    mbar_init(smem_u32(&bars.qfull), 1);
+    for (int s = 0; s < kAttnKStages; ++s) {
+      mbar_init(smem_u32(&bars.kfull[s]), 1);
+      mbar_init(smem_u32(&bars.kempty[s]), 1);
+    }
+    mbar_init(smem_u32(&bars.vfull), 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(smem_u32(&bars.sfull[s]), 1);
+      mbar_init(smem_u32(&bars.sfree[s]), 4);
+    }
+    mbar_init(smem_u32(&bars.pfull), 4);
+    mbar_init(smem_u32(&bars.pvdone), 1);
+    mbar_init(smem_u32(&bars.drain), 1);
+    bars.abort = 0;
+    fence_mbar_init();
+    prefetch_tensormap(&qmap);
+    prefetch_tensormap(&kvmap);
+    prefetch_tensormap(&krmap);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&bars.tmem_base), 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bars.tmem_base;
+
+  if (warp == 0) {
+    // ---- Q once, then the key tiles: k^C of head h (two 64-column boxes of
+    // the kv buffer) and the shared k^R rows
+    if (elect_one()) {
+      const uint64_t pol_q = policy_evict_first(), pol_k = policy_evict_last();
+      mbar_arrive_expect_tx(smem_u32(&bars.qfull), kAttnQBytes);
+      for (int c = 0; c < 3; ++c)
+        tma_load_2d(sbase + kOffQ + c * kPfAtom, &qmap, h * kPfDqk + c * kPfChunk, start + q0,
+                    smem_u32(&bars.qfull), pol_q);
+      int issued = 0;
+      for (int j = 0; j < nkt; ++j) {
+        const int s = j % kAttnKStages;
+        if (j >= kAttnKStages &&
+            !mbar_wait(smem_u32(&bars.kempty[s]), ((j / kAttnKStages) & 1) ^ 1, abort_flag, p.wait_ns))
+          break;
+        const uint32_t dst = sbase + kOffK + s * kAttnKBytes;
+        const int y = start + j * kPfRows;
+        mbar_arrive_expect_tx(smem_u32(&bars.kfull[s]), kAttnKBytes);
+        tma_load_2d(dst, &kvmap, h * kKvFeat, y, smem_u32(&bars.kfull[s]), pol_k);
+        tma_load_2d(dst + kPfAtom, &kvmap, h * kKvFeat + kPfChunk, y, smem_u32(&bars.kfull[s]), pol_k);
+        tma_load_2d(dst + 2 * kPfAtom, &krmap, 0, y, smem_u32(&bars.kfull[s]), pol_k);
+        issued = j + 1;
+      }
+      volatile int own = 0;
+      if (!mbar_wait(smem_u32(&bars.qfull), 0, &own, p.wait_ns)) *abort_flag = 1;
+      for (int j = issued > kAttnKStages ? issued - kAttnKStages : 0; j < issued; ++j)
+        if (!mbar_wait(smem_u32(&bars.kfull[j % kAttnKStages]), (j / kAttnKStages) & 1, &own, p.wait_ns))
+          *abort_flag = 1;
+    }
+    __syncwarp();
+  } else if (warp == kAttnVWarp) {
+    // ---- value tiles: v^C of head h, one stage, refilled once the PV MMA
+    // that read the previous tile has completed
+    if (elect_one()) {
+      const uint64_t pol_v = policy_evict_last();
+      int issued = 0;
+      for (int j = 0; j < nkt; ++j) {
+        if (j >= 1 && !mbar_wait(smem_u32(&bars.pvdone), (j - 1) & 1, abort_flag, p.wait_ns)) break;
+        const int y = start + j * kPfRows;
+        mbar_arrive_expect_tx(smem_u32(&bars.vfull), kAttnVBytes);
+        tma_load_2d(sbase + kOffV, &kvmap, h * kKvFeat + kPfDn, y, smem_u32(&bars.vfull), pol_v);
+        tma_load_2d(sbase + kOffV + kPfAtom, &kvmap, h * kKvFeat + kPfDn + kPfChunk, y, smem_u32(&bars.vfull),
+                    pol_v);
+        issued = j + 1;
+      }
+      volatile int own = 0;
+      if (issued > 0 && !mbar_wait(smem_u32(&bars.vfull), (issued - 1) & 1, &own, p.wait_ns)) *abort_flag = 1;
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ---- MMAs: S(j) into score buffer j % 2, then O += P(j - 1) V(j - 1)
+    constexpr uint32_t idesc_s = idesc_bf16(kPfRows, kPfRows, 0, 0);
+    constexpr uint32_t idesc_o = idesc_bf16(kPfRows, kPfDv, 0, 1);
+    const uint64_t qdesc = smem_desc(sbase + kOffQ, 16, 1024, kSwizzle128B);
+    const uint64_t kdesc = smem_desc(sbase + kOffK, 16, 1024, kSwizzle128B);
+    const uint64_t pdesc = smem_desc(sbase + kOffP, 16, 1024, kSwizzle128B);
+    // V [keys x features] is the B operand MN-major: 64-feature atoms 16 KB
+    // apart, 8-key groups 1 KB apart
+    const uint64_t vdesc = smem_desc(sbase + kOffV, kPfAtom, 1024, kSwizzle128B);
+    bool ok = pf_warp_wait(smem_u32(&bars.qfull), 0, abort_flag, p.wait_ns);
+    bool issued = false;
+    auto issue_pv = [&](int i) {
+      ok = ok && pf_warp_wait(smem_u32(&bars.vfull), i & 1, abort_flag, p.wait_ns);
+      ok = ok && pf_warp_wait(smem_u32(&bars.pfull), i & 1, abort_flag, p.wait_ns);
+      if (!ok) return;
+      tc_fence_after();
+      if (elect_one()) {
+#pragma unroll
+        for (int ks = 0; ks < kPfRows / 16; ++ks)
+          mma_bf16_ss(tmem + kColO, pdesc + (((ks >> 2) * kPfAtom + (ks & 3) * 32) >> 4),
+                      vdesc + ((ks * 2048) >> 4), idesc_o, (i > 0 || ks > 0) ? 1u : 0u);
+        mma_commit(smem_u32(&bars.pvdone));
+      }
+      __syncwarp();
+      issued = true;
+    };
+    for (int j = 0; ok && j < nkt; ++j) {
+      const int s = j % kAttnKStages, sb = j & 1;
+      ok = pf_warp_wait(smem_u32(&bars.kfull[s]), (j / kAttnKStages) & 1, abort_flag, p.wait_ns);
+      if (ok && j >= 2) ok = pf_warp_wait(smem_u32(&bars.sfree[sb]), ((j - 2) >> 1) & 1, abort_flag, p.wait_ns);
+      if (!ok) break;
+      tc_fence_after();
+      if (elect_one()) {
+        const uint64_t kd = kdesc + ((s * kAttnKBytes) >> 4);
+#pragma unroll
+        for (int kk = 0; kk < kPfDqk / 16; ++kk)
+          mma_bf16_ss(tmem + sb * kPfRows, qdesc + (((kk >> 2) * kPfAtom + (kk & 3) * 32) >> 4),
+                      kd + (((kk >> 2) * kPfAtom + (kk & 3) * 32) >> 4), idesc_s, kk > 0 ? 1u : 0u);
+        mma_commit(smem_u32(&bars.kempty[s]));
+        mma_commit(smem_u32(&bars.sfull[sb]));
+      }
+      __syncwarp();
+      issued = true;
+      if (j >= 1) issue_pv(j - 1);
+    }
+    if (ok) issue_pv(nkt - 1);
+    if (issued) {
+      if (elect_one()) mma_commit(smem_u32(&bars.drain));
+      __syncwarp();
+      volatile int own = 0;
+      if (!mbar_wait(smem_u32(&bars.drain), 0, &own, p.wait_ns)) *abort_flag = 1;
+    }
+    __syncwarp();
+  } else {
+    // ---- softmax and epilogue: query row r = TMEM lane r
+    const int quad = warp & 3;
+    const int r = 32 * quad + lane;
+    const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * quad) << 16);
+    const float sl2 = p.scale_log2;
+    // this row's place in the swizzled P tile: 8-row group, row in group
+    const uint32_t prow = sbase + kOffP + (r >> 3) * 1024 + (r & 7) * 128;
+    float m_ref = 0.f, l = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nkt; ++j) {
+      const int sb = j & 1;
+      ok = pf_warp_wait(smem_u32(&bars.sfull[sb]), (j >> 1) & 1, abort_flag, p.wait_ns);
+      if (!ok) break;
+      tc_fence_after();
+      float sv[kPfRows];
+#pragma unroll
+      for (int c = 0; c < kPfRows; c += 16)
+        tmem_ld16(lane_base + sb * kPfRows + c, *reinterpret_cast<float(*)[16]>(&sv[c]));
+      tmem_wait_ld();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&bars.sfree[sb]));
+      if (j == nkt - 1) {
+        // diagonal tile: key c is after query r when c > r
+#pragma unroll
+        for (int c = 0; c < kPfRows; ++c)
+          if (c > r) sv[c] = -INFINITY;
+      }
+      float mx = sv[0];
+#pragma unroll
+      for (int c = 1; c < kPfRows; ++c) mx = fmaxf(mx, sv[c]);
+      mx *= sl2;
+      float alpha = 1.f;
+      if (j == 0) {
+        m_ref = mx;
+      } else if (mx > m_ref + kRescaleLog2) {
+        alpha = pf_ex2(m_ref - mx);
+        m_ref = mx;
+      }
+      uint32_t pk[kPfRows / 2];
+      float rs = 0.f;
+#pragma unroll
+      for (int c = 0; c < kPfRows; c += 2) {
+        const float p0 = pf_ex2(fmaf(sv[c], sl2, -m_ref));
+        const float p1 = pf_ex2(fmaf(sv[c + 1], sl2, -m_ref));
+        rs += p0 + p1;
+        pk[c / 2] = pack_bf16x2(p0, p1);
+      }
+      l = fmaf(l, alpha, rs);
+      // P is single-buffered and O is updated by the previous tile's PV MMA:
+      // both wait for it
+      if (j >= 1) {
+        ok = pf_warp_wait(smem_u32(&bars.pvdone), (j - 1) & 1, abort_flag, p.wait_ns);
+        if (!ok) break;
+        tc_fence_after();
+        if (__any_sync(0xffffffffu, alpha != 1.f)) {
+#pragma unroll
+          for (int c = 0; c < kPfDv; c += 16) {
+            float o[16];
+            tmem_ld16(lane_base + kColO + c, o);
+            tmem_wait_ld();
+#pragma unroll
+            for (int e = 0; e < 16; ++e) o[e] *= alpha;
+            tmem_st16(lane_base + kColO + c, o);
+          }
+          tmem_wait_st();
+        }
+      }
+#pragma unroll
+      for (int kc = 0; kc < 2; ++kc)
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const uint32_t a = prow + kc * kPfAtom + ((u ^ (r & 7)) << 4);
+          const int w = kc * 32 + 4 * u;
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(pk[w]), "r"(pk[w + 1]),
+                       "r"(pk[w + 2]), "r"(pk[w + 3])
+                       : "memory");
+        }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&bars.pfull));
+    }
+    // ---- epilogue: O / l of the live rows
+    if (ok) ok = pf_warp_wait(smem_u32(&bars.pvdone), (nkt - 1) & 1, abort_flag, p.wait_ns);
+    if (ok) {
+      tc_fence_after();
+      const float inv = 1.f / l;
+      const bool live = q0 + r < L;
+      __nv_bfloat16* orow = p.out + (static_cast<size_t>(start + q0 + (live ? r : 0)) * p.H + h) * kPfDv;
+#pragma unroll
+      for (int c = 0; c < kPfDv; c += 32) {
+        float o[32];
+        tmem_ld16(lane_base + kColO + c, *reinterpret_cast<float(*)[16]>(&o[0]));
+        tmem_ld16(lane_base + kColO + c + 16, *reinterpret_cast<float(*)[16]>(&o[16]));
+        tmem_wait_ld();
+        if (live) {
+          uint4* d = reinterpret_cast<uint4*>(orow + c);
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            d[q] = make_uint4(pack_bf16x2(o[8 * q] * inv, o[8 * q + 1] * inv),
+                              pack_bf16x2(o[8 * q + 2] * inv, o[8 * q + 3] * inv),
+                              pack_bf16x2(o[8 * q + 4] * inv, o[8 * q + 5] * inv),
+                              pack_bf16x2(o[8 * q + 6] * inv, o[8 * q + 7] * inv));
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, 512);
+  if (tid == 0 && bars.abort) report_status(p.status, kStatusTimeout);
+}
+
+// ---------------------------------------------------------------- host
+using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                              const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                              CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeFn pf_encode_fn() {
+  static EncodeFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeFn>(ptr);
+  });
+  return fn;
+}
+
+// row-major bf16 [rows, cols] with row stride `ld` elements; boxes of 64
+// columns x 128 rows, 128-byte swizzle, rows past the end read as zero
+bool pf_encode(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld) {
+  EncodeFn enc = pf_encode_fn();
+  if (enc == nullptr) return false;
+  std::memset(map, 0, sizeof(*map));
+  const cuuint64_t dims[2] = {cols, rows};
+  const cuuint64_t strides[1] = {ld * 2};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(kPfChunk), static_cast<cuuint32_t>(kPfRows)};
+  const cuuint32_t estr[2] = {1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+struct PfWorkspace {
+  size_t off_ctil, off_kv, total;
+};
+
+PfWorkspace pf_layout(int total, int H, int d_c) {
+  PfWorkspace w;
+  size_t off = 0;
+  w.off_ctil = off;
+  off = align_up(off + static_cast<size_t>(total) * d_c * 2, 256);
+  w.off_kv = off;
+  off = align_up(off + static_cast<size_t>(total) * H * kKvFeat * 2, 256);
+  w.total = off;
+  return w;
+}
+
+}  // namespace
+
+size_t prefill_workspace_bytes(int total_tokens, int H, int d_c) { return pf_layout(total_tokens, H, d_c).total; }
+
+bool prefill_supported(int d_nope, int d_rope, int d_v, int d_c) {
+  return d_nope == kPfDn && d_rope == kPfDr && d_v == kPfDv && d_c % kPfChunk == 0 && d_c >= kPfChunk &&
+         d_c <= 512;
+}
+
+cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st) {
+  if (a.total <= 0 || a.batch <= 0) return cudaSuccess;
+  const PfWorkspace w = pf_layout(a.total, a.H, a.d_c);
+  uint8_t* ws = static_cast<uint8_t*>(a.workspace);
+  __nv_bfloat16* ctil = reinterpret_cast<__nv_bfloat16*>(ws + w.off_ctil);
+  __nv_bfloat16* kv = reinterpret_cast<__nv_bfloat16*>(ws + w.off_kv);
+
+  // 1. gate, LayerNorm, cache write
+  PfGateParams gp;
+  gp.c = static_cast<const __nv_bfloat16*>(a.c);
+  gp.kr = static_cast<const __nv_bfloat16*>(a.kr);
+  gp.ids = a.ids;
+  gp.cu = a.cu_seqlens;
+  gp.gate_table = static_cast<const __nv_bfloat16*>(a.gate_table);
+  gp.gamma = a.ln_gamma;
+  gp.beta = a.ln_beta;
+  gp.ctil = ctil;
+  gp.c_pool = static_cast<__nv_bfloat16*>(a.c_pool);
+  gp.kr_pool = static_cast<__nv_bfloat16*>(a.kr_pool);
+  gp.id_pool = a.id_pool;
+  gp.block_table = a.block_table;
+  gp.batch = a.batch;
+  gp.total = a.total;
+  gp.d_c = a.d_c;
+  gp.d_r = kPfDr;
+  gp.vocab = a.vocab;
+  gp.max_pages = a.max_pages;
+  gp.num_pages = a.num_pages;
+  gp.gate = a.gate;
+  gp.gate_add = a.gate_add;
+  gp.gate_ln = a.gate_ln;
+  gp.eps = a.eps;
+  gp.status = a.status;
+  prefill_gate_kernel<<<(a.total + kGateWarps - 1) / kGateWarps, 32 * kGateWarps, 0, st>>>(gp);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+
+  // 2. keys and values of every head
+  CUtensorMap cmap, wkmap, wvmap;
+  if (!pf_encode(&cmap, ctil, a.total, a.d_c, a.d_c)) return cudaErrorInvalidValue;
+  if (!pf_encode(&wkmap, a.w_uk, static_cast<uint64_t>(a.H) * kPfDn, a.d_c, a.d_c)) return cudaErrorInvalidValue;
+  if (!pf_encode(&wvmap, a.w_uv, static_cast<uint64_t>(a.H) * kPfDv, a.d_c, a.d_c)) return cudaErrorInvalidValue;
+  const int nkc = a.d_c / kPfChunk;
+  const int kv_smem = static_cast<int>(nkc * kPfAtom + kKvStages * kKvBBytes + sizeof(KvBars) + 1024);
+  e = cudaFuncSetAttribute(prefill_kv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kv_smem);
+  if (e != cudaSuccess) return e;
+  KvParams kp;
+  kp.kv = kv;
+  kp.total = a.total;
+  kp.H = a.H;
+  kp.nkc = nkc;
+  kp.wait_ns = kWaitLimitNs;
+  kp.status = a.status;
+  prefill_kv_kernel<<<(a.total + kPfRows - 1) / kPfRows, kKvThreads, kv_smem, st>>>(cmap, wkmap, wvmap, kp);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+
+  // 3. causal attention
+  CUtensorMap qmap, kvmap, krmap;
+  if (!pf_encode(&qmap, a.q, a.total, static_cast<uint64_t>(a.H) * kPfDqk, static_cast<uint64_t>(a.H) * kPfDqk))
+    return cudaErrorInvalidValue;
+  if (!pf_encode(&kvmap, kv, a.total, static_cast<uint64_t>(a.H) * kKvFeat, static_cast<uint64_t>(a.H) * kKvFeat))
+    return cudaErrorInvalidValue;
+  if (!pf_encode(&krmap, a.kr, a.total, kPfDr, kPfDr)) return cudaErrorInvalidValue;
+  e = cudaFuncSetAttribute(prefill_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(kAttnSmem));
+  if (e != cudaSuccess) return e;
+  AttnParams ap;
+  ap.cu = a.cu_seqlens;
+  ap.out = static_cast<__nv_bfloat16*>(a.out);
+  ap.batch = a.batch;
+  ap.H = a.H;
+  ap.total = a.total;
+  ap.qtiles = (a.max_seq_len + kPfRows - 1) / kPfRows;
+  ap.scale_log2 = a.scale_log2;
+  ap.wait_ns = kWaitLimitNs;
+  ap.status = a.status;
+  if (ap.qtiles == 0) return cudaSuccess;
+  const long long grid = static_cast<long long>(a.batch) * a.H * ap.qtiles;
+  if (grid > 0x7fffffffLL) return cudaErrorInvalidValue;
+  prefill_attn_kernel<<<static_cast<unsigned>(grid), kAttnThreads, kAttnSmem, st>>>(qmap, kvmap, krmap, ap);
+  return cudaGetLastError();
+}
+
+}  // namespace egmla

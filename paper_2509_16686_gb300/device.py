@@ -230,3 +230,69 @@ def clone_layer(dl: DeviceLayer, share=("workspace", "status")) -> DeviceLayer:
                        w_qkv_a=dl.w_qkv_a.clone(),
                        kv_norm_w=dl.kv_norm_w.clone(), w_o=dl.w_o.clone(),
                        y=torch.empty_like(dl.y), workspace=dl.workspace)
+
+
+# --------------------------------------------------------------------------
+# prompt processing (prefill)
+# --------------------------------------------------------------------------
+@dataclasses.dataclass
+class DevicePrefill:
+    dims: _lib.EgMlaDims
+    q: torch.Tensor
+    c: torch.Tensor
+    kr: torch.Tensor
+    ids: torch.Tensor
+    cu_seqlens: torch.Tensor
+    gate_table: torch.Tensor
+    ln_gamma: torch.Tensor
+    ln_beta: torch.Tensor
+    w_uk: torch.Tensor
+    w_uv: torch.Tensor
+    c_pool: torch.Tensor
+    kr_pool: torch.Tensor
+    id_pool: torch.Tensor
+    block_table: torch.Tensor
+    out: torch.Tensor
+    workspace: torch.Tensor
+    status: torch.Tensor
+    max_seq_len: int
+
+    def run(self, stream=None, write_cache: bool = True) -> torch.Tensor:
+        """eg_mla_prefill over the packed prompts (and the cache write)."""
+        pools = (self.c_pool, self.kr_pool, self.id_pool, self.block_table) if write_cache else (None,) * 4
+        _lib.eg_mla_prefill(self.dims, self.q, self.c, self.kr, self.ids, self.cu_seqlens, self.max_seq_len,
+                            self.gate_table, self.ln_gamma, self.ln_beta, self.w_uk, self.w_uv, self.out,
+                            self.workspace, *pools, dev_status=self.status, stream=stream)
+        return self.out
+
+    def read_status(self) -> int:
+        return int(self.status.item())
+
+
+def upload_prefill(pc, device="cuda") -> DevicePrefill:
+    d = pc.dims
+    dt = d.dtype
+    dims = dims_of(pc)
+    T = pc.total_tokens
+    return DevicePrefill(
+        dims=dims,
+        q=to_device_array(pc.q, dt, device),
+        c=to_device_array(pc.c, dt, device),
+        kr=to_device_array(pc.kr, dt, device),
+        ids=to_device_array(pc.ids, dt, device),
+        cu_seqlens=to_device_array(pc.cu_seqlens, dt, device),
+        gate_table=to_device_array(pc.gate_table, dt, device),
+        ln_gamma=torch.from_numpy(pc.ln_gamma.astype(np.float32)).to(device),
+        ln_beta=torch.from_numpy(pc.ln_beta.astype(np.float32)).to(device),
+        w_uk=to_device_array(pc.w_uk, dt, device),
+        w_uv=to_device_array(pc.w_uv, dt, device),
+        c_pool=to_device_array(pc.c_pool, dt, device),
+        kr_pool=to_device_array(pc.kr_pool, dt, device),
+        id_pool=to_device_array(pc.id_pool, dt, device),
+        block_table=to_device_array(pc.block_table, dt, device),
+        out=torch.empty((T, d.num_heads, d.d_v), dtype=torch.bfloat16, device=device),
+        workspace=torch.empty(max(_lib.eg_mla_prefill_workspace_size(dims, T), 1), dtype=torch.uint8,
+                              device=device),
+        status=torch.zeros(1, dtype=torch.int32, device=device),
+        max_seq_len=int(pc.seq_lens.max()) if pc.batch else 0,
+    )
