@@ -22,15 +22,16 @@
 //                        keys, K = d_n + d_r, the RoPE part read from the
 //                        shared k^R rows) into one of two TMEM score buffers;
 //                        one softmax thread per query row (its TMEM lane) turns
-//                        S into P in bf16 in shared memory; O += P V (M = 128
-//                        queries, N = d_v, K = 128 keys, V read MN-major) in a
-//                        third TMEM buffer.  Scores of tile j + 1 are computed
-//                        while the softmax threads work on tile j.
+//                        S into P in bf16, stored back to tensor memory; O += P
+//                        V (M = 128 queries, N = d_v, K = 128 keys; A = P read
+//                        from tensor memory, B = V read MN-major from shared
+//                        memory) in a third TMEM buffer.  Scores of tile j + 1
+//                        are computed while the softmax threads work on tile j.
 //
 // Warp roles of prefill_attn_kernel: warp 0 loads Q once and the key tiles
 // (two stages), warp 1 issues the MMAs, warps 2-5 run the softmax (warp w
 // owns TMEM lane quadrant w % 4) and the epilogue, warp 6 loads the value
-// tiles (one stage, refilled when the PV MMA that read it completes).
+// tiles (two stages, each refilled when the PV MMA that read it completes).
 //
 // Online softmax with a lazily moved reference: a row keeps the reference
 // maximum m of its exponentials until a tile's maximum exceeds it by more than
@@ -373,22 +374,22 @@ __global__ void __launch_bounds__(kKvThreads, 1)
 constexpr int kAttnKStages = 2;
 constexpr uint32_t kAttnQBytes = 3 * kPfAtom;               // 48 KB: Q [128 x 192]
 constexpr uint32_t kAttnKBytes = 3 * kPfAtom;               // 48 KB: k^C [128 x 128] + k^R [128 x 64]
+constexpr int kAttnVStages = 2;
 constexpr uint32_t kAttnVBytes = 2 * kPfAtom;               // 32 KB: V [128 keys x 128]
-constexpr uint32_t kAttnPBytes = 2 * kPfAtom;               // 32 KB: P [128 queries x 128 keys]
 constexpr uint32_t kOffQ = 0;
 constexpr uint32_t kOffK = kOffQ + kAttnQBytes;
 constexpr uint32_t kOffV = kOffK + kAttnKStages * kAttnKBytes;
-constexpr uint32_t kOffP = kOffV + kAttnVBytes;
-constexpr uint32_t kOffBars = kOffP + kAttnPBytes;
+constexpr uint32_t kOffBars = kOffV + kAttnVStages * kAttnVBytes;
 constexpr int kAttnVWarp = 6;
 constexpr int kAttnThreads = 32 * 7;
-constexpr uint32_t kColO = 2 * kPfRows;                     // TMEM: S0 at 0, S1 at 128, O at 256
+constexpr uint32_t kColO = 2 * kPfRows;                     // TMEM: S0 at 0, S1 at 128, O at 256,
+constexpr uint32_t kColP = kColO + kPfDv;                   // P (bf16 pairs, 64 columns) at 384
 constexpr float kRescaleLog2 = 8.f;
 
 struct AttnBars {
   uint64_t qfull;
   uint64_t kfull[kAttnKStages], kempty[kAttnKStages];
-  uint64_t vfull;
+  uint64_t vfull[kAttnVStages], vempty[kAttnVStages];
   uint64_t sfull[2], sfree[2];
   uint64_t pfull, pvdone;
   uint64_t drain;
@@ -439,7 +440,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       mbar_init(smem_u32(&bars.kfull[s]), 1);
       mbar_init(smem_u32(&bars.kempty[s]), 1);
     }
-    mbar_init(smem_u32(&bars.vfull), 1);
+    for (int s = 0; s < kAttnVStages; ++s) {
+      mbar_init(smem_u32(&bars.vfull[s]), 1);
+      mbar_init(smem_u32(&bars.vempty[s]), 1);
+    }
     for (int s = 0; s < 2; ++s) {
       mbar_init(smem_u32(&bars.sfull[s]), 1);
       mbar_init(smem_u32(&bars.sfree[s]), 4);
@@ -493,22 +497,27 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     }
     __syncwarp();
   } else if (warp == kAttnVWarp) {
-    // ---- value tiles: v^C of head h, one stage, refilled once the PV MMA
-    // that read the previous tile has completed
+    // ---- value tiles: v^C of head h, two stages, each refilled once the PV
+    // MMA that read it has completed
     if (elect_one()) {
       const uint64_t pol_v = policy_evict_last();
       int issued = 0;
       for (int j = 0; j < nkt; ++j) {
-        if (j >= 1 && !mbar_wait(smem_u32(&bars.pvdone), (j - 1) & 1, abort_flag, p.wait_ns)) break;
+        const int s = j % kAttnVStages;
+        if (j >= kAttnVStages &&
+            !mbar_wait(smem_u32(&bars.vempty[s]), ((j / kAttnVStages) & 1) ^ 1, abort_flag, p.wait_ns))
+          break;
         const int y = start + j * kPfRows;
-        mbar_arrive_expect_tx(smem_u32(&bars.vfull), kAttnVBytes);
-        tma_load_2d(sbase + kOffV, &kvmap, h * kKvFeat + kPfDn, y, smem_u32(&bars.vfull), pol_v);
-        tma_load_2d(sbase + kOffV + kPfAtom, &kvmap, h * kKvFeat + kPfDn + kPfChunk, y, smem_u32(&bars.vfull),
-                    pol_v);
+        const uint32_t dst = sbase + kOffV + s * kAttnVBytes;
+        mbar_arrive_expect_tx(smem_u32(&bars.vfull[s]), kAttnVBytes);
+        tma_load_2d(dst, &kvmap, h * kKvFeat + kPfDn, y, smem_u32(&bars.vfull[s]), pol_v);
+        tma_load_2d(dst + kPfAtom, &kvmap, h * kKvFeat + kPfDn + kPfChunk, y, smem_u32(&bars.vfull[s]), pol_v);
         issued = j + 1;
       }
       volatile int own = 0;
-      if (issued > 0 && !mbar_wait(smem_u32(&bars.vfull), (issued - 1) & 1, &own, p.wait_ns)) *abort_flag = 1;
+      for (int j = issued > kAttnVStages ? issued - kAttnVStages : 0; j < issued; ++j)
+        if (!mbar_wait(smem_u32(&bars.vfull[j % kAttnVStages]), (j / kAttnVStages) & 1, &own, p.wait_ns))
+          *abort_flag = 1;
     }
     __syncwarp();
   } else if (warp == 1) {
@@ -517,22 +526,25 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     constexpr uint32_t idesc_o = idesc_bf16(kPfRows, kPfDv, 0, 1);
     const uint64_t qdesc = smem_desc(sbase + kOffQ, 16, 1024, kSwizzle128B);
     const uint64_t kdesc = smem_desc(sbase + kOffK, 16, 1024, kSwizzle128B);
-    const uint64_t pdesc = smem_desc(sbase + kOffP, 16, 1024, kSwizzle128B);
     // V [keys x features] is the B operand MN-major: 64-feature atoms 16 KB
     // apart, 8-key groups 1 KB apart
     const uint64_t vdesc = smem_desc(sbase + kOffV, kPfAtom, 1024, kSwizzle128B);
     bool ok = pf_warp_wait(smem_u32(&bars.qfull), 0, abort_flag, p.wait_ns);
     bool issued = false;
     auto issue_pv = [&](int i) {
-      ok = ok && pf_warp_wait(smem_u32(&bars.vfull), i & 1, abort_flag, p.wait_ns);
+      const int vs = i % kAttnVStages;
+      ok = ok && pf_warp_wait(smem_u32(&bars.vfull[vs]), (i / kAttnVStages) & 1, abort_flag, p.wait_ns);
       ok = ok && pf_warp_wait(smem_u32(&bars.pfull), i & 1, abort_flag, p.wait_ns);
       if (!ok) return;
       tc_fence_after();
       if (elect_one()) {
+        const uint64_t vd = vdesc + ((vs * kAttnVBytes) >> 4);
+        // A = P from tensor memory: 16 keys per MMA are 8 columns of bf16 pairs
 #pragma unroll
         for (int ks = 0; ks < kPfRows / 16; ++ks)
-          mma_bf16_ss(tmem + kColO, pdesc + (((ks >> 2) * kPfAtom + (ks & 3) * 32) >> 4),
-                      vdesc + ((ks * 2048) >> 4), idesc_o, (i > 0 || ks > 0) ? 1u : 0u);
+          mma_bf16_ts(tmem + kColO, tmem + kColP + ks * 8, vd + ((ks * 2048) >> 4), idesc_o,
+                      (i > 0 || ks > 0) ? 1u : 0u);
+        mma_commit(smem_u32(&bars.vempty[vs]));
         mma_commit(smem_u32(&bars.pvdone));
       }
       __syncwarp();
@@ -571,8 +583,6 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     const int r = 32 * quad + lane;
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * quad) << 16);
     const float sl2 = p.scale_log2;
-    // this row's place in the swizzled P tile: 8-row group, row in group
-    const uint32_t prow = sbase + kOffP + (r >> 3) * 1024 + (r & 7) * 128;
     float m_ref = 0.f, l = 0.f;
     bool ok = true;
     for (int j = 0; j < nkt; ++j) {
@@ -594,9 +604,13 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         for (int c = 0; c < kPfRows; ++c)
           if (c > r) sv[c] = -INFINITY;
       }
-      float mx = sv[0];
+      // row maximum and sum as eight interleaved chains (short dependencies)
+      float m8[8];
 #pragma unroll
-      for (int c = 1; c < kPfRows; ++c) mx = fmaxf(mx, sv[c]);
+      for (int e = 0; e < 8; ++e) m8[e] = sv[e];
+#pragma unroll
+      for (int c = 8; c < kPfRows; ++c) m8[c & 7] = fmaxf(m8[c & 7], sv[c]);
+      float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])), fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
       mx *= sl2;
       float alpha = 1.f;
       if (j == 0) {
@@ -605,15 +619,16 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         alpha = pf_ex2(m_ref - mx);
         m_ref = mx;
       }
-      uint32_t pk[kPfRows / 2];
-      float rs = 0.f;
+      float pk[kPfRows / 2];   // bf16 pairs, kept as 32-bit words for the TMEM store
+      float r8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int c = 0; c < kPfRows; c += 2) {
         const float p0 = pf_ex2(fmaf(sv[c], sl2, -m_ref));
         const float p1 = pf_ex2(fmaf(sv[c + 1], sl2, -m_ref));
-        rs += p0 + p1;
-        pk[c / 2] = pack_bf16x2(p0, p1);
+        r8[(c >> 1) & 7] += p0 + p1;
+        pk[c / 2] = __uint_as_float(pack_bf16x2(p0, p1));
       }
+      const float rs = ((r8[0] + r8[1]) + (r8[2] + r8[3])) + ((r8[4] + r8[5]) + (r8[6] + r8[7]));
       l = fmaf(l, alpha, rs);
       // P is single-buffered and O is updated by the previous tile's PV MMA:
       // both wait for it
@@ -635,16 +650,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         }
       }
 #pragma unroll
-      for (int kc = 0; kc < 2; ++kc)
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          const uint32_t a = prow + kc * kPfAtom + ((u ^ (r & 7)) << 4);
-          const int w = kc * 32 + 4 * u;
-          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(pk[w]), "r"(pk[w + 1]),
-                       "r"(pk[w + 2]), "r"(pk[w + 3])
-                       : "memory");
-        }
-      fence_proxy_async_smem();
+      for (int c = 0; c < kPfRows / 2; c += 16)
+        tmem_st16(lane_base + kColP + c, *reinterpret_cast<const float(*)[16]>(&pk[c]));
+      tmem_wait_st();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&bars.pfull));
