@@ -3,6 +3,7 @@
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c32k] [--impl reference]
     python bench.py --sweep        (decode throughput vs context length)
     python bench.py --workload layers24_full   (24 whole attention layers per step)
+    python bench.py --workload prefill         (prompt processing: 8 prompts x 4096 tokens)
 
 A step is one pass of the whole decode hot path for one batch: append of each
 sequence's new token to the paged latent cache, query absorption, the split-KV
@@ -26,6 +27,14 @@ captured graph of the same steps, on the launching stream), against the
 measured HBM copy bandwidth.
 cpu_baseline / --impl reference: the fp64 oracle on the host cores on a bounded
 sample of the same workload, scaled to decode tokens/s.
+
+prefill / prefill_ragged: a step is one eg_mla_prefill call over the packed
+prompts (gate + LayerNorm and cache write per token, the per-head key/value
+up-projection, causal attention); value = prompt tokens/s, the roofline is the
+attention kernel's causal FLOPs over its own CUDA-event time against the bf16
+tensor peak, e2e copies the prompts' q, c, k^R and ids in from pinned host
+memory and the output back every step, and the oracle baseline times whole
+heads of the first prompt.
 
 Multi-GPU (torchrun): every rank runs its own replica of the workload (the
 sequences are independent; no data-path collective); the slowest rank's time
@@ -76,7 +85,8 @@ def parse():
                     help="timed steps (default 20000; 200 for layers24, 2000 per length for --sweep)")
     ap.add_argument("--warmup", type=int, default=30)
     ap.add_argument("--workload", default="c32k",
-                    choices=["c32k", "c4k", "ragged", "ragged_mla", "layers24", "layers24_full", "r0"])
+                    choices=["c32k", "c4k", "ragged", "ragged_mla", "layers24", "layers24_full", "r0", "prefill",
+                             "prefill_ragged"])
     ap.add_argument("--sweep", action="store_true",
                     help="decode throughput vs context length: batch 8, d_c 256, L = 1K .. 64K, one line per L")
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
@@ -322,6 +332,8 @@ def run_reference(args):
     ws, rank, _ = dist_env()
     if rank != 0:
         return 0
+    if args.workload.startswith("prefill"):
+        return run_reference_prefill(args)
     case, desc = make_workload(args.workload)
     from oracle import egmla_oracle as orc
     H = case.dims.num_heads
@@ -367,6 +379,53 @@ def run_reference(args):
                                       "attention work per token and are not timed"
                                       if args.workload == "layers24_full" else "")},
         "e2e": {"value": rate, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_reference_prefill(args):
+    """The reference arm of the prefill workloads: each step is the oracle's
+    prefill of one head of the first prompt over its first S tokens (S sized so
+    the run ends in about two minutes), scaled by the oracle's quadratic cost
+    in the prompt length to all heads and prompts."""
+    import dataclasses
+    from oracle import egmla_oracle as orc
+    pc, desc = prefill_case(args.workload)
+    H = pc.dims.num_heads
+    L = int(pc.seq_lens[0])
+    n_steps = max(1, args.steps if args.steps is not None else 10) + max(0, args.warmup)
+    t0 = time.perf_counter()
+    orc.prefill(pc, batches=[0], heads=[0])
+    t_full = time.perf_counter() - t0
+    S = int(min(L, max(64, L * ((110.0 / n_steps) / max(t_full, 1e-6)) ** 0.5)))
+    sub = dataclasses.replace(pc, seq_lens=np.array([S], np.int32), cu_seqlens=np.array([0, S], np.int32),
+                              q=pc.q[:S], c=pc.c[:S], kr=pc.kr[:S], ids=pc.ids[:S])
+    times = []
+    t_start = time.perf_counter()
+    for i in range(n_steps):
+        t1 = time.perf_counter()
+        orc.prefill(sub, batches=[0], heads=[i % H])
+        dt = time.perf_counter() - t1
+        if i >= args.warmup:
+            times.append(dt)
+        if time.perf_counter() - t_start > 170:
+            break
+    t_step = statistics.mean(times)
+    work = sum(int(x) ** 2 for x in pc.seq_lens) / float(S * S)
+    t_call = t_step * H * work
+    rate = pc.total_tokens / t_call
+    line = {
+        "impl": "reference", "metric": "prefill tokens/sec (prompt tokens through gate, cache write, up-projection "
+                                      "and causal attention)",
+        "value": rate, "unit": "tokens/s", "n_gpus": args.gpus, "steps": len(times), "warmup": args.warmup,
+        "ms_per_step": t_step * 1e3, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f64", "data": "synthetic", "config": {"workload": desc, "prompts": pc.batch, "tokens": pc.total_tokens},
+        "cpu_baseline": {"value": rate, "unit": "tokens/s", "cores": BLAS_THREADS, "threads": BLAS_THREADS,
+                         "host_cores": host_cores(), "kind": "oracle",
+                         "sample": f"per step one head of prompt 0 over its first {S} of {L} tokens, scaled x{H} "
+                                   f"heads x sum L^2 / S^2 = {work:.1f}"},
+        "e2e": {"value": rate, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
     return 0
@@ -722,8 +781,164 @@ def run_gpu_r0(args, workload, torch, dist, ws, rank):
     }
 
 
+def prefill_case(workload):
+    from paper_2509_16686_gb300 import synth
+    if workload == "prefill":
+        return synth.case_prefill(), ("prefill: 8 prompts x 4096 tokens, 16 heads, d_nope 128, d_rope 64, d_v 128, "
+                                      "d_c 256, vocabulary 32000 (uniform ids), gate LN(c (*) G[id]), page 64")
+    return synth.case_prefill_ragged(), ("prefill_ragged: 16 prompts of log-uniform lengths in [128, 4096], "
+                                         "16 heads, d_c 192, vocabulary 50000, Zipf(1.1) ids, page 64")
+
+
+def prefill_flops(pc):
+    """Algorithmic FLOPs of one call: the causal attention (2 (d_n + d_r + d_v)
+    per visible (query, key, head)) and the key/value up-projection
+    (2 H (d_n + d_v) d_c per token)."""
+    d = pc.dims
+    pairs = sum(int(L) * (int(L) + 1) // 2 for L in pc.seq_lens)
+    attn = 2.0 * pairs * d.num_heads * (d.d_nope + d.d_rope + d.d_v)
+    proj = 2.0 * pc.total_tokens * d.num_heads * (d.d_nope + d.d_v) * d.d_c
+    return attn, proj
+
+
+def oracle_prefill_rate(pc, budget_s):
+    """Prompt tokens/s of the fp64 oracle's prefill on host cores: whole heads
+    of the first prompt while the budget lasts (at least one)."""
+    from oracle import egmla_oracle as orc
+    H = pc.dims.num_heads
+    L = int(pc.seq_lens[0])
+    t0 = time.perf_counter()
+    done = 0
+    for h in range(H):
+        orc.prefill(pc, batches=[0], heads=[h])
+        done += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    dt = time.perf_counter() - t0
+    # prompt 0's tokens pass all H heads; the other prompts cost in proportion to L^2
+    work_full = sum(int(x) ** 2 for x in pc.seq_lens) / float(L * L)
+    rate = pc.total_tokens / (dt * H / done * work_full)
+    return rate, (f"{done} of {H} heads of prompt 0 ({L} tokens), {dt:.1f} s, scaled by heads and by "
+                  f"sum L^2 / L_0^2 = {work_full:.2f} to all prompts")
+
+
+def run_gpu_prefill(args, workload, torch, dist, ws, rank):
+    """Prompt processing through eg_mla_prefill (see the module docstring)."""
+    from paper_2509_16686_gb300 import _lib, device
+    dev = torch.cuda.current_device()
+    pc, desc = prefill_case(workload)
+    d = pc.dims
+    dp = device.upload_prefill(pc)
+    stream = torch.cuda.Stream()
+    T = pc.total_tokens
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, args.warmup)):
+            dp.run(stream)
+    stream.synchronize()
+    assert dp.read_status() == 0, "device status (prefill)"
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        dp.run(stream)
+    steps = args.steps if args.steps is not None else 200
+    with torch.cuda.stream(stream):
+        graph.replay()
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(nvsmi_id(torch, dev)) as clk:
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize()
+        with torch.cuda.stream(stream):
+            ev0.record(stream)
+            for _ in range(steps):
+                graph.replay()
+            ev1.record(stream)
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+    elapsed_ms = max_over_ranks(ev0.elapsed_time(ev1), dist, "cuda")
+    assert dp.read_status() == 0, "device status (prefill)"
+    ms = elapsed_ms / steps
+    value = ws * T * steps / (elapsed_ms * 1e-3)
+
+    # ---- the attention kernel alone: events around its launch in a captured
+    # graph of 10 calls, replayed twice (the events hold the second replay)
+    n_prof = 10
+    _lib.eg_mla_profile_begin(n_prof)
+    pgraph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(pgraph, stream=stream):
+        for _ in range(n_prof):
+            dp.run(stream)
+    with torch.cuda.stream(stream):
+        pgraph.replay()
+        pgraph.replay()
+    stream.synchronize()
+    del pgraph
+    ms_sum, n_l = _lib.eg_mla_profile_end()
+    k_ms = ms_sum / max(1, n_l)
+    attn_flops, proj_flops = prefill_flops(pc)
+    peaks_path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(peaks_path):
+        pk = json.load(open(peaks_path))
+        peak, src = float(pk.get("bf16_tflops_sustained", pk["bf16_tflops"])), "measured (sustained)"
+    else:
+        peak, src = 1700.0, "fallback (sustained)"
+    achieved = attn_flops / (k_ms * 1e-3) / 1e12
+
+    # ---- end to end through the C ABI with host buffers: every step copies the
+    # prompts' q, c, k^R and ids in from pinned host memory and reads the output back
+    names = ("q", "c", "kr", "ids")
+    h_in = {n: getattr(dp, n).cpu().pin_memory() for n in names}
+    h_out = torch.empty(dp.out.shape, dtype=dp.out.dtype).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for t in h_in.values())
+    d2h = h_out.numel() * h_out.element_size()
+    e2e_steps = args.e2e_steps or min(steps, 50)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(e2e_steps):
+            for n in names:
+                getattr(dp, n).copy_(h_in[n], non_blocking=True)
+            dp.run(stream)
+            h_out.copy_(dp.out, non_blocking=True)
+        e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), dist, "cuda")
+    e2e_value = ws * T * e2e_steps / (e2e_ms * 1e-3)
+    assert dp.read_status() == 0, "device status (prefill e2e)"
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        rate, sample = oracle_prefill_rate(pc, 12.0)
+        cpu = {"value": rate, "unit": "tokens/s", "cores": BLAS_THREADS, "threads": BLAS_THREADS,
+               "host_cores": host_cores(), "kind": "oracle", "sample": sample}
+    return {
+        "metric": "prefill tokens/sec (prompt tokens through gate, cache write, up-projection and causal attention)",
+        "value": value, "unit": "tokens/s", "n_gpus": ws, "steps": steps, "warmup": args.warmup,
+        "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": desc, "prompts": pc.batch, "tokens": T,
+                   "l2": "inputs larger than L2 (q alone is "
+                         f"{dp.q.numel() * 2 / 1e6:.0f} MB; the per-head keys and values "
+                         f"{T * d.num_heads * 256 * 2 / 1e6:.0f} MB are rewritten every step)",
+                   "graph": "one call per step, replayed from a CUDA graph"},
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "traffic": None, "kernel": "prefill_attn_kernel",
+                     "kernel_ms": k_ms, "flops_per_launch": attn_flops, "peak_source": src,
+                     "step_tflops": (attn_flops + proj_flops) / (ms * 1e-3) / 1e12,
+                     "proj_flops_per_step": proj_flops},
+        "cpu_baseline": cpu,
+        "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": 3 * steps,
+        "clocks": clk.summary(),
+    }
+
+
 def run_gpu(args, workload, torch, dist, ws, rank):
     """One bench line of `workload` (see the module docstring)."""
+    if workload.startswith("prefill"):
+        return run_gpu_prefill(args, workload, torch, dist, ws, rank)
     if workload == "r0":
         return run_gpu_r0(args, workload, torch, dist, ws, rank)
     if workload == "layers24_full":

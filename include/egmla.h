@@ -383,9 +383,11 @@ int eg_mla_debug_gather(const eg_mla_dims* dims, const void* c_pool, const void*
 
 /*
  * eg_mla_profile_begin / eg_mla_profile_end - per-launch timing of the split-KV
- * decode kernel (the one that streams the latent cache).  After begin, every
- * eg_mla_decode call records a CUDA event pair around that kernel's launch on
- * its stream, for at most max_launches launches.  end synchronises on the
+ * decode kernel (the one that streams the latent cache) and of the prefill's
+ * attention kernel.  After begin, every eg_mla_decode (eg_mla_step) call
+ * records a CUDA event pair around the decode kernel's launch on its stream,
+ * and every eg_mla_prefill call one around its attention kernel's launch, for
+ * at most max_launches launches in all.  end synchronises on the
  * events, returns the summed kernel time in milliseconds and the number of
  * launches timed, releases the events and stops recording.  During stream
  * capture the pair becomes event-record nodes of the graph

@@ -617,7 +617,7 @@ int eg_mla_prefill(const eg_mla_dims* dims, const void* q, const void* c_new, co
   a.gate_ln = (dims->gate_mode == EG_MLA_GATE_MUL_LN || dims->gate_mode == EG_MLA_GATE_ADD_LN) ? 1 : 0;
   a.eps = dims->ln_eps > 0.f ? dims->ln_eps : 1e-5f;
   a.scale_log2 = resolve_scale(dims) * 1.4426950408889634f;
-  return to_status(egmla::launch_prefill(a, static_cast<cudaStream_t>(stream)));
+  return to_status(egmla::launch_prefill(a, static_cast<cudaStream_t>(stream), prof_mark));
 }
 
 int eg_mla_debug_linear(const void* w, int32_t n_out, int32_t k, const void* x, int32_t batch, void* out,

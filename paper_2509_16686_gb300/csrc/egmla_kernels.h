@@ -134,7 +134,9 @@ struct PrefillArgs {
 };
 size_t prefill_workspace_bytes(int total_tokens, int H, int d_c);
 bool prefill_supported(int d_nope, int d_rope, int d_v, int d_c);
-cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st);
+// `mark` (may be null) is called with (stream, true) just before the
+// attention kernel's launch and (stream, false) just after it.
+cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st, void (*mark)(cudaStream_t, bool));
 // out[b][n] = sum_k x[b][k] W[n][k] for b < batch, n < n_out: W [n_out, k] and
 // x [batch, k] bf16 row-major (16-byte aligned, k % 8 == 0), out fp32 or
 // bf16 with row stride ldo elements (egmla_linear.cu).  Launched with

@@ -747,7 +747,7 @@ bool prefill_supported(int d_nope, int d_rope, int d_v, int d_c) {
          d_c <= 512;
 }
 
-cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st) {
+cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st, void (*mark)(cudaStream_t, bool)) {
   if (a.total <= 0 || a.batch <= 0) return cudaSuccess;
   const PfWorkspace w = pf_layout(a.total, a.H, a.d_c);
   uint8_t* ws = static_cast<uint8_t*>(a.workspace);
@@ -827,8 +827,11 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st) {
   if (ap.qtiles == 0) return cudaSuccess;
   const long long grid = static_cast<long long>(a.batch) * a.H * ap.qtiles;
   if (grid > 0x7fffffffLL) return cudaErrorInvalidValue;
+  if (mark) mark(st, true);
   prefill_attn_kernel<<<static_cast<unsigned>(grid), kAttnThreads, kAttnSmem, st>>>(qmap, kvmap, krmap, ap);
-  return cudaGetLastError();
+  e = cudaGetLastError();
+  if (mark) mark(st, false);
+  return e;
 }
 
 }  // namespace egmla
