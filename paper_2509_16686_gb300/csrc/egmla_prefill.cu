@@ -12,10 +12,11 @@
 //                        rounded to bf16, and the raw c, k^R and id written to
 //                        the token's cache slot through the block table.
 //   prefill_kv_kernel    (tcgen05) [k^C_h ; v^C_h] = [W_UK,h ; W_UV,h] c~ for
-//                        128 tokens per CTA and every head h (Eqs. 2 and 6): M =
-//                        128 tokens, N = 256 (d_n key rows, then d_v value
-//                        rows), K = d_c, two TMEM accumulators so the epilogue
-//                        of head h overlaps the MMAs of head h + 1.
+//                        256 tokens per CTA (128 at d_c > 256) and every head h
+//                        (Eqs. 2 and 6): per output block of 128 columns (the
+//                        key or the value rows of a head) M = 128 tokens per
+//                        row tile, N = 128, K = d_c; two TMEM accumulators so
+//                        the epilogue of one block overlaps the MMAs of the next.
 //   prefill_attn_kernel  (tcgen05) flash attention: one CTA per (prompt, head,
 //                        128-query tile), walking the key tiles 0..qt of the
 //                        same prompt.  S = Q K^T (M = 128 queries, N = 128
@@ -209,15 +210,25 @@ __global__ void __launch_bounds__(32 * kGateWarps) prefill_gate_kernel(const PfG
 }
 
 // ============================================================================ 2. key/value up-projection
+// Each CTA owns RT tiles of 128 token rows and walks the output blocks
+// (head h, key rows or value rows) in order; every 16 KB chunk of W (128
+// output rows x 64 of d_c) that it pulls in feeds the MMAs of all RT row
+// tiles, so the weights cross into the SM once per RT x 128 tokens (the
+// weight stream, not the tensor pipe, bounds a CTA of one row tile).
 constexpr int kKvFeat = kPfDn + kPfDv;                      // 256 output features per head
-constexpr uint32_t kKvBBytes = kKvFeat * kPfChunk * 2;      // 32 KB: one K chunk of a head's rows
-constexpr int kKvStages = 3;
-constexpr int kKvEpiWarps = 8;                              // two per lane quadrant: key / value half
+constexpr int kKvBlock = 128;                               // output columns per block (key or value rows)
+constexpr uint32_t kKvBBytes = kKvBlock * kPfChunk * 2;     // 16 KB: one K chunk of a block's W rows
+constexpr int kKvMaxStages = 4;
+constexpr int kKvEpiWarps = 8;
+// output staging: per epilogue warp two 4 KB buffers of 32 rows x 64 columns
+// (128-byte swizzle), each stored to global memory by one TMA box
+constexpr uint32_t kKvStageOut = 32 * kPfChunk * 2;         // 4 KB
+constexpr uint32_t kKvOutBytes = kKvEpiWarps * 2 * kKvStageOut;   // 64 KB
 constexpr int kKvThreads = 32 * (2 + kKvEpiWarps);          // warp 0 TMA, warp 1 MMA
 
 struct KvBars {
   uint64_t afull;
-  uint64_t bfull[kKvStages], bempty[kKvStages];
+  uint64_t bfull[kKvMaxStages], bempty[kKvMaxStages];
   uint64_t dfull[2], dfree[2];
   uint64_t drain;
   uint32_t tmem_base;
@@ -226,23 +237,42 @@ struct KvBars {
 
 struct KvParams {
   __nv_bfloat16* kv;   // [T, H, 256]
-  int total, H, nkc;
+  int total, H, nkc, stages;
   uint64_t wait_ns;
   int32_t* status;
 };
 
+// weight stages that fit next to RT x nkc latent atoms and the output staging
+template <int RT>
+__host__ __device__ constexpr int kv_stages(int nkc) {
+  const long long room = 227LL * 1024 - 2048 - static_cast<long long>(RT * nkc) * kPfAtom - kKvOutBytes;
+  const long long st = room / kKvBBytes;
+  return st > kKvMaxStages ? kKvMaxStages : static_cast<int>(st);
+}
+template <int RT>
+__host__ __device__ constexpr uint32_t kv_smem_bytes(int nkc) {
+  return static_cast<uint32_t>(RT * nkc) * kPfAtom + kKvOutBytes + kv_stages<RT>(nkc) * kKvBBytes + sizeof(KvBars) +
+         1024;
+}
+
+template <int RT>
 __global__ void __launch_bounds__(kKvThreads, 1)
     prefill_kv_kernel(const __grid_constant__ CUtensorMap cmap, const __grid_constant__ CUtensorMap wkmap,
-                      const __grid_constant__ CUtensorMap wvmap, const KvParams p) {
+                      const __grid_constant__ CUtensorMap wvmap, const __grid_constant__ CUtensorMap omap,
+                      const KvParams p) {
+  constexpr uint32_t kTmemCols = 2 * RT * kKvBlock;          // two accumulators of RT x 128 columns
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const uint32_t sbase = smem_u32(smem);
-  const uint32_t b_off = static_cast<uint32_t>(p.nkc) * kPfAtom;
+  const int kKvStages = p.stages;
+  const uint32_t o_off = static_cast<uint32_t>(RT * p.nkc) * kPfAtom;
+  const uint32_t b_off = o_off + kKvOutBytes;
   KvBars& bars = *reinterpret_cast<KvBars*>(smem + b_off + kKvStages * kKvBBytes);
   volatile int* abort_flag = &bars.abort;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int row0 = blockIdx.x * kPfRows;
-  const int nsteps = p.H * p.nkc;
+  const int row0 = blockIdx.x * RT * kPfRows;
+  const int nblocks = 2 * p.H;                 // (head, key or value rows)
+  const int nsteps = nblocks * p.nkc;
 
   if (tid == 0) {
     mbar_init(smem_u32(&bars.afull), 1);
@@ -260,9 +290,10 @@ __global__ void __launch_bounds__(kKvThreads, 1)
     prefetch_tensormap(&cmap);
     prefetch_tensormap(&wkmap);
     prefetch_tensormap(&wvmap);
+    prefetch_tensormap(&omap);
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32(&bars.tmem_base), 512);
+    tmem_alloc(smem_u32(&bars.tmem_base), kTmemCols);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -273,20 +304,21 @@ __global__ void __launch_bounds__(kKvThreads, 1)
   if (warp == 0) {
     if (elect_one()) {
       const uint64_t pol_stream = policy_evict_first(), pol_keep = policy_evict_last();
-      mbar_arrive_expect_tx(smem_u32(&bars.afull), static_cast<uint32_t>(p.nkc) * kPfAtom);
-      for (int kc = 0; kc < p.nkc; ++kc)
-        tma_load_2d(sbase + kc * kPfAtom, &cmap, kc * kPfChunk, row0, smem_u32(&bars.afull), pol_stream);
+      mbar_arrive_expect_tx(smem_u32(&bars.afull), static_cast<uint32_t>(RT * p.nkc) * kPfAtom);
+      for (int t = 0; t < RT; ++t)
+        for (int kc = 0; kc < p.nkc; ++kc)
+          tma_load_2d(sbase + (t * p.nkc + kc) * kPfAtom, &cmap, kc * kPfChunk, row0 + t * kPfRows,
+                      smem_u32(&bars.afull), pol_stream);
       int issued = 0;
       for (int i = 0; i < nsteps; ++i) {
         const int s = i % kKvStages;
         if (i >= kKvStages &&
             !mbar_wait(smem_u32(&bars.bempty[s]), ((i / kKvStages) & 1) ^ 1, abort_flag, p.wait_ns))
           break;
-        const int h = i / p.nkc, kc = i % p.nkc;
-        const uint32_t dst = sbase + b_off + s * kKvBBytes;
+        const int blk = i / p.nkc, kc = i % p.nkc;
         mbar_arrive_expect_tx(smem_u32(&bars.bfull[s]), kKvBBytes);
-        tma_load_2d(dst, &wkmap, kc * kPfChunk, h * kPfDn, smem_u32(&bars.bfull[s]), pol_keep);
-        tma_load_2d(dst + kKvBBytes / 2, &wvmap, kc * kPfChunk, h * kPfDv, smem_u32(&bars.bfull[s]), pol_keep);
+        tma_load_2d(sbase + b_off + s * kKvBBytes, (blk & 1) ? &wvmap : &wkmap, kc * kPfChunk,
+                    (blk >> 1) * kKvBlock, smem_u32(&bars.bfull[s]), pol_keep);
         issued = i + 1;
       }
       // every copy issued lands before the CTA can leave
@@ -298,24 +330,27 @@ __global__ void __launch_bounds__(kKvThreads, 1)
     }
     __syncwarp();
   } else if (warp == 1) {
-    constexpr uint32_t idesc = idesc_bf16(kPfRows, kKvFeat, 0, 0);
+    constexpr uint32_t idesc = idesc_bf16(kPfRows, kKvBlock, 0, 0);
     bool ok = pf_warp_wait(smem_u32(&bars.afull), 0, abort_flag, p.wait_ns);
     bool issued = false;
-    for (int h = 0; ok && h < p.H; ++h) {
-      const int db = h & 1;
-      if (h >= 2) ok = pf_warp_wait(smem_u32(&bars.dfree[db]), ((h - 2) >> 1) & 1, abort_flag, p.wait_ns);
+    for (int blk = 0; ok && blk < nblocks; ++blk) {
+      const int db = blk & 1;
+      if (blk >= 2) ok = pf_warp_wait(smem_u32(&bars.dfree[db]), ((blk - 2) >> 1) & 1, abort_flag, p.wait_ns);
       for (int kc = 0; ok && kc < p.nkc; ++kc) {
-        const int i = h * p.nkc + kc, s = i % kKvStages;
+        const int i = blk * p.nkc + kc, s = i % kKvStages;
         ok = pf_warp_wait(smem_u32(&bars.bfull[s]), (i / kKvStages) & 1, abort_flag, p.wait_ns);
         if (!ok) break;
         tc_fence_after();
         if (elect_one()) {
-          const uint64_t ad = smem_desc(sbase + kc * kPfAtom, 16, 1024, kSwizzle128B);
           const uint64_t bd = smem_desc(sbase + b_off + s * kKvBBytes, 16, 1024, kSwizzle128B);
 #pragma unroll
-          for (int kk = 0; kk < kPfChunk / 16; ++kk)
-            mma_bf16_ss(tmem + db * kKvFeat, ad + ((kk * 32) >> 4), bd + ((kk * 32) >> 4), idesc,
-                        (kc > 0 || kk > 0) ? 1u : 0u);
+          for (int t = 0; t < RT; ++t) {
+            const uint64_t ad = smem_desc(sbase + (t * p.nkc + kc) * kPfAtom, 16, 1024, kSwizzle128B);
+#pragma unroll
+            for (int kk = 0; kk < kPfChunk / 16; ++kk)
+              mma_bf16_ss(tmem + db * (RT * kKvBlock) + t * kKvBlock, ad + ((kk * 32) >> 4), bd + ((kk * 32) >> 4),
+                          idesc, (kc > 0 || kk > 0) ? 1u : 0u);
+          }
           mma_commit(smem_u32(&bars.bempty[s]));
           if (kc == p.nkc - 1) mma_commit(smem_u32(&bars.dfull[db]));
         }
@@ -331,42 +366,61 @@ __global__ void __launch_bounds__(kKvThreads, 1)
     }
     __syncwarp();
   } else {
-    // token row r = TMEM lane r; warps 2-5 store the key half (columns 0-127)
-    // of every head, warps 6-9 the value half
-    const int quad = warp & 3, half = (warp - 2) / 4;
-    const int r = 32 * quad + lane, row = row0 + r;
-    const bool live = row < p.total;
-    __nv_bfloat16* dst_row = p.kv + static_cast<size_t>(live ? row : 0) * p.H * kKvFeat + half * kPfDn;
+    // token row = TMEM lane of its row tile; RT = 2: warps 2-5 store row tile
+    // 0, warps 6-9 row tile 1 (all 128 columns of a block); RT = 1: warps 2-5
+    // store the block's first 64 columns, warps 6-9 the last 64.  Each warp
+    // writes its 32 rows x 64 columns into one of its two staging buffers
+    // (128-byte swizzle) and its lane 0 stores them with one TMA box.
+    const int quad = warp & 3, g = (warp - 2) / 4;
+    const int t = RT == 2 ? g : 0;
+    constexpr int kCols = RT == 2 ? kKvBlock : kKvBlock / 2;
+    const int cbase = RT == 2 ? 0 : g * kCols;
+    const int y0 = row0 + t * kPfRows + 32 * quad;           // the warp's first token row
+    const uint32_t stg = sbase + o_off + (warp - 2) * 2 * kKvStageOut;
+    const uint32_t rowoff = (lane >> 3) * 1024 + (lane & 7) * 128;
     bool ok = true;
-    for (int h = 0; h < p.H; ++h) {
-      const int db = h & 1;
-      ok = ok && pf_warp_wait(smem_u32(&bars.dfull[db]), (h >> 1) & 1, abort_flag, p.wait_ns);
+    int nst = 0;   // boxes stored so far (buffer nst % 2)
+    for (int blk = 0; blk < nblocks; ++blk) {
+      const int db = blk & 1;
+      ok = ok && pf_warp_wait(smem_u32(&bars.dfull[db]), (blk >> 1) & 1, abort_flag, p.wait_ns);
       if (!ok) break;
       tc_fence_after();
 #pragma unroll
-      for (int c0 = 0; c0 < kPfDn; c0 += 32) {
-        float v[32];
-        const uint32_t ta = tmem + (static_cast<uint32_t>(32 * quad) << 16) + db * kKvFeat + half * kPfDn + c0;
-        tmem_ld16(ta, *reinterpret_cast<float(*)[16]>(&v[0]));
-        tmem_ld16(ta + 16, *reinterpret_cast<float(*)[16]>(&v[16]));
-        tmem_wait_ld();
-        if (live) {
-          uint4* d = reinterpret_cast<uint4*>(dst_row + static_cast<size_t>(h) * kKvFeat + c0);
+      for (int c0 = 0; c0 < kCols; c0 += kPfChunk, ++nst) {
+        float v[kPfChunk];
+        const uint32_t ta =
+            tmem + (static_cast<uint32_t>(32 * quad) << 16) + db * (RT * kKvBlock) + t * kKvBlock + cbase + c0;
 #pragma unroll
-          for (int q = 0; q < 4; ++q)
-            d[q] = make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
-                              pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+        for (int c = 0; c < kPfChunk; c += 16) tmem_ld16(ta + c, *reinterpret_cast<float(*)[16]>(&v[c]));
+        tmem_wait_ld();
+        // the store that last read this buffer (two boxes ago) has read it
+        if (lane == 0 && nst >= 2) bulk_wait_group_read<1>();
+        __syncwarp();
+        const uint32_t buf = stg + (nst & 1) * kKvStageOut + rowoff;
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(buf + ((u ^ (lane & 7)) << 4)),
+                       "r"(pack_bf16x2(v[8 * u], v[8 * u + 1])), "r"(pack_bf16x2(v[8 * u + 2], v[8 * u + 3])),
+                       "r"(pack_bf16x2(v[8 * u + 4], v[8 * u + 5])), "r"(pack_bf16x2(v[8 * u + 6], v[8 * u + 7]))
+                       : "memory");
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_2d(&omap, blk * kKvBlock + cbase + c0, y0, stg + (nst & 1) * kKvStageOut);
+          bulk_commit_group();
         }
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&bars.dfree[db]));
     }
+    if (lane == 0) bulk_wait_group_all();
+    __syncwarp();
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  if (warp == 1) tmem_dealloc(tmem, 512);
+  if (warp == 1) tmem_dealloc(tmem, kTmemCols);
   if (tid == 0 && bars.abort) report_status(p.status, kStatusTimeout);
 }
 
@@ -709,14 +763,15 @@ EncodeFn pf_encode_fn() {
 }
 
 // row-major bf16 [rows, cols] with row stride `ld` elements; boxes of 64
-// columns x 128 rows, 128-byte swizzle, rows past the end read as zero
-bool pf_encode(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld) {
+// columns x box_rows rows, 128-byte swizzle, rows past the end read as zero
+bool pf_encode(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld,
+               uint32_t box_rows = kPfRows) {
   EncodeFn enc = pf_encode_fn();
   if (enc == nullptr) return false;
   std::memset(map, 0, sizeof(*map));
   const cuuint64_t dims[2] = {cols, rows};
   const cuuint64_t strides[1] = {ld * 2};
-  const cuuint32_t box[2] = {static_cast<cuuint32_t>(kPfChunk), static_cast<cuuint32_t>(kPfRows)};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(kPfChunk), box_rows};
   const cuuint32_t estr[2] = {1, 1};
   return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -784,15 +839,16 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st, void (*mark)(c
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
 
-  // 2. keys and values of every head
+  // 2. keys and values of every head: two row tiles per CTA while their
+  // latent tiles fit shared memory next to the weight stages (d_c <= 256)
   CUtensorMap cmap, wkmap, wvmap;
   if (!pf_encode(&cmap, ctil, a.total, a.d_c, a.d_c)) return cudaErrorInvalidValue;
   if (!pf_encode(&wkmap, a.w_uk, static_cast<uint64_t>(a.H) * kPfDn, a.d_c, a.d_c)) return cudaErrorInvalidValue;
   if (!pf_encode(&wvmap, a.w_uv, static_cast<uint64_t>(a.H) * kPfDv, a.d_c, a.d_c)) return cudaErrorInvalidValue;
   const int nkc = a.d_c / kPfChunk;
-  const int kv_smem = static_cast<int>(nkc * kPfAtom + kKvStages * kKvBBytes + sizeof(KvBars) + 1024);
-  e = cudaFuncSetAttribute(prefill_kv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kv_smem);
-  if (e != cudaSuccess) return e;
+  CUtensorMap omap;   // the kv buffer, stored in boxes of 64 columns x 32 rows
+  if (!pf_encode(&omap, kv, a.total, static_cast<uint64_t>(a.H) * kKvFeat, static_cast<uint64_t>(a.H) * kKvFeat, 32))
+    return cudaErrorInvalidValue;
   KvParams kp;
   kp.kv = kv;
   kp.total = a.total;
@@ -800,7 +856,21 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st, void (*mark)(c
   kp.nkc = nkc;
   kp.wait_ns = kWaitLimitNs;
   kp.status = a.status;
-  prefill_kv_kernel<<<(a.total + kPfRows - 1) / kPfRows, kKvThreads, kv_smem, st>>>(cmap, wkmap, wvmap, kp);
+  if (nkc <= 4) {
+    kp.stages = kv_stages<2>(nkc);
+    const int kv_smem = static_cast<int>(kv_smem_bytes<2>(nkc));
+    e = cudaFuncSetAttribute(prefill_kv_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, kv_smem);
+    if (e != cudaSuccess) return e;
+    prefill_kv_kernel<2><<<(a.total + 2 * kPfRows - 1) / (2 * kPfRows), kKvThreads, kv_smem, st>>>(
+        cmap, wkmap, wvmap, omap, kp);
+  } else {
+    kp.stages = kv_stages<1>(nkc);
+    const int kv_smem = static_cast<int>(kv_smem_bytes<1>(nkc));
+    e = cudaFuncSetAttribute(prefill_kv_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kv_smem);
+    if (e != cudaSuccess) return e;
+    prefill_kv_kernel<1><<<(a.total + kPfRows - 1) / kPfRows, kKvThreads, kv_smem, st>>>(cmap, wkmap, wvmap, omap,
+                                                                                         kp);
+  }
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
 
