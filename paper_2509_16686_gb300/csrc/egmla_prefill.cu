@@ -425,27 +425,48 @@ __global__ void __launch_bounds__(kKvThreads, 1)
 }
 
 // ============================================================================ 3. causal flash attention
-constexpr int kAttnKStages = 2;
-constexpr uint32_t kAttnQBytes = 3 * kPfAtom;               // 48 KB: Q [128 x 192]
-constexpr uint32_t kAttnKBytes = 3 * kPfAtom;               // 48 KB: k^C [128 x 128] + k^R [128 x 64]
-constexpr int kAttnVStages = 2;
+// One CTA per (prompt, head, block of 256 queries): two query tiles X = A
+// (queries q0 .. q0 + 127) and B (q0 + 128 .. q0 + 255) share every key and
+// value tile copied into shared memory, which halves the bytes a CTA pulls in
+// per flop (the per-SM copy rate into shared memory, not the tensor pipe,
+// bounds a CTA that owns one query tile).  Key tiles are 128 keys; A meets
+// tiles 0 .. 2 qb, B tiles 0 .. 2 qb + 1 (qb = q0 / 256).
+//
+// Tensor memory holds S_X (128 fp32 columns) and O_X (128) of both tiles.
+// The softmax threads write P_X in bf16 over the first 64 columns of S_X
+// once they have read S_X, and the MMA issuer orders, per key tile j,
+//   O_A += P_A(j - 1) V(j - 1);  S_A(j) = Q_A K(j)^T;
+//   O_B += P_B(j - 1) V(j - 1);  S_B(j) = Q_B K(j)^T
+// in one thread: the MMAs of one issuing thread run in order, so S_X(j)
+// overwrites P_X(j - 1) only after the PV MMA has read it, and the commit
+// after S_X(j) also covers that PV MMA (O_X is current when the softmax of
+// tile j sees S_X(j)).  While the softmax threads of one query tile work, the
+// tensor pipe runs the other tile's MMAs.
+constexpr int kAttnKeys = 128;                              // keys per tile
+constexpr uint32_t kAttnQBytes = 3 * kPfAtom;               // 48 KB: one query tile [128 x 192]
 constexpr uint32_t kAttnVBytes = 2 * kPfAtom;               // 32 KB: V [128 keys x 128]
+// key tiles arrive as three 16 KB chunks (k^C columns 0-63, 64-127, k^R)
+// in a ring of four chunk slots, so the next tile's first chunks land while
+// the last score MMAs of the current tile still read it; values in two stages
+constexpr int kAttnKSlots = 4;
+constexpr int kAttnVStages = 2;
 constexpr uint32_t kOffQ = 0;
-constexpr uint32_t kOffK = kOffQ + kAttnQBytes;
-constexpr uint32_t kOffV = kOffK + kAttnKStages * kAttnKBytes;
+constexpr uint32_t kOffK = kOffQ + 2 * kAttnQBytes;
+constexpr uint32_t kOffV = kOffK + kAttnKSlots * kPfAtom;
 constexpr uint32_t kOffBars = kOffV + kAttnVStages * kAttnVBytes;
-constexpr int kAttnVWarp = 6;
-constexpr int kAttnThreads = 32 * 7;
-constexpr uint32_t kColO = 2 * kPfRows;                     // TMEM: S0 at 0, S1 at 128, O at 256,
-constexpr uint32_t kColP = kColO + kPfDv;                   // P (bf16 pairs, 64 columns) at 384
+constexpr int kAttnSoftWarp0 = 2;                           // warps 2-5: tile A, warps 6-9: tile B
+constexpr int kAttnVWarp = 10;
+constexpr int kAttnThreads = 32 * (kAttnVWarp + 1);
+// TMEM columns: S_X (P_X over its first 64 columns) and O_X
+__host__ __device__ constexpr uint32_t col_s(int x) { return x * kAttnKeys; }
+__host__ __device__ constexpr uint32_t col_o(int x) { return 256 + x * kPfDv; }
 constexpr float kRescaleLog2 = 8.f;
 
 struct AttnBars {
   uint64_t qfull;
-  uint64_t kfull[kAttnKStages], kempty[kAttnKStages];
+  uint64_t kfull[kAttnKSlots], kempty[kAttnKSlots];
   uint64_t vfull[kAttnVStages], vempty[kAttnVStages];
-  uint64_t sfull[2], sfree[2];
-  uint64_t pfull, pvdone;
+  uint64_t sfull[2], pfull[2], odone[2];   // per query tile
   uint64_t drain;
   uint32_t tmem_base;
   int abort;
@@ -455,7 +476,7 @@ constexpr uint32_t kAttnSmem = kOffBars + sizeof(AttnBars) + 1024;
 struct AttnParams {
   const int32_t* cu;
   __nv_bfloat16* out;   // [T, H, d_v]
-  int batch, H, qtiles, total;
+  int batch, H, qblocks, total;
   float scale_log2;
   uint64_t wait_ns;
   int32_t* status;
@@ -464,22 +485,24 @@ struct AttnParams {
 __global__ void __launch_bounds__(kAttnThreads, 1)
     prefill_attn_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kvmap,
                         const __grid_constant__ CUtensorMap krmap, const AttnParams p) {
-  // heaviest query tiles of a (prompt, head) first; the tiles of one (prompt,
-  // head) are neighbours in launch order, so its keys stay in L2 while read
-  const int group = blockIdx.x / p.qtiles;
-  const int qt = p.qtiles - 1 - blockIdx.x % p.qtiles;
+  // heaviest query blocks of a (prompt, head) first; the blocks of one
+  // (prompt, head) are neighbours in launch order, so its keys stay in L2
+  const int group = blockIdx.x / p.qblocks;
+  const int qb = p.qblocks - 1 - blockIdx.x % p.qblocks;
   const int b = group / p.H, h = group % p.H;
   const int start = __ldg(p.cu + b);
   const int L = __ldg(p.cu + b + 1) - start;
-  const int q0 = qt * kPfRows;
+  const int q0 = qb * 2 * kPfRows;
   // prompt offsets that do not fit the packed rows, or a prompt longer than
   // the host bound the grid was sized for: report, compute nothing past it
-  if (start < 0 || L < 0 || start > p.total - L || (qt == p.qtiles - 1 && L > p.qtiles * kPfRows)) {
+  if (start < 0 || L < 0 || start > p.total - L || (qb == p.qblocks - 1 && L > p.qblocks * 2 * kPfRows)) {
     if (threadIdx.x == 0) report_status(p.status, kStatusOutOfRange);
     if (start < 0 || L < 0 || start > p.total - L) return;
   }
   if (q0 >= L) return;
-  const int nkt = qt + 1;   // key tiles 0..qt; the last one is the diagonal tile
+  const bool has_b = q0 + kPfRows < L;                     // tile B holds live queries
+  const int ntile[2] = {2 * qb + 1, has_b ? 2 * qb + 2 : 0};
+  const int nkt = has_b ? ntile[1] : ntile[0];
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
@@ -490,7 +513,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 
   if (tid == 0) {
     mbar_init(smem_u32(&bars.qfull), 1);
-    for (int s = 0; s < kAttnKStages; ++s) {
+    for (int s = 0; s < kAttnKSlots; ++s) {
       mbar_init(smem_u32(&bars.kfull[s]), 1);
       mbar_init(smem_u32(&bars.kempty[s]), 1);
     }
@@ -498,12 +521,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       mbar_init(smem_u32(&bars.vfull[s]), 1);
       mbar_init(smem_u32(&bars.vempty[s]), 1);
     }
-    for (int s = 0; s < 2; ++s) {
-      mbar_init(smem_u32(&bars.sfull[s]), 1);
-      mbar_init(smem_u32(&bars.sfree[s]), 4);
+    for (int x = 0; x < 2; ++x) {
+      mbar_init(smem_u32(&bars.sfull[x]), 1);
+      mbar_init(smem_u32(&bars.pfull[x]), 4);
+      mbar_init(smem_u32(&bars.odone[x]), 1);
     }
-    mbar_init(smem_u32(&bars.pfull), 4);
-    mbar_init(smem_u32(&bars.pvdone), 1);
     mbar_init(smem_u32(&bars.drain), 1);
     bars.abort = 0;
     fence_mbar_init();
@@ -521,38 +543,42 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const uint32_t tmem = bars.tmem_base;
 
   if (warp == 0) {
-    // ---- Q once, then the key tiles: k^C of head h (two 64-column boxes of
-    // the kv buffer) and the shared k^R rows
+    // ---- the query tiles once, then the key tiles: k^C of head h (two
+    // 64-column boxes of the kv buffer) and the shared k^R rows
     if (elect_one()) {
       const uint64_t pol_q = policy_evict_first(), pol_k = policy_evict_last();
-      mbar_arrive_expect_tx(smem_u32(&bars.qfull), kAttnQBytes);
-      for (int c = 0; c < 3; ++c)
-        tma_load_2d(sbase + kOffQ + c * kPfAtom, &qmap, h * kPfDqk + c * kPfChunk, start + q0,
-                    smem_u32(&bars.qfull), pol_q);
+      const int nq = has_b ? 2 : 1;
+      mbar_arrive_expect_tx(smem_u32(&bars.qfull), nq * kAttnQBytes);
+      for (int x = 0; x < nq; ++x)
+        for (int c = 0; c < 3; ++c)
+          tma_load_2d(sbase + kOffQ + x * kAttnQBytes + c * kPfAtom, &qmap, h * kPfDqk + c * kPfChunk,
+                      start + q0 + x * kPfRows, smem_u32(&bars.qfull), pol_q);
+      // chunk g = 3 j + c of key tile j goes to slot g % 4
       int issued = 0;
-      for (int j = 0; j < nkt; ++j) {
-        const int s = j % kAttnKStages;
-        if (j >= kAttnKStages &&
-            !mbar_wait(smem_u32(&bars.kempty[s]), ((j / kAttnKStages) & 1) ^ 1, abort_flag, p.wait_ns))
+      for (int g = 0; g < 3 * nkt; ++g) {
+        const int s = g % kAttnKSlots, j = g / 3, c = g % 3;
+        if (g >= kAttnKSlots &&
+            !mbar_wait(smem_u32(&bars.kempty[s]), ((g / kAttnKSlots) & 1) ^ 1, abort_flag, p.wait_ns))
           break;
-        const uint32_t dst = sbase + kOffK + s * kAttnKBytes;
-        const int y = start + j * kPfRows;
-        mbar_arrive_expect_tx(smem_u32(&bars.kfull[s]), kAttnKBytes);
-        tma_load_2d(dst, &kvmap, h * kKvFeat, y, smem_u32(&bars.kfull[s]), pol_k);
-        tma_load_2d(dst + kPfAtom, &kvmap, h * kKvFeat + kPfChunk, y, smem_u32(&bars.kfull[s]), pol_k);
-        tma_load_2d(dst + 2 * kPfAtom, &krmap, 0, y, smem_u32(&bars.kfull[s]), pol_k);
-        issued = j + 1;
+        const int y = start + j * kAttnKeys;
+        mbar_arrive_expect_tx(smem_u32(&bars.kfull[s]), kPfAtom);
+        if (c < 2)
+          tma_load_2d(sbase + kOffK + s * kPfAtom, &kvmap, h * kKvFeat + c * kPfChunk, y, smem_u32(&bars.kfull[s]),
+                      pol_k);
+        else
+          tma_load_2d(sbase + kOffK + s * kPfAtom, &krmap, 0, y, smem_u32(&bars.kfull[s]), pol_k);
+        issued = g + 1;
       }
       volatile int own = 0;
       if (!mbar_wait(smem_u32(&bars.qfull), 0, &own, p.wait_ns)) *abort_flag = 1;
-      for (int j = issued > kAttnKStages ? issued - kAttnKStages : 0; j < issued; ++j)
-        if (!mbar_wait(smem_u32(&bars.kfull[j % kAttnKStages]), (j / kAttnKStages) & 1, &own, p.wait_ns))
+      for (int g = issued > kAttnKSlots ? issued - kAttnKSlots : 0; g < issued; ++g)
+        if (!mbar_wait(smem_u32(&bars.kfull[g % kAttnKSlots]), (g / kAttnKSlots) & 1, &own, p.wait_ns))
           *abort_flag = 1;
     }
     __syncwarp();
   } else if (warp == kAttnVWarp) {
-    // ---- value tiles: v^C of head h, two stages, each refilled once the PV
-    // MMA that read it has completed
+    // ---- value tiles: v^C of head h, two stages, each refilled once both
+    // PV MMAs that read it have completed
     if (elect_one()) {
       const uint64_t pol_v = policy_evict_last();
       int issued = 0;
@@ -561,7 +587,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         if (j >= kAttnVStages &&
             !mbar_wait(smem_u32(&bars.vempty[s]), ((j / kAttnVStages) & 1) ^ 1, abort_flag, p.wait_ns))
           break;
-        const int y = start + j * kPfRows;
+        const int y = start + j * kAttnKeys;
         const uint32_t dst = sbase + kOffV + s * kAttnVBytes;
         mbar_arrive_expect_tx(smem_u32(&bars.vfull[s]), kAttnVBytes);
         tma_load_2d(dst, &kvmap, h * kKvFeat + kPfDn, y, smem_u32(&bars.vfull[s]), pol_v);
@@ -575,8 +601,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     }
     __syncwarp();
   } else if (warp == 1) {
-    // ---- MMAs: S(j) into score buffer j % 2, then O += P(j - 1) V(j - 1)
-    constexpr uint32_t idesc_s = idesc_bf16(kPfRows, kPfRows, 0, 0);
+    // ---- MMAs.  Per key tile j and query tile X: O_X += P_X(j - 1) V(j - 1),
+    // then S_X(j) = Q_X K(j)^T (see the header for why in this order)
+    constexpr uint32_t idesc_s = idesc_bf16(kPfRows, kAttnKeys, 0, 0);
     constexpr uint32_t idesc_o = idesc_bf16(kPfRows, kPfDv, 0, 1);
     const uint64_t qdesc = smem_desc(sbase + kOffQ, 16, 1024, kSwizzle128B);
     const uint64_t kdesc = smem_desc(sbase + kOffK, 16, 1024, kSwizzle128B);
@@ -585,45 +612,66 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     const uint64_t vdesc = smem_desc(sbase + kOffV, kPfAtom, 1024, kSwizzle128B);
     bool ok = pf_warp_wait(smem_u32(&bars.qfull), 0, abort_flag, p.wait_ns);
     bool issued = false;
-    auto issue_pv = [&](int i) {
+    int kseen = -1;   // the last key chunk whose arrival was waited for
+    auto wait_k = [&](int g) {
+      if (kseen < g) {
+        ok = ok && pf_warp_wait(smem_u32(&bars.kfull[g % kAttnKSlots]), (g / kAttnKSlots) & 1, abort_flag,
+                                p.wait_ns);
+        kseen = g;
+      }
+    };
+    // O_X += P_X(i) V(i); the last reader of V(i) frees it, the last PV of X signals its epilogue
+    auto issue_pv = [&](int x, int i) {
       const int vs = i % kAttnVStages;
-      ok = ok && pf_warp_wait(smem_u32(&bars.vfull[vs]), (i / kAttnVStages) & 1, abort_flag, p.wait_ns);
-      ok = ok && pf_warp_wait(smem_u32(&bars.pfull), i & 1, abort_flag, p.wait_ns);
+      if (x == 0 || (x == 1 && ntile[0] <= i)) {
+        // first reader of V(i): wait for its copy (A reads every tile B reads but the last)
+        ok = ok && pf_warp_wait(smem_u32(&bars.vfull[vs]), (i / kAttnVStages) & 1, abort_flag, p.wait_ns);
+      }
+      ok = ok && pf_warp_wait(smem_u32(&bars.pfull[x]), i & 1, abort_flag, p.wait_ns);
       if (!ok) return;
       tc_fence_after();
       if (elect_one()) {
-        const uint64_t vd = vdesc + ((vs * kAttnVBytes) >> 4);
-        // A = P from tensor memory: 16 keys per MMA are 8 columns of bf16 pairs
+        // A = P_X from tensor memory: 16 keys per MMA are 8 columns of bf16 pairs
 #pragma unroll
-        for (int ks = 0; ks < kPfRows / 16; ++ks)
-          mma_bf16_ts(tmem + kColO, tmem + kColP + ks * 8, vd + ((ks * 2048) >> 4), idesc_o,
+        const uint64_t vd = vdesc + ((vs * kAttnVBytes) >> 4);
+        for (int ks = 0; ks < kAttnKeys / 16; ++ks)
+          mma_bf16_ts(tmem + col_o(x), tmem + col_s(x) + ks * 8, vd + ((ks * 2048) >> 4), idesc_o,
                       (i > 0 || ks > 0) ? 1u : 0u);
-        mma_commit(smem_u32(&bars.vempty[vs]));
-        mma_commit(smem_u32(&bars.pvdone));
+        const bool last_reader = x == 1 || ntile[1] <= i;
+        if (last_reader) mma_commit(smem_u32(&bars.vempty[vs]));
+        if (i == ntile[x] - 1) mma_commit(smem_u32(&bars.odone[x]));
       }
       __syncwarp();
       issued = true;
     };
-    for (int j = 0; ok && j < nkt; ++j) {
-      const int s = j % kAttnKStages, sb = j & 1;
-      ok = pf_warp_wait(smem_u32(&bars.kfull[s]), (j / kAttnKStages) & 1, abort_flag, p.wait_ns);
-      if (ok && j >= 2) ok = pf_warp_wait(smem_u32(&bars.sfree[sb]), ((j - 2) >> 1) & 1, abort_flag, p.wait_ns);
-      if (!ok) break;
-      tc_fence_after();
-      if (elect_one()) {
-        const uint64_t kd = kdesc + ((s * kAttnKBytes) >> 4);
+    auto issue_s = [&](int x, int j) {
+      const uint64_t qd = qdesc + ((x * kAttnQBytes) >> 4);
+      // the last reader of a key chunk (B, or A when B has no tile j) frees its slot
+      const bool last_reader = x == 1 || ntile[1] <= j;
+      for (int c = 0; c < 3; ++c) {
+        const int g = 3 * j + c, s = g % kAttnKSlots;
+        wait_k(g);
+        if (!ok) return;
+        tc_fence_after();
+        if (elect_one()) {
+          const uint64_t kd = kdesc + ((s * kPfAtom) >> 4);
 #pragma unroll
-        for (int kk = 0; kk < kPfDqk / 16; ++kk)
-          mma_bf16_ss(tmem + sb * kPfRows, qdesc + (((kk >> 2) * kPfAtom + (kk & 3) * 32) >> 4),
-                      kd + (((kk >> 2) * kPfAtom + (kk & 3) * 32) >> 4), idesc_s, kk > 0 ? 1u : 0u);
-        mma_commit(smem_u32(&bars.kempty[s]));
-        mma_commit(smem_u32(&bars.sfull[sb]));
+          for (int kk = 0; kk < 4; ++kk)
+            mma_bf16_ss(tmem + col_s(x), qd + ((c * kPfAtom + kk * 32) >> 4), kd + ((kk * 32) >> 4), idesc_s,
+                        (c > 0 || kk > 0) ? 1u : 0u);
+          if (c == 2) mma_commit(smem_u32(&bars.sfull[x]));
+          if (last_reader) mma_commit(smem_u32(&bars.kempty[s]));
+        }
+        __syncwarp();
       }
-      __syncwarp();
       issued = true;
-      if (j >= 1) issue_pv(j - 1);
+    };
+    for (int j = 0; ok && j <= nkt; ++j) {
+      for (int x = 0; ok && x < 2; ++x) {
+        if (j >= 1 && j - 1 < ntile[x]) issue_pv(x, j - 1);
+        if (ok && j < ntile[x]) issue_s(x, j);
+      }
     }
-    if (ok) issue_pv(nkt - 1);
     if (issued) {
       if (elect_one()) mma_commit(smem_u32(&bars.drain));
       __syncwarp();
@@ -632,38 +680,39 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     }
     __syncwarp();
   } else {
-    // ---- softmax and epilogue: query row r = TMEM lane r
+    // ---- softmax and epilogue of query tile x: query row r = TMEM lane r
+    const int x = (warp - kAttnSoftWarp0) >> 2;
     const int quad = warp & 3;
     const int r = 32 * quad + lane;
+    const int qrow = q0 + x * kPfRows + r;   // this row's position in the prompt
+    const int nx = ntile[x];
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * quad) << 16);
     const float sl2 = p.scale_log2;
     float m_ref = 0.f, l = 0.f;
-    bool ok = true;
-    for (int j = 0; j < nkt; ++j) {
-      const int sb = j & 1;
-      ok = pf_warp_wait(smem_u32(&bars.sfull[sb]), (j >> 1) & 1, abort_flag, p.wait_ns);
+    bool ok = nx > 0;
+    for (int j = 0; ok && j < nx; ++j) {
+      // S_X(j) complete (and with it every earlier MMA: O_X is current)
+      ok = pf_warp_wait(smem_u32(&bars.sfull[x]), j & 1, abort_flag, p.wait_ns);
       if (!ok) break;
       tc_fence_after();
-      float sv[kPfRows];
+      float sv[kAttnKeys];
 #pragma unroll
-      for (int c = 0; c < kPfRows; c += 16)
-        tmem_ld16(lane_base + sb * kPfRows + c, *reinterpret_cast<float(*)[16]>(&sv[c]));
+      for (int c = 0; c < kAttnKeys; c += 16)
+        tmem_ld16(lane_base + col_s(x) + c, *reinterpret_cast<float(*)[16]>(&sv[c]));
       tmem_wait_ld();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&bars.sfree[sb]));
-      if (j == nkt - 1) {
-        // diagonal tile: key c is after query r when c > r
+      const int k0 = j * kAttnKeys;
+      if (k0 + kAttnKeys - 1 > qrow) {
+        // keys after the query (the tile on the diagonal)
 #pragma unroll
-        for (int c = 0; c < kPfRows; ++c)
-          if (c > r) sv[c] = -INFINITY;
+        for (int c = 0; c < kAttnKeys; ++c)
+          if (k0 + c > qrow) sv[c] = -INFINITY;
       }
       // row maximum and sum as eight interleaved chains (short dependencies)
       float m8[8];
 #pragma unroll
       for (int e = 0; e < 8; ++e) m8[e] = sv[e];
 #pragma unroll
-      for (int c = 8; c < kPfRows; ++c) m8[c & 7] = fmaxf(m8[c & 7], sv[c]);
+      for (int c = 8; c < kAttnKeys; ++c) m8[c & 7] = fmaxf(m8[c & 7], sv[c]);
       float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])), fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
       mx *= sl2;
       float alpha = 1.f;
@@ -673,10 +722,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         alpha = pf_ex2(m_ref - mx);
         m_ref = mx;
       }
-      float pk[kPfRows / 2];   // bf16 pairs, kept as 32-bit words for the TMEM store
+      float pk[kAttnKeys / 2];   // bf16 pairs, kept as 32-bit words for the TMEM store
       float r8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int c = 0; c < kPfRows; c += 2) {
+      for (int c = 0; c < kAttnKeys; c += 2) {
         const float p0 = pf_ex2(fmaf(sv[c], sl2, -m_ref));
         const float p1 = pf_ex2(fmaf(sv[c + 1], sl2, -m_ref));
         r8[(c >> 1) & 7] += p0 + p1;
@@ -684,45 +733,38 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       }
       const float rs = ((r8[0] + r8[1]) + (r8[2] + r8[3])) + ((r8[4] + r8[5]) + (r8[6] + r8[7]));
       l = fmaf(l, alpha, rs);
-      // P is single-buffered and O is updated by the previous tile's PV MMA:
-      // both wait for it
-      if (j >= 1) {
-        ok = pf_warp_wait(smem_u32(&bars.pvdone), (j - 1) & 1, abort_flag, p.wait_ns);
-        if (!ok) break;
-        tc_fence_after();
-        if (__any_sync(0xffffffffu, alpha != 1.f)) {
+      if (__any_sync(0xffffffffu, alpha != 1.f)) {
 #pragma unroll
-          for (int c = 0; c < kPfDv; c += 16) {
-            float o[16];
-            tmem_ld16(lane_base + kColO + c, o);
-            tmem_wait_ld();
+        for (int c = 0; c < kPfDv; c += 16) {
+          float o[16];
+          tmem_ld16(lane_base + col_o(x) + c, o);
+          tmem_wait_ld();
 #pragma unroll
-            for (int e = 0; e < 16; ++e) o[e] *= alpha;
-            tmem_st16(lane_base + kColO + c, o);
-          }
-          tmem_wait_st();
+          for (int e = 0; e < 16; ++e) o[e] *= alpha;
+          tmem_st16(lane_base + col_o(x) + c, o);
         }
       }
+      // P_X over the first 64 columns of S_X
 #pragma unroll
-      for (int c = 0; c < kPfRows / 2; c += 16)
-        tmem_st16(lane_base + kColP + c, *reinterpret_cast<const float(*)[16]>(&pk[c]));
+      for (int c = 0; c < kAttnKeys / 2; c += 16)
+        tmem_st16(lane_base + col_s(x) + c, *reinterpret_cast<const float(*)[16]>(&pk[c]));
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&bars.pfull));
+      if (lane == 0) mbar_arrive(smem_u32(&bars.pfull[x]));
     }
-    // ---- epilogue: O / l of the live rows
-    if (ok) ok = pf_warp_wait(smem_u32(&bars.pvdone), (nkt - 1) & 1, abort_flag, p.wait_ns);
+    // ---- epilogue: O_X / l of the live rows
+    if (ok) ok = pf_warp_wait(smem_u32(&bars.odone[x]), 0, abort_flag, p.wait_ns);
     if (ok) {
       tc_fence_after();
       const float inv = 1.f / l;
-      const bool live = q0 + r < L;
-      __nv_bfloat16* orow = p.out + (static_cast<size_t>(start + q0 + (live ? r : 0)) * p.H + h) * kPfDv;
+      const bool live = qrow < L;
+      __nv_bfloat16* orow = p.out + (static_cast<size_t>(start + (live ? qrow : 0)) * p.H + h) * kPfDv;
 #pragma unroll
       for (int c = 0; c < kPfDv; c += 32) {
         float o[32];
-        tmem_ld16(lane_base + kColO + c, *reinterpret_cast<float(*)[16]>(&o[0]));
-        tmem_ld16(lane_base + kColO + c + 16, *reinterpret_cast<float(*)[16]>(&o[16]));
+        tmem_ld16(lane_base + col_o(x) + c, *reinterpret_cast<float(*)[16]>(&o[0]));
+        tmem_ld16(lane_base + col_o(x) + c + 16, *reinterpret_cast<float(*)[16]>(&o[16]));
         tmem_wait_ld();
         if (live) {
           uint4* d = reinterpret_cast<uint4*>(orow + c);
@@ -890,12 +932,12 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st, void (*mark)(c
   ap.batch = a.batch;
   ap.H = a.H;
   ap.total = a.total;
-  ap.qtiles = (a.max_seq_len + kPfRows - 1) / kPfRows;
+  ap.qblocks = (a.max_seq_len + 2 * kPfRows - 1) / (2 * kPfRows);
   ap.scale_log2 = a.scale_log2;
   ap.wait_ns = kWaitLimitNs;
   ap.status = a.status;
-  if (ap.qtiles == 0) return cudaSuccess;
-  const long long grid = static_cast<long long>(a.batch) * a.H * ap.qtiles;
+  if (ap.qblocks == 0) return cudaSuccess;
+  const long long grid = static_cast<long long>(a.batch) * a.H * ap.qblocks;
   if (grid > 0x7fffffffLL) return cudaErrorInvalidValue;
   if (mark) mark(st, true);
   prefill_attn_kernel<<<static_cast<unsigned>(grid), kAttnThreads, kAttnSmem, st>>>(qmap, kvmap, krmap, ap);
