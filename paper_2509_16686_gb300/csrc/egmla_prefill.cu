@@ -7,7 +7,7 @@
 // in the unabsorbed per-head form of the Appendix E listing, which needs
 // 2 (d_n + d_r + d_v) = 640 flops per (query, key, head) instead of the
 // absorbed form's 2 (d_c + d_r + d_c) = 1152:
-//   prefill_gate_kernel  one warp per prompt token: c~ = LN(c (*) G[id]) (or the
+//   prefill_gate_kernel  one warp per four prompt tokens: c~ = LN(c (*) G[id]) (or the
 //                        gate mode's variant; Section 3 Eq. 5 in latent space),
 //                        rounded to bf16, and the raw c, k^R and id written to
 //                        the token's cache slot through the block table.
@@ -110,31 +110,17 @@ struct PfGateParams {
 };
 
 constexpr int kGateWarps = 8;
+constexpr int kGateRows = 4;   // rows per warp, their loads issued together
 
-__global__ void __launch_bounds__(32 * kGateWarps) prefill_gate_kernel(const PfGateParams p) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int t = blockIdx.x * kGateWarps + warp;
-  if (t >= p.total) return;
-  const int b = prompt_of_row(p.cu, p.batch, t);
-  const int pos = t - __ldg(p.cu + b);
-  const int nu = p.d_c / 8;   // 16-byte units of a row (at most 64: two per lane)
-  bool bad = false;
-  int id = p.ids ? __ldg(p.ids + t) : 0;
-  if (p.gate && static_cast<unsigned>(id) >= static_cast<unsigned>(p.vocab)) {
-    bad = true;
-    id = 0;
-  }
-  uint4 craw[2];
+// c~ of one row from its loaded c and g units, stored, and the row's cache write
+__device__ __forceinline__ void gate_row(const PfGateParams& p, int t, int b, int pos, int lane, int nu,
+                                         const uint4 (&craw)[2], const uint4 (&graw)[2], bool& bad) {
   float z[2][8];
 #pragma unroll
   for (int i = 0; i < 2; ++i) {
     const int u = lane + 32 * i;
-    craw[i] = make_uint4(0u, 0u, 0u, 0u);
-    if (u < nu) craw[i] = __ldg(reinterpret_cast<const uint4*>(p.c + static_cast<size_t>(t) * p.d_c) + u);
     const __nv_bfloat162* c2 = reinterpret_cast<const __nv_bfloat162*>(&craw[i]);
-    uint4 graw = make_uint4(0u, 0u, 0u, 0u);
-    if (p.gate && u < nu) graw = __ldg(reinterpret_cast<const uint4*>(p.gate_table + static_cast<size_t>(id) * p.d_c) + u);
-    const __nv_bfloat162* g2 = reinterpret_cast<const __nv_bfloat162*>(&graw);
+    const __nv_bfloat162* g2 = reinterpret_cast<const __nv_bfloat162*>(&graw[i]);
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
       const float2 cf = __bfloat1622float2(c2[e]);
@@ -206,6 +192,55 @@ __global__ void __launch_bounds__(32 * kGateWarps) prefill_gate_kernel(const PfG
       if (lane == 0 && p.id_pool && p.ids) p.id_pool[slot] = __ldg(p.ids + t);
     }
   }
+}
+
+// One warp per kGateRows consecutive token rows: their prompt found once,
+// then the rows' ids and latents requested together, then their gate rows.
+__global__ void __launch_bounds__(32 * kGateWarps) prefill_gate_kernel(const PfGateParams p) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int t0 = (blockIdx.x * kGateWarps + warp) * kGateRows;
+  if (t0 >= p.total) return;
+  const int nu = p.d_c / 8;   // 16-byte units of a row (at most 64: two per lane)
+  bool bad = false;
+  int tb[kGateRows], pos[kGateRows], id[kGateRows];
+  int b = prompt_of_row(p.cu, p.batch, t0);
+#pragma unroll
+  for (int r = 0; r < kGateRows; ++r) {
+    const int t = t0 + r;
+    while (b + 1 < p.batch && __ldg(p.cu + b + 1) <= t) ++b;
+    tb[r] = b;
+    pos[r] = t - __ldg(p.cu + b);
+  }
+  uint4 craw[kGateRows][2], graw[kGateRows][2];
+#pragma unroll
+  for (int r = 0; r < kGateRows; ++r) {
+    const int t = t0 + r;
+    id[r] = (p.ids && t < p.total) ? __ldg(p.ids + t) : 0;
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int u = lane + 32 * i;
+      craw[r][i] = make_uint4(0u, 0u, 0u, 0u);
+      if (u < nu && t < p.total)
+        craw[r][i] = __ldg(reinterpret_cast<const uint4*>(p.c + static_cast<size_t>(t) * p.d_c) + u);
+    }
+  }
+#pragma unroll
+  for (int r = 0; r < kGateRows; ++r) {
+    if (p.gate && static_cast<unsigned>(id[r]) >= static_cast<unsigned>(p.vocab)) {
+      if (t0 + r < p.total) bad = true;
+      id[r] = 0;
+    }
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int u = lane + 32 * i;
+      graw[r][i] = make_uint4(0u, 0u, 0u, 0u);
+      if (p.gate && u < nu)
+        graw[r][i] = __ldg(reinterpret_cast<const uint4*>(p.gate_table + static_cast<size_t>(id[r]) * p.d_c) + u);
+    }
+  }
+#pragma unroll
+  for (int r = 0; r < kGateRows; ++r)
+    if (t0 + r < p.total) gate_row(p, t0 + r, tb[r], pos[r], lane, nu, craw[r], graw[r], bad);
   if (bad && lane == 0) report_status(p.status, kStatusOutOfRange);
 }
 
@@ -877,7 +912,8 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st, void (*mark)(c
   gp.gate_ln = a.gate_ln;
   gp.eps = a.eps;
   gp.status = a.status;
-  prefill_gate_kernel<<<(a.total + kGateWarps - 1) / kGateWarps, 32 * kGateWarps, 0, st>>>(gp);
+  prefill_gate_kernel<<<(a.total + kGateWarps * kGateRows - 1) / (kGateWarps * kGateRows), 32 * kGateWarps, 0, st>>>(
+      gp);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
 
