@@ -470,8 +470,9 @@ int eg_mla_decode_r0(const eg_mla_dims* dims, const void* q, const void* c_pool,
  *                the paged cache as for eg_mla_append_latent; c_pool NULL
  *                skips the cache write (the other four are then ignored);
  *                id_pool may be NULL with EG_MLA_GATE_NONE
- *   workspace    >= eg_mla_prefill_workspace_size(dims, total_tokens) bytes,
- *                256-byte aligned: c~ of every token (d_c bf16) and its
+ *   workspace    >= eg_mla_prefill_workspace_size(dims, batch, total_tokens)
+ *                bytes, 256-byte aligned: the prompts' launch order (longest
+ *                first; batch int32), c~ of every token (d_c bf16) and its
  *                per-head keys and values (num_heads * 256 bf16)
  * All tensor arguments read or written in 16-byte pieces must be 16-byte
  * aligned.  Host errors return at once (nothing launched).  Device errors go
@@ -481,7 +482,7 @@ int eg_mla_decode_r0(const eg_mla_dims* dims, const void* q, const void* c_pool,
  * prompt longer than max_seq_len (its rows past the bound are not computed)
  * as EG_MLA_ERR_OUT_OF_RANGE; a timed-out pipeline wait as EG_MLA_ERR_TIMEOUT.
  */
-size_t eg_mla_prefill_workspace_size(const eg_mla_dims* dims, int32_t total_tokens);
+size_t eg_mla_prefill_workspace_size(const eg_mla_dims* dims, int32_t batch, int32_t total_tokens);
 int eg_mla_prefill(const eg_mla_dims* dims, const void* q, const void* c_new, const void* krope_new,
                    const int32_t* ids_new, const int32_t* cu_seqlens, int32_t batch, int32_t total_tokens,
                    int32_t max_seq_len, const void* gate_table, const float* ln_gamma, const float* ln_beta,

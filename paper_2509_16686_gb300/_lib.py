@@ -108,7 +108,7 @@ def _declare(lib: ctypes.CDLL) -> None:
     lib.eg_mla_decode_r0_workspace_size.restype = SZ
     lib.eg_mla_decode_r0.argtypes = [D, P, P, P, P, P, I32, P, I32, I32, P, P, P, P, P, P, SZ, P, P]
     lib.eg_mla_decode_r0.restype = ctypes.c_int
-    lib.eg_mla_prefill_workspace_size.argtypes = [D, I32]
+    lib.eg_mla_prefill_workspace_size.argtypes = [D, I32, I32]
     lib.eg_mla_prefill_workspace_size.restype = SZ
     lib.eg_mla_prefill.argtypes = [D, P, P, P, P, P, I32, I32, I32, P, P, P, P, P, P, P, P, P, P, I32, I32,
                                    P, SZ, P, P]
@@ -359,8 +359,8 @@ def eg_mla_decode_r0(dims: EgMlaDims, q, c_pool, krope_pool, id_pool, block_tabl
     _check(code, "eg_mla_decode_r0")
 
 
-def eg_mla_prefill_workspace_size(dims: EgMlaDims, total_tokens: int) -> int:
-    n = load().eg_mla_prefill_workspace_size(ctypes.byref(dims), int(total_tokens))
+def eg_mla_prefill_workspace_size(dims: EgMlaDims, batch: int, total_tokens: int) -> int:
+    n = load().eg_mla_prefill_workspace_size(ctypes.byref(dims), int(batch), int(total_tokens))
     if n == 0 and total_tokens > 0:
         raise EgMlaError(EG_MLA_ERR_UNSUPPORTED, "eg_mla_prefill_workspace_size")
     return int(n)

@@ -552,9 +552,9 @@ int eg_mla_decode_r0(const eg_mla_dims* dims, const void* q, const void* c_pool,
   return to_status(egmla::launch_decode_r0(a, static_cast<cudaStream_t>(stream)));
 }
 
-size_t eg_mla_prefill_workspace_size(const eg_mla_dims* dims, int32_t total_tokens) {
-  if (check_prefill_dims(dims) != EG_MLA_OK || total_tokens < 0) return 0;
-  return egmla::prefill_workspace_bytes(total_tokens, dims->num_heads, dims->d_c);
+size_t eg_mla_prefill_workspace_size(const eg_mla_dims* dims, int32_t batch, int32_t total_tokens) {
+  if (check_prefill_dims(dims) != EG_MLA_OK || total_tokens < 0 || batch < 0) return 0;
+  return egmla::prefill_workspace_bytes(batch, total_tokens, dims->num_heads, dims->d_c);
 }
 
 int eg_mla_prefill(const eg_mla_dims* dims, const void* q, const void* c_new, const void* krope_new,
@@ -583,7 +583,7 @@ int eg_mla_prefill(const eg_mla_dims* dims, const void* q, const void* c_new, co
   const int64_t qtiles = (static_cast<int64_t>(max_seq_len) + 127) / 128;
   if (static_cast<int64_t>(batch) * dims->num_heads * qtiles > INT32_MAX) return EG_MLA_ERR_UNSUPPORTED;
   if (workspace == nullptr || !aligned(workspace, 256) ||
-      workspace_bytes < egmla::prefill_workspace_bytes(total_tokens, dims->num_heads, dims->d_c))
+      workspace_bytes < egmla::prefill_workspace_bytes(batch, total_tokens, dims->num_heads, dims->d_c))
     return EG_MLA_ERR_WORKSPACE;
   egmla::PrefillArgs a;
   std::memset(&a, 0, sizeof(a));

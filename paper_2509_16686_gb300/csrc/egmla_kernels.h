@@ -132,7 +132,7 @@ struct PrefillArgs {
   int gate, gate_add, gate_ln;
   float eps, scale_log2;
 };
-size_t prefill_workspace_bytes(int total_tokens, int H, int d_c);
+size_t prefill_workspace_bytes(int batch, int total_tokens, int H, int d_c);
 bool prefill_supported(int d_nope, int d_rope, int d_v, int d_c);
 // `mark` (may be null) is called with (stream, true) just before the
 // attention kernel's launch and (stream, false) just after it.

@@ -7,7 +7,7 @@
 // in the unabsorbed per-head form of the Appendix E listing, which needs
 // 2 (d_n + d_r + d_v) = 640 flops per (query, key, head) instead of the
 // absorbed form's 2 (d_c + d_r + d_c) = 1152:
-//   prefill_gate_kernel  one warp per four prompt tokens: c~ = LN(c (*) G[id]) (or the
+//   prefill_gate_kernel  one warp per prompt token: c~ = LN(c (*) G[id]) (or the
 //                        gate mode's variant; Section 3 Eq. 5 in latent space),
 //                        rounded to bf16, and the raw c, k^R and id written to
 //                        the token's cache slot through the block table.
@@ -91,6 +91,7 @@ __device__ __forceinline__ int prompt_of_row(const int32_t* cu, int batch, int t
 
 // ============================================================================ 1. gate, LayerNorm, cache write
 struct PfGateParams {
+  int32_t* order;              // [batch]: prompts by decreasing length (written by block 0)
   const __nv_bfloat16* c;      // [T, d_c]
   const __nv_bfloat16* kr;     // [T, d_r]
   const int32_t* ids;          // [T] (null with the gate off)
@@ -110,7 +111,6 @@ struct PfGateParams {
 };
 
 constexpr int kGateWarps = 8;
-constexpr int kGateRows = 4;   // rows per warp, their loads issued together
 
 // c~ of one row from its loaded c and g units, stored, and the row's cache write
 __device__ __forceinline__ void gate_row(const PfGateParams& p, int t, int b, int pos, int lane, int nu,
@@ -194,53 +194,50 @@ __device__ __forceinline__ void gate_row(const PfGateParams& p, int t, int b, in
   }
 }
 
-// One warp per kGateRows consecutive token rows: their prompt found once,
-// then the rows' ids and latents requested together, then their gate rows.
+constexpr int kSortMaxBatch = 2048;   // larger batches keep the given order
+
+// One warp per token row.
 __global__ void __launch_bounds__(32 * kGateWarps) prefill_gate_kernel(const PfGateParams p) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int t0 = (blockIdx.x * kGateWarps + warp) * kGateRows;
-  if (t0 >= p.total) return;
+  if (blockIdx.x == 0) {
+    // the attention's launch order: longest prompts first (rank of each prompt
+    // among all by length, ties by index), so that the longest prompts'
+    // query blocks do not start last
+    for (int b = threadIdx.x; b < p.batch; b += blockDim.x) {
+      int rank = b;
+      if (p.batch <= kSortMaxBatch) {
+        const int Lb = __ldg(p.cu + b + 1) - __ldg(p.cu + b);
+        rank = 0;
+        for (int o = 0; o < p.batch; ++o) {
+          const int Lo = __ldg(p.cu + o + 1) - __ldg(p.cu + o);
+          rank += (Lo > Lb || (Lo == Lb && o < b)) ? 1 : 0;
+        }
+      }
+      p.order[rank] = b;
+    }
+  }
+  const int t = blockIdx.x * kGateWarps + warp;
+  if (t >= p.total) return;
   const int nu = p.d_c / 8;   // 16-byte units of a row (at most 64: two per lane)
+  const int b = prompt_of_row(p.cu, p.batch, t);
+  const int pos = t - __ldg(p.cu + b);
   bool bad = false;
-  int tb[kGateRows], pos[kGateRows], id[kGateRows];
-  int b = prompt_of_row(p.cu, p.batch, t0);
-#pragma unroll
-  for (int r = 0; r < kGateRows; ++r) {
-    const int t = t0 + r;
-    while (b + 1 < p.batch && __ldg(p.cu + b + 1) <= t) ++b;
-    tb[r] = b;
-    pos[r] = t - __ldg(p.cu + b);
+  int id = p.ids ? __ldg(p.ids + t) : 0;
+  if (p.gate && static_cast<unsigned>(id) >= static_cast<unsigned>(p.vocab)) {
+    bad = true;
+    id = 0;
   }
-  uint4 craw[kGateRows][2], graw[kGateRows][2];
+  uint4 craw[2], graw[2];
 #pragma unroll
-  for (int r = 0; r < kGateRows; ++r) {
-    const int t = t0 + r;
-    id[r] = (p.ids && t < p.total) ? __ldg(p.ids + t) : 0;
-#pragma unroll
-    for (int i = 0; i < 2; ++i) {
-      const int u = lane + 32 * i;
-      craw[r][i] = make_uint4(0u, 0u, 0u, 0u);
-      if (u < nu && t < p.total)
-        craw[r][i] = __ldg(reinterpret_cast<const uint4*>(p.c + static_cast<size_t>(t) * p.d_c) + u);
-    }
+  for (int i = 0; i < 2; ++i) {
+    const int u = lane + 32 * i;
+    craw[i] = make_uint4(0u, 0u, 0u, 0u);
+    graw[i] = make_uint4(0u, 0u, 0u, 0u);
+    if (u < nu) craw[i] = __ldg(reinterpret_cast<const uint4*>(p.c + static_cast<size_t>(t) * p.d_c) + u);
+    if (p.gate && u < nu)
+      graw[i] = __ldg(reinterpret_cast<const uint4*>(p.gate_table + static_cast<size_t>(id) * p.d_c) + u);
   }
-#pragma unroll
-  for (int r = 0; r < kGateRows; ++r) {
-    if (p.gate && static_cast<unsigned>(id[r]) >= static_cast<unsigned>(p.vocab)) {
-      if (t0 + r < p.total) bad = true;
-      id[r] = 0;
-    }
-#pragma unroll
-    for (int i = 0; i < 2; ++i) {
-      const int u = lane + 32 * i;
-      graw[r][i] = make_uint4(0u, 0u, 0u, 0u);
-      if (p.gate && u < nu)
-        graw[r][i] = __ldg(reinterpret_cast<const uint4*>(p.gate_table + static_cast<size_t>(id[r]) * p.d_c) + u);
-    }
-  }
-#pragma unroll
-  for (int r = 0; r < kGateRows; ++r)
-    if (t0 + r < p.total) gate_row(p, t0 + r, tb[r], pos[r], lane, nu, craw[r], graw[r], bad);
+  gate_row(p, t, b, pos, lane, nu, craw, graw, bad);
   if (bad && lane == 0) report_status(p.status, kStatusOutOfRange);
 }
 
@@ -510,6 +507,7 @@ constexpr uint32_t kAttnSmem = kOffBars + sizeof(AttnBars) + 1024;
 
 struct AttnParams {
   const int32_t* cu;
+  const int32_t* order;   // prompts in launch order
   __nv_bfloat16* out;   // [T, H, d_v]
   int batch, H, qblocks, total;
   float scale_log2;
@@ -524,7 +522,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   // (prompt, head) are neighbours in launch order, so its keys stay in L2
   const int group = blockIdx.x / p.qblocks;
   const int qb = p.qblocks - 1 - blockIdx.x % p.qblocks;
-  const int b = group / p.H, h = group % p.H;
+  const int b = __ldg(p.order + group / p.H), h = group % p.H;
   const int start = __ldg(p.cu + b);
   const int L = __ldg(p.cu + b + 1) - start;
   const int q0 = qb * 2 * kPfRows;
@@ -856,12 +854,14 @@ bool pf_encode(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols,
 }
 
 struct PfWorkspace {
-  size_t off_ctil, off_kv, total;
+  size_t off_order, off_ctil, off_kv, total;
 };
 
-PfWorkspace pf_layout(int total, int H, int d_c) {
+PfWorkspace pf_layout(int batch, int total, int H, int d_c) {
   PfWorkspace w;
   size_t off = 0;
+  w.off_order = off;
+  off = align_up(off + static_cast<size_t>(batch) * 4, 256);
   w.off_ctil = off;
   off = align_up(off + static_cast<size_t>(total) * d_c * 2, 256);
   w.off_kv = off;
@@ -872,7 +872,9 @@ PfWorkspace pf_layout(int total, int H, int d_c) {
 
 }  // namespace
 
-size_t prefill_workspace_bytes(int total_tokens, int H, int d_c) { return pf_layout(total_tokens, H, d_c).total; }
+size_t prefill_workspace_bytes(int batch, int total_tokens, int H, int d_c) {
+  return pf_layout(batch, total_tokens, H, d_c).total;
+}
 
 bool prefill_supported(int d_nope, int d_rope, int d_v, int d_c) {
   return d_nope == kPfDn && d_rope == kPfDr && d_v == kPfDv && d_c % kPfChunk == 0 && d_c >= kPfChunk &&
@@ -881,13 +883,15 @@ bool prefill_supported(int d_nope, int d_rope, int d_v, int d_c) {
 
 cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st, void (*mark)(cudaStream_t, bool)) {
   if (a.total <= 0 || a.batch <= 0) return cudaSuccess;
-  const PfWorkspace w = pf_layout(a.total, a.H, a.d_c);
+  const PfWorkspace w = pf_layout(a.batch, a.total, a.H, a.d_c);
   uint8_t* ws = static_cast<uint8_t*>(a.workspace);
+  int32_t* order = reinterpret_cast<int32_t*>(ws + w.off_order);
   __nv_bfloat16* ctil = reinterpret_cast<__nv_bfloat16*>(ws + w.off_ctil);
   __nv_bfloat16* kv = reinterpret_cast<__nv_bfloat16*>(ws + w.off_kv);
 
   // 1. gate, LayerNorm, cache write
   PfGateParams gp;
+  gp.order = order;
   gp.c = static_cast<const __nv_bfloat16*>(a.c);
   gp.kr = static_cast<const __nv_bfloat16*>(a.kr);
   gp.ids = a.ids;
@@ -912,8 +916,7 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st, void (*mark)(c
   gp.gate_ln = a.gate_ln;
   gp.eps = a.eps;
   gp.status = a.status;
-  prefill_gate_kernel<<<(a.total + kGateWarps * kGateRows - 1) / (kGateWarps * kGateRows), 32 * kGateWarps, 0, st>>>(
-      gp);
+  prefill_gate_kernel<<<(a.total + kGateWarps - 1) / kGateWarps, 32 * kGateWarps, 0, st>>>(gp);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
 
@@ -964,6 +967,7 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st, void (*mark)(c
   if (e != cudaSuccess) return e;
   AttnParams ap;
   ap.cu = a.cu_seqlens;
+  ap.order = order;
   ap.out = static_cast<__nv_bfloat16*>(a.out);
   ap.batch = a.batch;
   ap.H = a.H;

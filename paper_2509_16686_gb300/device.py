@@ -291,7 +291,7 @@ def upload_prefill(pc, device="cuda") -> DevicePrefill:
         id_pool=to_device_array(pc.id_pool, dt, device),
         block_table=to_device_array(pc.block_table, dt, device),
         out=torch.empty((T, d.num_heads, d.d_v), dtype=torch.bfloat16, device=device),
-        workspace=torch.empty(max(_lib.eg_mla_prefill_workspace_size(dims, T), 1), dtype=torch.uint8,
+        workspace=torch.empty(max(_lib.eg_mla_prefill_workspace_size(dims, pc.batch, T), 1), dtype=torch.uint8,
                               device=device),
         status=torch.zeros(1, dtype=torch.int32, device=device),
         max_seq_len=int(pc.seq_lens.max()) if pc.batch else 0,
