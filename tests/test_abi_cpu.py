@@ -159,3 +159,52 @@ def test_layer_attention_offset_is_inside_the_workspace(lib):
     ws = _lib.eg_mla_layer_workspace_size(dims, layer, 64, 152)
     off = _lib.eg_mla_layer_attn_offset(dims, layer, 64, 152)
     assert 0 < off and off % 256 == 0 and off + 64 * 16 * 128 * 2 <= ws
+
+
+# --------------------------------------------------------------------------- prefill: host-side checks
+def _prefill_call(lib, dims, **kw):
+    """eg_mla_prefill with fake, aligned device addresses; each case makes one
+    host check fail, so the call returns before anything is launched."""
+    P = lambda v: ctypes.c_void_p(v)
+    a = dict(q=0x1000, c=0x2000, kr=0x3000, ids=0x4000, cu=0x5000, batch=2, total=100, max_len=60, gate=0x6000,
+             gamma=None, beta=None, w_uk=0x7000, w_uv=0x8000, out=0x9000, c_pool=None, kr_pool=None, id_pool=None,
+             bt=None, max_pages=0, num_pages=0, ws=0xA000, ws_bytes=1 << 30, status=None)
+    a.update(kw)
+    return lib.eg_mla_prefill(ctypes.byref(dims), P(a["q"]), P(a["c"]), P(a["kr"]), P(a["ids"]), P(a["cu"]),
+                              a["batch"], a["total"], a["max_len"], P(a["gate"]), P(a["gamma"]), P(a["beta"]),
+                              P(a["w_uk"]), P(a["w_uv"]), P(a["out"]), P(a["c_pool"]), P(a["kr_pool"]),
+                              P(a["id_pool"]), P(a["bt"]), a["max_pages"], a["num_pages"], P(a["ws"]),
+                              ctypes.c_size_t(a["ws_bytes"]), P(a["status"]), None)
+
+
+def test_prefill_workspace_size(lib):
+    d = _lib.make_dims(16, 128, 64, 128, 256, 32000)
+    n = _lib.eg_mla_prefill_workspace_size(d, 8, 32768)
+    # launch order (8 int32), c~ (32768 x 256 bf16), keys and values (32768 x 16 x 256 bf16)
+    assert n == 256 + 32768 * 256 * 2 + 32768 * 16 * 256 * 2
+    assert lib.eg_mla_prefill_workspace_size(ctypes.byref(_lib.make_dims(16, 64, 64, 128, 256, 32000)), 8, 100) == 0
+
+
+def test_prefill_rejects_bad_arguments(lib):
+    d = _lib.make_dims(16, 128, 64, 128, 256, 32000)
+    assert _prefill_call(lib, d, batch=0) == _lib.EG_MLA_OK                 # nothing to do
+    assert _prefill_call(lib, d, total=0) == _lib.EG_MLA_OK
+    assert _prefill_call(lib, d, batch=-1) == _lib.EG_MLA_ERR_INVALID_ARG
+    assert _prefill_call(lib, d, max_len=0) == _lib.EG_MLA_ERR_INVALID_ARG
+    assert _prefill_call(lib, d, max_len=101) == _lib.EG_MLA_ERR_INVALID_ARG  # longer than all tokens
+    assert _prefill_call(lib, d, q=0) == _lib.EG_MLA_ERR_INVALID_ARG
+    assert _prefill_call(lib, d, ids=0) == _lib.EG_MLA_ERR_INVALID_ARG       # gated: ids needed
+    assert _prefill_call(lib, d, gate=0) == _lib.EG_MLA_ERR_INVALID_ARG
+    assert _prefill_call(lib, d, out=0x9008) == _lib.EG_MLA_ERR_INVALID_ARG  # 16-byte alignment
+    assert _prefill_call(lib, d, c_pool=0xB000) == _lib.EG_MLA_ERR_INVALID_ARG  # pool without block table
+    assert _prefill_call(lib, d, ws_bytes=1000) == _lib.EG_MLA_ERR_WORKSPACE
+    assert _prefill_call(lib, d, ws=0xA010) == _lib.EG_MLA_ERR_WORKSPACE     # 256-byte alignment
+    for bad in (_lib.make_dims(16, 64, 64, 128, 256, 32000),                   # d_nope 64
+                _lib.make_dims(16, 128, 32, 128, 256, 32000),                  # d_rope 32
+                _lib.make_dims(16, 128, 64, 128, 200, 32000),                  # d_c not a multiple of 64
+                _lib.make_dims(16, 128, 64, 128, 576, 32000),                  # d_c above 512
+                _lib.make_dims(4, 128, 64, 128, 256, 1000, dtype="fp32")):     # fp32
+        assert _prefill_call(lib, bad) == _lib.EG_MLA_ERR_UNSUPPORTED
+    # gate off: ids and gate table may be null
+    d_off = _lib.make_dims(16, 128, 64, 128, 256, 32000, gate=False)
+    assert _prefill_call(lib, d_off, ids=0, gate=0, ws_bytes=1000) == _lib.EG_MLA_ERR_WORKSPACE

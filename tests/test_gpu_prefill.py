@@ -60,6 +60,11 @@ CASES = {
     "add_ln": dict(dims=synth.dims_bf16(d_c=256, vocab=3000, gate_op="add_ln"), lens=(150, 70), affine=True),
     "heads5_dc128": dict(dims=synth.Dims(num_heads=5, d_nope=128, d_rope=64, d_v=128, d_c=128, page_size=64,
                                          vocab=700, dtype="bf16"), lens=(140, 257)),
+    # the gated latent at d_c 512 (one 128-row tile per up-projection CTA),
+    # and a single head at d_c 64
+    "gate512": dict(dims=synth.dims_bf16(d_c=512, vocab=3000), lens=(300, 129), affine=True),
+    "head1_dc64": dict(dims=synth.Dims(num_heads=1, d_nope=128, d_rope=64, d_v=128, d_c=64, page_size=64,
+                                       vocab=500, dtype="bf16"), lens=(64, 1, 200)),
 }
 
 
@@ -154,3 +159,35 @@ def test_prefill_full_size_sampled_rows(gpu_lib):
             refs.append(orc.decode_unabsorbed(case)[0])
             pos.append(t)
     check_close(np.stack(rows), np.stack(refs), pos)
+
+
+def test_prefill_prompt_longer_than_the_bound_is_reported(gpu_lib):
+    """max_seq_len below a prompt's length: the rows past the bound are not
+    computed and the call reports EG_MLA_ERR_OUT_OF_RANGE; the other rows are
+    right."""
+    pc = synth.make_prefill_case("bound", synth.dims_bf16(d_c=256, vocab=3000), [300, 200], seed=67)
+    dp = device.upload_prefill(pc)
+    dp.max_seq_len = 256
+    dp.out.fill_(float("nan"))
+    dp.run()
+    torch.cuda.synchronize()
+    assert dp.read_status() == _lib.EG_MLA_ERR_OUT_OF_RANGE
+    got = device.output_f64(dp.out)
+    ref = orc.prefill(pc)
+    rows = np.r_[0:256, 300:500]   # prompt 0 up to the bound, all of prompt 1
+    check_close(got[rows], ref[rows], positions_of(pc)[rows])
+
+
+def test_prefill_offsets_past_the_tokens_are_reported(gpu_lib):
+    """cu_seqlens claiming more rows than the call has: the prompt that does
+    not fit is skipped and reported; the prompts that fit are right."""
+    pc = synth.make_prefill_case("cu", synth.dims_bf16(d_c=256, vocab=3000), [150, 90], seed=68)
+    dp = device.upload_prefill(pc)
+    dp.cu_seqlens[2] = pc.total_tokens + 50
+    dp.out.fill_(float("nan"))
+    dp.run()
+    torch.cuda.synchronize()
+    assert dp.read_status() == _lib.EG_MLA_ERR_OUT_OF_RANGE
+    got = device.output_f64(dp.out)
+    ref = orc.prefill(pc)
+    check_close(got[:150], ref[:150], positions_of(pc)[:150])
