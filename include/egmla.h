@@ -491,6 +491,27 @@ int eg_mla_prefill(const eg_mla_dims* dims, const void* q, const void* c_new, co
                    void* workspace, size_t workspace_bytes, int32_t* dev_status, void* stream);
 
 /*
+ * eg_mla_gate_table - the gate table of every vocabulary entry,
+ * G[i] = W^UE Emb(i) (Section 3 Eqs. 3-4), computed on the GPU:
+ * G [vocab, d_c] = E [vocab, d_e] W^UE^T with fp32 accumulation, rounded to
+ * bf16.  EG-MLA-A keeps G from model load on; calling this before each
+ * eg_mla_step instead gates the decode with the embedding's projection
+ * computed in the step (the EG-MLA form without a stored table), at
+ * vocab x d_e x d_c MACs per call.
+ *
+ *   dims        dtype bf16; dims->vocab rows, dims->d_c a multiple of 64
+ *   d_e         embedding width, a multiple of 64 up to 512
+ *   emb         [vocab, d_e] bf16 row-major, 16-byte aligned
+ *   w_ue        [d_c, d_e] bf16 row-major (the Linear weight layout), 16-byte aligned
+ *   gate_table  [vocab, d_c] bf16 row-major, written; 16-byte aligned
+ * Returns EG_MLA_ERR_UNSUPPORTED for other shapes or dtypes,
+ * EG_MLA_ERR_INVALID_ARG for null or misaligned pointers; a timed-out
+ * pipeline wait is reported in *dev_status (may be NULL).
+ */
+int eg_mla_gate_table(const eg_mla_dims* dims, int32_t d_e, const void* emb, const void* w_ue, void* gate_table,
+                      int32_t* dev_status, void* stream);
+
+/*
  * eg_mla_debug_linear - the projection GEMM of eg_mla_layer_decode on its own
  * (a testing aid): out[b][n] = sum_j x[b][j] w[n][j] for b < batch,
  * n < n_out (Eq. 14 and the projections of Appendix C Eqs. 1, 8-10 are of

@@ -47,6 +47,7 @@ EXPORTED = [
     "eg_mla_decode_r0",
     "eg_mla_prefill_workspace_size",
     "eg_mla_prefill",
+    "eg_mla_gate_table",
     "eg_mla_kv_bytes_per_token",
     "eg_mla_status_string",
     "eg_mla_debug_gather",
@@ -113,6 +114,8 @@ def _declare(lib: ctypes.CDLL) -> None:
     lib.eg_mla_prefill.argtypes = [D, P, P, P, P, P, I32, I32, I32, P, P, P, P, P, P, P, P, P, P, I32, I32,
                                    P, SZ, P, P]
     lib.eg_mla_prefill.restype = ctypes.c_int
+    lib.eg_mla_gate_table.argtypes = [D, I32, P, P, P, P, P]
+    lib.eg_mla_gate_table.restype = ctypes.c_int
     lib.eg_mla_debug_linear.argtypes = [P, I32, I32, P, I32, P, I32, I32, P, P]
     lib.eg_mla_debug_linear.restype = ctypes.c_int
     lib.eg_mla_debug_linear_plan.argtypes = [I32, I32, I32, ctypes.POINTER(I32), ctypes.POINTER(I32),
@@ -379,6 +382,13 @@ def eg_mla_prefill(dims: EgMlaDims, q, c_new, krope_new, ids_new, cu_seqlens, ma
         block_table.shape[1] if block_table is not None else 0, c_pool.shape[0] if c_pool is not None else 0,
         _ptr(workspace), workspace.numel() * workspace.element_size(), _ptr(dev_status), _stream(stream))
     _check(code, "eg_mla_prefill")
+
+
+def eg_mla_gate_table(dims: EgMlaDims, emb, w_ue, gate_table, dev_status=None, stream=None) -> None:
+    """G = E W^UE^T for every vocabulary entry: emb [vocab, d_e], w_ue [d_c, d_e],
+    gate_table [vocab, d_c], all bf16 (see include/egmla.h)."""
+    _check(load().eg_mla_gate_table(ctypes.byref(dims), emb.shape[1], _ptr(emb), _ptr(w_ue), _ptr(gate_table),
+                                    _ptr(dev_status), _stream(stream)), "eg_mla_gate_table")
 
 
 def eg_mla_debug_linear(w, x, out, dev_status=None, stream=None) -> None:

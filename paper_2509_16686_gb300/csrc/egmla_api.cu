@@ -620,6 +620,16 @@ int eg_mla_prefill(const eg_mla_dims* dims, const void* q, const void* c_new, co
   return to_status(egmla::launch_prefill(a, static_cast<cudaStream_t>(stream), prof_mark));
 }
 
+int eg_mla_gate_table(const eg_mla_dims* dims, int32_t d_e, const void* emb, const void* w_ue, void* gate_table,
+                      int32_t* dev_status, void* stream) {
+  if (dims == nullptr || d_e <= 0 || dims->vocab <= 0 || dims->d_c <= 0) return EG_MLA_ERR_INVALID_ARG;
+  if (dims->dtype != EG_MLA_BF16 || d_e % 64 != 0 || d_e > 512 || dims->d_c % 64 != 0) return EG_MLA_ERR_UNSUPPORTED;
+  if (!emb || !w_ue || !gate_table || !aligned(emb, 16) || !aligned(w_ue, 16) || !aligned(gate_table, 16))
+    return EG_MLA_ERR_INVALID_ARG;
+  return to_status(egmla::launch_gate_table(emb, w_ue, dims->vocab, d_e, dims->d_c, gate_table, dev_status,
+                                            static_cast<cudaStream_t>(stream)));
+}
+
 int eg_mla_debug_linear(const void* w, int32_t n_out, int32_t k, const void* x, int32_t batch, void* out,
                         int32_t ldo, int32_t out_f32, int32_t* dev_status, void* stream) {
   if (n_out <= 0 || k <= 0 || batch < 0 || ldo < n_out || k % 8 != 0) return EG_MLA_ERR_INVALID_ARG;

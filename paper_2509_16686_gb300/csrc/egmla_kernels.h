@@ -137,6 +137,11 @@ bool prefill_supported(int d_nope, int d_rope, int d_v, int d_c);
 // `mark` (may be null) is called with (stream, true) just before the
 // attention kernel's launch and (stream, false) just after it.
 cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st, void (*mark)(cudaStream_t, bool));
+// The gate table G = E W^UE^T (Section 3 Eqs. 3-4 for every vocabulary
+// entry): E [vocab, d_e], W^UE [d_c, d_e] bf16 row-major, G [vocab, d_c] bf16;
+// d_e a multiple of 64 up to 512, d_c a multiple of 64 (egmla_prefill.cu).
+cudaError_t launch_gate_table(const void* emb, const void* w_ue, int vocab, int d_e, int d_c, void* table,
+                              int32_t* status, cudaStream_t st);
 // out[b][n] = sum_k x[b][k] W[n][k] for b < batch, n < n_out: W [n_out, k] and
 // x [batch, k] bf16 row-major (16-byte aligned, k % 8 == 0), out fp32 or
 // bf16 with row stride ldo elements (egmla_linear.cu).  Launched with

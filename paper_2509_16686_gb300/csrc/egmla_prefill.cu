@@ -270,6 +270,11 @@ struct KvBars {
 struct KvParams {
   __nv_bfloat16* kv;   // [T, H, 256]
   int total, H, nkc, stages;
+  // kv_mode 1: block b is the key (b even) or value (b odd) rows of head b / 2
+  // from the two weight maps; kv_mode 0: block b is rows 128 b .. 128 b + 127
+  // of the first map (a plain x W^T, e.g. the gate table E W^UE^T)
+  int nblocks, kv_mode;
+  int out_cols;   // output row width (elements): stores of chunks past it are skipped
   uint64_t wait_ns;
   int32_t* status;
 };
@@ -303,7 +308,7 @@ __global__ void __launch_bounds__(kKvThreads, 1)
   volatile int* abort_flag = &bars.abort;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int row0 = blockIdx.x * RT * kPfRows;
-  const int nblocks = 2 * p.H;                 // (head, key or value rows)
+  const int nblocks = p.nblocks;
   const int nsteps = nblocks * p.nkc;
 
   if (tid == 0) {
@@ -349,8 +354,8 @@ __global__ void __launch_bounds__(kKvThreads, 1)
           break;
         const int blk = i / p.nkc, kc = i % p.nkc;
         mbar_arrive_expect_tx(smem_u32(&bars.bfull[s]), kKvBBytes);
-        tma_load_2d(sbase + b_off + s * kKvBBytes, (blk & 1) ? &wvmap : &wkmap, kc * kPfChunk,
-                    (blk >> 1) * kKvBlock, smem_u32(&bars.bfull[s]), pol_keep);
+        tma_load_2d(sbase + b_off + s * kKvBBytes, (p.kv_mode && (blk & 1)) ? &wvmap : &wkmap, kc * kPfChunk,
+                    (p.kv_mode ? blk >> 1 : blk) * kKvBlock, smem_u32(&bars.bfull[s]), pol_keep);
         issued = i + 1;
       }
       // every copy issued lands before the CTA can leave
@@ -438,7 +443,10 @@ __global__ void __launch_bounds__(kKvThreads, 1)
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) {
-          tma_store_2d(&omap, blk * kKvBlock + cbase + c0, y0, stg + (nst & 1) * kKvStageOut);
+          // every chunk commits a group (possibly empty), so the buffer
+          // rotation above stays in step
+          if (blk * kKvBlock + cbase + c0 < p.out_cols)
+            tma_store_2d(&omap, blk * kKvBlock + cbase + c0, y0, stg + (nst & 1) * kKvStageOut);
           bulk_commit_group();
         }
       }
@@ -937,6 +945,9 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st, void (*mark)(c
   kp.nkc = nkc;
   kp.wait_ns = kWaitLimitNs;
   kp.status = a.status;
+  kp.nblocks = 2 * a.H;
+  kp.kv_mode = 1;
+  kp.out_cols = a.H * kKvFeat;
   if (nkc <= 4) {
     kp.stages = kv_stages<2>(nkc);
     const int kv_smem = static_cast<int>(kv_smem_bytes<2>(nkc));
@@ -984,6 +995,42 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st, void (*mark)(c
   e = cudaGetLastError();
   if (mark) mark(st, false);
   return e;
+}
+
+cudaError_t launch_gate_table(const void* emb, const void* w_ue, int vocab, int d_e, int d_c, void* table,
+                              int32_t* status, cudaStream_t st) {
+  if (vocab <= 0) return cudaSuccess;
+  CUtensorMap amap, wmap, omap;
+  if (!pf_encode(&amap, emb, vocab, d_e, d_e)) return cudaErrorInvalidValue;
+  if (!pf_encode(&wmap, w_ue, d_c, d_e, d_e)) return cudaErrorInvalidValue;
+  if (!pf_encode(&omap, table, vocab, d_c, d_c, 32)) return cudaErrorInvalidValue;
+  const int nkc = d_e / kPfChunk;
+  KvParams kp;
+  kp.kv = static_cast<__nv_bfloat16*>(table);
+  kp.total = vocab;
+  kp.H = 0;
+  kp.nkc = nkc;
+  kp.wait_ns = kWaitLimitNs;
+  kp.status = status;
+  kp.nblocks = (d_c + kKvBlock - 1) / kKvBlock;   // the last block's rows past d_c read as zero
+  kp.kv_mode = 0;
+  kp.out_cols = d_c;
+  cudaError_t e;
+  if (nkc <= 4) {
+    kp.stages = kv_stages<2>(nkc);
+    const int smem = static_cast<int>(kv_smem_bytes<2>(nkc));
+    e = cudaFuncSetAttribute(prefill_kv_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    prefill_kv_kernel<2><<<(vocab + 2 * kPfRows - 1) / (2 * kPfRows), kKvThreads, smem, st>>>(amap, wmap, wmap, omap,
+                                                                                              kp);
+  } else {
+    kp.stages = kv_stages<1>(nkc);
+    const int smem = static_cast<int>(kv_smem_bytes<1>(nkc));
+    e = cudaFuncSetAttribute(prefill_kv_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    prefill_kv_kernel<1><<<(vocab + kPfRows - 1) / kPfRows, kKvThreads, smem, st>>>(amap, wmap, wmap, omap, kp);
+  }
+  return cudaGetLastError();
 }
 
 }  // namespace egmla

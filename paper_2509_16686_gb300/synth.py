@@ -472,3 +472,14 @@ def case_prefill_ragged(seed: int = 6, batch: int = 16, lo: int = 128, hi: int =
     lens = log_uniform_lengths(np.random.default_rng(seed + 1000), batch, lo, hi)
     kw.setdefault("id_dist", "zipf")
     return make_prefill_case("prefill_ragged", dims_bf16(d_c=192, vocab=50000), lens, seed=seed, **kw)
+
+
+def make_embedding(case, d_e: int, *, seed: int):
+    """Gate embedding of the non-precomputed EG-MLA form (Section 3 Eqs. 3-4):
+    E [V, d_e] ~ N(0, 1) and W^UE [d_c, d_e] ~ N(0, d_e^-1/2), stored in the
+    model dtype, so that E W^UE^T has unit-variance entries."""
+    d = case.dims
+    rng = np.random.default_rng(seed)
+    emb = _store(_normal(rng, (d.vocab, d_e), 1.0), d.dtype)
+    w_ue = _store(_normal(rng, (d.d_c, d_e), d_e ** -0.5), d.dtype)
+    return emb, w_ue
