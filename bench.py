@@ -85,8 +85,8 @@ def parse():
                     help="timed steps (default 20000; 200 for layers24, 2000 per length for --sweep)")
     ap.add_argument("--warmup", type=int, default=30)
     ap.add_argument("--workload", default="c32k",
-                    choices=["c32k", "c4k", "ragged", "ragged_mla", "layers24", "layers24_full", "r0", "prefill",
-                             "prefill_ragged"])
+                    choices=["c32k", "c32k_embed", "c4k", "ragged", "ragged_mla", "layers24", "layers24_full", "r0",
+                             "prefill", "prefill_ragged"])
     ap.add_argument("--sweep", action="store_true",
                     help="decode throughput vs context length: batch 8, d_c 256, L = 1K .. 64K, one line per L")
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
@@ -105,12 +105,21 @@ def parse():
     return ap.parse_args()
 
 
+def synth_mod():
+    from paper_2509_16686_gb300 import synth
+    return synth
+
+
 def make_workload(name):
     from paper_2509_16686_gb300 import synth
     if name == "c32k":
         case = synth.case_c32k(keep_logical=False)
         desc = "c32k: batch 8 x context 32768, 16 heads, d_nope 128, d_rope 64, d_c 256, vocab 32000, " \
                "64-token pages permuted over one pool, uniform ids"
+    elif name == "c32k_embed":
+        case = synth.case_c32k(keep_logical=False)
+        desc = "c32k_embed: the c32k step with its gate table computed in the step from the gate embedding " \
+               "(eg_mla_gate_table: E [32000 x 256] W^UE^T, then eg_mla_step), the EG-MLA form without a stored table"
     elif name == "c4k":
         case = synth.case_c4k(keep_logical=False)
         desc = "c4k: batch 32 x context 4096, 16 heads, d_c 256, d_rope 64, vocab 32000, contiguous pages"
@@ -986,9 +995,21 @@ def run_gpu(args, workload, torch, dist, ws, rank):
     # of at most one CTA per SM); fp32: append + decode + combine
     fused = d.dtype == "bf16" and d.d_c in (192, 256) and splits <= sms
     launches_per_step = n_layers * ((2 if fused else 3) if d.dtype == "bf16" else 3)
+    if workload.endswith("_embed"):
+        launches_per_step += n_layers
+
+    embed = workload.endswith("_embed")
+    if embed:
+        # the gate table of the step, computed in it from the embedding (the
+        # units share the table tensor of the first)
+        emb_h, w_ue_h = synth_mod().make_embedding(case, d.d_c, seed=75)
+        emb_d = device.to_device_array(emb_h, "bf16", "cuda")
+        w_ue_d = device.to_device_array(w_ue_h, "bf16", "cuda")
 
     def run_group(g):
         for u in g:
+            if embed:
+                _lib.eg_mla_gate_table(u.dims, emb_d, w_ue_d, u.gate_table, u.status, stream)
             u.step(stream)
 
     # ---- warm-up, then capture one graph of every group (one step each)
@@ -1101,6 +1122,8 @@ def run_gpu(args, workload, torch, dist, ws, rank):
             stream.wait_event(ev_in[k])
             if used[k]:
                 stream.wait_event(ev_out[k])          # this unit's last output has been read back
+            if embed:
+                _lib.eg_mla_gate_table(units[k].dims, emb_d, w_ue_d, units[k].gate_table, units[k].status, stream)
             steps_bound[k]()
             ev_comp[k].record(stream)
             if i + 1 < len(seq):
@@ -1119,6 +1142,28 @@ def run_gpu(args, workload, torch, dist, ws, rank):
     e2e_ms = max_over_ranks(e0.elapsed_time(e1), dist, "cuda")
     e2e_value = whole_job_rate(ws, B, e2e_steps, e2e_ms)
     assert units[0].read_status() == 0, "device status after end-to-end run"
+
+    # ---- the gate table from the embedding alone (c32k_embed): a graph of 20 calls
+    gate_table = None
+    if embed:
+        gg = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gg, stream=stream):
+            for _ in range(20):
+                _lib.eg_mla_gate_table(units[0].dims, emb_d, w_ue_d, units[0].gate_table, units[0].status, stream)
+        with torch.cuda.stream(stream):
+            gg.replay()
+            g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            g0.record(stream)
+            gg.replay()
+            g1.record(stream)
+        torch.cuda.synchronize()
+        gt_ms = g0.elapsed_time(g1) / 20
+        V, d_e = case.dims.vocab, d.d_c
+        gate_table = {"kernel": "prefill_kv_kernel (x W^T mode)", "ms": gt_ms, "vocab": V, "d_e": d_e,
+                      "tflops": 2.0 * V * d_e * d.d_c / (gt_ms * 1e-3) / 1e12,
+                      "bytes": (V * d_e + d.d_c * d_e + V * d.d_c) * 2,
+                      "gbs": (V * d_e + d.d_c * d_e + V * d.d_c) * 2 / (gt_ms * 1e-3) / 1e9}
+        del gg
 
     # ---- the gate-off (plain MLA) result of the same workload, beside the gated one
     mla = None
@@ -1149,6 +1194,7 @@ def run_gpu(args, workload, torch, dist, ws, rank):
         "gpu_launches": steps * launches_per_step,
         "clocks": clk.summary(),
         "mla_baseline": mla,
+        "gate_table": gate_table,
     }
 
 
