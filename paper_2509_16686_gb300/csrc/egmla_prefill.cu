@@ -92,6 +92,7 @@ __device__ __forceinline__ int prompt_of_row(const int32_t* cu, int batch, int t
 // ============================================================================ 1. gate, LayerNorm, cache write
 struct PfGateParams {
   int32_t* order;              // [batch]: prompts by decreasing length (written by block 0)
+  int32_t* next_item;          // the attention's work counter, zeroed by block 0
   const __nv_bfloat16* c;      // [T, d_c]
   const __nv_bfloat16* kr;     // [T, d_r]
   const int32_t* ids;          // [T] (null with the gate off)
@@ -200,6 +201,7 @@ constexpr int kSortMaxBatch = 2048;   // larger batches keep the given order
 __global__ void __launch_bounds__(32 * kGateWarps) prefill_gate_kernel(const PfGateParams p) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (blockIdx.x == 0) {
+    if (threadIdx.x == 0) *p.next_item = 0;
     // the attention's launch order: longest prompts first (rank of each prompt
     // among all by length, ties by index), so that the longest prompts'
     // query blocks do not start last
@@ -502,49 +504,42 @@ __host__ __device__ constexpr uint32_t col_s(int x) { return x * kAttnKeys; }
 __host__ __device__ constexpr uint32_t col_o(int x) { return 256 + x * kPfDv; }
 constexpr float kRescaleLog2 = 8.f;
 
+struct AttnItem {
+  int b, h, qb, start, L;   // b < 0: no more work
+};
+
 struct AttnBars {
-  uint64_t qfull;
+  uint64_t qfull, qempty;
   uint64_t kfull[kAttnKSlots], kempty[kAttnKSlots];
   uint64_t vfull[kAttnVStages], vempty[kAttnVStages];
-  uint64_t sfull[2], pfull[2], odone[2];   // per query tile
+  uint64_t sfull[2], pfull[2], odone[2], ofree[2];   // per query tile
+  uint64_t ifull[2], iempty[2];                      // the work-item ring
   uint64_t drain;
+  AttnItem item[2];
   uint32_t tmem_base;
   int abort;
 };
 constexpr uint32_t kAttnSmem = kOffBars + sizeof(AttnBars) + 1024;
+constexpr int kAttnItemReaders = 2 + 8;   // MMA warp, value loader, eight softmax warps
 
 struct AttnParams {
   const int32_t* cu;
   const int32_t* order;   // prompts in launch order
-  __nv_bfloat16* out;   // [T, H, d_v]
-  int batch, H, qblocks, total;
+  int32_t* next_item;     // work counter, zeroed by the gate kernel
+  __nv_bfloat16* out;     // [T, H, d_v]
+  int batch, H, qblocks, total, items;
   float scale_log2;
   uint64_t wait_ns;
   int32_t* status;
 };
 
+// Persistent: one CTA per SM takes (prompt, head, 256-query block) items from
+// a counter, in launch order (prompts longest first, heads, blocks heaviest
+// first), so that the next item's query and key copies overlap the current
+// item's last tiles and epilogue.  Every barrier's phases run on across items.
 __global__ void __launch_bounds__(kAttnThreads, 1)
     prefill_attn_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kvmap,
                         const __grid_constant__ CUtensorMap krmap, const AttnParams p) {
-  // heaviest query blocks of a (prompt, head) first; the blocks of one
-  // (prompt, head) are neighbours in launch order, so its keys stay in L2
-  const int group = blockIdx.x / p.qblocks;
-  const int qb = p.qblocks - 1 - blockIdx.x % p.qblocks;
-  const int b = __ldg(p.order + group / p.H), h = group % p.H;
-  const int start = __ldg(p.cu + b);
-  const int L = __ldg(p.cu + b + 1) - start;
-  const int q0 = qb * 2 * kPfRows;
-  // prompt offsets that do not fit the packed rows, or a prompt longer than
-  // the host bound the grid was sized for: report, compute nothing past it
-  if (start < 0 || L < 0 || start > p.total - L || (qb == p.qblocks - 1 && L > p.qblocks * 2 * kPfRows)) {
-    if (threadIdx.x == 0) report_status(p.status, kStatusOutOfRange);
-    if (start < 0 || L < 0 || start > p.total - L) return;
-  }
-  if (q0 >= L) return;
-  const bool has_b = q0 + kPfRows < L;                     // tile B holds live queries
-  const int ntile[2] = {2 * qb + 1, has_b ? 2 * qb + 2 : 0};
-  const int nkt = has_b ? ntile[1] : ntile[0];
-
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const uint32_t sbase = smem_u32(smem);
@@ -554,6 +549,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 
   if (tid == 0) {
     mbar_init(smem_u32(&bars.qfull), 1);
+    mbar_init(smem_u32(&bars.qempty), 1);
     for (int s = 0; s < kAttnKSlots; ++s) {
       mbar_init(smem_u32(&bars.kfull[s]), 1);
       mbar_init(smem_u32(&bars.kempty[s]), 1);
@@ -566,6 +562,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       mbar_init(smem_u32(&bars.sfull[x]), 1);
       mbar_init(smem_u32(&bars.pfull[x]), 4);
       mbar_init(smem_u32(&bars.odone[x]), 1);
+      mbar_init(smem_u32(&bars.ofree[x]), 4);
+      mbar_init(smem_u32(&bars.ifull[x]), 1);
+      mbar_init(smem_u32(&bars.iempty[x]), kAttnItemReaders);
     }
     mbar_init(smem_u32(&bars.drain), 1);
     bars.abort = 0;
@@ -583,61 +582,129 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   tc_fence_after();
   const uint32_t tmem = bars.tmem_base;
 
+  // item n of this CTA sits in ring slot n % 2; a reader copies it out, then frees the slot
+  auto read_item = [&](int n, AttnItem& it, bool arrive) -> bool {
+    if (!pf_warp_wait(smem_u32(&bars.ifull[n & 1]), (n >> 1) & 1, abort_flag, p.wait_ns)) return false;
+    it = bars.item[n & 1];
+    __syncwarp();
+    if (arrive && lane == 0) mbar_arrive(smem_u32(&bars.iempty[n & 1]));
+    return true;
+  };
+  auto tiles_of = [&](const AttnItem& it, int (&nt)[2]) {
+    const int q0 = it.qb * 2 * kPfRows;
+    const bool has_b = q0 + kPfRows < it.L;
+    nt[0] = 2 * it.qb + 1;
+    nt[1] = has_b ? 2 * it.qb + 2 : 0;
+  };
+
   if (warp == 0) {
-    // ---- the query tiles once, then the key tiles: k^C of head h (two
-    // 64-column boxes of the kv buffer) and the shared k^R rows
+    // ---- work items, the query tiles of each, and the key tiles: k^C of
+    // head h (two 64-column chunks of the kv buffer) and the shared k^R rows
     if (elect_one()) {
       const uint64_t pol_q = policy_evict_first(), pol_k = policy_evict_last();
-      const int nq = has_b ? 2 : 1;
-      mbar_arrive_expect_tx(smem_u32(&bars.qfull), nq * kAttnQBytes);
-      for (int x = 0; x < nq; ++x)
-        for (int c = 0; c < 3; ++c)
-          tma_load_2d(sbase + kOffQ + x * kAttnQBytes + c * kPfAtom, &qmap, h * kPfDqk + c * kPfChunk,
-                      start + q0 + x * kPfRows, smem_u32(&bars.qfull), pol_q);
-      // chunk g = 3 j + c of key tile j goes to slot g % 4
-      int issued = 0;
-      for (int g = 0; g < 3 * nkt; ++g) {
-        const int s = g % kAttnKSlots, j = g / 3, c = g % 3;
-        if (g >= kAttnKSlots &&
-            !mbar_wait(smem_u32(&bars.kempty[s]), ((g / kAttnKSlots) & 1) ^ 1, abort_flag, p.wait_ns))
+      int g = 0;       // key chunks issued (chunk g in slot g % 4)
+      int n = 0;       // items published
+      bool ok = true;
+      while (ok) {
+        // the next non-empty item, or the end
+        AttnItem it;
+        it.b = -1;
+        for (;;) {
+          const int i = atomicAdd(p.next_item, 1);
+          if (i >= p.items) break;
+          const int group = i / p.qblocks;
+          const int qb = p.qblocks - 1 - i % p.qblocks;
+          const int b = __ldg(p.order + group / p.H), h = group % p.H;
+          const int start = __ldg(p.cu + b);
+          const int L = __ldg(p.cu + b + 1) - start;
+          // prompt offsets that do not fit the packed rows, or a prompt longer
+          // than the host bound: report, compute nothing past it
+          if (start < 0 || L < 0 || start > p.total - L) {
+            report_status(p.status, kStatusOutOfRange);
+            continue;
+          }
+          if (qb == p.qblocks - 1 && L > p.qblocks * 2 * kPfRows) report_status(p.status, kStatusOutOfRange);
+          if (qb * 2 * kPfRows >= L) continue;
+          it.b = b; it.h = h; it.qb = qb; it.start = start; it.L = L;
           break;
-        const int y = start + j * kAttnKeys;
-        mbar_arrive_expect_tx(smem_u32(&bars.kfull[s]), kPfAtom);
-        if (c < 2)
-          tma_load_2d(sbase + kOffK + s * kPfAtom, &kvmap, h * kKvFeat + c * kPfChunk, y, smem_u32(&bars.kfull[s]),
-                      pol_k);
-        else
-          tma_load_2d(sbase + kOffK + s * kPfAtom, &krmap, 0, y, smem_u32(&bars.kfull[s]), pol_k);
-        issued = g + 1;
+        }
+        if (n >= 2 && !mbar_wait(smem_u32(&bars.iempty[n & 1]), ((n >> 1) & 1) ^ 1, abort_flag, p.wait_ns)) break;
+        bars.item[n & 1] = it;
+        mbar_arrive(smem_u32(&bars.ifull[n & 1]));
+        if (it.b < 0) break;
+        int nt[2];
+        tiles_of(it, nt);
+        const int nkt = nt[1] > 0 ? nt[1] : nt[0];
+        // the query tiles once the previous item's score MMAs are done with them
+        if (n >= 1 && !mbar_wait(smem_u32(&bars.qempty), (n - 1) & 1, abort_flag, p.wait_ns)) break;
+        const int nq = nt[1] > 0 ? 2 : 1;
+        mbar_arrive_expect_tx(smem_u32(&bars.qfull), nq * kAttnQBytes);
+        for (int x = 0; x < nq; ++x)
+          for (int c = 0; c < 3; ++c)
+            tma_load_2d(sbase + kOffQ + x * kAttnQBytes + c * kPfAtom, &qmap, it.h * kPfDqk + c * kPfChunk,
+                        it.start + it.qb * 2 * kPfRows + x * kPfRows, smem_u32(&bars.qfull), pol_q);
+        for (int j = 0; ok && j < nkt; ++j) {
+          const int y = it.start + j * kAttnKeys;
+          for (int c = 0; c < 3; ++c, ++g) {
+            const int s = g % kAttnKSlots;
+            if (g >= kAttnKSlots &&
+                !mbar_wait(smem_u32(&bars.kempty[s]), ((g / kAttnKSlots) & 1) ^ 1, abort_flag, p.wait_ns)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(smem_u32(&bars.kfull[s]), kPfAtom);
+            if (c < 2)
+              tma_load_2d(sbase + kOffK + s * kPfAtom, &kvmap, it.h * kKvFeat + c * kPfChunk, y,
+                          smem_u32(&bars.kfull[s]), pol_k);
+            else
+              tma_load_2d(sbase + kOffK + s * kPfAtom, &krmap, 0, y, smem_u32(&bars.kfull[s]), pol_k);
+          }
+        }
+        ++n;
       }
+      // every copy issued lands before the CTA can leave (own flag: bounded, not cut short)
       volatile int own = 0;
-      if (!mbar_wait(smem_u32(&bars.qfull), 0, &own, p.wait_ns)) *abort_flag = 1;
-      for (int g = issued > kAttnKSlots ? issued - kAttnKSlots : 0; g < issued; ++g)
-        if (!mbar_wait(smem_u32(&bars.kfull[g % kAttnKSlots]), (g / kAttnKSlots) & 1, &own, p.wait_ns))
+      for (int q = g > kAttnKSlots ? g - kAttnKSlots : 0; q < g; ++q)
+        if (!mbar_wait(smem_u32(&bars.kfull[q % kAttnKSlots]), (q / kAttnKSlots) & 1, &own, p.wait_ns))
           *abort_flag = 1;
+      if (n >= 1 && !mbar_wait(smem_u32(&bars.qfull), (n - 1) & 1, &own, p.wait_ns)) *abort_flag = 1;
     }
     __syncwarp();
   } else if (warp == kAttnVWarp) {
     // ---- value tiles: v^C of head h, two stages, each refilled once both
     // PV MMAs that read it have completed
-    if (elect_one()) {
-      const uint64_t pol_v = policy_evict_last();
-      int issued = 0;
-      for (int j = 0; j < nkt; ++j) {
-        const int s = j % kAttnVStages;
-        if (j >= kAttnVStages &&
-            !mbar_wait(smem_u32(&bars.vempty[s]), ((j / kAttnVStages) & 1) ^ 1, abort_flag, p.wait_ns))
-          break;
-        const int y = start + j * kAttnKeys;
-        const uint32_t dst = sbase + kOffV + s * kAttnVBytes;
-        mbar_arrive_expect_tx(smem_u32(&bars.vfull[s]), kAttnVBytes);
-        tma_load_2d(dst, &kvmap, h * kKvFeat + kPfDn, y, smem_u32(&bars.vfull[s]), pol_v);
-        tma_load_2d(dst + kPfAtom, &kvmap, h * kKvFeat + kPfDn + kPfChunk, y, smem_u32(&bars.vfull[s]), pol_v);
-        issued = j + 1;
+    // (lane 0 issues; the whole warp reads the items)
+    int vt = 0;   // value tiles issued (tile vt in stage vt % 2), kept by lane 0
+    const uint64_t pol_v = policy_evict_last();
+    for (int n = 0;; ++n) {
+      AttnItem it;
+      if (!read_item(n, it, true) || it.b < 0) break;
+      int nt[2];
+      tiles_of(it, nt);
+      const int nkt = nt[1] > 0 ? nt[1] : nt[0];
+      int ok = 1;
+      if (lane == 0) {
+        for (int j = 0; j < nkt; ++j, ++vt) {
+          const int s = vt % kAttnVStages;
+          if (vt >= kAttnVStages &&
+              !mbar_wait(smem_u32(&bars.vempty[s]), ((vt / kAttnVStages) & 1) ^ 1, abort_flag, p.wait_ns)) {
+            ok = 0;
+            break;
+          }
+          const int y = it.start + j * kAttnKeys;
+          const uint32_t dst = sbase + kOffV + s * kAttnVBytes;
+          mbar_arrive_expect_tx(smem_u32(&bars.vfull[s]), kAttnVBytes);
+          tma_load_2d(dst, &kvmap, it.h * kKvFeat + kPfDn, y, smem_u32(&bars.vfull[s]), pol_v);
+          tma_load_2d(dst + kPfAtom, &kvmap, it.h * kKvFeat + kPfDn + kPfChunk, y, smem_u32(&bars.vfull[s]),
+                      pol_v);
+        }
       }
+      if (!__shfl_sync(0xffffffffu, ok, 0)) break;
+    }
+    if (lane == 0) {
       volatile int own = 0;
-      for (int j = issued > kAttnVStages ? issued - kAttnVStages : 0; j < issued; ++j)
-        if (!mbar_wait(smem_u32(&bars.vfull[j % kAttnVStages]), (j / kAttnVStages) & 1, &own, p.wait_ns))
+      for (int q = vt > kAttnVStages ? vt - kAttnVStages : 0; q < vt; ++q)
+        if (!mbar_wait(smem_u32(&bars.vfull[q % kAttnVStages]), (q / kAttnVStages) & 1, &own, p.wait_ns))
           *abort_flag = 1;
     }
     __syncwarp();
@@ -651,66 +718,84 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     // V [keys x features] is the B operand MN-major: 64-feature atoms 16 KB
     // apart, 8-key groups 1 KB apart
     const uint64_t vdesc = smem_desc(sbase + kOffV, kPfAtom, 1024, kSwizzle128B);
-    bool ok = pf_warp_wait(smem_u32(&bars.qfull), 0, abort_flag, p.wait_ns);
-    bool issued = false;
-    int kseen = -1;   // the last key chunk whose arrival was waited for
-    auto wait_k = [&](int g) {
-      if (kseen < g) {
-        ok = ok && pf_warp_wait(smem_u32(&bars.kfull[g % kAttnKSlots]), (g / kAttnKSlots) & 1, abort_flag,
-                                p.wait_ns);
-        kseen = g;
-      }
-    };
-    // O_X += P_X(i) V(i); the last reader of V(i) frees it, the last PV of X signals its epilogue
-    auto issue_pv = [&](int x, int i) {
-      const int vs = i % kAttnVStages;
-      if (x == 0 || (x == 1 && ntile[0] <= i)) {
-        // first reader of V(i): wait for its copy (A reads every tile B reads but the last)
-        ok = ok && pf_warp_wait(smem_u32(&bars.vfull[vs]), (i / kAttnVStages) & 1, abort_flag, p.wait_ns);
-      }
-      ok = ok && pf_warp_wait(smem_u32(&bars.pfull[x]), i & 1, abort_flag, p.wait_ns);
-      if (!ok) return;
-      tc_fence_after();
-      if (elect_one()) {
-        // A = P_X from tensor memory: 16 keys per MMA are 8 columns of bf16 pairs
-#pragma unroll
-        const uint64_t vd = vdesc + ((vs * kAttnVBytes) >> 4);
-        for (int ks = 0; ks < kAttnKeys / 16; ++ks)
-          mma_bf16_ts(tmem + col_o(x), tmem + col_s(x) + ks * 8, vd + ((ks * 2048) >> 4), idesc_o,
-                      (i > 0 || ks > 0) ? 1u : 0u);
-        const bool last_reader = x == 1 || ntile[1] <= i;
-        if (last_reader) mma_commit(smem_u32(&bars.vempty[vs]));
-        if (i == ntile[x] - 1) mma_commit(smem_u32(&bars.odone[x]));
-      }
-      __syncwarp();
-      issued = true;
-    };
-    auto issue_s = [&](int x, int j) {
-      const uint64_t qd = qdesc + ((x * kAttnQBytes) >> 4);
-      // the last reader of a key chunk (B, or A when B has no tile j) frees its slot
-      const bool last_reader = x == 1 || ntile[1] <= j;
-      for (int c = 0; c < 3; ++c) {
-        const int g = 3 * j + c, s = g % kAttnKSlots;
-        wait_k(g);
+    bool ok = true, issued = false;
+    int g0 = 0, v0 = 0;              // first key chunk and value tile of the item
+    int tx[2] = {0, 0};              // tiles of query tile X before this item
+    int kx[2] = {0, 0};              // items in which query tile X had rows
+    int kseen = -1;                  // the last key chunk whose arrival was waited for
+    for (int n = 0; ok; ++n) {
+      AttnItem it;
+      if (!read_item(n, it, true) || it.b < 0) break;
+      int ntile[2];
+      tiles_of(it, ntile);
+      const int nkt = ntile[1] > 0 ? ntile[1] : ntile[0];
+      ok = pf_warp_wait(smem_u32(&bars.qfull), n & 1, abort_flag, p.wait_ns);
+      auto wait_k = [&](int g) {
+        if (kseen < g) {
+          ok = ok && pf_warp_wait(smem_u32(&bars.kfull[g % kAttnKSlots]), (g / kAttnKSlots) & 1, abort_flag,
+                                  p.wait_ns);
+          kseen = g;
+        }
+      };
+      // O_X += P_X(i) V(i); the last reader of V(i) frees it, the last PV of X signals its epilogue
+      auto issue_pv = [&](int x, int i) {
+        const int vi = v0 + i, vs = vi % kAttnVStages;
+        if (x == 0 || ntile[0] <= i)   // first reader of V(i)
+          ok = ok && pf_warp_wait(smem_u32(&bars.vfull[vs]), (vi / kAttnVStages) & 1, abort_flag, p.wait_ns);
+        // the first PV MMA of X in this item overwrites O_X: its last item's epilogue has read it
+        if (i == 0 && kx[x] >= 1)
+          ok = ok && pf_warp_wait(smem_u32(&bars.ofree[x]), (kx[x] - 1) & 1, abort_flag, p.wait_ns);
+        ok = ok && pf_warp_wait(smem_u32(&bars.pfull[x]), (tx[x] + i) & 1, abort_flag, p.wait_ns);
         if (!ok) return;
         tc_fence_after();
         if (elect_one()) {
-          const uint64_t kd = kdesc + ((s * kPfAtom) >> 4);
+          const uint64_t vd = vdesc + ((vs * kAttnVBytes) >> 4);
+          // A = P_X from tensor memory: 16 keys per MMA are 8 columns of bf16 pairs
 #pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            mma_bf16_ss(tmem + col_s(x), qd + ((c * kPfAtom + kk * 32) >> 4), kd + ((kk * 32) >> 4), idesc_s,
-                        (c > 0 || kk > 0) ? 1u : 0u);
-          if (c == 2) mma_commit(smem_u32(&bars.sfull[x]));
-          if (last_reader) mma_commit(smem_u32(&bars.kempty[s]));
+          for (int ks = 0; ks < kAttnKeys / 16; ++ks)
+            mma_bf16_ts(tmem + col_o(x), tmem + col_s(x) + ks * 8, vd + ((ks * 2048) >> 4), idesc_o,
+                        (i > 0 || ks > 0) ? 1u : 0u);
+          if (x == 1 || ntile[1] <= i) mma_commit(smem_u32(&bars.vempty[vs]));
+          if (i == ntile[x] - 1) mma_commit(smem_u32(&bars.odone[x]));
         }
         __syncwarp();
+        issued = true;
+      };
+      auto issue_s = [&](int x, int j) {
+        const uint64_t qd = qdesc + ((x * kAttnQBytes) >> 4);
+        // the last reader of a key chunk (B, or A when B has no tile j) frees its slot
+        const bool last_reader = x == 1 || ntile[1] <= j;
+        for (int c = 0; c < 3; ++c) {
+          const int g = g0 + 3 * j + c, s = g % kAttnKSlots;
+          wait_k(g);
+          if (!ok) return;
+          tc_fence_after();
+          if (elect_one()) {
+            const uint64_t kd = kdesc + ((s * kPfAtom) >> 4);
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+              mma_bf16_ss(tmem + col_s(x), qd + ((c * kPfAtom + kk * 32) >> 4), kd + ((kk * 32) >> 4), idesc_s,
+                          (c > 0 || kk > 0) ? 1u : 0u);
+            if (c == 2) mma_commit(smem_u32(&bars.sfull[x]));
+            if (last_reader) mma_commit(smem_u32(&bars.kempty[s]));
+            // the item's last score MMAs done: the query tiles may be refilled
+            if (c == 2 && last_reader && j == nkt - 1) mma_commit(smem_u32(&bars.qempty));
+          }
+          __syncwarp();
+        }
+        issued = true;
+      };
+      for (int j = 0; ok && j <= nkt; ++j) {
+        for (int x = 0; ok && x < 2; ++x) {
+          if (j >= 1 && j - 1 < ntile[x]) issue_pv(x, j - 1);
+          if (ok && j < ntile[x]) issue_s(x, j);
+        }
       }
-      issued = true;
-    };
-    for (int j = 0; ok && j <= nkt; ++j) {
-      for (int x = 0; ok && x < 2; ++x) {
-        if (j >= 1 && j - 1 < ntile[x]) issue_pv(x, j - 1);
-        if (ok && j < ntile[x]) issue_s(x, j);
+      g0 += 3 * nkt;
+      v0 += nkt;
+      for (int x = 0; x < 2; ++x) {
+        tx[x] += ntile[x];
+        if (ntile[x] > 0) ++kx[x];
       }
     }
     if (issued) {
@@ -725,98 +810,108 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     const int x = (warp - kAttnSoftWarp0) >> 2;
     const int quad = warp & 3;
     const int r = 32 * quad + lane;
-    const int qrow = q0 + x * kPfRows + r;   // this row's position in the prompt
-    const int nx = ntile[x];
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * quad) << 16);
     const float sl2 = p.scale_log2;
-    float m_ref = 0.f, l = 0.f;
-    bool ok = nx > 0;
-    for (int j = 0; ok && j < nx; ++j) {
-      // S_X(j) complete (and with it every earlier MMA: O_X is current)
-      ok = pf_warp_wait(smem_u32(&bars.sfull[x]), j & 1, abort_flag, p.wait_ns);
+    int tx = 0, kx = 0;   // tiles and items of X before this item
+    bool ok = true;
+    for (int n = 0; ok; ++n) {
+      AttnItem it;
+      if (!read_item(n, it, true) || it.b < 0) break;
+      int ntile[2];
+      tiles_of(it, ntile);
+      const int nx = ntile[x];
+      if (nx == 0) continue;
+      const int qrow = it.qb * 2 * kPfRows + x * kPfRows + r;   // this row's position in the prompt
+      float m_ref = 0.f, l = 0.f;
+      for (int j = 0; ok && j < nx; ++j) {
+        // S_X(j) complete (and with it every earlier MMA: O_X is current)
+        ok = pf_warp_wait(smem_u32(&bars.sfull[x]), (tx + j) & 1, abort_flag, p.wait_ns);
+        if (!ok) break;
+        tc_fence_after();
+        float sv[kAttnKeys];
+#pragma unroll
+        for (int c = 0; c < kAttnKeys; c += 16)
+          tmem_ld16(lane_base + col_s(x) + c, *reinterpret_cast<float(*)[16]>(&sv[c]));
+        tmem_wait_ld();
+        const int k0 = j * kAttnKeys;
+        if (k0 + kAttnKeys - 1 > qrow) {
+          // keys after the query (the tile on the diagonal)
+#pragma unroll
+          for (int c = 0; c < kAttnKeys; ++c)
+            if (k0 + c > qrow) sv[c] = -INFINITY;
+        }
+        // row maximum and sum as eight interleaved chains (short dependencies)
+        float m8[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) m8[e] = sv[e];
+#pragma unroll
+        for (int c = 8; c < kAttnKeys; ++c) m8[c & 7] = fmaxf(m8[c & 7], sv[c]);
+        float mx =
+            fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])), fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
+        mx *= sl2;
+        float alpha = 1.f;
+        if (j == 0) {
+          m_ref = mx;
+        } else if (mx > m_ref + kRescaleLog2) {
+          alpha = pf_ex2(m_ref - mx);
+          m_ref = mx;
+        }
+        float pk[kAttnKeys / 2];   // bf16 pairs, kept as 32-bit words for the TMEM store
+        float r8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int c = 0; c < kAttnKeys; c += 2) {
+          const float p0 = pf_ex2(fmaf(sv[c], sl2, -m_ref));
+          const float p1 = pf_ex2(fmaf(sv[c + 1], sl2, -m_ref));
+          r8[(c >> 1) & 7] += p0 + p1;
+          pk[c / 2] = __uint_as_float(pack_bf16x2(p0, p1));
+        }
+        const float rs = ((r8[0] + r8[1]) + (r8[2] + r8[3])) + ((r8[4] + r8[5]) + (r8[6] + r8[7]));
+        l = fmaf(l, alpha, rs);
+        if (__any_sync(0xffffffffu, alpha != 1.f)) {
+#pragma unroll
+          for (int c = 0; c < kPfDv; c += 16) {
+            float o[16];
+            tmem_ld16(lane_base + col_o(x) + c, o);
+            tmem_wait_ld();
+#pragma unroll
+            for (int e = 0; e < 16; ++e) o[e] *= alpha;
+            tmem_st16(lane_base + col_o(x) + c, o);
+          }
+        }
+        // P_X over the first 64 columns of S_X
+#pragma unroll
+        for (int c = 0; c < kAttnKeys / 2; c += 16)
+          tmem_st16(lane_base + col_s(x) + c, *reinterpret_cast<const float(*)[16]>(&pk[c]));
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&bars.pfull[x]));
+      }
+      // ---- epilogue: O_X / l of the live rows, then O_X is free for the next item
+      if (ok) ok = pf_warp_wait(smem_u32(&bars.odone[x]), kx & 1, abort_flag, p.wait_ns);
       if (!ok) break;
       tc_fence_after();
-      float sv[kAttnKeys];
+      const float inv = 1.f / l;
+      const bool live = qrow < it.L;
+      __nv_bfloat16* orow = p.out + (static_cast<size_t>(it.start + (live ? qrow : 0)) * p.H + it.h) * kPfDv;
+      float o[kPfDv];
 #pragma unroll
-      for (int c = 0; c < kAttnKeys; c += 16)
-        tmem_ld16(lane_base + col_s(x) + c, *reinterpret_cast<float(*)[16]>(&sv[c]));
+      for (int c = 0; c < kPfDv; c += 16) tmem_ld16(lane_base + col_o(x) + c, *reinterpret_cast<float(*)[16]>(&o[c]));
       tmem_wait_ld();
-      const int k0 = j * kAttnKeys;
-      if (k0 + kAttnKeys - 1 > qrow) {
-        // keys after the query (the tile on the diagonal)
-#pragma unroll
-        for (int c = 0; c < kAttnKeys; ++c)
-          if (k0 + c > qrow) sv[c] = -INFINITY;
-      }
-      // row maximum and sum as eight interleaved chains (short dependencies)
-      float m8[8];
-#pragma unroll
-      for (int e = 0; e < 8; ++e) m8[e] = sv[e];
-#pragma unroll
-      for (int c = 8; c < kAttnKeys; ++c) m8[c & 7] = fmaxf(m8[c & 7], sv[c]);
-      float mx = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])), fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
-      mx *= sl2;
-      float alpha = 1.f;
-      if (j == 0) {
-        m_ref = mx;
-      } else if (mx > m_ref + kRescaleLog2) {
-        alpha = pf_ex2(m_ref - mx);
-        m_ref = mx;
-      }
-      float pk[kAttnKeys / 2];   // bf16 pairs, kept as 32-bit words for the TMEM store
-      float r8[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int c = 0; c < kAttnKeys; c += 2) {
-        const float p0 = pf_ex2(fmaf(sv[c], sl2, -m_ref));
-        const float p1 = pf_ex2(fmaf(sv[c + 1], sl2, -m_ref));
-        r8[(c >> 1) & 7] += p0 + p1;
-        pk[c / 2] = __uint_as_float(pack_bf16x2(p0, p1));
-      }
-      const float rs = ((r8[0] + r8[1]) + (r8[2] + r8[3])) + ((r8[4] + r8[5]) + (r8[6] + r8[7]));
-      l = fmaf(l, alpha, rs);
-      if (__any_sync(0xffffffffu, alpha != 1.f)) {
-#pragma unroll
-        for (int c = 0; c < kPfDv; c += 16) {
-          float o[16];
-          tmem_ld16(lane_base + col_o(x) + c, o);
-          tmem_wait_ld();
-#pragma unroll
-          for (int e = 0; e < 16; ++e) o[e] *= alpha;
-          tmem_st16(lane_base + col_o(x) + c, o);
-        }
-      }
-      // P_X over the first 64 columns of S_X
-#pragma unroll
-      for (int c = 0; c < kAttnKeys / 2; c += 16)
-        tmem_st16(lane_base + col_s(x) + c, *reinterpret_cast<const float(*)[16]>(&pk[c]));
-      tmem_wait_st();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&bars.pfull[x]));
-    }
-    // ---- epilogue: O_X / l of the live rows
-    if (ok) ok = pf_warp_wait(smem_u32(&bars.odone[x]), 0, abort_flag, p.wait_ns);
-    if (ok) {
-      tc_fence_after();
-      const float inv = 1.f / l;
-      const bool live = qrow < L;
-      __nv_bfloat16* orow = p.out + (static_cast<size_t>(start + (live ? qrow : 0)) * p.H + h) * kPfDv;
+      if (lane == 0) mbar_arrive(smem_u32(&bars.ofree[x]));
+      if (live) {
+        uint4* d = reinterpret_cast<uint4*>(orow);
 #pragma unroll
-      for (int c = 0; c < kPfDv; c += 32) {
-        float o[32];
-        tmem_ld16(lane_base + col_o(x) + c, *reinterpret_cast<float(*)[16]>(&o[0]));
-        tmem_ld16(lane_base + col_o(x) + c + 16, *reinterpret_cast<float(*)[16]>(&o[16]));
-        tmem_wait_ld();
-        if (live) {
-          uint4* d = reinterpret_cast<uint4*>(orow + c);
-#pragma unroll
-          for (int q = 0; q < 4; ++q)
-            d[q] = make_uint4(pack_bf16x2(o[8 * q] * inv, o[8 * q + 1] * inv),
-                              pack_bf16x2(o[8 * q + 2] * inv, o[8 * q + 3] * inv),
-                              pack_bf16x2(o[8 * q + 4] * inv, o[8 * q + 5] * inv),
-                              pack_bf16x2(o[8 * q + 6] * inv, o[8 * q + 7] * inv));
-        }
+        for (int q = 0; q < kPfDv / 8; ++q)
+          d[q] = make_uint4(pack_bf16x2(o[8 * q] * inv, o[8 * q + 1] * inv),
+                            pack_bf16x2(o[8 * q + 2] * inv, o[8 * q + 3] * inv),
+                            pack_bf16x2(o[8 * q + 4] * inv, o[8 * q + 5] * inv),
+                            pack_bf16x2(o[8 * q + 6] * inv, o[8 * q + 7] * inv));
       }
+      tx += nx;
+      ++kx;
     }
   }
   tc_fence_before();
@@ -868,8 +963,8 @@ struct PfWorkspace {
 PfWorkspace pf_layout(int batch, int total, int H, int d_c) {
   PfWorkspace w;
   size_t off = 0;
-  w.off_order = off;
-  off = align_up(off + static_cast<size_t>(batch) * 4, 256);
+  w.off_order = off;   // the prompt order, then the attention's work counter
+  off = align_up(off + static_cast<size_t>(batch + 1) * 4, 256);
   w.off_ctil = off;
   off = align_up(off + static_cast<size_t>(total) * d_c * 2, 256);
   w.off_kv = off;
@@ -900,6 +995,7 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st, void (*mark)(c
   // 1. gate, LayerNorm, cache write
   PfGateParams gp;
   gp.order = order;
+  gp.next_item = order + a.batch;
   gp.c = static_cast<const __nv_bfloat16*>(a.c);
   gp.kr = static_cast<const __nv_bfloat16*>(a.kr);
   gp.ids = a.ids;
@@ -979,6 +1075,7 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st, void (*mark)(c
   AttnParams ap;
   ap.cu = a.cu_seqlens;
   ap.order = order;
+  ap.next_item = order + a.batch;
   ap.out = static_cast<__nv_bfloat16*>(a.out);
   ap.batch = a.batch;
   ap.H = a.H;
@@ -988,10 +1085,16 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st, void (*mark)(c
   ap.wait_ns = kWaitLimitNs;
   ap.status = a.status;
   if (ap.qblocks == 0) return cudaSuccess;
-  const long long grid = static_cast<long long>(a.batch) * a.H * ap.qblocks;
-  if (grid > 0x7fffffffLL) return cudaErrorInvalidValue;
+  const long long items = static_cast<long long>(a.batch) * a.H * ap.qblocks;
+  if (items > 0x7fffffffLL) return cudaErrorInvalidValue;
+  ap.items = static_cast<int>(items);
+  int dev = 0, sms = 0;
+  e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  const int grid = static_cast<int>(items < sms ? items : sms);
   if (mark) mark(st, true);
-  prefill_attn_kernel<<<static_cast<unsigned>(grid), kAttnThreads, kAttnSmem, st>>>(qmap, kvmap, krmap, ap);
+  prefill_attn_kernel<<<grid, kAttnThreads, kAttnSmem, st>>>(qmap, kvmap, krmap, ap);
   e = cudaGetLastError();
   if (mark) mark(st, false);
   return e;
