@@ -10,29 +10,23 @@
 //   prefill_gate_kernel  one warp per prompt token: c~ = LN(c (*) G[id]) (or the
 //                        gate mode's variant; Section 3 Eq. 5 in latent space),
 //                        rounded to bf16, and the raw c, k^R and id written to
-//                        the token's cache slot through the block table.
+//                        the token's cache slot through the block table; its
+//                        first block also ranks the prompts by length (the
+//                        attention's launch order) and zeroes the attention's
+//                        work counter.
 //   prefill_kv_kernel    (tcgen05) [k^C_h ; v^C_h] = [W_UK,h ; W_UV,h] c~ for
 //                        256 tokens per CTA (128 at d_c > 256) and every head h
 //                        (Eqs. 2 and 6): per output block of 128 columns (the
 //                        key or the value rows of a head) M = 128 tokens per
 //                        row tile, N = 128, K = d_c; two TMEM accumulators so
-//                        the epilogue of one block overlaps the MMAs of the next.
-//   prefill_attn_kernel  (tcgen05) flash attention: one CTA per (prompt, head,
-//                        128-query tile), walking the key tiles 0..qt of the
-//                        same prompt.  S = Q K^T (M = 128 queries, N = 128
-//                        keys, K = d_n + d_r, the RoPE part read from the
-//                        shared k^R rows) into one of two TMEM score buffers;
-//                        one softmax thread per query row (its TMEM lane) turns
-//                        S into P in bf16, stored back to tensor memory; O += P
-//                        V (M = 128 queries, N = d_v, K = 128 keys; A = P read
-//                        from tensor memory, B = V read MN-major from shared
-//                        memory) in a third TMEM buffer.  Scores of tile j + 1
-//                        are computed while the softmax threads work on tile j.
-//
-// Warp roles of prefill_attn_kernel: warp 0 loads Q once and the key tiles
-// (two stages), warp 1 issues the MMAs, warps 2-5 run the softmax (warp w
-// owns TMEM lane quadrant w % 4) and the epilogue, warp 6 loads the value
-// tiles (two stages, each refilled when the PV MMA that read it completes).
+//                        the epilogue of one block overlaps the MMAs of the
+//                        next; the output leaves through TMA tensor stores.
+//                        The same kernel in plain x W^T mode computes the gate
+//                        table E W^UE^T (eg_mla_gate_table).
+//   prefill_attn_kernel  (tcgen05) causal flash attention, persistent: one CTA
+//                        per SM takes (prompt, head, 256-query block) items,
+//                        two query tiles of 128 rows each sharing every key and
+//                        value tile (see the kernel's own header).
 //
 // Online softmax with a lazily moved reference: a row keeps the reference
 // maximum m of its exponentials until a tile's maximum exceeds it by more than
@@ -467,7 +461,7 @@ __global__ void __launch_bounds__(kKvThreads, 1)
 }
 
 // ============================================================================ 3. causal flash attention
-// One CTA per (prompt, head, block of 256 queries): two query tiles X = A
+// Work item (prompt, head, block of 256 queries): two query tiles X = A
 // (queries q0 .. q0 + 127) and B (q0 + 128 .. q0 + 255) share every key and
 // value tile copied into shared memory, which halves the bytes a CTA pulls in
 // per flop (the per-SM copy rate into shared memory, not the tensor pipe,
