@@ -490,7 +490,10 @@ constexpr uint32_t kOffQ = 0;
 constexpr uint32_t kOffK = kOffQ + 2 * kAttnQBytes;
 constexpr uint32_t kOffV = kOffK + kAttnKSlots * kPfAtom;
 constexpr uint32_t kOffBars = kOffV + kAttnVStages * kAttnVBytes;
-constexpr int kAttnSoftWarp0 = 2;                           // warps 2-5: tile A, warps 6-9: tile B
+// warp 0: work items, query and key copies; warp 1: MMAs; warps 2-9: softmax
+// and epilogue (2-5 tile A, 6-9 tile B, warp w reading TMEM lane quadrant
+// w % 4); warp 10: value copies
+constexpr int kAttnSoftWarp0 = 2;
 constexpr int kAttnVWarp = 10;
 constexpr int kAttnThreads = 32 * (kAttnVWarp + 1);
 // TMEM columns: S_X (P_X over its first 64 columns) and O_X
