@@ -51,3 +51,32 @@ def test_page_layouts_and_unused_slots():
     filled = ~np.isnan(f(rows)).all(axis=1)
     assert filled.sum() == 129 + 63
     assert (perm.id_pool.reshape(-1)[~filled] < 0).all()
+
+
+def test_prefill_inputs_follow_the_recipe():
+    """Packed prompts: offsets from the lengths, each prompt's pages distinct
+    across the pool, the pool empty (NaN latents, ids -7), value ranges as in
+    the decode workloads."""
+    lens = [300, 0, 1, 129, 64]
+    pc = synth.make_prefill_case("recipe", synth.dims_bf16(), lens, seed=3, extra_pages=2)
+    assert list(pc.cu_seqlens) == [0, 300, 300, 301, 430, 494]
+    assert pc.q.shape == (494, 16, 192) and pc.c.shape == (494, 256) and pc.kr.shape == (494, 64)
+    P = pc.dims.page_size
+    used = [int(p) for b, L in enumerate(lens) for p in pc.block_table[b, :(L + P - 1) // P]]
+    assert len(used) == len(set(used)) == sum((L + P - 1) // P for L in lens)
+    assert pc.num_pages == len(used) + 2 and max(used) < pc.num_pages
+    assert np.isnan(f(pc.c_pool)).all() and (pc.id_pool == -7).all()
+    assert (pc.ids >= 0).all() and (pc.ids < pc.dims.vocab).all()
+    big = synth.case_prefill(batch=2, prompt=2048)
+    c = f(big.c)
+    assert abs(c.std() - 0.5) < 0.01 and abs(f(big.q).std() - 1.0) < 0.01
+
+
+def test_prefill_ragged_lengths_and_embedding_inputs():
+    pc = synth.case_prefill_ragged()
+    L = pc.seq_lens
+    assert L.min() >= 128 and L.max() <= 4096 and pc.dims.d_c == 192
+    case = synth.make_case("emb", synth.dims_bf16(vocab=2000), [64], seed=4)
+    emb, w_ue = synth.make_embedding(case, 256, seed=5)
+    assert emb.shape == (2000, 256) and w_ue.shape == (256, 256)
+    assert abs(f(emb).std() - 1.0) < 0.01 and abs(f(w_ue).std() - 1.0 / 16) < 0.002
