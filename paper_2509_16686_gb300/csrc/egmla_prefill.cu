@@ -15,7 +15,8 @@
 //                        attention's launch order) and zeroes the attention's
 //                        work counter.
 //   prefill_kv_kernel    (tcgen05) [k^C_h ; v^C_h] = [W_UK,h ; W_UV,h] c~ for
-//                        256 tokens per CTA (128 at d_c > 256) and every head h
+//                        128 tokens per CTA (RT = 1; RT = 2 row tiles share each
+//                        weight chunk in the gate-table mode) and every head h
 //                        (Eqs. 2 and 6): per output block of 128 columns (the
 //                        key or the value rows of a head) M = 128 tokens per
 //                        row tile, N = 128, K = d_c; two TMEM accumulators so
@@ -1021,8 +1022,9 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st, void (*mark)(c
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
 
-  // 2. keys and values of every head: two row tiles per CTA while their
-  // latent tiles fit shared memory next to the weight stages (d_c <= 256)
+  // 2. keys and values of every head: one 128-row tile per CTA (measured:
+  // the kernel is bound by its output stores per SM, so more CTAs beat fewer
+  // weight reads; two tiles per CTA took 114 us against 109 at 8 x 4096)
   CUtensorMap cmap, wkmap, wvmap;
   if (!pf_encode(&cmap, ctil, a.total, a.d_c, a.d_c)) return cudaErrorInvalidValue;
   if (!pf_encode(&wkmap, a.w_uk, static_cast<uint64_t>(a.H) * kPfDn, a.d_c, a.d_c)) return cudaErrorInvalidValue;
@@ -1041,14 +1043,7 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st, void (*mark)(c
   kp.nblocks = 2 * a.H;
   kp.kv_mode = 1;
   kp.out_cols = a.H * kKvFeat;
-  if (nkc <= 4) {
-    kp.stages = kv_stages<2>(nkc);
-    const int kv_smem = static_cast<int>(kv_smem_bytes<2>(nkc));
-    e = cudaFuncSetAttribute(prefill_kv_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, kv_smem);
-    if (e != cudaSuccess) return e;
-    prefill_kv_kernel<2><<<(a.total + 2 * kPfRows - 1) / (2 * kPfRows), kKvThreads, kv_smem, st>>>(
-        cmap, wkmap, wvmap, omap, kp);
-  } else {
+  {
     kp.stages = kv_stages<1>(nkc);
     const int kv_smem = static_cast<int>(kv_smem_bytes<1>(nkc));
     e = cudaFuncSetAttribute(prefill_kv_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kv_smem);
