@@ -1022,9 +1022,10 @@ cudaError_t launch_prefill(const PrefillArgs& a, cudaStream_t st, void (*mark)(c
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
 
-  // 2. keys and values of every head: one 128-row tile per CTA (measured:
-  // the kernel is bound by its output stores per SM, so more CTAs beat fewer
-  // weight reads; two tiles per CTA took 114 us against 109 at 8 x 4096)
+  // 2. keys and values of every head: one 128-row tile per CTA.  Its output
+  // stores and its weight copies bound it about equally per SM, so spreading
+  // the stores over more CTAs beats reading the weights fewer times (measured:
+  // two tiles per CTA took 114 us against 109 at 8 x 4096)
   CUtensorMap cmap, wkmap, wvmap;
   if (!pf_encode(&cmap, ctil, a.total, a.d_c, a.d_c)) return cudaErrorInvalidValue;
   if (!pf_encode(&wkmap, a.w_uk, static_cast<uint64_t>(a.H) * kPfDn, a.d_c, a.d_c)) return cudaErrorInvalidValue;
