@@ -729,7 +729,8 @@ def run_gpu_r0(args, workload, torch, dist, ws, rank):
     w_ukv = device.to_device_array(r0.w_ukv, "bf16", "cuda")
     gate = device.to_device_array(r0.gate_r0, "bf16", "cuda")
     gamma, beta = torch.from_numpy(r0.gamma).cuda(), torch.from_numpy(r0.beta).cuda()
-    wsb = torch.empty(_lib.eg_mla_decode_r0_workspace_size(units[0].dims, case.num_pages), dtype=torch.uint8,
+    wsb = torch.empty(_lib.eg_mla_decode_r0_workspace_size(units[0].dims, case.batch, units[0].block_table.shape[1],
+                                                           case.num_pages), dtype=torch.uint8,
                       device="cuda")
     out = torch.empty((case.batch, 16, 128), dtype=torch.bfloat16, device="cuda")
     stream = torch.cuda.Stream()
@@ -778,8 +779,9 @@ def run_gpu_r0(args, workload, torch, dist, ws, rank):
                                "d_c 256, vocabulary 32000; seeded synthetic W^UKV (the case's W_UK, W_UV), "
                                "R0 gate table N(1, 0.1), gamma N(1, 0.1), beta N(0, 0.1)",
                    "batch": case.batch, "ctx_tokens_cached": tokens,
-                   "l2": f"{REPLICAS} rotating cache replicas; the gated projections of the pool "
-                         f"({case.num_pages * 64 * width * 2 / 1e6:.0f} MB) are written and read every step"},
+                   "l2": f"{REPLICAS} rotating cache replicas; the gated values of the pool "
+                         f"({case.num_pages * 64 * d.num_heads * d.d_v * 2 / 1e6:.0f} MB) are written and read "
+                         f"every step, and the R0 gate rows ({case.num_pages * 64 * width * 2 / 1e6:.0f} MB) read"},
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "traffic": None, "kernel": "r0_project_kernel (+ r0_attend_kernel)",
                      "flops_per_launch": flops, "peak_source": src,

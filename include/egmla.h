@@ -421,16 +421,20 @@ int eg_mla_profile_end(double* ms_sum, int32_t* launches);
  *   gate_r0    [vocab, 4096] bf16: the gate in that space per token id
  *   ln_gamma_r0, ln_beta_r0  [4096] fp32, may be NULL (1, 0)
  *   out        [batch, 16, 128] bf16
- *   workspace  >= eg_mla_decode_r0_workspace_size(dims, num_pages) bytes,
- *              256-byte aligned: the gated projections of every pool row
- *              (4096 bf16 each) and their LayerNorm statistics
+ *   workspace  >= eg_mla_decode_r0_workspace_size(dims, batch,
+ *              max_pages_per_seq, num_pages) bytes, 256-byte aligned: the
+ *              gated values of every pool row (16 x 128 bf16, head-major),
+ *              the rows' LayerNorm statistics, and the logits of every
+ *              (sequence, position) the block table can hold (16 fp32 each)
  *
- * Device errors: a page id outside [0, num_pages) or a token id outside
+ * Device errors: a page id outside [0, num_pages), a sequence longer than
+ * its block table (positions past it are not read), or a token id outside
  * [0, vocab) of a cached token is reported as EG_MLA_ERR_OUT_OF_RANGE (the
  * gate then uses row 0); a timed-out pipeline wait as EG_MLA_ERR_TIMEOUT.
  * All 16-byte-read arguments must be 16-byte aligned.
  */
-size_t eg_mla_decode_r0_workspace_size(const eg_mla_dims* dims, int32_t num_pages);
+size_t eg_mla_decode_r0_workspace_size(const eg_mla_dims* dims, int32_t batch, int32_t max_pages_per_seq,
+                                       int32_t num_pages);
 int eg_mla_decode_r0(const eg_mla_dims* dims, const void* q, const void* c_pool, const void* krope_pool,
                      const int32_t* id_pool, const int32_t* block_table, int32_t max_pages_per_seq,
                      const int32_t* seq_lens, int32_t batch, int32_t num_pages, const void* w_ukv,

@@ -105,7 +105,7 @@ def _declare(lib: ctypes.CDLL) -> None:
     lib.eg_mla_step.argtypes = [D, P, P, P, P, P, P, P, P, P, I32, P, I32, I32, I32, P, P, P, P, P, P, I32, P, SZ,
                                 P, P]
     lib.eg_mla_step.restype = ctypes.c_int
-    lib.eg_mla_decode_r0_workspace_size.argtypes = [D, I32]
+    lib.eg_mla_decode_r0_workspace_size.argtypes = [D, I32, I32, I32]
     lib.eg_mla_decode_r0_workspace_size.restype = SZ
     lib.eg_mla_decode_r0.argtypes = [D, P, P, P, P, P, I32, P, I32, I32, P, P, P, P, P, P, SZ, P, P]
     lib.eg_mla_decode_r0.restype = ctypes.c_int
@@ -344,8 +344,9 @@ def bind_step(dims: EgMlaDims, c_pool, krope_pool, id_pool, c_new, krope_new, id
     return step
 
 
-def eg_mla_decode_r0_workspace_size(dims: EgMlaDims, num_pages: int) -> int:
-    n = load().eg_mla_decode_r0_workspace_size(ctypes.byref(dims), num_pages)
+def eg_mla_decode_r0_workspace_size(dims: EgMlaDims, batch: int, max_pages_per_seq: int, num_pages: int) -> int:
+    n = load().eg_mla_decode_r0_workspace_size(ctypes.byref(dims), int(batch), int(max_pages_per_seq),
+                                               int(num_pages))
     if n == 0:
         raise EgMlaError(EG_MLA_ERR_UNSUPPORTED, "eg_mla_decode_r0_workspace_size")
     return int(n)

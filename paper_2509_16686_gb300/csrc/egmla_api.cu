@@ -502,11 +502,12 @@ int eg_mla_decode_static(const eg_mla_dims* dims, const void* q, const void* c_p
                        EG_MLA_STATIC_SCRATCH_BYTES, dev_status, stream);
 }
 
-size_t eg_mla_decode_r0_workspace_size(const eg_mla_dims* dims, int32_t num_pages) {
-  if (check_dims(dims) != EG_MLA_OK || num_pages <= 0) return 0;
+size_t eg_mla_decode_r0_workspace_size(const eg_mla_dims* dims, int32_t batch, int32_t max_pages_per_seq,
+                                       int32_t num_pages) {
+  if (check_dims(dims) != EG_MLA_OK || num_pages <= 0 || batch < 0 || max_pages_per_seq <= 0) return 0;
   if (dims->dtype != EG_MLA_BF16 || dims->d_nope != 128 || dims->d_v != 128 || (dims->d_c != 192 && dims->d_c != 256))
     return 0;
-  return egmla::r0_workspace_bytes(num_pages);
+  return egmla::r0_workspace_bytes(batch, max_pages_per_seq, num_pages);
 }
 
 int eg_mla_decode_r0(const eg_mla_dims* dims, const void* q, const void* c_pool, const void* krope_pool,
@@ -526,7 +527,7 @@ int eg_mla_decode_r0(const eg_mla_dims* dims, const void* q, const void* c_pool,
       !aligned(gate_r0, 16) || !aligned(out, 16))
     return EG_MLA_ERR_INVALID_ARG;
   if (static_cast<int64_t>(num_pages) * dims->page_size > INT32_MAX) return EG_MLA_ERR_UNSUPPORTED;
-  if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < egmla::r0_workspace_bytes(num_pages))
+  if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < egmla::r0_workspace_bytes(batch, max_pages_per_seq, num_pages))
     return EG_MLA_ERR_WORKSPACE;
   egmla::R0Args a;
   a.q = q;

@@ -104,7 +104,7 @@ struct R0Args {
   int d_c, vocab, batch, max_pages, num_pages;
   float eps, scale_log2;
 };
-size_t r0_workspace_bytes(int num_pages);
+size_t r0_workspace_bytes(int batch, int max_pages, int num_pages);
 cudaError_t launch_decode_r0(const R0Args& a, cudaStream_t st);
 // Prefill (egmla_prefill.cu): bf16, d_n = d_v = 128, d_r = 64, d_c a
 // multiple of 64 up to 512, any head count.  Prompts packed row after row

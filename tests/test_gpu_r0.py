@@ -29,8 +29,8 @@ def run_r0(case, r0):
     gate = device.to_device_array(r0.gate_r0, "bf16", "cuda")
     gamma = torch.from_numpy(r0.gamma).cuda()
     beta = torch.from_numpy(r0.beta).cuda()
-    ws = torch.empty(_lib.eg_mla_decode_r0_workspace_size(dc.dims, case.num_pages), dtype=torch.uint8,
-                     device="cuda")
+    ws = torch.empty(_lib.eg_mla_decode_r0_workspace_size(dc.dims, case.batch, dc.block_table.shape[1],
+                                                          case.num_pages), dtype=torch.uint8, device="cuda")
     out = torch.full((case.batch, 16, 128), float("nan"), dtype=torch.bfloat16, device="cuda")
     _lib.eg_mla_decode_r0(dc.dims, dc.q, dc.c_pool, dc.kr_pool, dc.id_pool, dc.block_table, dc.seq_lens, w_ukv,
                           gate, gamma, beta, out, ws, dc.status)
