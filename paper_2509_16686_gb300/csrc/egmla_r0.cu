@@ -339,17 +339,18 @@ __global__ void __launch_bounds__(kR0Threads, 1)
     const bool store_v = half == 1 && n > 0;   // uniform in the warp
     float s1 = 0.f, s2 = 0.f;
     bool ok = true;
+    // this half of the row's gate values of a head (128 bf16): each quarter
+    // of them is requested for head h + 1 as soon as head h has used it, so
+    // that the loads run while the rest of head h is processed
+    uint4 g[kR0Half / 8];
+    auto load_g = [&](int hh, int i) { ldg_32_na_hint(grow + hh * kR0Feat + 16 * i, pol_gate, g[2 * i], g[2 * i + 1]); };
+#pragma unroll
+    for (int i = 0; i < kR0Half / 16; ++i) load_g(0, i);
     for (int h = 0; h < kR0Heads; ++h) {
       const int db = h & 1;
-      // this half of the row's gate values of the head, requested at once
-      // while the head's MMAs may still run; the next head's brought into L2
-      uint4 g[kR0Half / 8];
-#pragma unroll
-      for (int i = 0; i < kR0Half / 16; ++i)
-        ldg_32_na_hint(grow + h * kR0Feat + 16 * i, pol_gate, g[2 * i], g[2 * i + 1]);
-      if (h + 1 < kR0Heads) {
-        prefetch_l2(grow + (h + 1) * kR0Feat);
-        prefetch_l2(grow + (h + 1) * kR0Feat + 64);
+      if (h + 2 < kR0Heads) {   // two heads ahead into L2
+        prefetch_l2(grow + (h + 2) * kR0Feat);
+        prefetch_l2(grow + (h + 2) * kR0Feat + 64);
       }
       ok = ok && warp_all_wait(smem_u32(&sm.dfull[db]), (h >> 1) & 1, abort_flag, p.wait_ns);
       if (!ok) break;
@@ -392,6 +393,10 @@ __global__ void __launch_bounds__(kR0Threads, 1)
               make_uint4(packed[0], packed[1], packed[2], packed[3]);
           *reinterpret_cast<uint4*>(vst + lane * kR0RowBytes + (((ch + 1) ^ (lane & 15)) << 4)) =
               make_uint4(packed[4], packed[5], packed[6], packed[7]);
+        }
+        if (c0 % 32 == 16 && h + 1 < kR0Heads) {   // columns c0 - 16 .. c0 + 15 done
+          load_g(h + 1, c0 / 16 - 1);
+          load_g(h + 1, c0 / 16);
         }
       }
       tc_fence_before();
