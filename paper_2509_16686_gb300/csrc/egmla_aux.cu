@@ -184,11 +184,11 @@ __device__ void split_starts(const int32_t* cu, const int32_t* seq_lens, int bat
 // splits' start records.
 //  - All 16-byte global loads of a thread are issued before any is stored
 //    (W_UK with an L2 evict-last hint: it stays in L2 across steps).
-//  - W_UK and q^C are staged row-major; a warp takes a quad of sequences and
-//    a part of the n range, reading per 8 n the lane's feature of 8 W rows
-//    and 8 n of each q^C row (one 16-byte broadcast per sequence) for 32
-//    FMAs.  With few sequences the spare warps split n further; the parts
-//    are added in shared memory.
+//  - W_UK (bf16) and q^C (converted to fp32 once, as it is staged) are held
+//    row-major; a warp takes a quad of sequences and a part of the n range,
+//    reading per 8 n the lane's feature of 8 W rows and 8 n of each q^C row
+//    (two 16-byte broadcasts per sequence) for 32 FMAs.  With few sequences
+//    the spare warps split n further; the parts are added in shared memory.
 constexpr int kPBatch = 32;
 constexpr int kPMaxNope = 256;
 constexpr int kPThreads = 256;
@@ -202,7 +202,7 @@ __global__ void prologue_tc_kernel(const __nv_bfloat16* __restrict__ q, const __
                        uint32_t* __restrict__ seq_done, int num_splits, const int32_t* __restrict__ block_table,
                        int max_pages, SplitStart* __restrict__ starts, const AppendArgs app) {
   __shared__ __align__(16) __nv_bfloat16 ws[kPMaxNope][kSumFeatures];  // W_UK,h[n][f0 + f]
-  __shared__ __align__(16) __nv_bfloat16 qs[kPBatch][kPMaxNope];      // q^C_{b0 + j, h}[n]
+  __shared__ __align__(16) float qs[kPBatch][kPMaxNope];              // q^C_{b0 + j, h}[n]
   // partial sums [n part * 4 quads + j][f], written once every warp is done with ws
   float (*red)[kSumFeatures] = reinterpret_cast<float (*)[kSumFeatures]>(&ws[0][0]);
   static_assert(sizeof(ws) >= 32 * kSumFeatures * sizeof(float), "reduction buffer aliases ws");
@@ -266,7 +266,13 @@ __global__ void prologue_tc_kernel(const __nv_bfloat16* __restrict__ q, const __
   for (int k = 0; k < kPLoads; ++k) {
     const int i = tid + k * kPThreads;
     if (i < wpieces) *reinterpret_cast<uint4*>(&ws[i / 4][8 * (i % 4)]) = wv[k];
-    if (i < qpieces) *reinterpret_cast<uint4*>(&qs[i / qpr][8 * (i % qpr)]) = qv[k];
+    if (i < qpieces) {
+      float x[8];
+      unpack16(qv[k], x);
+      float4* d = reinterpret_cast<float4*>(&qs[i / qpr][8 * (i % qpr)]);
+      d[0] = make_float4(x[0], x[1], x[2], x[3]);
+      d[1] = make_float4(x[4], x[5], x[6], x[7]);
+    }
   }
   __syncthreads();
   // warp -> (sequence quad sq, n part kp); nq quads, ks parts of the n range
@@ -283,10 +289,16 @@ __global__ void prologue_tc_kernel(const __nv_bfloat16* __restrict__ q, const __
       for (int e = 0; e < 8; ++e) w[e] = __bfloat162float(ws[blk * 8 + e][lane]);
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
-        float x[8];
-        unpack16(*reinterpret_cast<const uint4*>(&qs[4 * sq + i][blk * 8]), x);
-#pragma unroll
-        for (int e = 0; e < 8; ++e) acc[i] = fmaf(w[e], x[e], acc[i]);
+        const float4 x0 = *reinterpret_cast<const float4*>(&qs[4 * sq + i][blk * 8]);
+        const float4 x1 = *reinterpret_cast<const float4*>(&qs[4 * sq + i][blk * 8 + 4]);
+        acc[i] = fmaf(w[0], x0.x, acc[i]);
+        acc[i] = fmaf(w[1], x0.y, acc[i]);
+        acc[i] = fmaf(w[2], x0.z, acc[i]);
+        acc[i] = fmaf(w[3], x0.w, acc[i]);
+        acc[i] = fmaf(w[4], x1.x, acc[i]);
+        acc[i] = fmaf(w[5], x1.y, acc[i]);
+        acc[i] = fmaf(w[6], x1.z, acc[i]);
+        acc[i] = fmaf(w[7], x1.w, acc[i]);
       }
     }
   }
