@@ -62,3 +62,35 @@ def test_r0_out_of_range_id_is_reported(gpu_lib):
     dc, got = run_r0(case, r0)
     assert dc.read_status() == _lib.EG_MLA_ERR_OUT_OF_RANGE
     assert np.isfinite(got).all()
+
+
+def test_r0_batch_past_one_warp_of_sequences(gpu_lib):
+    """40 sequences: the projection finds its pages with a prefix sum over the
+    lanes 32 sequences at a time, so the second round of that scan is used."""
+    rng = np.random.default_rng(55)
+    lens = [int(x) for x in rng.integers(1, 300, size=40)]
+    lens[7], lens[33] = 0, 64
+    case = synth.make_case("r0-b40", synth.dims_bf16(d_c=192, vocab=3000), lens, seed=56, latent_scale=0.5,
+                           layout="permuted", affine_ln=True, extra_pages=5)
+    r0 = synth.make_r0_inputs(case, seed=57)
+    dc, got = run_r0(case, r0)
+    assert dc.read_status() == 0
+    ref = orc.decode_r0(case, gate_r0=orc.widen(r0.gate_r0, "bf16"), ln_gamma_r0=r0.gamma, ln_beta_r0=r0.beta)
+    diff = np.abs(got - ref)
+    assert (diff <= 1e-2 * np.maximum(1.0, np.abs(ref))).all() and rel_l2(got, ref) <= 5e-3, (diff.max(),)
+
+
+def test_r0_pages_shared_between_sequences(gpu_lib):
+    """A page in two sequences' block tables (a shared prefix) is projected for
+    each of them; both write the same gated values, and each sequence's logits
+    are its own."""
+    case = synth.make_case("r0-shared", synth.dims_bf16(d_c=256, vocab=3000), [300, 200, 150], seed=58,
+                           latent_scale=0.5, layout="permuted", affine_ln=True)
+    case.block_table[1, 0] = case.block_table[0, 0]
+    case.block_table[2, 1] = case.block_table[0, 2]
+    r0 = synth.make_r0_inputs(case, seed=59)
+    dc, got = run_r0(case, r0)
+    assert dc.read_status() == 0
+    ref = orc.decode_r0(case, gate_r0=orc.widen(r0.gate_r0, "bf16"), ln_gamma_r0=r0.gamma, ln_beta_r0=r0.beta)
+    diff = np.abs(got - ref)
+    assert (diff <= 1e-2 * np.maximum(1.0, np.abs(ref))).all() and rel_l2(got, ref) <= 5e-3, (diff.max(),)
