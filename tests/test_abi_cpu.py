@@ -208,3 +208,54 @@ def test_prefill_rejects_bad_arguments(lib):
     # gate off: ids and gate table may be null
     d_off = _lib.make_dims(16, 128, 64, 128, 256, 32000, gate=False)
     assert _prefill_call(lib, d_off, ids=0, gate=0, ws_bytes=1000) == _lib.EG_MLA_ERR_WORKSPACE
+
+
+# --------------------------------------------------------------------------- R0 decode: host-side checks
+def _r0_call(lib, dims, **kw):
+    """eg_mla_decode_r0 with fake, aligned device addresses; each case makes one
+    host check fail, so the call returns before anything is launched."""
+    P = lambda v: ctypes.c_void_p(v)
+    a = dict(q=0x1000, c_pool=0x2000, kr_pool=0x3000, id_pool=0x4000, bt=0x5000, max_pages=4, seq_lens=0x6000,
+             batch=2, num_pages=8, w_ukv=0x7000, gate=0x8000, gamma=None, beta=None, out=0x9000, ws=0xA000,
+             ws_bytes=1 << 30, status=None)
+    a.update(kw)
+    return lib.eg_mla_decode_r0(ctypes.byref(dims), P(a["q"]), P(a["c_pool"]), P(a["kr_pool"]), P(a["id_pool"]),
+                                P(a["bt"]), a["max_pages"], P(a["seq_lens"]), a["batch"], a["num_pages"],
+                                P(a["w_ukv"]), P(a["gate"]), P(a["gamma"]), P(a["beta"]), P(a["out"]), P(a["ws"]),
+                                ctypes.c_size_t(a["ws_bytes"]), P(a["status"]), None)
+
+
+def test_r0_workspace_size(lib):
+    d = _lib.make_dims(16, 128, 64, 128, 256, 32000)
+    # gated values (16 x 128 bf16 per pool row), row statistics (2 fp32), and
+    # 16 fp32 logits per (sequence, position) of the block table; 256-byte pieces
+    rows, positions = 512 * 64, 8 * 64 * 64
+    expect = rows * 16 * 128 * 2 + rows * 8 + positions * 16 * 4
+    assert _lib.eg_mla_decode_r0_workspace_size(d, 8, 64, 512) == expect
+    assert _lib.eg_mla_decode_r0_workspace_size(d, 8, 64, 512) < _lib.eg_mla_decode_r0_workspace_size(d, 9, 64, 512)
+    for bad in (_lib.make_dims(16, 128, 64, 128, 512, 32000, gate=False),   # d_c 512
+                _lib.make_dims(16, 64, 64, 64, 256, 32000),                 # d_nope, d_v 64
+                _lib.make_dims(4, 32, 16, 32, 64, 1000, dtype="fp32")):     # fp32
+        assert lib.eg_mla_decode_r0_workspace_size(ctypes.byref(bad), 8, 64, 512) == 0
+    assert lib.eg_mla_decode_r0_workspace_size(ctypes.byref(d), 8, 0, 512) == 0       # no block table
+    assert lib.eg_mla_decode_r0_workspace_size(ctypes.byref(d), 8, 64, 0) == 0        # no pool
+
+
+def test_r0_rejects_bad_arguments(lib):
+    d = _lib.make_dims(16, 128, 64, 128, 256, 32000)
+    assert _r0_call(lib, d, batch=0) == _lib.EG_MLA_OK                       # nothing to do
+    assert _r0_call(lib, d, batch=-1) == _lib.EG_MLA_ERR_INVALID_ARG
+    assert _r0_call(lib, d, max_pages=0) == _lib.EG_MLA_ERR_INVALID_ARG
+    assert _r0_call(lib, d, num_pages=0) == _lib.EG_MLA_ERR_INVALID_ARG
+    for name in ("q", "c_pool", "kr_pool", "id_pool", "bt", "seq_lens", "w_ukv", "gate", "out"):
+        assert _r0_call(lib, d, **{name: 0}) == _lib.EG_MLA_ERR_INVALID_ARG, name
+    assert _r0_call(lib, d, out=0x9008) == _lib.EG_MLA_ERR_INVALID_ARG      # 16-byte alignment
+    assert _r0_call(lib, d, gate=0x8004) == _lib.EG_MLA_ERR_INVALID_ARG
+    need = _lib.eg_mla_decode_r0_workspace_size(d, 2, 4, 8)
+    assert _r0_call(lib, d, ws_bytes=need - 1) == _lib.EG_MLA_ERR_WORKSPACE
+    assert _r0_call(lib, d, ws=0xA010) == _lib.EG_MLA_ERR_WORKSPACE          # 256-byte alignment
+    assert _r0_call(lib, d, ws=0) == _lib.EG_MLA_ERR_WORKSPACE
+    for bad in (_lib.make_dims(16, 128, 64, 128, 512, 32000, gate=False),
+                _lib.make_dims(16, 128, 64, 128, 128, 32000),                 # d_c 128
+                _lib.make_dims(4, 32, 16, 32, 64, 1000, dtype="fp32")):
+        assert _r0_call(lib, bad) == _lib.EG_MLA_ERR_UNSUPPORTED
