@@ -635,14 +635,12 @@ size_t r0_workspace_bytes(int batch, int max_pages, int num_pages) {
 
 cudaError_t launch_decode_r0(const R0Args& a, cudaStream_t st) {
   const size_t rows = static_cast<size_t>(a.num_pages) * kPage;
-  const size_t positions = static_cast<size_t>(a.batch) * a.max_pages * kPage;
   uint8_t* ws = static_cast<uint8_t*>(a.workspace);
   __nv_bfloat16* zv = reinterpret_cast<__nv_bfloat16*>(ws);
   size_t off = align_up(rows * kR0Heads * kR0Half * 2, 256);
   float2* stats = reinterpret_cast<float2*>(ws + off);
   off += align_up(rows * sizeof(float2), 256);
   float* logit = reinterpret_cast<float*>(ws + off);
-  (void)positions;
   CUtensorMap cmap, wmap;
   if (!r0_encode(&cmap, a.c_pool, rows, static_cast<uint64_t>(a.d_c), kPage)) return cudaErrorInvalidValue;
   if (!r0_encode(&wmap, a.w_ukv, kR0Width, static_cast<uint64_t>(a.d_c), kR0Feat)) return cudaErrorInvalidValue;
