@@ -94,3 +94,19 @@ def test_r0_pages_shared_between_sequences(gpu_lib):
     ref = orc.decode_r0(case, gate_r0=orc.widen(r0.gate_r0, "bf16"), ln_gamma_r0=r0.gamma, ln_beta_r0=r0.beta)
     diff = np.abs(got - ref)
     assert (diff <= 1e-2 * np.maximum(1.0, np.abs(ref))).all() and rel_l2(got, ref) <= 5e-3, (diff.max(),)
+
+
+def test_r0_full_size_sampled(gpu_lib):
+    """The R0 bench workload itself (8 sequences x 4096 tokens, d_c 256,
+    vocabulary 32000, the bench's seeds and launch): sequences 0 and 5, every
+    head, against the oracle."""
+    case = synth.case_c4k(batch=8, ctx=4096, keep_logical=False)
+    r0 = synth.make_r0_inputs(case, seed=61)
+    dc, got = run_r0(case, r0)
+    assert dc.read_status() == 0
+    picked = [0, 5]
+    ref = orc.decode_r0(case, gate_r0=orc.widen(r0.gate_r0, "bf16"), ln_gamma_r0=r0.gamma, ln_beta_r0=r0.beta,
+                        batches=picked)
+    g, r = got[picked], ref[picked]
+    diff = np.abs(g - r)
+    assert (diff <= 1e-2 * np.maximum(1.0, np.abs(r))).all() and rel_l2(g, r) <= 5e-3, (diff.max(), rel_l2(g, r))
