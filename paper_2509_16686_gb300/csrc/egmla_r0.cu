@@ -15,12 +15,15 @@
 //                      for each head h, D = C W^UKV_h^T (N = 256 = d_n + d_v
 //                      features, K = d_c) in one of two TMEM accumulators, so
 //                      that the epilogue of head h overlaps the MMAs of head
-//                      h + 1.  Epilogue warps, one row each: the key half
-//                      gates its 128 features (R0 gate G_R0[id]), rounds z to
-//                      bf16 and adds (q gamma) . z to the row's head dots; the
-//                      value half gates and rounds its 128 features and
-//                      stores them head-major through a per-warp shared-memory
-//                      tile (whole 512-byte rows per store instruction).  Both
+//                      h + 1.  Epilogue warps, one row each (their R0 gate
+//                      values G_R0[id] of head h + 1 requested a quarter at a
+//                      time while head h is processed): the key half gates
+//                      its 128 features, rounds z to bf16 and adds
+//                      (q gamma) . z to the row's head dots; the value half
+//                      gates and rounds its 128 features and stores them
+//                      head-major through a per-warp shared-memory tile (two
+//                      256-byte rows, 512 contiguous bytes, per store
+//                      instruction).  Both
 //                      add z and z^2 of the rounded values into the row's
 //                      statistics.  After the last head: (mu, 1/sqrt(var +
 //                      eps)) and every head's logit
